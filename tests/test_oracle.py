@@ -1,0 +1,196 @@
+"""Pins for the oracle: facts fixed by mathematics, independent of the oracle's code.
+
+Each test is chosen so that a plausible slip in the oracle (a dropped k term, a wrong
+index or sign, a transposed operand, bias added per k, a lost batch stride) fails at
+least one of them.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import B_KN, B_NK
+from synthetic import small_ints, uniform, normal, to_f32, f32_to_bf16_bits
+
+pytestmark = pytest.mark.filterwarnings("ignore::RuntimeWarning")
+
+
+def _int_operands(seed, batch, M, N, K, layout):
+    A = small_ints(seed, batch * M * K).reshape(batch, M, K).astype(np.float32)
+    bs = (K, N) if layout == B_KN else (N, K)
+    B = small_ints(seed + 1, batch * K * N).reshape((batch,) + bs).astype(np.float32)
+    bias = small_ints(seed + 2, N).astype(np.float32)
+    return A, B, bias
+
+
+def _exact_python(A, B, bias, layout):
+    """Brute force with Python integers: independent of the C code and of floating point."""
+    batch, M, K = A.shape
+    N = B.shape[2] if layout == B_KN else B.shape[1]
+    out = np.zeros((batch, M, N), dtype=object)
+    for b in range(batch):
+        for i in range(M):
+            for j in range(N):
+                s = 0
+                for k in range(K):
+                    bkj = B[b, k, j] if layout == B_KN else B[b, j, k]
+                    s += int(A[b, i, k]) * int(bkj)
+                out[b, i, j] = s + (int(bias[j]) if bias is not None else 0)
+    return out
+
+
+@pytest.mark.parametrize("layout", [B_KN, B_NK])
+@pytest.mark.parametrize("dims", [(1, 1, 1, 1), (1, 3, 5, 7), (2, 4, 3, 9), (3, 7, 6, 1),
+                                  (1, 5, 1, 11), (2, 1, 8, 4)])
+@pytest.mark.parametrize("with_bias", [False, True])
+def test_bruteforce_exact_integers(layout, dims, with_bias):
+    batch, M, N, K = dims
+    A, B, bias = _int_operands(100 + sum(dims), batch, M, N, K, layout)
+    bias = bias if with_bias else None
+    C64, C32 = oracle.matmul(A, B, bias, layout)
+    ref = _exact_python(A, B, bias, layout)
+    assert C64.shape == (batch, M, N)
+    assert np.array_equal(C64, ref.astype(np.float64))
+    assert np.array_equal(C32, ref.astype(np.float32))
+
+
+@pytest.mark.parametrize("layout", [B_KN, B_NK])
+def test_identity_bit_exact(layout):
+    K = 37
+    A = to_f32(uniform(7, 19 * K)).reshape(19, K)
+    eye = np.eye(K, dtype=np.float32)
+    C64, C32 = oracle.matmul(A, eye, None, layout)
+    assert np.array_equal(C32, A)
+    assert np.array_equal(C64, A.astype(np.float64))
+    # identity on the left: I . B = B (B given in either storage)
+    Bm = to_f32(normal(8, K * 23)).reshape(K, 23)
+    Bs = Bm if layout == B_KN else np.ascontiguousarray(Bm.T)
+    C64, _ = oracle.matmul(eye, Bs, None, layout)
+    assert np.array_equal(C64, Bm.astype(np.float64))
+
+
+def test_permutation_columns_exact():
+    K = N = 29
+    rng_perm = np.argsort(uniform(9, N))          # a permutation drawn from the generator
+    P = np.zeros((K, N), dtype=np.float32)
+    P[rng_perm, np.arange(N)] = 1.0               # column j of A.P is column perm[j] of A
+    A = to_f32(normal(10, 11 * K)).reshape(11, K)
+    C64, _ = oracle.matmul(A, P, None, B_KN)
+    assert np.array_equal(C64, A[:, rng_perm].astype(np.float64))
+    C64nk, _ = oracle.matmul(A, np.ascontiguousarray(P.T), None, B_NK)
+    assert np.array_equal(C64nk, C64)
+
+
+def test_all_ones_closed_form():
+    M, N, K = 5, 6, 1000
+    A = np.ones((M, K), dtype=np.float32)
+    B = np.ones((K, N), dtype=np.float32)
+    bias = to_f32(uniform(11, N))
+    C64, _ = oracle.matmul(A, B, bias, B_KN)
+    assert np.array_equal(C64, np.broadcast_to(K + bias.astype(np.float64), (M, N)))
+
+
+def test_k1_outer_product():
+    M, N = 13, 17
+    a = to_f32(uniform(12, M)).reshape(M, 1)
+    b = to_f32(uniform(13, N)).reshape(1, N)
+    C64, _ = oracle.matmul(a, b, None, B_KN)
+    # the product of two f32 values is exact in f64
+    assert np.array_equal(C64, a.astype(np.float64) * b.astype(np.float64))
+
+
+def test_zero_a_gives_bias_and_k0():
+    bias = to_f32(normal(14, 9))
+    C64, C32 = oracle.matmul(np.zeros((4, 5), np.float32), np.ones((5, 9), np.float32),
+                             bias, B_KN)
+    assert np.array_equal(C32, np.broadcast_to(bias, (4, 9)))
+    C64, _ = oracle.matmul(np.zeros((4, 0), np.float32), np.zeros((0, 9), np.float32),
+                           bias, B_KN)
+    assert np.array_equal(C64, np.broadcast_to(bias.astype(np.float64), (4, 9)))
+
+
+def test_empty_shapes():
+    C64, C32 = oracle.matmul(np.zeros((0, 5), np.float32), np.zeros((5, 3), np.float32))
+    assert C64.shape == (0, 3) and C32.shape == (0, 3)
+    C64, _ = oracle.matmul(np.zeros((2, 5), np.float32), np.zeros((5, 0), np.float32))
+    assert C64.shape == (2, 0)
+
+
+@pytest.mark.parametrize("layout", [B_KN, B_NK])
+def test_numpy_float64_matmul_agreement(layout):
+    M, N, K = 67, 129, 300
+    A = to_f32(normal(15, M * K)).reshape(M, K)
+    Bm = to_f32(normal(16, K * N, 0.02)).reshape(K, N)
+    Bs = Bm if layout == B_KN else np.ascontiguousarray(Bm.T)
+    bias = to_f32(normal(17, N, 0.02))
+    C64, _ = oracle.matmul(A, Bs, bias, layout)
+    ref = A.astype(np.float64) @ Bm.astype(np.float64) + bias.astype(np.float64)
+    assert oracle.rel_fro(C64, ref) <= 1e-12
+
+
+def test_layouts_agree_bit_exact():
+    M, N, K = 9, 21, 50
+    A = to_f32(normal(18, M * K)).reshape(M, K)
+    Bm = to_f32(normal(19, K * N)).reshape(K, N)
+    c_kn, _ = oracle.matmul(A, Bm, None, B_KN)
+    c_nk, _ = oracle.matmul(A, np.ascontiguousarray(Bm.T), None, B_NK)
+    assert np.array_equal(c_kn, c_nk)
+
+
+def test_batched_equals_per_matrix_and_broadcast_b():
+    batch, M, N, K = 4, 6, 10, 12
+    A = to_f32(normal(20, batch * M * K)).reshape(batch, M, K)
+    B = to_f32(normal(21, batch * N * K)).reshape(batch, N, K)
+    C64, _ = oracle.matmul(A, B, None, B_NK)
+    for b in range(batch):
+        cb, _ = oracle.matmul(A[b], B[b], None, B_NK)
+        assert np.array_equal(C64[b], cb)
+    Cbc, _ = oracle.matmul(A, B[1], None, B_NK)
+    for b in range(batch):
+        cb, _ = oracle.matmul(A[b], B[1], None, B_NK)
+        assert np.array_equal(Cbc[b], cb)
+
+
+def test_thread_count_invariance():
+    A = to_f32(normal(22, 33 * 70)).reshape(33, 70)
+    B = to_f32(normal(23, 70 * 45)).reshape(70, 45)
+    c1, _ = oracle.matmul(A, B, None, B_KN, nthreads=1)
+    c8, _ = oracle.matmul(A, B, None, B_KN, nthreads=8)
+    assert np.array_equal(c1, c8)
+
+
+def test_rows_subset_equals_full():
+    A = to_f32(normal(24, 40 * 30)).reshape(40, 30)
+    B = to_f32(normal(25, 30 * 20)).reshape(20, 30)
+    full, _ = oracle.matmul(A, B, None, B_NK)
+    rows = [0, 7, 39]
+    sub, _ = oracle.matmul_rows(A, B, None, B_NK, rows)
+    assert np.array_equal(sub, full[rows])
+
+
+def test_bf16_widening_known_patterns():
+    bits = np.array([0x0000, 0x8000, 0x3F80, 0xBF80, 0x4000, 0xC000, 0x3F81, 0x4049,
+                     0x0001, 0x7F7F], dtype=np.uint16)
+    want = np.array([0.0, -0.0, 1.0, -1.0, 2.0, -2.0, 1.0 + 2.0 ** -7,
+                     2.0 * (1.0 + 73.0 / 128.0), 2.0 ** -133,
+                     (2.0 - 2.0 ** -7) * 2.0 ** 127])
+    got = oracle.bf16_bits_to_f64(bits)
+    assert np.array_equal(got, want)
+    assert np.signbit(got[1])
+
+
+def test_bf16_operands_match_f32_operands():
+    """An operand given as bf16 bits equals the same values given as f32."""
+    A = to_f32(normal(26, 8 * 16)).reshape(8, 16)
+    B = to_f32(normal(27, 16 * 4)).reshape(16, 4)
+    Ab, Bb = f32_to_bf16_bits(A), f32_to_bf16_bits(B)
+    from synthetic import bf16_bits_to_f32
+    c_bits, _ = oracle.matmul(Ab, Bb, None, B_KN)
+    c_f32, _ = oracle.matmul(bf16_bits_to_f32(Ab), bf16_bits_to_f32(Bb), None, B_KN)
+    assert np.array_equal(c_bits, c_f32)
+
+
+def test_rel_fro_closed_form():
+    ref = np.array([[3.0, 4.0]])
+    assert oracle.rel_fro(ref, ref) == 0.0
+    assert oracle.rel_fro(np.array([[3.0, 0.0]]), ref) == pytest.approx(4.0 / 5.0)
+    assert oracle.rel_fro(np.zeros((1, 1)), np.zeros((1, 1))) == 0.0
