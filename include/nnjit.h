@@ -1,0 +1,255 @@
+/*
+ * nnjit.h -- C ABI of a JIT-tuned dense MatMul / BatchMatMul library for one NVIDIA
+ * GB300 (sm_103a).
+ *
+ * The operator is the one every kernel experiment of nnJIT (arXiv 2309.08978) tunes:
+ * MatMul (Sec. 2.2; Table 3, K0/K1) and BatchMatMul (Table 3, K2/K3):
+ *
+ *     C[b,i,j] = sum_k A[b,i,k] * Bt[b,k,j] (+ bias[j]),   Bt = B or B^T (see nnjit_blayout)
+ *
+ * The library keeps the paper's JIT scheme (Sec. 3): for each (kernel type, shape, device)
+ * it builds a small "lite" space of kernel configurations pruned by tile-based hardware
+ * usage formulas (Sec. 5.2, Table 1), times the candidates on the device, keeps the
+ * fastest, and caches it under a key made of the kernel type, shape and device (Sec. 5.3).
+ *
+ * Conventions for every function below:
+ *   - Every call returns an nnjit_status; no C++ exception crosses this boundary.  On
+ *     failure nnjit_last_error() returns a thread-local, human-readable detail string.
+ *   - Device pointers are plain CUDA device addresses (e.g. from cudaMalloc or a PyTorch
+ *     tensor's data_ptr()) on the device that was current when the plan was made; the
+ *     caller owns them.  `stream` is a cudaStream_t passed as void* (NULL = legacy
+ *     default stream).
+ *   - All sizes, leading dimensions and batch strides are in ELEMENTS, not bytes.
+ *   - Matrices are row-major.  A is [batch][M][K] (row i at A + b*stride_a + i*lda).
+ *     C is [batch][M][N] float32 (row i at C + b*stride_c + i*ldc).
+ *   - Operand element types: NNJIT_F32_FFMA and NNJIT_TF32 take float32 A and B;
+ *     NNJIT_BF16 takes bfloat16 A and B (16-bit patterns).  bias and C are always float32;
+ *     accumulation is always float32.
+ */
+#ifndef NNJIT_H
+#define NNJIT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+typedef enum {
+    NNJIT_OK = 0,
+    NNJIT_ERR_INVALID_ARG = 1,   /* bad shape (<0), NULL operand, unknown enum, bad stride */
+    NNJIT_ERR_UNSUPPORTED = 2,   /* legal request this library does not serve, e.g. a
+                                    tensor-core path whose row stride or pointer is not
+                                    16-byte aligned */
+    NNJIT_ERR_CUDA = 3,          /* a CUDA runtime/driver call failed (detail in last_error) */
+    NNJIT_ERR_OOM = 4,           /* device or host allocation failed */
+    NNJIT_ERR_TIMEOUT = 5,       /* a kernel's bounded wait expired and it stopped early
+                                    (device watchdog word set); results are invalid */
+    NNJIT_ERR_BUDGET = 6         /* tuning budget too small to evaluate any candidate;
+                                    only returned when NNJIT_PLAN_REQUIRE_TIMED is set */
+} nnjit_status;
+
+/* Arithmetic path.  C and bias are float32 for all three. */
+typedef enum {
+    NNJIT_F32_FFMA = 0,  /* float32 operands, exact float32 fused multiply-add (SIMT) */
+    NNJIT_TF32 = 1,      /* float32 operands consumed as TF32 by the tensor cores
+                            (tcgen05 .kind::tf32), float32 accumulation */
+    NNJIT_BF16 = 2       /* bfloat16 operands, float32 accumulation (tcgen05 .kind::f16,
+                            or the split-K GEMV when M <= 8) */
+} nnjit_dtype;
+
+/* Storage of B. */
+typedef enum {
+    NNJIT_B_KN = 0,      /* B is [K][N] row-major (ldb >= N): Bt = B */
+    NNJIT_B_NK = 1       /* B is [N][K] row-major (ldb >= K): Bt = B^T.  This is the
+                            PyTorch Linear weight layout and K^T of attention QK^T. */
+} nnjit_blayout;
+
+/* Kernel families of the lite space. */
+typedef enum {
+    NNJIT_FAMILY_FFMA = 0,  /* register-tiled SIMT GEMM, exact FP32 */
+    NNJIT_FAMILY_TC = 1,    /* TMA + tcgen05/TMEM tensor-core GEMM, persistent */
+    NNJIT_FAMILY_GEMV = 2   /* streaming split-K GEMV for M <= 8 (BF16 weights) */
+} nnjit_family;
+
+/* Plan descriptor flags. */
+#define NNJIT_PLAN_NO_CACHE      0x1u  /* neither read nor write the process plan cache */
+#define NNJIT_PLAN_EXHAUSTIVE    0x2u  /* time every candidate, ignoring the budget */
+#define NNJIT_PLAN_REQUIRE_TIMED 0x4u  /* fail with NNJIT_ERR_BUDGET instead of taking the
+                                          top-ranked candidate untimed */
+
+/*
+ * Full problem description.  Zero leading dimensions / strides mean "packed":
+ * lda = K, ldb = (B_KN ? N : K), ldc = N, stride_a = M*lda, stride_b = (B_KN ? K : N)*ldb,
+ * stride_c = M*ldc.  batch >= 1.  M, N, K >= 0 (an empty M or N is a no-op; K = 0 gives
+ * C = bias, or 0 without bias).
+ */
+typedef struct {
+    int64_t M, N, K;
+    int64_t batch;
+    int32_t dtype;        /* nnjit_dtype */
+    int32_t b_layout;     /* nnjit_blayout */
+    int64_t lda, ldb, ldc;
+    int64_t stride_a, stride_b, stride_c;
+    int32_t has_bias;     /* 1: run() takes a float32 bias[N] added to every row */
+    uint32_t flags;       /* NNJIT_PLAN_* */
+} nnjit_matmul_desc;
+
+/*
+ * Device resources the lite space is built against (the "hardware constraints" that
+ * the formulas of Table 1 take: registers, L1/shared memory and warps per core), plus
+ * the Blackwell-specific tensor-memory column count.
+ */
+typedef struct {
+    int32_t sm_count;
+    int32_t smem_per_sm;           /* bytes of shared memory per SM */
+    int32_t smem_per_block_optin;  /* bytes a CTA may opt in to */
+    int32_t regs_per_sm;
+    int32_t max_threads_per_sm;
+    int32_t max_blocks_per_sm;
+    int32_t tmem_cols_per_sm;      /* tensor-memory columns per SM (512 on sm_10x) */
+    int32_t l2_bytes;
+    int32_t cc_major, cc_minor;
+} nnjit_device_limits;
+
+/*
+ * One candidate of the lite space (the "sequence of primitives and configurations"
+ * of Sec. 2.2; tile symbols follow Table 1: x1, y1, r1 = bm, bn, bk; x0, y0 = tm, tn).
+ */
+typedef struct {
+    int32_t family;          /* nnjit_family */
+    int32_t bm, bn, bk;      /* CTA tile */
+    int32_t tm, tn;          /* FFMA: thread tile; GEMV: tm = rows per warp */
+    int32_t stages;          /* TC: shared-memory ring depth; GEMV: loads in flight per row */
+    int32_t split_k;         /* K slices reduced in a fixed order afterwards (1 = none) */
+    int32_t raster;          /* TC tile order: 0 = M fastest, 1 = N fastest */
+    int32_t threads;         /* threads per CTA */
+    int32_t smem_bytes;      /* shared memory per CTA */
+    int32_t tmem_cols;       /* TMEM columns per CTA (TC only) */
+    int32_t regs_per_thread; /* register figure used by the usage model */
+    int32_t blocks_per_sm;   /* Block_core of Table 1 */
+    int32_t grid;            /* CTAs per launch of the main kernel */
+    int32_t wave_eff_ppm;    /* predicted wave efficiency, parts per million */
+    int32_t instance;        /* index of the precompiled kernel instance */
+    int64_t predicted_cost;  /* model cost used for ordering (arbitrary units, lower first) */
+} nnjit_candidate;
+
+typedef struct nnjit_plan_s* nnjit_plan;
+
+/* ---------------------------------------------------------------------------------- */
+
+/* Static string for a status code.  Never NULL. */
+const char* nnjit_status_string(nnjit_status s);
+
+/* Detail of the last failing call on this thread ("" if none).  Valid until the next
+ * call on this thread. */
+const char* nnjit_last_error(void);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int32_t nnjit_version(void);
+
+/* Query the limits of CUDA device `device` (host call; needs a GPU). */
+nnjit_status nnjit_device_limits_query(int32_t device, nnjit_device_limits* out);
+
+/*
+ * Build the lite space for `d` against `lim` (host only; needs no GPU).  Sec. 5.2 and
+ * Table 1: enumerate power-of-two tiles (heuristic 2), keep those whose shared memory,
+ * TMEM, register and thread usage fit the device, compute Block_core =
+ * min(RegLimit, L1Limit, WarpLimit, ...), and order the survivors from most to fewest
+ * blocks per core, then by the predicted cost.  Writes at most `capacity` candidates to
+ * `out` (may be NULL when capacity is 0), the full count to *count, and the size of the
+ * unpruned space (every tile/stage/split combination of the family's axes before the
+ * usage rules and heuristics) to *naive_count (may be NULL).
+ * INVALID_ARG for a bad descriptor; UNSUPPORTED when no family serves it.
+ */
+nnjit_status nnjit_space_enumerate(const nnjit_matmul_desc* d, const nnjit_device_limits* lim,
+                                   nnjit_candidate* out, int32_t capacity, int32_t* count,
+                                   int64_t* naive_count);
+
+/*
+ * JIT-tune a plan for C[M,N] = A[M,K] . B[K,N] (B_KN, batch 1, packed, with a bias slot
+ * that may be NULL at run time).  Shorthand for nnjit_matmul_plan_ex.
+ */
+nnjit_status nnjit_matmul_plan(int64_t M, int64_t N, int64_t K, nnjit_dtype dt,
+                               double tune_budget_ms, nnjit_plan* out);
+
+/*
+ * JIT-tune a plan (Sec. 3: compose the lite space, evaluate candidates on the device,
+ * keep the fastest).  Candidates are evaluated in space order on device scratch buffers
+ * the call allocates and frees itself, while the wall-clock time spent stays under
+ * tune_budget_ms (at least one candidate is timed when the budget is > 0).  Budget 0
+ * takes the top-ranked candidate untimed (unless NNJIT_PLAN_REQUIRE_TIMED).  The choice
+ * is the fastest median time; ties go to the lower space index.  The result is cached
+ * per (type, shape, layout, strides, dtype, device) unless NNJIT_PLAN_NO_CACHE; a cache
+ * hit returns at once.  Uses the current CUDA device.  Synchronises the device.
+ * The plan owns its split-K workspace and its kernel-watchdog word.
+ */
+nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double tune_budget_ms,
+                                  nnjit_plan* out);
+
+/*
+ * Plan that uses candidate `index` of the space nnjit_space_enumerate builds for `d` on
+ * the current device, without tuning and without the cache (testing every candidate;
+ * exhaustive sweeps).  INVALID_ARG if index is out of range.
+ */
+nnjit_status nnjit_matmul_plan_candidate(const nnjit_matmul_desc* d, int32_t index,
+                                         nnjit_plan* out);
+
+/*
+ * C = A . Bt (+ bias) with the plan's kernel, asynchronously on `stream`.
+ * A, B: device pointers (float32 or bf16 per the plan's dtype); bias: float32[N] device
+ * pointer or NULL (NULL means no bias even if the plan was made with has_bias);
+ * C: float32 device pointer.  C must not overlap A, B or bias.  Tensor-core and GEMV
+ * paths need A, B (and C for the GEMV's vector stores) 16-byte aligned, else
+ * UNSUPPORTED.  Never synchronises.  A kernel watchdog expiry is reported by
+ * nnjit_plan_check.  Batched plans run all batch items.
+ */
+nnjit_status nnjit_matmul_run(nnjit_plan p, const void* A, const void* B, const float* bias,
+                              float* C, void* stream);
+
+/* Batched form of nnjit_matmul_run for attention QK^T / PV (Table 3, K2/K3): no bias. */
+nnjit_status nnjit_matmul_run_batched(nnjit_plan p, const void* A, const void* B, float* C,
+                                      void* stream);
+
+/*
+ * End-to-end form with HOST buffers: copies A, B (and bias when non-NULL) host->device
+ * into device staging buffers the plan owns (allocated on first use, packed layout),
+ * runs the plan, and copies C device->host, all asynchronously on `stream`; the caller
+ * synchronises the stream before reading hC.  Host buffers should be page-locked for
+ * asynchronous copies.  Plans with non-packed strides are UNSUPPORTED here.
+ */
+nnjit_status nnjit_matmul_run_host(nnjit_plan p, const void* hA, const void* hB,
+                                   const float* hbias, float* hC, void* stream);
+
+/* Synchronise the plan's device and read its watchdog word: TIMEOUT if any kernel of
+ * this plan stopped on an expired wait since the last check (the word is then reset). */
+nnjit_status nnjit_plan_check(nnjit_plan p);
+
+/*
+ * JSON description of the plan: shape, family and parameters of the chosen candidate,
+ * space size, naive count, tuning wall time, and every timed candidate with its median
+ * microseconds.  Truncated to len-1 characters (always NUL-terminated when len > 0);
+ * *needed (may be NULL) receives the full length + 1.
+ */
+nnjit_status nnjit_plan_describe(nnjit_plan p, char* buf, size_t len, size_t* needed);
+
+/* The chosen candidate. */
+nnjit_status nnjit_plan_candidate(nnjit_plan p, nnjit_candidate* out);
+
+/* Free the plan and everything it owns.  NULL is a no-op.  The caller must ensure no
+ * launch of this plan is still running (e.g. synchronise the stream first). */
+nnjit_status nnjit_plan_destroy(nnjit_plan p);
+
+/* Drop every cached plan choice of this process. */
+nnjit_status nnjit_cache_clear(void);
+
+/* Number of choices currently in the process plan cache. */
+int32_t nnjit_cache_size(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NNJIT_H */

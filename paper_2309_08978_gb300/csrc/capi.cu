@@ -1,0 +1,769 @@
+// C ABI: plans, the JIT tuner, the process plan cache and the run entry points.
+//
+// Sec. 3 of the paper: compose the lite space for the operator, evaluate the candidates
+// on the device one after another, keep the fastest, and store it in a kernel database
+// keyed by (kernel type t, shape s, primitive vector rho, device id) (Sec. 5.3).  Here
+// the database is an in-process map keyed by type, shape, layout, strides, dtype and
+// the device's name, compute capability and SM count.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <chrono>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <map>
+#include <memory>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "../../include/nnjit.h"
+#include "launch.h"
+#include "space.h"
+
+using namespace nnjit;
+
+// ------------------------------------------------------------------------ errors
+namespace {
+
+thread_local std::string t_last_error;
+
+nnjit_status fail(nnjit_status s, const std::string& msg) {
+    t_last_error = msg;
+    return s;
+}
+
+nnjit_status cuda_fail(cudaError_t e, const char* what) {
+    std::string m = std::string(what) + ": " + cudaGetErrorName(e) + " (" + cudaGetErrorString(e) + ")";
+    t_last_error = m;
+    if (e == cudaErrorMemoryAllocation) return NNJIT_ERR_OOM;
+    return NNJIT_ERR_CUDA;
+}
+
+bool env_flag(const char* name) {
+    const char* v = std::getenv(name);
+    return v && *v && std::strcmp(v, "0") != 0;
+}
+
+// Host-side fault injection for testing the tuner's failure handling without faulting
+// the GPU: NNJIT_FAULT="launch:<i>" makes candidate i's launch report an error,
+// "timeout:<i>" makes it report an expired kernel watchdog.
+struct FaultSpec {
+    int kind = 0;  // 0 none, 1 launch, 2 timeout
+    int index = -1;
+};
+
+FaultSpec read_fault() {
+    FaultSpec f;
+    const char* v = std::getenv("NNJIT_FAULT");
+    if (!v) return f;
+    int idx = -1;
+    if (std::sscanf(v, "launch:%d", &idx) == 1) { f.kind = 1; f.index = idx; }
+    else if (std::sscanf(v, "timeout:%d", &idx) == 1) { f.kind = 2; f.index = idx; }
+    return f;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------------ plan
+struct nnjit_plan_s {
+    Problem p;
+    int family = 0;
+    int device = 0;
+    nnjit_candidate cand{};
+    int chosen_index = 0;
+    int space_size = 0;
+    int64_t naive = 0;
+    std::vector<std::pair<int, double>> timings;  // (space index, median microseconds)
+    std::vector<int> failed;                      // space indices skipped as failing
+    double tune_ms = 0.0;
+    bool from_cache = false;
+    bool timed = false;
+    float* ws = nullptr;
+    size_t ws_bytes = 0;
+    int* err = nullptr;
+    std::mutex mu;  // guards the tensor-map cache and the host staging buffers
+    const void* tm_A = nullptr;
+    const void* tm_B = nullptr;
+    bool tm_valid = false;
+    CUtensorMap ta, tb;
+    void* hA = nullptr;  // device staging for run_host
+    void* hB = nullptr;
+    float* hbias = nullptr;
+    float* hC = nullptr;
+};
+
+namespace {
+
+struct CacheEntry {
+    nnjit_candidate cand;
+    int chosen_index;
+    int space_size;
+    int64_t naive;
+    std::vector<std::pair<int, double>> timings;
+    double tune_ms;
+    bool timed;
+};
+
+std::mutex g_cache_mu;
+std::map<std::string, CacheEntry>& cache() {
+    static std::map<std::string, CacheEntry> m;
+    return m;
+}
+
+std::mutex g_lim_mu;
+std::map<int, nnjit_device_limits> g_limits;
+std::map<int, std::string> g_dev_name;
+
+nnjit_status query_limits(int dev, nnjit_device_limits* out) {
+    {
+        std::lock_guard<std::mutex> lk(g_lim_mu);
+        auto it = g_limits.find(dev);
+        if (it != g_limits.end()) { *out = it->second; return NNJIT_OK; }
+    }
+    cudaDeviceProp prop;
+    cudaError_t e = cudaGetDeviceProperties(&prop, dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDeviceProperties");
+    nnjit_device_limits L{};
+    L.sm_count = prop.multiProcessorCount;
+    L.smem_per_sm = (int32_t)prop.sharedMemPerMultiprocessor;
+    L.smem_per_block_optin = (int32_t)prop.sharedMemPerBlockOptin;
+    L.regs_per_sm = prop.regsPerMultiprocessor;
+    L.max_threads_per_sm = prop.maxThreadsPerMultiProcessor;
+    L.max_blocks_per_sm = prop.maxBlocksPerMultiProcessor;
+    L.tmem_cols_per_sm = prop.major == 10 ? 512 : 0;
+    L.l2_bytes = prop.l2CacheSize;
+    L.cc_major = prop.major;
+    L.cc_minor = prop.minor;
+    std::lock_guard<std::mutex> lk(g_lim_mu);
+    g_limits[dev] = L;
+    g_dev_name[dev] = prop.name;
+    *out = L;
+    return NNJIT_OK;
+}
+
+std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L) {
+    char buf[512];
+    std::string name;
+    {
+        std::lock_guard<std::mutex> lk(g_lim_mu);
+        name = g_dev_name[dev];
+    }
+    std::snprintf(buf, sizeof buf,
+                  "t=matmul|s=%lld,%lld,%lld,%lld|dt=%d|bl=%d|ld=%lld,%lld,%lld|st=%lld,%lld,%lld|"
+                  "bias=%d|dev=%s,cc%d%d,sm%d",
+                  (long long)p.M, (long long)p.N, (long long)p.K, (long long)p.batch, p.dtype,
+                  p.b_layout, (long long)p.lda, (long long)p.ldb, (long long)p.ldc,
+                  (long long)p.stride_a, (long long)p.stride_b, (long long)p.stride_c, p.has_bias,
+                  name.c_str(), L.cc_major, L.cc_minor, L.sm_count);
+    return buf;
+}
+
+size_t ws_bytes_for(const Problem& p, const nnjit_candidate& c) {
+    if (c.split_k <= 1) return 0;
+    return (size_t)c.split_k * (size_t)p.batch * (size_t)p.M * (size_t)p.N * sizeof(float);
+}
+
+// Launch the plan's kernels for one product (the body of nnjit_matmul_run).
+nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* bias, float* C,
+                      cudaStream_t s, const nnjit_candidate* override_cand = nullptr,
+                      float* override_ws = nullptr) {
+    const Problem& p = pl->p;
+    const nnjit_candidate& c = override_cand ? *override_cand : pl->cand;
+    float* ws = override_ws ? override_ws : pl->ws;
+    if (p.M == 0 || p.N == 0) return NNJIT_OK;
+    if (!C) return fail(NNJIT_ERR_INVALID_ARG, "C is NULL");
+    if (p.K == 0) {
+        cudaError_t e = launch_fill_bias(p, bias, C, s);
+        return e == cudaSuccess ? NNJIT_OK : cuda_fail(e, "fill (K = 0)");
+    }
+    if (!A || !B) return fail(NNJIT_ERR_INVALID_ARG, "A or B is NULL");
+    const uintptr_t ua = reinterpret_cast<uintptr_t>(A), ub = reinterpret_cast<uintptr_t>(B);
+    if ((reinterpret_cast<uintptr_t>(C) & 3) || (bias && (reinterpret_cast<uintptr_t>(bias) & 3)))
+        return fail(NNJIT_ERR_INVALID_ARG, "C and bias must be 4-byte aligned");
+    if (c.family == NNJIT_FAMILY_FFMA) {
+        if ((ua & 3) || (ub & 3)) return fail(NNJIT_ERR_INVALID_ARG, "A and B must be 4-byte aligned");
+    } else if ((ua & 15) || (ub & 15)) {
+        return fail(NNJIT_ERR_UNSUPPORTED, "tensor-core and GEMV paths need 16-byte aligned A and B");
+    }
+    if (c.split_k > 1 && !ws) return fail(NNJIT_ERR_INVALID_ARG, "split-K workspace missing");
+    LaunchArgs la;
+    la.p = &p;
+    la.c = &c;
+    la.A = A;
+    la.B = B;
+    la.bias = c.split_k > 1 ? nullptr : bias;
+    la.C = C;
+    la.ws = ws;
+    la.err = pl->err;
+    la.stream = s;
+    cudaError_t e = cudaSuccess;
+    if (c.family == NNJIT_FAMILY_TC) {
+        CUtensorMap ta, tb;
+        const char* why = "";
+        {
+            std::lock_guard<std::mutex> lk(pl->mu);
+            if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B) {
+                e = encode_tc_tensor_maps(p, c, A, B, &ta, &tb, &why);
+                if (e != cudaSuccess) return fail(NNJIT_ERR_UNSUPPORTED, why);
+                if (!override_cand) {
+                    pl->ta = ta; pl->tb = tb; pl->tm_A = A; pl->tm_B = B; pl->tm_valid = true;
+                }
+            } else {
+                ta = pl->ta; tb = pl->tb;
+            }
+        }
+        la.tmap_a = &ta;
+        la.tmap_b = &tb;
+        e = launch_tc(la);
+    } else if (c.family == NNJIT_FAMILY_FFMA) {
+        e = launch_ffma(la);
+    } else {
+        e = launch_gemv(la);
+    }
+    if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+    if (c.split_k > 1) {
+        e = launch_splitk_reduce(ws, c.split_k, p, bias, C, s);
+        if (e != cudaSuccess) return cuda_fail(e, "split-K reduce launch");
+    }
+    return NNJIT_OK;
+}
+
+double now_ms() {
+    using namespace std::chrono;
+    return duration<double, std::milli>(steady_clock::now().time_since_epoch()).count();
+}
+
+struct DevBuf {
+    void* p = nullptr;
+    ~DevBuf() { if (p) cudaFree(p); }
+};
+
+// Tuning scratch: `sets` independent operand sets so that back-to-back repetitions do
+// not find their operands in L2 (rotation), plus one workspace big enough for any
+// candidate's split-K partials.
+struct Scratch {
+    DevBuf A, B, bias, C, ws;
+    int sets = 1;
+    size_t a_elems = 0, b_elems = 0, c_elems = 0;
+};
+
+nnjit_status make_scratch(const Problem& p, const std::vector<nnjit_candidate>& space,
+                          const nnjit_device_limits& L, Scratch* s) {
+    const int e = p.elem_bytes();
+    // element extents covering every batch item with the plan's strides
+    s->a_elems = (size_t)((p.batch - 1) * p.stride_a + (p.M - 1) * p.lda + p.K);
+    const int64_t b_rows = p.b_layout == NNJIT_B_KN ? p.K : p.N;
+    const int64_t b_cols = p.b_layout == NNJIT_B_KN ? p.N : p.K;
+    s->b_elems = (size_t)((p.batch - 1) * p.stride_b + (b_rows - 1) * p.ldb + b_cols);
+    s->c_elems = (size_t)((p.batch - 1) * p.stride_c + (p.M - 1) * p.ldc + p.N);
+    // round each set up to 256 bytes so every set keeps 16-byte alignment
+    auto r256 = [](size_t b) { return (b + 255) / 256 * 256; };
+    const size_t set_bytes = r256(s->a_elems * e) + r256(s->b_elems * e) + r256(s->c_elems * 4);
+    const size_t want = 3ull * (size_t)std::max(L.l2_bytes, 1);
+    size_t sets = (want + set_bytes - 1) / set_bytes;
+    sets = std::max<size_t>(1, std::min<size_t>(sets, 16));
+    while (sets > 1 && sets * set_bytes > (size_t)4 << 30) --sets;
+    s->sets = (int)sets;
+    size_t ws_max = 0;
+    for (const auto& c : space) ws_max = std::max(ws_max, ws_bytes_for(p, c));
+    cudaError_t err;
+    if ((err = cudaMalloc(&s->A.p, sets * r256(s->a_elems * e))) != cudaSuccess) return cuda_fail(err, "scratch A");
+    if ((err = cudaMalloc(&s->B.p, sets * r256(s->b_elems * e))) != cudaSuccess) return cuda_fail(err, "scratch B");
+    if ((err = cudaMalloc(&s->C.p, sets * r256(s->c_elems * 4))) != cudaSuccess) return cuda_fail(err, "scratch C");
+    if ((err = cudaMalloc(&s->bias.p, r256((size_t)p.N * 4))) != cudaSuccess) return cuda_fail(err, "scratch bias");
+    if (ws_max && (err = cudaMalloc(&s->ws.p, ws_max)) != cudaSuccess) return cuda_fail(err, "scratch workspace");
+    if ((err = launch_fill_scratch(s->A.p, (int64_t)(sets * r256(s->a_elems * e) / e), e, 1u, 0)) != cudaSuccess ||
+        (err = launch_fill_scratch(s->B.p, (int64_t)(sets * r256(s->b_elems * e) / e), e, 2u, 0)) != cudaSuccess ||
+        (err = launch_fill_scratch(s->bias.p, p.N, 4, 3u, 0)) != cudaSuccess)
+        return cuda_fail(err, "scratch fill");
+    err = cudaDeviceSynchronize();
+    if (err != cudaSuccess) return cuda_fail(err, "scratch fill sync");
+    return NNJIT_OK;
+}
+
+const void* set_ptr(const DevBuf& b, size_t elems, int e, int i) {
+    const size_t stride = (elems * e + 255) / 256 * 256;
+    return static_cast<const char*>(b.p) + (size_t)i * stride;
+}
+
+// Time one candidate: median over 3 trials of (R back-to-back launches rotating operand
+// sets, captured in a CUDA graph so host launch overhead is not measured) / R, in
+// microseconds.  Returns false if the candidate failed (it is then skipped); *fatal is
+// set for a sticky CUDA error.
+bool time_candidate(nnjit_plan pl, const nnjit_candidate& c, const Scratch& sc, int idx,
+                    const FaultSpec& fault, double* us, nnjit_status* fatal) {
+    const Problem& p = pl->p;
+    const int e = p.elem_bytes();
+    const float* bias = p.has_bias ? static_cast<const float*>(sc.bias.p) : nullptr;
+    float* ws = static_cast<float*>(sc.ws.p);
+    if (fault.kind == 1 && fault.index == idx) return false;
+    cudaStream_t s = nullptr;
+    if (cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking) != cudaSuccess) {
+        *fatal = fail(NNJIT_ERR_CUDA, "stream create");
+        return false;
+    }
+    struct StreamGuard {
+        cudaStream_t s;
+        ~StreamGuard() { cudaStreamDestroy(s); }
+    } sg{s};
+    auto launch = [&](int set) -> nnjit_status {
+        return run_impl(pl, set_ptr(sc.A, sc.a_elems, e, set), set_ptr(sc.B, sc.b_elems, e, set), bias,
+                        const_cast<float*>(static_cast<const float*>(set_ptr(sc.C, sc.c_elems, 4, set))),
+                        s, &c, ws);
+    };
+    auto sticky = [&](cudaError_t err, const char* what) {
+        cudaGetLastError();
+        if (cudaDeviceSynchronize() != cudaSuccess) *fatal = cuda_fail(err, what);
+    };
+    auto watchdog_fired = [&]() {
+        int word = 0;
+        cudaMemcpy(&word, pl->err, sizeof(int), cudaMemcpyDeviceToHost);
+        if (fault.kind == 2 && fault.index == idx) word = 0x1FF;
+        if (word != 0) cudaMemset(pl->err, 0, sizeof(int));
+        return word != 0;
+    };
+    nnjit_status st = launch(0);
+    cudaError_t err = cudaStreamSynchronize(s);
+    if (err != cudaSuccess) { sticky(err, "tuning launch"); return false; }
+    if (st != NNJIT_OK) return false;
+    if (watchdog_fired()) return false;
+    cudaEvent_t e0, e1;
+    cudaEventCreate(&e0);
+    cudaEventCreate(&e1);
+    struct EventGuard {
+        cudaEvent_t a, b;
+        ~EventGuard() { cudaEventDestroy(a); cudaEventDestroy(b); }
+    } eg{e0, e1};
+    // estimate one launch, then size the repetitions to ~1 ms of device time (3..50)
+    cudaEventRecord(e0, s);
+    launch(1 % sc.sets);
+    cudaEventRecord(e1, s);
+    cudaEventSynchronize(e1);
+    float ms1 = 0.f;
+    cudaEventElapsedTime(&ms1, e0, e1);
+    const int reps = (int)std::min(50.0, std::max(3.0, 1.0 / std::max(1e-4, (double)ms1)));
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    int set = 0;
+    bool captured = cudaStreamBeginCapture(s, cudaStreamCaptureModeThreadLocal) == cudaSuccess;
+    if (captured) {
+        for (int r = 0; r < reps; ++r) {
+            launch(set);
+            set = (set + 1) % sc.sets;
+        }
+        captured = cudaStreamEndCapture(s, &graph) == cudaSuccess && graph &&
+                   cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess;
+    }
+    if (!captured) cudaGetLastError();
+    std::vector<double> trials;
+    for (int t = 0; t < 3; ++t) {
+        cudaEventRecord(e0, s);
+        if (captured) {
+            cudaGraphLaunch(exec, s);
+        } else {
+            for (int r = 0; r < reps; ++r) {
+                launch(set);
+                set = (set + 1) % sc.sets;
+            }
+        }
+        cudaEventRecord(e1, s);
+        cudaEventSynchronize(e1);
+        float ms = 0.f;
+        cudaEventElapsedTime(&ms, e0, e1);
+        trials.push_back(1000.0 * ms / reps);
+    }
+    if (exec) cudaGraphExecDestroy(exec);
+    if (graph) cudaGraphDestroy(graph);
+    err = cudaStreamSynchronize(s);
+    if (err == cudaSuccess) err = cudaGetLastError();
+    if (err != cudaSuccess) { sticky(err, "tuning repetitions"); return false; }
+    if (watchdog_fired()) return false;
+    std::sort(trials.begin(), trials.end());
+    *us = trials[trials.size() / 2];
+    return true;
+}
+
+nnjit_status alloc_plan_buffers(nnjit_plan pl) {
+    cudaError_t e = cudaMalloc(&pl->err, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "watchdog word");
+    e = cudaMemset(pl->err, 0, sizeof(int));
+    if (e != cudaSuccess) return cuda_fail(e, "watchdog word");
+    pl->ws_bytes = ws_bytes_for(pl->p, pl->cand);
+    if (pl->ws_bytes) {
+        e = cudaMalloc(&pl->ws, pl->ws_bytes);
+        if (e != cudaSuccess) return cuda_fail(e, "split-K workspace");
+    }
+    return NNJIT_OK;
+}
+
+void free_plan(nnjit_plan pl) {
+    if (!pl) return;
+    if (pl->err) cudaFree(pl->err);
+    if (pl->ws) cudaFree(pl->ws);
+    if (pl->hA) cudaFree(pl->hA);
+    if (pl->hB) cudaFree(pl->hB);
+    if (pl->hbias) cudaFree(pl->hbias);
+    if (pl->hC) cudaFree(pl->hC);
+    delete pl;
+}
+
+nnjit_status plan_common(const nnjit_matmul_desc* d, nnjit_plan* out, Problem* prob,
+                         nnjit_device_limits* L, int* dev, std::vector<nnjit_candidate>* space,
+                         int64_t* naive) {
+    if (!out) return fail(NNJIT_ERR_INVALID_ARG, "out is NULL");
+    *out = nullptr;
+    std::string err;
+    nnjit_status st = resolve_problem(d, prob, &err);
+    if (st != NNJIT_OK) return fail(st, err);
+    cudaError_t e = cudaGetDevice(dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    e = cudaFree(nullptr);  // make sure a context exists
+    if (e != cudaSuccess) return cuda_fail(e, "context");
+    st = query_limits(*dev, L);
+    if (st != NNJIT_OK) return st;
+    st = build_space(*prob, *L, space, naive, &err);
+    if (st != NNJIT_OK) return fail(st, err);
+    return NNJIT_OK;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------------ C ABI
+extern "C" {
+
+const char* nnjit_status_string(nnjit_status s) {
+    switch (s) {
+        case NNJIT_OK: return "NNJIT_OK";
+        case NNJIT_ERR_INVALID_ARG: return "NNJIT_ERR_INVALID_ARG";
+        case NNJIT_ERR_UNSUPPORTED: return "NNJIT_ERR_UNSUPPORTED";
+        case NNJIT_ERR_CUDA: return "NNJIT_ERR_CUDA";
+        case NNJIT_ERR_OOM: return "NNJIT_ERR_OOM";
+        case NNJIT_ERR_TIMEOUT: return "NNJIT_ERR_TIMEOUT";
+        case NNJIT_ERR_BUDGET: return "NNJIT_ERR_BUDGET";
+    }
+    return "NNJIT_ERR_UNKNOWN";
+}
+
+const char* nnjit_last_error(void) { return t_last_error.c_str(); }
+
+int32_t nnjit_version(void) { return 100; }
+
+nnjit_status nnjit_device_limits_query(int32_t device, nnjit_device_limits* out) {
+    if (!out) return fail(NNJIT_ERR_INVALID_ARG, "out is NULL");
+    return query_limits(device, out);
+}
+
+nnjit_status nnjit_space_enumerate(const nnjit_matmul_desc* d, const nnjit_device_limits* lim,
+                                   nnjit_candidate* out, int32_t capacity, int32_t* count,
+                                   int64_t* naive_count) {
+    if (!lim || !count || capacity < 0 || (capacity > 0 && !out))
+        return fail(NNJIT_ERR_INVALID_ARG, "bad output arguments");
+    Problem p;
+    std::string err;
+    nnjit_status st = resolve_problem(d, &p, &err);
+    if (st != NNJIT_OK) return fail(st, err);
+    std::vector<nnjit_candidate> v;
+    int64_t naive = 0;
+    st = build_space(p, *lim, &v, &naive, &err);
+    if (st != NNJIT_OK) return fail(st, err);
+    *count = (int32_t)v.size();
+    for (int32_t i = 0; i < capacity && i < (int32_t)v.size(); ++i) out[i] = v[i];
+    if (naive_count) *naive_count = naive;
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, nnjit_plan* out) {
+    const double t0 = now_ms();
+    if (!(budget_ms >= 0.0)) return fail(NNJIT_ERR_INVALID_ARG, "tune_budget_ms must be >= 0");
+    Problem p;
+    nnjit_device_limits L;
+    int dev = 0;
+    std::vector<nnjit_candidate> space;
+    int64_t naive = 0;
+    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive);
+    if (st != NNJIT_OK) return st;
+    std::unique_ptr<nnjit_plan_s> pl(new nnjit_plan_s);
+    pl->p = p;
+    pl->device = dev;
+    pl->family = space[0].family;
+    pl->space_size = (int)space.size();
+    pl->naive = naive;
+    const bool use_cache = !(p.flags & NNJIT_PLAN_NO_CACHE) && !(p.flags & NNJIT_PLAN_EXHAUSTIVE);
+    const std::string key = cache_key(p, dev, L);
+    if (use_cache) {
+        std::lock_guard<std::mutex> lk(g_cache_mu);
+        auto it = cache().find(key);
+        if (it != cache().end()) {
+            const CacheEntry& ce = it->second;
+            pl->cand = ce.cand;
+            pl->chosen_index = ce.chosen_index;
+            pl->timings = ce.timings;
+            pl->tune_ms = ce.tune_ms;
+            pl->timed = ce.timed;
+            pl->from_cache = true;
+        }
+    }
+    if (!pl->from_cache) {
+        const bool require = (p.flags & NNJIT_PLAN_REQUIRE_TIMED) != 0;
+        const bool exhaustive = (p.flags & NNJIT_PLAN_EXHAUSTIVE) != 0;
+        if (p.degenerate() || (budget_ms == 0.0 && !exhaustive)) {
+            if (!p.degenerate() && require)
+                return fail(NNJIT_ERR_BUDGET, "budget 0 with NNJIT_PLAN_REQUIRE_TIMED");
+            pl->cand = space[0];
+            pl->chosen_index = 0;
+        } else {
+            // the plan's watchdog word is needed while timing candidates
+            cudaError_t e = cudaMalloc(&pl->err, sizeof(int));
+            if (e != cudaSuccess) return cuda_fail(e, "watchdog word");
+            cudaMemset(pl->err, 0, sizeof(int));
+            Scratch sc;
+            st = make_scratch(p, space, L, &sc);
+            if (st != NNJIT_OK) { cudaFree(pl->err); pl->err = nullptr; return st; }
+            const FaultSpec fault = read_fault();
+            const bool log = env_flag("NNJIT_LOG");
+            std::vector<std::pair<int, double>> timed;
+            nnjit_status fatal = NNJIT_OK;
+            for (int i = 0; i < (int)space.size(); ++i) {
+                if (!exhaustive && !timed.empty() && now_ms() - t0 >= budget_ms) break;
+                double us = 0.0;
+                if (time_candidate(pl.get(), space[i], sc, i, fault, &us, &fatal)) {
+                    timed.emplace_back(i, us);
+                    if (log) std::fprintf(stderr, "[nnjit] cand %d family %d bn %d split %d: %.3f us\n",
+                                          i, space[i].family, space[i].bn, space[i].split_k, us);
+                } else {
+                    pl->failed.push_back(i);
+                    if (log) std::fprintf(stderr, "[nnjit] cand %d failed (skipped)\n", i);
+                }
+                if (fatal != NNJIT_OK) { cudaFree(pl->err); pl->err = nullptr; return fatal; }
+            }
+            if (timed.empty()) {
+                cudaFree(pl->err);
+                pl->err = nullptr;
+                return fail(NNJIT_ERR_CUDA, "every timed candidate failed");
+            }
+            // Re-time the three fastest interleaved (noise between the first pass and now
+            // hits all of them alike); keep the fastest re-timed one, ties to lower index.
+            std::vector<std::pair<int, double>> order = timed;
+            std::stable_sort(order.begin(), order.end(),
+                             [](const std::pair<int, double>& a, const std::pair<int, double>& b) {
+                                 return a.second < b.second;
+                             });
+            const int top = std::min<int>(3, (int)order.size());
+            std::vector<std::vector<double>> again(top);
+            if (top > 1) {
+                for (int round = 0; round < 3; ++round)
+                    for (int j = 0; j < top; ++j) {
+                        double us = 0.0;
+                        if (time_candidate(pl.get(), space[order[j].first], sc, order[j].first,
+                                           FaultSpec{}, &us, &fatal))
+                            again[j].push_back(us);
+                        if (fatal != NNJIT_OK) { cudaFree(pl->err); pl->err = nullptr; return fatal; }
+                    }
+            }
+            int best = order[0].first;
+            double best_us = 1e300;
+            for (int j = 0; j < top; ++j) {
+                double med = order[j].second;
+                if (!again[j].empty()) {
+                    std::sort(again[j].begin(), again[j].end());
+                    med = again[j][again[j].size() / 2];
+                }
+                if (med < best_us || (med == best_us && order[j].first < best)) {
+                    best_us = med;
+                    best = order[j].first;
+                }
+                for (auto& t : timed)
+                    if (t.first == order[j].first) t.second = med;
+            }
+            pl->cand = space[best];
+            pl->chosen_index = best;
+            pl->timings = timed;
+            pl->timed = true;
+            cudaFree(pl->err);
+            pl->err = nullptr;
+        }
+        pl->tune_ms = now_ms() - t0;
+        if (use_cache) {
+            CacheEntry ce{pl->cand, pl->chosen_index, pl->space_size, pl->naive, pl->timings,
+                          pl->tune_ms, pl->timed};
+            std::lock_guard<std::mutex> lk(g_cache_mu);
+            cache()[key] = ce;
+        }
+    }
+    st = alloc_plan_buffers(pl.get());
+    if (st != NNJIT_OK) { free_plan(pl.release()); return st; }
+    *out = pl.release();
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_matmul_plan(int64_t M, int64_t N, int64_t K, nnjit_dtype dt, double budget_ms,
+                               nnjit_plan* out) {
+    nnjit_matmul_desc d{};
+    d.M = M; d.N = N; d.K = K; d.batch = 1;
+    d.dtype = dt;
+    d.b_layout = NNJIT_B_KN;
+    d.has_bias = 1;
+    return nnjit_matmul_plan_ex(&d, budget_ms, out);
+}
+
+nnjit_status nnjit_matmul_plan_candidate(const nnjit_matmul_desc* d, int32_t index, nnjit_plan* out) {
+    Problem p;
+    nnjit_device_limits L;
+    int dev = 0;
+    std::vector<nnjit_candidate> space;
+    int64_t naive = 0;
+    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive);
+    if (st != NNJIT_OK) return st;
+    if (index < 0 || index >= (int32_t)space.size())
+        return fail(NNJIT_ERR_INVALID_ARG, "candidate index out of range");
+    std::unique_ptr<nnjit_plan_s> pl(new nnjit_plan_s);
+    pl->p = p;
+    pl->device = dev;
+    pl->family = space[index].family;
+    pl->cand = space[index];
+    pl->chosen_index = index;
+    pl->space_size = (int)space.size();
+    pl->naive = naive;
+    st = alloc_plan_buffers(pl.get());
+    if (st != NNJIT_OK) { free_plan(pl.release()); return st; }
+    *out = pl.release();
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_matmul_run(nnjit_plan p, const void* A, const void* B, const float* bias,
+                              float* C, void* stream) {
+    if (!p) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    return run_impl(p, A, B, bias, C, static_cast<cudaStream_t>(stream));
+}
+
+nnjit_status nnjit_matmul_run_batched(nnjit_plan p, const void* A, const void* B, float* C,
+                                      void* stream) {
+    if (!p) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    return run_impl(p, A, B, nullptr, C, static_cast<cudaStream_t>(stream));
+}
+
+nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB,
+                                   const float* hbias, float* hC, void* stream) {
+    if (!pl) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    const Problem& p = pl->p;
+    const int64_t b_rows = p.b_layout == NNJIT_B_KN ? p.K : p.N;
+    const int64_t b_cols = p.b_layout == NNJIT_B_KN ? p.N : p.K;
+    const bool packed = p.lda == std::max<int64_t>(p.K, 1) && p.ldb == std::max<int64_t>(b_cols, 1) &&
+                        p.ldc == std::max<int64_t>(p.N, 1) && p.stride_a == p.M * p.lda &&
+                        p.stride_b == b_rows * p.ldb && p.stride_c == p.M * p.ldc;
+    if (!packed) return fail(NNJIT_ERR_UNSUPPORTED, "run_host needs a packed plan");
+    if (p.M == 0 || p.N == 0) return NNJIT_OK;
+    if (!hC || (p.K > 0 && (!hA || !hB))) return fail(NNJIT_ERR_INVALID_ARG, "NULL host buffer");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const size_t e = (size_t)p.elem_bytes();
+    const size_t a_bytes = (size_t)(p.batch * p.M * p.K) * e;
+    const size_t b_bytes = (size_t)(p.batch * p.K * p.N) * e;
+    const size_t c_bytes = (size_t)(p.batch * p.M * p.N) * 4;
+    {
+        std::lock_guard<std::mutex> lk(pl->mu);
+        cudaError_t err = cudaSuccess;
+        if (!pl->hA && a_bytes && (err = cudaMalloc(&pl->hA, a_bytes)) != cudaSuccess) return cuda_fail(err, "staging A");
+        if (!pl->hB && b_bytes && (err = cudaMalloc(&pl->hB, b_bytes)) != cudaSuccess) return cuda_fail(err, "staging B");
+        if (!pl->hbias && (err = cudaMalloc(&pl->hbias, (size_t)p.N * 4)) != cudaSuccess) return cuda_fail(err, "staging bias");
+        if (!pl->hC && (err = cudaMalloc(&pl->hC, c_bytes)) != cudaSuccess) return cuda_fail(err, "staging C");
+    }
+    cudaError_t err;
+    if (a_bytes && (err = cudaMemcpyAsync(pl->hA, hA, a_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(err, "copy A");
+    if (b_bytes && (err = cudaMemcpyAsync(pl->hB, hB, b_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(err, "copy B");
+    if (hbias && (err = cudaMemcpyAsync(pl->hbias, hbias, (size_t)p.N * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
+        return cuda_fail(err, "copy bias");
+    nnjit_status st = run_impl(pl, pl->hA, pl->hB, hbias ? pl->hbias : nullptr, pl->hC, s);
+    if (st != NNJIT_OK) return st;
+    if ((err = cudaMemcpyAsync(hC, pl->hC, c_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
+        return cuda_fail(err, "copy C");
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_plan_check(nnjit_plan p) {
+    if (!p) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    int cur = 0;
+    cudaGetDevice(&cur);
+    if (cur != p->device) cudaSetDevice(p->device);
+    cudaError_t e = cudaDeviceSynchronize();
+    int word = 0;
+    if (e == cudaSuccess) e = cudaMemcpy(&word, p->err, sizeof(int), cudaMemcpyDeviceToHost);
+    if (e == cudaSuccess && word != 0) cudaMemset(p->err, 0, sizeof(int));
+    if (cur != p->device) cudaSetDevice(cur);
+    if (e != cudaSuccess) return cuda_fail(e, "plan check");
+    if (word != 0) {
+        char buf[96];
+        std::snprintf(buf, sizeof buf, "kernel watchdog expired (code 0x%x)", word);
+        return fail(NNJIT_ERR_TIMEOUT, buf);
+    }
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_plan_candidate(nnjit_plan p, nnjit_candidate* out) {
+    if (!p || !out) return fail(NNJIT_ERR_INVALID_ARG, "NULL argument");
+    *out = p->cand;
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_plan_describe(nnjit_plan pl, char* buf, size_t len, size_t* needed) {
+    if (!pl) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    const Problem& p = pl->p;
+    const nnjit_candidate& c = pl->cand;
+    std::string s;
+    char tmp[1024];
+    std::snprintf(tmp, sizeof tmp,
+                  "{\"M\":%lld,\"N\":%lld,\"K\":%lld,\"batch\":%lld,\"dtype\":%d,\"b_layout\":%d,"
+                  "\"family\":%d,\"chosen_index\":%d,\"space_size\":%d,\"naive_space\":%lld,"
+                  "\"tune_ms\":%.3f,\"from_cache\":%s,\"timed\":%s,"
+                  "\"candidate\":{\"bm\":%d,\"bn\":%d,\"bk\":%d,\"tm\":%d,\"tn\":%d,\"stages\":%d,"
+                  "\"split_k\":%d,\"raster\":%d,\"threads\":%d,\"smem_bytes\":%d,\"tmem_cols\":%d,"
+                  "\"regs_per_thread\":%d,\"blocks_per_sm\":%d,\"grid\":%d,\"wave_eff_ppm\":%d,"
+                  "\"instance\":%d,\"predicted_cost\":%lld},\"timings_us\":[",
+                  (long long)p.M, (long long)p.N, (long long)p.K, (long long)p.batch, p.dtype,
+                  p.b_layout, pl->family, pl->chosen_index, pl->space_size, (long long)pl->naive,
+                  pl->tune_ms, pl->from_cache ? "true" : "false", pl->timed ? "true" : "false",
+                  c.bm, c.bn, c.bk, c.tm, c.tn, c.stages, c.split_k, c.raster, c.threads,
+                  c.smem_bytes, c.tmem_cols, c.regs_per_thread, c.blocks_per_sm, c.grid,
+                  c.wave_eff_ppm, c.instance, (long long)c.predicted_cost);
+    s += tmp;
+    for (size_t i = 0; i < pl->timings.size(); ++i) {
+        std::snprintf(tmp, sizeof tmp, "%s[%d,%.4f]", i ? "," : "", pl->timings[i].first,
+                      pl->timings[i].second);
+        s += tmp;
+    }
+    s += "],\"failed\":[";
+    for (size_t i = 0; i < pl->failed.size(); ++i) {
+        std::snprintf(tmp, sizeof tmp, "%s%d", i ? "," : "", pl->failed[i]);
+        s += tmp;
+    }
+    s += "]}";
+    if (needed) *needed = s.size() + 1;
+    if (buf && len > 0) {
+        const size_t n = std::min(len - 1, s.size());
+        std::memcpy(buf, s.data(), n);
+        buf[n] = '\0';
+    }
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_plan_destroy(nnjit_plan p) {
+    free_plan(p);
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_cache_clear(void) {
+    std::lock_guard<std::mutex> lk(g_cache_mu);
+    cache().clear();
+    return NNJIT_OK;
+}
+
+int32_t nnjit_cache_size(void) {
+    std::lock_guard<std::mutex> lk(g_cache_mu);
+    return (int32_t)cache().size();
+}
+
+}  // extern "C"

@@ -1,0 +1,431 @@
+// Tensor-core GEMM for sm_103a: TMA -> shared-memory ring -> tcgen05.mma (cta_group::1,
+// M = 128) -> TMEM f32 accumulators -> tcgen05.ld epilogue (+ bias) -> f32 global stores.
+//
+// This is the tensor-core member of the kernel family the JIT tunes (the MatMul and
+// BatchMatMul operators of Table 3).  One CTA per SM runs persistently over output tiles
+// of BM x BN = 128 x BN; per tile it streams K in blocks of 128 bytes (64 bf16 / 32 tf32
+// elements), so every shared-memory row is one 128-byte swizzle row.
+//
+// Warp roles (192 threads):
+//   warp 0      TMA producer: waits "empty[s]", arms "full[s]" with the stage bytes and
+//               issues the A and B tile loads.
+//   warp 1      TMEM owner and MMA issuer: waits "full[s]", issues BK/UMMA_K MMAs into
+//               accumulator buffer (tile & 1), commits to "empty[s]"; after the last
+//               k-block commits to "tmem_full[acc]".
+//   warps 2..5  epilogue: wait "tmem_full[acc]", tcgen05.ld 32 columns at a time, add
+//               bias, store f32; then arrive on "tmem_empty[acc]" (128 arrivals).
+// Two accumulator buffers let the epilogue of one tile overlap the mainloop of the next.
+// Every wait is bounded (ptx::mbar_wait); an expired wait records an error code in the
+// plan's watchdog word, all roles leave their loops, in-flight copies and MMAs are
+// drained (bounded), TMEM is freed and the CTA exits.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+#include <mutex>
+
+#include "launch.h"
+#include "ptx.cuh"
+
+namespace nnjit {
+
+namespace {
+
+constexpr int kBM = 128;
+constexpr int kThreads = 192;
+constexpr int kMaxStages = 8;
+
+struct TcParams {
+    CUtensorMap tmap_a;  // A [batch][M][K]: dims {K, M, batch}, box {BK, 128, 1}
+    CUtensorMap tmap_b;  // NK: dims {K, N, batch}, box {BK, BN, 1}; KN: dims {N, K, batch}, box {atom, BK, 1}
+    float* C;
+    const float* bias;
+    float* ws;
+    int* err;
+    int M, N, K, batch;
+    long long ldc, stride_c;
+    int num_kb, split, tiles_m, tiles_n, total_tiles, stages, raster;
+};
+
+struct TileCoord {
+    int b, s, tm, tn;
+};
+
+__device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p) {
+    TileCoord c;
+    const int per = p.tiles_m * p.tiles_n;
+    const int r = t % per;
+    const int q = t / per;
+    c.s = q % p.split;
+    c.b = q / p.split;
+    if (p.raster == 0) {
+        c.tm = r % p.tiles_m;
+        c.tn = r / p.tiles_m;
+    } else {
+        c.tn = r % p.tiles_n;
+        c.tm = r / p.tiles_n;
+    }
+    return c;
+}
+
+// Error codes written to the watchdog word: 0x100 | role << 4 | which wait.
+constexpr int kErrProducerEmpty = 0x101;
+constexpr int kErrMmaTmemEmpty = 0x111;
+constexpr int kErrMmaFull = 0x112;
+constexpr int kErrEpiTmemFull = 0x121;
+constexpr int kErrDrain = 0x131;
+
+template <int kKind, bool kBMn, int BN>
+__global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
+    constexpr int kElem = kKind == 0 ? 2 : 4;
+    constexpr int BK = 128 / kElem;                     // K elements per stage (one swizzle row)
+    constexpr int kUmmaK = 32 / kElem;                  // K per MMA instruction (32 bytes)
+    constexpr int kKSteps = BK / kUmmaK;                // 4
+    constexpr int kAtom = 128 / kElem;                  // MN-major swizzle atom width (elements)
+    constexpr uint32_t kABytes = kBM * 128;             // 16 KB
+    constexpr uint32_t kBBytes = BN * 128;
+    constexpr uint32_t kStageBytes = kABytes + kBBytes;
+    constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
+    constexpr uint32_t kIdesc = ptx::instr_desc(kKind == 0 ? 1u : 2u, kBMn, kBM, BN);
+
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~static_cast<uintptr_t>(1023));
+    const int S = p.stages;
+    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * kStageBytes);
+    // bars[0..S): full, [S..2S): empty, 2S..2S+1: tmem_full, 2S+2..2S+3: tmem_empty,
+    // 2S+4: drain
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kMaxStages + 5);
+    volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t smem_base = ptx::smem_u32(smem);
+    auto full_bar = [&](int s) { return ptx::smem_u32(bars + s); };
+    auto empty_bar = [&](int s) { return ptx::smem_u32(bars + S + s); };
+    auto tfull_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + a); };
+    auto tempty_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + 2 + a); };
+    const uint32_t drain_bar = ptx::smem_u32(bars + 2 * S + 4);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < S; ++s) {
+            ptx::mbar_init(full_bar(s), 1);
+            ptx::mbar_init(empty_bar(s), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            ptx::mbar_init(tfull_bar(a), 1);
+            ptx::mbar_init(tempty_bar(a), 4 * 32);
+        }
+        ptx::mbar_init(drain_bar, 1);
+        *abort_flag = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        ptx::prefetch_tmap(&p.tmap_a);
+        ptx::prefetch_tmap(&p.tmap_b);
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(tmem_slot), kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem_base = *tmem_slot;
+
+    if (warp == 0) {
+        // ---------------------------------------------------------------- TMA producer
+        int stage = 0;
+        uint32_t phase = 0;
+        uint32_t armed = 0, armed_parity = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+            const TileCoord tc = decode_tile(t, p);
+            const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
+            const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
+            for (int kb = kb0; kb < kb1; ++kb) {
+                if (!ptx::mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, p.err,
+                                    kErrProducerEmpty)) {
+                    ok = false;
+                    break;
+                }
+                if (lane == 0) {
+                    const uint32_t sa = smem_base + stage * kStageBytes;
+                    const uint32_t sb = sa + kABytes;
+                    ptx::mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
+                    ptx::tma_load_3d(sa, &p.tmap_a, kb * BK, tc.tm * kBM, tc.b, full_bar(stage));
+                    if constexpr (!kBMn) {
+                        ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, full_bar(stage));
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < BN / kAtom; ++j)
+                            ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom,
+                                             kb * BK, tc.b, full_bar(stage));
+                    }
+                }
+                __syncwarp();
+                armed |= 1u << stage;
+                armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
+                if (++stage == S) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+        }
+        // Drain: every load this warp issued has landed before the CTA may exit.
+        for (int s = 0; s < S; ++s) {
+            if (armed & (1u << s)) {
+                volatile int no_abort = 0;
+                ptx::mbar_wait(full_bar(s), (armed_parity >> s) & 1u, &no_abort, p.err, kErrDrain,
+                               ptx::kWaitLimitNs / 4);
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------------- MMA issuer
+        int stage = 0;
+        uint32_t phase = 0;
+        uint32_t iter = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x, ++iter) {
+            const TileCoord tc = decode_tile(t, p);
+            const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
+            const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
+            const uint32_t acc = iter & 1u;
+            const uint32_t acc_phase = (iter >> 1) & 1u;
+            if (!ptx::mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty)) {
+                ok = false;
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t d_tmem = tmem_base + acc * BN;
+            for (int kb = kb0; kb < kb1; ++kb) {
+                if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull)) {
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+                if (lane == 0) {
+                    const uint32_t sa = smem_base + stage * kStageBytes;
+                    const uint32_t sb = sa + kABytes;
+#pragma unroll
+                    for (int kk = 0; kk < kKSteps; ++kk) {
+                        const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
+                        uint64_t bdesc;
+                        if constexpr (!kBMn)
+                            bdesc = ptx::smem_desc_sw128(sb + kk * 32, 16, 1024);
+                        else
+                            bdesc = ptx::smem_desc_sw128(sb + kk * kUmmaK * 128, BK * 128, 1024);
+                        ptx::mma_ss<kKind>(d_tmem, adesc, bdesc, kIdesc,
+                                           (kb > kb0 || kk > 0) ? 1u : 0u);
+                    }
+                    ptx::tc_commit(empty_bar(stage));
+                }
+                __syncwarp();
+                if (++stage == S) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            if (!ok) break;
+            if (lane == 0) ptx::tc_commit(tfull_bar(acc));
+            __syncwarp();
+        }
+        // Drain: all MMAs this thread issued have completed before TMEM is released.
+        if (lane == 0) ptx::tc_commit(drain_bar);
+        __syncwarp();
+        volatile int no_abort = 0;
+        ptx::mbar_wait(drain_bar, 0, &no_abort, p.err, kErrDrain, ptx::kWaitLimitNs / 4);
+    } else {
+        // ---------------------------------------------------------------- epilogue
+        const int q = warp & 3;              // TMEM sub-partition this warp may access
+        const int row_in_tile = q * 32 + lane;
+        uint32_t iter = 0;
+        const long long MN = (long long)p.M * p.N;
+        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++iter) {
+            const TileCoord tc = decode_tile(t, p);
+            const uint32_t acc = iter & 1u;
+            const uint32_t acc_phase = (iter >> 1) & 1u;
+            if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
+            ptx::tc_fence_after();
+            const int row = tc.tm * kBM + row_in_tile;
+            float* dst_row;
+            const float* bias = nullptr;
+            if (p.split == 1) {
+                dst_row = p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc;
+                bias = p.bias;
+            } else {
+                dst_row = p.ws + ((long long)tc.s * p.batch + tc.b) * MN + (long long)row * p.N;
+            }
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                uint32_t r[32];
+                const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32;
+                ptx::tmem_ld32(taddr, r);
+                ptx::tmem_wait_ld(r);
+                const int col0 = tc.tn * BN + c * 32;
+                if (row < p.M) {
+                    float v[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+                    if (bias) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (col0 + j < p.N) v[j] += __ldg(bias + col0 + j);
+                    }
+                    float* dst = dst_row + col0;
+                    if (col0 + 32 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+#pragma unroll
+                        for (int j = 0; j < 32; j += 4)
+                            *reinterpret_cast<float4*>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (col0 + j < p.N) dst[j] = v[j];
+                    }
+                }
+            }
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(tempty_bar(acc));
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem_base, kTmemCols);
+}
+
+using TcKernel = void (*)(TcParams);
+
+// Instance table, indexed as tc_instance(): ((dtype_i * 2 + kn) * 3 + bn_i).
+const TcKernel kTcKernels[12] = {
+    tc_gemm_kernel<0, false, 64>, tc_gemm_kernel<0, false, 128>, tc_gemm_kernel<0, false, 256>,
+    tc_gemm_kernel<0, true, 64>,  tc_gemm_kernel<0, true, 128>,  tc_gemm_kernel<0, true, 256>,
+    tc_gemm_kernel<1, false, 64>, tc_gemm_kernel<1, false, 128>, tc_gemm_kernel<1, false, 256>,
+    tc_gemm_kernel<1, true, 64>,  tc_gemm_kernel<1, true, 128>,  tc_gemm_kernel<1, true, 256>,
+};
+
+std::mutex g_prep_mu;
+int g_prepared_smem[12] = {0};
+
+// Driver entry point for cuTensorMapEncodeTiled, fetched through the runtime so the
+// library does not link against libcuda.
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    static std::once_flag once;
+    std::call_once(once, [] {
+        void* ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPoint("cuTensorMapEncodeTiled", &ptr, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    });
+    return fn;
+}
+
+}  // namespace
+
+cudaError_t prepare_tc_instance(int instance, int smem_bytes) {
+    if (instance < 0 || instance >= 12) return cudaErrorInvalidValue;
+    std::lock_guard<std::mutex> lk(g_prep_mu);
+    if (g_prepared_smem[instance] >= smem_bytes) return cudaSuccess;
+    cudaError_t e = cudaFuncSetAttribute(kTcKernels[instance],
+                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+    if (e == cudaSuccess) g_prepared_smem[instance] = smem_bytes;
+    return e;
+}
+
+cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,
+                                  const void* B, CUtensorMap* ta, CUtensorMap* tb,
+                                  const char** why) {
+    EncodeTiledFn enc = get_encode_fn();
+    if (!enc) {
+        *why = "cuTensorMapEncodeTiled entry point unavailable";
+        return cudaErrorNotSupported;
+    }
+    const int e = p.elem_bytes();
+    const CUtensorMapDataType dt =
+        p.dtype == NNJIT_BF16 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32;
+    const cuuint32_t bk = 128 / e;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    {
+        const cuuint64_t dims[3] = {(cuuint64_t)p.K, (cuuint64_t)p.M, (cuuint64_t)p.batch};
+        const cuuint64_t strides[2] = {(cuuint64_t)(p.lda * e), (cuuint64_t)(p.stride_a * e)};
+        const cuuint32_t box[3] = {bk, (cuuint32_t)kBM, 1};
+        CUresult r = enc(ta, dt, 3, const_cast<void*>(A), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) {
+            *why = "cuTensorMapEncodeTiled failed for A";
+            return cudaErrorInvalidValue;
+        }
+    }
+    {
+        cuuint64_t dims[3];
+        cuuint32_t box[3];
+        if (p.b_layout == NNJIT_B_NK) {
+            dims[0] = (cuuint64_t)p.K; dims[1] = (cuuint64_t)p.N;
+            box[0] = bk; box[1] = (cuuint32_t)c.bn;
+        } else {
+            dims[0] = (cuuint64_t)p.N; dims[1] = (cuuint64_t)p.K;
+            box[0] = 128 / e; box[1] = bk;
+        }
+        dims[2] = (cuuint64_t)p.batch;
+        box[2] = 1;
+        const cuuint64_t strides[2] = {(cuuint64_t)(p.ldb * e), (cuuint64_t)(p.stride_b * e)};
+        CUresult r = enc(tb, dt, 3, const_cast<void*>(B), dims, strides, box, estr,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+        if (r != CUDA_SUCCESS) {
+            *why = "cuTensorMapEncodeTiled failed for B";
+            return cudaErrorInvalidValue;
+        }
+    }
+    return cudaSuccess;
+}
+
+cudaError_t launch_tc(const LaunchArgs& a) {
+    const Problem& p = *a.p;
+    const nnjit_candidate& c = *a.c;
+    if (c.instance < 0 || c.instance >= 12 || !a.tmap_a || !a.tmap_b) return cudaErrorInvalidValue;
+    if (c.stages < 2 || c.stages > kMaxStages) return cudaErrorInvalidValue;
+    TcParams prm;
+    prm.tmap_a = *a.tmap_a;
+    prm.tmap_b = *a.tmap_b;
+    prm.C = a.C;
+    prm.bias = a.bias;
+    prm.ws = a.ws;
+    prm.err = a.err;
+    prm.M = (int)p.M;
+    prm.N = (int)p.N;
+    prm.K = (int)p.K;
+    prm.batch = (int)p.batch;
+    prm.ldc = p.ldc;
+    prm.stride_c = p.stride_c;
+    prm.num_kb = (int)((p.K + c.bk - 1) / c.bk);
+    prm.split = c.split_k;
+    prm.tiles_m = (int)((p.M + kBM - 1) / kBM);
+    prm.tiles_n = (int)((p.N + c.bn - 1) / c.bn);
+    const long long total = (long long)p.batch * c.split_k * prm.tiles_m * prm.tiles_n;
+    if (total >= (1LL << 31)) return cudaErrorInvalidValue;
+    if (c.split_k > prm.num_kb) return cudaErrorInvalidValue;  // every split owns >= 1 k-block
+    prm.total_tiles = (int)total;
+    prm.stages = c.stages;
+    prm.raster = c.raster;
+    const int grid = (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
+    // ring + alignment slack + barriers/TMEM slot/abort flag
+    const int stage_bytes = (kBM + c.bn) * 128;
+    const int smem = c.stages * stage_bytes + 1024 + 256;
+    cudaError_t e = prepare_tc_instance(c.instance, smem);
+    if (e != cudaSuccess) return e;
+    kTcKernels[c.instance]<<<grid, kThreads, smem, a.stream>>>(prm);
+    return cudaGetLastError();
+}
+
+}  // namespace nnjit

@@ -1,0 +1,56 @@
+// Internal interface between the C-ABI layer (capi.cu) and the kernel translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "space.h"
+
+namespace nnjit {
+
+// Everything one launch of the plan's main kernel needs.
+struct LaunchArgs {
+    const Problem* p = nullptr;
+    const nnjit_candidate* c = nullptr;
+    const void* A = nullptr;
+    const void* B = nullptr;
+    const float* bias = nullptr;   // NULL: no bias
+    float* C = nullptr;
+    float* ws = nullptr;           // split-K partials [split][batch][M][N], or NULL if split == 1
+    int* err = nullptr;            // device watchdog word
+    cudaStream_t stream = nullptr;
+    const CUtensorMap* tmap_a = nullptr;  // TC family only
+    const CUtensorMap* tmap_b = nullptr;
+};
+
+// Main kernels.  Each returns the launch status (cudaGetLastError after the launch).
+cudaError_t launch_ffma(const LaunchArgs& a);
+cudaError_t launch_gemv(const LaunchArgs& a);
+cudaError_t launch_tc(const LaunchArgs& a);
+
+// C[b,m,n] = sum_{s < split} ws[s][b][m][n] (+ bias[n]), s ascending.
+cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, const float* bias,
+                                 float* C, cudaStream_t s);
+
+// C = bias broadcast over rows (or 0 when bias is NULL): the K = 0 product.
+cudaError_t launch_fill_bias(const Problem& p, const float* bias, float* C, cudaStream_t s);
+
+// Arbitrary finite data for tuning scratch buffers (not the test inputs).
+cudaError_t launch_fill_scratch(void* dst, int64_t n_elems, int elem_bytes, uint32_t seed,
+                                cudaStream_t s);
+
+// Write `bytes` of `buf` (evicts the L2 between timed repetitions).
+cudaError_t launch_l2_flush(void* buf, int64_t bytes, cudaStream_t s);
+
+// One-time per-process kernel attribute setup (opt-in shared memory).  Idempotent.
+cudaError_t prepare_tc_instance(int instance, int smem_bytes);
+cudaError_t prepare_gemv_instance(int instance, int smem_bytes);
+
+// Tensor maps for the TC family (host; uses the driver entry point).
+cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,
+                                  const void* B, CUtensorMap* ta, CUtensorMap* tb,
+                                  const char** why);
+
+}  // namespace nnjit

@@ -1,0 +1,423 @@
+// Lite kernel-configuration space: descriptor resolution, family choice, enumeration,
+// pruning by hardware-usage formulas and ordering (Sec. 5.2, Table 1, Table 2).
+#include "space.h"
+
+#include <algorithm>
+#include <cstdio>
+
+namespace nnjit {
+
+namespace {
+
+int64_t ceil_div(int64_t a, int64_t b) { return (a + b - 1) / b; }
+
+int64_t pow2_ceil(int64_t x) {
+    int64_t p = 1;
+    while (p < x) p <<= 1;
+    return p;
+}
+
+int min4(int a, int b, int c, int d) { return std::min(std::min(a, b), std::min(c, d)); }
+
+// Block_core of Table 1 generalised: the number of CTAs one SM can hold is the smallest
+// of the per-resource limits (registers, shared memory = L1Limit, warps, TMEM, blocks).
+int blocks_per_core(const nnjit_device_limits& L, int regs, int threads, int smem, int tmem) {
+    const int reg_lim = L.regs_per_sm / std::max(1, regs * threads);
+    const int smem_lim = smem > 0 ? L.smem_per_sm / smem : L.max_blocks_per_sm;
+    const int warp_lim = (L.max_threads_per_sm / 32) / std::max(1, threads / 32);
+    const int tmem_lim = tmem > 0 ? L.tmem_cols_per_sm / tmem : L.max_blocks_per_sm;
+    return std::min(min4(reg_lim, smem_lim, warp_lim, tmem_lim), L.max_blocks_per_sm);
+}
+
+nnjit_candidate blank() {
+    nnjit_candidate c{};
+    c.split_k = 1;
+    c.instance = -1;
+    return c;
+}
+
+// ---------------------------------------------------------------------------------
+// tcgen05 tensor-core family.  The CTA tile is BM x BN with BM = 128 (one cta_group::1
+// UMMA covers 128 TMEM lanes).  BK is fixed at one 128-byte swizzle row of K (64 bf16,
+// 32 tf32): the Blackwell counterpart of the paper's "consistent" primitive settings
+// (Sec. 5.1), fixed once instead of searched.  The searched axes are BN, split-K and
+// the tile raster order; the stage count is derived, not searched: the ring fills the
+// shared memory a CTA may opt in to (the counterpart of heuristic 7, "use all of the
+// fastest storage").
+// ---------------------------------------------------------------------------------
+void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_candidate>& v,
+              int64_t* naive) {
+    using MC = ModelConstants;
+    const int e = p.elem_bytes();
+    const int BM = MC::kTcBM, BK = 128 / e;
+    const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
+    const int64_t K = std::max<int64_t>(p.K, 1);
+    const int64_t num_kb = ceil_div(K, BK);
+    const int bns[3] = {64, 128, 256};
+    const int splits[4] = {1, 2, 4, 8};
+    *naive = 3 * (MC::kTcMaxStages - 1) * 4 * 2;  // BN x stage count 2..8 x split x raster
+    for (int bn : bns) {
+        if (bn > 64 && bn > pow2_ceil(N)) continue;  // no tile wider than the padded N
+        const int stage_bytes = (BM + bn) * 128;
+        const int stages = std::min(MC::kTcMaxStages,
+                                    (L.smem_per_block_optin - MC::kTcFixedSmem) / stage_bytes);
+        if (stages < 2) continue;
+        const int smem = stages * stage_bytes + MC::kTcFixedSmem;
+        const int tmem = (int)pow2_ceil(std::max(32, 2 * bn));  // two accumulator buffers
+        if (tmem > L.tmem_cols_per_sm) continue;
+        const int threads = MC::kTcThreads, regs = MC::kTcRegsPerThread;
+        const int blk = blocks_per_core(L, regs, threads, smem, tmem);
+        if (blk < 1) continue;
+        const int64_t tiles_m = ceil_div(M, BM), tiles_n = ceil_div(N, bn);
+        const int64_t tiles = p.batch * tiles_m * tiles_n;
+        for (int split : splits) {
+            // split only while the previous split count still leaves SMs idle
+            if (split > 1 && (tiles * (split / 2) >= L.sm_count || num_kb < 4 * split)) continue;
+            for (int raster = 0; raster < 2; ++raster) {
+                if (raster == 1 && (tiles_m == 1 || tiles_n == 1)) continue;
+                nnjit_candidate c = blank();
+                c.family = NNJIT_FAMILY_TC;
+                c.bm = BM; c.bn = bn; c.bk = BK;
+                c.tm = 0; c.tn = 0;
+                c.stages = stages;
+                c.split_k = split;
+                c.raster = raster;
+                c.threads = threads;
+                c.smem_bytes = smem;
+                c.tmem_cols = tmem;
+                c.regs_per_thread = regs;
+                c.blocks_per_sm = blk;
+                const int64_t work = tiles * split;
+                const int64_t slots = (int64_t)L.sm_count * blk;
+                const int64_t grid = std::min(work, slots);
+                const int64_t waves = ceil_div(work, grid);
+                c.grid = (int32_t)grid;
+                c.wave_eff_ppm = (int32_t)(work * 1000000 / (waves * grid));
+                // per k-block: MMA clocks (2*BN for both bf16 and tf32 at BK = 128 bytes)
+                // against the operand feed (stage bytes over the per-SM L2 feed)
+                const int64_t t_kb = std::max<int64_t>(2 * bn, ceil_div(stage_bytes,
+                                                                        MC::kFeedBytesPerClk));
+                int64_t cost = waves * t_kb * ceil_div(num_kb, split);
+                if (split > 1)
+                    cost += MC::kLaunchClk +
+                            ceil_div(2LL * split * p.batch * M * N * 4, MC::kHbmBytesPerClk);
+                c.predicted_cost = cost;
+                c.instance = tc_instance(p.dtype, p.b_layout, bn);
+                v.push_back(c);
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------
+// FP32-FFMA SIMT family: the direct descendant of the paper's WebGPU tile template
+// (Table 2): thread tile x0 = y0 in {4, 8} (inner range [4..32]), block tile x1, y1 in
+// {32, 64, 128} (range [32..256]), r1 = BK in {8, 16}, r0 = 1.  Table 1's usage formulas
+// are applied as written; heuristic 5 (Thread_block <= 256) is kept, the WebGPU 16 KB
+// limit of heuristic 6 becomes the CTA's shared-memory limit.
+// ---------------------------------------------------------------------------------
+void ffma_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_candidate>& v,
+                int64_t* naive) {
+    using MC = ModelConstants;
+    const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
+    const int64_t K = std::max<int64_t>(p.K, 1);
+    const int tiles_x[3] = {32, 64, 128};
+    const int bks[2] = {8, 16};
+    const int splits[4] = {1, 2, 4, 8};
+    *naive = 2 * 3 * 3 * 2 * 4;
+    for (int t0 : {4, 8}) {
+        for (int bm : tiles_x) {
+            for (int bn : tiles_x) {
+                const int threads = (bm / t0) * (bn / t0);       // Thread_block
+                if (threads < 64 || threads > 256) continue;     // >= 2 warps; heuristic 5
+                if ((bm > 32 && bm > pow2_ceil(M)) || (bn > 32 && bn > pow2_ceil(N))) continue;
+                for (int bk : bks) {
+                    // Table 1: Reg_thread = x0 r0 + r0 y0 + x0 y0 (r0 = 1), divided by the
+                    // relaxation share for the kernel's other variables.
+                    const int reg_paper = t0 * 1 + 1 * t0 + t0 * t0;
+                    const int regs = (int)ceil_div(reg_paper * 100, MC::kRegRelaxPct);
+                    // shared memory: double-buffered A and B tiles, rows padded by 4 floats
+                    const int smem = 2 * bk * ((bm + 4) + (bn + 4)) * 4;
+                    if (smem > L.smem_per_block_optin) continue;
+                    const int blk = blocks_per_core(L, regs, threads, smem, 0);
+                    if (blk < 1) continue;
+                    const int64_t tiles = p.batch * ceil_div(M, bm) * ceil_div(N, bn);
+                    for (int split : splits) {
+                        if (split > 1 && (tiles * (split / 2) >= L.sm_count || K < 2LL * split * bk))
+                            continue;
+                        nnjit_candidate c = blank();
+                        c.family = NNJIT_FAMILY_FFMA;
+                        c.bm = bm; c.bn = bn; c.bk = bk;
+                        c.tm = t0; c.tn = t0;
+                        c.stages = 2;
+                        c.split_k = split;
+                        c.threads = threads;
+                        c.smem_bytes = smem;
+                        c.regs_per_thread = regs;
+                        c.blocks_per_sm = blk;
+                        const int64_t grid = tiles * split;
+                        const int64_t slots = (int64_t)L.sm_count * blk;
+                        const int64_t waves = ceil_div(grid, slots);
+                        c.grid = (int32_t)grid;
+                        c.wave_eff_ppm = (int32_t)(grid * 1000000 / (waves * slots));
+                        const int64_t per_sm = ceil_div(grid, L.sm_count);
+                        const int64_t resident = std::min<int64_t>(per_sm, blk);
+                        const int64_t warps = resident * threads / 32;
+                        const int64_t util_pct = std::min<int64_t>(100, std::max<int64_t>(1, warps * 100 / 16));
+                        int64_t cost = per_sm * ceil_div((int64_t)bm * bn * ceil_div(K, split), 128) *
+                                       100 / util_pct;
+                        if (split > 1)
+                            cost += MC::kLaunchClk +
+                                    ceil_div(2LL * split * p.batch * M * N * 4, MC::kHbmBytesPerClk);
+                        c.predicted_cost = cost;
+                        c.instance = ffma_instance(t0, bm, bn, bk, p.b_layout);
+                        v.push_back(c);
+                    }
+                }
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------
+// Split-K GEMV family (M <= 8, bf16 weights): bandwidth-bound, so the axes are those
+// that set the bytes in flight per SM: threads per CTA, rows per warp, 16-byte loads in
+// flight per lane and row (unroll), and split-K.
+// ---------------------------------------------------------------------------------
+void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_candidate>& v,
+                int64_t* naive) {
+    using MC = ModelConstants;
+    const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
+    const int64_t K = std::max<int64_t>(p.K, 1);
+    const int64_t wbytes = N * K * 2;
+    if (p.b_layout == NNJIT_B_NK) {
+        *naive = 2 * 3 * 2 * 4;
+        for (int threads : {128, 256}) {
+            for (int rows : {1, 2, 4}) {
+                for (int unroll : {2, 4}) {
+                    const int warps = threads / 32;
+                    const int64_t ctas_n = ceil_div(N, (int64_t)warps * rows);
+                    for (int split : {1, 2, 4, 8}) {
+                        const int64_t kper = ceil_div(ceil_div(K, split), 8) * 8;
+                        if (split > 1 && (kper < 256LL * unroll ||
+                                          ctas_n * (split / 2) >= 2LL * L.sm_count))
+                            continue;
+                        const int64_t smem = ceil_div(M * kper * 2, 16) * 16;
+                        if (smem > MC::kGemvMaxSmem || smem > L.smem_per_block_optin) continue;
+                        const int regs = 40 + rows * (int)M + 4 * unroll * rows + 8;
+                        const int blk = blocks_per_core(L, regs, threads, (int)smem, 0);
+                        if (blk < 1) continue;
+                        nnjit_candidate c = blank();
+                        c.family = NNJIT_FAMILY_GEMV;
+                        c.bm = (int)M; c.bn = warps * rows; c.bk = (int)std::min<int64_t>(kper, 1 << 30);
+                        c.tm = rows; c.tn = 1;
+                        c.stages = unroll;
+                        c.split_k = split;
+                        c.threads = threads;
+                        c.smem_bytes = (int)smem;
+                        c.regs_per_thread = regs;
+                        c.blocks_per_sm = blk;
+                        const int64_t grid = ctas_n * split;
+                        const int64_t slots = (int64_t)L.sm_count * blk;
+                        const int64_t waves = ceil_div(grid, slots);
+                        c.grid = (int32_t)grid;
+                        c.wave_eff_ppm = (int32_t)(grid * 1000000 / (waves * slots));
+                        const int64_t resident = std::min<int64_t>(ceil_div(grid, L.sm_count), blk);
+                        const int64_t inflight = resident * threads * unroll * rows * 16;
+                        const int64_t eff_pct = std::min<int64_t>(100, std::max<int64_t>(1, inflight * 100 / 32768));
+                        int64_t cost = ceil_div(wbytes, MC::kHbmBytesPerClk) * 100 / eff_pct;
+                        if (split > 1)
+                            cost += MC::kLaunchClk +
+                                    ceil_div(2LL * split * M * N * 4, MC::kHbmBytesPerClk);
+                        c.predicted_cost = cost;
+                        c.instance = gemv_instance(p.b_layout, rows, unroll);
+                        v.push_back(c);
+                    }
+                }
+            }
+        }
+    } else {
+        *naive = 2 * 2 * 6;
+        for (int threads : {128, 256}) {
+            for (int unroll : {2, 4}) {
+                const int warps = threads / 32;
+                const int64_t ctas_n = ceil_div(N, 256);
+                for (int split : {1, 2, 4, 8, 16, 32}) {
+                    const int64_t kper = ceil_div(K, split);
+                    if (split > 1 && (kper < (int64_t)warps * unroll ||
+                                      ctas_n * (split / 2) >= 2LL * L.sm_count))
+                        continue;
+                    const int64_t smem = (int64_t)warps * M * 256 * 4;
+                    if (smem > MC::kGemvMaxSmem || smem > L.smem_per_block_optin) continue;
+                    const int regs = 40 + 8 * (int)M + 4 * unroll + 8;
+                    const int blk = blocks_per_core(L, regs, threads, (int)smem, 0);
+                    if (blk < 1) continue;
+                    nnjit_candidate c = blank();
+                    c.family = NNJIT_FAMILY_GEMV;
+                    c.bm = (int)M; c.bn = 256; c.bk = (int)std::min<int64_t>(kper, 1 << 30);
+                    c.tm = 1; c.tn = 8;
+                    c.stages = unroll;
+                    c.split_k = split;
+                    c.threads = threads;
+                    c.smem_bytes = (int)smem;
+                    c.regs_per_thread = regs;
+                    c.blocks_per_sm = blk;
+                    const int64_t grid = ctas_n * split;
+                    const int64_t slots = (int64_t)L.sm_count * blk;
+                    const int64_t waves = ceil_div(grid, slots);
+                    c.grid = (int32_t)grid;
+                    c.wave_eff_ppm = (int32_t)(grid * 1000000 / (waves * slots));
+                    const int64_t resident = std::min<int64_t>(ceil_div(grid, L.sm_count), blk);
+                    const int64_t inflight = resident * threads * unroll * 16;
+                    const int64_t eff_pct = std::min<int64_t>(100, std::max<int64_t>(1, inflight * 100 / 32768));
+                    int64_t cost = ceil_div(wbytes, MC::kHbmBytesPerClk) * 100 / eff_pct;
+                    if (split > 1)
+                        cost += MC::kLaunchClk + ceil_div(2LL * split * M * N * 4, MC::kHbmBytesPerClk);
+                    c.predicted_cost = cost;
+                    c.instance = gemv_instance(p.b_layout, 1, unroll);
+                    v.push_back(c);
+                }
+            }
+        }
+    }
+}
+
+}  // namespace
+
+int tc_instance(int dtype, int b_layout, int bn) {
+    const int bi = bn == 64 ? 0 : bn == 128 ? 1 : bn == 256 ? 2 : -1;
+    if (bi < 0) return -1;
+    const int di = dtype == NNJIT_BF16 ? 0 : 1;
+    return (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
+}
+
+// The 12 (thread tile, block tile) pairs with 64..256 threads, in enumeration order.
+static const int kFfmaTiles[12][3] = {
+    {4, 32, 32}, {4, 32, 64}, {4, 32, 128}, {4, 64, 32}, {4, 64, 64}, {4, 128, 32},
+    {8, 32, 128}, {8, 64, 64}, {8, 64, 128}, {8, 128, 32}, {8, 128, 64}, {8, 128, 128}};
+
+int ffma_instance(int tm, int bm, int bn, int bk, int b_layout) {
+    int ti = -1;
+    for (int i = 0; i < 12; ++i)
+        if (kFfmaTiles[i][0] == tm && kFfmaTiles[i][1] == bm && kFfmaTiles[i][2] == bn) ti = i;
+    if (ti < 0 || (bk != 8 && bk != 16)) return -1;
+    return (ti * 2 + (bk == 16 ? 1 : 0)) * 2 + (b_layout == NNJIT_B_NK ? 1 : 0);
+}
+
+int gemv_instance(int b_layout, int rows, int unroll) {
+    const int ui = unroll == 2 ? 0 : unroll == 4 ? 1 : -1;
+    if (ui < 0) return -1;
+    if (b_layout == NNJIT_B_KN) return rows == 1 ? 6 + ui : -1;
+    const int ri = rows == 1 ? 0 : rows == 2 ? 1 : rows == 4 ? 2 : -1;
+    if (ri < 0) return -1;
+    return ri * 2 + ui;
+}
+
+nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string* err) {
+    if (!d || !p) { *err = "descriptor is NULL"; return NNJIT_ERR_INVALID_ARG; }
+    if (d->M < 0 || d->N < 0 || d->K < 0) { *err = "M, N, K must be >= 0"; return NNJIT_ERR_INVALID_ARG; }
+    if (d->batch < 1) { *err = "batch must be >= 1"; return NNJIT_ERR_INVALID_ARG; }
+    if (d->dtype < NNJIT_F32_FFMA || d->dtype > NNJIT_BF16) { *err = "unknown dtype"; return NNJIT_ERR_INVALID_ARG; }
+    if (d->b_layout != NNJIT_B_KN && d->b_layout != NNJIT_B_NK) { *err = "unknown b_layout"; return NNJIT_ERR_INVALID_ARG; }
+    if (d->has_bias != 0 && d->has_bias != 1) { *err = "has_bias must be 0 or 1"; return NNJIT_ERR_INVALID_ARG; }
+    const int64_t lim = (int64_t)1 << 31;
+    if (d->M >= lim || d->N >= lim || d->K >= lim || d->batch >= lim) {
+        *err = "dimensions must be < 2^31"; return NNJIT_ERR_INVALID_ARG;
+    }
+    if (d->lda < 0 || d->ldb < 0 || d->ldc < 0 || d->stride_a < 0 || d->stride_b < 0 || d->stride_c < 0) {
+        *err = "leading dimensions and strides must be >= 0"; return NNJIT_ERR_INVALID_ARG;
+    }
+    Problem q;
+    q.M = d->M; q.N = d->N; q.K = d->K; q.batch = d->batch;
+    q.dtype = d->dtype; q.b_layout = d->b_layout; q.has_bias = d->has_bias; q.flags = d->flags;
+    const int64_t b_rows = q.b_layout == NNJIT_B_KN ? q.K : q.N;
+    const int64_t b_cols = q.b_layout == NNJIT_B_KN ? q.N : q.K;
+    q.lda = d->lda ? d->lda : std::max<int64_t>(q.K, 1);
+    q.ldb = d->ldb ? d->ldb : std::max<int64_t>(b_cols, 1);
+    q.ldc = d->ldc ? d->ldc : std::max<int64_t>(q.N, 1);
+    if (q.lda < q.K) { *err = "lda < K"; return NNJIT_ERR_INVALID_ARG; }
+    if (q.ldb < b_cols) { *err = "ldb smaller than the row length of B"; return NNJIT_ERR_INVALID_ARG; }
+    if (q.ldc < q.N) { *err = "ldc < N"; return NNJIT_ERR_INVALID_ARG; }
+    q.stride_a = d->stride_a ? d->stride_a : q.M * q.lda;
+    q.stride_b = d->stride_b ? d->stride_b : b_rows * q.ldb;
+    q.stride_c = d->stride_c ? d->stride_c : q.M * q.ldc;
+    if (q.batch > 1 && q.stride_c < q.M * q.ldc) {
+        *err = "stride_c smaller than one C matrix: batch items would overlap";
+        return NNJIT_ERR_INVALID_ARG;
+    }
+    const int64_t elim = (int64_t)1 << 40;
+    if (q.batch * std::max<int64_t>(q.stride_a, q.M * q.lda) >= elim ||
+        q.batch * std::max<int64_t>(q.stride_b, b_rows * q.ldb) >= elim ||
+        q.batch * std::max<int64_t>(q.stride_c, q.M * q.ldc) >= elim) {
+        *err = "operand extent too large"; return NNJIT_ERR_INVALID_ARG;
+    }
+    *p = q;
+    return NNJIT_OK;
+}
+
+nnjit_status choose_family(const Problem& p, int* family, std::string* err) {
+    if (p.dtype == NNJIT_F32_FFMA) { *family = NNJIT_FAMILY_FFMA; return NNJIT_OK; }
+    const int e = p.elem_bytes();
+    if (p.dtype == NNJIT_BF16 && p.M <= ModelConstants::kGemvMaxM && p.batch == 1) {
+        if (!p.degenerate() && ((p.lda * e) % 16 != 0 || (p.ldb * e) % 16 != 0)) {
+            *err = "GEMV path needs 16-byte aligned rows of A and B (lda, ldb multiples of 8)";
+            return NNJIT_ERR_UNSUPPORTED;
+        }
+        *family = NNJIT_FAMILY_GEMV;
+        return NNJIT_OK;
+    }
+    if (!p.degenerate()) {
+        if ((p.lda * e) % 16 != 0 || (p.ldb * e) % 16 != 0) {
+            *err = "tensor-core path needs 16-byte aligned row strides (TMA): lda*elem and "
+                   "ldb*elem must be multiples of 16 bytes";
+            return NNJIT_ERR_UNSUPPORTED;
+        }
+        if (p.batch > 1 && ((p.stride_a * e) % 16 != 0 || (p.stride_b * e) % 16 != 0)) {
+            *err = "tensor-core path needs 16-byte aligned batch strides";
+            return NNJIT_ERR_UNSUPPORTED;
+        }
+    }
+    *family = NNJIT_FAMILY_TC;
+    return NNJIT_OK;
+}
+
+nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
+                         std::vector<nnjit_candidate>* out, int64_t* naive, std::string* err) {
+    if (lim.sm_count <= 0 || lim.smem_per_sm <= 0 || lim.smem_per_block_optin <= 0 ||
+        lim.regs_per_sm <= 0 || lim.max_threads_per_sm <= 0 || lim.max_blocks_per_sm <= 0 ||
+        lim.tmem_cols_per_sm < 0) {
+        *err = "device limits must be positive";
+        return NNJIT_ERR_INVALID_ARG;
+    }
+    int family = 0;
+    nnjit_status st = choose_family(p, &family, err);
+    if (st != NNJIT_OK) return st;
+    std::vector<nnjit_candidate> v;
+    int64_t nv = 0;
+    if (family == NNJIT_FAMILY_TC) {
+        if (lim.cc_major != 10 || lim.tmem_cols_per_sm < 128) {
+            *err = "tensor-core family needs an sm_10x device with tensor memory";
+            return NNJIT_ERR_UNSUPPORTED;
+        }
+        tc_space(p, lim, v, &nv);
+    } else if (family == NNJIT_FAMILY_FFMA) {
+        ffma_space(p, lim, v, &nv);
+    } else {
+        gemv_space(p, lim, v, &nv);
+    }
+    if (v.empty()) {
+        *err = "no candidate fits the device limits";
+        return NNJIT_ERR_UNSUPPORTED;
+    }
+    // Evaluation order (Sec. 5.2): most blocks per core first; then the predicted cost;
+    // ties keep enumeration order.
+    std::stable_sort(v.begin(), v.end(), [](const nnjit_candidate& a, const nnjit_candidate& b) {
+        if (a.blocks_per_sm != b.blocks_per_sm) return a.blocks_per_sm > b.blocks_per_sm;
+        return a.predicted_cost < b.predicted_cost;
+    });
+    *out = std::move(v);
+    if (naive) *naive = nv;
+    return NNJIT_OK;
+}
+
+}  // namespace nnjit

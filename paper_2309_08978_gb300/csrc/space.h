@@ -1,0 +1,61 @@
+// Lite kernel-configuration space (host only).
+//
+// Sec. 5.2 and Table 1 of the paper: tile sizes decide how a kernel uses registers,
+// L1/shared memory, threads and warps; formulas of those usages plus a few heuristics
+// prune the space to a few dozen candidates, evaluated from the most to the fewest
+// blocks per core.  This file restates that scheme for three sm_103a kernel families.
+#pragma once
+
+#include <cstdint>
+#include <string>
+#include <vector>
+
+#include "../../include/nnjit.h"
+
+namespace nnjit {
+
+// Descriptor with every default resolved and validated.
+struct Problem {
+    int64_t M = 0, N = 0, K = 0, batch = 1;
+    int dtype = NNJIT_BF16;
+    int b_layout = NNJIT_B_NK;
+    int64_t lda = 0, ldb = 0, ldc = 0;
+    int64_t stride_a = 0, stride_b = 0, stride_c = 0;
+    int has_bias = 0;
+    uint32_t flags = 0;
+    int elem_bytes() const { return dtype == NNJIT_BF16 ? 2 : 4; }
+    bool degenerate() const { return M == 0 || N == 0 || K == 0; }
+};
+
+// Model constants of the ordering cost (readings; see the design notes).
+struct ModelConstants {
+    static constexpr int kFeedBytesPerClk = 64;      // L2->SM operand feed per SM
+    static constexpr int kHbmBytesPerClk = 3500;     // chip-wide HBM bytes per SM clock
+    static constexpr int kLaunchClk = 2000;          // cost of one extra kernel launch
+    static constexpr int kRegRelaxPct = 50;          // Table 1 register formula covers half
+    static constexpr int kTcRegsPerThread = 72;      // tcgen05 kernel: ptxas reports 64-65, allocated in 8s
+    static constexpr int kTcThreads = 192;           // 6 warps: TMA, MMA, 4 x epilogue
+    static constexpr int kTcBM = 128;
+    static constexpr int kTcFixedSmem = 1024 + 256;  // 1 KB alignment slack + barriers
+    static constexpr int kTcMaxStages = 8;
+    static constexpr int kGemvMaxM = 8;
+    static constexpr int kGemvMaxSmem = 64 * 1024;
+};
+
+// Resolve defaults and validate.  Returns NNJIT_OK or an error with `err` set.
+nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string* err);
+
+// Which family serves the problem (a1 of the hot path), or UNSUPPORTED with `err`.
+nnjit_status choose_family(const Problem& p, int* family, std::string* err);
+
+// Build the ordered lite space.  naive = size before pruning.
+nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
+                         std::vector<nnjit_candidate>* out, int64_t* naive, std::string* err);
+
+// Precompiled-instance index helpers (kept in one place so the registry and the space
+// agree).
+int tc_instance(int dtype, int b_layout, int bn);            // 0..11
+int ffma_instance(int tm, int bm, int bn, int bk, int b_layout);  // 0..47, -1 if none
+int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if none
+
+}  // namespace nnjit

@@ -1,0 +1,78 @@
+"""The C-ABI library builds, loads without a GPU, and exports every function that
+include/nnjit.h declares; host-only entry points behave as documented."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2309_08978_gb300.build_lib import build
+    path = build()
+    return ctypes.CDLL(path)
+
+
+def _declared():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        if h.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", h)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names |= set(re.findall(r"\b(nnjit_[a-z0-9_]+)\s*\(", src))
+    return sorted(names)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert "nnjit_matmul_plan" in names and "nnjit_matmul_run" in names
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, f"declared but not exported: {missing}"
+
+
+def test_status_strings_and_version(lib):
+    import paper_2309_08978_gb300 as nj
+    assert nj.nnjit_status_string(0) == "NNJIT_OK"
+    assert nj.nnjit_status_string(5) == "NNJIT_ERR_TIMEOUT"
+    assert nj.nnjit_status_string(99) == "NNJIT_ERR_UNKNOWN"
+    assert nj.nnjit_version() >= 100
+
+
+def test_null_plan_arguments_are_rejected(lib):
+    import paper_2309_08978_gb300 as nj
+    st = nj.load_library().nnjit_matmul_run(None, None, None, None, None, None)
+    assert st == nj.NNJIT_ERR_INVALID_ARG
+    assert "plan" in nj.nnjit_last_error()
+    assert nj.load_library().nnjit_plan_destroy(None) == nj.NNJIT_OK
+
+
+def test_invalid_descriptors(lib):
+    import paper_2309_08978_gb300 as nj
+    from conftest_limits import gb300_limits
+    L = gb300_limits()
+    bad = [nj.make_desc(-1, 4, 4, "bf16"), nj.make_desc(4, 4, 4, "bf16", batch=0),
+           nj.make_desc(4, 4, 4, 7), nj.make_desc(4, 4, 4, "bf16", b_layout=5),
+           nj.make_desc(4, 4, 8, "bf16", lda=4), nj.make_desc(4, 8, 4, "bf16", "KN", ldb=4),
+           nj.make_desc(4, 8, 4, "bf16", ldc=7)]
+    for d in bad:
+        with pytest.raises(nj.NnjitError) as ei:
+            nj.nnjit_space_enumerate(d, L)
+        assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
+
+
+def test_unaligned_tensor_core_strides_unsupported(lib):
+    import paper_2309_08978_gb300 as nj
+    from conftest_limits import gb300_limits
+    L = gb300_limits()
+    with pytest.raises(nj.NnjitError) as ei:
+        nj.nnjit_space_enumerate(nj.make_desc(64, 64, 30, "bf16", "NK"), L)   # 60-byte rows
+    assert ei.value.status == nj.NNJIT_ERR_UNSUPPORTED
+    with pytest.raises(nj.NnjitError) as ei:
+        nj.nnjit_space_enumerate(nj.make_desc(64, 30, 64, "tf32", "KN"), L)   # 120-byte rows of B
+    assert ei.value.status == nj.NNJIT_ERR_UNSUPPORTED
+    # the exact FFMA path takes any stride
+    cands, _ = nj.nnjit_space_enumerate(nj.make_desc(64, 30, 31, "f32_ffma", "KN"), L)
+    assert cands and all(c["family"] == nj.NNJIT_FAMILY_FFMA for c in cands)

@@ -1,0 +1,154 @@
+"""GPU parity: the CUDA path through the C ABI against the oracle, element by element.
+
+Integer-valued inputs in [-8, 8] are exact in bf16, tf32 and f32, and every partial sum
+stays below 2^24, so every kernel must reproduce the oracle bit for bit in any
+summation order (split-K included).  Random inputs with the workloads' distributions are
+held to the relative-Frobenius tolerances 1e-5 (FP32-FFMA), 5e-3 (TF32), 1e-2 (BF16).
+Shapes span several tiles and ragged tails in M, N and K.
+"""
+import numpy as np
+import pytest
+
+from synthetic import Shape, make_operands
+from gpu_util import run_plan, compare
+
+pytestmark = pytest.mark.gpu
+
+nj = pytest.importorskip("paper_2309_08978_gb300")
+
+
+def _plan(shape, dtype, budget=0.0, flags=0, **kw):
+    desc = nj.make_desc(shape.M, shape.N, shape.K, dtype, shape.b_layout, batch=shape.batch,
+                        has_bias=shape.has_bias, flags=flags, **kw)
+    return nj.nnjit_matmul_plan_ex(desc, budget)
+
+
+FFMA_SHAPES = [(1, 1, 1, "KN"), (7, 63, 65, "NK"), (129, 130, 67, "KN"), (64, 768, 768, "KN"),
+               (33, 257, 40, "NK")]
+TC_BF16_SHAPES = [(9, 40, 24, "NK"), (129, 200, 72, "NK"), (300, 264, 136, "KN"),
+                  (256, 512, 1024, "NK"), (130, 72, 200, "KN"), (512, 768, 64, "NK")]
+TC_TF32_SHAPES = [(5, 36, 12, "NK"), (130, 96, 100, "KN"), (257, 300, 68, "NK"),
+                  (64, 768, 768, "KN"), (512, 768, 256, "NK")]
+GEMV_SHAPES = [(1, 1, 8, "NK"), (1, 7, 16, "NK"), (3, 300, 520, "NK"), (8, 4096, 256, "NK"),
+               (1, 1000, 4104, "NK"), (2, 300, 520, "KN"), (1, 513, 4096, "KN"), (8, 33, 24, "KN")]
+
+CASES = ([("f32_ffma",) + s for s in FFMA_SHAPES] + [("bf16",) + s for s in TC_BF16_SHAPES] +
+         [("tf32",) + s for s in TC_TF32_SHAPES] + [("bf16",) + s for s in GEMV_SHAPES])
+
+
+def _ids(c):
+    return f"{c[0]}-{c[1]}x{c[2]}x{c[3]}-{c[4]}"
+
+
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+@pytest.mark.parametrize("with_bias", [False, True])
+def test_exact_integer_inputs(case, with_bias):
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, with_bias)
+    A, B, bias = make_operands(shape, 7, dtype, ints=True)
+    with _plan(shape, dtype) as plan:
+        C = run_plan(plan, A, B, bias, M, N)
+    compare(C, A, B, bias, layout, dtype, exact=True)
+
+
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_random_inputs_tolerance(case):
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    A, B, bias = make_operands(shape, 8, dtype)
+    with _plan(shape, dtype) as plan:
+        C = run_plan(plan, A, B, bias, M, N)
+    compare(C, A, B, bias, layout, dtype)
+
+
+EVERY_CANDIDATE = [("f32_ffma", 64, 768, 768, "KN"), ("f32_ffma", 100, 90, 300, "NK"),
+                   ("tf32", 64, 768, 768, "KN"), ("tf32", 200, 300, 520, "NK"),
+                   ("bf16", 300, 520, 1040, "NK"), ("bf16", 200, 600, 520, "KN"),
+                   ("bf16", 1, 4096, 4096, "NK"), ("bf16", 4, 1000, 2048, "KN")]
+
+
+@pytest.mark.parametrize("case", EVERY_CANDIDATE, ids=_ids)
+def test_every_candidate_is_exact(case):
+    """Legality invariant of the lite space: every enumerated candidate launches and
+    reproduces the oracle exactly on integer inputs."""
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    A, B, bias = make_operands(shape, 9, dtype, ints=True)
+    desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True)
+    lim = nj.nnjit_device_limits_query(0)
+    cands, _ = nj.nnjit_space_enumerate(desc, lim)
+    assert 1 <= len(cands) <= 64
+    for i, c in enumerate(cands):
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            C = run_plan(plan, A, B, bias, M, N)
+        try:
+            compare(C, A, B, bias, layout, dtype, exact=True)
+        except AssertionError as e:
+            raise AssertionError(f"candidate {i} {c}: {e}") from None
+
+
+BATCHED = [("bf16", 3, 130, 72, 64, "NK"), ("bf16", 4, 256, 64, 256, "KN"),
+           ("tf32", 2, 129, 40, 36, "NK"), ("bf16", 5, 64, 128, 128, "NK"),
+           ("f32_ffma", 3, 33, 20, 17, "KN")]
+
+
+@pytest.mark.parametrize("case", BATCHED, ids=lambda c: f"{c[0]}-b{c[1]}-{c[2]}x{c[3]}x{c[4]}-{c[5]}")
+@pytest.mark.parametrize("exact", [True, False])
+def test_batched(case, exact):
+    dtype, batch, M, N, K, layout = case
+    shape = Shape("t", M, N, K, batch, layout, False)
+    A, B, _ = make_operands(shape, 10, dtype, ints=exact)
+    with _plan(shape, dtype) as plan:
+        C = run_plan(plan, A, B, None, M, N, batch=batch)
+    compare(C, A, B, None, layout, dtype, exact=exact)
+
+
+@pytest.mark.parametrize("dtype", ["f32_ffma", "tf32", "bf16"])
+def test_degenerate_shapes(dtype):
+    import torch
+    bias = np.arange(5, dtype=np.float32)
+    # K = 0: C = bias
+    with nj.nnjit_matmul_plan_ex(nj.make_desc(3, 5, 0, dtype, "KN", has_bias=True), 10.0) as plan:
+        C = torch.full((3, 5), float("nan"), device="cuda")
+        plan.run(None, None, torch.from_numpy(bias).cuda(), C)
+        torch.cuda.synchronize()
+        assert np.array_equal(C.cpu().numpy(), np.broadcast_to(bias, (3, 5)))
+        C.fill_(float("nan"))
+        plan.run(None, None, None, C)
+        torch.cuda.synchronize()
+        assert np.array_equal(C.cpu().numpy(), np.zeros((3, 5), np.float32))
+    # M = 0 or N = 0: nothing to do, nothing written
+    for M, N in [(0, 5), (3, 0)]:
+        with nj.nnjit_matmul_plan_ex(nj.make_desc(M, N, 8, dtype, "KN"), 10.0) as plan:
+            plan.run(None, None, None, None)
+
+
+def test_gemv_ragged_k_with_padded_rows():
+    """K = 100 is not a multiple of the 8-element vector: lda = ldb = 104 keeps rows
+    16-byte aligned and the kernel's scalar tail covers the last 4 elements."""
+    M, N, K, ld = 2, 77, 100, 104
+    shape = Shape("t", M, N, ld, 1, "NK", True)
+    Ap, Bp, bias = make_operands(shape, 11, "bf16", ints=True)
+    desc = nj.make_desc(M, N, K, "bf16", "NK", has_bias=True, lda=ld, ldb=ld)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        assert plan.describe()["family"] == nj.NNJIT_FAMILY_GEMV
+        C = run_plan(plan, Ap, Bp, bias, M, N)
+    compare(C, np.ascontiguousarray(Ap[:, :K]), np.ascontiguousarray(Bp[:, :K]), bias, "NK",
+            "bf16", exact=True)
+
+
+def test_tc_strided_c():
+    """ldc > N: the epilogue honours the output row stride and leaves the gap alone."""
+    import torch
+    M, N, K, ldc = 130, 72, 64, 80
+    shape = Shape("t", M, N, K, 1, "NK", True)
+    A, B, bias = make_operands(shape, 12, "bf16", ints=True)
+    desc = nj.make_desc(M, N, K, "bf16", "NK", has_bias=True, ldc=ldc)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        from gpu_util import dev
+        Cbuf = torch.full((M, ldc), -7.0, device="cuda")
+        plan.run(dev(A), dev(B), dev(bias), Cbuf)
+        torch.cuda.synchronize()
+    Cn = Cbuf.cpu().numpy()
+    compare(np.ascontiguousarray(Cn[:, :N]), A, B, bias, "NK", "bf16", exact=True)
+    assert np.all(Cn[:, N:] == -7.0)
