@@ -1,0 +1,510 @@
+"""Benchmark of the JIT-tuned MatMul hot path on one workload (one JSON line on stdout).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME] [--budget-ms B] [--no-sweep]
+
+A step is one pass of the workload's products (for the default workload, the four
+Linears of a BART-base encoder layer at batch 4 x seq 128, TF32) over one batch of
+synthetic input.  Plans are tuned first (the JIT phase, timed separately and reported
+under "tune"); the timed region then runs K steps.  Each product's K launches run as a
+block of CUDA-graph replays that rotate over enough operand copies to exceed the L2, so
+operands come from HBM; CUDA events at the block boundaries give every kernel's average
+launch duration.  Under torchrun each rank runs its own replica (weak scaling).
+
+--impl reference times the oracle (the plain CPU definition) on the host cores on the
+same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+DEFAULT_WORKLOAD = "bart_base_encoder_m512"
+METRIC = "GEMM TFLOP/s (GEMV GB/s) vs GB300 roofline per shape; JIT tune time to plan"
+TF32_OVER_BF16 = 1.1 / 2.25     # nominal dense TF32 / BF16 tensor rates
+FFMA_PEAK_NOTE = "FP32 FFMA: 152 SMs x 128 FMA/clk x 2 x SM clock"
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+# ------------------------------------------------------------------------- helpers
+
+def shape_bytes(s, dtype):
+    e = 2 if dtype == "bf16" else 4
+    b = s.batch * (s.M * s.K * e + s.K * s.N * e + s.M * s.N * 4)
+    return b + (4 * s.N if s.has_bias else 0)
+
+
+def load_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained"), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0,
+            "source": "fallback"}
+
+
+def dtype_peak_tflops(dtype, peaks, sm_mhz):
+    if dtype == "bf16":
+        return peaks["bf16_tflops"]
+    if dtype == "tf32":
+        return peaks["bf16_tflops"] * TF32_OVER_BF16
+    return 152 * 128 * 2 * sm_mhz * 1e6 / 1e12
+
+
+class ClockSampler:
+    """nvidia-smi sampling during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index=0):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_rank{index}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"], stdout=self.f,
+                stderr=subprocess.DEVNULL)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        self.f.close()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 8:
+                    continue
+                try:
+                    rows.append((float(parts[0]), float(parts[1]), parts[3:]))
+                except ValueError:
+                    continue
+        if not rows:
+            return None
+        mx = max(r[1] for r in rows)
+        load = sorted(r[0] for r in rows)
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = set()
+        for r in rows:
+            for n, v in zip(names, r[2][1:5]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": load[len(load) // 2], "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(rows)}
+
+
+# ------------------------------------------------------------------------- reference arm
+
+def run_reference(args, workload, rank):
+    """The oracle as it stands, on the host cores, on the same workload and metric."""
+    if rank != 0:
+        return 0
+    import numpy as np
+    import oracle
+    from synthetic import make_operands
+    oracle.build()
+    dtype = workload.dtypes[-1]
+    cores = oracle.hw_threads()
+    # one step = every product of the workload on a row sample of A (the oracle cost is
+    # linear in the rows), sized to a few seconds of host work per step
+    budget_s = float(os.environ.get("NNJIT_REF_STEP_S", "3.0"))
+    ops = []
+    for s in workload.shapes:
+        A, B, bias = make_operands(s, workload.index, dtype)
+        ops.append((s, A, B, bias))
+    # calibrate the row fraction on one small probe
+    t0 = time.perf_counter()
+    s, A, B, bias = ops[0]
+    probe_rows = max(1, min(s.M, 8))
+    _ = oracle.matmul(A[..., :probe_rows, :] if s.batch > 1 else A[:probe_rows], B, bias,
+                      oracle.B_KN if s.b_layout == "KN" else oracle.B_NK)
+    dt_probe = max(1e-4, time.perf_counter() - t0)
+    probe_flops = 2 * s.batch * probe_rows * s.N * s.K
+    rate = probe_flops / dt_probe
+    full_flops = sum(x[0].flops for x in ops)
+    frac = min(1.0, budget_s * rate / full_flops)
+    sample_flops = 0
+    timings = []
+    for step in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        fl = 0
+        for s, A, B, bias in ops:
+            rows = max(1, int(round(s.M * frac)))
+            Ar = A[:, :rows] if s.batch > 1 else A[:rows]
+            oracle.matmul(np.ascontiguousarray(Ar), B, bias,
+                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores)
+            fl += 2 * s.batch * rows * s.N * s.K
+        dt = time.perf_counter() - t0
+        if step >= args.warmup:
+            timings.append(dt)
+            sample_flops = fl
+    total = sum(timings)
+    value = sample_flops * len(timings) / total / 1e12
+    sample = (f"each step: every product of the workload on the first {frac:.4f} of its rows "
+              f"({sample_flops / 1e9:.3f} GFLOP of {full_flops / 1e9:.3f}), fp64 oracle")
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TFLOP/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1000 * total / len(timings), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": workload.key, "shapes": [[s.batch, s.M, s.N, s.K] for s in workload.shapes]},
+        "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def cpu_baseline(workload, dtype, seconds=12.0):
+    """Oracle throughput on the host cores on a bounded sample of the workload."""
+    import numpy as np
+    import oracle
+    from synthetic import make_operands
+    oracle.build()
+    cores = oracle.hw_threads()
+    ops = [(s,) + make_operands(s, workload.index, dtype) for s in workload.shapes]
+    done_flops, t_used, reps = 0, 0.0, 0
+    # rows of every product, grown until the sample takes ~`seconds`
+    rows_frac = 1.0 / 64
+    while t_used < seconds and reps < 64:
+        t0 = time.perf_counter()
+        fl = 0
+        for s, A, B, bias in ops:
+            rows = max(1, int(round(s.M * rows_frac)))
+            Ar = A[:, :rows] if s.batch > 1 else A[:rows]
+            oracle.matmul(np.ascontiguousarray(Ar), B, bias,
+                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores)
+            fl += 2 * s.batch * rows * s.N * s.K
+        dt = time.perf_counter() - t0
+        done_flops += fl
+        t_used += dt
+        reps += 1
+        if dt < seconds / 8 and rows_frac < 1.0:
+            rows_frac = min(1.0, rows_frac * 2)
+    return {"value": done_flops / t_used / 1e12, "unit": "TFLOP/s", "cores": cores,
+            "kind": "oracle",
+            "sample": f"{reps} passes over every product on up to {rows_frac:.4f} of its rows "
+                      f"({done_flops / 1e9:.2f} GFLOP in {t_used:.1f} s, fp64, all host threads)"}
+
+
+# ------------------------------------------------------------------------- our arm
+
+def run_ours(args, workload, rank, world, local_rank):
+    import numpy as np
+    import torch
+    import paper_2309_08978_gb300 as nj
+    from synthetic import make_operands
+
+    torch.cuda.set_device(local_rank)
+    dev = torch.device("cuda", local_rank)
+    dtype = workload.dtypes[-1]
+    peaks = load_peaks()
+    lim = nj.nnjit_device_limits_query(local_rank)
+    l2 = lim.l2_bytes
+
+    def to_dev(x):
+        if x is None:
+            return None
+        if x.dtype == np.uint16:
+            return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).to(dev)
+        return torch.from_numpy(x).to(dev)
+
+    def to_pinned(x):
+        if x is None:
+            return None
+        if x.dtype == np.uint16:
+            t = torch.from_numpy(x.view(np.int16)).view(torch.bfloat16)
+        else:
+            t = torch.from_numpy(x)
+        return t.pin_memory()
+
+    # ---- operands, plans (the JIT phase), tuner vs exhaustive sweep
+    items = []
+    tune = {"budget_ms_per_shape": args.budget_ms, "shapes": []}
+    for s in workload.shapes:
+        A, B, bias = make_operands(s, workload.index, dtype)
+        desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
+                            has_bias=s.has_bias)
+        t0 = time.perf_counter()
+        plan = nj.nnjit_matmul_plan_ex(desc, args.budget_ms)
+        plan_ms = 1000 * (time.perf_counter() - t0)
+        info = plan.describe()
+        entry = {"shape": [s.batch, s.M, s.N, s.K], "plan_ms": round(plan_ms, 2),
+                 "space_size": info["space_size"], "naive_space": info["naive_space"],
+                 "chosen_index": info["chosen_index"], "family": info["family"],
+                 "candidate": {k: info["candidate"][k] for k in ("bm", "bn", "bk", "stages", "split_k", "raster")}}
+        if not args.no_sweep:
+            sweep_desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
+                                      has_bias=s.has_bias,
+                                      flags=nj.NNJIT_PLAN_EXHAUSTIVE | nj.NNJIT_PLAN_NO_CACHE)
+            t0 = time.perf_counter()
+            sweep = nj.nnjit_matmul_plan_ex(sweep_desc, 0.0)
+            sweep_ms = 1000 * (time.perf_counter() - t0)
+            sinfo = sweep.describe()
+            sweep.destroy()
+            times = {int(i): t for i, t in sinfo["timings_us"]}
+            best_i = min(times, key=lambda i: (times[i], i))
+            pick = times.get(info["chosen_index"])
+            entry.update({"sweep_ms": round(sweep_ms, 2), "best_index": best_i,
+                          "best_us": round(times[best_i], 3),
+                          "pick_us": round(pick, 3) if pick is not None else None,
+                          "pick_over_best": round(pick / times[best_i], 4) if pick else None})
+        tune["shapes"].append(entry)
+        nsets = int(min(64, max(1, math.ceil(3 * l2 / shape_bytes(s, dtype)))))
+        if s.batch > 1:
+            out_shape = (s.batch, s.M, s.N)
+        else:
+            out_shape = (s.M, s.N)
+        dA, dB, dbias = to_dev(A), to_dev(B), to_dev(bias)
+        sets = [(dA, dB, dbias, torch.empty(out_shape, dtype=torch.float32, device=dev))]
+        for _ in range(nsets - 1):
+            sets.append((dA.clone(), dB.clone(), dbias.clone() if dbias is not None else None,
+                         torch.empty(out_shape, dtype=torch.float32, device=dev)))
+        cand = plan.candidate()
+        launches = 1 + (1 if cand["split_k"] > 1 else 0)
+        items.append({"shape": s, "plan": plan, "sets": sets, "host": (A, B, bias),
+                      "launches": launches, "family": info["family"]})
+    tune["total_plan_ms"] = round(sum(e["plan_ms"] for e in tune["shapes"]), 2)
+    ratios = [e["pick_over_best"] for e in tune["shapes"] if e.get("pick_over_best")]
+    if ratios:
+        tune["max_pick_over_best"] = max(ratios)
+    torch.cuda.synchronize()
+
+    stream = torch.cuda.Stream(device=dev)
+
+    def run_item(it, k):
+        A, B, bias, C = it["sets"][k % len(it["sets"])]
+        it["plan"].run(A, B, bias, C, stream)
+
+    # ---- graphs: per product, one replay = one launch on each operand copy
+    graphs = []
+    with torch.cuda.stream(stream):
+        for it in items:
+            run_item(it, 0)  # warm the tensor-map cache outside capture
+        torch.cuda.synchronize()
+        for it in items:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for k in range(len(it["sets"])):
+                    run_item(it, k)
+            graphs.append(g)
+    torch.cuda.synchronize()
+
+    def block(i, n):
+        """n launches of product i, as graph replays (+ a tail of single launches)."""
+        it = items[i]
+        G = len(it["sets"])
+        for _ in range(n // G):
+            graphs[i].replay()
+        for k in range(n % G):
+            run_item(it, k)
+
+    # warm-up steps
+    with torch.cuda.stream(stream):
+        for i in range(len(items)):
+            block(i, args.warmup)
+    torch.cuda.synchronize()
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+        torch.cuda.synchronize()
+
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    time.sleep(0.3)
+    barrier()
+    evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(items) + 1)]
+    t_wall = time.perf_counter()
+    with torch.cuda.stream(stream):
+        evs[0].record(stream)
+        for i in range(len(items)):
+            block(i, args.steps)
+            evs[i + 1].record(stream)
+    stream.synchronize()
+    barrier()
+    wall = time.perf_counter() - t_wall
+    clocks = sampler.stop()
+    per_item_ms = [evs[i].elapsed_time(evs[i + 1]) for i in range(len(items))]
+    total_ms = sum(per_item_ms)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    for it in items:
+        it["plan"].check()
+
+    flops_step = sum(it["shape"].flops for it in items)
+    ms_per_step = total_ms / args.steps
+    value = world * flops_step * args.steps / (total_ms / 1e3) / 1e12
+
+    # ---- roofline of the dominant kernel (largest share of the timed region)
+    dom = max(range(len(items)), key=lambda i: per_item_ms[i])
+    ds = items[dom]["shape"]
+    dur_s = per_item_ms[dom] / 1e3 / args.steps
+    alg_bytes = shape_bytes(ds, dtype)
+    sm_mhz = clocks["sm_mhz"] if clocks else 1900.0
+    peak_t = dtype_peak_tflops(dtype, peaks, sm_mhz)
+    ai = ds.flops / alg_bytes
+    ridge = peak_t * 1e12 / (peaks["hbm_gbs"] * 1e9)
+    if items[dom]["family"] == nj.NNJIT_FAMILY_GEMV or ai < ridge:
+        ach = alg_bytes / dur_s / 1e9
+        roof = {"bound": "hbm", "achieved": round(ach, 1), "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                "frac": round(ach / peaks["hbm_gbs"], 4)}
+    else:
+        ach = ds.flops / dur_s / 1e12
+        roof = {"bound": "tensor", "achieved": round(ach, 2), "peak": round(peak_t, 1),
+                "unit": "TFLOP/s", "frac": round(ach / peak_t, 4)}
+    roof.update({"traffic": None, "kernel": f"{ds.name} {ds.batch}x{ds.M}x{ds.N}x{ds.K} {dtype}",
+                 "peak_source": ("measured bf16 x nominal tf32/bf16 ratio" if dtype == "tf32"
+                                 else peaks["source"]) + f" ({peaks['source']})",
+                 "units_per_launch": f"{ds.flops} flop, {alg_bytes} algorithmic bytes"})
+    per_shape = []
+    for i, it in enumerate(items):
+        s = it["shape"]
+        d = per_item_ms[i] / 1e3 / args.steps
+        per_shape.append({"shape": [s.batch, s.M, s.N, s.K], "us": round(d * 1e6, 3),
+                          "tflops": round(s.flops / d / 1e12, 2),
+                          "gbs": round(shape_bytes(s, dtype) / d / 1e9, 1),
+                          "share": round(per_item_ms[i] / sum(per_item_ms), 4)})
+
+    # ---- end to end through the C ABI with host buffers (copies inside the region)
+    e2e_steps = max(3, min(args.steps, args.e2e_steps))
+    hosts = []
+    for it in items:
+        A, B, bias = it["host"]
+        s = it["shape"]
+        out = torch.empty(((s.batch, s.M, s.N) if s.batch > 1 else (s.M, s.N)),
+                          dtype=torch.float32).pin_memory()
+        hosts.append((to_pinned(A), to_pinned(B), to_pinned(bias), out))
+    h2d = sum(h[0].numel() * h[0].element_size() + h[1].numel() * h[1].element_size() +
+              (h[2].numel() * 4 if h[2] is not None else 0) for h in hosts)
+    d2h = sum(h[3].numel() * 4 for h in hosts)
+    with torch.cuda.stream(stream):
+        for it, h in zip(items, hosts):
+            nj.nnjit_matmul_run_host(it["plan"], *h, stream)
+    stream.synchronize()
+    barrier()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(e2e_steps):
+            for it, h in zip(items, hosts):
+                nj.nnjit_matmul_run_host(it["plan"], *h, stream)
+        e1.record(stream)
+    stream.synchronize()
+    barrier()
+    e2e_ms = e0.elapsed_time(e1)
+    if world > 1:
+        import torch.distributed as dist
+        t = torch.tensor([e2e_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+    e2e_value = world * flops_step * e2e_steps / (e2e_ms / 1e3) / 1e12
+
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(workload, dtype, seconds=args.cpu_seconds)
+
+    l2_note = ("each product rotates over " + ", ".join(str(len(it["sets"])) for it in items) +
+               f" operand copies (>= 3 x L2 = {3 * l2 / 2**20:.0f} MiB per product), so "
+               "operands stream from HBM")
+    line = {
+        "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
+        "data": "synthetic (seeded SplitMix64, the workload's distributions; no trained weights)",
+        "config": {"workload": workload.key, "title": workload.title,
+                   "shapes": [[s.batch, s.M, s.N, s.K, s.b_layout] for s in workload.shapes],
+                   "parallelism": f"replicas{world}", "l2": l2_note,
+                   "schedule": "per product: K launches as CUDA-graph replays, products in sequence"},
+        "roofline": roof,
+        "per_shape": per_shape,
+        "tune": tune,
+        "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
+                "d2h_bytes_per_step": d2h, "steps": e2e_steps,
+                "how": "nnjit_matmul_run_host per product: pinned host -> device copies, kernel, "
+                       "device -> host copy of C, all inside the timed region"},
+        "gpu_launches": int(args.steps * sum(it["launches"] for it in items)),
+        "clocks": clocks,
+        "wall_s": round(wall, 3),
+    }
+    if cpu is not None:
+        line["cpu_baseline"] = cpu
+    for it in items:
+        it["plan"].destroy()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    return 0
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=50000)
+    ap.add_argument("--warmup", type=int, default=500)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
+    ap.add_argument("--budget-ms", type=float, default=2000.0, help="tuning budget per product")
+    ap.add_argument("--no-sweep", action="store_true", help="skip the exhaustive sweep")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--e2e-steps", type=int, default=200)
+    args = ap.parse_args(argv)
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    from synthetic import WORKLOADS
+    workload = WORKLOADS[args.workload]
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        return run_reference(args, workload, rank)
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    import __graft_entry__
+    __graft_entry__.build()
+    try:
+        return run_ours(args, workload, rank, world, local_rank)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -11,7 +11,7 @@ FfmaKernel ffma_kernel_nk(int i);
 cudaError_t launch_ffma(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
-    if (c.instance < 0 || c.instance >= 48) return cudaErrorInvalidValue;
+    if (c.instance < 0 || c.instance >= 24) return cudaErrorInvalidValue;
     const bool nk = (c.instance & 1) != 0;
     FfmaKernel k = nk ? ffma_kernel_nk(c.instance >> 1) : ffma_kernel_kn(c.instance >> 1);
     if (!k || nk != (p.b_layout == NNJIT_B_NK)) return cudaErrorInvalidValue;

@@ -1,20 +1,20 @@
 // FP32-FFMA GEMM instances with B stored [N][K]: the 12 (thread tile, block tile)
-// pairs of the lite space x BK in {8, 16}, in the order of ffma_instance().
+// pairs of the lite space (BK = 16), in the order of ffma_instance().
 #include "ffma.cuh"
 
 namespace nnjit {
 
 using FfmaKernel = void (*)(FfmaParams);
 
-#define NNJIT_FFMA_PAIR(TM, BM, BN) ffma_gemm_kernel<BM, BN, 8, TM, TM, true>, ffma_gemm_kernel<BM, BN, 16, TM, TM, true>
+#define NNJIT_FFMA_PAIR(TM, BM, BN) ffma_gemm_kernel<BM, BN, 16, TM, TM, true>
 
-static const FfmaKernel kFfma_nk[24] = {
+static const FfmaKernel kFfma_nk[12] = {
     NNJIT_FFMA_PAIR(4, 32, 32),  NNJIT_FFMA_PAIR(4, 32, 64),  NNJIT_FFMA_PAIR(4, 32, 128),
     NNJIT_FFMA_PAIR(4, 64, 32),  NNJIT_FFMA_PAIR(4, 64, 64),  NNJIT_FFMA_PAIR(4, 128, 32),
     NNJIT_FFMA_PAIR(8, 32, 128), NNJIT_FFMA_PAIR(8, 64, 64),  NNJIT_FFMA_PAIR(8, 64, 128),
     NNJIT_FFMA_PAIR(8, 128, 32), NNJIT_FFMA_PAIR(8, 128, 64), NNJIT_FFMA_PAIR(8, 128, 128),
 };
 
-FfmaKernel ffma_kernel_nk(int i) { return (i >= 0 && i < 24) ? kFfma_nk[i] : nullptr; }
+FfmaKernel ffma_kernel_nk(int i) { return (i >= 0 && i < 12) ? kFfma_nk[i] : nullptr; }
 
 }  // namespace nnjit

@@ -28,6 +28,7 @@ struct GemvParams {
     float* C;            // [M][ldc]
     float* ws;           // [split][M][N]
     int M, N, K, split, kper;
+    int vec_ok;          // KN: rows of W are 16-byte aligned (ldb % 8 == 0)
     long long lda, ldb, ldc;
 };
 
@@ -158,7 +159,7 @@ __global__ void __launch_bounds__(256) gemv_kn_kernel(const GemvParams p) {
     const int k1 = min(p.K, k0 + p.kper);
     const int M = p.M;
     const int n0 = blockIdx.x * 256 + lane * 8;
-    const bool vec = n0 + 8 <= p.N;
+    const bool vec = p.vec_ok && n0 + 8 <= p.N;
     float acc[kMaxM][8];
 #pragma unroll
     for (int m = 0; m < kMaxM; ++m)
@@ -312,6 +313,7 @@ cudaError_t launch_gemv(const LaunchArgs& a) {
     prm.M = (int)p.M; prm.N = (int)p.N; prm.K = (int)p.K;
     prm.split = c.split_k;
     prm.lda = p.lda; prm.ldb = p.ldb; prm.ldc = p.ldc;
+    prm.vec_ok = (p.ldb % 8 == 0 && (reinterpret_cast<uintptr_t>(a.B) & 15) == 0) ? 1 : 0;
     const int warps = c.threads / 32;
     dim3 grid;
     int smem;

@@ -87,6 +87,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     constexpr uint32_t kStageBytes = kABytes + kBBytes;
     constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
     constexpr uint32_t kIdesc = ptx::instr_desc(kKind == 0 ? 1u : 2u, kBMn, kBM, BN);
+    // MN-major 32-bit (tf32) operands use the 32-byte-atom variant of the 128-byte swizzle
+    // (the TMA load writes the matching CU_TENSOR_MAP_SWIZZLE_128B_ATOM_32B pattern).
+    constexpr uint32_t kBLayout = (kKind == 1 && kBMn) ? ptx::kLayoutSw128Atom32 : ptx::kLayoutSw128;
+    // In that layout the MMA walks K in groups of 4 rows of 128 bytes, so consecutive
+    // K groups sit 512 bytes apart (8-row groups, 1024 bytes, for the other layouts).
+    constexpr uint32_t kBSbo = (kKind == 1 && kBMn) ? 512u : 1024u;
 
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -209,12 +215,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     const uint32_t sb = sa + kABytes;
 #pragma unroll
                     for (int kk = 0; kk < kKSteps; ++kk) {
-                        const uint64_t adesc = ptx::smem_desc_sw128(sa + kk * 32, 16, 1024);
+                        const uint64_t adesc = ptx::smem_desc(sa + kk * 32, 16, 1024);
                         uint64_t bdesc;
                         if constexpr (!kBMn)
-                            bdesc = ptx::smem_desc_sw128(sb + kk * 32, 16, 1024);
+                            bdesc = ptx::smem_desc(sb + kk * 32, 16, 1024);
                         else
-                            bdesc = ptx::smem_desc_sw128(sb + kk * kUmmaK * 128, BK * 128, 1024);
+                            bdesc = ptx::smem_desc(sb + kk * kUmmaK * 128, BK * 128, kBSbo, kBLayout);
                         ptx::mma_ss<kKind>(d_tmem, adesc, bdesc, kIdesc,
                                            (kb > kb0 || kk > 0) ? 1u : 0u);
                     }
@@ -379,8 +385,11 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
         dims[2] = (cuuint64_t)p.batch;
         box[2] = 1;
         const cuuint64_t strides[2] = {(cuuint64_t)(p.ldb * e), (cuuint64_t)(p.stride_b * e)};
+        const CUtensorMapSwizzle swz = (p.dtype != NNJIT_BF16 && p.b_layout == NNJIT_B_KN)
+                                           ? CU_TENSOR_MAP_SWIZZLE_128B_ATOM_32B
+                                           : CU_TENSOR_MAP_SWIZZLE_128B;
         CUresult r = enc(tb, dt, 3, const_cast<void*>(B), dims, strides, box, estr,
-                         CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                         CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
         if (r != CUDA_SUCCESS) {
             *why = "cuTensorMapEncodeTiled failed for B";

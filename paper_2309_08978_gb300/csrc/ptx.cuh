@@ -111,17 +111,21 @@ __device__ __forceinline__ void tc_fence_after() {
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
-// Shared-memory matrix descriptor, 128-byte swizzle (layout type 2 in bits 61-63),
-// descriptor version 1 (bits 46-47), base offset 0, absolute LBO mode.
-// Start address, leading-dimension byte offset and stride-dimension byte offset are
-// stored >> 4 in 14-bit fields at bits 0, 16 and 32.
-__device__ __forceinline__ uint64_t smem_desc_sw128(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+// Shared-memory matrix descriptor layout types (bits 61-63).
+constexpr uint32_t kLayoutSw128 = 2;        // 128-byte swizzle, 16-byte atoms
+constexpr uint32_t kLayoutSw128Atom32 = 1;  // 128-byte swizzle, 32-byte atoms (MN-major tf32)
+
+// Shared-memory matrix descriptor: descriptor version 1 (bits 46-47), base offset 0,
+// absolute LBO mode.  Start address, leading-dimension byte offset and stride-dimension
+// byte offset are stored >> 4 in 14-bit fields at bits 0, 16 and 32.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo,
+                                              uint32_t layout = kLayoutSw128) {
     uint64_t d = 0;
     d |= (uint64_t)((saddr >> 4) & 0x3FFFu);
     d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
     d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
     d |= (uint64_t)1u << 46;
-    d |= (uint64_t)2u << 61;
+    d |= (uint64_t)(layout & 7u) << 61;
     return d;
 }
 

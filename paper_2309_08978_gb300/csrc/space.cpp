@@ -112,7 +112,7 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
 // ---------------------------------------------------------------------------------
 // FP32-FFMA SIMT family: the direct descendant of the paper's WebGPU tile template
 // (Table 2): thread tile x0 = y0 in {4, 8} (inner range [4..32]), block tile x1, y1 in
-// {32, 64, 128} (range [32..256]), r1 = BK in {8, 16}, r0 = 1.  Table 1's usage formulas
+// {32, 64, 128} (range [32..256]), r1 = BK = 16, r0 = 1.  Table 1's usage formulas
 // are applied as written; heuristic 5 (Thread_block <= 256) is kept, the WebGPU 16 KB
 // limit of heuristic 6 becomes the CTA's shared-memory limit.
 // ---------------------------------------------------------------------------------
@@ -122,9 +122,9 @@ void ffma_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
     const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
     const int64_t K = std::max<int64_t>(p.K, 1);
     const int tiles_x[3] = {32, 64, 128};
-    const int bks[2] = {8, 16};
+    const int bks[1] = {16};
     const int splits[4] = {1, 2, 4, 8};
-    *naive = 2 * 3 * 3 * 2 * 4;
+    *naive = 2 * 3 * 3 * 2 * 4;  // thread tile x block tile x BK {8, 16} x split
     for (int t0 : {4, 8}) {
         for (int bm : tiles_x) {
             for (int bn : tiles_x) {
@@ -300,8 +300,8 @@ int ffma_instance(int tm, int bm, int bn, int bk, int b_layout) {
     int ti = -1;
     for (int i = 0; i < 12; ++i)
         if (kFfmaTiles[i][0] == tm && kFfmaTiles[i][1] == bm && kFfmaTiles[i][2] == bn) ti = i;
-    if (ti < 0 || (bk != 8 && bk != 16)) return -1;
-    return (ti * 2 + (bk == 16 ? 1 : 0)) * 2 + (b_layout == NNJIT_B_NK ? 1 : 0);
+    if (ti < 0 || bk != 16) return -1;
+    return ti * 2 + (b_layout == NNJIT_B_NK ? 1 : 0);
 }
 
 int gemv_instance(int b_layout, int rows, int unroll) {
@@ -359,8 +359,12 @@ nnjit_status choose_family(const Problem& p, int* family, std::string* err) {
     if (p.dtype == NNJIT_F32_FFMA) { *family = NNJIT_FAMILY_FFMA; return NNJIT_OK; }
     const int e = p.elem_bytes();
     if (p.dtype == NNJIT_BF16 && p.M <= ModelConstants::kGemvMaxM && p.batch == 1) {
-        if (!p.degenerate() && ((p.lda * e) % 16 != 0 || (p.ldb * e) % 16 != 0)) {
-            *err = "GEMV path needs 16-byte aligned rows of A and B (lda, ldb multiples of 8)";
+        // B as [N][K]: x is staged and W streamed with 16-byte loads along K.  B as [K][N]
+        // falls back to 2-byte loads when rows of W are not 16-byte aligned.
+        if (!p.degenerate() && p.b_layout == NNJIT_B_NK &&
+            ((p.lda * e) % 16 != 0 || (p.ldb * e) % 16 != 0)) {
+            *err = "GEMV path with B as [N][K] needs 16-byte aligned rows of A and B "
+                   "(lda, ldb multiples of 8)";
             return NNJIT_ERR_UNSUPPORTED;
         }
         *family = NNJIT_FAMILY_GEMV;
