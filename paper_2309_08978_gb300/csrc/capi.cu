@@ -87,8 +87,10 @@ struct nnjit_plan_s {
     std::mutex mu;  // guards the tensor-map cache and the host staging buffers
     const void* tm_A = nullptr;
     const void* tm_B = nullptr;
+    const void* tm_C = nullptr;
     bool tm_valid = false;
-    CUtensorMap ta, tb;
+    bool tm_c_ok = false;
+    CUtensorMap ta, tb, tc;
     void* hA = nullptr;  // device staging for run_host
     void* hB = nullptr;
     float* hbias = nullptr;
@@ -201,22 +203,27 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
     la.stream = s;
     cudaError_t e = cudaSuccess;
     if (c.family == NNJIT_FAMILY_TC) {
-        CUtensorMap ta, tb;
+        CUtensorMap ta, tb, tcm;
+        bool c_ok = false;
         const char* why = "";
+        float* out = c.split_k > 1 ? ws : C;
         {
             std::lock_guard<std::mutex> lk(pl->mu);
-            if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B) {
+            if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B || pl->tm_C != out) {
                 e = encode_tc_tensor_maps(p, c, A, B, &ta, &tb, &why);
                 if (e != cudaSuccess) return fail(NNJIT_ERR_UNSUPPORTED, why);
+                encode_tc_output_map(p, c, out, c.split_k > 1, &tcm, &c_ok);
                 if (!override_cand) {
-                    pl->ta = ta; pl->tb = tb; pl->tm_A = A; pl->tm_B = B; pl->tm_valid = true;
+                    pl->ta = ta; pl->tb = tb; pl->tc = tcm; pl->tm_c_ok = c_ok;
+                    pl->tm_A = A; pl->tm_B = B; pl->tm_C = out; pl->tm_valid = true;
                 }
             } else {
-                ta = pl->ta; tb = pl->tb;
+                ta = pl->ta; tb = pl->tb; tcm = pl->tc; c_ok = pl->tm_c_ok;
             }
         }
         la.tmap_a = &ta;
         la.tmap_b = &tb;
+        la.tmap_c = c_ok ? &tcm : nullptr;
         e = launch_tc(la);
     } else if (c.family == NNJIT_FAMILY_FFMA) {
         e = launch_ffma(la);

@@ -34,10 +34,13 @@ namespace {
 constexpr int kBM = 128;
 constexpr int kThreads = 192;
 constexpr int kMaxStages = 8;
+constexpr int kEpiStageBytes = 4 * 2 * 4096;  // 4 epilogue warps x 2 buffers x (32 x 32 f32)
 
 struct TcParams {
     CUtensorMap tmap_a;  // A [batch][M][K]: dims {K, M, batch}, box {BK, 128, 1}
     CUtensorMap tmap_b;  // NK: dims {K, N, batch}, box {BK, BN, 1}; KN: dims {N, K, batch}, box {atom, BK, 1}
+    CUtensorMap tmap_c;  // output (C, or the split-K partials): dims {N, M, z}, box {32, 32, 1}
+    int tma_store;       // 1: epilogue stores through tmap_c; 0: direct global stores
     float* C;
     const float* bias;
     float* ws;
@@ -98,7 +101,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
     const int S = p.stages;
-    uint64_t* bars = reinterpret_cast<uint64_t*>(smem + (size_t)S * kStageBytes);
+    uint8_t* epi_smem = smem + (size_t)S * kStageBytes;  // 1024-aligned (stage bytes are)
+    uint64_t* bars = reinterpret_cast<uint64_t*>(epi_smem + kEpiStageBytes);
     // bars[0..S): full, [S..2S): empty, 2S..2S+1: tmem_full, 2S+2..2S+3: tmem_empty,
     // 2S+4: drain
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kMaxStages + 5);
@@ -129,6 +133,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     if (warp == 0 && lane == 0) {
         ptx::prefetch_tmap(&p.tmap_a);
         ptx::prefetch_tmap(&p.tmap_b);
+        if (p.tma_store) ptx::prefetch_tmap(&p.tmap_c);
     }
     if (warp == 1) {
         ptx::tmem_alloc(ptx::smem_u32(tmem_slot), kTmemCols);
@@ -243,8 +248,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         ptx::mbar_wait(drain_bar, 0, &no_abort, p.err, kErrDrain, ptx::kWaitLimitNs / 4);
     } else {
         // ---------------------------------------------------------------- epilogue
-        const int q = warp & 3;              // TMEM sub-partition this warp may access
+        // Warp (2 + e) owns TMEM sub-partition q = warp % 4, i.e. tile rows 32q .. 32q+31;
+        // thread `lane` holds one row.  Each 32 x 32 chunk goes either through a 128B-
+        // swizzled shared-memory buffer and a TMA store (coalesced, bounds-clipped), or,
+        // when the output's strides do not allow TMA, straight to global memory.
+        const int q = warp & 3;
         const int row_in_tile = q * 32 + lane;
+        uint8_t* stage_buf = epi_smem + (warp - 2) * 8192;
+        uint32_t chunk_ctr = 0;
         uint32_t iter = 0;
         const long long MN = (long long)p.M * p.N;
         for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++iter) {
@@ -254,30 +265,47 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
             ptx::tc_fence_after();
             const int row = tc.tm * kBM + row_in_tile;
-            float* dst_row;
-            const float* bias = nullptr;
-            if (p.split == 1) {
-                dst_row = p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc;
-                bias = p.bias;
-            } else {
-                dst_row = p.ws + ((long long)tc.s * p.batch + tc.b) * MN + (long long)row * p.N;
-            }
+            const float* bias = p.split == 1 ? p.bias : nullptr;
+            float* dst_row = p.split == 1
+                                 ? p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc
+                                 : p.ws + ((long long)tc.s * p.batch + tc.b) * MN + (long long)row * p.N;
+            const int zc = p.split == 1 ? tc.b : tc.s * p.batch + tc.b;
 #pragma unroll 1
             for (int c = 0; c < BN / 32; ++c) {
                 uint32_t r[32];
                 const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32;
                 ptx::tmem_ld32(taddr, r);
                 ptx::tmem_wait_ld(r);
+                if (c == BN / 32 - 1) {
+                    // the accumulator is in registers: hand TMEM back to the MMA warp
+                    ptx::tc_fence_before();
+                    ptx::mbar_arrive(tempty_bar(acc));
+                }
                 const int col0 = tc.tn * BN + c * 32;
-                if (row < p.M) {
-                    float v[32];
+                float v[32];
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-                    if (bias) {
+                for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+                if (bias) {
 #pragma unroll
-                        for (int j = 0; j < 32; ++j)
-                            if (col0 + j < p.N) v[j] += __ldg(bias + col0 + j);
+                    for (int j = 0; j < 32; ++j)
+                        if (col0 + j < p.N) v[j] += __ldg(bias + col0 + j);
+                }
+                if (p.tma_store) {
+                    uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
+                    if (lane == 0) ptx::bulk_wait_read<1>();  // the store that used buf is done
+                    __syncwarp();
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        *reinterpret_cast<float4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                    ptx::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        ptx::tma_store_3d(&p.tmap_c, ptx::smem_u32(buf), col0, tc.tm * kBM + q * 32, zc);
+                        ptx::bulk_commit();
                     }
+                    ++chunk_ctr;
+                } else if (row < p.M) {
                     float* dst = dst_row + col0;
                     if (col0 + 32 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
 #pragma unroll
@@ -290,9 +318,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     }
                 }
             }
-            ptx::tc_fence_before();
-            ptx::mbar_arrive(tempty_bar(acc));
         }
+        if (p.tma_store && lane == 0) ptx::bulk_wait_all();
+        __syncwarp();
     }
 
     ptx::tc_fence_before();
@@ -399,6 +427,26 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
     return cudaSuccess;
 }
 
+cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, float* out,
+                                 bool partials, CUtensorMap* tc_map, bool* ok) {
+    *ok = false;
+    EncodeTiledFn enc = get_encode_fn();
+    if (!enc || !out) return cudaSuccess;
+    const long long ld = partials ? p.N : p.ldc;
+    const long long zs = partials ? p.M * p.N : p.stride_c;
+    const long long nz = partials ? p.batch * c.split_k : p.batch;
+    if ((reinterpret_cast<uintptr_t>(out) & 15) || (ld * 4) % 16 || (zs * 4) % 16) return cudaSuccess;
+    const cuuint64_t dims[3] = {(cuuint64_t)p.N, (cuuint64_t)p.M, (cuuint64_t)nz};
+    const cuuint64_t strides[2] = {(cuuint64_t)(ld * 4), (cuuint64_t)(zs * 4)};
+    const cuuint32_t box[3] = {32, 32, 1};
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(tc_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, out, dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    *ok = (r == CUDA_SUCCESS);
+    return cudaSuccess;
+}
+
 cudaError_t launch_tc(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
@@ -407,6 +455,8 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     TcParams prm;
     prm.tmap_a = *a.tmap_a;
     prm.tmap_b = *a.tmap_b;
+    prm.tma_store = a.tmap_c ? 1 : 0;
+    if (a.tmap_c) prm.tmap_c = *a.tmap_c;
     prm.C = a.C;
     prm.bias = a.bias;
     prm.ws = a.ws;
@@ -430,7 +480,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     const int grid = (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
     // ring + alignment slack + barriers/TMEM slot/abort flag
     const int stage_bytes = (kBM + c.bn) * 128;
-    const int smem = c.stages * stage_bytes + 1024 + 256;
+    const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     cudaError_t e = prepare_tc_instance(c.instance, smem);
     if (e != cudaSuccess) return e;
     kTcKernels[c.instance]<<<grid, kThreads, smem, a.stream>>>(prm);

@@ -23,6 +23,8 @@ struct LaunchArgs {
     cudaStream_t stream = nullptr;
     const CUtensorMap* tmap_a = nullptr;  // TC family only
     const CUtensorMap* tmap_b = nullptr;
+    const CUtensorMap* tmap_c = nullptr;  // TC output map (C, or partials when split > 1);
+                                          // NULL: the epilogue stores directly
 };
 
 // Main kernels.  Each returns the launch status (cudaGetLastError after the launch).
@@ -47,6 +49,11 @@ cudaError_t launch_l2_flush(void* buf, int64_t bytes, cudaStream_t s);
 // One-time per-process kernel attribute setup (opt-in shared memory).  Idempotent.
 cudaError_t prepare_tc_instance(int instance, int smem_bytes);
 cudaError_t prepare_gemv_instance(int instance, int smem_bytes);
+
+// Output tensor map for the TC epilogue's TMA stores: C (partials = false) or the split-K
+// partials buffer.  *ok is false when the output's alignment or strides rule TMA out.
+cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, float* out,
+                                 bool partials, CUtensorMap* tc_map, bool* ok);
 
 // Tensor maps for the TC family (host; uses the driver entry point).
 cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,

@@ -36,7 +36,8 @@ struct ModelConstants {
     static constexpr int kTcRegsPerThread = 72;      // tcgen05 kernel: ptxas reports 64-65, allocated in 8s
     static constexpr int kTcThreads = 192;           // 6 warps: TMA, MMA, 4 x epilogue
     static constexpr int kTcBM = 128;
-    static constexpr int kTcFixedSmem = 1024 + 256;  // 1 KB alignment slack + barriers
+    static constexpr int kTcFixedSmem = 1024 + 256 + 32768;  // alignment slack, barriers,
+                                                              // epilogue staging buffers
     static constexpr int kTcMaxStages = 8;
     static constexpr int kGemvMaxM = 8;
     static constexpr int kGemvMaxSmem = 64 * 1024;

@@ -137,10 +137,12 @@ def test_gemv_ragged_k_with_padded_rows():
             "bf16", exact=True)
 
 
-def test_tc_strided_c():
-    """ldc > N: the epilogue honours the output row stride and leaves the gap alone."""
+@pytest.mark.parametrize("ldc", [80, 75])
+def test_tc_strided_c(ldc):
+    """ldc > N: the epilogue honours the output row stride and leaves the gap alone.
+    ldc = 80 keeps 16-byte rows (TMA-store epilogue); ldc = 75 does not (direct stores)."""
     import torch
-    M, N, K, ldc = 130, 72, 64, 80
+    M, N, K = 130, 72, 64
     shape = Shape("t", M, N, K, 1, "NK", True)
     A, B, bias = make_operands(shape, 12, "bf16", ints=True)
     desc = nj.make_desc(M, N, K, "bf16", "NK", has_bias=True, ldc=ldc)
