@@ -242,6 +242,33 @@ nnjit_status nnjit_plan_candidate(nnjit_plan p, nnjit_candidate* out);
  * launch of this plan is still running (e.g. synchronise the stream first). */
 nnjit_status nnjit_plan_destroy(nnjit_plan p);
 
+/*
+ * Decode GEMV that allocates nothing (the paper has no counterpart; this serves callers
+ * that cannot allocate device memory when they run a product, e.g. a process whose
+ * device memory a framework's caching allocator has already reserved, or a decode loop
+ * that must not pay for cudaMalloc / cudaFree, which may synchronise the device).
+ *
+ * C[m,n] = sum_k x[m,k] * W[n,k] (+ bias[n]) for 1 <= M <= 8, with x [M][K] and W [N][K]
+ * packed bf16, C [M][N] packed float32, bias float32[N] or NULL, all device pointers the
+ * caller owns; K % 8 == 0 and x, W 16-byte aligned.  K is split into split_k slices
+ * (1..64) whose float32 partial sums are kept in one fixed device array inside the
+ * library of NNJIT_NOALLOC_SCRATCH_FLOATS floats (4 MiB, held by every GPU that loads
+ * the library until the process exits) and then added in slice order.  Requests with
+ * split_k * M * N above that size, or whose x slice (M * K / split_k bf16 values) exceeds
+ * 96 KiB of shared memory, fail with UNSUPPORTED and a message in nnjit_last_error().
+ * On success the call makes no allocation: it calls no cudaMalloc, cudaMallocAsync,
+ * cudaFree or other allocating routine, and no host heap allocation of its own; it makes
+ * no plan and does no tuning (one fixed GEMV configuration).  The first call on a device looks
+ * up the array's device address (cudaGetSymbolAddress) and keeps it; make that first
+ * call before any stream capture.  Every call on a device shares the one array: calls
+ * that may overlap on the GPU (different streams, or another thread) race on it and
+ * must be serialised by the caller.  Every partial is written before it is read, so the
+ * array's previous contents never matter.  Asynchronous on `stream`.
+ */
+#define NNJIT_NOALLOC_SCRATCH_FLOATS (1 << 20)
+nnjit_status nnjit_gemv_bf16_noalloc(int64_t M, int64_t N, int64_t K, const void* x, const void* W,
+                                     const float* bias, float* C, int32_t split_k, void* stream);
+
 /* Drop every cached plan choice of this process. */
 nnjit_status nnjit_cache_clear(void);
 

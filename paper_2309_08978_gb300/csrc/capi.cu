@@ -67,6 +67,11 @@ FaultSpec read_fault() {
 
 }  // namespace
 
+namespace nnjit {
+// Record a failure detail for nnjit_last_error() from other translation units.
+void set_last_error(const char* msg) { t_last_error = msg; }
+}  // namespace nnjit
+
 // ------------------------------------------------------------------------ plan
 struct nnjit_plan_s {
     Problem p;

@@ -55,6 +55,9 @@ cudaError_t prepare_gemv_instance(int instance, int smem_bytes);
 cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, float* out,
                                  bool partials, CUtensorMap* tc_map, bool* ok);
 
+// Detail string for nnjit_last_error() (defined with the C ABI).
+void set_last_error(const char* msg);
+
 // Tensor maps for the TC family (host; uses the driver entry point).
 cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,
                                   const void* B, CUtensorMap* ta, CUtensorMap* tb,

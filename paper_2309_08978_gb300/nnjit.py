@@ -109,6 +109,7 @@ def load_library(path: str = LIB_PATH):
             "nnjit_plan_candidate": [vp, P(nnjit_candidate)],
             "nnjit_plan_destroy": [vp],
             "nnjit_cache_clear": [],
+            "nnjit_gemv_bf16_noalloc": [i64, i64, i64, vp, vp, vp, vp, i32, vp],
         }
         for name, args in sigs.items():
             f = getattr(lib, name)
@@ -291,6 +292,17 @@ def nnjit_plan_candidate(plan: Plan) -> dict:
 def nnjit_plan_destroy(plan: Plan):
     _check(load_library().nnjit_plan_destroy(plan.handle), "nnjit_plan_destroy")
     plan.handle = None
+
+
+NNJIT_NOALLOC_SCRATCH_FLOATS = 1 << 20
+
+
+def nnjit_gemv_bf16_noalloc(M: int, N: int, K: int, x, W, bias, C, split_k: int, stream=None):
+    """Decode GEMV whose split-K partials live in a fixed array inside the library; it
+    allocates nothing (see include/nnjit.h)."""
+    _check(load_library().nnjit_gemv_bf16_noalloc(M, N, K, _ptr(x), _ptr(W), _ptr(bias), _ptr(C),
+                                                  split_k, _stream(stream)),
+           "nnjit_gemv_bf16_noalloc")
 
 
 def nnjit_cache_clear():
