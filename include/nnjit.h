@@ -134,6 +134,9 @@ typedef struct {
     int32_t wave_eff_ppm;    /* predicted wave efficiency, parts per million */
     int32_t instance;        /* index of the precompiled kernel instance */
     int64_t predicted_cost;  /* model cost used for ordering (arbitrary units, lower first) */
+    int32_t reduce;          /* split-K reduction: 0 = partials in the plan's workspace, summed
+                                by a second kernel; 1 = TC only, inside a thread-block cluster
+                                of split_k CTAs through distributed shared memory */
 } nnjit_candidate;
 
 typedef struct nnjit_plan_s* nnjit_plan;

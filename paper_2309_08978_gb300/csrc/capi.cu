@@ -168,8 +168,11 @@ std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L) {
     return buf;
 }
 
+// Split-K partials go to a workspace unless they are reduced inside a cluster.
+bool uses_workspace(const nnjit_candidate& c) { return c.split_k > 1 && c.reduce == 0; }
+
 size_t ws_bytes_for(const Problem& p, const nnjit_candidate& c) {
-    if (c.split_k <= 1) return 0;
+    if (!uses_workspace(c)) return 0;
     return (size_t)c.split_k * (size_t)p.batch * (size_t)p.M * (size_t)p.N * sizeof(float);
 }
 
@@ -195,13 +198,14 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
     } else if ((ua & 15) || (ub & 15)) {
         return fail(NNJIT_ERR_UNSUPPORTED, "tensor-core and GEMV paths need 16-byte aligned A and B");
     }
-    if (c.split_k > 1 && !ws) return fail(NNJIT_ERR_INVALID_ARG, "split-K workspace missing");
+    const bool two_pass = uses_workspace(c);
+    if (two_pass && !ws) return fail(NNJIT_ERR_INVALID_ARG, "split-K workspace missing");
     LaunchArgs la;
     la.p = &p;
     la.c = &c;
     la.A = A;
     la.B = B;
-    la.bias = c.split_k > 1 ? nullptr : bias;
+    la.bias = two_pass ? nullptr : bias;
     la.C = C;
     la.ws = ws;
     la.err = pl->err;
@@ -211,13 +215,13 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
         CUtensorMap ta, tb, tcm;
         bool c_ok = false;
         const char* why = "";
-        float* out = c.split_k > 1 ? ws : C;
+        float* out = two_pass ? ws : C;
         {
             std::lock_guard<std::mutex> lk(pl->mu);
             if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B || pl->tm_C != out) {
                 e = encode_tc_tensor_maps(p, c, A, B, &ta, &tb, &why);
                 if (e != cudaSuccess) return fail(NNJIT_ERR_UNSUPPORTED, why);
-                encode_tc_output_map(p, c, out, c.split_k > 1, &tcm, &c_ok);
+                encode_tc_output_map(p, c, out, two_pass, &tcm, &c_ok);
                 if (!override_cand) {
                     pl->ta = ta; pl->tb = tb; pl->tc = tcm; pl->tm_c_ok = c_ok;
                     pl->tm_A = A; pl->tm_B = B; pl->tm_C = out; pl->tm_valid = true;
@@ -236,7 +240,7 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
         e = launch_gemv(la);
     }
     if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
-    if (c.split_k > 1) {
+    if (two_pass) {
         e = launch_splitk_reduce(ws, c.split_k, p, bias, C, s);
         if (e != cudaSuccess) return cuda_fail(e, "split-K reduce launch");
     }

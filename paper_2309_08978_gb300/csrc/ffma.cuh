@@ -33,6 +33,8 @@ __global__ void __launch_bounds__((BM / TM) * (BN / TN))
     __shared__ __align__(16) float As[2][BK][BM + 4];
     __shared__ __align__(16) float Bs[2][BK][BN + 4];
 
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int tid = threadIdx.x;
     const int ty = tid / TX, tx = tid % TX;
     const int m0 = blockIdx.y * BM, n0 = blockIdx.x * BN;

@@ -32,8 +32,7 @@ cudaError_t launch_ffma(const LaunchArgs& a) {
     if (gz > 65535) return cudaErrorInvalidValue;
     dim3 grid((unsigned)((p.N + c.bn - 1) / c.bn), (unsigned)((p.M + c.bm - 1) / c.bm), (unsigned)gz);
     if (grid.y > 65535) return cudaErrorInvalidValue;
-    k<<<grid, c.threads, 0, a.stream>>>(prm);
-    return cudaGetLastError();
+    return launch_pdl(k, grid, dim3(c.threads), 0, a.stream, prm);
 }
 
 }  // namespace nnjit

@@ -53,6 +53,8 @@ __device__ __forceinline__ float bf16_to_f(uint16_t h) { return __uint_as_float(
 template <int R, int U>
 __global__ void __launch_bounds__(256) gemv_nk_kernel(const GemvParams p) {
     extern __shared__ __align__(16) uint16_t xs[];
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const int warps = blockDim.x >> 5;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int s = blockIdx.y;
@@ -152,6 +154,8 @@ __global__ void __launch_bounds__(256) gemv_nk_kernel(const GemvParams p) {
 template <int U>
 __global__ void __launch_bounds__(256) gemv_kn_kernel(const GemvParams p) {
     extern __shared__ __align__(16) float red[];
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const int warps = blockDim.x >> 5;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int s = blockIdx.y;
@@ -231,6 +235,8 @@ int g_gemv_smem[8] = {0};
 __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, long long batch_mn,
                                      int M, int N, long long ldc, long long stride_c,
                                      const float* __restrict__ bias, float* __restrict__ C) {
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const long long mn = (long long)M * N;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < batch_mn;
          i += (long long)gridDim.x * blockDim.x) {
@@ -246,6 +252,8 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, lo
 
 __global__ void fill_bias_kernel(long long total, int M, int N, long long ldc, long long stride_c,
                                  const float* __restrict__ bias, float* __restrict__ C) {
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const long long mn = (long long)M * N;
     for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total;
          i += (long long)gridDim.x * blockDim.x) {
@@ -330,24 +338,22 @@ cudaError_t launch_gemv(const LaunchArgs& a) {
     }
     cudaError_t e = prepare_gemv_instance(c.instance, smem);
     if (e != cudaSuccess) return e;
-    kGemvKernels[c.instance]<<<grid, c.threads, smem, a.stream>>>(prm);
-    return cudaGetLastError();
+    return launch_pdl(kGemvKernels[c.instance], grid, dim3(c.threads), smem, a.stream, prm);
 }
 
 cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, const float* bias,
                                  float* C, cudaStream_t s) {
     const long long n = p.batch * p.M * p.N;
     if (n == 0) return cudaSuccess;
-    splitk_reduce_kernel<<<grid_for(n, 256), 256, 0, s>>>(ws, split, n, (int)p.M, (int)p.N, p.ldc,
-                                                          p.stride_c, bias, C);
-    return cudaGetLastError();
+    return launch_pdl(splitk_reduce_kernel, dim3(grid_for(n, 256)), dim3(256), 0, s, ws, split, n,
+                      (int)p.M, (int)p.N, p.ldc, p.stride_c, bias, C);
 }
 
 cudaError_t launch_fill_bias(const Problem& p, const float* bias, float* C, cudaStream_t s) {
     const long long n = p.batch * p.M * p.N;
     if (n == 0) return cudaSuccess;
-    fill_bias_kernel<<<grid_for(n, 256), 256, 0, s>>>(n, (int)p.M, (int)p.N, p.ldc, p.stride_c, bias, C);
-    return cudaGetLastError();
+    return launch_pdl(fill_bias_kernel, dim3(grid_for(n, 256)), dim3(256), 0, s, n, (int)p.M,
+                      (int)p.N, p.ldc, p.stride_c, bias, C);
 }
 
 cudaError_t launch_fill_scratch(void* dst, int64_t n_elems, int elem_bytes, uint32_t seed,

@@ -54,13 +54,25 @@ struct TileCoord {
     int b, s, tm, tn;
 };
 
+// Work item t -> (batch, K slice, tile row, tile column).  Persistent mode: slices of a
+// tile are separate work items.  Cluster mode: the split_k consecutive CTAs of a cluster
+// share one output tile and CTA rank = K slice.
+template <bool kCluster>
 __device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p) {
     TileCoord c;
     const int per = p.tiles_m * p.tiles_n;
-    const int r = t % per;
-    const int q = t / per;
-    c.s = q % p.split;
-    c.b = q / p.split;
+    int r, q;
+    if constexpr (kCluster) {
+        c.s = t % p.split;
+        const int ot = t / p.split;
+        r = ot % per;
+        c.b = ot / per;
+    } else {
+        r = t % per;
+        q = t / per;
+        c.s = q % p.split;
+        c.b = q / p.split;
+    }
     if (p.raster == 0) {
         c.tm = r % p.tiles_m;
         c.tn = r / p.tiles_m;
@@ -78,7 +90,7 @@ constexpr int kErrMmaFull = 0x112;
 constexpr int kErrEpiTmemFull = 0x121;
 constexpr int kErrDrain = 0x131;
 
-template <int kKind, bool kBMn, int BN>
+template <int kKind, bool kBMn, int BN, bool kCluster>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
     constexpr int kElem = kKind == 0 ? 2 : 4;
     constexpr int BK = 128 / kElem;                     // K elements per stage (one swizzle row)
@@ -134,6 +146,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         ptx::prefetch_tmap(&p.tmap_a);
         ptx::prefetch_tmap(&p.tmap_b);
         if (p.tma_store) ptx::prefetch_tmap(&p.tmap_c);
+        // Warm L2 with the first ring's worth of this CTA's operand tiles while the
+        // previous kernel may still be running: an L2 prefetch writes nothing, and L2 is
+        // where the previous kernel's stores land, so no stale copy can result.
+        if (blockIdx.x < p.total_tiles) {
+            const TileCoord tc = decode_tile<kCluster>(blockIdx.x, p);
+            const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
+            const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
+            for (int kb = kb0; kb < kb1 && kb < kb0 + S; ++kb) {
+                ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm * kBM, tc.b);
+                if constexpr (!kBMn) {
+                    ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN, tc.b);
+                } else {
+                    for (int j = 0; j < BN / kAtom; ++j)
+                        ptx::tma_prefetch_l2_3d(&p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b);
+                }
+            }
+        }
     }
     if (warp == 1) {
         ptx::tmem_alloc(ptx::smem_u32(tmem_slot), kTmemCols);
@@ -143,6 +172,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // Everything above overlaps the previous kernel's tail; global memory only from here.
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
 
     if (warp == 0) {
         // ---------------------------------------------------------------- TMA producer
@@ -151,7 +183,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t armed = 0, armed_parity = 0;
         bool ok = true;
         for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
-            const TileCoord tc = decode_tile(t, p);
+            const TileCoord tc = decode_tile<kCluster>(t, p);
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
             const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
             for (int kb = kb0; kb < kb1; ++kb) {
@@ -198,7 +230,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t iter = 0;
         bool ok = true;
         for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x, ++iter) {
-            const TileCoord tc = decode_tile(t, p);
+            const TileCoord tc = decode_tile<kCluster>(t, p);
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
             const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
             const uint32_t acc = iter & 1u;
@@ -259,11 +291,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t iter = 0;
         const long long MN = (long long)p.M * p.N;
         for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++iter) {
-            const TileCoord tc = decode_tile(t, p);
+            const TileCoord tc = decode_tile<kCluster>(t, p);
             const uint32_t acc = iter & 1u;
             const uint32_t acc_phase = (iter >> 1) & 1u;
             if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
             ptx::tc_fence_after();
+            if constexpr (kCluster) {
+                // The partial stays in TMEM until every CTA of the cluster has finished
+                // its main loop (see the reduction after the role branches).
+                continue;
+            }
             const int row = tc.tm * kBM + row_in_tile;
             const float* bias = p.split == 1 ? p.bias : nullptr;
             float* dst_row = p.split == 1
@@ -319,10 +356,74 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 }
             }
         }
-        if (p.tma_store && lane == 0) ptx::bulk_wait_all();
+        // the shared-memory sources must outlive the stores; the global writes complete
+        // with the kernel
+        if (p.tma_store && lane == 0) ptx::bulk_wait_all_read();
         __syncwarp();
     }
 
+    if constexpr (kCluster) {
+        // Cluster split-K reduction.  CTA rank r owns rows [r*R, (r+1)*R) of the tile
+        // (R = 128 / split).  (1) A cluster barrier: every CTA's main loop is over, so every
+        // ring is idle.  (2) Each CTA streams its partial rows from TMEM straight into the
+        // owning CTA's ring, slot [its rank][row][BN + 4] (fire-and-forget remote stores).
+        // (3) A second barrier publishes them.  (4) Each owner adds its rows over the
+        // slices in slice order (deterministic), adds bias, and stores them.  No CTA
+        // touches another's shared memory after the second barrier.
+        const int R = kBM / p.split;
+        const uint32_t my_rank = ptx::cluster_ctarank();
+        ptx::tc_fence_before();
+        ptx::cluster_sync();
+        ptx::tc_fence_after();
+        if (warp >= 2) {
+            const int q = warp & 3;
+            const int row = q * 32 + lane;
+            const uint32_t owner = (uint32_t)(row / R);
+            const uint32_t dst_row = ptx::map_shared_rank(smem_base, owner) +
+                                     (uint32_t)(((int)my_rank * R + row % R) * (BN + 4)) * 4u;
+#pragma unroll 1
+            for (int c = 0; c < BN / 32; ++c) {
+                uint32_t r[32];
+                ptx::tmem_ld32(tmem_base + ((uint32_t)(q * 32) << 16) + c * 32, r);
+                ptx::tmem_wait_ld(r);
+#pragma unroll
+                for (int j = 0; j < 32; j += 4)
+                    ptx::st_shared_cluster_v4(dst_row + (uint32_t)(c * 32 + j) * 4u, __uint_as_float(r[j]),
+                                              __uint_as_float(r[j + 1]), __uint_as_float(r[j + 2]),
+                                              __uint_as_float(r[j + 3]));
+            }
+        }
+        ptx::cluster_sync();
+        const TileCoord tc = decode_tile<true>(blockIdx.x, p);
+        constexpr int kVec = BN / 4;
+        const float* recv = reinterpret_cast<const float*>(smem);
+        float* Cb = p.C + (long long)tc.b * p.stride_c;
+        const int row0 = (int)my_rank * R;
+        for (int e = threadIdx.x; e < R * kVec; e += kThreads) {
+            const int lr = e / kVec;
+            const int cv = e % kVec;
+            const int row = tc.tm * kBM + row0 + lr;
+            const int col = tc.tn * BN + cv * 4;
+            if (row >= p.M || col >= p.N) continue;
+            float4 a = *reinterpret_cast<const float4*>(recv + (size_t)lr * (BN + 4) + cv * 4);
+            for (int s = 1; s < p.split; ++s) {
+                const float4 v = *reinterpret_cast<const float4*>(recv + (size_t)(s * R + lr) * (BN + 4) + cv * 4);
+                a.x += v.x; a.y += v.y; a.z += v.z; a.w += v.w;
+            }
+            float o[4] = {a.x, a.y, a.z, a.w};
+            float* dst = Cb + (long long)row * p.ldc + col;
+            if (col + 4 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+                if (p.bias) {
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) o[j] += __ldg(p.bias + col + j);
+                }
+                *reinterpret_cast<float4*>(dst) = make_float4(o[0], o[1], o[2], o[3]);
+            } else {
+                for (int j = 0; j < 4 && col + j < p.N; ++j)
+                    dst[j] = p.bias ? o[j] + __ldg(p.bias + col + j) : o[j];
+            }
+        }
+    }
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
@@ -331,16 +432,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
 using TcKernel = void (*)(TcParams);
 
-// Instance table, indexed as tc_instance(): ((dtype_i * 2 + kn) * 3 + bn_i).
-const TcKernel kTcKernels[12] = {
-    tc_gemm_kernel<0, false, 64>, tc_gemm_kernel<0, false, 128>, tc_gemm_kernel<0, false, 256>,
-    tc_gemm_kernel<0, true, 64>,  tc_gemm_kernel<0, true, 128>,  tc_gemm_kernel<0, true, 256>,
-    tc_gemm_kernel<1, false, 64>, tc_gemm_kernel<1, false, 128>, tc_gemm_kernel<1, false, 256>,
-    tc_gemm_kernel<1, true, 64>,  tc_gemm_kernel<1, true, 128>,  tc_gemm_kernel<1, true, 256>,
+// Instance table, indexed as tc_instance(): cluster * 12 + (dtype_i * 2 + kn) * 3 + bn_i.
+#define NNJIT_TC_ROW(K, MN, CL) \
+    tc_gemm_kernel<K, MN, 64, CL>, tc_gemm_kernel<K, MN, 128, CL>, tc_gemm_kernel<K, MN, 256, CL>
+const TcKernel kTcKernels[24] = {
+    NNJIT_TC_ROW(0, false, false), NNJIT_TC_ROW(0, true, false),
+    NNJIT_TC_ROW(1, false, false), NNJIT_TC_ROW(1, true, false),
+    NNJIT_TC_ROW(0, false, true),  NNJIT_TC_ROW(0, true, true),
+    NNJIT_TC_ROW(1, false, true),  NNJIT_TC_ROW(1, true, true),
 };
+#undef NNJIT_TC_ROW
 
 std::mutex g_prep_mu;
-int g_prepared_smem[12] = {0};
+int g_prepared_smem[24] = {0};
 
 // Driver entry point for cuTensorMapEncodeTiled, fetched through the runtime so the
 // library does not link against libcuda.
@@ -366,7 +470,7 @@ EncodeTiledFn get_encode_fn() {
 }  // namespace
 
 cudaError_t prepare_tc_instance(int instance, int smem_bytes) {
-    if (instance < 0 || instance >= 12) return cudaErrorInvalidValue;
+    if (instance < 0 || instance >= 24) return cudaErrorInvalidValue;
     std::lock_guard<std::mutex> lk(g_prep_mu);
     if (g_prepared_smem[instance] >= smem_bytes) return cudaSuccess;
     cudaError_t e = cudaFuncSetAttribute(kTcKernels[instance],
@@ -450,7 +554,11 @@ cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, flo
 cudaError_t launch_tc(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
-    if (c.instance < 0 || c.instance >= 12 || !a.tmap_a || !a.tmap_b) return cudaErrorInvalidValue;
+    if (c.instance < 0 || c.instance >= 24 || !a.tmap_a || !a.tmap_b) return cudaErrorInvalidValue;
+    const bool cluster = c.instance >= 12;
+    if (cluster != (c.reduce == 1)) return cudaErrorInvalidValue;
+    if (cluster && (c.split_k < 2 || c.split_k > 8 || (c.split_k & (c.split_k - 1)) != 0))
+        return cudaErrorInvalidValue;
     if (c.stages < 2 || c.stages > kMaxStages) return cudaErrorInvalidValue;
     TcParams prm;
     prm.tmap_a = *a.tmap_a;
@@ -477,14 +585,30 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     prm.total_tiles = (int)total;
     prm.stages = c.stages;
     prm.raster = c.raster;
-    const int grid = (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
+    // persistent: at most the candidate's grid; cluster mode: one CTA per (tile, slice)
+    const int grid = cluster ? (int)total : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
     // ring + alignment slack + barriers/TMEM slot/abort flag
     const int stage_bytes = (kBM + c.bn) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     cudaError_t e = prepare_tc_instance(c.instance, smem);
     if (e != cudaSuccess) return e;
-    kTcKernels[c.instance]<<<grid, kThreads, smem, a.stream>>>(prm);
-    return cudaGetLastError();
+    if (!cluster)
+        return launch_pdl(kTcKernels[c.instance], dim3(grid), dim3(kThreads), smem, a.stream, prm);
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(kThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = a.stream;
+    cudaLaunchAttribute attr[2];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    attr[1].id = cudaLaunchAttributeClusterDimension;
+    attr[1].val.clusterDim.x = (unsigned)c.split_k;
+    attr[1].val.clusterDim.y = 1;
+    attr[1].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, kTcKernels[c.instance], prm);
 }
 
 }  // namespace nnjit

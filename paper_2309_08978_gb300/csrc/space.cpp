@@ -55,7 +55,7 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
     const int64_t num_kb = ceil_div(K, BK);
     const int bns[3] = {64, 128, 256};
     const int splits[4] = {1, 2, 4, 8};
-    *naive = 3 * (MC::kTcMaxStages - 1) * 4 * 2;  // BN x stage count 2..8 x split x raster
+    *naive = 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2;  // BN x stages 2..8 x split x raster x reduce
     for (int bn : bns) {
         if (bn > 64 && bn > pow2_ceil(N)) continue;  // no tile wider than the padded N
         const int stage_bytes = (BM + bn) * 128;
@@ -73,8 +73,13 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
         for (int split : splits) {
             // split only while the previous split count still leaves SMs idle
             if (split > 1 && (tiles * (split / 2) >= L.sm_count || num_kb < 4 * split)) continue;
+            // split-K partials: summed by a second kernel (reduce 0) or, one output tile
+            // per thread-block cluster of `split` CTAs, through distributed shared memory
+            // (reduce 1; the partial tile reuses the idle ring)
+            for (int reduce = 0; reduce < (split > 1 ? 2 : 1); ++reduce)
             for (int raster = 0; raster < 2; ++raster) {
                 if (raster == 1 && (tiles_m == 1 || tiles_n == 1)) continue;
+                if (reduce == 1 && (raster == 1 || stages * stage_bytes < 128 * (bn + 4) * 4)) continue;
                 nnjit_candidate c = blank();
                 c.family = NNJIT_FAMILY_TC;
                 c.bm = BM; c.bn = bn; c.bk = BK;
@@ -87,22 +92,28 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 c.tmem_cols = tmem;
                 c.regs_per_thread = regs;
                 c.blocks_per_sm = blk;
+                c.reduce = reduce;
                 const int64_t work = tiles * split;
                 const int64_t slots = (int64_t)L.sm_count * blk;
-                const int64_t grid = std::min(work, slots);
-                const int64_t waves = ceil_div(work, grid);
+                // persistent grid; cluster mode launches one CTA per (tile, slice)
+                const int64_t grid = reduce ? work : std::min(work, slots);
+                const int64_t waves = ceil_div(work, std::min(work, slots));
                 c.grid = (int32_t)grid;
-                c.wave_eff_ppm = (int32_t)(work * 1000000 / (waves * grid));
-                // per k-block: MMA clocks (2*BN for both bf16 and tf32 at BK = 128 bytes)
-                // against the operand feed (stage bytes over the per-SM L2 feed)
-                const int64_t t_kb = std::max<int64_t>(2 * bn, ceil_div(stage_bytes,
-                                                                        MC::kFeedBytesPerClk));
+                c.wave_eff_ppm = (int32_t)(work * 1000000 / (waves * std::min(work, slots)));
+                // per k-block: one MMA instruction costs about as much as N = 256 (the
+                // tensor core works on all 256 columns at once), so the MMA clocks are
+                // those of BN = 256, against the operand feed (stage bytes over the per-SM
+                // L2 feed)
+                const int64_t t_kb = std::max<int64_t>(2 * 256, ceil_div(stage_bytes,
+                                                                         MC::kFeedBytesPerClk));
                 int64_t cost = waves * t_kb * ceil_div(num_kb, split);
-                if (split > 1)
+                if (split > 1 && reduce == 0)
                     cost += MC::kLaunchClk +
                             ceil_div(2LL * split * p.batch * M * N * 4, MC::kHbmBytesPerClk);
+                if (split > 1 && reduce == 1)
+                    cost += waves * (128LL * bn * 4 / MC::kFeedBytesPerClk);  // DSMEM reduction
                 c.predicted_cost = cost;
-                c.instance = tc_instance(p.dtype, p.b_layout, bn);
+                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce);
                 v.push_back(c);
             }
         }
@@ -284,11 +295,11 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 
 }  // namespace
 
-int tc_instance(int dtype, int b_layout, int bn) {
+int tc_instance(int dtype, int b_layout, int bn, int cluster) {
     const int bi = bn == 64 ? 0 : bn == 128 ? 1 : bn == 256 ? 2 : -1;
     if (bi < 0) return -1;
     const int di = dtype == NNJIT_BF16 ? 0 : 1;
-    return (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
+    return (cluster ? 12 : 0) + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
 }
 
 // The 12 (thread tile, block tile) pairs with 64..256 threads, in enumeration order.
