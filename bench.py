@@ -46,6 +46,30 @@ def shape_bytes(s, dtype):
     return b + (4 * s.N if s.has_bias else 0)
 
 
+def kernel_key(s, dtype, cand):
+    """Identifies one kernel configuration on one product (the traffic table's key)."""
+    fam = {0: "ffma", 1: "tc", 2: "gemv"}[cand["family"]]
+    return (f"{fam} {dtype} {s.batch}x{s.M}x{s.N}x{s.K} {s.b_layout} bm{cand['bm']} bn{cand['bn']} "
+            f"st{cand['stages']} split{cand['split_k']} red{cand['reduce']} rast{cand['raster']}")
+
+
+def lookup_traffic(key):
+    """DRAM bytes per launch (ncu dram__bytes_read.sum + dram__bytes_write.sum) recorded in
+    profiles/dram_traffic.txt for exactly this kernel configuration, else None."""
+    path = os.path.join(ROOT, "profiles", "dram_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        for line in f:
+            line = line.strip()
+            if not line or line.startswith("#") or "|" not in line:
+                continue
+            k, v = line.rsplit("|", 1)
+            if k.strip() == key:
+                return int(float(v.strip()))
+    return None
+
+
 def load_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -248,6 +272,8 @@ def run_ours(args, workload, rank, world, local_rank):
         return t.pin_memory()
 
     # ---- operands, plans (the JIT phase), tuner vs exhaustive sweep
+    if args.cache and os.path.exists(args.cache):
+        nj.nnjit_cache_load(args.cache)
     items = []
     tune = {"budget_ms_per_shape": args.budget_ms, "shapes": []}
     for s in workload.shapes:
@@ -294,6 +320,8 @@ def run_ours(args, workload, rank, world, local_rank):
         items.append({"shape": s, "plan": plan, "sets": sets, "host": (A, B, bias),
                       "launches": launches, "family": info["family"]})
     tune["total_plan_ms"] = round(sum(e["plan_ms"] for e in tune["shapes"]), 2)
+    if args.cache:
+        nj.nnjit_cache_save(args.cache)
     ratios = [e["pick_over_best"] for e in tune["shapes"] if e.get("pick_over_best")]
     if ratios:
         tune["max_pick_over_best"] = max(ratios)
@@ -346,12 +374,14 @@ def run_ours(args, workload, rank, world, local_rank):
     barrier()
     evs = [torch.cuda.Event(enable_timing=True) for _ in range(len(items) + 1)]
     t_wall = time.perf_counter()
+    torch.cuda.nvtx.range_push("timed_region")
     with torch.cuda.stream(stream):
         evs[0].record(stream)
         for i in range(len(items)):
             block(i, args.steps)
             evs[i + 1].record(stream)
     stream.synchronize()
+    torch.cuda.nvtx.range_pop()
     barrier()
     wall = time.perf_counter() - t_wall
     clocks = sampler.stop()
@@ -386,7 +416,8 @@ def run_ours(args, workload, rank, world, local_rank):
         ach = ds.flops / dur_s / 1e12
         roof = {"bound": "tensor", "achieved": round(ach, 2), "peak": round(peak_t, 1),
                 "unit": "TFLOP/s", "frac": round(ach / peak_t, 4)}
-    roof.update({"traffic": None, "kernel": f"{ds.name} {ds.batch}x{ds.M}x{ds.N}x{ds.K} {dtype}",
+    dom_key = kernel_key(ds, dtype, items[dom]["plan"].candidate())
+    roof.update({"traffic": lookup_traffic(dom_key), "kernel": dom_key,
                  "peak_source": ("measured bf16 x nominal tf32/bf16 ratio" if dtype == "tf32"
                                  else peaks["source"]) + f" ({peaks['source']})",
                  "units_per_launch": f"{ds.flops} flop, {alg_bytes} algorithmic bytes"})
@@ -481,11 +512,21 @@ def main(argv=None):
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--e2e-steps", type=int, default=200)
+    ap.add_argument("--cache", default=None,
+                    help="plan-cache file: loaded before tuning if present, saved after")
+    ap.add_argument("--only", default=None,
+                    help="run a single product of the workload (by name), e.g. for profiling")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from synthetic import WORKLOADS
     workload = WORKLOADS[args.workload]
+    if args.only:
+        import dataclasses
+        shapes = tuple(s for s in workload.shapes if s.name == args.only)
+        if not shapes:
+            ap.error(f"--only: no product named {args.only} in {args.workload}")
+        workload = dataclasses.replace(workload, shapes=shapes)
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))

@@ -278,6 +278,23 @@ nnjit_status nnjit_cache_clear(void);
 /* Number of choices currently in the process plan cache. */
 int32_t nnjit_cache_size(void);
 
+/*
+ * Persist the plan cache -- the kernel database of Sec. 5.3, keyed by kernel type, shape,
+ * layout, strides, dtype and device (name, compute capability, SM count) -- to a text
+ * file at `path` (overwritten), so that tuning results outlive the process.
+ * NNJIT_ERR_INVALID_ARG if the file cannot be written.
+ */
+nnjit_status nnjit_cache_save(const char* path);
+
+/*
+ * Merge the entries of a file written by nnjit_cache_save into the plan cache (entries
+ * already present are replaced); *loaded (may be NULL) receives the number read.  An entry
+ * is used by nnjit_matmul_plan_ex only if its candidate is still a member of the lite
+ * space this library builds for that problem on this device; otherwise the problem is
+ * tuned afresh.  INVALID_ARG if the file cannot be read or is not a cache file.
+ */
+nnjit_status nnjit_cache_load(const char* path, int32_t* loaded);
+
 #ifdef __cplusplus
 }
 #endif

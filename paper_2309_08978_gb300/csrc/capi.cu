@@ -512,10 +512,16 @@ nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, 
     if (use_cache) {
         std::lock_guard<std::mutex> lk(g_cache_mu);
         auto it = cache().find(key);
-        if (it != cache().end()) {
+        // an entry (possibly loaded from a file) is honoured only if its candidate is
+        // still a member of the space built now
+        int member = -1;
+        if (it != cache().end())
+            for (size_t i = 0; i < space.size() && member < 0; ++i)
+                if (std::memcmp(&space[i], &it->second.cand, sizeof(nnjit_candidate)) == 0) member = (int)i;
+        if (it != cache().end() && member >= 0) {
             const CacheEntry& ce = it->second;
             pl->cand = ce.cand;
-            pl->chosen_index = ce.chosen_index;
+            pl->chosen_index = member;
             pl->timings = ce.timings;
             pl->tune_ms = ce.tune_ms;
             pl->timed = ce.timed;
@@ -780,6 +786,94 @@ nnjit_status nnjit_cache_clear(void) {
 int32_t nnjit_cache_size(void) {
     std::lock_guard<std::mutex> lk(g_cache_mu);
     return (int32_t)cache().size();
+}
+
+// File format: a header line, then one line per entry:
+//   key \t 19 candidate integers \t chosen_index space_size naive tune_ms timed \t
+//   n (index us)*n
+static const char* kCacheHeader = "nnjit-plan-cache v1";
+
+nnjit_status nnjit_cache_save(const char* path) {
+    if (!path) return fail(NNJIT_ERR_INVALID_ARG, "path is NULL");
+    std::string tmp = std::string(path) + ".tmp";
+    FILE* f = std::fopen(tmp.c_str(), "w");
+    if (!f) return fail(NNJIT_ERR_INVALID_ARG, std::string("cannot write ") + path);
+    std::fprintf(f, "%s\n", kCacheHeader);
+    {
+        std::lock_guard<std::mutex> lk(g_cache_mu);
+        for (const auto& kv : cache()) {
+            const CacheEntry& e = kv.second;
+            const nnjit_candidate& c = e.cand;
+            std::fprintf(f, "%s\t%d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %lld %d\t%d %d %lld %.6f %d\t%zu",
+                         kv.first.c_str(), c.family, c.bm, c.bn, c.bk, c.tm, c.tn, c.stages,
+                         c.split_k, c.raster, c.threads, c.smem_bytes, c.tmem_cols,
+                         c.regs_per_thread, c.blocks_per_sm, c.grid, c.wave_eff_ppm, c.instance,
+                         (long long)c.predicted_cost, c.reduce, e.chosen_index, e.space_size,
+                         (long long)e.naive, e.tune_ms, e.timed ? 1 : 0, e.timings.size());
+            for (const auto& t : e.timings) std::fprintf(f, " %d %.6f", t.first, t.second);
+            std::fprintf(f, "\n");
+        }
+    }
+    const bool ok = std::fclose(f) == 0 && std::rename(tmp.c_str(), path) == 0;
+    if (!ok) return fail(NNJIT_ERR_INVALID_ARG, std::string("cannot write ") + path);
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_cache_load(const char* path, int32_t* loaded) {
+    if (!path) return fail(NNJIT_ERR_INVALID_ARG, "path is NULL");
+    FILE* f = std::fopen(path, "r");
+    if (!f) return fail(NNJIT_ERR_INVALID_ARG, std::string("cannot read ") + path);
+    std::string content;
+    char buf[4096];
+    size_t n;
+    while ((n = std::fread(buf, 1, sizeof buf, f)) > 0) content.append(buf, n);
+    std::fclose(f);
+    size_t pos = content.find('\n');
+    if (pos == std::string::npos || content.substr(0, pos) != kCacheHeader)
+        return fail(NNJIT_ERR_INVALID_ARG, "not an nnjit plan cache file");
+    std::map<std::string, CacheEntry> got;
+    while (pos != std::string::npos && pos + 1 < content.size()) {
+        const size_t end = content.find('\n', pos + 1);
+        const std::string line = content.substr(pos + 1, end == std::string::npos ? std::string::npos : end - pos - 1);
+        pos = end;
+        if (line.empty()) continue;
+        const size_t t1 = line.find('\t');
+        if (t1 == std::string::npos) return fail(NNJIT_ERR_INVALID_ARG, "malformed cache line");
+        CacheEntry e{};
+        nnjit_candidate& c = e.cand;
+        long long cost = 0, naive = 0;
+        int timed = 0;
+        size_t ntim = 0;
+        int used = 0;
+        const char* rest = line.c_str() + t1 + 1;
+        if (std::sscanf(rest, "%d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %lld %d %d %d %lld %lf %d %zu%n",
+                        &c.family, &c.bm, &c.bn, &c.bk, &c.tm, &c.tn, &c.stages, &c.split_k,
+                        &c.raster, &c.threads, &c.smem_bytes, &c.tmem_cols, &c.regs_per_thread,
+                        &c.blocks_per_sm, &c.grid, &c.wave_eff_ppm, &c.instance, &cost, &c.reduce,
+                        &e.chosen_index, &e.space_size, &naive, &e.tune_ms, &timed, &ntim, &used) != 25 ||
+            ntim > 4096)
+            return fail(NNJIT_ERR_INVALID_ARG, "malformed cache line");
+        c.predicted_cost = cost;
+        e.naive = naive;
+        e.timed = timed != 0;
+        rest += used;
+        for (size_t i = 0; i < ntim; ++i) {
+            int idx = 0;
+            double us = 0;
+            int u2 = 0;
+            if (std::sscanf(rest, " %d %lf%n", &idx, &us, &u2) != 2)
+                return fail(NNJIT_ERR_INVALID_ARG, "malformed cache timings");
+            rest += u2;
+            e.timings.emplace_back(idx, us);
+        }
+        got[line.substr(0, t1)] = e;
+    }
+    {
+        std::lock_guard<std::mutex> lk(g_cache_mu);
+        for (auto& kv : got) cache()[kv.first] = kv.second;
+    }
+    if (loaded) *loaded = (int32_t)got.size();
+    return NNJIT_OK;
 }
 
 }  // extern "C"

@@ -110,6 +110,8 @@ def load_library(path: str = LIB_PATH):
             "nnjit_plan_destroy": [vp],
             "nnjit_cache_clear": [],
             "nnjit_gemv_bf16_noalloc": [i64, i64, i64, vp, vp, vp, vp, i32, vp],
+            "nnjit_cache_save": [ctypes.c_char_p],
+            "nnjit_cache_load": [ctypes.c_char_p, P(i32)],
         }
         for name, args in sigs.items():
             f = getattr(lib, name)
@@ -311,3 +313,13 @@ def nnjit_cache_clear():
 
 def nnjit_cache_size() -> int:
     return int(load_library().nnjit_cache_size())
+
+
+def nnjit_cache_save(path: str):
+    _check(load_library().nnjit_cache_save(os.fsencode(path)), "nnjit_cache_save")
+
+
+def nnjit_cache_load(path: str) -> int:
+    n = ctypes.c_int32(0)
+    _check(load_library().nnjit_cache_load(os.fsencode(path), ctypes.byref(n)), "nnjit_cache_load")
+    return n.value

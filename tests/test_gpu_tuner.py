@@ -1,0 +1,127 @@
+"""The JIT tuner and plan cache on the GPU: budget semantics, cache hits, exhaustive
+sweeps, the persisted kernel database, host-side fault injection, end-to-end host path."""
+import os
+
+import numpy as np
+import pytest
+
+from synthetic import Shape, make_operands
+from gpu_util import run_plan, compare
+
+pytestmark = pytest.mark.gpu
+
+nj = pytest.importorskip("paper_2309_08978_gb300")
+
+
+def _desc(flags=0):
+    return nj.make_desc(512, 768, 768, "bf16", "NK", has_bias=True, flags=flags)
+
+
+def test_budget_zero_takes_top_ranked_untimed():
+    desc = _desc(nj.NNJIT_PLAN_NO_CACHE)
+    lim = nj.nnjit_device_limits_query(0)
+    cands, _ = nj.nnjit_space_enumerate(desc, lim)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        info = plan.describe()
+        assert info["chosen_index"] == 0 and info["timed"] is False
+        assert plan.candidate() == cands[0]
+    with pytest.raises(nj.NnjitError) as ei:
+        nj.nnjit_matmul_plan_ex(_desc(nj.NNJIT_PLAN_NO_CACHE | nj.NNJIT_PLAN_REQUIRE_TIMED), 0.0)
+    assert ei.value.status == nj.NNJIT_ERR_BUDGET
+
+
+def test_exhaustive_times_every_candidate_and_picks_the_fastest():
+    desc = _desc(nj.NNJIT_PLAN_EXHAUSTIVE)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        info = plan.describe()
+    assert len(info["timings_us"]) + len(info["failed"]) == info["space_size"]
+    assert not info["failed"]
+    # the pick is the fastest re-timed candidate (re-timing can reorder near-ties)
+    times = dict((int(i), t) for i, t in info["timings_us"])
+    assert times[info["chosen_index"]] <= min(times.values()) * 1.05
+
+
+def test_cache_hit_and_persistence(tmp_path):
+    nj.nnjit_cache_clear()
+    desc = _desc()
+    with nj.nnjit_matmul_plan_ex(desc, 200.0) as p1:
+        i1 = p1.describe()
+        assert i1["from_cache"] is False and i1["timed"] is True
+    assert nj.nnjit_cache_size() == 1
+    with nj.nnjit_matmul_plan_ex(desc, 200.0) as p2:
+        i2 = p2.describe()
+        assert i2["from_cache"] is True and i2["candidate"] == i1["candidate"]
+    path = str(tmp_path / "plans.cache")
+    nj.nnjit_cache_save(path)
+    nj.nnjit_cache_clear()
+    assert nj.nnjit_cache_load(path) == 1
+    with nj.nnjit_matmul_plan_ex(desc, 200.0) as p3:
+        i3 = p3.describe()
+        assert i3["from_cache"] is True and i3["candidate"] == i1["candidate"]
+        shape = Shape("t", 512, 768, 768, 1, "NK", True)
+        A, B, bias = make_operands(shape, 30, "bf16", ints=True)
+        compare(run_plan(p3, A, B, bias, 512, 768), A, B, bias, "NK", "bf16", exact=True)
+    nj.nnjit_cache_clear()
+
+
+def test_cached_candidate_outside_the_space_is_retuned(tmp_path):
+    nj.nnjit_cache_clear()
+    desc = _desc()
+    with nj.nnjit_matmul_plan_ex(desc, 50.0):
+        pass
+    path = tmp_path / "plans.cache"
+    nj.nnjit_cache_save(str(path))
+    lines = path.read_text().splitlines()
+    key, cand, rest, tim = lines[1].split("\t")
+    fields = cand.split()
+    fields[2] = "96"                      # BN = 96 is not a member of any space
+    path.write_text(lines[0] + "\n" + "\t".join([key, " ".join(fields), rest, tim]) + "\n")
+    nj.nnjit_cache_clear()
+    assert nj.nnjit_cache_load(str(path)) == 1
+    with nj.nnjit_matmul_plan_ex(desc, 50.0) as plan:
+        info = plan.describe()
+        assert info["from_cache"] is False and info["candidate"]["bn"] != 96
+    nj.nnjit_cache_clear()
+
+
+@pytest.mark.parametrize("kind", ["launch", "timeout"])
+def test_fault_injection_skips_the_candidate(kind, monkeypatch):
+    """Host-side injection: candidate 0 reports a launch error or an expired watchdog;
+    the tuner must skip it and still deliver a correct plan."""
+    monkeypatch.setenv("NNJIT_FAULT", f"{kind}:0")
+    desc = _desc(nj.NNJIT_PLAN_NO_CACHE | nj.NNJIT_PLAN_EXHAUSTIVE)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        info = plan.describe()
+        assert 0 in info["failed"] and info["chosen_index"] != 0
+        shape = Shape("t", 512, 768, 768, 1, "NK", True)
+        A, B, bias = make_operands(shape, 31, "bf16", ints=True)
+        compare(run_plan(plan, A, B, bias, 512, 768), A, B, bias, "NK", "bf16", exact=True)
+
+
+def test_run_host_end_to_end():
+    import torch
+    shape = Shape("t", 300, 520, 264, 1, "KN", True)
+    A, B, bias = make_operands(shape, 32, "tf32")
+    desc = nj.make_desc(300, 520, 264, "tf32", "KN", has_bias=True)
+    with nj.nnjit_matmul_plan_ex(desc, 20.0) as plan:
+        hA = torch.from_numpy(A).pin_memory()
+        hB = torch.from_numpy(B).pin_memory()
+        hbias = torch.from_numpy(bias).pin_memory()
+        hC = torch.empty((300, 520), dtype=torch.float32).pin_memory()
+        nj.nnjit_matmul_run_host(plan, hA, hB, hbias, hC)
+        torch.cuda.synchronize()
+        plan.check()
+        compare(hC.numpy(), A, B, bias, "KN", "tf32")
+
+
+def test_invalid_run_arguments():
+    import torch
+    with nj.nnjit_matmul_plan_ex(nj.make_desc(256, 256, 256, "bf16", "NK"), 0.0) as plan:
+        A = torch.zeros((256, 256), dtype=torch.bfloat16, device="cuda")
+        C = torch.zeros((256, 256), dtype=torch.float32, device="cuda")
+        with pytest.raises(nj.NnjitError) as ei:
+            plan.run(A.data_ptr() + 2, A, None, C)          # misaligned A
+        assert ei.value.status == nj.NNJIT_ERR_UNSUPPORTED
+        with pytest.raises(nj.NnjitError) as ei:
+            plan.run(A, None, None, C)
+        assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
