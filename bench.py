@@ -46,6 +46,22 @@ def shape_bytes(s, dtype):
     return b + (4 * s.N if s.has_bias else 0)
 
 
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The largest of every rank's value (the slowest rank's time); identity at world 1."""
+    if world <= 1:
+        return float(x)
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, flops_per_step: int, steps: int, ms: float) -> float:
+    """Whole-job TFLOP/s: every replica ran `steps` steps; `ms` is the slowest rank's time."""
+    return world * flops_per_step * steps / (ms / 1e3) / 1e12
+
+
 def kernel_key(s, dtype, cand):
     """Identifies one kernel configuration on one product (the traffic table's key)."""
     fam = {0: "ffma", 1: "tc", 2: "gemv"}[cand["family"]]
@@ -386,18 +402,13 @@ def run_ours(args, workload, rank, world, local_rank):
     wall = time.perf_counter() - t_wall
     clocks = sampler.stop()
     per_item_ms = [evs[i].elapsed_time(evs[i + 1]) for i in range(len(items))]
-    total_ms = sum(per_item_ms)
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([total_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(per_item_ms), world, dev)
     for it in items:
         it["plan"].check()
 
     flops_step = sum(it["shape"].flops for it in items)
     ms_per_step = total_ms / args.steps
-    value = world * flops_step * args.steps / (total_ms / 1e3) / 1e12
+    value = job_throughput(world, flops_step, args.steps, total_ms)
 
     # ---- roofline of the dominant kernel (largest share of the timed region)
     dom = max(range(len(items)), key=lambda i: per_item_ms[i])
@@ -456,13 +467,8 @@ def run_ours(args, workload, rank, world, local_rank):
         e1.record(stream)
     stream.synchronize()
     barrier()
-    e2e_ms = e0.elapsed_time(e1)
-    if world > 1:
-        import torch.distributed as dist
-        t = torch.tensor([e2e_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        e2e_ms = float(t.item())
-    e2e_value = world * flops_step * e2e_steps / (e2e_ms / 1e3) / 1e12
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    e2e_value = job_throughput(world, flops_step, e2e_steps, e2e_ms)
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
