@@ -173,8 +173,9 @@ def _blank():
     return c
 
 
-def tc_instance(dtype, b_layout, bn, cluster):
-    return (12 if cluster else 0) + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 3 + \
+def tc_instance(dtype, b_layout, bn, cluster, bm):
+    variant = 2 if bm == 64 else (1 if cluster else 0)
+    return variant * 12 + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 3 + \
         {64: 0, 128: 1, 256: 2}[bn]
 
 
@@ -201,10 +202,13 @@ def _tc(p, lim):
     M, N, K = max(p.M, 1), max(p.N, 1), max(p.K, 1)
     num_kb = cdiv(K, bk)
     out = []
-    for bn in (64, 128, 256):
+    for bm, bn in [(m, n) for m in (TC_BM, 64) for n in (64, 128, 256)]:
         if bn > 64 and bn > pow2_at_least(N):
             continue
-        stage = (TC_BM + bn) * 128
+        # 64-row tiles only where 128-row tiles would leave SMs idle
+        if bm == 64 and p.batch * cdiv(M, TC_BM) * cdiv(N, bn) >= lim["sm_count"]:
+            continue
+        stage = (bm + bn) * 128
         stages = min(TC_MAX_STAGES, (lim["smem_per_block_optin"] - TC_FIXED_SMEM) // stage)
         if stages < 2:
             continue
@@ -215,7 +219,7 @@ def _tc(p, lim):
         blk = block_core(lim, TC_REGS, TC_THREADS, smem, tmem)
         if blk < 1:
             continue
-        tiles_m, tiles_n = cdiv(M, TC_BM), cdiv(N, bn)
+        tiles_m, tiles_n = cdiv(M, bm), cdiv(N, bn)
         tiles = p.batch * tiles_m * tiles_n
         for split in (1, 2, 4, 8):
             if split > 1 and (tiles * (split // 2) >= lim["sm_count"] or num_kb < 4 * split):
@@ -224,27 +228,27 @@ def _tc(p, lim):
                 for raster in (0, 1):
                     if raster == 1 and (tiles_m == 1 or tiles_n == 1):
                         continue
-                    if reduce == 1 and (raster == 1 or stages * stage < TC_BM * (bn + 4) * 4):
+                    if reduce == 1 and (bm != TC_BM or raster == 1 or stages * stage < TC_BM * (bn + 4) * 4):
                         continue
                     c = _blank()
                     work = tiles * split
                     slots = lim["sm_count"] * blk
                     live = min(work, slots)
                     waves = cdiv(work, live)
-                    t_kb = max(2 * 256, cdiv(stage, FEED_BYTES_PER_CLK))
+                    t_kb = max(2 * 256 * bm // TC_BM, cdiv(stage, FEED_BYTES_PER_CLK))
                     cost = waves * t_kb * cdiv(num_kb, split)
                     if split > 1 and reduce == 0:
                         cost += LAUNCH_CLK + cdiv(2 * split * p.batch * M * N * 4, HBM_BYTES_PER_CLK)
                     if split > 1 and reduce == 1:
                         cost += waves * (TC_BM * bn * 4 // FEED_BYTES_PER_CLK)
-                    c.update(family=FAMILY_TC, bm=TC_BM, bn=bn, bk=bk, stages=stages, split_k=split,
+                    c.update(family=FAMILY_TC, bm=bm, bn=bn, bk=bk, stages=stages, split_k=split,
                              raster=raster, threads=TC_THREADS, smem_bytes=smem, tmem_cols=tmem,
                              regs_per_thread=TC_REGS, blocks_per_sm=blk,
                              grid=work if reduce else live, wave_eff_ppm=work * 1000000 // (waves * live),
-                             instance=tc_instance(p.dtype, p.b_layout, bn, reduce),
+                             instance=tc_instance(p.dtype, p.b_layout, bn, reduce, bm),
                              predicted_cost=cost, reduce=reduce)
                     out.append(c)
-    return out, 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2
+    return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2
 
 
 def _ffma(p, lim):

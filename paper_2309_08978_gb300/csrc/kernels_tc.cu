@@ -31,7 +31,6 @@ namespace nnjit {
 
 namespace {
 
-constexpr int kBM = 128;
 constexpr int kThreads = 192;
 constexpr int kMaxStages = 8;
 constexpr int kEpiStageBytes = 4 * 2 * 4096;  // 4 epilogue warps x 2 buffers x (32 x 32 f32)
@@ -90,18 +89,22 @@ constexpr int kErrMmaFull = 0x112;
 constexpr int kErrEpiTmemFull = 0x121;
 constexpr int kErrDrain = 0x131;
 
-template <int kKind, bool kBMn, int BN, bool kCluster>
+template <int kKind, bool kBMn, int BN, bool kCluster, int BM>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
+    static_assert(BM == 128 || (BM == 64 && !kCluster), "BM 64 tiles run persistent only");
+    // Rows of the accumulator per epilogue warp.  An M = 128 MMA puts row r in TMEM lane
+    // r; an M = 64 MMA puts rows 16q .. 16q+15 in lanes 32q .. 32q+15 of sub-partition q.
+    constexpr int kRowsPerWarp = BM / 4;
     constexpr int kElem = kKind == 0 ? 2 : 4;
     constexpr int BK = 128 / kElem;                     // K elements per stage (one swizzle row)
     constexpr int kUmmaK = 32 / kElem;                  // K per MMA instruction (32 bytes)
     constexpr int kKSteps = BK / kUmmaK;                // 4
     constexpr int kAtom = 128 / kElem;                  // MN-major swizzle atom width (elements)
-    constexpr uint32_t kABytes = kBM * 128;             // 16 KB
+    constexpr uint32_t kABytes = BM * 128;              // 16 KB (BM 128) or 8 KB
     constexpr uint32_t kBBytes = BN * 128;
     constexpr uint32_t kStageBytes = kABytes + kBBytes;
     constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
-    constexpr uint32_t kIdesc = ptx::instr_desc(kKind == 0 ? 1u : 2u, kBMn, kBM, BN);
+    constexpr uint32_t kIdesc = ptx::instr_desc(kKind == 0 ? 1u : 2u, kBMn, BM, BN);
     // MN-major 32-bit (tf32) operands use the 32-byte-atom variant of the 128-byte swizzle
     // (the TMA load writes the matching CU_TENSOR_MAP_SWIZZLE_128B_ATOM_32B pattern).
     constexpr uint32_t kBLayout = (kKind == 1 && kBMn) ? ptx::kLayoutSw128Atom32 : ptx::kLayoutSw128;
@@ -154,7 +157,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
             const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
             for (int kb = kb0; kb < kb1 && kb < kb0 + S; ++kb) {
-                ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm * kBM, tc.b);
+                ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm * BM, tc.b);
                 if constexpr (!kBMn) {
                     ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN, tc.b);
                 } else {
@@ -196,7 +199,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     const uint32_t sa = smem_base + stage * kStageBytes;
                     const uint32_t sb = sa + kABytes;
                     ptx::mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
-                    ptx::tma_load_3d(sa, &p.tmap_a, kb * BK, tc.tm * kBM, tc.b, full_bar(stage));
+                    ptx::tma_load_3d(sa, &p.tmap_a, kb * BK, tc.tm * BM, tc.b, full_bar(stage));
                     if constexpr (!kBMn) {
                         ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, full_bar(stage));
                     } else {
@@ -285,7 +288,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         // swizzled shared-memory buffer and a TMA store (coalesced, bounds-clipped), or,
         // when the output's strides do not allow TMA, straight to global memory.
         const int q = warp & 3;
-        const int row_in_tile = q * 32 + lane;
+        const int row_in_tile = q * kRowsPerWarp + lane;   // valid for lane < kRowsPerWarp
+        const bool row_lane = lane < kRowsPerWarp;
         uint8_t* stage_buf = epi_smem + (warp - 2) * 8192;
         uint32_t chunk_ctr = 0;
         uint32_t iter = 0;
@@ -301,7 +305,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 // its main loop (see the reduction after the role branches).
                 continue;
             }
-            const int row = tc.tm * kBM + row_in_tile;
+            const int row = tc.tm * BM + row_in_tile;
             const float* bias = p.split == 1 ? p.bias : nullptr;
             float* dst_row = p.split == 1
                                  ? p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc
@@ -331,18 +335,20 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
                     if (lane == 0) ptx::bulk_wait_read<1>();  // the store that used buf is done
                     __syncwarp();
+                    if (row_lane) {
 #pragma unroll
-                    for (int j = 0; j < 8; ++j)
-                        *reinterpret_cast<float4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
-                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                        for (int j = 0; j < 8; ++j)
+                            *reinterpret_cast<float4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
+                                make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                    }
                     ptx::fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        ptx::tma_store_3d(&p.tmap_c, ptx::smem_u32(buf), col0, tc.tm * kBM + q * 32, zc);
+                        ptx::tma_store_3d(&p.tmap_c, ptx::smem_u32(buf), col0, tc.tm * BM + q * kRowsPerWarp, zc);
                         ptx::bulk_commit();
                     }
                     ++chunk_ctr;
-                } else if (row < p.M) {
+                } else if (row_lane && row < p.M) {
                     float* dst = dst_row + col0;
                     if (col0 + 32 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
 #pragma unroll
@@ -370,7 +376,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         // (3) A second barrier publishes them.  (4) Each owner adds its rows over the
         // slices in slice order (deterministic), adds bias, and stores them.  No CTA
         // touches another's shared memory after the second barrier.
-        const int R = kBM / p.split;
+        const int R = BM / p.split;
         const uint32_t my_rank = ptx::cluster_ctarank();
         ptx::tc_fence_before();
         ptx::cluster_sync();
@@ -402,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         for (int e = threadIdx.x; e < R * kVec; e += kThreads) {
             const int lr = e / kVec;
             const int cv = e % kVec;
-            const int row = tc.tm * kBM + row0 + lr;
+            const int row = tc.tm * BM + row0 + lr;
             const int col = tc.tn * BN + cv * 4;
             if (row >= p.M || col >= p.N) continue;
             float4 a = *reinterpret_cast<const float4*>(recv + (size_t)lr * (BN + 4) + cv * 4);
@@ -432,19 +438,23 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 
 using TcKernel = void (*)(TcParams);
 
-// Instance table, indexed as tc_instance(): cluster * 12 + (dtype_i * 2 + kn) * 3 + bn_i.
-#define NNJIT_TC_ROW(K, MN, CL) \
-    tc_gemm_kernel<K, MN, 64, CL>, tc_gemm_kernel<K, MN, 128, CL>, tc_gemm_kernel<K, MN, 256, CL>
-const TcKernel kTcKernels[24] = {
-    NNJIT_TC_ROW(0, false, false), NNJIT_TC_ROW(0, true, false),
-    NNJIT_TC_ROW(1, false, false), NNJIT_TC_ROW(1, true, false),
-    NNJIT_TC_ROW(0, false, true),  NNJIT_TC_ROW(0, true, true),
-    NNJIT_TC_ROW(1, false, true),  NNJIT_TC_ROW(1, true, true),
+// Instance table, indexed as tc_instance(): variant * 12 + (dtype_i * 2 + kn) * 3 + bn_i,
+// variant 0 = 128-row persistent, 1 = 128-row cluster split-K, 2 = 64-row persistent.
+constexpr int kNumTcInstances = 36;
+#define NNJIT_TC_ROW(K, MN, CL, BM) \
+    tc_gemm_kernel<K, MN, 64, CL, BM>, tc_gemm_kernel<K, MN, 128, CL, BM>, tc_gemm_kernel<K, MN, 256, CL, BM>
+const TcKernel kTcKernels[kNumTcInstances] = {
+    NNJIT_TC_ROW(0, false, false, 128), NNJIT_TC_ROW(0, true, false, 128),
+    NNJIT_TC_ROW(1, false, false, 128), NNJIT_TC_ROW(1, true, false, 128),
+    NNJIT_TC_ROW(0, false, true, 128),  NNJIT_TC_ROW(0, true, true, 128),
+    NNJIT_TC_ROW(1, false, true, 128),  NNJIT_TC_ROW(1, true, true, 128),
+    NNJIT_TC_ROW(0, false, false, 64),  NNJIT_TC_ROW(0, true, false, 64),
+    NNJIT_TC_ROW(1, false, false, 64),  NNJIT_TC_ROW(1, true, false, 64),
 };
 #undef NNJIT_TC_ROW
 
 std::mutex g_prep_mu;
-int g_prepared_smem[24] = {0};
+int g_prepared_smem[kNumTcInstances] = {0};
 
 // Driver entry point for cuTensorMapEncodeTiled, fetched through the runtime so the
 // library does not link against libcuda.
@@ -470,7 +480,7 @@ EncodeTiledFn get_encode_fn() {
 }  // namespace
 
 cudaError_t prepare_tc_instance(int instance, int smem_bytes) {
-    if (instance < 0 || instance >= 24) return cudaErrorInvalidValue;
+    if (instance < 0 || instance >= kNumTcInstances) return cudaErrorInvalidValue;
     std::lock_guard<std::mutex> lk(g_prep_mu);
     if (g_prepared_smem[instance] >= smem_bytes) return cudaSuccess;
     cudaError_t e = cudaFuncSetAttribute(kTcKernels[instance],
@@ -495,7 +505,7 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
     {
         const cuuint64_t dims[3] = {(cuuint64_t)p.K, (cuuint64_t)p.M, (cuuint64_t)p.batch};
         const cuuint64_t strides[2] = {(cuuint64_t)(p.lda * e), (cuuint64_t)(p.stride_a * e)};
-        const cuuint32_t box[3] = {bk, (cuuint32_t)kBM, 1};
+        const cuuint32_t box[3] = {bk, (cuuint32_t)c.bm, 1};
         CUresult r = enc(ta, dt, 3, const_cast<void*>(A), dims, strides, box, estr,
                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -542,7 +552,7 @@ cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, flo
     if ((reinterpret_cast<uintptr_t>(out) & 15) || (ld * 4) % 16 || (zs * 4) % 16) return cudaSuccess;
     const cuuint64_t dims[3] = {(cuuint64_t)p.N, (cuuint64_t)p.M, (cuuint64_t)nz};
     const cuuint64_t strides[2] = {(cuuint64_t)(ld * 4), (cuuint64_t)(zs * 4)};
-    const cuuint32_t box[3] = {32, 32, 1};
+    const cuuint32_t box[3] = {32, (cuuint32_t)(c.bm / 4), 1};  // one epilogue warp's rows
     const cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = enc(tc_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, out, dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -554,8 +564,10 @@ cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, flo
 cudaError_t launch_tc(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
-    if (c.instance < 0 || c.instance >= 24 || !a.tmap_a || !a.tmap_b) return cudaErrorInvalidValue;
-    const bool cluster = c.instance >= 12;
+    if (c.instance < 0 || c.instance >= kNumTcInstances || !a.tmap_a || !a.tmap_b)
+        return cudaErrorInvalidValue;
+    const bool cluster = c.instance >= 12 && c.instance < 24;
+    if ((c.instance >= 24) != (c.bm == 64) || (c.bm != 64 && c.bm != 128)) return cudaErrorInvalidValue;
     if (cluster != (c.reduce == 1)) return cudaErrorInvalidValue;
     if (cluster && (c.split_k < 2 || c.split_k > 8 || (c.split_k & (c.split_k - 1)) != 0))
         return cudaErrorInvalidValue;
@@ -577,7 +589,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     prm.stride_c = p.stride_c;
     prm.num_kb = (int)((p.K + c.bk - 1) / c.bk);
     prm.split = c.split_k;
-    prm.tiles_m = (int)((p.M + kBM - 1) / kBM);
+    prm.tiles_m = (int)((p.M + c.bm - 1) / c.bm);
     prm.tiles_n = (int)((p.N + c.bn - 1) / c.bn);
     const long long total = (long long)p.batch * c.split_k * prm.tiles_m * prm.tiles_n;
     if (total >= (1LL << 31)) return cudaErrorInvalidValue;
@@ -588,7 +600,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     // persistent: at most the candidate's grid; cluster mode: one CTA per (tile, slice)
     const int grid = cluster ? (int)total : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
     // ring + alignment slack + barriers/TMEM slot/abort flag
-    const int stage_bytes = (kBM + c.bn) * 128;
+    const int stage_bytes = (c.bm + c.bn) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     cudaError_t e = prepare_tc_instance(c.instance, smem);
     if (e != cudaSuccess) return e;

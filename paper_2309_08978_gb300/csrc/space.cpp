@@ -37,8 +37,10 @@ nnjit_candidate blank() {
 }
 
 // ---------------------------------------------------------------------------------
-// tcgen05 tensor-core family.  The CTA tile is BM x BN with BM = 128 (one cta_group::1
-// UMMA covers 128 TMEM lanes).  BK is fixed at one 128-byte swizzle row of K (64 bf16,
+// tcgen05 tensor-core family.  The CTA tile is BM x BN with BM = 128, or BM = 64 when the
+// 128-row tiles leave SMs idle (an M = 64 MMA costs about half as long, so 64-row tiles
+// double the CTAs without split-K partial traffic).  BK is fixed at one 128-byte swizzle
+// row of K (64 bf16,
 // 32 tf32): the Blackwell counterpart of the paper's "consistent" primitive settings
 // (Sec. 5.1), fixed once instead of searched.  The searched axes are BN, split-K and
 // the tile raster order; the stage count is derived, not searched: the ring fills the
@@ -49,15 +51,17 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
               int64_t* naive) {
     using MC = ModelConstants;
     const int e = p.elem_bytes();
-    const int BM = MC::kTcBM, BK = 128 / e;
+    const int BK = 128 / e;
     const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
     const int64_t K = std::max<int64_t>(p.K, 1);
     const int64_t num_kb = ceil_div(K, BK);
     const int bns[3] = {64, 128, 256};
     const int splits[4] = {1, 2, 4, 8};
-    *naive = 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2;  // BN x stages 2..8 x split x raster x reduce
+    *naive = 2 * 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2;  // BM x BN x stages x split x raster x reduce
+    for (int BM : {MC::kTcBM, 64})
     for (int bn : bns) {
         if (bn > 64 && bn > pow2_ceil(N)) continue;  // no tile wider than the padded N
+        if (BM == 64 && p.batch * ceil_div(M, MC::kTcBM) * ceil_div(N, bn) >= L.sm_count) continue;
         const int stage_bytes = (BM + bn) * 128;
         const int stages = std::min(MC::kTcMaxStages,
                                     (L.smem_per_block_optin - MC::kTcFixedSmem) / stage_bytes);
@@ -79,7 +83,8 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
             for (int reduce = 0; reduce < (split > 1 ? 2 : 1); ++reduce)
             for (int raster = 0; raster < 2; ++raster) {
                 if (raster == 1 && (tiles_m == 1 || tiles_n == 1)) continue;
-                if (reduce == 1 && (raster == 1 || stages * stage_bytes < 128 * (bn + 4) * 4)) continue;
+                if (reduce == 1 && (BM != MC::kTcBM || raster == 1 || stages * stage_bytes < 128 * (bn + 4) * 4))
+                    continue;
                 nnjit_candidate c = blank();
                 c.family = NNJIT_FAMILY_TC;
                 c.bm = BM; c.bn = bn; c.bk = BK;
@@ -104,8 +109,8 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 // tensor core works on all 256 columns at once), so the MMA clocks are
                 // those of BN = 256, against the operand feed (stage bytes over the per-SM
                 // L2 feed)
-                const int64_t t_kb = std::max<int64_t>(2 * 256, ceil_div(stage_bytes,
-                                                                         MC::kFeedBytesPerClk));
+                const int64_t t_kb = std::max<int64_t>(2 * 256 * BM / MC::kTcBM,
+                                                       ceil_div(stage_bytes, MC::kFeedBytesPerClk));
                 int64_t cost = waves * t_kb * ceil_div(num_kb, split);
                 if (split > 1 && reduce == 0)
                     cost += MC::kLaunchClk +
@@ -113,7 +118,7 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 if (split > 1 && reduce == 1)
                     cost += waves * (128LL * bn * 4 / MC::kFeedBytesPerClk);  // DSMEM reduction
                 c.predicted_cost = cost;
-                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce);
+                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM);
                 v.push_back(c);
             }
         }
@@ -295,11 +300,12 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 
 }  // namespace
 
-int tc_instance(int dtype, int b_layout, int bn, int cluster) {
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm) {
     const int bi = bn == 64 ? 0 : bn == 128 ? 1 : bn == 256 ? 2 : -1;
-    if (bi < 0) return -1;
+    if (bi < 0 || (bm != 64 && bm != 128) || (bm == 64 && cluster)) return -1;
     const int di = dtype == NNJIT_BF16 ? 0 : 1;
-    return (cluster ? 12 : 0) + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
+    const int variant = bm == 64 ? 2 : cluster ? 1 : 0;
+    return variant * 12 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
 }
 
 // The 12 (thread tile, block tile) pairs with 64..256 threads, in enumeration order.
