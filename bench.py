@@ -294,8 +294,9 @@ def run_ours(args, workload, rank, world, local_rank):
     tune = {"budget_ms_per_shape": args.budget_ms, "shapes": []}
     for s in workload.shapes:
         A, B, bias = make_operands(s, workload.index, dtype)
+        bflag = nj.NNJIT_PLAN_B_CONSTANT if s.b_is_weight else 0   # weights never change
         desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
-                            has_bias=s.has_bias)
+                            has_bias=s.has_bias, flags=bflag)
         t0 = time.perf_counter()
         plan = nj.nnjit_matmul_plan_ex(desc, args.budget_ms)
         plan_ms = 1000 * (time.perf_counter() - t0)
@@ -307,7 +308,7 @@ def run_ours(args, workload, rank, world, local_rank):
         if not args.no_sweep:
             sweep_desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
                                       has_bias=s.has_bias,
-                                      flags=nj.NNJIT_PLAN_EXHAUSTIVE | nj.NNJIT_PLAN_NO_CACHE)
+                                      flags=nj.NNJIT_PLAN_EXHAUSTIVE | nj.NNJIT_PLAN_NO_CACHE | bflag)
             t0 = time.perf_counter()
             sweep = nj.nnjit_matmul_plan_ex(sweep_desc, 0.0)
             sweep_ms = 1000 * (time.perf_counter() - t0)

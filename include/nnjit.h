@@ -79,6 +79,11 @@ typedef enum {
 #define NNJIT_PLAN_EXHAUSTIVE    0x2u  /* time every candidate, ignoring the budget */
 #define NNJIT_PLAN_REQUIRE_TIMED 0x4u  /* fail with NNJIT_ERR_BUDGET instead of taking the
                                           top-ranked candidate untimed */
+#define NNJIT_PLAN_B_CONSTANT    0x8u  /* promise: B (e.g. Linear weights) is never written by
+                                          a kernel launched earlier in the same stream, so the
+                                          kernels may start reading B while that kernel still
+                                          runs (programmatic dependent launch); A and bias are
+                                          read only after it has completed */
 
 /*
  * Full problem description.  Zero leading dimensions / strides mean "packed":

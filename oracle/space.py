@@ -314,7 +314,9 @@ def _gemv(p, lim):
                         blk = block_core(lim, regs, threads, smem, 0)
                         if blk < 1:
                             continue
-                        grid = ctas_n * split
+                        # at most as many CTAs as fit at once; beyond that warps take
+                        # row groups round-robin
+                        grid = min(ctas_n, lim["sm_count"] * blk) * split
                         slots = lim["sm_count"] * blk
                         waves = cdiv(grid, slots)
                         inflight = min(cdiv(grid, lim["sm_count"]), blk) * threads * unroll * rows * 16

@@ -10,6 +10,7 @@
 #include <cuda_runtime.h>
 
 #include <cstdint>
+#include <algorithm>
 #include <mutex>
 
 #include "launch.h"
@@ -29,6 +30,7 @@ struct GemvParams {
     float* ws;           // [split][M][N]
     int M, N, K, split, kper;
     int vec_ok;          // KN: rows of W are 16-byte aligned (ldb % 8 == 0)
+    int b_const;         // W is not written by kernels launched before this one
     long long lda, ldb, ldc;
 };
 
@@ -49,18 +51,55 @@ __device__ __forceinline__ float dot8(const uint4& w, const uint4& x, float acc)
 
 __device__ __forceinline__ float bf16_to_f(uint16_t h) { return __uint_as_float((uint32_t)h << 16); }
 
-// grid: (ceil(N / (warps * R)), split); dynamic smem: M * kper bf16 (x slice).
+// grid: (CTAs, split) with CTAs <= ceil(N / (warps * R)); dynamic smem: M * kper bf16.
+// Each warp streams R weight rows in batches of U 16-byte loads per lane and row; the
+// other warps of the SM hide each batch's latency.
 template <int R, int U>
 __global__ void __launch_bounds__(256) gemv_nk_kernel(const GemvParams p) {
     extern __shared__ __align__(16) uint16_t xs[];
-    ptx::griddep_wait();
-    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const int warps = blockDim.x >> 5;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int s = blockIdx.y;
     const int k0 = s * p.kper;
     const int klen = max(0, min(p.K, k0 + p.kper) - k0);
     const int M = p.M;
+    const int nvec = klen >> 3;  // full 16-byte chunks in this slice
+    // Row groups of R weight rows are dealt to warps round-robin over the whole grid.
+    const int groups = (p.N + R - 1) / R;
+    const int g_first = blockIdx.x * warps + warp;
+
+    auto row_ptrs = [&](int g, const uint16_t* (&wrow)[R]) {
+#pragma unroll
+        for (int r = 0; r < R; ++r) {
+            const int n = min(g * R + r, p.N - 1);  // rows past N repeat the last row, unused
+            wrow[r] = p.W + (long long)n * p.ldb + k0;
+        }
+    };
+    auto load_batch = [&](const uint16_t* const (&wrow)[R], int c0, uint4 (&w)[U][R]) {
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int c = c0 + u * 32 + lane;
+#pragma unroll
+            for (int r = 0; r < R; ++r)
+                w[u][r] = c < nvec ? ptx::ld_stream_v4(wrow[r] + c * 8) : make_uint4(0, 0, 0, 0);
+        }
+    };
+
+    // With constant weights the first batch is requested before the dependency wait, so
+    // the weight stream overlaps the previous kernel's tail; x is read only after it.
+    uint4 w[U][R];
+    const uint16_t* wrow[R];
+    bool have_first = false;
+    if (g_first < groups) {
+        row_ptrs(g_first, wrow);
+        if (p.b_const && nvec > 0) {
+            load_batch(wrow, 0, w);
+            have_first = true;
+        }
+    }
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
+
     // x slice -> shared memory (16-byte copies when the slice allows, else scalar)
     const int kl8 = klen & ~7;
     for (int m = 0; m < M; ++m) {
@@ -72,79 +111,66 @@ __global__ void __launch_bounds__(256) gemv_nk_kernel(const GemvParams p) {
     }
     __syncthreads();
 
-    const int n_base = (blockIdx.x * warps + warp) * R;
-    if (n_base >= p.N) return;
-    float acc[R][kMaxM];
+    for (int g = g_first; g < groups; g += gridDim.x * warps) {
+        const int n_base = g * R;
+        if (g != g_first) row_ptrs(g, wrow);
+        float acc[R][kMaxM];
 #pragma unroll
-    for (int r = 0; r < R; ++r)
+        for (int r = 0; r < R; ++r)
 #pragma unroll
-        for (int m = 0; m < kMaxM; ++m) acc[r][m] = 0.0f;
-
-    const uint16_t* wrow[R];
+            for (int m = 0; m < kMaxM; ++m) acc[r][m] = 0.0f;
+        for (int c0 = 0; c0 < nvec; c0 += 32 * U) {
+            if (!(c0 == 0 && g == g_first && have_first)) load_batch(wrow, c0, w);
 #pragma unroll
-    for (int r = 0; r < R; ++r) {
-        const int n = min(n_base + r, p.N - 1);  // rows past N repeat the last row, unused
-        wrow[r] = p.W + (long long)n * p.ldb + k0;
-    }
-    const int nvec = klen >> 3;  // full 16-byte chunks in this slice
-    for (int c0 = 0; c0 < nvec; c0 += 32 * U) {
-        uint4 w[U][R];
+            for (int u = 0; u < U; ++u) {
+                const int c = c0 + u * 32 + lane;
+                if (c < nvec) {
 #pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int c = c0 + u * 32 + lane;
+                    for (int m = 0; m < kMaxM; ++m) {
+                        if (m < M) {
+                            const uint4 xv = *reinterpret_cast<const uint4*>(xs + (long long)m * p.kper + c * 8);
 #pragma unroll
-            for (int r = 0; r < R; ++r)
-                w[u][r] = c < nvec ? ptx::ld_stream_v4(wrow[r] + c * 8) : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int u = 0; u < U; ++u) {
-            const int c = c0 + u * 32 + lane;
-            if (c < nvec) {
-#pragma unroll
-                for (int m = 0; m < kMaxM; ++m) {
-                    if (m < M) {
-                        const uint4 xv = *reinterpret_cast<const uint4*>(xs + (long long)m * p.kper + c * 8);
-#pragma unroll
-                        for (int r = 0; r < R; ++r) acc[r][m] = dot8(w[u][r], xv, acc[r][m]);
+                            for (int r = 0; r < R; ++r) acc[r][m] = dot8(w[u][r], xv, acc[r][m]);
+                        }
                     }
                 }
             }
         }
-    }
-    // ragged K tail (fewer than 8 elements)
-    for (int k = (nvec << 3) + lane; k < klen; k += 32) {
+        // ragged K tail (fewer than 8 elements)
+        for (int k = (nvec << 3) + lane; k < klen; k += 32) {
 #pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const float wv = bf16_to_f(wrow[r][k]);
+            for (int r = 0; r < R; ++r) {
+                const float wv = bf16_to_f(wrow[r][k]);
 #pragma unroll
-            for (int m = 0; m < kMaxM; ++m)
-                if (m < M) acc[r][m] = fmaf(wv, bf16_to_f(xs[(long long)m * p.kper + k]), acc[r][m]);
-        }
-    }
-    // butterfly reduction over the warp
-#pragma unroll
-    for (int r = 0; r < R; ++r)
-#pragma unroll
-        for (int m = 0; m < kMaxM; ++m) {
-            if (m < M) {
-                float v = acc[r][m];
-#pragma unroll
-                for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                acc[r][m] = v;
+                for (int m = 0; m < kMaxM; ++m)
+                    if (m < M) acc[r][m] = fmaf(wv, bf16_to_f(xs[(long long)m * p.kper + k]), acc[r][m]);
             }
         }
-    if (lane == 0) {
+        // butterfly reduction over the warp
 #pragma unroll
-        for (int r = 0; r < R; ++r) {
-            const int n = n_base + r;
-            if (n >= p.N) continue;
+        for (int r = 0; r < R; ++r)
 #pragma unroll
             for (int m = 0; m < kMaxM; ++m) {
-                if (m >= M) continue;
-                if (p.split == 1)
-                    p.C[(long long)m * p.ldc + n] = p.bias ? acc[r][m] + p.bias[n] : acc[r][m];
-                else
-                    p.ws[((long long)s * M + m) * p.N + n] = acc[r][m];
+                if (m < M) {
+                    float v = acc[r][m];
+#pragma unroll
+                    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+                    acc[r][m] = v;
+                }
+            }
+        if (lane == 0) {
+#pragma unroll
+            for (int r = 0; r < R; ++r) {
+                const int n = n_base + r;
+                if (n >= p.N) continue;
+#pragma unroll
+                for (int m = 0; m < kMaxM; ++m) {
+                    if (m >= M) continue;
+                    if (p.split == 1)
+                        p.C[(long long)m * p.ldc + n] = p.bias ? acc[r][m] + p.bias[n] : acc[r][m];
+                    else
+                        p.ws[((long long)s * M + m) * p.N + n] = acc[r][m];
+                }
             }
         }
     }
@@ -322,14 +348,14 @@ cudaError_t launch_gemv(const LaunchArgs& a) {
     prm.split = c.split_k;
     prm.lda = p.lda; prm.ldb = p.ldb; prm.ldc = p.ldc;
     prm.vec_ok = (p.ldb % 8 == 0 && (reinterpret_cast<uintptr_t>(a.B) & 15) == 0) ? 1 : 0;
+    prm.b_const = (p.flags & NNJIT_PLAN_B_CONSTANT) ? 1 : 0;
     const int warps = c.threads / 32;
     dim3 grid;
     int smem;
     if (!kn_inst) {
         // K slice: a multiple of 8 elements so every slice starts 16-byte aligned
         prm.kper = (int)((((p.K + c.split_k - 1) / c.split_k) + 7) / 8 * 8);
-        grid = dim3((unsigned)((p.N + (long long)warps * c.tm - 1) / ((long long)warps * c.tm)),
-                    (unsigned)c.split_k);
+        grid = dim3((unsigned)std::max(1, c.grid / c.split_k), (unsigned)c.split_k);
         smem = (int)((p.M * (long long)prm.kper * 2 + 15) / 16 * 16);
     } else {
         prm.kper = (int)((p.K + c.split_k - 1) / c.split_k);

@@ -40,6 +40,7 @@ struct TcParams {
     CUtensorMap tmap_b;  // NK: dims {K, N, batch}, box {BK, BN, 1}; KN: dims {N, K, batch}, box {atom, BK, 1}
     CUtensorMap tmap_c;  // output (C, or the split-K partials): dims {N, M, z}, box {32, 32, 1}
     int tma_store;       // 1: epilogue stores through tmap_c; 0: direct global stores
+    int b_const;         // B is not written by kernels launched earlier in the stream
     float* C;
     const float* bias;
     float* ws;
@@ -175,7 +176,33 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    // Everything above overlaps the previous kernel's tail; global memory only from here.
+    // With a constant B the producer arms the first ring and starts its B tiles before
+    // the dependency wait (the ring is empty, so no "empty" wait is needed); the loop
+    // below then only adds the A tiles of those stages.
+    int b_preloaded = 0;
+    if (p.b_const && warp == 0 && blockIdx.x < p.total_tiles) {
+        const TileCoord tc = decode_tile<kCluster>(blockIdx.x, p);
+        const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
+        const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
+        b_preloaded = min(S, kb1 - kb0);
+        if (lane == 0) {
+            for (int i = 0; i < b_preloaded; ++i) {
+                const int kb = kb0 + i;
+                const uint32_t sb = smem_base + i * kStageBytes + kABytes;
+                ptx::mbar_arrive_expect_tx(full_bar(i), kStageBytes);
+                if constexpr (!kBMn) {
+                    ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, full_bar(i));
+                } else {
+#pragma unroll
+                    for (int j = 0; j < BN / kAtom; ++j)
+                        ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK,
+                                         tc.b, full_bar(i));
+                }
+            }
+        }
+        __syncwarp();
+    }
+    // Global memory that earlier kernels may write is touched only from here.
     ptx::griddep_wait();
     if (threadIdx.x == 0) ptx::griddep_launch_dependents();
 
@@ -185,6 +212,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t phase = 0;
         uint32_t armed = 0, armed_parity = 0;
         bool ok = true;
+        int issued = 0;  // k-blocks issued so far by this CTA
         for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
             const TileCoord tc = decode_tile<kCluster>(t, p);
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
@@ -195,7 +223,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     ok = false;
                     break;
                 }
-                if (lane == 0) {
+                const bool pre = issued < b_preloaded;  // B of this stage already on its way
+                ++issued;
+                if (lane == 0 && pre) {
+                    ptx::tma_load_3d(smem_base + stage * kStageBytes, &p.tmap_a, kb * BK, tc.tm * BM, tc.b,
+                                     full_bar(stage));
+                } else if (lane == 0) {
                     const uint32_t sa = smem_base + stage * kStageBytes;
                     const uint32_t sb = sa + kABytes;
                     ptx::mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
@@ -576,6 +609,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     prm.tmap_a = *a.tmap_a;
     prm.tmap_b = *a.tmap_b;
     prm.tma_store = a.tmap_c ? 1 : 0;
+    prm.b_const = (p.flags & NNJIT_PLAN_B_CONSTANT) ? 1 : 0;
     if (a.tmap_c) prm.tmap_c = *a.tmap_c;
     prm.C = a.C;
     prm.bias = a.bias;

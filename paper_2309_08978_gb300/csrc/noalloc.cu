@@ -112,6 +112,7 @@ extern "C" nnjit_status nnjit_gemv_bf16_noalloc(int64_t M, int64_t N, int64_t K,
     c.split_k = split_k;
     c.threads = 256;
     c.bn = 8 * 2;
+    c.grid = (int32_t)(((N + c.bn - 1) / c.bn) * split_k);  // one CTA per 16-row block
     c.instance = gemv_instance(NNJIT_B_NK, 2, 4);
 
     LaunchArgs la;

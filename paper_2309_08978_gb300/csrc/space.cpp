@@ -233,7 +233,11 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
                         c.smem_bytes = (int)smem;
                         c.regs_per_thread = regs;
                         c.blocks_per_sm = blk;
-                        const int64_t grid = ctas_n * split;
+                        // at most as many CTAs as fit at once (bytes in flight are
+                        // what a streaming kernel needs); beyond that the warps take
+                        // row groups round-robin
+                        const int64_t per_split = std::min<int64_t>(ctas_n, (int64_t)L.sm_count * blk);
+                        const int64_t grid = per_split * split;
                         const int64_t slots = (int64_t)L.sm_count * blk;
                         const int64_t waves = ceil_div(grid, slots);
                         c.grid = (int32_t)grid;

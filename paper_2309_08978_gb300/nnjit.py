@@ -36,6 +36,7 @@ NNJIT_FAMILY_GEMV = 2
 NNJIT_PLAN_NO_CACHE = 0x1
 NNJIT_PLAN_EXHAUSTIVE = 0x2
 NNJIT_PLAN_REQUIRE_TIMED = 0x4
+NNJIT_PLAN_B_CONSTANT = 0x8
 
 DTYPES = {"f32_ffma": NNJIT_F32_FFMA, "tf32": NNJIT_TF32, "bf16": NNJIT_BF16}
 LAYOUTS = {"KN": NNJIT_B_KN, "NK": NNJIT_B_NK}

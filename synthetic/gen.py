@@ -119,6 +119,7 @@ class Shape:
     b_dist: tuple = ("normal", 0.02)
     bias_dist: tuple = ("normal", 0.02)
     ids: tuple = (0, 1, 2)        # tensor ids of A, B, bias
+    b_is_weight: bool = True      # B is a model weight (constant across calls)
 
     @property
     def flops(self) -> int:
@@ -163,9 +164,9 @@ WORKLOADS = {
         _linears(2048, [(1024, 1024), (4096, 1024), (1024, 4096), (4096, 4096)],
                  ["q_k_v_o", "wi", "wo", "n4096_k4096"]) + (
             Shape("qk_t", 256, 256, 64, 128, "NK", False, ("normal", 1.0), ("normal", 1.0),
-                  ("normal", 0.0), (12, 13, 2)),
+                  ("normal", 0.0), (12, 13, 2), False),
             Shape("pv", 256, 64, 256, 128, "KN", False, ("normal", 1.0), ("normal", 1.0),
-                  ("normal", 0.0), (14, 15, 2)))),
+                  ("normal", 0.0), (14, 15, 2), False))),
     "llama2_7b_decode_m1": Workload(
         "llama2_7b_decode_m1", 3,
         "Llama-2-7B decoder block decode GEMVs, batch 1 (M=1), BF16",
@@ -179,9 +180,9 @@ WORKLOADS = {
         _linears(4096, [(12288, 4096), (4096, 4096), (22016, 4096), (4096, 11008)],
                  ["qkv", "o_proj", "gate_up", "down"]) + (
             Shape("qk_t", 1024, 1024, 128, 128, "NK", False, ("normal", 1.0), ("normal", 1.0),
-                  ("normal", 0.0), (12, 13, 2)),
+                  ("normal", 0.0), (12, 13, 2), False),
             Shape("pv", 1024, 128, 1024, 128, "KN", False, ("normal", 1.0), ("normal", 1.0),
-                  ("normal", 0.0), (14, 15, 2)))),
+                  ("normal", 0.0), (14, 15, 2), False))),
 }
 
 

@@ -154,3 +154,55 @@ def test_tc_strided_c(ldc):
     Cn = Cbuf.cpu().numpy()
     compare(np.ascontiguousarray(Cn[:, :N]), A, B, bias, "NK", "bf16", exact=True)
     assert np.all(Cn[:, N:] == -7.0)
+
+
+CONST_B_CASES = [("bf16", 300, 520, 1040, "NK"), ("tf32", 130, 96, 100, "KN"),
+                 ("bf16", 1, 4096, 4096, "NK"), ("bf16", 3, 300, 520, "NK"),
+                 ("bf16", 512, 768, 3072, "NK")]
+
+
+@pytest.mark.parametrize("case", CONST_B_CASES, ids=_ids)
+def test_constant_b_flag_is_exact(case):
+    """NNJIT_PLAN_B_CONSTANT lets the kernels start reading B before the dependency
+    wait; results must not change."""
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    A, B, bias = make_operands(shape, 13, dtype, ints=True)
+    desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True,
+                        flags=nj.NNJIT_PLAN_B_CONSTANT | nj.NNJIT_PLAN_NO_CACHE)
+    lim = nj.nnjit_device_limits_query(0)
+    cands, _ = nj.nnjit_space_enumerate(desc, lim)
+    for i in range(min(len(cands), 6)):
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            C = run_plan(plan, A, B, bias, M, N)
+        compare(C, A, B, bias, layout, dtype, exact=True)
+
+
+def test_chain_waits_for_the_producer_of_a():
+    """Two TF32 products on one stream, the second reading the first's output as A while
+    its (constant) B is fetched early: the second must still see the finished A.
+    Integer operands keep every value exact (C1 <= 64 is exact in TF32)."""
+    import torch
+    from synthetic import small_ints
+    M, K1, N1, N2 = 256, 16, 64, 128
+    A0 = (small_ints(40, M * K1, -2, 2).reshape(M, K1)).astype(np.float32)
+    B1 = (small_ints(41, N1 * K1, -2, 2).reshape(N1, K1)).astype(np.float32)
+    B2 = (small_ints(42, N2 * N1).reshape(N2, N1)).astype(np.float32)
+    flags = nj.NNJIT_PLAN_B_CONSTANT | nj.NNJIT_PLAN_NO_CACHE
+    p1 = nj.nnjit_matmul_plan_ex(nj.make_desc(M, N1, K1, "tf32", "NK", flags=flags), 0.0)
+    p2 = nj.nnjit_matmul_plan_ex(nj.make_desc(M, N2, N1, "tf32", "NK", flags=flags), 0.0)
+    dA0, dB1, dB2 = (torch.from_numpy(x).cuda() for x in (A0, B1, B2))
+    want1 = A0.astype(np.int64) @ B1.T.astype(np.int64)
+    want2 = want1 @ B2.T.astype(np.int64)
+    s = torch.cuda.Stream()
+    for rep in range(20):
+        C1 = torch.full((M, N1), float("nan"), device="cuda")
+        C2 = torch.full((M, N2), float("nan"), device="cuda")
+        torch.cuda.synchronize()
+        with torch.cuda.stream(s):
+            p1.run(dA0, dB1, None, C1, s)
+            p2.run(C1, dB2, None, C2, s)
+        s.synchronize()
+        assert np.array_equal(C2.cpu().numpy(), want2.astype(np.float32)), f"repetition {rep}"
+    p1.destroy()
+    p2.destroy()
