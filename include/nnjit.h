@@ -142,6 +142,8 @@ typedef struct {
     int32_t reduce;          /* split-K reduction: 0 = partials in the plan's workspace, summed
                                 by a second kernel; 1 = TC only, inside a thread-block cluster
                                 of split_k CTAs through distributed shared memory */
+    int32_t cluster_m;       /* TC only: 2 = the two CTAs of a cluster take vertically adjacent
+                                tiles and share each B tile by TMA multicast; else 1 */
 } nnjit_candidate;
 
 typedef struct nnjit_plan_s* nnjit_plan;

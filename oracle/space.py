@@ -41,7 +41,7 @@ GEMV_MAX_SMEM = 64 * 1024
 
 CANDIDATE_FIELDS = ("family", "bm", "bn", "bk", "tm", "tn", "stages", "split_k", "raster",
                     "threads", "smem_bytes", "tmem_cols", "regs_per_thread", "blocks_per_sm",
-                    "grid", "wave_eff_ppm", "instance", "predicted_cost", "reduce")
+                    "grid", "wave_eff_ppm", "instance", "predicted_cost", "reduce", "cluster_m")
 
 
 def cdiv(a: int, b: int) -> int:
@@ -170,10 +170,13 @@ def _blank():
     c = dict.fromkeys(CANDIDATE_FIELDS, 0)
     c["split_k"] = 1
     c["instance"] = -1
+    c["cluster_m"] = 1
     return c
 
 
-def tc_instance(dtype, b_layout, bn, cluster, bm):
+def tc_instance(dtype, b_layout, bn, cluster, bm, mcast=False):
+    if mcast:
+        return 36 + (0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)
     variant = 2 if bm == 64 else (1 if cluster else 0)
     return variant * 12 + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 3 + \
         {64: 0, 128: 1, 256: 2}[bn]
@@ -248,7 +251,18 @@ def _tc(p, lim):
                              instance=tc_instance(p.dtype, p.b_layout, bn, reduce, bm),
                              predicted_cost=cost, reduce=reduce)
                     out.append(c)
-    return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2
+                    # multicast pair: two CTAs of a cluster share each B tile
+                    if bm == TC_BM and bn == 256 and split == 1 and tiles >= lim["sm_count"]:
+                        m = dict(c)
+                        pairs = p.batch * cdiv(tiles_m, 2) * tiles_n
+                        live = min(pairs, max(1, slots // 2))
+                        pw = cdiv(pairs, live)
+                        feed = cdiv(stage - bn * 128 // 2, FEED_BYTES_PER_CLK)
+                        m.update(cluster_m=2, grid=2 * live, wave_eff_ppm=pairs * 1000000 // (pw * live),
+                                 predicted_cost=pw * max(2 * 256, feed) * num_kb,
+                                 instance=tc_instance(p.dtype, p.b_layout, bn, 0, bm, True))
+                        out.append(m)
+    return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2
 
 
 def _ffma(p, lim):

@@ -789,9 +789,9 @@ int32_t nnjit_cache_size(void) {
 }
 
 // File format: a header line, then one line per entry:
-//   key \t 19 candidate integers \t chosen_index space_size naive tune_ms timed \t
+//   key \t 20 candidate integers \t chosen_index space_size naive tune_ms timed \t
 //   n (index us)*n
-static const char* kCacheHeader = "nnjit-plan-cache v1";
+static const char* kCacheHeader = "nnjit-plan-cache v2";
 
 nnjit_status nnjit_cache_save(const char* path) {
     if (!path) return fail(NNJIT_ERR_INVALID_ARG, "path is NULL");
@@ -804,11 +804,11 @@ nnjit_status nnjit_cache_save(const char* path) {
         for (const auto& kv : cache()) {
             const CacheEntry& e = kv.second;
             const nnjit_candidate& c = e.cand;
-            std::fprintf(f, "%s\t%d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %lld %d\t%d %d %lld %.6f %d\t%zu",
+            std::fprintf(f, "%s\t%d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %lld %d %d\t%d %d %lld %.6f %d\t%zu",
                          kv.first.c_str(), c.family, c.bm, c.bn, c.bk, c.tm, c.tn, c.stages,
                          c.split_k, c.raster, c.threads, c.smem_bytes, c.tmem_cols,
                          c.regs_per_thread, c.blocks_per_sm, c.grid, c.wave_eff_ppm, c.instance,
-                         (long long)c.predicted_cost, c.reduce, e.chosen_index, e.space_size,
+                         (long long)c.predicted_cost, c.reduce, c.cluster_m, e.chosen_index, e.space_size,
                          (long long)e.naive, e.tune_ms, e.timed ? 1 : 0, e.timings.size());
             for (const auto& t : e.timings) std::fprintf(f, " %d %.6f", t.first, t.second);
             std::fprintf(f, "\n");
@@ -846,11 +846,12 @@ nnjit_status nnjit_cache_load(const char* path, int32_t* loaded) {
         size_t ntim = 0;
         int used = 0;
         const char* rest = line.c_str() + t1 + 1;
-        if (std::sscanf(rest, "%d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %lld %d %d %d %lld %lf %d %zu%n",
+        if (std::sscanf(rest, "%d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %d %lld %d %d %d %d %lld %lf %d %zu%n",
                         &c.family, &c.bm, &c.bn, &c.bk, &c.tm, &c.tn, &c.stages, &c.split_k,
                         &c.raster, &c.threads, &c.smem_bytes, &c.tmem_cols, &c.regs_per_thread,
                         &c.blocks_per_sm, &c.grid, &c.wave_eff_ppm, &c.instance, &cost, &c.reduce,
-                        &e.chosen_index, &e.space_size, &naive, &e.tune_ms, &timed, &ntim, &used) != 25 ||
+                        &c.cluster_m, &e.chosen_index, &e.space_size, &naive, &e.tune_ms, &timed,
+                        &ntim, &used) != 26 ||
             ntim > 4096)
             return fail(NNJIT_ERR_INVALID_ARG, "malformed cache line");
         c.predicted_cost = cost;

@@ -54,15 +54,22 @@ struct TileCoord {
     int b, s, tm, tn;
 };
 
-// Work item t -> (batch, K slice, tile row, tile column).  Persistent mode: slices of a
-// tile are separate work items.  Cluster mode: the split_k consecutive CTAs of a cluster
-// share one output tile and CTA rank = K slice.
-template <bool kCluster>
-__device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p) {
+// Kernel modes: persistent CTAs (slices of a tile are separate work items), cluster
+// split-K (the split_k consecutive CTAs of a cluster share one output tile, CTA rank =
+// K slice), and multicast pairs (a cluster of 2 CTAs takes the two vertically adjacent
+// tiles 2*mp and 2*mp + 1 of one tile column; work item = pair).
+constexpr int kModePersistent = 0;
+constexpr int kModeClusterSplitK = 1;
+constexpr int kModeMcastPair = 2;
+
+// Work item t -> (batch, K slice, tile row, tile column).
+template <int kMode>
+__device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p, int rank) {
     TileCoord c;
-    const int per = p.tiles_m * p.tiles_n;
+    const int rows = kMode == kModeMcastPair ? (p.tiles_m + 1) / 2 : p.tiles_m;
+    const int per = rows * p.tiles_n;
     int r, q;
-    if constexpr (kCluster) {
+    if constexpr (kMode == kModeClusterSplitK) {
         c.s = t % p.split;
         const int ot = t / p.split;
         r = ot % per;
@@ -74,12 +81,13 @@ __device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p) {
         c.b = q / p.split;
     }
     if (p.raster == 0) {
-        c.tm = r % p.tiles_m;
-        c.tn = r / p.tiles_m;
+        c.tm = r % rows;
+        c.tn = r / rows;
     } else {
         c.tn = r % p.tiles_n;
         c.tm = r / p.tiles_n;
     }
+    if constexpr (kMode == kModeMcastPair) c.tm = 2 * c.tm + rank;
     return c;
 }
 
@@ -90,9 +98,11 @@ constexpr int kErrMmaFull = 0x112;
 constexpr int kErrEpiTmemFull = 0x121;
 constexpr int kErrDrain = 0x131;
 
-template <int kKind, bool kBMn, int BN, bool kCluster, int BM>
+template <int kKind, bool kBMn, int BN, int kMode, int BM>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
-    static_assert(BM == 128 || (BM == 64 && !kCluster), "BM 64 tiles run persistent only");
+    constexpr bool kCluster = kMode == kModeClusterSplitK;
+    constexpr bool kMcast = kMode == kModeMcastPair;
+    static_assert(BM == 128 || (BM == 64 && kMode == kModePersistent), "BM 64 tiles run persistent only");
     // Rows of the accumulator per epilogue warp.  An M = 128 MMA puts row r in TMEM lane
     // r; an M = 64 MMA puts rows 16q .. 16q+15 in lanes 32q .. 32q+15 of sub-partition q.
     constexpr int kRowsPerWarp = BM / 4;
@@ -132,11 +142,41 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     auto tfull_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + a); };
     auto tempty_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + 2 + a); };
     const uint32_t drain_bar = ptx::smem_u32(bars + 2 * S + 4);
+    // Multicast pairs: this CTA's rank in its cluster; work items are pairs.
+    const int rank = kMcast ? (int)ptx::cluster_ctarank() : 0;
+    const int t_begin = kMcast ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int t_step = kMcast ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+    // B tile of k-block kb into the ring slot at `sb`.  In a multicast pair each CTA
+    // fetches one half of the tile and the copy lands in both CTAs' slots.
+    auto load_b = [&](uint32_t sb, const TileCoord& tc, int kb, uint32_t bar) {
+        if constexpr (!kBMn) {
+            if constexpr (kMcast) {
+                constexpr int kHalf = BN / 2;
+                ptx::tma_load_3d_mc(sb + rank * kHalf * 128, &p.tmap_b, kb * BK, tc.tn * BN + rank * kHalf,
+                                    tc.b, bar, 0x3);
+            } else {
+                ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, bar);
+            }
+        } else {
+            constexpr int kBoxes = BN / kAtom;
+            constexpr int kPer = kMcast ? kBoxes / 2 : kBoxes;
+#pragma unroll
+            for (int i = 0; i < kPer; ++i) {
+                const int j = (kMcast ? rank * kPer : 0) + i;
+                if constexpr (kMcast)
+                    ptx::tma_load_3d_mc(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b,
+                                        bar, 0x3);
+                else
+                    ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b, bar);
+            }
+        }
+    };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             ptx::mbar_init(full_bar(s), 1);
-            ptx::mbar_init(empty_bar(s), 1);
+            // multicast pairs: a slot is free once both CTAs' MMAs have read it
+            ptx::mbar_init(empty_bar(s), kMcast ? 2 : 1);
         }
         for (int a = 0; a < 2; ++a) {
             ptx::mbar_init(tfull_bar(a), 1);
@@ -153,14 +193,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         // Warm L2 with the first ring's worth of this CTA's operand tiles while the
         // previous kernel may still be running: an L2 prefetch writes nothing, and L2 is
         // where the previous kernel's stores land, so no stale copy can result.
-        if (blockIdx.x < p.total_tiles) {
-            const TileCoord tc = decode_tile<kCluster>(blockIdx.x, p);
+        if (t_begin < p.total_tiles) {
+            const TileCoord tc = decode_tile<kMode>(t_begin, p, rank);
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
             const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
             for (int kb = kb0; kb < kb1 && kb < kb0 + S; ++kb) {
                 ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm * BM, tc.b);
                 if constexpr (!kBMn) {
-                    ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN, tc.b);
+                    ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN + (kMcast ? rank * (BN / 2) : 0), tc.b);
                 } else {
                     for (int j = 0; j < BN / kAtom; ++j)
                         ptx::tma_prefetch_l2_3d(&p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b);
@@ -176,12 +216,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // multicast pairs: the partner's barriers must be initialised before any copy or
+    // commit of this CTA can reach them
+    if constexpr (kMcast) ptx::cluster_sync();
     // With a constant B the producer arms the first ring and starts its B tiles before
     // the dependency wait (the ring is empty, so no "empty" wait is needed); the loop
     // below then only adds the A tiles of those stages.
     int b_preloaded = 0;
-    if (p.b_const && warp == 0 && blockIdx.x < p.total_tiles) {
-        const TileCoord tc = decode_tile<kCluster>(blockIdx.x, p);
+    if (p.b_const && warp == 0 && t_begin < p.total_tiles) {
+        const TileCoord tc = decode_tile<kMode>(t_begin, p, rank);
         const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
         const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
         b_preloaded = min(S, kb1 - kb0);
@@ -190,14 +233,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                 const int kb = kb0 + i;
                 const uint32_t sb = smem_base + i * kStageBytes + kABytes;
                 ptx::mbar_arrive_expect_tx(full_bar(i), kStageBytes);
-                if constexpr (!kBMn) {
-                    ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, full_bar(i));
-                } else {
-#pragma unroll
-                    for (int j = 0; j < BN / kAtom; ++j)
-                        ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK,
-                                         tc.b, full_bar(i));
-                }
+                load_b(sb, tc, kb, full_bar(i));
             }
         }
         __syncwarp();
@@ -213,8 +249,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t armed = 0, armed_parity = 0;
         bool ok = true;
         int issued = 0;  // k-blocks issued so far by this CTA
-        for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
-            const TileCoord tc = decode_tile<kCluster>(t, p);
+        for (int t = t_begin; ok && t < p.total_tiles; t += t_step) {
+            const TileCoord tc = decode_tile<kMode>(t, p, rank);
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
             const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
             for (int kb = kb0; kb < kb1; ++kb) {
@@ -233,14 +269,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     const uint32_t sb = sa + kABytes;
                     ptx::mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
                     ptx::tma_load_3d(sa, &p.tmap_a, kb * BK, tc.tm * BM, tc.b, full_bar(stage));
-                    if constexpr (!kBMn) {
-                        ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, full_bar(stage));
-                    } else {
-#pragma unroll
-                        for (int j = 0; j < BN / kAtom; ++j)
-                            ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom,
-                                             kb * BK, tc.b, full_bar(stage));
-                    }
+                    load_b(sb, tc, kb, full_bar(stage));
                 }
                 __syncwarp();
                 armed |= 1u << stage;
@@ -265,8 +294,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t phase = 0;
         uint32_t iter = 0;
         bool ok = true;
-        for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x, ++iter) {
-            const TileCoord tc = decode_tile<kCluster>(t, p);
+        for (int t = t_begin; ok && t < p.total_tiles; t += t_step, ++iter) {
+            const TileCoord tc = decode_tile<kMode>(t, p, rank);
             const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
             const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
             const uint32_t acc = iter & 1u;
@@ -297,7 +326,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                         ptx::mma_ss<kKind>(d_tmem, adesc, bdesc, kIdesc,
                                            (kb > kb0 || kk > 0) ? 1u : 0u);
                     }
-                    ptx::tc_commit(empty_bar(stage));
+                    if constexpr (kMcast)
+                        ptx::tc_commit_mc(empty_bar(stage), 0x3);  // frees the slot in both CTAs
+                    else
+                        ptx::tc_commit(empty_bar(stage));
                 }
                 __syncwarp();
                 if (++stage == S) {
@@ -327,8 +359,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t chunk_ctr = 0;
         uint32_t iter = 0;
         const long long MN = (long long)p.M * p.N;
-        for (int t = blockIdx.x; t < p.total_tiles; t += gridDim.x, ++iter) {
-            const TileCoord tc = decode_tile<kCluster>(t, p);
+        for (int t = t_begin; t < p.total_tiles; t += t_step, ++iter) {
+            const TileCoord tc = decode_tile<kMode>(t, p, rank);
             const uint32_t acc = iter & 1u;
             const uint32_t acc_phase = (iter >> 1) & 1u;
             if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
@@ -433,7 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
         }
         ptx::cluster_sync();
-        const TileCoord tc = decode_tile<true>(blockIdx.x, p);
+        const TileCoord tc = decode_tile<kModeClusterSplitK>(blockIdx.x, p, 0);
         constexpr int kVec = BN / 4;
         const float* recv = reinterpret_cast<const float*>(smem);
         float* Cb = p.C + (long long)tc.b * p.stride_c;
@@ -466,23 +498,29 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
+    // multicast pairs: neither CTA leaves while the other may still copy into it or
+    // signal its barriers
+    if constexpr (kMcast) ptx::cluster_sync();
     if (warp == 1) ptx::tmem_dealloc(tmem_base, kTmemCols);
 }
 
 using TcKernel = void (*)(TcParams);
 
-// Instance table, indexed as tc_instance(): variant * 12 + (dtype_i * 2 + kn) * 3 + bn_i,
-// variant 0 = 128-row persistent, 1 = 128-row cluster split-K, 2 = 64-row persistent.
-constexpr int kNumTcInstances = 36;
-#define NNJIT_TC_ROW(K, MN, CL, BM) \
-    tc_gemm_kernel<K, MN, 64, CL, BM>, tc_gemm_kernel<K, MN, 128, CL, BM>, tc_gemm_kernel<K, MN, 256, CL, BM>
+// Instance table, indexed as tc_instance(): variant * 12 + (dtype_i * 2 + kn) * 3 + bn_i
+// for variant 0 = 128-row persistent, 1 = 128-row cluster split-K, 2 = 64-row persistent;
+// then 36 + dtype_i * 2 + kn for the 128 x 256 multicast pairs.
+constexpr int kNumTcInstances = 40;
+#define NNJIT_TC_ROW(K, MN, MODE, BM) \
+    tc_gemm_kernel<K, MN, 64, MODE, BM>, tc_gemm_kernel<K, MN, 128, MODE, BM>, tc_gemm_kernel<K, MN, 256, MODE, BM>
 const TcKernel kTcKernels[kNumTcInstances] = {
-    NNJIT_TC_ROW(0, false, false, 128), NNJIT_TC_ROW(0, true, false, 128),
-    NNJIT_TC_ROW(1, false, false, 128), NNJIT_TC_ROW(1, true, false, 128),
-    NNJIT_TC_ROW(0, false, true, 128),  NNJIT_TC_ROW(0, true, true, 128),
-    NNJIT_TC_ROW(1, false, true, 128),  NNJIT_TC_ROW(1, true, true, 128),
-    NNJIT_TC_ROW(0, false, false, 64),  NNJIT_TC_ROW(0, true, false, 64),
-    NNJIT_TC_ROW(1, false, false, 64),  NNJIT_TC_ROW(1, true, false, 64),
+    NNJIT_TC_ROW(0, false, 0, 128), NNJIT_TC_ROW(0, true, 0, 128),
+    NNJIT_TC_ROW(1, false, 0, 128), NNJIT_TC_ROW(1, true, 0, 128),
+    NNJIT_TC_ROW(0, false, 1, 128), NNJIT_TC_ROW(0, true, 1, 128),
+    NNJIT_TC_ROW(1, false, 1, 128), NNJIT_TC_ROW(1, true, 1, 128),
+    NNJIT_TC_ROW(0, false, 0, 64),  NNJIT_TC_ROW(0, true, 0, 64),
+    NNJIT_TC_ROW(1, false, 0, 64),  NNJIT_TC_ROW(1, true, 0, 64),
+    tc_gemm_kernel<0, false, 256, 2, 128>, tc_gemm_kernel<0, true, 256, 2, 128>,
+    tc_gemm_kernel<1, false, 256, 2, 128>, tc_gemm_kernel<1, true, 256, 2, 128>,
 };
 #undef NNJIT_TC_ROW
 
@@ -552,7 +590,8 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
         cuuint32_t box[3];
         if (p.b_layout == NNJIT_B_NK) {
             dims[0] = (cuuint64_t)p.K; dims[1] = (cuuint64_t)p.N;
-            box[0] = bk; box[1] = (cuuint32_t)c.bn;
+            // a multicast pair fetches each B tile in two halves
+            box[0] = bk; box[1] = (cuuint32_t)(c.bn / (c.cluster_m == 2 ? 2 : 1));
         } else {
             dims[0] = (cuuint64_t)p.N; dims[1] = (cuuint64_t)p.K;
             box[0] = 128 / e; box[1] = bk;
@@ -600,7 +639,11 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     if (c.instance < 0 || c.instance >= kNumTcInstances || !a.tmap_a || !a.tmap_b)
         return cudaErrorInvalidValue;
     const bool cluster = c.instance >= 12 && c.instance < 24;
-    if ((c.instance >= 24) != (c.bm == 64) || (c.bm != 64 && c.bm != 128)) return cudaErrorInvalidValue;
+    const bool mcast = c.instance >= 36;
+    if ((c.instance >= 24 && c.instance < 36) != (c.bm == 64) || (c.bm != 64 && c.bm != 128))
+        return cudaErrorInvalidValue;
+    if (mcast != (c.cluster_m == 2) || (mcast && (c.bn != 256 || c.split_k != 1 || c.grid < 2 || (c.grid & 1))))
+        return cudaErrorInvalidValue;
     if (cluster != (c.reduce == 1)) return cudaErrorInvalidValue;
     if (cluster && (c.split_k < 2 || c.split_k > 8 || (c.split_k & (c.split_k - 1)) != 0))
         return cudaErrorInvalidValue;
@@ -625,20 +668,24 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     prm.split = c.split_k;
     prm.tiles_m = (int)((p.M + c.bm - 1) / c.bm);
     prm.tiles_n = (int)((p.N + c.bn - 1) / c.bn);
-    const long long total = (long long)p.batch * c.split_k * prm.tiles_m * prm.tiles_n;
+    // work items: tiles (x K slices), or pairs of vertically adjacent tiles
+    const long long total = mcast ? (long long)p.batch * ((prm.tiles_m + 1) / 2) * prm.tiles_n
+                                  : (long long)p.batch * c.split_k * prm.tiles_m * prm.tiles_n;
     if (total >= (1LL << 31)) return cudaErrorInvalidValue;
     if (c.split_k > prm.num_kb) return cudaErrorInvalidValue;  // every split owns >= 1 k-block
     prm.total_tiles = (int)total;
     prm.stages = c.stages;
     prm.raster = c.raster;
     // persistent: at most the candidate's grid; cluster mode: one CTA per (tile, slice)
-    const int grid = cluster ? (int)total : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
+    const int grid = cluster ? (int)total
+                     : mcast ? (int)std::min<long long>(2 * total, c.grid)
+                             : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
     // ring + alignment slack + barriers/TMEM slot/abort flag
     const int stage_bytes = (c.bm + c.bn) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     cudaError_t e = prepare_tc_instance(c.instance, smem);
     if (e != cudaSuccess) return e;
-    if (!cluster)
+    if (!cluster && !mcast)
         return launch_pdl(kTcKernels[c.instance], dim3(grid), dim3(kThreads), smem, a.stream, prm);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -649,7 +696,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = (unsigned)c.split_k;
+    attr[1].val.clusterDim.x = mcast ? 2u : (unsigned)c.split_k;
     attr[1].val.clusterDim.y = 1;
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;

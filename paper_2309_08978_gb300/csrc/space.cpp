@@ -33,6 +33,7 @@ nnjit_candidate blank() {
     nnjit_candidate c{};
     c.split_k = 1;
     c.instance = -1;
+    c.cluster_m = 1;
     return c;
 }
 
@@ -57,7 +58,7 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
     const int64_t num_kb = ceil_div(K, BK);
     const int bns[3] = {64, 128, 256};
     const int splits[4] = {1, 2, 4, 8};
-    *naive = 2 * 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2;  // BM x BN x stages x split x raster x reduce
+    *naive = 2 * 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2 * 2;  // BM x BN x stages x split x raster x reduce x pair
     for (int BM : {MC::kTcBM, 64})
     for (int bn : bns) {
         if (bn > 64 && bn > pow2_ceil(N)) continue;  // no tile wider than the padded N
@@ -118,8 +119,25 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 if (split > 1 && reduce == 1)
                     cost += waves * (128LL * bn * 4 / MC::kFeedBytesPerClk);  // DSMEM reduction
                 c.predicted_cost = cost;
-                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM);
+                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM, 0);
                 v.push_back(c);
+                // Multicast pair of the same tile: for full waves of 128 x 256 tiles, two
+                // CTAs of a cluster take vertically adjacent tiles and share each B tile,
+                // halving the B bytes each SM pulls from L2 (32 instead of 48 KB per k-block).
+                if (BM == MC::kTcBM && bn == 256 && split == 1 && tiles >= L.sm_count) {
+                    nnjit_candidate m = c;
+                    m.cluster_m = 2;
+                    const int64_t pairs = p.batch * ceil_div(tiles_m, 2) * tiles_n;
+                    const int64_t pair_slots = std::max<int64_t>(1, slots / 2);
+                    const int64_t live_pairs = std::min(pairs, pair_slots);
+                    const int64_t pwaves = ceil_div(pairs, live_pairs);
+                    m.grid = (int32_t)(2 * live_pairs);
+                    m.wave_eff_ppm = (int32_t)(pairs * 1000000 / (pwaves * live_pairs));
+                    const int64_t feed = ceil_div(stage_bytes - bn * 128 / 2, MC::kFeedBytesPerClk);
+                    m.predicted_cost = pwaves * std::max<int64_t>(2 * 256, feed) * num_kb;
+                    m.instance = tc_instance(p.dtype, p.b_layout, bn, 0, BM, 1);
+                    v.push_back(m);
+                }
             }
         }
     }
@@ -304,10 +322,11 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 
 }  // namespace
 
-int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm) {
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast) {
     const int bi = bn == 64 ? 0 : bn == 128 ? 1 : bn == 256 ? 2 : -1;
     if (bi < 0 || (bm != 64 && bm != 128) || (bm == 64 && cluster)) return -1;
     const int di = dtype == NNJIT_BF16 ? 0 : 1;
+    if (mcast) return (bn == 256 && bm == 128 && !cluster) ? 36 + di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0) : -1;
     const int variant = bm == 64 ? 2 : cluster ? 1 : 0;
     return variant * 12 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
 }

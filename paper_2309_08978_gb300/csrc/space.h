@@ -55,7 +55,7 @@ nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
 
 // Precompiled-instance index helpers (kept in one place so the registry and the space
 // agree).
-int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm);  // 0..35
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast);  // 0..39
 int ffma_instance(int tm, int bm, int bn, int bk, int b_layout);  // 0..23, -1 if none
 int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if none
 

@@ -61,7 +61,8 @@ class nnjit_candidate(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "family", "bm", "bn", "bk", "tm", "tn", "stages", "split_k", "raster", "threads",
         "smem_bytes", "tmem_cols", "regs_per_thread", "blocks_per_sm", "grid", "wave_eff_ppm",
-        "instance")] + [("predicted_cost", ctypes.c_int64), ("reduce", ctypes.c_int32)]
+        "instance")] + [("predicted_cost", ctypes.c_int64), ("reduce", ctypes.c_int32),
+                        ("cluster_m", ctypes.c_int32)]
 
 
 def struct_to_dict(s) -> dict:

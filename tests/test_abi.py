@@ -83,7 +83,7 @@ def test_cache_file_format(lib, tmp_path):
     nj.nnjit_cache_clear()
     empty = tmp_path / "empty.cache"
     nj.nnjit_cache_save(str(empty))
-    assert empty.read_text().splitlines() == ["nnjit-plan-cache v1"]
+    assert empty.read_text().splitlines() == ["nnjit-plan-cache v2"]
     assert nj.nnjit_cache_load(str(empty)) == 0
     bad = tmp_path / "bad.cache"
     bad.write_text("something else\n")
@@ -92,15 +92,15 @@ def test_cache_file_format(lib, tmp_path):
     assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
     # a well-formed entry round-trips through load and save
     entry = ("t=matmul|s=1,2,3,1|dt=2|bl=1|ld=3,3,2|st=3,6,2|bias=0|dev=X,cc103,sm152\t"
-             "1 128 256 64 0 0 4 1 0 192 230656 512 72 1 1 1000000 2 9 0\t0 6 336 12.5 1\t2 0 3.5 1 4.25\n")
+             "1 128 256 64 0 0 4 1 0 192 230656 512 72 1 1 1000000 2 9 0 1\t0 6 336 12.5 1\t2 0 3.5 1 4.25\n")
     good = tmp_path / "good.cache"
-    good.write_text("nnjit-plan-cache v1\n" + entry)
+    good.write_text("nnjit-plan-cache v2\n" + entry)
     assert nj.nnjit_cache_load(str(good)) == 1
     assert nj.nnjit_cache_size() == 1
     out = tmp_path / "out.cache"
     nj.nnjit_cache_save(str(out))
     lines = out.read_text().splitlines()
-    assert lines[0] == "nnjit-plan-cache v1" and lines[1].split("\t")[0] == entry.split("\t")[0]
+    assert lines[0] == "nnjit-plan-cache v2" and lines[1].split("\t")[0] == entry.split("\t")[0]
     assert lines[1].split("\t")[1] == entry.split("\t")[1]
     nj.nnjit_cache_clear()
     assert nj.nnjit_cache_size() == 0

@@ -206,3 +206,26 @@ def test_chain_waits_for_the_producer_of_a():
         assert np.array_equal(C2.cpu().numpy(), want2.astype(np.float32)), f"repetition {rep}"
     p1.destroy()
     p2.destroy()
+
+
+PAIR_CASES = [("bf16", 2048, 2560, 192, "NK"), ("bf16", 2176, 2560, 136, "KN"),
+              ("tf32", 2048, 2560, 64, "NK"), ("tf32", 2200, 2560, 40, "KN")]
+
+
+@pytest.mark.parametrize("case", PAIR_CASES, ids=_ids)
+def test_multicast_pairs_exact(case):
+    """Two CTAs of a cluster take vertically adjacent 128 x 256 tiles and share each B tile
+    through TMA multicast (each fetches one half).  Includes an odd number of tile rows,
+    where the second tile of the last pair lies entirely past M."""
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    A, B, bias = make_operands(shape, 14, dtype, ints=True)
+    for flags in (0, nj.NNJIT_PLAN_B_CONSTANT):
+        desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, flags=flags)
+        cands, _ = nj.nnjit_space_enumerate(desc, nj.nnjit_device_limits_query(0))
+        pairs = [i for i, c in enumerate(cands) if c["cluster_m"] == 2]
+        assert pairs, "expected multicast-pair candidates for a full-wave shape"
+        for i in pairs:
+            with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+                C = run_plan(plan, A, B, bias, M, N)
+            compare(C, A, B, bias, layout, dtype, exact=True)
