@@ -208,6 +208,29 @@ nnjit_status nnjit_matmul_plan_candidate(const nnjit_matmul_desc* d, int32_t ind
                                          nnjit_plan* out);
 
 /*
+ * Online plan (Sec. 3: kernels are evaluated on the device between inferences, and a
+ * newly measured kernel replaces the registered one only if it is significantly faster).
+ * No tuning happens here: the plan serves every nnjit_matmul_run / _run_batched call at
+ * once, with the top-ranked candidate at first.  While the queue (the lite space in
+ * evaluation order) lasts, each call is run instead with the candidate under evaluation
+ * and timed with CUDA events recorded around that call's own launches; the timings are
+ * read back on later calls without synchronising.  After 3 timed calls a candidate
+ * replaces the incumbent if its median is more than 2 % lower.  Every call's result is
+ * correct whichever candidate ran.  When the queue is exhausted the choice is stored in
+ * the plan cache (unless NNJIT_PLAN_NO_CACHE), so later nnjit_matmul_plan_ex calls hit.
+ * Calls on one online plan must not overlap on the GPU (share one stream); synchronise
+ * before nnjit_plan_destroy.  Allocates the plan's workspace (for the widest candidate),
+ * watchdog word and 16 CUDA events.
+ */
+nnjit_status nnjit_matmul_plan_online(const nnjit_matmul_desc* d, nnjit_plan* out);
+
+/* Progress of an online plan: candidates fully evaluated, space size, the index of the
+ * candidate now serving calls, and whether the queue is exhausted (1).  For other plans:
+ * evaluated = space size, done = 1. */
+nnjit_status nnjit_plan_online_progress(nnjit_plan p, int32_t* evaluated, int32_t* space_size,
+                                        int32_t* current_index, int32_t* done);
+
+/*
  * C = A . Bt (+ bias) with the plan's kernel, asynchronously on `stream`.
  * A, B: device pointers (float32 or bf16 per the plan's dtype); bias: float32[N] device
  * pointer or NULL (NULL means no bias even if the plan was made with has_bias);

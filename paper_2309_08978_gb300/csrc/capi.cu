@@ -100,6 +100,24 @@ struct nnjit_plan_s {
     void* hB = nullptr;
     float* hbias = nullptr;
     float* hC = nullptr;
+    // Online tuning (Sec. 3): serve each call with the incumbent candidate or with the
+    // next one of the queue, timed by CUDA events read back on later calls.
+    struct Online {
+        bool active = false;
+        bool done = false;
+        std::vector<nnjit_candidate> space;
+        std::string key;
+        bool store = true;
+        int best = 0;            // incumbent (space index)
+        double best_us = -1.0;   // its median, once measured
+        int eval = 0;            // candidate being evaluated
+        int issued = 0;          // timed launches issued for `eval`
+        std::vector<std::vector<double>> samples;
+        struct Pending { int idx; cudaEvent_t e0, e1; };
+        std::vector<Pending> pending;
+        std::vector<cudaEvent_t> free_events;
+    } online;
+    std::mutex online_mu;
 };
 
 namespace {
@@ -417,6 +435,11 @@ nnjit_status alloc_plan_buffers(nnjit_plan pl) {
 
 void free_plan(nnjit_plan pl) {
     if (!pl) return;
+    for (auto e : pl->online.free_events) cudaEventDestroy(e);
+    for (auto& pd : pl->online.pending) {
+        cudaEventDestroy(pd.e0);
+        cudaEventDestroy(pd.e1);
+    }
     if (pl->err) cudaFree(pl->err);
     if (pl->ws) cudaFree(pl->ws);
     if (pl->hA) cudaFree(pl->hA);
@@ -443,6 +466,82 @@ nnjit_status plan_common(const nnjit_matmul_desc* d, nnjit_plan* out, Problem* p
     st = build_space(*prob, *L, space, naive, &err);
     if (st != NNJIT_OK) return fail(st, err);
     return NNJIT_OK;
+}
+
+// Online tuning parameters: timed launches per candidate and the margin by which a
+// newcomer must beat the incumbent ("significantly faster", Sec. 3).
+constexpr int kOnlineSamples = 3;
+constexpr double kOnlineMargin = 0.02;
+constexpr int kOnlineEventPairs = 8;
+
+double median_of(std::vector<double> v) {
+    std::sort(v.begin(), v.end());
+    return v[v.size() / 2];
+}
+
+// Read back finished timings and advance the evaluation queue.  Caller holds online_mu.
+void online_poll(nnjit_plan pl) {
+    auto& o = pl->online;
+    for (size_t i = 0; i < o.pending.size();) {
+        auto& pd = o.pending[i];
+        if (cudaEventQuery(pd.e1) != cudaSuccess) { ++i; continue; }
+        float ms = 0.f;
+        if (cudaEventElapsedTime(&ms, pd.e0, pd.e1) == cudaSuccess) o.samples[pd.idx].push_back(1000.0 * ms);
+        o.free_events.push_back(pd.e0);
+        o.free_events.push_back(pd.e1);
+        o.pending.erase(o.pending.begin() + (long)i);
+    }
+    while (!o.done && (int)o.samples[o.eval].size() >= kOnlineSamples) {
+        const double med = median_of(o.samples[o.eval]);
+        pl->timings.emplace_back(o.eval, med);
+        if (o.best_us < 0 || (o.eval != o.best && med < o.best_us * (1.0 - kOnlineMargin))) {
+            o.best = o.eval;
+            o.best_us = med;
+        }
+        o.issued = 0;
+        if (++o.eval >= (int)o.space.size()) o.done = true;
+    }
+    pl->cand = o.space[o.best];
+    pl->chosen_index = o.best;
+    if (o.done && o.store && !o.key.empty()) {
+        CacheEntry ce{pl->cand, pl->chosen_index, pl->space_size, pl->naive, pl->timings,
+                      pl->tune_ms, true};
+        std::lock_guard<std::mutex> lk(g_cache_mu);
+        cache()[o.key] = ce;
+        o.store = false;
+    }
+}
+
+// One call of an online plan.
+nnjit_status online_run(nnjit_plan pl, const void* A, const void* B, const float* bias, float* C,
+                        cudaStream_t s) {
+    std::lock_guard<std::mutex> lk(pl->online_mu);
+    auto& o = pl->online;
+    online_poll(pl);
+    const bool explore = !o.done && o.issued < kOnlineSamples && o.free_events.size() >= 2;
+    const int idx = explore ? o.eval : o.best;
+    cudaEvent_t e0 = nullptr, e1 = nullptr;
+    if (explore) {
+        e0 = o.free_events.back(); o.free_events.pop_back();
+        e1 = o.free_events.back(); o.free_events.pop_back();
+        cudaEventRecord(e0, s);
+    }
+    nnjit_status st = run_impl(pl, A, B, bias, C, s, &o.space[idx], pl->ws);
+    if (explore) {
+        if (st != NNJIT_OK) {
+            // a failing newcomer is skipped; the call is served by the incumbent
+            o.free_events.push_back(e0);
+            o.free_events.push_back(e1);
+            pl->failed.push_back(idx);
+            o.samples[idx].assign(kOnlineSamples, 1e300);
+            online_poll(pl);
+            return run_impl(pl, A, B, bias, C, s, &o.space[o.best], pl->ws);
+        }
+        cudaEventRecord(e1, s);
+        o.pending.push_back({idx, e0, e1});
+        ++o.issued;
+    }
+    return st;
 }
 
 }  // namespace
@@ -658,13 +757,66 @@ nnjit_status nnjit_matmul_plan_candidate(const nnjit_matmul_desc* d, int32_t ind
 nnjit_status nnjit_matmul_run(nnjit_plan p, const void* A, const void* B, const float* bias,
                               float* C, void* stream) {
     if (!p) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    if (p->online.active) return online_run(p, A, B, bias, C, static_cast<cudaStream_t>(stream));
     return run_impl(p, A, B, bias, C, static_cast<cudaStream_t>(stream));
+}
+
+nnjit_status nnjit_matmul_plan_online(const nnjit_matmul_desc* d, nnjit_plan* out) {
+    const double t0 = now_ms();
+    Problem p;
+    nnjit_device_limits L;
+    int dev = 0;
+    std::vector<nnjit_candidate> space;
+    int64_t naive = 0;
+    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive);
+    if (st != NNJIT_OK) return st;
+    std::unique_ptr<nnjit_plan_s> pl(new nnjit_plan_s);
+    pl->p = p;
+    pl->device = dev;
+    pl->family = space[0].family;
+    pl->cand = space[0];
+    pl->chosen_index = 0;
+    pl->space_size = (int)space.size();
+    pl->naive = naive;
+    pl->timed = true;
+    auto& o = pl->online;
+    o.active = !p.degenerate();
+    o.space = space;
+    o.samples.assign(space.size(), {});
+    o.key = (p.flags & NNJIT_PLAN_NO_CACHE) ? std::string() : cache_key(p, dev, L);
+    // the workspace serves every candidate of the queue
+    nnjit_candidate widest = space[0];
+    for (const auto& c : space)
+        if (ws_bytes_for(p, c) > ws_bytes_for(p, widest)) widest = c;
+    pl->cand = widest;
+    st = alloc_plan_buffers(pl.get());
+    pl->cand = space[0];
+    if (st != NNJIT_OK) { free_plan(pl.release()); return st; }
+    for (int i = 0; i < 2 * kOnlineEventPairs; ++i) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) { free_plan(pl.release()); return fail(NNJIT_ERR_CUDA, "event create"); }
+        o.free_events.push_back(e);
+    }
+    pl->tune_ms = now_ms() - t0;
+    *out = pl.release();
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_plan_online_progress(nnjit_plan p, int32_t* evaluated, int32_t* space_size,
+                                        int32_t* current_index, int32_t* done) {
+    if (!p) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    std::lock_guard<std::mutex> lk(p->online_mu);
+    if (p->online.active) online_poll(p);
+    if (evaluated) *evaluated = p->online.active ? p->online.eval : p->space_size;
+    if (space_size) *space_size = p->space_size;
+    if (current_index) *current_index = p->chosen_index;
+    if (done) *done = (!p->online.active || p->online.done) ? 1 : 0;
+    return NNJIT_OK;
 }
 
 nnjit_status nnjit_matmul_run_batched(nnjit_plan p, const void* A, const void* B, float* C,
                                       void* stream) {
-    if (!p) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
-    return run_impl(p, A, B, nullptr, C, static_cast<cudaStream_t>(stream));
+    return nnjit_matmul_run(p, A, B, nullptr, C, stream);
 }
 
 nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB,

@@ -112,6 +112,8 @@ def load_library(path: str = LIB_PATH):
             "nnjit_plan_destroy": [vp],
             "nnjit_cache_clear": [],
             "nnjit_gemv_bf16_noalloc": [i64, i64, i64, vp, vp, vp, vp, i32, vp],
+            "nnjit_matmul_plan_online": [P(nnjit_matmul_desc), P(vp)],
+            "nnjit_plan_online_progress": [vp, P(i32), P(i32), P(i32), P(i32)],
             "nnjit_cache_save": [ctypes.c_char_p],
             "nnjit_cache_load": [ctypes.c_char_p, P(i32)],
         }
@@ -255,6 +257,21 @@ def nnjit_matmul_plan_candidate(desc: nnjit_matmul_desc, index: int) -> Plan:
     _check(load_library().nnjit_matmul_plan_candidate(ctypes.byref(desc), index, ctypes.byref(h)),
            "nnjit_matmul_plan_candidate")
     return Plan(h.value, desc)
+
+
+def nnjit_matmul_plan_online(desc: nnjit_matmul_desc) -> Plan:
+    h = ctypes.c_void_p()
+    _check(load_library().nnjit_matmul_plan_online(ctypes.byref(desc), ctypes.byref(h)),
+           "nnjit_matmul_plan_online")
+    return Plan(h.value, desc)
+
+
+def nnjit_plan_online_progress(plan: Plan) -> dict:
+    v = [ctypes.c_int32(0) for _ in range(4)]
+    _check(load_library().nnjit_plan_online_progress(plan.handle, *[ctypes.byref(x) for x in v]),
+           "nnjit_plan_online_progress")
+    return {"evaluated": v[0].value, "space_size": v[1].value, "current_index": v[2].value,
+            "done": bool(v[3].value)}
 
 
 def nnjit_matmul_run(plan: Plan, A, B, bias, C, stream=None):

@@ -125,3 +125,43 @@ def test_invalid_run_arguments():
         with pytest.raises(nj.NnjitError) as ei:
             plan.run(A, None, None, C)
         assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
+
+
+def test_online_plan_serves_exact_results_while_it_tunes():
+    import torch
+    from gpu_util import dev
+    nj.nnjit_cache_clear()
+    M, N, K = 512, 768, 768
+    shape = Shape("t", M, N, K, 1, "NK", True)
+    A, B, bias = make_operands(shape, 33, "bf16", ints=True)
+    from oracle import matmul, B_NK
+    _, ref32 = matmul(A, B, bias, B_NK)
+    desc = nj.make_desc(M, N, K, "bf16", "NK", has_bias=True)
+    plan = nj.nnjit_matmul_plan_online(desc)
+    dA, dB, dbias = dev(A), dev(B), dev(bias)
+    C = torch.empty((M, N), dtype=torch.float32, device="cuda")
+    prog = nj.nnjit_plan_online_progress(plan)
+    assert prog["done"] is False and prog["evaluated"] == 0
+    calls = 0
+    while not prog["done"] and calls < 1000:
+        C.fill_(float("nan"))
+        plan.run(dA, dB, dbias, C)
+        torch.cuda.synchronize()
+        assert np.array_equal(C.cpu().numpy(), ref32), f"call {calls}"
+        calls += 1
+        prog = nj.nnjit_plan_online_progress(plan)
+    assert prog["done"], calls
+    info = plan.describe()
+    assert len(info["timings_us"]) + len(info["failed"]) == info["space_size"]
+    times = dict((int(i), t) for i, t in info["timings_us"])
+    # the incumbent is never beaten by more than the 2 % margin
+    assert times[prog["current_index"]] <= min(times.values()) / 0.98 + 1e-9
+    plan.run(dA, dB, dbias, C)
+    torch.cuda.synchronize()
+    assert np.array_equal(C.cpu().numpy(), ref32)
+    plan.destroy()
+    # the finished choice is in the kernel database
+    with nj.nnjit_matmul_plan_ex(desc, 1000.0) as p2:
+        i2 = p2.describe()
+        assert i2["from_cache"] is True and i2["chosen_index"] == prog["current_index"]
+    nj.nnjit_cache_clear()
