@@ -38,6 +38,9 @@ TC_FIXED_SMEM = 1024 + 256 + 32768   # alignment slack, barriers, epilogue stagi
 TC_MAX_STAGES = 8
 GEMV_MAX_M = 8
 GEMV_MAX_SMEM = 64 * 1024
+GEMV_TMA_KC = 256             # K elements per ring stage of the TMA-fed GEMV
+GEMV_TMA_THREADS = 160        # producer warp + 4 consumer warps
+GEMV_TMA_FIRST = 8            # first instance id of the TMA-fed GEMV kernels
 
 CANDIDATE_FIELDS = ("family", "bm", "bn", "bk", "tm", "tn", "stages", "split_k", "raster",
                     "threads", "smem_bytes", "tmem_cols", "regs_per_thread", "blocks_per_sm",
@@ -197,6 +200,10 @@ def gemv_instance(layout, rows, unroll):
     return {1: 0, 2: 1, 4: 2}[rows] * 2 + u
 
 
+def gemv_tma_instance(rows, maxm):
+    return GEMV_TMA_FIRST + {8: 0, 16: 1, 32: 2}[rows] * 2 + {1: 0, GEMV_MAX_M: 1}[maxm]
+
+
 # ---------------------------------------------------------------------------- families
 
 def _tc(p, lim):
@@ -345,7 +352,42 @@ def _gemv(p, lim):
                                  wave_eff_ppm=grid * 1000000 // (waves * slots),
                                  instance=gemv_instance(B_NK, rows, unroll), predicted_cost=cost)
                         out.append(c)
-        return out, 2 * 3 * 2 * 4
+        # TMA-fed kernels: `stages` boxes of `rows` weight rows x 256 K elements in flight
+        maxm = 1 if M == 1 else GEMV_MAX_M
+        chunks = cdiv(K, GEMV_TMA_KC)
+        for rows in (8, 16, 32):
+            groups = cdiv(N, rows)
+            for stages in (4, 8):
+                for split in (1, 2, 4, 8):
+                    cps = cdiv(chunks, split)
+                    if split > 1 and (cps < 2 or (split - 1) * cps >= chunks or
+                                      groups * (split // 2) >= 2 * lim["sm_count"]):
+                        continue
+                    smem = 128 + stages * (rows + M) * GEMV_TMA_KC * 2
+                    if smem > lim["smem_per_block_optin"]:
+                        continue
+                    regs = 40 if maxm == 1 else 96 + 3 * rows
+                    blk = block_core(lim, regs, GEMV_TMA_THREADS, smem, 0)
+                    if blk < 1:
+                        continue
+                    items = groups * split
+                    slots = lim["sm_count"] * blk
+                    grid = min(items, slots)
+                    inflight = min(cdiv(grid, lim["sm_count"]), blk) * stages * rows * GEMV_TMA_KC * 2
+                    eff = min(100, max(1, inflight * 100 // 32768))
+                    cost = cdiv(wbytes, HBM_BYTES_PER_CLK) * 100 // eff
+                    # the SM with the most items finishes last
+                    cost = cost * cdiv(items, lim["sm_count"]) * lim["sm_count"] // items
+                    if split > 1:
+                        cost += LAUNCH_CLK + cdiv(2 * split * M * N * 4, HBM_BYTES_PER_CLK)
+                    c = _blank()
+                    c.update(family=FAMILY_GEMV, bm=M, bn=rows, bk=GEMV_TMA_KC, tm=rows // 4, tn=1,
+                             stages=stages, split_k=split, threads=GEMV_TMA_THREADS, smem_bytes=smem,
+                             regs_per_thread=regs, blocks_per_sm=blk, grid=grid,
+                             wave_eff_ppm=grid * 1000000 // slots,
+                             instance=gemv_tma_instance(rows, maxm), predicted_cost=cost)
+                    out.append(c)
+        return out, 2 * 3 * 2 * 4 + 3 * 2 * 4
     for threads in (128, 256):
         for unroll in (2, 4):
             warps = threads // 32

@@ -94,6 +94,7 @@ struct nnjit_plan_s {
     const void* tm_B = nullptr;
     const void* tm_C = nullptr;
     bool tm_valid = false;
+    nnjit_candidate tm_cand{};  // the candidate the cached tensor maps were encoded for
     bool tm_c_ok = false;
     CUtensorMap ta, tb, tc;
     void* hA = nullptr;  // device staging for run_host
@@ -229,20 +230,23 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
     la.err = pl->err;
     la.stream = s;
     cudaError_t e = cudaSuccess;
-    if (c.family == NNJIT_FAMILY_TC) {
+    const bool tc = c.family == NNJIT_FAMILY_TC;
+    if (tc || gemv_uses_tma(c)) {
         CUtensorMap ta, tb, tcm;
         bool c_ok = false;
         const char* why = "";
         float* out = two_pass ? ws : C;
         {
             std::lock_guard<std::mutex> lk(pl->mu);
-            if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B || pl->tm_C != out) {
-                e = encode_tc_tensor_maps(p, c, A, B, &ta, &tb, &why);
+            if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B || pl->tm_C != out ||
+                std::memcmp(&pl->tm_cand, &c, sizeof(c)) != 0) {
+                e = tc ? encode_tc_tensor_maps(p, c, A, B, &ta, &tb, &why)
+                       : encode_gemv_tensor_maps(p, c, A, B, &ta, &tb, &why);
                 if (e != cudaSuccess) return fail(NNJIT_ERR_UNSUPPORTED, why);
-                encode_tc_output_map(p, c, out, two_pass, &tcm, &c_ok);
+                if (tc) encode_tc_output_map(p, c, out, two_pass, &tcm, &c_ok);
                 if (!override_cand) {
                     pl->ta = ta; pl->tb = tb; pl->tc = tcm; pl->tm_c_ok = c_ok;
-                    pl->tm_A = A; pl->tm_B = B; pl->tm_C = out; pl->tm_valid = true;
+                    pl->tm_A = A; pl->tm_B = B; pl->tm_C = out; pl->tm_cand = c; pl->tm_valid = true;
                 }
             } else {
                 ta = pl->ta; tb = pl->tb; tcm = pl->tc; c_ok = pl->tm_c_ok;
@@ -251,7 +255,7 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
         la.tmap_a = &ta;
         la.tmap_b = &tb;
         la.tmap_c = c_ok ? &tcm : nullptr;
-        e = launch_tc(la);
+        e = tc ? launch_tc(la) : launch_gemv(la);
     } else if (c.family == NNJIT_FAMILY_FFMA) {
         e = launch_ffma(la);
     } else {

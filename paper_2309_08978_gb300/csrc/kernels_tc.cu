@@ -527,12 +527,7 @@ const TcKernel kTcKernels[kNumTcInstances] = {
 std::mutex g_prep_mu;
 int g_prepared_smem[kNumTcInstances] = {0};
 
-// Driver entry point for cuTensorMapEncodeTiled, fetched through the runtime so the
-// library does not link against libcuda.
-using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
-                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
-                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
-                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+}  // namespace
 
 EncodeTiledFn get_encode_fn() {
     static EncodeTiledFn fn = nullptr;
@@ -547,8 +542,6 @@ EncodeTiledFn get_encode_fn() {
     });
     return fn;
 }
-
-}  // namespace
 
 cudaError_t prepare_tc_instance(int instance, int smem_bytes) {
     if (instance < 0 || instance >= kNumTcInstances) return cudaErrorInvalidValue;

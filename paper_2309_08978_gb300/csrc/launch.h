@@ -78,6 +78,22 @@ cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, flo
 // Detail string for nnjit_last_error() (defined with the C ABI).
 void set_last_error(const char* msg);
 
+// Driver entry point for cuTensorMapEncodeTiled, fetched through the runtime so the
+// library does not link against libcuda (NULL if unavailable).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                   const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn get_encode_fn();
+
+// GEMV candidates whose weights are streamed by TMA (instances kGemvTmaFirstInstance..+5).
+bool gemv_uses_tma(const nnjit_candidate& c);
+cudaError_t launch_gemv_tma(const LaunchArgs& a);
+// Tensor maps of x (*tx, from A) and the weights (*tw, from B) for a TMA GEMV candidate.
+cudaError_t encode_gemv_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,
+                                    const void* B, CUtensorMap* tx, CUtensorMap* tw,
+                                    const char** why);
+
 // Tensor maps for the TC family (host; uses the driver entry point).
 cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,
                                   const void* B, CUtensorMap* ta, CUtensorMap* tb,

@@ -274,6 +274,53 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
                 }
             }
         }
+        // TMA-fed instances: a producer warp keeps `stages` boxes of `rows` weight rows x
+        // 256 K elements in flight; axes rows per stage, ring stages and split-K.
+        const int maxm = M == 1 ? 1 : MC::kGemvMaxM;
+        const int64_t chunks = ceil_div(K, MC::kGemvTmaKc);
+        *naive += 3 * 2 * 4;
+        for (int rows : {8, 16, 32}) {
+            const int64_t groups = ceil_div(N, rows);
+            for (int stages : {4, 8}) {
+                for (int split : {1, 2, 4, 8}) {
+                    const int64_t cps = ceil_div(chunks, split);
+                    if (split > 1 && (cps < 2 || (split - 1) * cps >= chunks ||
+                                      groups * (split / 2) >= 2LL * L.sm_count))
+                        continue;
+                    const int64_t smem = 128 + (int64_t)stages * (rows + M) * MC::kGemvTmaKc * 2;
+                    if (smem > L.smem_per_block_optin) continue;
+                    const int regs = maxm == 1 ? 40 : 96 + 3 * rows;
+                    const int blk = blocks_per_core(L, regs, MC::kGemvTmaThreads, (int)smem, 0);
+                    if (blk < 1) continue;
+                    const int64_t items = groups * split;
+                    const int64_t slots = (int64_t)L.sm_count * blk;
+                    const int64_t grid = std::min<int64_t>(items, slots);
+                    nnjit_candidate c = blank();
+                    c.family = NNJIT_FAMILY_GEMV;
+                    c.bm = (int)M; c.bn = rows; c.bk = MC::kGemvTmaKc;
+                    c.tm = rows / 4; c.tn = 1;
+                    c.stages = stages;
+                    c.split_k = split;
+                    c.threads = MC::kGemvTmaThreads;
+                    c.smem_bytes = (int)smem;
+                    c.regs_per_thread = regs;
+                    c.blocks_per_sm = blk;
+                    c.grid = (int32_t)grid;
+                    c.wave_eff_ppm = (int32_t)(grid * 1000000 / slots);
+                    const int64_t resident = std::min<int64_t>(ceil_div(grid, L.sm_count), blk);
+                    const int64_t inflight = resident * stages * rows * MC::kGemvTmaKc * 2;
+                    const int64_t eff_pct = std::min<int64_t>(100, std::max<int64_t>(1, inflight * 100 / 32768));
+                    int64_t cost = ceil_div(wbytes, MC::kHbmBytesPerClk) * 100 / eff_pct;
+                    // the SM with the most items finishes last
+                    cost = cost * ceil_div(items, L.sm_count) * L.sm_count / items;
+                    if (split > 1)
+                        cost += MC::kLaunchClk + ceil_div(2LL * split * M * N * 4, MC::kHbmBytesPerClk);
+                    c.predicted_cost = cost;
+                    c.instance = gemv_tma_instance(rows, maxm);
+                    v.push_back(c);
+                }
+            }
+        }
     } else {
         *naive = 2 * 2 * 6;
         for (int threads : {128, 256}) {
@@ -351,6 +398,13 @@ int gemv_instance(int b_layout, int rows, int unroll) {
     const int ri = rows == 1 ? 0 : rows == 2 ? 1 : rows == 4 ? 2 : -1;
     if (ri < 0) return -1;
     return ri * 2 + ui;
+}
+
+int gemv_tma_instance(int rows, int maxm) {
+    const int ri = rows == 8 ? 0 : rows == 16 ? 1 : rows == 32 ? 2 : -1;
+    const int mi = maxm == 1 ? 0 : maxm == ModelConstants::kGemvMaxM ? 1 : -1;
+    if (ri < 0 || mi < 0) return -1;
+    return kGemvTmaFirstInstance + ri * 2 + mi;
 }
 
 nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string* err) {

@@ -41,6 +41,8 @@ struct ModelConstants {
     static constexpr int kTcMaxStages = 8;
     static constexpr int kGemvMaxM = 8;
     static constexpr int kGemvMaxSmem = 64 * 1024;
+    static constexpr int kGemvTmaKc = 256;           // K elements per TMA GEMV ring stage
+    static constexpr int kGemvTmaThreads = 160;      // producer warp + 4 consumer warps
 };
 
 // Resolve defaults and validate.  Returns NNJIT_OK or an error with `err` set.
@@ -58,5 +60,8 @@ nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
 int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast);  // 0..39
 int ffma_instance(int tm, int bm, int bn, int bk, int b_layout);  // 0..23, -1 if none
 int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if none
+// TMA-fed GEMV (B as [N][K]): rows per stage 8/16/32, M <= maxm (1 or 8).
+constexpr int kGemvTmaFirstInstance = 8;
+int gemv_tma_instance(int rows, int maxm);                     // 8..13, -1 if none
 
 }  // namespace nnjit

@@ -9,8 +9,9 @@ Shapes span several tiles and ragged tails in M, N and K.
 import numpy as np
 import pytest
 
+import oracle
 from synthetic import Shape, make_operands
-from gpu_util import run_plan, compare
+from gpu_util import compare, dev, layout_code, run_plan
 
 pytestmark = pytest.mark.gpu
 
@@ -64,7 +65,8 @@ def test_random_inputs_tolerance(case):
 EVERY_CANDIDATE = [("f32_ffma", 64, 768, 768, "KN"), ("f32_ffma", 100, 90, 300, "NK"),
                    ("tf32", 64, 768, 768, "KN"), ("tf32", 200, 300, 520, "NK"),
                    ("bf16", 300, 520, 1040, "NK"), ("bf16", 200, 600, 520, "KN"),
-                   ("bf16", 1, 4096, 4096, "NK"), ("bf16", 4, 1000, 2048, "KN")]
+                   ("bf16", 1, 4096, 4096, "NK"), ("bf16", 4, 1000, 2048, "KN"),
+                   ("bf16", 3, 1000, 2056, "NK"), ("bf16", 8, 520, 4096, "NK")]
 
 
 @pytest.mark.parametrize("case", EVERY_CANDIDATE, ids=_ids)
@@ -77,7 +79,7 @@ def test_every_candidate_is_exact(case):
     desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True)
     lim = nj.nnjit_device_limits_query(0)
     cands, _ = nj.nnjit_space_enumerate(desc, lim)
-    assert 1 <= len(cands) <= 64, len(cands)
+    assert 1 <= len(cands) <= 96, len(cands)
     for i, c in enumerate(cands):
         with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
             C = run_plan(plan, A, B, bias, M, N)
@@ -123,18 +125,26 @@ def test_degenerate_shapes(dtype):
             plan.run(None, None, None, None)
 
 
-def test_gemv_ragged_k_with_padded_rows():
+@pytest.mark.parametrize("M", [2, 1])
+def test_gemv_ragged_k_with_padded_rows(M):
     """K = 100 is not a multiple of the 8-element vector: lda = ldb = 104 keeps rows
-    16-byte aligned and the kernel's scalar tail covers the last 4 elements."""
-    M, N, K, ld = 2, 77, 100, 104
+    16-byte aligned; the streaming kernels' scalar tail covers the last 4 elements and
+    the TMA-fed kernels' zero fill past K does.  Every candidate of the space runs."""
+    N, K, ld = 77, 100, 104
     shape = Shape("t", M, N, ld, 1, "NK", True)
     Ap, Bp, bias = make_operands(shape, 11, "bf16", ints=True)
     desc = nj.make_desc(M, N, K, "bf16", "NK", has_bias=True, lda=ld, ldb=ld)
-    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
-        assert plan.describe()["family"] == nj.NNJIT_FAMILY_GEMV
-        C = run_plan(plan, Ap, Bp, bias, M, N)
-    compare(C, np.ascontiguousarray(Ap[:, :K]), np.ascontiguousarray(Bp[:, :K]), bias, "NK",
-            "bf16", exact=True)
+    cands, _ = nj.nnjit_space_enumerate(desc, nj.nnjit_device_limits_query(0))
+    assert any(c["instance"] >= 8 for c in cands)
+    for i, c in enumerate(cands):
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            assert plan.describe()["family"] == nj.NNJIT_FAMILY_GEMV
+            C = run_plan(plan, Ap, Bp, bias, M, N)
+        try:
+            compare(C, np.ascontiguousarray(Ap[:, :K]), np.ascontiguousarray(Bp[:, :K]), bias,
+                    "NK", "bf16", exact=True)
+        except AssertionError as e:
+            raise AssertionError(f"candidate {i} {c}: {e}") from None
 
 
 @pytest.mark.parametrize("ldc", [80, 75])
@@ -206,6 +216,59 @@ def test_chain_waits_for_the_producer_of_a():
         assert np.array_equal(C2.cpu().numpy(), want2.astype(np.float32)), f"repetition {rep}"
     p1.destroy()
     p2.destroy()
+
+
+@pytest.mark.parametrize("M", [1, 3])
+def test_gemv_tma_constant_b_every_candidate(M):
+    """TMA-fed GEMV candidates with NNJIT_PLAN_B_CONSTANT: the weight boxes of the first
+    ring are requested before the dependency wait, x boxes after it.  N and K are not
+    multiples of the box (rows past N and K past 2056 are zero-filled)."""
+    N, K = 1000, 2056
+    shape = Shape("t", M, N, K, 1, "NK", True)
+    A, B, bias = make_operands(shape, 15, "bf16", ints=True)
+    desc = nj.make_desc(M, N, K, "bf16", "NK", has_bias=True,
+                        flags=nj.NNJIT_PLAN_B_CONSTANT | nj.NNJIT_PLAN_NO_CACHE)
+    cands, _ = nj.nnjit_space_enumerate(desc, nj.nnjit_device_limits_query(0))
+    tma = [i for i, c in enumerate(cands) if c["instance"] >= 8]
+    assert tma
+    for i in tma:
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            C = run_plan(plan, A, B, bias, M, N)
+        compare(C, A, B, bias, "NK", "bf16", exact=True)
+
+
+def test_gemv_tma_writes_after_the_previous_kernel():
+    """A slow product writes C, then a TMA-fed GEMV with constant weights writes the same
+    C on the same stream: the second one's results must be the ones left in C."""
+    import torch
+    M, N, K1, K2 = 1, 4096, 8192, 512
+    s1 = Shape("t", M, N, K1, 1, "NK", False)
+    s2 = Shape("t", M, N, K2, 1, "NK", False)
+    A1, B1, _ = make_operands(s1, 16, "bf16", ints=True)
+    A2, B2, _ = make_operands(s2, 17, "bf16", ints=True)
+    flags = nj.NNJIT_PLAN_B_CONSTANT | nj.NNJIT_PLAN_NO_CACHE
+    d1 = nj.make_desc(M, N, K1, "bf16", "NK", flags=flags)
+    d2 = nj.make_desc(M, N, K2, "bf16", "NK", flags=flags)
+    c2, _ = nj.nnjit_space_enumerate(d2, nj.nnjit_device_limits_query(0))
+    tma = [i for i, c in enumerate(c2) if c["instance"] >= 8]
+    _, ref32 = oracle.matmul(A2, B2, None, layout_code("NK"))
+    dA1, dB1, dA2, dB2 = dev(A1), dev(B1), dev(A2), dev(B2)
+    p1 = nj.nnjit_matmul_plan_candidate(d1, 0)
+    st = torch.cuda.Stream()
+    try:
+        for i in tma:
+            with nj.nnjit_matmul_plan_candidate(d2, i) as p2:
+                for rep in range(5):
+                    C = torch.full((M, N), float("nan"), device="cuda")
+                    torch.cuda.synchronize()
+                    with torch.cuda.stream(st):
+                        p1.run(dA1, dB1, None, C, st)
+                        p2.run(dA2, dB2, None, C, st)
+                    st.synchronize()
+                    p2.check()
+                    assert np.array_equal(C.cpu().numpy(), ref32), f"candidate {i} repetition {rep}"
+    finally:
+        p1.destroy()
 
 
 PAIR_CASES = [("bf16", 2048, 2560, 192, "NK"), ("bf16", 2176, 2560, 136, "KN"),
