@@ -66,7 +66,7 @@ def kernel_key(s, dtype, cand):
     """Identifies one kernel configuration on one product (the traffic table's key)."""
     fam = {0: "ffma", 1: "tc", 2: "gemv"}[cand["family"]]
     return (f"{fam} {dtype} {s.batch}x{s.M}x{s.N}x{s.K} {s.b_layout} bm{cand['bm']} bn{cand['bn']} "
-            f"st{cand['stages']} split{cand['split_k']} red{cand['reduce']} rast{cand['raster']}")
+            f"bk{cand['bk']} st{cand['stages']} split{cand['split_k']} red{cand['reduce']} rast{cand['raster']}")
 
 
 def lookup_traffic(key):

@@ -31,11 +31,14 @@ FEED_BYTES_PER_CLK = 64       # per-SM L2 -> SM operand feed
 HBM_BYTES_PER_CLK = 3500      # chip-wide HBM bytes per SM clock
 LAUNCH_CLK = 2000             # one extra kernel launch
 REG_SHARE_PCT = 50            # Table 1's Reg_thread is this share of a thread's registers
-TC_REGS = 72                  # registers per thread of the tensor-core kernel
+TC_REGS = 80                  # registers per thread of the tensor-core kernel (ptxas: 72-80)
 TC_THREADS = 192
 TC_BM = 128
 TC_FIXED_SMEM = 1024 + 256 + 32768   # alignment slack, barriers, epilogue staging
 TC_MAX_STAGES = 8
+MMA_N256_CLK = 128            # tensor pipe: one M = 128, N = 256 MMA instruction
+MMA_ISSUE_CLK = 57            # issuing thread: one tcgen05.mma
+SLOT_SYNC_CLK = 226           # issuing thread: one ring-slot barrier wait + commit
 GEMV_MAX_M = 8
 GEMV_MAX_SMEM = 64 * 1024
 GEMV_TMA_KC = 256             # K elements per ring stage of the TMA-fed GEMV
@@ -177,7 +180,9 @@ def _blank():
     return c
 
 
-def tc_instance(dtype, b_layout, bn, cluster, bm, mcast=False):
+def tc_instance(dtype, b_layout, bn, cluster, bm, mcast=False, kg=1):
+    if kg == 2:
+        return 40 + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 2 + {64: 0, 128: 1}[bn]
     if mcast:
         return 36 + (0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)
     variant = 2 if bm == 64 else (1 if cluster else 0)
@@ -212,13 +217,17 @@ def _tc(p, lim):
     M, N, K = max(p.M, 1), max(p.N, 1), max(p.K, 1)
     num_kb = cdiv(K, bk)
     out = []
-    for bm, bn in [(m, n) for m in (TC_BM, 64) for n in (64, 128, 256)]:
+    for bm, bn, kg in [(m, n, g) for m in (TC_BM, 64) for n in (64, 128, 256) for g in (1, 2)]:
         if bn > 64 and bn > pow2_at_least(N):
             continue
         # 64-row tiles only where 128-row tiles would leave SMs idle
         if bm == 64 and p.batch * cdiv(M, TC_BM) * cdiv(N, bn) >= lim["sm_count"]:
             continue
-        stage = (bm + bn) * 128
+        # two k-blocks per ring slot only where the MMA issue path is the bottleneck
+        if kg == 2 and (bm != TC_BM or bn > 128):
+            continue
+        kb_bytes = (bm + bn) * 128
+        stage = kg * kb_bytes
         stages = min(TC_MAX_STAGES, (lim["smem_per_block_optin"] - TC_FIXED_SMEM) // stage)
         if stages < 2:
             continue
@@ -234,7 +243,7 @@ def _tc(p, lim):
         for split in (1, 2, 4, 8):
             if split > 1 and (tiles * (split // 2) >= lim["sm_count"] or num_kb < 4 * split):
                 continue
-            for reduce in ((0, 1) if split > 1 else (0,)):
+            for reduce in ((0, 1) if split > 1 and kg == 1 else (0,)):
                 for raster in (0, 1):
                     if raster == 1 and (tiles_m == 1 or tiles_n == 1):
                         continue
@@ -245,17 +254,20 @@ def _tc(p, lim):
                     slots = lim["sm_count"] * blk
                     live = min(work, slots)
                     waves = cdiv(work, live)
-                    t_kb = max(2 * 256 * bm // TC_BM, cdiv(stage, FEED_BYTES_PER_CLK))
+                    # per k-block: tensor pipe, issuing thread, operand feed
+                    t_tensor = 4 * max(MMA_N256_CLK // 4, MMA_N256_CLK * bn // 256)
+                    t_issue = 4 * MMA_ISSUE_CLK + SLOT_SYNC_CLK // kg
+                    t_kb = max(t_tensor, t_issue, cdiv(kb_bytes, FEED_BYTES_PER_CLK))
                     cost = waves * t_kb * cdiv(num_kb, split)
                     if split > 1 and reduce == 0:
                         cost += LAUNCH_CLK + cdiv(2 * split * p.batch * M * N * 4, HBM_BYTES_PER_CLK)
                     if split > 1 and reduce == 1:
                         cost += waves * (TC_BM * bn * 4 // FEED_BYTES_PER_CLK)
-                    c.update(family=FAMILY_TC, bm=bm, bn=bn, bk=bk, stages=stages, split_k=split,
+                    c.update(family=FAMILY_TC, bm=bm, bn=bn, bk=bk * kg, stages=stages, split_k=split,
                              raster=raster, threads=TC_THREADS, smem_bytes=smem, tmem_cols=tmem,
                              regs_per_thread=TC_REGS, blocks_per_sm=blk,
                              grid=work if reduce else live, wave_eff_ppm=work * 1000000 // (waves * live),
-                             instance=tc_instance(p.dtype, p.b_layout, bn, reduce, bm),
+                             instance=tc_instance(p.dtype, p.b_layout, bn, reduce, bm, kg=kg),
                              predicted_cost=cost, reduce=reduce)
                     out.append(c)
                     # multicast pair: two CTAs of a cluster share each B tile
@@ -269,7 +281,7 @@ def _tc(p, lim):
                                  predicted_cost=pw * max(2 * 256, feed) * num_kb,
                                  instance=tc_instance(p.dtype, p.b_layout, bn, 0, bm, True))
                         out.append(m)
-    return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2
+    return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2 * 2
 
 
 def _ffma(p, lim):

@@ -33,6 +33,7 @@ constexpr int kKc = 256;              // K elements per stage
 constexpr int kRowBytes = kKc * 2;    // bytes of one row of one stage
 constexpr int kThreads = 160;         // producer warp + 4 consumer warps
 constexpr int kMaxStages = 8;
+constexpr long long kPrefetchBytes = 48ll << 20;
 constexpr int kErrGemvEmpty = 0x201;
 constexpr int kErrGemvFull = 0x202;
 constexpr int kErrGemvDrain = 0x203;
@@ -51,6 +52,7 @@ struct GemvTmaParams {
     int items;           // groups * split
     int stages;
     int b_const;         // W is not written by kernels launched earlier in the stream
+    int pf_chunks;       // b_const: chunks of the first item past the ring to prefetch into L2
     long long ldc;
 };
 
@@ -117,6 +119,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
             // With constant weights the first ring's worth of weight boxes is requested
             // before the dependency wait; their x boxes follow once the previous kernel
             // (which may produce x) has finished.
+            // Weights are read once: their lines go first when L2 needs room, so they do
+            // not evict what the next kernel has prefetched.
+            const uint64_t pol = ptx::l2_policy_evict_first();
             int pre = 0;
             int pre_chunk[kMaxStages];
             Item first{};
@@ -124,9 +129,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
                 first = item_of(blockIdx.x, p);
                 for (int c = first.c0; c < first.c1 && pre < S; ++c, ++pre) {
                     ptx::mbar_arrive_expect_tx(full_bar(pre), kWBytes + xbytes);
-                    ptx::tma_load_2d(w_base + pre * kWBytes, &p.tmap_w, c * kKc, first.g * ROWS, full_bar(pre));
+                    ptx::tma_load_2d_hint(w_base + pre * kWBytes, &p.tmap_w, c * kKc, first.g * ROWS,
+                                          full_bar(pre), pol);
                     pre_chunk[pre] = c;
                 }
+                // ... and the next part of the first item is brought into L2, so the
+                // weight stream keeps HBM busy while the previous kernel drains.
+                const int pf_end = min(first.c1, first.c0 + pre + p.pf_chunks);
+                for (int c = first.c0 + pre; c < pf_end; ++c)
+                    ptx::tma_prefetch_l2_2d(&p.tmap_w, c * kKc, first.g * ROWS);
             }
             ptx::griddep_wait();
             ptx::griddep_launch_dependents();
@@ -146,7 +157,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
                         break;
                     }
                     ptx::mbar_arrive_expect_tx(full_bar(stage), kWBytes + xbytes);
-                    ptx::tma_load_2d(w_base + stage * kWBytes, &p.tmap_w, c * kKc, w.g * ROWS, full_bar(stage));
+                    ptx::tma_load_2d_hint(w_base + stage * kWBytes, &p.tmap_w, c * kKc, w.g * ROWS,
+                                          full_bar(stage), pol);
                     ptx::tma_load_2d(x_base + stage * xbytes, &p.tmap_x, c * kKc, 0, full_bar(stage));
                     armed |= 1u << stage;
                     armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
@@ -336,6 +348,13 @@ cudaError_t launch_gemv_tma(const LaunchArgs& a) {
     prm.b_const = (p.flags & NNJIT_PLAN_B_CONSTANT) ? 1 : 0;
     prm.ldc = p.ldc;
     const int grid = (int)std::min<long long>(items, std::max(1, c.grid));
+    // L2 prefetch ahead of the dependency wait: at most kPrefetchBytes over the grid
+    // (well under the 129 MB L2, which the previous kernel is also streaming through).
+    prm.pf_chunks = 0;
+    if (prm.b_const) {
+        const long long per_cta = kPrefetchBytes / grid / ((long long)kRowsOf[i] * kRowBytes);
+        prm.pf_chunks = (int)std::min<long long>(per_cta, prm.cps);
+    }
     const int smem = 128 + c.stages * (kRowsOf[i] + (int)p.M) * kRowBytes;
     {
         std::lock_guard<std::mutex> lk(g_mu);

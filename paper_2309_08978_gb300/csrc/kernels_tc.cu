@@ -98,11 +98,15 @@ constexpr int kErrMmaFull = 0x112;
 constexpr int kErrEpiTmemFull = 0x121;
 constexpr int kErrDrain = 0x131;
 
-template <int kKind, bool kBMn, int BN, int kMode, int BM>
+// KG: k-blocks per ring slot.  Each slot is guarded by one pair of barriers, so the MMA
+// issuer pays one barrier wait and one commit per KG k-blocks (4 * KG instructions);
+// with N <= 128 the issue path, not the tensor pipe, sets the pace, and KG = 2 shortens it.
+template <int kKind, bool kBMn, int BN, int kMode, int BM, int KG>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
     constexpr bool kCluster = kMode == kModeClusterSplitK;
     constexpr bool kMcast = kMode == kModeMcastPair;
     static_assert(BM == 128 || (BM == 64 && kMode == kModePersistent), "BM 64 tiles run persistent only");
+    static_assert(KG == 1 || (KG == 2 && kMode == kModePersistent), "k-block groups run persistent only");
     // Rows of the accumulator per epilogue warp.  An M = 128 MMA puts row r in TMEM lane
     // r; an M = 64 MMA puts rows 16q .. 16q+15 in lanes 32q .. 32q+15 of sub-partition q.
     constexpr int kRowsPerWarp = BM / 4;
@@ -113,7 +117,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     constexpr int kAtom = 128 / kElem;                  // MN-major swizzle atom width (elements)
     constexpr uint32_t kABytes = BM * 128;              // 16 KB (BM 128) or 8 KB
     constexpr uint32_t kBBytes = BN * 128;
-    constexpr uint32_t kStageBytes = kABytes + kBBytes;
+    constexpr uint32_t kStageBytes = kABytes + kBBytes;  // one k-block
+    constexpr uint32_t kGroupBytes = KG * kStageBytes;   // one ring slot
     constexpr uint32_t kTmemCols = 2 * BN < 32 ? 32 : 2 * BN;
     constexpr uint32_t kIdesc = ptx::instr_desc(kKind == 0 ? 1u : 2u, kBMn, BM, BN);
     // MN-major 32-bit (tf32) operands use the 32-byte-atom variant of the 128-byte swizzle
@@ -127,7 +132,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~static_cast<uintptr_t>(1023));
     const int S = p.stages;
-    uint8_t* epi_smem = smem + (size_t)S * kStageBytes;  // 1024-aligned (stage bytes are)
+    uint8_t* epi_smem = smem + (size_t)S * kGroupBytes;  // 1024-aligned (stage bytes are)
     uint64_t* bars = reinterpret_cast<uint64_t*>(epi_smem + kEpiStageBytes);
     // bars[0..S): full, [S..2S): empty, 2S..2S+1: tmem_full, 2S+2..2S+3: tmem_empty,
     // 2S+4: drain
@@ -142,6 +147,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     auto tfull_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + a); };
     auto tempty_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + 2 + a); };
     const uint32_t drain_bar = ptx::smem_u32(bars + 2 * S + 4);
+    // k-blocks [kb0, kb1) of a work item
+    auto kb_range = [&](const TileCoord& tc, int& kb0, int& kb1) {
+        kb0 = (int)((long long)tc.s * p.num_kb / p.split);
+        kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
+    };
     // Multicast pairs: this CTA's rank in its cluster; work items are pairs.
     const int rank = kMcast ? (int)ptx::cluster_ctarank() : 0;
     const int t_begin = kMcast ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
@@ -195,9 +205,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         // where the previous kernel's stores land, so no stale copy can result.
         if (t_begin < p.total_tiles) {
             const TileCoord tc = decode_tile<kMode>(t_begin, p, rank);
-            const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
-            const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
-            for (int kb = kb0; kb < kb1 && kb < kb0 + S; ++kb) {
+            int kb0, kb1;
+            kb_range(tc, kb0, kb1);
+            for (int kb = kb0; kb < kb1 && kb < kb0 + S * KG; ++kb) {
                 ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm * BM, tc.b);
                 if constexpr (!kBMn) {
                     ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN + (kMcast ? rank * (BN / 2) : 0), tc.b);
@@ -222,18 +232,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     // With a constant B the producer arms the first ring and starts its B tiles before
     // the dependency wait (the ring is empty, so no "empty" wait is needed); the loop
     // below then only adds the A tiles of those stages.
-    int b_preloaded = 0;
+    int b_preloaded = 0;  // ring slots whose B tiles are already requested
     if (p.b_const && warp == 0 && t_begin < p.total_tiles) {
         const TileCoord tc = decode_tile<kMode>(t_begin, p, rank);
-        const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
-        const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
-        b_preloaded = min(S, kb1 - kb0);
+        int kb0, kb1;
+        kb_range(tc, kb0, kb1);
+        b_preloaded = min(S, (kb1 - kb0 + KG - 1) / KG);
         if (lane == 0) {
             for (int i = 0; i < b_preloaded; ++i) {
-                const int kb = kb0 + i;
-                const uint32_t sb = smem_base + i * kStageBytes + kABytes;
-                ptx::mbar_arrive_expect_tx(full_bar(i), kStageBytes);
-                load_b(sb, tc, kb, full_bar(i));
+                const int g0 = kb0 + i * KG;
+                const int nk = min(KG, kb1 - g0);
+                ptx::mbar_arrive_expect_tx(full_bar(i), nk * kStageBytes);
+                for (int j = 0; j < nk; ++j)
+                    load_b(smem_base + i * kGroupBytes + j * kStageBytes + kABytes, tc, g0 + j, full_bar(i));
             }
         }
         __syncwarp();
@@ -248,28 +259,27 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t phase = 0;
         uint32_t armed = 0, armed_parity = 0;
         bool ok = true;
-        int issued = 0;  // k-blocks issued so far by this CTA
+        int issued = 0;  // ring slots filled so far by this CTA
         for (int t = t_begin; ok && t < p.total_tiles; t += t_step) {
             const TileCoord tc = decode_tile<kMode>(t, p, rank);
-            const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
-            const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
-            for (int kb = kb0; kb < kb1; ++kb) {
+            int kb0, kb1;
+            kb_range(tc, kb0, kb1);
+            for (int g0 = kb0; g0 < kb1; g0 += KG) {
+                const int nk = min(KG, kb1 - g0);
                 if (!ptx::mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, p.err,
                                     kErrProducerEmpty)) {
                     ok = false;
                     break;
                 }
-                const bool pre = issued < b_preloaded;  // B of this stage already on its way
+                const bool pre = issued < b_preloaded;  // B of this slot already on its way
                 ++issued;
-                if (lane == 0 && pre) {
-                    ptx::tma_load_3d(smem_base + stage * kStageBytes, &p.tmap_a, kb * BK, tc.tm * BM, tc.b,
-                                     full_bar(stage));
-                } else if (lane == 0) {
-                    const uint32_t sa = smem_base + stage * kStageBytes;
-                    const uint32_t sb = sa + kABytes;
-                    ptx::mbar_arrive_expect_tx(full_bar(stage), kStageBytes);
-                    ptx::tma_load_3d(sa, &p.tmap_a, kb * BK, tc.tm * BM, tc.b, full_bar(stage));
-                    load_b(sb, tc, kb, full_bar(stage));
+                if (lane == 0) {
+                    if (!pre) ptx::mbar_arrive_expect_tx(full_bar(stage), nk * kStageBytes);
+                    for (int j = 0; j < nk; ++j) {
+                        const uint32_t sa = smem_base + stage * kGroupBytes + j * kStageBytes;
+                        ptx::tma_load_3d(sa, &p.tmap_a, (g0 + j) * BK, tc.tm * BM, tc.b, full_bar(stage));
+                        if (!pre) load_b(sa + kABytes, tc, g0 + j, full_bar(stage));
+                    }
                 }
                 __syncwarp();
                 armed |= 1u << stage;
@@ -294,10 +304,16 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t phase = 0;
         uint32_t iter = 0;
         bool ok = true;
+        // Descriptors of ring slot 0; a slot's are these plus its byte offset >> 4 (the
+        // start-address field holds shared addresses >> 4, below 2^14, so no carry).
+        const uint64_t a_desc0 = ptx::smem_desc(smem_base, 16, 1024);
+        const uint64_t b_desc0 = kBMn ? ptx::smem_desc(smem_base + kABytes, BK * 128, kBSbo, kBLayout)
+                                      : ptx::smem_desc(smem_base + kABytes, 16, 1024);
+        constexpr uint32_t kBStep = kBMn ? (kUmmaK * 128) >> 4 : 32 >> 4;  // per MMA along K
         for (int t = t_begin; ok && t < p.total_tiles; t += t_step, ++iter) {
             const TileCoord tc = decode_tile<kMode>(t, p, rank);
-            const int kb0 = (int)((long long)tc.s * p.num_kb / p.split);
-            const int kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
+            int kb0, kb1;
+            kb_range(tc, kb0, kb1);
             const uint32_t acc = iter & 1u;
             const uint32_t acc_phase = (iter >> 1) & 1u;
             if (!ptx::mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty)) {
@@ -306,25 +322,24 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
             ptx::tc_fence_after();
             const uint32_t d_tmem = tmem_base + acc * BN;
-            for (int kb = kb0; kb < kb1; ++kb) {
+            for (int g0 = kb0; g0 < kb1; g0 += KG) {
+                const int nk = min(KG, kb1 - g0);
                 if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull)) {
                     ok = false;
                     break;
                 }
                 ptx::tc_fence_after();
                 if (lane == 0) {
-                    const uint32_t sa = smem_base + stage * kStageBytes;
-                    const uint32_t sb = sa + kABytes;
 #pragma unroll
-                    for (int kk = 0; kk < kKSteps; ++kk) {
-                        const uint64_t adesc = ptx::smem_desc(sa + kk * 32, 16, 1024);
-                        uint64_t bdesc;
-                        if constexpr (!kBMn)
-                            bdesc = ptx::smem_desc(sb + kk * 32, 16, 1024);
-                        else
-                            bdesc = ptx::smem_desc(sb + kk * kUmmaK * 128, BK * 128, kBSbo, kBLayout);
-                        ptx::mma_ss<kKind>(d_tmem, adesc, bdesc, kIdesc,
-                                           (kb > kb0 || kk > 0) ? 1u : 0u);
+                    for (int j = 0; j < KG; ++j) {
+                        if (j < nk) {
+                            const uint64_t off = (uint64_t)((stage * kGroupBytes + j * kStageBytes) >> 4);
+                            const uint64_t ad = a_desc0 + off, bd = b_desc0 + off;
+#pragma unroll
+                            for (int kk = 0; kk < kKSteps; ++kk)
+                                ptx::mma_ss<kKind>(d_tmem, ad + 2 * kk, bd + kBStep * kk, kIdesc,
+                                                   (g0 > kb0 || j > 0 || kk > 0) ? 1u : 0u);
+                        }
                     }
                     if constexpr (kMcast)
                         ptx::tc_commit_mc(empty_bar(stage), 0x3);  // frees the slot in both CTAs
@@ -508,10 +523,14 @@ using TcKernel = void (*)(TcParams);
 
 // Instance table, indexed as tc_instance(): variant * 12 + (dtype_i * 2 + kn) * 3 + bn_i
 // for variant 0 = 128-row persistent, 1 = 128-row cluster split-K, 2 = 64-row persistent;
-// then 36 + dtype_i * 2 + kn for the 128 x 256 multicast pairs.
-constexpr int kNumTcInstances = 40;
-#define NNJIT_TC_ROW(K, MN, MODE, BM) \
-    tc_gemm_kernel<K, MN, 64, MODE, BM>, tc_gemm_kernel<K, MN, 128, MODE, BM>, tc_gemm_kernel<K, MN, 256, MODE, BM>
+// then 36 + dtype_i * 2 + kn for the 128 x 256 multicast pairs; then
+// 40 + (dtype_i * 2 + kn) * 2 + (BN == 128) for 128-row persistent tiles with two k-blocks
+// per ring slot.
+constexpr int kNumTcInstances = 48;
+#define NNJIT_TC_ROW(K, MN, MODE, BM)                                                  \
+    tc_gemm_kernel<K, MN, 64, MODE, BM, 1>, tc_gemm_kernel<K, MN, 128, MODE, BM, 1>, \
+        tc_gemm_kernel<K, MN, 256, MODE, BM, 1>
+#define NNJIT_TC_KG2(K, MN) tc_gemm_kernel<K, MN, 64, 0, 128, 2>, tc_gemm_kernel<K, MN, 128, 0, 128, 2>
 const TcKernel kTcKernels[kNumTcInstances] = {
     NNJIT_TC_ROW(0, false, 0, 128), NNJIT_TC_ROW(0, true, 0, 128),
     NNJIT_TC_ROW(1, false, 0, 128), NNJIT_TC_ROW(1, true, 0, 128),
@@ -519,10 +538,12 @@ const TcKernel kTcKernels[kNumTcInstances] = {
     NNJIT_TC_ROW(1, false, 1, 128), NNJIT_TC_ROW(1, true, 1, 128),
     NNJIT_TC_ROW(0, false, 0, 64),  NNJIT_TC_ROW(0, true, 0, 64),
     NNJIT_TC_ROW(1, false, 0, 64),  NNJIT_TC_ROW(1, true, 0, 64),
-    tc_gemm_kernel<0, false, 256, 2, 128>, tc_gemm_kernel<0, true, 256, 2, 128>,
-    tc_gemm_kernel<1, false, 256, 2, 128>, tc_gemm_kernel<1, true, 256, 2, 128>,
+    tc_gemm_kernel<0, false, 256, 2, 128, 1>, tc_gemm_kernel<0, true, 256, 2, 128, 1>,
+    tc_gemm_kernel<1, false, 256, 2, 128, 1>, tc_gemm_kernel<1, true, 256, 2, 128, 1>,
+    NNJIT_TC_KG2(0, false), NNJIT_TC_KG2(0, true), NNJIT_TC_KG2(1, false), NNJIT_TC_KG2(1, true),
 };
 #undef NNJIT_TC_ROW
+#undef NNJIT_TC_KG2
 
 std::mutex g_prep_mu;
 int g_prepared_smem[kNumTcInstances] = {0};
@@ -632,8 +653,12 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     if (c.instance < 0 || c.instance >= kNumTcInstances || !a.tmap_a || !a.tmap_b)
         return cudaErrorInvalidValue;
     const bool cluster = c.instance >= 12 && c.instance < 24;
-    const bool mcast = c.instance >= 36;
+    const bool mcast = c.instance >= 36 && c.instance < 40;
+    const int kg = c.instance >= 40 ? 2 : 1;  // k-blocks per ring slot
+    const int bk = 128 / p.elem_bytes();      // K elements per k-block
     if ((c.instance >= 24 && c.instance < 36) != (c.bm == 64) || (c.bm != 64 && c.bm != 128))
+        return cudaErrorInvalidValue;
+    if (c.bk != bk * kg || (kg == 2 && (c.bm != 128 || c.bn > 128 || c.split_k < 1 || c.reduce != 0)))
         return cudaErrorInvalidValue;
     if (mcast != (c.cluster_m == 2) || (mcast && (c.bn != 256 || c.split_k != 1 || c.grid < 2 || (c.grid & 1))))
         return cudaErrorInvalidValue;
@@ -657,7 +682,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     prm.batch = (int)p.batch;
     prm.ldc = p.ldc;
     prm.stride_c = p.stride_c;
-    prm.num_kb = (int)((p.K + c.bk - 1) / c.bk);
+    prm.num_kb = (int)((p.K + bk - 1) / bk);
     prm.split = c.split_k;
     prm.tiles_m = (int)((p.M + c.bm - 1) / c.bm);
     prm.tiles_n = (int)((p.N + c.bn - 1) / c.bn);
@@ -674,7 +699,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
                      : mcast ? (int)std::min<long long>(2 * total, c.grid)
                              : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
     // ring + alignment slack + barriers/TMEM slot/abort flag
-    const int stage_bytes = (c.bm + c.bn) * 128;
+    const int stage_bytes = kg * (c.bm + c.bn) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     cudaError_t e = prepare_tc_instance(c.instance, smem);
     if (e != cudaSuccess) return e;

@@ -58,12 +58,17 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
     const int64_t num_kb = ceil_div(K, BK);
     const int bns[3] = {64, 128, 256};
     const int splits[4] = {1, 2, 4, 8};
-    *naive = 2 * 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2 * 2;  // BM x BN x stages x split x raster x reduce x pair
+    // BM x BN x stages x split x raster x reduce x pair x k-blocks per ring slot
+    *naive = 2 * 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2 * 2 * 2;
     for (int BM : {MC::kTcBM, 64})
-    for (int bn : bns) {
+    for (int bn : bns)
+    for (int kg : {1, 2}) {
         if (bn > 64 && bn > pow2_ceil(N)) continue;  // no tile wider than the padded N
         if (BM == 64 && p.batch * ceil_div(M, MC::kTcBM) * ceil_div(N, bn) >= L.sm_count) continue;
-        const int stage_bytes = (BM + bn) * 128;
+        // two k-blocks per ring slot only where the MMA issue path is the bottleneck
+        if (kg == 2 && (BM != MC::kTcBM || bn > 128)) continue;
+        const int kb_bytes = (BM + bn) * 128;
+        const int stage_bytes = kg * kb_bytes;
         const int stages = std::min(MC::kTcMaxStages,
                                     (L.smem_per_block_optin - MC::kTcFixedSmem) / stage_bytes);
         if (stages < 2) continue;
@@ -81,14 +86,14 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
             // split-K partials: summed by a second kernel (reduce 0) or, one output tile
             // per thread-block cluster of `split` CTAs, through distributed shared memory
             // (reduce 1; the partial tile reuses the idle ring)
-            for (int reduce = 0; reduce < (split > 1 ? 2 : 1); ++reduce)
+            for (int reduce = 0; reduce < (split > 1 && kg == 1 ? 2 : 1); ++reduce)
             for (int raster = 0; raster < 2; ++raster) {
                 if (raster == 1 && (tiles_m == 1 || tiles_n == 1)) continue;
                 if (reduce == 1 && (BM != MC::kTcBM || raster == 1 || stages * stage_bytes < 128 * (bn + 4) * 4))
                     continue;
                 nnjit_candidate c = blank();
                 c.family = NNJIT_FAMILY_TC;
-                c.bm = BM; c.bn = bn; c.bk = BK;
+                c.bm = BM; c.bn = bn; c.bk = BK * kg;
                 c.tm = 0; c.tn = 0;
                 c.stages = stages;
                 c.split_k = split;
@@ -106,12 +111,15 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 const int64_t waves = ceil_div(work, std::min(work, slots));
                 c.grid = (int32_t)grid;
                 c.wave_eff_ppm = (int32_t)(work * 1000000 / (waves * std::min(work, slots)));
-                // per k-block: one MMA instruction costs about as much as N = 256 (the
-                // tensor core works on all 256 columns at once), so the MMA clocks are
-                // those of BN = 256, against the operand feed (stage bytes over the per-SM
+                // per k-block (4 MMA instructions): the slowest of the tensor pipe (an
+                // instruction takes kMmaN256Clk * N / 256, at least a quarter of that),
+                // the issuing thread (kMmaIssueClk per instruction plus one barrier wait
+                // and commit per ring slot) and the operand feed (bytes over the per-SM
                 // L2 feed)
-                const int64_t t_kb = std::max<int64_t>(2 * 256 * BM / MC::kTcBM,
-                                                       ceil_div(stage_bytes, MC::kFeedBytesPerClk));
+                const int64_t t_tensor = 4LL * std::max(MC::kMmaN256Clk / 4, MC::kMmaN256Clk * bn / 256);
+                const int64_t t_issue = 4LL * MC::kMmaIssueClk + MC::kSlotSyncClk / kg;
+                const int64_t t_kb = std::max(std::max(t_tensor, t_issue),
+                                              ceil_div(kb_bytes, MC::kFeedBytesPerClk));
                 int64_t cost = waves * t_kb * ceil_div(num_kb, split);
                 if (split > 1 && reduce == 0)
                     cost += MC::kLaunchClk +
@@ -119,7 +127,7 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 if (split > 1 && reduce == 1)
                     cost += waves * (128LL * bn * 4 / MC::kFeedBytesPerClk);  // DSMEM reduction
                 c.predicted_cost = cost;
-                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM, 0);
+                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM, 0, kg);
                 v.push_back(c);
                 // Multicast pair of the same tile: for full waves of 128 x 256 tiles, two
                 // CTAs of a cluster take vertically adjacent tiles and share each B tile,
@@ -369,10 +377,15 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 
 }  // namespace
 
-int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast) {
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast, int kg) {
     const int bi = bn == 64 ? 0 : bn == 128 ? 1 : bn == 256 ? 2 : -1;
     if (bi < 0 || (bm != 64 && bm != 128) || (bm == 64 && cluster)) return -1;
     const int di = dtype == NNJIT_BF16 ? 0 : 1;
+    if (kg == 2) {
+        if (bm != 128 || cluster || mcast || bn > 128) return -1;
+        return 40 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 2 + bi;
+    }
+    if (kg != 1) return -1;
     if (mcast) return (bn == 256 && bm == 128 && !cluster) ? 36 + di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0) : -1;
     const int variant = bm == 64 ? 2 : cluster ? 1 : 0;
     return variant * 12 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;

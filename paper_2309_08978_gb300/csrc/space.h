@@ -33,12 +33,15 @@ struct ModelConstants {
     static constexpr int kHbmBytesPerClk = 3500;     // chip-wide HBM bytes per SM clock
     static constexpr int kLaunchClk = 2000;          // cost of one extra kernel launch
     static constexpr int kRegRelaxPct = 50;          // Table 1 register formula covers half
-    static constexpr int kTcRegsPerThread = 72;      // tcgen05 kernel: ptxas reports 64-65, allocated in 8s
+    static constexpr int kTcRegsPerThread = 80;      // tcgen05 kernel: ptxas reports 72-80
     static constexpr int kTcThreads = 192;           // 6 warps: TMA, MMA, 4 x epilogue
     static constexpr int kTcBM = 128;
     static constexpr int kTcFixedSmem = 1024 + 256 + 32768;  // alignment slack, barriers,
                                                               // epilogue staging buffers
     static constexpr int kTcMaxStages = 8;
+    static constexpr int kMmaN256Clk = 128;           // tensor pipe: one M = 128, N = 256 MMA
+    static constexpr int kMmaIssueClk = 57;           // issuing thread: one tcgen05.mma
+    static constexpr int kSlotSyncClk = 226;          // issuing thread: ring-slot wait + commit
     static constexpr int kGemvMaxM = 8;
     static constexpr int kGemvMaxSmem = 64 * 1024;
     static constexpr int kGemvTmaKc = 256;           // K elements per TMA GEMV ring stage
@@ -57,7 +60,8 @@ nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
 
 // Precompiled-instance index helpers (kept in one place so the registry and the space
 // agree).
-int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast);  // 0..39
+// kg: k-blocks per ring slot (2 only for 128-row persistent tiles with BN <= 128)
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast, int kg = 1);  // 0..47
 int ffma_instance(int tm, int bm, int bn, int bk, int b_layout);  // 0..23, -1 if none
 int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if none
 // TMA-fed GEMV (B as [N][K]): rows per stage 8/16/32, M <= maxm (1 or 8).

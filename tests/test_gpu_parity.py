@@ -182,7 +182,11 @@ def test_constant_b_flag_is_exact(case):
                         flags=nj.NNJIT_PLAN_B_CONSTANT | nj.NNJIT_PLAN_NO_CACHE)
     lim = nj.nnjit_device_limits_query(0)
     cands, _ = nj.nnjit_space_enumerate(desc, lim)
-    for i in range(min(len(cands), 6)):
+    # the first few candidates, plus every tensor-core one with two k-blocks per ring slot
+    # (whose preloaded B tiles are grouped two to a barrier)
+    picks = sorted(set(range(min(len(cands), 6))) |
+                   {i for i, c in enumerate(cands) if c["family"] == nj.NNJIT_FAMILY_TC and c["instance"] >= 40})
+    for i in picks:
         with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
             C = run_plan(plan, A, B, bias, M, N)
         compare(C, A, B, bias, layout, dtype, exact=True)
