@@ -31,7 +31,7 @@ FEED_BYTES_PER_CLK = 64       # per-SM L2 -> SM operand feed
 HBM_BYTES_PER_CLK = 3500      # chip-wide HBM bytes per SM clock
 LAUNCH_CLK = 2000             # one extra kernel launch
 REG_SHARE_PCT = 50            # Table 1's Reg_thread is this share of a thread's registers
-TC_REGS = 80                  # registers per thread of the tensor-core kernel (ptxas: 72-80)
+TC_REGS = 176                 # registers per thread of the tensor-core kernel (ptxas: 72-173)
 TC_THREADS = 192
 TC_BM = 128
 TC_FIXED_SMEM = 1024 + 256 + 32768   # alignment slack, barriers, epilogue staging
@@ -223,7 +223,8 @@ def _tc(p, lim):
         # 64-row tiles only where 128-row tiles would leave SMs idle
         if bm == 64 and p.batch * cdiv(M, TC_BM) * cdiv(N, bn) >= lim["sm_count"]:
             continue
-        # two k-blocks per ring slot only where the MMA issue path is the bottleneck
+        # two k-blocks per ring slot where the MMA issue path, not the tensor pipe, sets
+        # the pace: 128-row tiles with BN <= 128
         if kg == 2 and (bm != TC_BM or bn > 128):
             continue
         kb_bytes = (bm + bn) * 128
@@ -276,10 +277,10 @@ def _tc(p, lim):
                         pairs = p.batch * cdiv(tiles_m, 2) * tiles_n
                         live = min(pairs, max(1, slots // 2))
                         pw = cdiv(pairs, live)
-                        feed = cdiv(stage - bn * 128 // 2, FEED_BYTES_PER_CLK)
+                        feed = cdiv(kb_bytes - bn * 128 // 2, FEED_BYTES_PER_CLK)
                         m.update(cluster_m=2, grid=2 * live, wave_eff_ppm=pairs * 1000000 // (pw * live),
-                                 predicted_cost=pw * max(2 * 256, feed) * num_kb,
-                                 instance=tc_instance(p.dtype, p.b_layout, bn, 0, bm, True))
+                                 predicted_cost=pw * max(t_tensor, t_issue, feed) * num_kb,
+                                 instance=tc_instance(p.dtype, p.b_layout, bn, 0, bm, True, kg))
                         out.append(m)
     return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2 * 2
 

@@ -106,7 +106,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     constexpr bool kCluster = kMode == kModeClusterSplitK;
     constexpr bool kMcast = kMode == kModeMcastPair;
     static_assert(BM == 128 || (BM == 64 && kMode == kModePersistent), "BM 64 tiles run persistent only");
-    static_assert(KG == 1 || (KG == 2 && kMode == kModePersistent), "k-block groups run persistent only");
+    static_assert(KG == 1 || (KG == 2 && kMode == kModePersistent && BN <= 128),
+                  "k-block groups: persistent tiles with BN <= 128");
     // Rows of the accumulator per epilogue warp.  An M = 128 MMA puts row r in TMEM lane
     // r; an M = 64 MMA puts rows 16q .. 16q+15 in lanes 32q .. 32q+15 of sub-partition q.
     constexpr int kRowsPerWarp = BM / 4;
@@ -391,25 +392,19 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                                  ? p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc
                                  : p.ws + ((long long)tc.s * p.batch + tc.b) * MN + (long long)row * p.N;
             const int zc = p.split == 1 ? tc.b : tc.s * p.batch + tc.b;
-#pragma unroll 1
-            for (int c = 0; c < BN / 32; ++c) {
-                uint32_t r[32];
-                const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN + c * 32;
-                ptx::tmem_ld32(taddr, r);
-                ptx::tmem_wait_ld(r);
-                if (c == BN / 32 - 1) {
-                    // the accumulator is in registers: hand TMEM back to the MMA warp
-                    ptx::tc_fence_before();
-                    ptx::mbar_arrive(tempty_bar(acc));
-                }
+            const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN;
+            constexpr int kChunks = BN / 32;
+            static_assert(kChunks % 2 == 0, "chunks are processed in pairs");
+            // One 32-column chunk: bias (lane j fetched column j; broadcast by shuffles),
+            // then the staged TMA store or the direct stores.
+            auto emit = [&](const uint32_t (&r)[32], float bl, int c) {
                 const int col0 = tc.tn * BN + c * 32;
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
                 if (bias) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        if (col0 + j < p.N) v[j] += __ldg(bias + col0 + j);
+                    for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
                 }
                 if (p.tma_store) {
                     uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
@@ -440,6 +435,34 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                             if (col0 + j < p.N) dst[j] = v[j];
                     }
                 }
+            };
+            auto bias_of = [&](int c) {
+                const int col = tc.tn * BN + c * 32 + lane;
+                return (bias && col < p.N) ? __ldg(bias + col) : 0.0f;
+            };
+            // The load of chunk c + 1 (TMEM and bias) is in flight while chunk c is stored;
+            // TMEM goes back to the MMA warp as soon as its last chunk is in registers.
+            auto release = [&]() {
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(tempty_bar(acc));
+            };
+            uint32_t ra[32], rb[32];
+            ptx::tmem_ld32(tbase, ra);
+            float ba = bias_of(0), bb = 0.0f;
+            ptx::tmem_wait_ld(ra);
+#pragma unroll 1
+            for (int c = 0; c < kChunks; c += 2) {
+                ptx::tmem_ld32(tbase + (c + 1) * 32, rb);
+                bb = bias_of(c + 1);
+                emit(ra, ba, c);
+                ptx::tmem_wait_ld(rb);
+                if (c + 2 == kChunks) release();
+                if (c + 2 < kChunks) {
+                    ptx::tmem_ld32(tbase + (c + 2) * 32, ra);
+                    ba = bias_of(c + 2);
+                }
+                emit(rb, bb, c + 1);
+                if (c + 2 < kChunks) ptx::tmem_wait_ld(ra);
             }
         }
         // the shared-memory sources must outlive the stores; the global writes complete
@@ -524,8 +547,9 @@ using TcKernel = void (*)(TcParams);
 // Instance table, indexed as tc_instance(): variant * 12 + (dtype_i * 2 + kn) * 3 + bn_i
 // for variant 0 = 128-row persistent, 1 = 128-row cluster split-K, 2 = 64-row persistent;
 // then 36 + dtype_i * 2 + kn for the 128 x 256 multicast pairs; then
-// 40 + (dtype_i * 2 + kn) * 2 + (BN == 128) for 128-row persistent tiles with two k-blocks
-// per ring slot.
+// 40 + (dtype_i * 2 + kn) * 2 + bn_i for 128-row persistent tiles with BN = 64, 128 and
+// two k-blocks per ring slot.  (With BN = 256 the tensor pipe, not the issue path, sets
+// the pace, and halving the number of slots only shortens the lookahead.)
 constexpr int kNumTcInstances = 48;
 #define NNJIT_TC_ROW(K, MN, MODE, BM)                                                  \
     tc_gemm_kernel<K, MN, 64, MODE, BM, 1>, tc_gemm_kernel<K, MN, 128, MODE, BM, 1>, \
@@ -658,7 +682,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     const int bk = 128 / p.elem_bytes();      // K elements per k-block
     if ((c.instance >= 24 && c.instance < 36) != (c.bm == 64) || (c.bm != 64 && c.bm != 128))
         return cudaErrorInvalidValue;
-    if (c.bk != bk * kg || (kg == 2 && (c.bm != 128 || c.bn > 128 || c.split_k < 1 || c.reduce != 0)))
+    if (c.bk != bk * kg || (kg == 2 && (c.bm != 128 || c.bn > 128 || c.reduce != 0)))
         return cudaErrorInvalidValue;
     if (mcast != (c.cluster_m == 2) || (mcast && (c.bn != 256 || c.split_k != 1 || c.grid < 2 || (c.grid & 1))))
         return cudaErrorInvalidValue;

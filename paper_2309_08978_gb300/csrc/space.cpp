@@ -65,7 +65,8 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
     for (int kg : {1, 2}) {
         if (bn > 64 && bn > pow2_ceil(N)) continue;  // no tile wider than the padded N
         if (BM == 64 && p.batch * ceil_div(M, MC::kTcBM) * ceil_div(N, bn) >= L.sm_count) continue;
-        // two k-blocks per ring slot only where the MMA issue path is the bottleneck
+        // two k-blocks per ring slot where the MMA issue path, not the tensor pipe, sets
+        // the pace: 128-row tiles with BN <= 128
         if (kg == 2 && (BM != MC::kTcBM || bn > 128)) continue;
         const int kb_bytes = (BM + bn) * 128;
         const int stage_bytes = kg * kb_bytes;
@@ -141,9 +142,9 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                     const int64_t pwaves = ceil_div(pairs, live_pairs);
                     m.grid = (int32_t)(2 * live_pairs);
                     m.wave_eff_ppm = (int32_t)(pairs * 1000000 / (pwaves * live_pairs));
-                    const int64_t feed = ceil_div(stage_bytes - bn * 128 / 2, MC::kFeedBytesPerClk);
-                    m.predicted_cost = pwaves * std::max<int64_t>(2 * 256, feed) * num_kb;
-                    m.instance = tc_instance(p.dtype, p.b_layout, bn, 0, BM, 1);
+                    const int64_t feed = ceil_div(kb_bytes - bn * 128 / 2, MC::kFeedBytesPerClk);
+                    m.predicted_cost = pwaves * std::max(std::max(t_tensor, t_issue), feed) * num_kb;
+                    m.instance = tc_instance(p.dtype, p.b_layout, bn, 0, BM, 1, kg);
                     v.push_back(m);
                 }
             }

@@ -33,7 +33,7 @@ struct ModelConstants {
     static constexpr int kHbmBytesPerClk = 3500;     // chip-wide HBM bytes per SM clock
     static constexpr int kLaunchClk = 2000;          // cost of one extra kernel launch
     static constexpr int kRegRelaxPct = 50;          // Table 1 register formula covers half
-    static constexpr int kTcRegsPerThread = 80;      // tcgen05 kernel: ptxas reports 72-80
+    static constexpr int kTcRegsPerThread = 176;     // tcgen05 kernel: ptxas reports 72-173
     static constexpr int kTcThreads = 192;           // 6 warps: TMA, MMA, 4 x epilogue
     static constexpr int kTcBM = 128;
     static constexpr int kTcFixedSmem = 1024 + 256 + 32768;  // alignment slack, barriers,
