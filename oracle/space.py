@@ -36,6 +36,8 @@ TC_THREADS = 192
 TC_BM = 128
 TC_FIXED_SMEM = 1024 + 256 + 32768   # alignment slack, barriers, epilogue staging
 TC_MAX_STAGES = 8
+TC_PAIR_ACC_COLS = 512        # TMEM columns of the CTA-pair tile kernel (2 x 256)
+TC_PAIR_FIRST = 48            # instance ids of the CTA-pair tile kernel (bf16, tf32)
 MMA_N256_CLK = 128            # tensor pipe: one M = 128, N = 256 MMA instruction
 MMA_ISSUE_CLK = 57            # issuing thread: one tcgen05.mma
 SLOT_SYNC_CLK = 226           # issuing thread: one ring-slot barrier wait + commit
@@ -282,6 +284,31 @@ def _tc(p, lim):
                                  predicted_cost=pw * max(t_tensor, t_issue, feed) * num_kb,
                                  instance=tc_instance(p.dtype, p.b_layout, bn, 0, bm, True, kg))
                         out.append(m)
+    # 256 x 256 tiles on CTA pairs (tcgen05 cta_group::2), B as [N][K]: an SM receives its
+    # 128 rows of A and half of the B tile per k-block; one thread issues for both SMs
+    if p.b_layout == B_NK and M > TC_BM and lim["sm_count"] >= 2:
+        kb_bytes = (TC_BM + 128) * 128
+        stages = min(TC_MAX_STAGES, (lim["smem_per_block_optin"] - TC_FIXED_SMEM) // kb_bytes)
+        smem = stages * kb_bytes + TC_FIXED_SMEM
+        tmem = TC_PAIR_ACC_COLS
+        blk = block_core(lim, TC_REGS, TC_THREADS, smem, tmem)
+        tiles2_m, tiles_n = cdiv(M, 256), cdiv(N, 256)
+        pairs = p.batch * tiles2_m * tiles_n
+        if stages >= 2 and blk >= 1 and tmem <= lim["tmem_cols_per_sm"]:
+            for raster in (0, 1):
+                if raster == 1 and (tiles2_m == 1 or tiles_n == 1):
+                    continue
+                live = min(pairs, max(1, lim["sm_count"] * blk // 2))
+                waves = cdiv(pairs, live)
+                t_kb = max(4 * MMA_N256_CLK, 4 * MMA_ISSUE_CLK + SLOT_SYNC_CLK, cdiv(kb_bytes, FEED_BYTES_PER_CLK))
+                c = _blank()
+                c.update(family=FAMILY_TC, bm=256, bn=256, bk=bk, stages=stages, raster=raster,
+                         threads=TC_THREADS, smem_bytes=smem, tmem_cols=tmem, regs_per_thread=TC_REGS,
+                         blocks_per_sm=blk, cluster_m=2, grid=2 * live,
+                         wave_eff_ppm=pairs * 1000000 // (waves * live),
+                         predicted_cost=waves * t_kb * num_kb,
+                         instance=TC_PAIR_FIRST + (0 if p.dtype == BF16 else 1))
+                out.append(c)
     return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2 * 2
 
 

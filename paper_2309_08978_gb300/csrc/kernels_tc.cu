@@ -21,6 +21,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cstdint>
 #include <mutex>
 
@@ -614,7 +615,8 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
     {
         const cuuint64_t dims[3] = {(cuuint64_t)p.K, (cuuint64_t)p.M, (cuuint64_t)p.batch};
         const cuuint64_t strides[2] = {(cuuint64_t)(p.lda * e), (cuuint64_t)(p.stride_a * e)};
-        const cuuint32_t box[3] = {bk, (cuuint32_t)c.bm, 1};
+        // a CTA of a pair tile loads its own 128 rows
+        const cuuint32_t box[3] = {bk, (cuuint32_t)std::min(c.bm, 128), 1};
         CUresult r = enc(ta, dt, 3, const_cast<void*>(A), dims, strides, box, estr,
                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
@@ -662,7 +664,7 @@ cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, flo
     if ((reinterpret_cast<uintptr_t>(out) & 15) || (ld * 4) % 16 || (zs * 4) % 16) return cudaSuccess;
     const cuuint64_t dims[3] = {(cuuint64_t)p.N, (cuuint64_t)p.M, (cuuint64_t)nz};
     const cuuint64_t strides[2] = {(cuuint64_t)(ld * 4), (cuuint64_t)(zs * 4)};
-    const cuuint32_t box[3] = {32, (cuuint32_t)(c.bm / 4), 1};  // one epilogue warp's rows
+    const cuuint32_t box[3] = {32, (cuuint32_t)(std::min(c.bm, 128) / 4), 1};  // one epilogue warp's rows
     const cuuint32_t estr[3] = {1, 1, 1};
     CUresult r = enc(tc_map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, out, dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
@@ -674,6 +676,7 @@ cudaError_t encode_tc_output_map(const Problem& p, const nnjit_candidate& c, flo
 cudaError_t launch_tc(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
+    if (c.instance >= kTcPairFirstInstance && c.instance < kTcPairFirstInstance + 2) return launch_tc_pair(a);
     if (c.instance < 0 || c.instance >= kNumTcInstances || !a.tmap_a || !a.tmap_b)
         return cudaErrorInvalidValue;
     const bool cluster = c.instance >= 12 && c.instance < 24;

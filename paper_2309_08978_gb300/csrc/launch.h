@@ -51,6 +51,8 @@ struct LaunchArgs {
 cudaError_t launch_ffma(const LaunchArgs& a);
 cudaError_t launch_gemv(const LaunchArgs& a);
 cudaError_t launch_tc(const LaunchArgs& a);
+// CTA-pair (cta_group::2) tensor-core instances kTcPairFirstInstance.. (bf16, tf32).
+cudaError_t launch_tc_pair(const LaunchArgs& a);
 
 // C[b,m,n] = sum_{s < split} ws[s][b][m][n] (+ bias[n]), s ascending.
 cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, const float* bias,

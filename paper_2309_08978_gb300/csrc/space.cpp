@@ -150,6 +150,45 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
             }
         }
     }
+    // 256 x 256 tiles on CTA pairs (tcgen05 cta_group::2), B as [N][K]: an SM receives its
+    // 128 rows of A and half of the B tile per k-block (32 KB), one thread issues the MMAs
+    // of both SMs.  Unsplit, persistent over pair tiles.
+    if (p.b_layout == NNJIT_B_NK && M > MC::kTcBM && L.sm_count >= 2) {
+        const int kb_bytes = (MC::kTcBM + 128) * 128;
+        const int stages = std::min(MC::kTcMaxStages, (L.smem_per_block_optin - MC::kTcFixedSmem) / kb_bytes);
+        const int smem = stages * kb_bytes + MC::kTcFixedSmem;
+        const int tmem = MC::kTcPairAccCols;
+        const int blk = blocks_per_core(L, MC::kTcRegsPerThread, MC::kTcThreads, smem, tmem);
+        const int64_t tiles2_m = ceil_div(M, 256), tiles_n = ceil_div(N, 256);
+        const int64_t pairs = p.batch * tiles2_m * tiles_n;
+        if (stages >= 2 && blk >= 1 && tmem <= L.tmem_cols_per_sm) {
+            for (int raster = 0; raster < 2; ++raster) {
+                if (raster == 1 && (tiles2_m == 1 || tiles_n == 1)) continue;
+                nnjit_candidate c = blank();
+                c.family = NNJIT_FAMILY_TC;
+                c.bm = 256; c.bn = 256; c.bk = BK;
+                c.stages = stages;
+                c.raster = raster;
+                c.threads = MC::kTcThreads;
+                c.smem_bytes = smem;
+                c.tmem_cols = tmem;
+                c.regs_per_thread = MC::kTcRegsPerThread;
+                c.blocks_per_sm = blk;
+                c.cluster_m = 2;
+                const int64_t pair_slots = std::max<int64_t>(1, (int64_t)L.sm_count * blk / 2);
+                const int64_t live = std::min(pairs, pair_slots);
+                const int64_t waves = ceil_div(pairs, live);
+                c.grid = (int32_t)(2 * live);
+                c.wave_eff_ppm = (int32_t)(pairs * 1000000 / (waves * live));
+                const int64_t t_tensor = 4LL * MC::kMmaN256Clk;
+                const int64_t t_issue = 4LL * MC::kMmaIssueClk + MC::kSlotSyncClk;
+                const int64_t t_kb = std::max(std::max(t_tensor, t_issue), ceil_div(kb_bytes, MC::kFeedBytesPerClk));
+                c.predicted_cost = waves * t_kb * num_kb;
+                c.instance = kTcPairFirstInstance + (p.dtype == NNJIT_BF16 ? 0 : 1);
+                v.push_back(c);
+            }
+        }
+    }
 }
 
 // ---------------------------------------------------------------------------------

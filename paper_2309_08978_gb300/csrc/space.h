@@ -39,6 +39,7 @@ struct ModelConstants {
     static constexpr int kTcFixedSmem = 1024 + 256 + 32768;  // alignment slack, barriers,
                                                               // epilogue staging buffers
     static constexpr int kTcMaxStages = 8;
+    static constexpr int kTcPairAccCols = 512;        // TMEM columns of a CTA-pair tile kernel (2 x 256)
     static constexpr int kMmaN256Clk = 128;           // tensor pipe: one M = 128, N = 256 MMA
     static constexpr int kMmaIssueClk = 57;           // issuing thread: one tcgen05.mma
     static constexpr int kSlotSyncClk = 226;          // issuing thread: ring-slot wait + commit
@@ -62,6 +63,8 @@ nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
 // agree).
 // kg: k-blocks per ring slot (2 only for 128-row persistent tiles with BN <= 128)
 int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast, int kg = 1);  // 0..47
+// 256 x 256 tiles on CTA pairs (tcgen05 cta_group::2), B as [N][K]: 48 (bf16), 49 (tf32).
+constexpr int kTcPairFirstInstance = 48;
 int ffma_instance(int tm, int bm, int bn, int bk, int b_layout);  // 0..23, -1 if none
 int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if none
 // TMA-fed GEMV (B as [N][K]): rows per stage 8/16/32, M <= maxm (1 or 8).
