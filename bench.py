@@ -272,6 +272,21 @@ def cpu_baseline(workload, dtype, seconds=12.0):
 
 # ------------------------------------------------------------------------- our arm
 
+def custom_workload(ap, spec):
+    """A one-product workload from "MxNxK:dtype:layout" (weights-like B, no bias, the
+    default distributions), seeded with index 5."""
+    from synthetic import Shape, Workload
+    try:
+        dims, dtype, layout = spec.split(":")
+        M, N, K = (int(x) for x in dims.lower().split("x"))
+    except ValueError:
+        ap.error(f"--shape: expected MxNxK:dtype:layout, got {spec!r}")
+    if dtype not in ("f32_ffma", "tf32", "bf16") or layout not in ("NK", "KN") or min(M, N, K) < 1:
+        ap.error(f"--shape: bad dtype, layout or size in {spec!r}")
+    shape = Shape(f"{M}x{N}x{K}", M, N, K, 1, layout)
+    return Workload(f"custom_{M}x{N}x{K}_{dtype}_{layout}", 5, f"custom product {spec}", (dtype,), (shape,))
+
+
 def run_ours(args, workload, rank, world, local_rank):
     import numpy as np
     import torch
@@ -540,11 +555,16 @@ def main(argv=None):
                     help="plan-cache file: loaded before tuning if present, saved after")
     ap.add_argument("--only", default=None,
                     help="run a single product of the workload (by name), e.g. for profiling")
+    ap.add_argument("--shape", default=None,
+                    help="run one custom product instead of a workload: MxNxK:dtype:layout "
+                         "(dtype f32_ffma, tf32 or bf16; layout NK or KN), e.g. 4096x8192x4096:bf16:NK")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from synthetic import WORKLOADS
     workload = WORKLOADS[args.workload]
+    if args.shape:
+        workload = custom_workload(ap, args.shape)
     if args.only:
         import dataclasses
         shapes = tuple(s for s in workload.shapes if s.name == args.only)
