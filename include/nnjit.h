@@ -125,9 +125,13 @@ typedef struct {
  */
 typedef struct {
     int32_t family;          /* nnjit_family */
-    int32_t bm, bn, bk;      /* CTA tile */
+    int32_t bm, bn, bk;      /* CTA tile (TC: bm = 256 is a tile of a CTA pair; bk = K elements
+                                per ring slot, 2 k-blocks of 128 bytes when it is 256 bytes;
+                                GEMV: bm = M, bn = weight rows per CTA or stage, bk = K slice
+                                or K elements per ring stage) */
     int32_t tm, tn;          /* FFMA: thread tile; GEMV: tm = rows per warp */
-    int32_t stages;          /* TC: shared-memory ring depth; GEMV: loads in flight per row */
+    int32_t stages;          /* TC: shared-memory ring depth; GEMV: loads in flight per row,
+                                or ring stages of the TMA-fed kernels (instance >= 8) */
     int32_t split_k;         /* K slices reduced in a fixed order afterwards (1 = none) */
     int32_t raster;          /* TC tile order: 0 = M fastest, 1 = N fastest */
     int32_t threads;         /* threads per CTA */
@@ -142,8 +146,10 @@ typedef struct {
     int32_t reduce;          /* split-K reduction: 0 = partials in the plan's workspace, summed
                                 by a second kernel; 1 = TC only, inside a thread-block cluster
                                 of split_k CTAs through distributed shared memory */
-    int32_t cluster_m;       /* TC only: 2 = the two CTAs of a cluster take vertically adjacent
-                                tiles and share each B tile by TMA multicast; else 1 */
+    int32_t cluster_m;       /* TC only: 2 = a cluster of two CTAs; with bm = 128 they take
+                                vertically adjacent tiles and share each B tile by TMA
+                                multicast, with bm = 256 they compute one 256-row tile with
+                                tcgen05 cta_group::2 MMAs; else 1 */
 } nnjit_candidate;
 
 typedef struct nnjit_plan_s* nnjit_plan;
