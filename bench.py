@@ -187,6 +187,7 @@ def run_reference(args, workload, rank):
     oracle.build()
     dtype = workload.dtypes[-1]
     cores = oracle.hw_threads()
+    act = args.epilogue
     # one step = every product of the workload on a row sample of A (the oracle cost is
     # linear in the rows), sized to a few seconds of host work per step
     budget_s = float(os.environ.get("NNJIT_REF_STEP_S", "3.0"))
@@ -214,7 +215,7 @@ def run_reference(args, workload, rank):
             rows = max(1, int(round(s.M * frac)))
             Ar = A[:, :rows] if s.batch > 1 else A[:rows]
             oracle.matmul(np.ascontiguousarray(Ar), B, bias,
-                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores)
+                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores, act=act)
             fl += 2 * s.batch * rows * s.N * s.K
         dt = time.perf_counter() - t0
         if step >= args.warmup:
@@ -238,7 +239,7 @@ def run_reference(args, workload, rank):
     return 0
 
 
-def cpu_baseline(workload, dtype, seconds=12.0):
+def cpu_baseline(workload, dtype, seconds=12.0, act="none"):
     """Oracle throughput on the host cores on a bounded sample of the workload."""
     import numpy as np
     import oracle
@@ -256,7 +257,7 @@ def cpu_baseline(workload, dtype, seconds=12.0):
             rows = max(1, int(round(s.M * rows_frac)))
             Ar = A[:, :rows] if s.batch > 1 else A[:rows]
             oracle.matmul(np.ascontiguousarray(Ar), B, bias,
-                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores)
+                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores, act=act)
             fl += 2 * s.batch * rows * s.N * s.K
         dt = time.perf_counter() - t0
         done_flops += fl
@@ -325,7 +326,7 @@ def run_ours(args, workload, rank, world, local_rank):
         A, B, bias = make_operands(s, workload.index, dtype)
         bflag = nj.NNJIT_PLAN_B_CONSTANT if s.b_is_weight else 0   # weights never change
         desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
-                            has_bias=s.has_bias, flags=bflag)
+                            has_bias=s.has_bias, flags=bflag, epilogue=args.epilogue)
         t0 = time.perf_counter()
         plan = nj.nnjit_matmul_plan_ex(desc, args.budget_ms)
         plan_ms = 1000 * (time.perf_counter() - t0)
@@ -336,7 +337,7 @@ def run_ours(args, workload, rank, world, local_rank):
                  "candidate": {k: info["candidate"][k] for k in ("bm", "bn", "bk", "stages", "split_k", "raster")}}
         if not args.no_sweep:
             sweep_desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
-                                      has_bias=s.has_bias,
+                                      has_bias=s.has_bias, epilogue=args.epilogue,
                                       flags=nj.NNJIT_PLAN_EXHAUSTIVE | nj.NNJIT_PLAN_NO_CACHE | bflag)
             t0 = time.perf_counter()
             sweep = nj.nnjit_matmul_plan_ex(sweep_desc, 0.0)
@@ -505,7 +506,7 @@ def run_ours(args, workload, rank, world, local_rank):
 
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(workload, dtype, seconds=args.cpu_seconds)
+        cpu = cpu_baseline(workload, dtype, seconds=args.cpu_seconds, act=args.epilogue)
 
     l2_note = ("each product rotates over " + ", ".join(str(len(it["sets"])) for it in items) +
                f" operand copies (>= 3 x L2 = {3 * l2 / 2**20:.0f} MiB per product), so "
@@ -515,7 +516,7 @@ def run_ours(args, workload, rank, world, local_rank):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
         "data": "synthetic (seeded SplitMix64, the workload's distributions; no trained weights)",
-        "config": {"workload": workload.key, "title": workload.title,
+        "config": {"workload": workload.key, "title": workload.title, "epilogue": args.epilogue,
                    "shapes": [[s.batch, s.M, s.N, s.K, s.b_layout] for s in workload.shapes],
                    "parallelism": f"replicas{world}", "l2": l2_note,
                    "schedule": "per product: K launches as CUDA-graph replays, products in sequence"},
@@ -555,6 +556,8 @@ def main(argv=None):
                     help="plan-cache file: loaded before tuning if present, saved after")
     ap.add_argument("--only", default=None,
                     help="run a single product of the workload (by name), e.g. for profiling")
+    ap.add_argument("--epilogue", default="none", choices=["none", "relu", "gelu", "silu"],
+                    help="activation fused after the bias into every product (nnjit_epilogue)")
     ap.add_argument("--shape", default=None,
                     help="run one custom product instead of a workload: MxNxK:dtype:layout "
                          "(dtype f32_ffma, tf32 or bf16; layout NK or KN), e.g. 4096x8192x4096:bf16:NK")

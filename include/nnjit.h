@@ -67,6 +67,18 @@ typedef enum {
                             PyTorch Linear weight layout and K^T of attention QK^T. */
 } nnjit_blayout;
 
+/*
+ * Elementwise activation applied to every output after the bias, inside the kernel that
+ * writes C (the epilogue fusion of a Linear with its activation; in split-K plans the
+ * reduction applies it once the slices are summed):  C = act(A * Bt + bias).
+ */
+typedef enum {
+    NNJIT_EPI_NONE = 0,
+    NNJIT_EPI_RELU = 1,  /* max(x, 0) */
+    NNJIT_EPI_GELU = 2,  /* x * Phi(x) = 0.5 x (1 + erf(x / sqrt(2)))  (exact, erf form) */
+    NNJIT_EPI_SILU = 3   /* x * sigmoid(x) = x / (1 + exp(-x)) */
+} nnjit_epilogue;
+
 /* Kernel families of the lite space. */
 typedef enum {
     NNJIT_FAMILY_FFMA = 0,  /* register-tiled SIMT GEMM, exact FP32 */
@@ -100,6 +112,7 @@ typedef struct {
     int64_t stride_a, stride_b, stride_c;
     int32_t has_bias;     /* 1: run() takes a float32 bias[N] added to every row */
     uint32_t flags;       /* NNJIT_PLAN_* */
+    int32_t epilogue;     /* nnjit_epilogue, applied after the bias (0 = none) */
 } nnjit_matmul_desc;
 
 /*

@@ -8,8 +8,8 @@ written from the paper:
   * ``space``   -- the tile-based hardware-usage formulas and lite-space heuristics
     (Sec. 5.2, Table 1, Table 2) and the candidate evaluation order, restated in
     plain Python, plus the Blackwell readings of those rules used by the library.
-  * ``tuner``   -- the JIT selection rule (Sec. 3): keep the fastest measured
-    candidate; replace the current one only when the newcomer is faster.
+  * ``epilogue`` -- the activations a kernel may apply after the bias (textbook
+    definitions of ReLU, GELU and SiLU in FP64).
 
 Only tests/, ``__graft_entry__.smoke()`` and bench.py's CPU-baseline / reference legs
 may import this package.  The GPU library shares no code with it.

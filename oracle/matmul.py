@@ -91,11 +91,12 @@ def to_f64(x: np.ndarray) -> np.ndarray:
 
 
 def matmul(A: np.ndarray, B: np.ndarray, bias: np.ndarray | None = None,
-           b_layout: int = B_KN, nthreads: int = 0):
+           b_layout: int = B_KN, nthreads: int = 0, act: str = "none"):
     """Reference product.
 
     A: [M,K] or [batch,M,K]; B: [K,N] / [N,K] (KN / NK), optionally with a leading batch
-    dimension.  uint16 arrays are bf16 bit patterns.  bias: [N] or None.
+    dimension.  uint16 arrays are bf16 bit patterns.  bias: [N] or None.  act: an
+    activation of oracle.epilogue applied in FP64 after the bias (the fused epilogue).
     Returns (C64, C32): float64 and float32 arrays of shape [M,N] or [batch,M,N].
     """
     A64, B64 = to_f64(A), to_f64(B)
@@ -134,6 +135,9 @@ def matmul(A: np.ndarray, B: np.ndarray, bias: np.ndarray | None = None,
         raise RuntimeError(f"oracle_matmul_f64 failed with code {rc}")
     if squeeze:
         C = C[0]
+    if act != "none":
+        from .epilogue import apply
+        C = apply(C, act)
     return C, C.astype(np.float32)
 
 
@@ -148,8 +152,8 @@ def rel_fro(C_test: np.ndarray, C_ref64: np.ndarray) -> float:
 
 
 def matmul_rows(A: np.ndarray, B: np.ndarray, bias, b_layout: int, rows,
-                nthreads: int = 0):
+                nthreads: int = 0, act: str = "none"):
     """Reference values for a subset of output rows (one full row each) of a single
     (non-batched) product: the oracle run on A[rows]."""
     rows = np.asarray(rows, dtype=np.int64)
-    return matmul(np.ascontiguousarray(A[rows]), B, bias, b_layout, nthreads)
+    return matmul(np.ascontiguousarray(A[rows]), B, bias, b_layout, nthreads, act)

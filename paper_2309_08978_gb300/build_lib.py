@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 CUDA_SOURCES = ["capi.cu", "kernels_tc.cu", "kernels_tc2.cu", "kernels_gemv.cu", "kernels_gemv_tma.cu", "kernels_ffma.cu",
                 "kernels_ffma_kn.cu", "kernels_ffma_nk.cu", "noalloc.cu"]
 CXX_SOURCES = ["space.cpp"]
-HEADERS = ["space.h", "launch.h", "ptx.cuh", "ffma.cuh"]
+HEADERS = ["space.h", "launch.h", "ptx.cuh", "ffma.cuh", "epilogue.cuh"]
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 

@@ -184,7 +184,9 @@ std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L) {
                   p.b_layout, (long long)p.lda, (long long)p.ldb, (long long)p.ldc,
                   (long long)p.stride_a, (long long)p.stride_b, (long long)p.stride_c, p.has_bias,
                   name.c_str(), L.cc_major, L.cc_minor, L.sm_count);
-    return buf;
+    std::string key = buf;
+    if (p.epilogue != NNJIT_EPI_NONE) key += "|ep=" + std::to_string(p.epilogue);
+    return key;
 }
 
 // Split-K partials go to a workspace unless they are reduced inside a cluster.

@@ -9,6 +9,8 @@
 
 #include <cstdint>
 
+#include "epilogue.cuh"
+
 namespace nnjit {
 
 struct FfmaParams {
@@ -18,6 +20,7 @@ struct FfmaParams {
     float* C;
     float* ws;
     int M, N, K, batch, split, kper;
+    int act;            // nnjit_epilogue, applied when split == 1
     long long lda, ldb, ldc, stride_a, stride_b, stride_c;
 };
 
@@ -135,7 +138,10 @@ __global__ void __launch_bounds__((BM / TM) * (BN / TN))
 #pragma unroll
         for (int j = 0; j < TN; ++j) {
             const int gn = n0 + tx * TN + j;
-            if (gn < p.N) dst[gn] = bias ? acc[i][j] + __ldg(bias + gn) : acc[i][j];
+            if (gn < p.N) {
+                const float v = bias ? acc[i][j] + __ldg(bias + gn) : acc[i][j];
+                dst[gn] = p.split == 1 ? apply_act(v, p.act) : v;
+            }
         }
     }
 }

@@ -19,6 +19,7 @@ cudaError_t launch_ffma(const LaunchArgs& a) {
     prm.A = static_cast<const float*>(a.A);
     prm.B = static_cast<const float*>(a.B);
     prm.bias = a.bias;
+    prm.act = p.epilogue;
     prm.C = a.C;
     prm.ws = a.ws;
     prm.M = (int)p.M; prm.N = (int)p.N; prm.K = (int)p.K; prm.batch = (int)p.batch;

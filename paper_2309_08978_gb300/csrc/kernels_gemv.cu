@@ -13,6 +13,7 @@
 #include <algorithm>
 #include <mutex>
 
+#include "epilogue.cuh"
 #include "launch.h"
 #include "ptx.cuh"
 
@@ -31,6 +32,7 @@ struct GemvParams {
     int M, N, K, split, kper;
     int vec_ok;          // KN: rows of W are 16-byte aligned (ldb % 8 == 0)
     int b_const;         // W is not written by kernels launched before this one
+    int act;             // nnjit_epilogue, applied when split == 1
     long long lda, ldb, ldc;
 };
 
@@ -167,7 +169,7 @@ __global__ void __launch_bounds__(256) gemv_nk_kernel(const GemvParams p) {
                 for (int m = 0; m < kMaxM; ++m) {
                     if (m >= M) continue;
                     if (p.split == 1)
-                        p.C[(long long)m * p.ldc + n] = p.bias ? acc[r][m] + p.bias[n] : acc[r][m];
+                        p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act);
                     else
                         p.ws[((long long)s * M + m) * p.N + n] = acc[r][m];
                 }
@@ -242,7 +244,7 @@ __global__ void __launch_bounds__(256) gemv_kn_kernel(const GemvParams p) {
         float v = 0.0f;
         for (int w = 0; w < warps; ++w) v += red[((long long)w * M + m) * 256 + col];
         if (p.split == 1)
-            p.C[(long long)m * p.ldc + n] = p.bias ? v + p.bias[n] : v;
+            p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? v + p.bias[n] : v, p.act);
         else
             p.ws[((long long)s * M + m) * p.N + n] = v;
     }
@@ -260,7 +262,7 @@ int g_gemv_smem[8] = {0};
 
 __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, long long batch_mn,
                                      int M, int N, long long ldc, long long stride_c,
-                                     const float* __restrict__ bias, float* __restrict__ C) {
+                                     const float* __restrict__ bias, int act, float* __restrict__ C) {
     ptx::griddep_wait();
     if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const long long mn = (long long)M * N;
@@ -272,12 +274,12 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, lo
         const long long r = i % mn;
         const int m = (int)(r / N), n = (int)(r % N);
         if (bias) v += bias[n];
-        C[b * stride_c + (long long)m * ldc + n] = v;
+        C[b * stride_c + (long long)m * ldc + n] = apply_act(v, act);
     }
 }
 
 __global__ void fill_bias_kernel(long long total, int M, int N, long long ldc, long long stride_c,
-                                 const float* __restrict__ bias, float* __restrict__ C) {
+                                 const float* __restrict__ bias, int act, float* __restrict__ C) {
     ptx::griddep_wait();
     if (threadIdx.x == 0) ptx::griddep_launch_dependents();
     const long long mn = (long long)M * N;
@@ -285,7 +287,7 @@ __global__ void fill_bias_kernel(long long total, int M, int N, long long ldc, l
          i += (long long)gridDim.x * blockDim.x) {
         const long long b = i / mn, r = i % mn;
         const int m = (int)(r / N), n = (int)(r % N);
-        C[b * stride_c + (long long)m * ldc + n] = bias ? bias[n] : 0.0f;
+        C[b * stride_c + (long long)m * ldc + n] = apply_act(bias ? bias[n] : 0.0f, act);
     }
 }
 
@@ -350,6 +352,7 @@ cudaError_t launch_gemv(const LaunchArgs& a) {
     prm.lda = p.lda; prm.ldb = p.ldb; prm.ldc = p.ldc;
     prm.vec_ok = (p.ldb % 8 == 0 && (reinterpret_cast<uintptr_t>(a.B) & 15) == 0) ? 1 : 0;
     prm.b_const = (p.flags & NNJIT_PLAN_B_CONSTANT) ? 1 : 0;
+    prm.act = prm.split == 1 ? p.epilogue : NNJIT_EPI_NONE;
     const int warps = c.threads / 32;
     dim3 grid;
     int smem;
@@ -373,14 +376,14 @@ cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, c
     const long long n = p.batch * p.M * p.N;
     if (n == 0) return cudaSuccess;
     return launch_pdl(splitk_reduce_kernel, dim3(grid_for(n, 256)), dim3(256), 0, s, ws, split, n,
-                      (int)p.M, (int)p.N, p.ldc, p.stride_c, bias, C);
+                      (int)p.M, (int)p.N, p.ldc, p.stride_c, bias, p.epilogue, C);
 }
 
 cudaError_t launch_fill_bias(const Problem& p, const float* bias, float* C, cudaStream_t s) {
     const long long n = p.batch * p.M * p.N;
     if (n == 0) return cudaSuccess;
     return launch_pdl(fill_bias_kernel, dim3(grid_for(n, 256)), dim3(256), 0, s, n, (int)p.M,
-                      (int)p.N, p.ldc, p.stride_c, bias, C);
+                      (int)p.N, p.ldc, p.stride_c, bias, p.epilogue, C);
 }
 
 cudaError_t launch_fill_scratch(void* dst, int64_t n_elems, int elem_bytes, uint32_t seed,

@@ -22,6 +22,7 @@
 #include <cstdint>
 #include <mutex>
 
+#include "epilogue.cuh"
 #include "launch.h"
 #include "ptx.cuh"
 
@@ -53,6 +54,7 @@ struct GemvTmaParams {
     int stages;
     int b_const;         // W is not written by kernels launched earlier in the stream
     int pf_chunks;       // b_const: chunks of the first item past the ring to prefetch into L2
+    int act;             // nnjit_epilogue, applied when split == 1
     long long ldc;
 };
 
@@ -250,7 +252,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
                 for (int m = 0; m < MAXM; ++m) {
                     if (m >= M) continue;
                     if (p.split == 1)
-                        p.C[(long long)m * p.ldc + n] = p.bias ? acc[r][m] + p.bias[n] : acc[r][m];
+                        p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act);
                     else
                         p.ws[((long long)w.s * M + m) * p.N + n] = acc[r][m];
                 }
@@ -347,6 +349,7 @@ cudaError_t launch_gemv_tma(const LaunchArgs& a) {
     prm.stages = c.stages;
     prm.b_const = (p.flags & NNJIT_PLAN_B_CONSTANT) ? 1 : 0;
     prm.ldc = p.ldc;
+    prm.act = c.split_k == 1 ? p.epilogue : NNJIT_EPI_NONE;
     const int grid = (int)std::min<long long>(items, std::max(1, c.grid));
     // L2 prefetch ahead of the dependency wait: at most kPrefetchBytes over the grid
     // (well under the 129 MB L2, which the previous kernel is also streaming through).

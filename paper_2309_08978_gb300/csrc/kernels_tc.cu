@@ -25,6 +25,7 @@
 #include <cstdint>
 #include <mutex>
 
+#include "epilogue.cuh"
 #include "launch.h"
 #include "ptx.cuh"
 
@@ -49,6 +50,7 @@ struct TcParams {
     int M, N, K, batch;
     long long ldc, stride_c;
     int num_kb, split, tiles_m, tiles_n, total_tiles, stages, raster;
+    int act;             // nnjit_epilogue, applied where C is written (not to partials)
 };
 
 struct TileCoord {
@@ -389,6 +391,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
             const int row = tc.tm * BM + row_in_tile;
             const float* bias = p.split == 1 ? p.bias : nullptr;
+            const int act = p.split == 1 ? p.act : NNJIT_EPI_NONE;  // partials stay raw
             float* dst_row = p.split == 1
                                  ? p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc
                                  : p.ws + ((long long)tc.s * p.batch + tc.b) * MN + (long long)row * p.N;
@@ -407,6 +410,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
                 }
+                apply_act32(v, act);
                 if (p.tma_store) {
                     uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
                     if (lane == 0) ptx::bulk_wait_read<1>();  // the store that used buf is done
@@ -523,14 +527,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             float o[4] = {a.x, a.y, a.z, a.w};
             float* dst = Cb + (long long)row * p.ldc + col;
             if (col + 4 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
-                if (p.bias) {
 #pragma unroll
-                    for (int j = 0; j < 4; ++j) o[j] += __ldg(p.bias + col + j);
-                }
+                for (int j = 0; j < 4; ++j) o[j] = apply_act(p.bias ? o[j] + __ldg(p.bias + col + j) : o[j], p.act);
                 *reinterpret_cast<float4*>(dst) = make_float4(o[0], o[1], o[2], o[3]);
             } else {
                 for (int j = 0; j < 4 && col + j < p.N; ++j)
-                    dst[j] = p.bias ? o[j] + __ldg(p.bias + col + j) : o[j];
+                    dst[j] = apply_act(p.bias ? o[j] + __ldg(p.bias + col + j) : o[j], p.act);
             }
         }
     }
@@ -701,6 +703,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     if (a.tmap_c) prm.tmap_c = *a.tmap_c;
     prm.C = a.C;
     prm.bias = a.bias;
+    prm.act = p.epilogue;
     prm.ws = a.ws;
     prm.err = a.err;
     prm.M = (int)p.M;

@@ -27,6 +27,7 @@
 #include <cstdint>
 #include <mutex>
 
+#include "epilogue.cuh"
 #include "launch.h"
 #include "ptx.cuh"
 
@@ -57,6 +58,7 @@ struct Tc2Params {
     int M, N, K, batch;
     long long ldc, stride_c;
     int num_kb, tiles2_m, tiles_n, total, stages, raster;
+    int act;  // nnjit_epilogue
 };
 
 struct PairTile {
@@ -293,6 +295,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
                 }
+                apply_act32(v, p.act);
                 if (p.tma_store) {
                     uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
                     if (lane == 0) ptx::bulk_wait_read<1>();
@@ -389,6 +392,7 @@ cudaError_t launch_tc_pair(const LaunchArgs& a) {
     prm.b_const = (p.flags & NNJIT_PLAN_B_CONSTANT) ? 1 : 0;
     prm.C = a.C;
     prm.bias = a.bias;
+    prm.act = p.epilogue;
     prm.err = a.err;
     prm.M = (int)p.M;
     prm.N = (int)p.N;

@@ -23,6 +23,7 @@ struct Problem {
     int64_t stride_a = 0, stride_b = 0, stride_c = 0;
     int has_bias = 0;
     uint32_t flags = 0;
+    int epilogue = NNJIT_EPI_NONE;
     int elem_bytes() const { return dtype == NNJIT_BF16 ? 2 : 4; }
     bool degenerate() const { return M == 0 || N == 0 || K == 0; }
 };

@@ -26,6 +26,11 @@ NNJIT_F32_FFMA = 0
 NNJIT_TF32 = 1
 NNJIT_BF16 = 2
 
+NNJIT_EPI_NONE = 0
+NNJIT_EPI_RELU = 1
+NNJIT_EPI_GELU = 2
+NNJIT_EPI_SILU = 3
+
 NNJIT_B_KN = 0
 NNJIT_B_NK = 1
 
@@ -48,7 +53,7 @@ class nnjit_matmul_desc(ctypes.Structure):
                 ("lda", ctypes.c_int64), ("ldb", ctypes.c_int64), ("ldc", ctypes.c_int64),
                 ("stride_a", ctypes.c_int64), ("stride_b", ctypes.c_int64),
                 ("stride_c", ctypes.c_int64), ("has_bias", ctypes.c_int32),
-                ("flags", ctypes.c_uint32)]
+                ("flags", ctypes.c_uint32), ("epilogue", ctypes.c_int32)]
 
 
 class nnjit_device_limits(ctypes.Structure):
@@ -179,8 +184,11 @@ def nnjit_device_limits_query(device: int = 0) -> nnjit_device_limits:
     return out
 
 
+EPILOGUES = {"none": 0, "relu": 1, "gelu": 2, "silu": 3}
+
+
 def make_desc(M, N, K, dtype, b_layout="KN", batch=1, has_bias=False, flags=0, lda=0, ldb=0,
-              ldc=0, stride_a=0, stride_b=0, stride_c=0) -> nnjit_matmul_desc:
+              ldc=0, stride_a=0, stride_b=0, stride_c=0, epilogue="none") -> nnjit_matmul_desc:
     d = nnjit_matmul_desc()
     d.M, d.N, d.K, d.batch = M, N, K, batch
     d.dtype = DTYPES[dtype] if isinstance(dtype, str) else dtype
@@ -189,6 +197,7 @@ def make_desc(M, N, K, dtype, b_layout="KN", batch=1, has_bias=False, flags=0, l
     d.stride_a, d.stride_b, d.stride_c = stride_a, stride_b, stride_c
     d.has_bias = 1 if has_bias else 0
     d.flags = flags
+    d.epilogue = EPILOGUES[epilogue] if isinstance(epilogue, str) else epilogue
     return d
 
 

@@ -296,3 +296,64 @@ def test_multicast_pairs_exact(case):
             with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
                 C = run_plan(plan, A, B, bias, M, N)
             compare(C, A, B, bias, layout, dtype, exact=True)
+
+
+EPI_CASES = [("f32_ffma", 64, 768, 768, "KN"), ("tf32", 200, 300, 520, "NK"),
+             ("bf16", 300, 520, 1040, "NK"), ("bf16", 200, 600, 520, "KN"),
+             ("bf16", 1, 4096, 4096, "NK"), ("bf16", 3, 1000, 2056, "NK"), ("bf16", 4, 1000, 2048, "KN")]
+
+
+@pytest.mark.parametrize("case", EPI_CASES, ids=_ids)
+def test_fused_activation_every_candidate(case):
+    """C = act(A.B + bias) written by the kernel that writes C (split-K plans: by the
+    reduction).  Every candidate of the space runs -- split-K reduces, cluster reduces,
+    CTA pairs, TMA-fed GEMVs.  ReLU on integer inputs must be exact; GELU on random
+    inputs stays within the dtype's tolerance; SiLU runs on the top-ranked plan."""
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    Ai, Bi, biasi = make_operands(shape, 30, dtype, ints=True)
+    Ar, Br, biasr = make_operands(shape, 31, dtype)
+    lim = nj.nnjit_device_limits_query(0)
+    for act in ("relu", "gelu"):
+        desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, epilogue=act,
+                            flags=nj.NNJIT_PLAN_NO_CACHE)
+        cands, _ = nj.nnjit_space_enumerate(desc, lim)
+        for i, c in enumerate(cands):
+            with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+                if act == "relu":
+                    C = run_plan(plan, Ai, Bi, biasi, M, N)
+                else:
+                    C = run_plan(plan, Ar, Br, biasr, M, N)
+            try:
+                if act == "relu":
+                    compare(C, Ai, Bi, biasi, layout, dtype, exact=True, act=act)
+                else:
+                    compare(C, Ar, Br, biasr, layout, dtype, act=act)
+            except AssertionError as e:
+                raise AssertionError(f"{act} candidate {i} {c}: {e}") from None
+    desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, epilogue="silu",
+                        flags=nj.NNJIT_PLAN_NO_CACHE)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        C = run_plan(plan, Ar, Br, biasr, M, N)
+    compare(C, Ar, Br, biasr, layout, dtype, act="silu")
+
+
+@pytest.mark.parametrize("act", ["relu", "gelu", "silu"])
+def test_fused_activation_k0_applies_to_bias(act):
+    """K = 0: C = act(bias) on every row.  The kernels evaluate GELU with the erf of
+    Abramowitz & Stegun 7.1.26 (|error| <= 1.5e-7) and SiLU with the hardware exp2 and
+    reciprocal approximations; against the FP64 definitions the error stays within
+    2e-7 + 1e-6 |x| over [-10, 10]."""
+    import torch
+    from oracle.epilogue import apply
+    bias = np.linspace(-10.0, 10.0, 801).astype(np.float32)
+    N = bias.size
+    with nj.nnjit_matmul_plan_ex(nj.make_desc(4, N, 0, "bf16", "NK", has_bias=True, epilogue=act), 0.0) as plan:
+        C = torch.full((4, N), float("nan"), device="cuda")
+        plan.run(None, None, torch.from_numpy(bias).cuda(), C)
+        torch.cuda.synchronize()
+    got = C.cpu().numpy().astype(np.float64)
+    x = bias.astype(np.float64)
+    err = np.abs(got - apply(x, act)[None, :])
+    bound = 2e-7 + 1e-6 * np.abs(x)
+    assert np.all(err <= bound[None, :]), f"max excess {np.max(err - bound):.3e} at x = {x[np.argmax(np.max(err, 0) - bound)]}"

@@ -194,3 +194,52 @@ def test_rel_fro_closed_form():
     assert oracle.rel_fro(ref, ref) == 0.0
     assert oracle.rel_fro(np.array([[3.0, 0.0]]), ref) == pytest.approx(4.0 / 5.0)
     assert oracle.rel_fro(np.zeros((1, 1)), np.zeros((1, 1))) == 0.0
+
+
+# ---------------------------------------------------------------- fused activations
+
+def test_relu_exact():
+    from oracle.epilogue import apply
+    x = np.array([-3.5, -0.0, 0.0, 1e-300, 2.25, -1e300])
+    assert np.array_equal(apply(x, "relu"), np.array([0.0, 0.0, 0.0, 1e-300, 2.25, 0.0]))
+
+
+def test_gelu_known_values_and_odd_part():
+    """gelu(x) = x Phi(x): Phi(1) = 0.8413447460685429 and Phi(2) = 0.9772498680518208
+    (standard normal table); gelu(x) - gelu(-x) = x because Phi(x) + Phi(-x) = 1;
+    gelu(0) = 0; for large x, gelu(x) -> x and gelu(-x) -> 0."""
+    from oracle.epilogue import apply
+    g = apply(np.array([1.0, -1.0, 2.0, 0.0, 12.0, -12.0]), "gelu")
+    assert abs(g[0] - 0.8413447460685429) < 1e-15
+    assert abs(g[1] + (1.0 - 0.8413447460685429)) < 1e-15
+    assert abs(g[2] - 2.0 * 0.9772498680518208) < 1e-15
+    assert g[3] == 0.0 and abs(g[4] - 12.0) < 1e-14 and abs(g[5]) < 1e-14
+    x = np.random.default_rng(3).normal(0.0, 3.0, 1000)
+    assert np.max(np.abs(apply(x, "gelu") - apply(-x, "gelu") - x)) < 1e-13
+
+
+def test_silu_known_values_and_odd_part():
+    """silu(x) = x sigma(x): sigma(ln 3) = 3/4 exactly; silu(x) - silu(-x) = x because
+    sigma(x) + sigma(-x) = 1; silu(0) = 0; silu(-800) is -0 without overflow."""
+    from oracle.epilogue import apply
+    s = apply(np.array([np.log(3.0), 0.0, -800.0, 40.0]), "silu")
+    assert abs(s[0] - 0.75 * np.log(3.0)) < 1e-15
+    assert s[1] == 0.0 and s[2] == 0.0 and abs(s[3] - 40.0) < 1e-12
+    x = np.random.default_rng(4).normal(0.0, 3.0, 1000)
+    assert np.max(np.abs(apply(x, "silu") - apply(-x, "silu") - x)) < 1e-13
+
+
+def test_matmul_applies_activation_after_bias():
+    """The fused epilogue acts on the biased sum: with A = 0 the result is act(bias)."""
+    from oracle.epilogue import apply
+    bias = np.array([-2.0, -0.5, 0.0, 0.5, 2.0], dtype=np.float32)
+    A = np.zeros((3, 4), np.float32)
+    B = np.ones((4, 5), np.float32)
+    for act in ("relu", "gelu", "silu"):
+        C64, _ = oracle.matmul(A, B, bias, oracle.B_KN, act=act)
+        assert np.array_equal(C64, np.broadcast_to(apply(bias.astype(np.float64), act), (3, 5)))
+    # integer sums through relu: negative sums clamp to 0 exactly
+    A = np.array([[1, -2], [3, 1]], np.float32)
+    B = np.array([[1, 1], [2, -1]], np.float32)
+    C64, _ = oracle.matmul(A, B, None, oracle.B_KN, act="relu")
+    assert np.array_equal(C64, np.array([[0.0, 3.0], [5.0, 2.0]]))
