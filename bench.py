@@ -40,8 +40,19 @@ def log(*a):
 
 # ------------------------------------------------------------------------- helpers
 
+def ref_product(oracle, A, B, bias, s, dtype, nthreads=0, act="none"):
+    """The oracle on one product's operands (4-bit weights: dequantised first)."""
+    if dtype == "w4_bf16":
+        from oracle.quant import matmul as w4_matmul
+        return w4_matmul(A, B, s.N, s.K, 0, bias, act, nthreads)
+    return oracle.matmul(A, B, bias, oracle.B_KN if s.b_layout == "KN" else oracle.B_NK,
+                         nthreads=nthreads, act=act)
+
+
 def shape_bytes(s, dtype):
-    e = 2 if dtype == "bf16" else 4
+    if dtype == "w4_bf16":  # x bf16, 4-bit codes, bf16 group scales, f32 C
+        return s.M * s.K * 2 + s.N * s.K // 2 + (s.K + 127) // 128 * s.N * 2 + s.M * s.N * 4
+    e = 2 if dtype in ("bf16",) else 4
     b = s.batch * (s.M * s.K * e + s.K * s.N * e + s.M * s.N * 4)
     return b + (4 * s.N if s.has_bias else 0)
 
@@ -199,8 +210,8 @@ def run_reference(args, workload, rank):
     t0 = time.perf_counter()
     s, A, B, bias = ops[0]
     probe_rows = max(1, min(s.M, 8))
-    _ = oracle.matmul(A[..., :probe_rows, :] if s.batch > 1 else A[:probe_rows], B, bias,
-                      oracle.B_KN if s.b_layout == "KN" else oracle.B_NK)
+    _ = ref_product(oracle, np.ascontiguousarray(A[..., :probe_rows, :] if s.batch > 1 else A[:probe_rows]),
+                    B, bias, s, dtype)
     dt_probe = max(1e-4, time.perf_counter() - t0)
     probe_flops = 2 * s.batch * probe_rows * s.N * s.K
     rate = probe_flops / dt_probe
@@ -214,8 +225,7 @@ def run_reference(args, workload, rank):
         for s, A, B, bias in ops:
             rows = max(1, int(round(s.M * frac)))
             Ar = A[:, :rows] if s.batch > 1 else A[:rows]
-            oracle.matmul(np.ascontiguousarray(Ar), B, bias,
-                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores, act=act)
+            ref_product(oracle, np.ascontiguousarray(Ar), B, bias, s, dtype, cores, act)
             fl += 2 * s.batch * rows * s.N * s.K
         dt = time.perf_counter() - t0
         if step >= args.warmup:
@@ -256,8 +266,7 @@ def cpu_baseline(workload, dtype, seconds=12.0, act="none"):
         for s, A, B, bias in ops:
             rows = max(1, int(round(s.M * rows_frac)))
             Ar = A[:, :rows] if s.batch > 1 else A[:rows]
-            oracle.matmul(np.ascontiguousarray(Ar), B, bias,
-                          oracle.B_KN if s.b_layout == "KN" else oracle.B_NK, nthreads=cores, act=act)
+            ref_product(oracle, np.ascontiguousarray(Ar), B, bias, s, dtype, cores, act)
             fl += 2 * s.batch * rows * s.N * s.K
         dt = time.perf_counter() - t0
         done_flops += fl
@@ -282,7 +291,7 @@ def custom_workload(ap, spec):
         M, N, K = (int(x) for x in dims.lower().split("x"))
     except ValueError:
         ap.error(f"--shape: expected MxNxK:dtype:layout, got {spec!r}")
-    if dtype not in ("f32_ffma", "tf32", "bf16") or layout not in ("NK", "KN") or min(M, N, K) < 1:
+    if dtype not in ("f32_ffma", "tf32", "bf16", "w4_bf16") or layout not in ("NK", "KN") or min(M, N, K) < 1:
         ap.error(f"--shape: bad dtype, layout or size in {spec!r}")
     shape = Shape(f"{M}x{N}x{K}", M, N, K, 1, layout)
     return Workload(f"custom_{M}x{N}x{K}_{dtype}_{layout}", 5, f"custom product {spec}", (dtype,), (shape,))
@@ -560,7 +569,7 @@ def main(argv=None):
                     help="activation fused after the bias into every product (nnjit_epilogue)")
     ap.add_argument("--shape", default=None,
                     help="run one custom product instead of a workload: MxNxK:dtype:layout "
-                         "(dtype f32_ffma, tf32 or bf16; layout NK or KN), e.g. 4096x8192x4096:bf16:NK")
+                         "(dtype f32_ffma, tf32, bf16 or w4_bf16; layout NK or KN), e.g. 4096x8192x4096:bf16:NK")
     args = ap.parse_args(argv)
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

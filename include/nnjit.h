@@ -56,9 +56,27 @@ typedef enum {
     NNJIT_F32_FFMA = 0,  /* float32 operands, exact float32 fused multiply-add (SIMT) */
     NNJIT_TF32 = 1,      /* float32 operands consumed as TF32 by the tensor cores
                             (tcgen05 .kind::tf32), float32 accumulation */
-    NNJIT_BF16 = 2       /* bfloat16 operands, float32 accumulation (tcgen05 .kind::f16,
+    NNJIT_BF16 = 2,      /* bfloat16 operands, float32 accumulation (tcgen05 .kind::f16,
                             or the split-K GEMV when M <= 8) */
+    NNJIT_W4_BF16 = 3    /* bfloat16 A, 4-bit weights B with bfloat16 group scales (the
+                            "4-bit quantization" of the paper's Llama 2 result, Sec. 7:
+                            decode, M <= 8, B as [N][K] only); float32 accumulation.  B
+                            points to a weight blob laid out as described below. */
 } nnjit_dtype;
+
+/*
+ * 4-bit weight blob (NNJIT_W4_BF16).  Weight w[n][k] = (q[n][k] - 8) * s[k / 128][n]:
+ *   - q are unsigned 4-bit codes, two per byte, row n at byte n * ldb / 2, code k in byte
+ *     k / 2, the low nibble holding the even k.  ldb (in codes) >= K and a multiple of 32
+ *     (16-byte rows).
+ *   - s are bfloat16 scales, one per row and group of 128 consecutive k, stored
+ *     group-major: s[g][n] at element g * N + n of the scale block, which starts at byte
+ *     nnjit_w4_layout()'s scale_offset (the code block rounded up to 256 bytes).  N must be
+ *     a multiple of 8.
+ * The blob is read-only for the library; like any B it is owned by the caller.
+ */
+nnjit_status nnjit_w4_layout(int64_t N, int64_t K, int64_t ldb, int64_t* scale_offset_bytes,
+                             int64_t* total_bytes);
 
 /* Storage of B. */
 typedef enum {

@@ -21,7 +21,7 @@ from __future__ import annotations
 from dataclasses import dataclass
 
 # enum values of the C ABI
-F32_FFMA, TF32, BF16 = 0, 1, 2
+F32_FFMA, TF32, BF16, W4_BF16 = 0, 1, 2, 3
 B_KN, B_NK = 0, 1
 FAMILY_FFMA, FAMILY_TC, FAMILY_GEMV = 0, 1, 2
 INVALID_ARG, UNSUPPORTED = 1, 2
@@ -46,6 +46,8 @@ GEMV_MAX_SMEM = 64 * 1024
 GEMV_TMA_KC = 256             # K elements per ring stage of the TMA-fed GEMV
 GEMV_TMA_THREADS = 160        # producer warp + 4 consumer warps
 GEMV_TMA_FIRST = 8            # first instance id of the TMA-fed GEMV kernels
+GEMV_W4_FIRST = 14            # first instance id of the 4-bit-weight GEMV kernels
+GEMV_W4_KC = 1024             # 4-bit codes per ring stage and row
 
 CANDIDATE_FIELDS = ("family", "bm", "bn", "bk", "tm", "tn", "stages", "split_k", "raster",
                     "threads", "smem_bytes", "tmem_cols", "regs_per_thread", "blocks_per_sm",
@@ -101,7 +103,7 @@ class Problem:
 
     @property
     def elem(self) -> int:
-        return 2 if self.dtype == BF16 else 4
+        return 2 if self.dtype in (BF16, W4_BF16) else 4
 
     @property
     def degenerate(self) -> bool:
@@ -119,7 +121,7 @@ def resolve(M, N, K, batch=1, dtype=BF16, b_layout=B_NK, lda=0, ldb=0, ldc=0, st
     """Defaults and validation of the problem descriptor (packed when zero)."""
     if M < 0 or N < 0 or K < 0 or batch < 1:
         raise SpaceError(INVALID_ARG)
-    if dtype not in (F32_FFMA, TF32, BF16) or b_layout not in (B_KN, B_NK) or has_bias not in (0, 1):
+    if dtype not in (F32_FFMA, TF32, BF16, W4_BF16) or b_layout not in (B_KN, B_NK) or has_bias not in (0, 1):
         raise SpaceError(INVALID_ARG)
     if max(M, N, K, batch) >= 2 ** 31:
         raise SpaceError(INVALID_ARG)
@@ -150,6 +152,13 @@ def family_of(p: Problem) -> int:
     if p.dtype == F32_FFMA:
         return FAMILY_FFMA
     e = p.elem
+    if p.dtype == W4_BF16:
+        # 4-bit weights: decode products only, 16-byte rows of x, codes and group scales
+        if p.M > GEMV_MAX_M or p.batch != 1 or p.b_layout != B_NK:
+            raise SpaceError(UNSUPPORTED)
+        if not p.degenerate and ((p.lda * 2) % 16 or p.ldb % 32 or p.N % 8):
+            raise SpaceError(UNSUPPORTED)
+        return FAMILY_GEMV
     if p.dtype == BF16 and p.M <= GEMV_MAX_M and p.batch == 1:
         if not p.degenerate and p.b_layout == B_NK and ((p.lda * e) % 16 or (p.ldb * e) % 16):
             raise SpaceError(UNSUPPORTED)
@@ -354,7 +363,56 @@ def _ffma(p, lim):
     return out, 2 * 3 * 3 * 2 * 4
 
 
+def gemv_w4_instance(rows, maxm):
+    return GEMV_W4_FIRST + {8: 0, 16: 1, 32: 2}[rows] * 2 + {1: 0, GEMV_MAX_M: 1}[maxm]
+
+
+def _gemv_w4(p, lim):
+    """4-bit weights: a ring stage holds `rows` weight rows x 1024 codes (512 bytes a row),
+    their 8 group scales, and 1024 elements of every row of x."""
+    M, N, K = max(p.M, 1), max(p.N, 1), max(p.K, 1)
+    wbytes = N * K // 2 + cdiv(K, 128) * N * 2
+    maxm = 1 if M == 1 else GEMV_MAX_M
+    chunks = cdiv(K, GEMV_W4_KC)
+    out = []
+    for rows in (8, 16, 32):
+        groups = cdiv(N, rows)
+        for stages in (4, 8):
+            for split in (1, 2, 4, 8):
+                cps = cdiv(chunks, split)
+                if split > 1 and (cps < 2 or (split - 1) * cps >= chunks or
+                                  groups * (split // 2) >= 2 * lim["sm_count"]):
+                    continue
+                stage_bytes = rows * (GEMV_W4_KC // 2 + 16) + M * GEMV_W4_KC * 2
+                smem = 128 + stages * stage_bytes
+                if smem > lim["smem_per_block_optin"]:
+                    continue
+                regs = 72 if maxm == 1 else 104 + 5 * rows
+                blk = block_core(lim, regs, GEMV_TMA_THREADS, smem, 0)
+                if blk < 1:
+                    continue
+                items = groups * split
+                slots = lim["sm_count"] * blk
+                grid = min(items, slots)
+                inflight = min(cdiv(grid, lim["sm_count"]), blk) * stages * rows * GEMV_W4_KC // 2
+                eff = min(100, max(1, inflight * 100 // 32768))
+                cost = cdiv(wbytes, HBM_BYTES_PER_CLK) * 100 // eff
+                cost = cost * cdiv(items, lim["sm_count"]) * lim["sm_count"] // items
+                if split > 1:
+                    cost += LAUNCH_CLK + cdiv(2 * split * M * N * 4, HBM_BYTES_PER_CLK)
+                c = _blank()
+                c.update(family=FAMILY_GEMV, bm=M, bn=rows, bk=GEMV_W4_KC, tm=rows // 4, tn=1,
+                         stages=stages, split_k=split, threads=GEMV_TMA_THREADS, smem_bytes=smem,
+                         regs_per_thread=regs, blocks_per_sm=blk, grid=grid,
+                         wave_eff_ppm=grid * 1000000 // slots,
+                         instance=gemv_w4_instance(rows, maxm), predicted_cost=cost)
+                out.append(c)
+    return out, 3 * 2 * 4
+
+
 def _gemv(p, lim):
+    if p.dtype == W4_BF16:
+        return _gemv_w4(p, lim)
     M, N, K = max(p.M, 1), max(p.N, 1), max(p.K, 1)
     wbytes = N * K * 2
     out = []

@@ -233,7 +233,9 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
     la.stream = s;
     cudaError_t e = cudaSuccess;
     const bool tc = c.family == NNJIT_FAMILY_TC;
-    if (tc || gemv_uses_tma(c)) {
+    const bool w4 = gemv_uses_w4(c);
+    if (w4 != (p.dtype == NNJIT_W4_BF16)) return fail(NNJIT_ERR_INVALID_ARG, "candidate does not match the dtype");
+    if (tc || gemv_uses_tma(c) || w4) {
         CUtensorMap ta, tb, tcm;
         bool c_ok = false;
         const char* why = "";
@@ -243,9 +245,11 @@ nnjit_status run_impl(nnjit_plan pl, const void* A, const void* B, const float* 
             if (override_cand || !pl->tm_valid || pl->tm_A != A || pl->tm_B != B || pl->tm_C != out ||
                 std::memcmp(&pl->tm_cand, &c, sizeof(c)) != 0) {
                 e = tc ? encode_tc_tensor_maps(p, c, A, B, &ta, &tb, &why)
-                       : encode_gemv_tensor_maps(p, c, A, B, &ta, &tb, &why);
+                    : w4 ? encode_gemv_w4_maps(p, c, A, B, &ta, &tb, &tcm, &why)
+                         : encode_gemv_tensor_maps(p, c, A, B, &ta, &tb, &why);
                 if (e != cudaSuccess) return fail(NNJIT_ERR_UNSUPPORTED, why);
                 if (tc) encode_tc_output_map(p, c, out, two_pass, &tcm, &c_ok);
+                if (w4) c_ok = true;  // third map: the group scales
                 if (!override_cand) {
                     pl->ta = ta; pl->tb = tb; pl->tc = tcm; pl->tm_c_ok = c_ok;
                     pl->tm_A = A; pl->tm_B = B; pl->tm_C = out; pl->tm_cand = c; pl->tm_valid = true;
@@ -293,11 +297,10 @@ struct Scratch {
 nnjit_status make_scratch(const Problem& p, const std::vector<nnjit_candidate>& space,
                           const nnjit_device_limits& L, Scratch* s) {
     const int e = p.elem_bytes();
-    // element extents covering every batch item with the plan's strides
+    // element extents covering every batch item with the plan's strides (B in units of
+    // e bytes, so 4-bit weight blobs are covered too)
     s->a_elems = (size_t)((p.batch - 1) * p.stride_a + (p.M - 1) * p.lda + p.K);
-    const int64_t b_rows = p.b_layout == NNJIT_B_KN ? p.K : p.N;
-    const int64_t b_cols = p.b_layout == NNJIT_B_KN ? p.N : p.K;
-    s->b_elems = (size_t)((p.batch - 1) * p.stride_b + (b_rows - 1) * p.ldb + b_cols);
+    s->b_elems = (size_t)((p.b_bytes() + e - 1) / e);
     s->c_elems = (size_t)((p.batch - 1) * p.stride_c + (p.M - 1) * p.ldc + p.N);
     // round each set up to 256 bytes so every set keeps 16-byte alignment
     auto r256 = [](size_t b) { return (b + 255) / 256 * 256; };
@@ -572,6 +575,18 @@ const char* nnjit_last_error(void) { return t_last_error.c_str(); }
 
 int32_t nnjit_version(void) { return 100; }
 
+nnjit_status nnjit_w4_layout(int64_t N, int64_t K, int64_t ldb, int64_t* scale_offset_bytes,
+                             int64_t* total_bytes) {
+    if (N < 0 || K < 0 || ldb < K || ldb % 32 != 0 || N % 8 != 0)
+        return fail(NNJIT_ERR_INVALID_ARG, "4-bit layout needs N >= 0 a multiple of 8, ldb >= K a multiple of 32");
+    Problem p;
+    p.dtype = NNJIT_W4_BF16;
+    p.N = N; p.K = K; p.ldb = ldb;
+    if (scale_offset_bytes) *scale_offset_bytes = p.w4_scale_offset();
+    if (total_bytes) *total_bytes = p.w4_blob_bytes();
+    return NNJIT_OK;
+}
+
 nnjit_status nnjit_device_limits_query(int32_t device, nnjit_device_limits* out) {
     if (!out) return fail(NNJIT_ERR_INVALID_ARG, "out is NULL");
     return query_limits(device, out);
@@ -840,7 +855,7 @@ nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB
     cudaStream_t s = static_cast<cudaStream_t>(stream);
     const size_t e = (size_t)p.elem_bytes();
     const size_t a_bytes = (size_t)(p.batch * p.M * p.K) * e;
-    const size_t b_bytes = (size_t)(p.batch * p.K * p.N) * e;
+    const size_t b_bytes = (size_t)p.b_bytes();
     const size_t c_bytes = (size_t)(p.batch * p.M * p.N) * 4;
     {
         std::lock_guard<std::mutex> lk(pl->mu);

@@ -338,6 +338,7 @@ cudaError_t launch_gemv(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
     if (gemv_uses_tma(c)) return launch_gemv_tma(a);
+    if (gemv_uses_w4(c)) return launch_gemv_w4(a);
     if (c.instance < 0 || c.instance >= 8 || p.M > kMaxM) return cudaErrorInvalidValue;
     const bool kn_inst = c.instance >= 6;
     if (kn_inst != (p.b_layout == NNJIT_B_KN)) return cudaErrorInvalidValue;

@@ -266,9 +266,69 @@ void ffma_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 // that set the bytes in flight per SM: threads per CTA, rows per warp, 16-byte loads in
 // flight per lane and row (unroll), and split-K.
 // ---------------------------------------------------------------------------------
+// 4-bit weights (NNJIT_W4_BF16): the TMA-fed kernel only.  A ring stage holds `rows`
+// weight rows x 1024 codes (512 bytes a row), their 8 group scales, and the matching
+// 1024-element slice of every row of x; axes rows per stage, ring stages, split-K.
+void gemv_w4_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_candidate>& v,
+                   int64_t* naive) {
+    using MC = ModelConstants;
+    const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
+    const int64_t K = std::max<int64_t>(p.K, 1);
+    const int64_t wbytes = N * K / 2 + ceil_div(K, 128) * N * 2;
+    const int maxm = M == 1 ? 1 : MC::kGemvMaxM;
+    const int64_t chunks = ceil_div(K, MC::kGemvW4Kc);
+    *naive = 3 * 2 * 4;
+    for (int rows : {8, 16, 32}) {
+        const int64_t groups = ceil_div(N, rows);
+        for (int stages : {4, 8}) {
+            for (int split : {1, 2, 4, 8}) {
+                const int64_t cps = ceil_div(chunks, split);
+                if (split > 1 && (cps < 2 || (split - 1) * cps >= chunks ||
+                                  groups * (split / 2) >= 2LL * L.sm_count))
+                    continue;
+                const int64_t stage_bytes = rows * (MC::kGemvW4Kc / 2 + 16) + M * MC::kGemvW4Kc * 2;
+                const int64_t smem = 128 + stages * stage_bytes;
+                if (smem > L.smem_per_block_optin) continue;
+                const int regs = maxm == 1 ? 72 : 104 + 5 * rows;  // ptxas: 58-68 / 144-252
+                const int blk = blocks_per_core(L, regs, MC::kGemvTmaThreads, (int)smem, 0);
+                if (blk < 1) continue;
+                const int64_t items = groups * split;
+                const int64_t slots = (int64_t)L.sm_count * blk;
+                const int64_t grid = std::min<int64_t>(items, slots);
+                nnjit_candidate c = blank();
+                c.family = NNJIT_FAMILY_GEMV;
+                c.bm = (int)M; c.bn = rows; c.bk = MC::kGemvW4Kc;
+                c.tm = rows / 4; c.tn = 1;
+                c.stages = stages;
+                c.split_k = split;
+                c.threads = MC::kGemvTmaThreads;
+                c.smem_bytes = (int)smem;
+                c.regs_per_thread = regs;
+                c.blocks_per_sm = blk;
+                c.grid = (int32_t)grid;
+                c.wave_eff_ppm = (int32_t)(grid * 1000000 / slots);
+                const int64_t resident = std::min<int64_t>(ceil_div(grid, L.sm_count), blk);
+                const int64_t inflight = resident * stages * rows * MC::kGemvW4Kc / 2;
+                const int64_t eff_pct = std::min<int64_t>(100, std::max<int64_t>(1, inflight * 100 / 32768));
+                int64_t cost = ceil_div(wbytes, MC::kHbmBytesPerClk) * 100 / eff_pct;
+                cost = cost * ceil_div(items, L.sm_count) * L.sm_count / items;
+                if (split > 1)
+                    cost += MC::kLaunchClk + ceil_div(2LL * split * M * N * 4, MC::kHbmBytesPerClk);
+                c.predicted_cost = cost;
+                c.instance = gemv_w4_instance(rows, maxm);
+                v.push_back(c);
+            }
+        }
+    }
+}
+
 void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_candidate>& v,
                 int64_t* naive) {
     using MC = ModelConstants;
+    if (p.dtype == NNJIT_W4_BF16) {
+        gemv_w4_space(p, L, v, naive);
+        return;
+    }
     const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
     const int64_t K = std::max<int64_t>(p.K, 1);
     const int64_t wbytes = N * K * 2;
@@ -453,6 +513,13 @@ int gemv_instance(int b_layout, int rows, int unroll) {
     return ri * 2 + ui;
 }
 
+int gemv_w4_instance(int rows, int maxm) {
+    const int ri = rows == 8 ? 0 : rows == 16 ? 1 : rows == 32 ? 2 : -1;
+    const int mi = maxm == 1 ? 0 : maxm == ModelConstants::kGemvMaxM ? 1 : -1;
+    if (ri < 0 || mi < 0) return -1;
+    return kGemvW4FirstInstance + ri * 2 + mi;
+}
+
 int gemv_tma_instance(int rows, int maxm) {
     const int ri = rows == 8 ? 0 : rows == 16 ? 1 : rows == 32 ? 2 : -1;
     const int mi = maxm == 1 ? 0 : maxm == ModelConstants::kGemvMaxM ? 1 : -1;
@@ -464,7 +531,7 @@ nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string
     if (!d || !p) { *err = "descriptor is NULL"; return NNJIT_ERR_INVALID_ARG; }
     if (d->M < 0 || d->N < 0 || d->K < 0) { *err = "M, N, K must be >= 0"; return NNJIT_ERR_INVALID_ARG; }
     if (d->batch < 1) { *err = "batch must be >= 1"; return NNJIT_ERR_INVALID_ARG; }
-    if (d->dtype < NNJIT_F32_FFMA || d->dtype > NNJIT_BF16) { *err = "unknown dtype"; return NNJIT_ERR_INVALID_ARG; }
+    if (d->dtype < NNJIT_F32_FFMA || d->dtype > NNJIT_W4_BF16) { *err = "unknown dtype"; return NNJIT_ERR_INVALID_ARG; }
     if (d->b_layout != NNJIT_B_KN && d->b_layout != NNJIT_B_NK) { *err = "unknown b_layout"; return NNJIT_ERR_INVALID_ARG; }
     if (d->has_bias != 0 && d->has_bias != 1) { *err = "has_bias must be 0 or 1"; return NNJIT_ERR_INVALID_ARG; }
     if (d->epilogue < NNJIT_EPI_NONE || d->epilogue > NNJIT_EPI_SILU) { *err = "unknown epilogue"; return NNJIT_ERR_INVALID_ARG; }
@@ -506,6 +573,19 @@ nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string
 
 nnjit_status choose_family(const Problem& p, int* family, std::string* err) {
     if (p.dtype == NNJIT_F32_FFMA) { *family = NNJIT_FAMILY_FFMA; return NNJIT_OK; }
+    if (p.dtype == NNJIT_W4_BF16) {
+        if (p.M > ModelConstants::kGemvMaxM || p.batch != 1 || p.b_layout != NNJIT_B_NK) {
+            *err = "4-bit weights are served for decode products: M <= 8, batch 1, B as [N][K]";
+            return NNJIT_ERR_UNSUPPORTED;
+        }
+        if (!p.degenerate() && ((p.lda * 2) % 16 != 0 || p.ldb % 32 != 0 || p.N % 8 != 0)) {
+            *err = "4-bit GEMV needs 16-byte rows of A (lda multiple of 8), of the codes (ldb "
+                   "multiple of 32) and of the group-major scales (N multiple of 8)";
+            return NNJIT_ERR_UNSUPPORTED;
+        }
+        *family = NNJIT_FAMILY_GEMV;
+        return NNJIT_OK;
+    }
     const int e = p.elem_bytes();
     if (p.dtype == NNJIT_BF16 && p.M <= ModelConstants::kGemvMaxM && p.batch == 1) {
         // B as [N][K]: x is staged and W streamed with 16-byte loads along K.  B as [K][N]

@@ -24,8 +24,19 @@ struct Problem {
     int has_bias = 0;
     uint32_t flags = 0;
     int epilogue = NNJIT_EPI_NONE;
-    int elem_bytes() const { return dtype == NNJIT_BF16 ? 2 : 4; }
+    // bytes per element of A (and of B, except for 4-bit weights)
+    int elem_bytes() const { return dtype == NNJIT_BF16 || dtype == NNJIT_W4_BF16 ? 2 : 4; }
     bool degenerate() const { return M == 0 || N == 0 || K == 0; }
+    // 4-bit weight blob: scale block offset and total bytes (see nnjit.h)
+    int64_t w4_scale_offset() const { return (N * (ldb / 2) + 255) / 256 * 256; }
+    int64_t w4_groups() const { return (K + 127) / 128; }
+    int64_t w4_blob_bytes() const { return w4_scale_offset() + w4_groups() * N * 2; }
+    // extent of B in bytes over every batch item
+    int64_t b_bytes() const {
+        if (dtype == NNJIT_W4_BF16) return w4_blob_bytes();
+        const int64_t rows = b_layout == NNJIT_B_KN ? K : N, cols = b_layout == NNJIT_B_KN ? N : K;
+        return ((batch - 1) * stride_b + (rows - 1) * ldb + cols) * elem_bytes();
+    }
 };
 
 // Model constants of the ordering cost (readings; see the design notes).
@@ -48,6 +59,7 @@ struct ModelConstants {
     static constexpr int kGemvMaxSmem = 64 * 1024;
     static constexpr int kGemvTmaKc = 256;           // K elements per TMA GEMV ring stage
     static constexpr int kGemvTmaThreads = 160;      // producer warp + 4 consumer warps
+    static constexpr int kGemvW4Kc = 1024;           // K codes per 4-bit GEMV ring stage
 };
 
 // Resolve defaults and validate.  Returns NNJIT_OK or an error with `err` set.
@@ -71,5 +83,8 @@ int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if non
 // TMA-fed GEMV (B as [N][K]): rows per stage 8/16/32, M <= maxm (1 or 8).
 constexpr int kGemvTmaFirstInstance = 8;
 int gemv_tma_instance(int rows, int maxm);                     // 8..13, -1 if none
+// TMA-fed GEMV over 4-bit weights (NNJIT_W4_BF16): rows per stage 8/16/32, maxm 1 or 8.
+constexpr int kGemvW4FirstInstance = 14;
+int gemv_w4_instance(int rows, int maxm);                      // 14..19, -1 if none
 
 }  // namespace nnjit

@@ -25,6 +25,7 @@ NNJIT_ERR_BUDGET = 6
 NNJIT_F32_FFMA = 0
 NNJIT_TF32 = 1
 NNJIT_BF16 = 2
+NNJIT_W4_BF16 = 3
 
 NNJIT_EPI_NONE = 0
 NNJIT_EPI_RELU = 1
@@ -43,7 +44,7 @@ NNJIT_PLAN_EXHAUSTIVE = 0x2
 NNJIT_PLAN_REQUIRE_TIMED = 0x4
 NNJIT_PLAN_B_CONSTANT = 0x8
 
-DTYPES = {"f32_ffma": NNJIT_F32_FFMA, "tf32": NNJIT_TF32, "bf16": NNJIT_BF16}
+DTYPES = {"f32_ffma": NNJIT_F32_FFMA, "tf32": NNJIT_TF32, "bf16": NNJIT_BF16, "w4_bf16": NNJIT_W4_BF16}
 LAYOUTS = {"KN": NNJIT_B_KN, "NK": NNJIT_B_NK}
 
 
@@ -121,6 +122,7 @@ def load_library(path: str = LIB_PATH):
             "nnjit_plan_online_progress": [vp, P(i32), P(i32), P(i32), P(i32)],
             "nnjit_cache_save": [ctypes.c_char_p],
             "nnjit_cache_load": [ctypes.c_char_p, P(i32)],
+            "nnjit_w4_layout": [i64, i64, i64, P(i64), P(i64)],
         }
         for name, args in sigs.items():
             f = getattr(lib, name)
@@ -337,6 +339,14 @@ def nnjit_gemv_bf16_noalloc(M: int, N: int, K: int, x, W, bias, C, split_k: int,
 
 def nnjit_cache_clear():
     _check(load_library().nnjit_cache_clear(), "nnjit_cache_clear")
+
+
+def nnjit_w4_layout(N: int, K: int, ldb: int = 0):
+    """(scale_offset_bytes, total_bytes) of a 4-bit weight blob (ldb = 0: K)."""
+    off, tot = ctypes.c_int64(0), ctypes.c_int64(0)
+    _check(load_library().nnjit_w4_layout(N, K, ldb or K, ctypes.byref(off), ctypes.byref(tot)),
+           "nnjit_w4_layout")
+    return off.value, tot.value
 
 
 def nnjit_cache_size() -> int:

@@ -183,6 +183,13 @@ WORKLOADS = {
                   ("normal", 0.0), (12, 13, 2), False),
             Shape("pv", 1024, 128, 1024, 128, "KN", False, ("normal", 1.0), ("normal", 1.0),
                   ("normal", 0.0), (14, 15, 2), False))),
+    "llama2_7b_decode_w4_m1": Workload(
+        "llama2_7b_decode_w4_m1", 6,
+        "Llama-2-7B decoder block decode GEMVs, batch 1 (M=1), 4-bit weights with bf16 group "
+        "scales (group 128), bf16 activations",
+        ("w4_bf16",),
+        _linears(1, [(12288, 4096), (4096, 4096), (22016, 4096), (4096, 11008)],
+                 ["qkv", "o_proj", "gate_up", "down"])),
 }
 
 
@@ -197,6 +204,47 @@ def _draw(dist: tuple, seed: int, n: int, ints: bool) -> np.ndarray:
     raise ValueError(kind)
 
 
+def w4_blob(codes: np.ndarray, scale_bits: np.ndarray, ldb: int = 0) -> np.ndarray:
+    """The storage of 4-bit weights (nnjit_w4_layout): codes [N][K] in 0..15, two per byte
+    (row n at byte n * ldb / 2, code k in byte k / 2, the low nibble holding the even k),
+    then, from the code block rounded up to 256 bytes, the bf16 scale bit patterns
+    [ceil(K / 128)][N] (group-major)."""
+    N, K = codes.shape
+    ldb = ldb or K
+    row = ldb // 2
+    off = (N * row + 255) // 256 * 256
+    blob = np.zeros(off + scale_bits.size * 2, dtype=np.uint8)
+    c = np.zeros((N, 2 * row), dtype=np.uint8)
+    c[:, :K] = codes
+    blob[:N * row] = (c[:, 0::2] | (c[:, 1::2] << 4)).ravel()
+    blob[off:] = np.ascontiguousarray(scale_bits, dtype=np.uint16).view(np.uint8).ravel()
+    return blob
+
+
+def make_w4_operands(shape: Shape, base_seed: int, ints: bool = False, ldb: int = 0):
+    """Operands of one product over 4-bit weights: x as bf16 bit patterns [M][K] (the
+    shape's A distribution), the weight blob (codes drawn uniformly from 0..15, scales
+    uniform in [0.002, 0.01) rounded to bf16 -- about the magnitude of a symmetric 4-bit
+    quantisation of N(0, 0.02^2) weights), and the bias.  `ints`: x in [-8, 8] and every
+    scale 1, so every product and sum is an exact integer."""
+    ida, idb, idbias = shape.ids
+    N, K = shape.N, shape.K
+    x = _draw(shape.a_dist, tensor_seed(base_seed, ida), shape.M * K, ints)
+    x_bits = f32_to_bf16_bits(to_f32(x).reshape(shape.M, K))
+    seed_b = tensor_seed(base_seed, idb)
+    codes = np.floor(16.0 * _unit(seed_b, N * K)).astype(np.uint8).reshape(N, K)
+    groups = (K + 127) // 128
+    if ints:
+        scales = np.ones((groups, N), dtype=np.float32)
+    else:
+        scales = to_f32(uniform(seed_b ^ 0x5CA1E, groups * N, 0.002, 0.01)).reshape(groups, N)
+    blob = w4_blob(codes, f32_to_bf16_bits(scales), ldb)
+    bias = None
+    if shape.has_bias:
+        bias = to_f32(_draw(shape.bias_dist, tensor_seed(base_seed, idbias), N, ints))
+    return x_bits, blob, bias
+
+
 def make_operands(shape: Shape, base_seed: int, dtype: str, ints: bool = False,
                   M: int | None = None):
     """Operands of one product in their storage form.
@@ -207,6 +255,10 @@ def make_operands(shape: Shape, base_seed: int, dtype: str, ints: bool = False,
     `M` overrides the row count (the first M rows of the full-size A are drawn, so a
     sample of rows equals the corresponding rows of the full operand).
     """
+    if dtype == "w4_bf16":
+        if M is not None:
+            raise ValueError("row override not supported for 4-bit weights")
+        return make_w4_operands(shape, base_seed, ints)
     Mr = shape.M if M is None else M
     ida, idb, idbias = shape.ids
     bshape = (shape.K, shape.N) if shape.b_layout == "KN" else (shape.N, shape.K)

@@ -6,7 +6,7 @@ import numpy as np
 
 import oracle
 
-TOL = {"f32_ffma": 1e-5, "tf32": 5e-3, "bf16": 1e-2}
+TOL = {"f32_ffma": 1e-5, "tf32": 5e-3, "bf16": 1e-2, "w4_bf16": 1e-2}
 
 
 def torch_mod():

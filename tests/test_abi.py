@@ -105,3 +105,15 @@ def test_cache_file_format(lib, tmp_path):
     assert lines[1].split("\t")[1] == entry.split("\t")[1]
     nj.nnjit_cache_clear()
     assert nj.nnjit_cache_size() == 0
+
+
+def test_w4_layout_matches_the_documented_blob(lib):
+    import paper_2309_08978_gb300 as nj
+    # code block N * ldb / 2 bytes rounded up to 256, then ceil(K / 128) * N bf16 scales
+    assert nj.nnjit_w4_layout(4096, 11008) == (4096 * 5504, 4096 * 5504 + 86 * 4096 * 2)
+    assert nj.nnjit_w4_layout(8, 200, 224) == (1024, 1024 + 2 * 8 * 2)
+    assert nj.nnjit_w4_layout(24, 32) == (512, 512 + 24 * 2)
+    for bad in ((4096, 4096, 4100), (4096, 100, 0), (1004, 4096, 0), (8, 64, 32)):
+        with pytest.raises(nj.NnjitError) as ei:
+            nj.nnjit_w4_layout(*bad)
+        assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG

@@ -357,3 +357,71 @@ def test_fused_activation_k0_applies_to_bias(act):
     err = np.abs(got - apply(x, act)[None, :])
     bound = 2e-7 + 1e-6 * np.abs(x)
     assert np.all(err <= bound[None, :]), f"max excess {np.max(err - bound):.3e} at x = {x[np.argmax(np.max(err, 0) - bound)]}"
+
+
+W4_CASES = [(1, 4096, 4096, 0), (1, 4096, 11008, 0), (3, 1000, 2056, 2080), (8, 520, 4096, 0),
+            (2, 264, 640, 0)]
+
+
+def _w4_ids(c):
+    return f"w4-{c[0]}x{c[1]}x{c[2]}" + (f"-ldb{c[3]}" if c[3] else "")
+
+
+def _w4_compare(C, x, blob, N, K, ldb, bias, exact, act="none"):
+    from oracle.quant import matmul as w4_matmul
+    ref64, ref32 = w4_matmul(x, blob, N, K, ldb, bias, act)
+    assert np.all(np.isfinite(C)), "non-finite output (unwritten element?)"
+    if exact:
+        bad = np.argwhere(C != ref32)
+        assert bad.size == 0, f"{len(bad)} elements differ, first at {bad[:5].tolist()}"
+    else:
+        err = oracle.rel_fro(C, ref64)
+        assert err <= 1e-2, f"rel_fro {err:.3e}"
+
+
+@pytest.mark.parametrize("case", W4_CASES, ids=_w4_ids)
+def test_w4_gemv_every_candidate(case):
+    """4-bit weights: every candidate of the space, exact on integer x with unit scales
+    (products (q - 8) x and all sums are integers below 2^24), within the BF16 tolerance
+    on the workload's distributions, with and without constant-weight preloading.  K =
+    2056 and 11008 end in a partial stage; K = 2056 also pads rows to ldb = 2080 codes."""
+    from synthetic import make_w4_operands
+    M, N, K, ldb = case
+    shape = Shape("t", M, N, K, 1, "NK", True)
+    xi, blob_i, bias_i = make_w4_operands(shape, 40, ints=True, ldb=ldb)
+    xr, blob_r, bias_r = make_w4_operands(shape, 41, ldb=ldb)
+    for flags in (nj.NNJIT_PLAN_NO_CACHE, nj.NNJIT_PLAN_NO_CACHE | nj.NNJIT_PLAN_B_CONSTANT):
+        desc = nj.make_desc(M, N, K, "w4_bf16", "NK", has_bias=True, ldb=ldb, flags=flags)
+        cands, _ = nj.nnjit_space_enumerate(desc, nj.nnjit_device_limits_query(0))
+        assert cands and all(c["instance"] >= 14 for c in cands)
+        for i, c in enumerate(cands):
+            with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+                Ce = run_plan(plan, xi, blob_i, bias_i, M, N)
+                Cr = run_plan(plan, xr, blob_r, bias_r, M, N)
+            try:
+                _w4_compare(Ce, xi, blob_i, N, K, ldb, bias_i, exact=True)
+                _w4_compare(Cr, xr, blob_r, N, K, ldb, bias_r, exact=False)
+            except AssertionError as e:
+                raise AssertionError(f"candidate {i} {c}: {e}") from None
+
+
+def test_w4_gemv_tuned_plan_with_activation():
+    from synthetic import make_w4_operands
+    M, N, K = 1, 4096, 4096
+    shape = Shape("t", M, N, K, 1, "NK", True)
+    x, blob, bias = make_w4_operands(shape, 42)
+    desc = nj.make_desc(M, N, K, "w4_bf16", "NK", has_bias=True, epilogue="silu",
+                        flags=nj.NNJIT_PLAN_NO_CACHE)
+    with nj.nnjit_matmul_plan_ex(desc, 50.0) as plan:
+        C = run_plan(plan, x, blob, bias, M, N)
+    _w4_compare(C, x, blob, N, K, 0, bias, exact=False, act="silu")
+
+
+def test_w4_refusals():
+    """Prefill-sized M, B as [K][N], unaligned code rows and a ragged N are refused."""
+    L = nj.nnjit_device_limits_query(0)
+    for d in (nj.make_desc(16, 64, 256, "w4_bf16", "NK"), nj.make_desc(1, 64, 256, "w4_bf16", "KN"),
+              nj.make_desc(1, 64, 100, "w4_bf16", "NK"), nj.make_desc(1, 60, 256, "w4_bf16", "NK")):
+        with pytest.raises(nj.NnjitError) as ei:
+            nj.nnjit_space_enumerate(d, L)
+        assert ei.value.status == nj.NNJIT_ERR_UNSUPPORTED

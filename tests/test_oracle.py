@@ -243,3 +243,59 @@ def test_matmul_applies_activation_after_bias():
     B = np.array([[1, 1], [2, -1]], np.float32)
     C64, _ = oracle.matmul(A, B, None, oracle.B_KN, act="relu")
     assert np.array_equal(C64, np.array([[0.0, 3.0], [5.0, 2.0]]))
+
+
+# ---------------------------------------------------------------- 4-bit weights
+
+def test_w4_dequant_hand_packed_blob():
+    """A blob written byte by byte: row 1 holds codes 1, 2 (byte 0x21: the even k in the
+    low nibble), code 15 at k = 127 and code 0 at k = 128; scales 0.5 (group 0) and 2.0
+    (group 1) of row 1 sit at element N + 1 and 2N + 1 of the group-major scale block,
+    which starts at the code block (8 rows x 128 bytes = 1024) rounded up to 256."""
+    from oracle.quant import dequant
+    N, K = 8, 256
+    blob = np.full(1024 + 2 * N * 2, 0x88, dtype=np.uint8)      # every code 8 -> weight 0
+    blob[1 * 128 + 0] = 0x21
+    blob[1 * 128 + 63] = 0xF8                                     # k = 126 -> 8, k = 127 -> 15
+    blob[1 * 128 + 64] = 0x80                                     # k = 128 -> 0, k = 129 -> 8
+    scales = np.zeros((2, N), dtype=np.uint16)
+    scales[0, 1] = 0x3F00                                         # 0.5
+    scales[1, 1] = 0x4000                                         # 2.0
+    blob[1024:] = scales.view(np.uint8).ravel()
+    W = dequant(blob, N, K)
+    assert W.shape == (N, K)
+    assert W[1, 0] == (1 - 8) * 0.5 and W[1, 1] == (2 - 8) * 0.5
+    assert W[1, 127] == 7 * 0.5 and W[1, 128] == -8 * 2.0
+    nz = np.argwhere(W != 0).tolist()
+    assert nz == [[1, 0], [1, 1], [1, 127], [1, 128]], nz
+
+
+def test_w4_dequant_padded_rows_and_ragged_groups():
+    """K = 200 (two groups, the second partial) with rows padded to ldb = 224 codes: the
+    padding codes are ignored and k = 128..199 take the second group's scale."""
+    from oracle.quant import dequant
+    from synthetic import w4_blob
+    N, K, ldb = 16, 200, 224
+    rng = np.random.default_rng(5)
+    codes = rng.integers(0, 16, (N, K)).astype(np.uint8)
+    sb = np.array([[0x3F80] * N, [0x3E80] * N], dtype=np.uint16)   # 1.0, 0.25
+    blob = w4_blob(codes, sb, ldb)
+    assert blob.size == (N * ldb // 2 + 255) // 256 * 256 + 2 * N * 2
+    W = dequant(blob, N, K, ldb)
+    want = (codes.astype(np.float64) - 8) * np.where(np.arange(K) < 128, 1.0, 0.25)
+    assert np.array_equal(W, want)
+
+
+def test_w4_matmul_small_integers_bruteforce():
+    """x . W^T with integer x and scale 1: the exact integer sums of (q - 8) x."""
+    from oracle.quant import matmul as w4_matmul
+    from synthetic import w4_blob
+    rng = np.random.default_rng(6)
+    M, N, K = 3, 8, 130
+    codes = rng.integers(0, 16, (N, K)).astype(np.uint8)
+    xi = rng.integers(-8, 9, (M, K))
+    blob = w4_blob(codes, np.full((2, N), 0x3F80, np.uint16))
+    x_bits = f32_to_bf16_bits(xi.astype(np.float32))
+    C64, _ = w4_matmul(x_bits, blob, N, K)
+    want = [[sum(int(xi[m, k]) * (int(codes[n, k]) - 8) for k in range(K)) for n in range(N)] for m in range(M)]
+    assert np.array_equal(C64, np.array(want, dtype=np.float64))

@@ -45,7 +45,7 @@ def _limits(d):
 
 def _problems():
     from synthetic import WORKLOADS
-    code = {"f32_ffma": osp.F32_FFMA, "tf32": osp.TF32, "bf16": osp.BF16}
+    code = {"f32_ffma": osp.F32_FFMA, "tf32": osp.TF32, "bf16": osp.BF16, "w4_bf16": osp.W4_BF16}
     out = []
     for w in WORKLOADS.values():
         for dt in w.dtypes:
@@ -67,6 +67,11 @@ def _problems():
     # explicit strides, unaligned strides (UNSUPPORTED), invalid descriptors
     out.append(dict(M=2, N=77, K=100, dtype=osp.BF16, b_layout=osp.B_NK, lda=104, ldb=104))
     out.append(dict(M=64, N=64, K=30, dtype=osp.BF16, b_layout=osp.B_NK))
+    # 4-bit weights: decode shapes, a padded row, a ragged N, and refusals
+    for M, N, K, ldb in ((1, 4096, 4096, 0), (1, 4096, 11008, 0), (3, 1000, 2056, 2080),
+                         (8, 520, 4096, 0), (1, 1000, 100, 0), (1, 1004, 4096, 0), (9, 64, 256, 0)):
+        out.append(dict(M=M, N=N, K=K, dtype=osp.W4_BF16, b_layout=osp.B_NK, ldb=ldb))
+    out.append(dict(M=1, N=64, K=256, dtype=osp.W4_BF16, b_layout=osp.B_KN))
     out.append(dict(M=64, N=30, K=64, dtype=osp.TF32, b_layout=osp.B_KN))
     out.append(dict(M=130, N=72, K=64, dtype=osp.BF16, b_layout=osp.B_NK, ldc=75))
     out.append(dict(M=4, N=4, K=8, dtype=osp.BF16, b_layout=osp.B_NK, lda=4))
