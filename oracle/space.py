@@ -363,19 +363,18 @@ def _ffma(p, lim):
     return out, 2 * 3 * 3 * 2 * 4
 
 
-def gemv_w4_instance(rows, maxm):
-    return GEMV_W4_FIRST + {8: 0, 16: 1, 32: 2}[rows] * 2 + {1: 0, GEMV_MAX_M: 1}[maxm]
+def gemv_w4_instance(rows):
+    return GEMV_W4_FIRST + {16: 0, 32: 1}[rows]
 
 
 def _gemv_w4(p, lim):
     """4-bit weights: a ring stage holds `rows` weight rows x 1024 codes (512 bytes a row),
-    their 8 group scales, and 1024 elements of every row of x."""
+    1024 elements of every row of x and the rows' 8 group scales, padded to 1 KB."""
     M, N, K = max(p.M, 1), max(p.N, 1), max(p.K, 1)
     wbytes = N * K // 2 + cdiv(K, 128) * N * 2
-    maxm = 1 if M == 1 else GEMV_MAX_M
     chunks = cdiv(K, GEMV_W4_KC)
     out = []
-    for rows in (8, 16, 32):
+    for rows in (16, 32):
         groups = cdiv(N, rows)
         for stages in (4, 8):
             for split in (1, 2, 4, 8):
@@ -383,11 +382,11 @@ def _gemv_w4(p, lim):
                 if split > 1 and (cps < 2 or (split - 1) * cps >= chunks or
                                   groups * (split // 2) >= 2 * lim["sm_count"]):
                     continue
-                stage_bytes = rows * (GEMV_W4_KC // 2 + 16) + M * GEMV_W4_KC * 2
-                smem = 128 + stages * stage_bytes
+                stage_bytes = cdiv(rows * (GEMV_W4_KC // 2 + 16) + M * GEMV_W4_KC * 2, 1024) * 1024
+                smem = 1024 + stages * stage_bytes + 256 + rows * 128
                 if smem > lim["smem_per_block_optin"]:
                     continue
-                regs = 72 if maxm == 1 else 104 + 5 * rows
+                regs = 88 if rows == 16 else 112
                 blk = block_core(lim, regs, GEMV_TMA_THREADS, smem, 0)
                 if blk < 1:
                     continue
@@ -401,13 +400,13 @@ def _gemv_w4(p, lim):
                 if split > 1:
                     cost += LAUNCH_CLK + cdiv(2 * split * M * N * 4, HBM_BYTES_PER_CLK)
                 c = _blank()
-                c.update(family=FAMILY_GEMV, bm=M, bn=rows, bk=GEMV_W4_KC, tm=rows // 4, tn=1,
+                c.update(family=FAMILY_GEMV, bm=M, bn=rows, bk=GEMV_W4_KC, tm=rows // 16, tn=1,
                          stages=stages, split_k=split, threads=GEMV_TMA_THREADS, smem_bytes=smem,
                          regs_per_thread=regs, blocks_per_sm=blk, grid=grid,
                          wave_eff_ppm=grid * 1000000 // slots,
-                         instance=gemv_w4_instance(rows, maxm), predicted_cost=cost)
+                         instance=gemv_w4_instance(rows), predicted_cost=cost)
                 out.append(c)
-    return out, 3 * 2 * 4
+    return out, 2 * 2 * 4
 
 
 def _gemv(p, lim):

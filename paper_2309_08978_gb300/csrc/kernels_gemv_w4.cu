@@ -1,26 +1,35 @@
 // Decode-sized products over 4-bit weights (NNJIT_W4_BF16): C[m][n] = sum_k x[m][k] *
-// (q[n][k] - 8) * s[k / 128][n] (+ bias[n]), M <= 8, fed by the tensor memory accelerator.
+// (q[n][k] - 8) * s[k / 128][n] (+ bias[n]), M <= 8.  The weight rows are the M dimension
+// of warp-level tensor-core MMAs (mma.sync m16n8k16, bf16 x bf16 -> f32) and the (up to 8)
+// rows of x are their N dimension, so the CUDA cores only dequantise.
 //
-// The structure is that of the bf16 TMA-fed GEMV: warp 0 (one lane) streams ring stages
-// of ROWS weight rows x 1024 codes (512 bytes a row, one 2-D box of 32-bit words), the 8
-// group scales of those rows (a second box, group-major) and the matching 1024-element
-// slice of every row of x (four boxes of 256); warps 1..4 each own ROWS / 4 rows of a
-// stage.  Lane l takes 8 consecutive codes at k = 8l + 256i for i = 0..3 (a 4-byte word
-// of codes at byte 4l + 128i, 16 bytes of x at 16l + 512i: both conflict-free), whose
-// group is 2i + l / 16.
+// Ring (one producer lane, TMA): a stage holds ROWS weight rows x 1024 codes as four
+// 128-byte-swizzled boxes of 256 codes (box b = K quarter b), the 8 group scales of those
+// rows, and the matching 1024 elements of every row of x (four boxes of 256).  Consumer
+// warp w takes K quarter w of every stage for all ROWS rows (16-row MMA tiles); the four
+// warps' partial sums meet in shared memory at the end of a work item (ROWS output
+// columns x one K slice), in a fixed order.
 //
-// Dequantisation costs one logic operation per weight and one packed add and one packed
-// FMA (f32x2) per two weights.  Masking a code in place (nibble t of a 16-bit half at
-// bits 4t) and or-ing the exponent of 2^23 gives the float 2^23 + c 16^t exactly;
-// subtracting 2^23 + 8 16^t leaves (c - 8) 16^t exactly, and x, pre-scaled once per
-// stage by 16^-t, turns the FMA into (c - 8) x.  Nibble t of the low and of the high half
-// share the constant and the scale, so they travel as one f32x2 pair.  Every product is
-// exact in float32 (a 4-bit integer times a bfloat16); the 8 products of a group slice
-// are summed in a pair, which is multiplied by the group scale into the pair
-// accumulator of its row; the pair's two halves are added when the work item ends.
+// Fragments (m16n8k16; lane = 4 g + t): A rows g and g + 8, B column (token) g.  Within a
+// block of 128 codes (one scale group) thread t loads 32 consecutive codes of each of its
+// rows (a conflict-free 16-byte read of the swizzled box) and, for its token, the 32
+// matching x.  The k order inside an MMA is free as long as A and B agree, so each 8-code
+// word feeds two MMAs in the order the bit tricks produce: with (c0 .. c7) the codes of
+// the word, or-ing the exponent of 128 onto the masked nibbles of the word shifted by 0,
+// 4, 8 and 12 bits gives the bf16 pairs (128 + c0, 128 + c4), (128 + c1, 128 + c5),
+// (128 + c2, 128 + c6) and (128 + c3, 128 + c7); one packed subtract leaves (c - 8) exactly.
+// MMA 1 takes the pairs (c0, c4), (c1, c5) and x pairs (x0, x4), (x1, x5); MMA 2 the rest.
+// Two shared-memory bank conflicts are taken out by choices the MMA does not see: MMA row
+// g reads stage row ((g & 1) << 2 | g >> 1) (a row permutation undone at the output), and
+// thread t walks its 4 words in the order pp ^ (t & 2).
+// The 8 MMAs of a scale group accumulate from zero; the group sum is then scaled per row
+// and added to the thread's float32 accumulators.  Products are exact ((c - 8) times a
+// bf16 value); only the float32 accumulation rounds.
 //
-// Codes past K are zero-filled by the copy engine, and so are the scales of groups past
-// K and the x elements: nothing past K contributes.  Every wait is bounded.
+// Codes past K are zero-filled, and so are the scales of groups past K and x: nothing
+// past K contributes.  Every wait is bounded; an expired wait raises the CTA's abort
+// flag, and every consumer warp still meets the others at the item-end barriers before
+// all leave together.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -37,10 +46,9 @@ namespace nnjit {
 namespace {
 
 constexpr int kKc = 1024;             // codes per stage and row
-constexpr int kWRowBytes = kKc / 2;   // 512
+constexpr int kQuarter = 256;         // codes per box (one consumer warp's K share)
 constexpr int kGroupsPerStage = kKc / 128;
-constexpr int kXBox = 256;            // x elements per TMA box
-constexpr int kThreads = 160;
+constexpr int kThreads = 160;         // producer warp + 4 consumer warps
 constexpr int kMaxStages = 8;
 constexpr long long kPrefetchBytes = 48ll << 20;
 constexpr int kErrEmpty = 0x211;
@@ -48,7 +56,7 @@ constexpr int kErrFull = 0x212;
 constexpr int kErrDrain = 0x213;
 
 struct GemvW4Params {
-    CUtensorMap tmap_w;  // codes as 32-bit words: dims {ceil(K/8), N}, box {128, ROWS}
+    CUtensorMap tmap_w;  // codes as 32-bit words: dims {ceil(K/8), N}, box {32, ROWS}, 128B swizzle
     CUtensorMap tmap_s;  // scales bf16, group-major: dims {N, groups}, box {ROWS, 8}
     CUtensorMap tmap_x;  // x bf16: dims {K, M}, box {256, M}
     const float* bias;
@@ -72,73 +80,86 @@ __device__ __forceinline__ Item item_of(int it, const GemvW4Params& p) {
     return r;
 }
 
-// Packed float32 pairs (f32x2 arithmetic of sm_10x).
-__device__ __forceinline__ uint64_t pk2(float a, float b) {
-    uint64_t r;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+__device__ __forceinline__ uint32_t lop_or(uint32_t a, uint32_t mask, uint32_t bits) {
+    return (a & mask) | bits;
+}
+// bf16x2 a - b
+__device__ __forceinline__ uint32_t sub_bf2(uint32_t a, uint32_t b) {
+    uint32_t r;
+    asm("sub.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
     return r;
 }
-__device__ __forceinline__ void unpk2(uint64_t v, float& a, float& b) {
-    asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
-}
-__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
-    uint64_t r;
-    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
-}
-__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
-    uint64_t r;
-    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
-}
-__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
-    uint64_t r;
-    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+    uint32_t r;
+    asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
     return r;
 }
 
-// The 8 codes of one 32-bit word w (code t of the word at bits 4t) as pairs (code t of the
-// low half, code t of the high half) minus 8, times xs[t] = (x[t], x[t + 4]) * 16^-t,
-// summed over t: the pair (sum over the low codes, sum over the high codes).
-__device__ __forceinline__ uint64_t dot8_w4(uint32_t w, const uint64_t (&xs)[4]) {
-    const uint32_t lo = w, hi = w >> 16;
-    const uint64_t c0 = pk2(-8388616.0f, -8388616.0f), c1 = pk2(-8388736.0f, -8388736.0f),
-                   c2 = pk2(-8390656.0f, -8390656.0f), c3 = pk2(-8421376.0f, -8421376.0f);
-    auto code2 = [&](uint32_t mask) {
-        return pk2(__uint_as_float((lo & mask) | 0x4B000000u), __uint_as_float((hi & mask) | 0x4B000000u));
-    };
-    uint64_t s = mul2(add2(code2(0x000Fu), c0), xs[0]);
-    s = fma2(add2(code2(0x00F0u), c1), xs[1], s);
-    s = fma2(add2(code2(0x0F00u), c2), xs[2], s);
-    s = fma2(add2(code2(0xF000u), c3), xs[3], s);
-    return s;
+// The 8 codes of word q as four bf16 pairs (c - 8): P[0] = (c0, c4), P[1] = (c1, c5),
+// P[2] = (c2, c6), P[3] = (c3, c7) (low half first).  A nibble or-ed into the low mantissa
+// bits of bf16 128 (exponent 134, mantissa unit 1) reads 128 + c; bf16 has 7 mantissa
+// bits, so each nibble is first shifted down to bits 0-3 (at bits 4-7 it would reach the
+// exponent).
+__device__ __forceinline__ void dequant8(uint32_t q, uint32_t (&P)[4]) {
+    constexpr uint32_t kE128 = 0x43004300u;  // bf16 (128, 128)
+    constexpr uint32_t k136 = 0x43084308u;   // bf16 (136, 136)
+    P[0] = sub_bf2(lop_or(q, 0x000F000Fu, kE128), k136);
+    P[1] = sub_bf2(lop_or(q >> 4, 0x000F000Fu, kE128), k136);
+    P[2] = sub_bf2(lop_or(q >> 8, 0x000F000Fu, kE128), k136);
+    P[3] = sub_bf2(lop_or(q >> 12, 0x000F000Fu, kE128), k136);
 }
 
-__device__ __forceinline__ float bf_lo(uint32_t w) { return __uint_as_float(w << 16); }
-__device__ __forceinline__ float bf_hi(uint32_t w) { return __uint_as_float(w & 0xFFFF0000u); }
+__device__ __forceinline__ void mma_bf16(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, "
+        "{%8, %9}, {%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
 
-template <int ROWS, int MAXM>
+// Named barrier 1 over the 4 consumer warps; the second form also returns whether any of
+// their threads passed v = true (the same answer in all of them).
+__device__ __forceinline__ void consumers_sync() {
+    asm volatile("bar.sync 1, 128;" ::: "memory");
+}
+__device__ __forceinline__ bool consumers_sync_any(bool v) {
+    uint32_t r;
+    asm volatile(
+        "{\n\t.reg .pred p, q;\n\t"
+        "setp.ne.u32 p, %1, 0;\n\t"
+        "barrier.cta.red.or.pred q, 1, 128, p;\n\t"
+        "selp.u32 %0, 1, 0, q;\n\t}"
+        : "=r"(r)
+        : "r"((uint32_t)v)
+        : "memory");
+    return r != 0;
+}
+
+template <int ROWS>
 __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_constant__ GemvW4Params p) {
-    constexpr int RW = ROWS / 4;
-    constexpr uint32_t kWBytes = ROWS * kWRowBytes;
+    constexpr int kTiles = ROWS / 16;                 // 16-row MMA tiles per stage
+    constexpr uint32_t kBoxBytes = ROWS * 128;        // one 256-code quarter of ROWS rows
+    constexpr uint32_t kWBytes = 4 * kBoxBytes;
     constexpr uint32_t kSBytes = ROWS * kGroupsPerStage * 2;
-    static_assert(ROWS % 8 == 0 && ROWS <= 256, "rows per stage");
+    static_assert(ROWS == 16 || ROWS == 32, "rows per stage");
     extern __shared__ uint8_t gsm_raw[];
     __shared__ __align__(8) uint64_t bars[2 * kMaxStages];
     __shared__ int abort_word;
+    __shared__ float red[4][ROWS][8];                 // per-warp partial sums of an item
     volatile int* abort_flag = &abort_word;
 
     const int S = p.stages, M = p.M;
-    const uint32_t xbytes = (uint32_t)M * kKc * 2;  // four boxes of [M][256]
-    const uint32_t stage_bytes = kWBytes + kSBytes + xbytes;
-    const uint32_t base = (ptx::smem_u32(gsm_raw) + 127u) & ~127u;
-    const uint8_t* gbase = gsm_raw + (base - ptx::smem_u32(gsm_raw));  // generic address of `base`
-    auto w_at = [&](int s) { return base + (uint32_t)s * stage_bytes; };
-    auto s_at = [&](int s) { return w_at(s) + kWBytes; };
-    auto x_at = [&](int s) { return w_at(s) + kWBytes + kSBytes; };
+    const uint32_t xbytes = (uint32_t)M * kKc * 2;
+    const uint32_t stride = (kWBytes + xbytes + kSBytes + 1023u) & ~1023u;
+    const uint32_t base = (ptx::smem_u32(gsm_raw) + 1023u) & ~1023u;
+    const uint8_t* gbase = gsm_raw + (base - ptx::smem_u32(gsm_raw));
+    auto w_at = [&](int s) { return base + (uint32_t)s * stride; };
+    auto x_at = [&](int s) { return w_at(s) + kWBytes; };
+    auto s_at = [&](int s) { return w_at(s) + kWBytes + xbytes; };
     auto full_bar = [&](int s) { return ptx::smem_u32(bars + s); };
     auto empty_bar = [&](int s) { return ptx::smem_u32(bars + kMaxStages + s); };
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const uint32_t tx_bytes = kWBytes + kSBytes + xbytes;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -158,13 +179,17 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
             ptx::prefetch_tmap(&p.tmap_x);
             const uint64_t pol = ptx::l2_policy_evict_first();
             auto load_w = [&](int st, int c, int g) {  // codes and scales of chunk c, row group g
-                ptx::tma_load_2d_hint(w_at(st), &p.tmap_w, c * (kKc / 8), g * ROWS, full_bar(st), pol);
+#pragma unroll
+                for (int b = 0; b < 4; ++b)
+                    ptx::tma_load_2d_hint(w_at(st) + b * kBoxBytes, &p.tmap_w, c * (kKc / 8) + b * (kQuarter / 8),
+                                          g * ROWS, full_bar(st), pol);
                 ptx::tma_load_2d_hint(s_at(st), &p.tmap_s, g * ROWS, c * kGroupsPerStage, full_bar(st), pol);
             };
             auto load_x = [&](int st, int c) {
 #pragma unroll
-                for (int j = 0; j < kKc / kXBox; ++j)
-                    ptx::tma_load_2d(x_at(st) + j * M * kXBox * 2, &p.tmap_x, c * kKc + j * kXBox, 0, full_bar(st));
+                for (int j = 0; j < 4; ++j)
+                    ptx::tma_load_2d(x_at(st) + j * M * kQuarter * 2, &p.tmap_x, c * kKc + j * kQuarter, 0,
+                                     full_bar(st));
             };
             int stage = 0;
             uint32_t phase = 0;
@@ -174,13 +199,15 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
             if (p.b_const && (int)blockIdx.x < p.items) {
                 const Item first = item_of(blockIdx.x, p);
                 for (int c = first.c0; c < first.c1 && pre < S; ++c, ++pre) {
-                    ptx::mbar_arrive_expect_tx(full_bar(pre), stage_bytes);
+                    ptx::mbar_arrive_expect_tx(full_bar(pre), tx_bytes);
                     load_w(pre, c, first.g);
                     pre_chunk[pre] = c;
                 }
                 const int pf_end = min(first.c1, first.c0 + pre + p.pf_chunks);
                 for (int c = first.c0 + pre; c < pf_end; ++c)
-                    ptx::tma_prefetch_l2_2d(&p.tmap_w, c * (kKc / 8), first.g * ROWS);
+#pragma unroll
+                    for (int b = 0; b < 4; ++b)
+                        ptx::tma_prefetch_l2_2d(&p.tmap_w, c * (kKc / 8) + b * (kQuarter / 8), first.g * ROWS);
             }
             ptx::griddep_wait();
             ptx::griddep_launch_dependents();
@@ -199,7 +226,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
                         ok = false;
                         break;
                     }
-                    ptx::mbar_arrive_expect_tx(full_bar(stage), stage_bytes);
+                    ptx::mbar_arrive_expect_tx(full_bar(stage), tx_bytes);
                     load_w(stage, c, w.g);
                     load_x(stage, c);
                     armed |= 1u << stage;
@@ -223,53 +250,75 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
 
     // ---------------------------------------------------------------------- consumers
     ptx::griddep_wait();
-    const int cw = warp - 1;
+    const int cw = warp - 1;          // K quarter of every stage
+    const int g = lane >> 2, t = lane & 3;
+    const bool tok = g < M;           // this lane's B column is a real row of x
+    // MMA row g of a tile is stage row sg (and g + 8 is sg + 8): g = 2i and 2i + 1 land
+    // in different halves of the 128-byte swizzle, so the 8 lanes of a 16-byte load phase
+    // read 8 distinct bank quads.
+    const int sg = ((g & 1) << 2) | (g >> 1);
+    // Thread t takes the 4 words of its 16-byte unit in the order pp ^ rot: the x reads of
+    // t and t + 2 (64 bytes apart) then hit different bank quads.
+    const int rot = t & 2;
     int stage = 0;
     uint32_t phase = 0;
     for (int it = blockIdx.x; it < p.items; it += gridDim.x) {
         const Item w = item_of(it, p);
-        uint64_t acc2[RW][MAXM];
+        float acc[kTiles][4];
 #pragma unroll
-        for (int r = 0; r < RW; ++r)
+        for (int r = 0; r < kTiles; ++r)
 #pragma unroll
-            for (int m = 0; m < MAXM; ++m) acc2[r][m] = 0ull;  // (+0.0f, +0.0f)
-        bool ok = true;
+            for (int j = 0; j < 4; ++j) acc[r][j] = 0.0f;
         for (int c = w.c0; c < w.c1; ++c) {
-            if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrFull)) {
-                ok = false;
-                break;
-            }
+            // one answer for the whole warp: mma.sync needs all 32 lanes
+            const bool ready = ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrFull);
+            if (!__all_sync(0xffffffffu, ready)) break;
             const uint8_t* wst = gbase + (w_at(stage) - base);
-            const uint32_t* codes = reinterpret_cast<const uint32_t*>(wst) + lane;
-            const uint16_t* sc = reinterpret_cast<const uint16_t*>(wst + kWBytes);
-            const uint8_t* xst = wst + kWBytes + kSBytes;
+            const uint8_t* box = wst + cw * kBoxBytes;
+            const uint8_t* xq = wst + kWBytes + (cw * M + (tok ? g : 0)) * kQuarter * 2;
+            const uint16_t* sc = reinterpret_cast<const uint16_t*>(wst + kWBytes + xbytes);
 #pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                // (x[m][8l + 256i + t], x[m][8l + 256i + t + 4]) * 16^-t, t = 0..3
-                uint64_t xs[MAXM][4];
+            for (int h = 0; h < 2; ++h) {  // scale group 2 cw + h of the stage
+                // x[g][128h + 32t + 8(pp ^ rot) .. +7], as the B pairs of MMA 1 and 2
+                uint32_t B[4][4];
 #pragma unroll
-                for (int m = 0; m < MAXM; ++m) {
-                    if (m < M) {
-                        const uint4 v = *reinterpret_cast<const uint4*>(xst + (i * M + m) * kXBox * 2 + lane * 16);
-                        xs[m][0] = pk2(bf_lo(v.x), bf_lo(v.z));
-                        xs[m][1] = mul2(pk2(bf_hi(v.x), bf_hi(v.z)), pk2(0.0625f, 0.0625f));
-                        xs[m][2] = mul2(pk2(bf_lo(v.y), bf_lo(v.w)), pk2(0.00390625f, 0.00390625f));
-                        xs[m][3] = mul2(pk2(bf_hi(v.y), bf_hi(v.w)), pk2(0.000244140625f, 0.000244140625f));
-                    } else {
-#pragma unroll
-                        for (int t = 0; t < 4; ++t) xs[m][t] = 0ull;
-                    }
+                for (int pp = 0; pp < 4; ++pp) {
+                    uint4 v = make_uint4(0, 0, 0, 0);
+                    if (tok) v = *reinterpret_cast<const uint4*>(xq + (128 * h + 32 * t + 8 * (pp ^ rot)) * 2);
+                    B[pp][0] = prmt(v.x, v.z, 0x5410u);  // (x0, x4)
+                    B[pp][1] = prmt(v.x, v.z, 0x7632u);  // (x1, x5)
+                    B[pp][2] = prmt(v.y, v.w, 0x5410u);  // (x2, x6)
+                    B[pp][3] = prmt(v.y, v.w, 0x7632u);  // (x3, x7)
                 }
-                const int grp = 2 * i + (lane >> 4);
+                const int grp = 2 * cw + h;
+                // 16-byte unit 4h + t of a row, at (4h + t) ^ (row % 8) under the swizzle
+                const uint32_t u = (uint32_t)(4 * h + t) ^ (uint32_t)sg;
 #pragma unroll
-                for (int r = 0; r < RW; ++r) {
-                    const int row = cw * RW + r;
-                    const uint32_t code = codes[row * (kWRowBytes / 4) + i * 32];
-                    const float scale = __uint_as_float((uint32_t)sc[grp * ROWS + row] << 16);
-                    const uint64_t scale2 = pk2(scale, scale);
+                for (int r = 0; r < kTiles; ++r) {
+                    const int r0 = 16 * r + sg, r1 = r0 + 8;
+                    uint4 q0 = *reinterpret_cast<const uint4*>(box + r0 * 128 + u * 16);
+                    uint4 q1 = *reinterpret_cast<const uint4*>(box + r1 * 128 + u * 16);
+                    if (rot) {
+                        q0 = make_uint4(q0.z, q0.w, q0.x, q0.y);
+                        q1 = make_uint4(q1.z, q1.w, q1.x, q1.y);
+                    }
+                    const uint32_t w0[4] = {q0.x, q0.y, q0.z, q0.w}, w1[4] = {q1.x, q1.y, q1.z, q1.w};
+                    // two accumulation chains (codes (c0, c4, c1, c5) and (c2, c6, c3, c7))
+                    float d[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e[4] = {0.0f, 0.0f, 0.0f, 0.0f};
 #pragma unroll
-                    for (int m = 0; m < MAXM; ++m)
-                        if (m < M) acc2[r][m] = fma2(scale2, dot8_w4(code, xs[m]), acc2[r][m]);
+                    for (int pp = 0; pp < 4; ++pp) {
+                        uint32_t P0[4], P1[4];
+                        dequant8(w0[pp], P0);
+                        dequant8(w1[pp], P1);
+                        mma_bf16(d, P0[0], P1[0], P0[1], P1[1], B[pp][0], B[pp][1]);
+                        mma_bf16(e, P0[2], P1[2], P0[3], P1[3], B[pp][2], B[pp][3]);
+                    }
+                    const float s0 = __uint_as_float((uint32_t)sc[grp * ROWS + r0] << 16);
+                    const float s1 = __uint_as_float((uint32_t)sc[grp * ROWS + r1] << 16);
+                    acc[r][0] = fmaf(s0, d[0] + e[0], acc[r][0]);
+                    acc[r][1] = fmaf(s0, d[1] + e[1], acc[r][1]);
+                    acc[r][2] = fmaf(s1, d[2] + e[2], acc[r][2]);
+                    acc[r][3] = fmaf(s1, d[3] + e[3], acc[r][3]);
                 }
             }
             __syncwarp();
@@ -279,58 +328,46 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
                 phase ^= 1u;
             }
         }
-        if (!ok) break;
-        float acc[RW][MAXM];
+        // the four K quarters meet: D element (row, token 2t + j) of tile r
 #pragma unroll
-        for (int r = 0; r < RW; ++r)
-#pragma unroll
-            for (int m = 0; m < MAXM; ++m) {
-                float a, b;
-                unpk2(acc2[r][m], a, b);
-                acc[r][m] = a + b;
-                if (m < M) {
-                    float v = acc[r][m];
-#pragma unroll
-                    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-                    acc[r][m] = v;
-                }
-            }
-        if (lane == 0) {
-#pragma unroll
-            for (int r = 0; r < RW; ++r) {
-                const int n = w.g * ROWS + cw * RW + r;
+        for (int r = 0; r < kTiles; ++r) {
+            red[cw][16 * r + sg][2 * t] = acc[r][0];
+            red[cw][16 * r + sg][2 * t + 1] = acc[r][1];
+            red[cw][16 * r + sg + 8][2 * t] = acc[r][2];
+            red[cw][16 * r + sg + 8][2 * t + 1] = acc[r][3];
+        }
+        // one vote for all four warps, so that they leave the item loop together
+        const bool aborted = consumers_sync_any(*abort_flag != 0);
+        if (!aborted) {
+            for (int o = threadIdx.x - 32; o < ROWS * M; o += 128) {
+                const int row = o / M, m = o % M;
+                const int n = w.g * ROWS + row;
                 if (n >= p.N) continue;
-#pragma unroll
-                for (int m = 0; m < MAXM; ++m) {
-                    if (m >= M) continue;
-                    if (p.split == 1)
-                        p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act);
-                    else
-                        p.ws[((long long)w.s * M + m) * p.N + n] = acc[r][m];
-                }
+                const float v = ((red[0][row][m] + red[1][row][m]) + red[2][row][m]) + red[3][row][m];
+                if (p.split == 1)
+                    p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? v + p.bias[n] : v, p.act);
+                else
+                    p.ws[((long long)w.s * M + m) * p.N + n] = v;
             }
         }
+        consumers_sync();
+        if (aborted) break;
     }
 }
 
 using GemvW4Kernel = void (*)(GemvW4Params);
-// Instance table, indexed as gemv_w4_instance() - kGemvW4FirstInstance:
-// (ROWS 8, 16, 32) x (MAXM 1, 8).
-const GemvW4Kernel kKernels[6] = {
-    gemv_w4_kernel<8, 1>,  gemv_w4_kernel<8, 8>,  gemv_w4_kernel<16, 1>,
-    gemv_w4_kernel<16, 8>, gemv_w4_kernel<32, 1>, gemv_w4_kernel<32, 8>,
-};
-const int kRowsOf[6] = {8, 8, 16, 16, 32, 32};
-const int kMaxMOf[6] = {1, 8, 1, 8, 1, 8};
+// Instance table, indexed as gemv_w4_instance() - kGemvW4FirstInstance: ROWS 16, 32.
+const GemvW4Kernel kKernels[2] = {gemv_w4_kernel<16>, gemv_w4_kernel<32>};
+const int kRowsOf[2] = {16, 32};
 
 std::mutex g_mu;
-int g_smem[6] = {0};
+int g_smem[2] = {0, 0};
 
 }  // namespace
 
 bool gemv_uses_w4(const nnjit_candidate& c) {
     return c.family == NNJIT_FAMILY_GEMV && c.instance >= kGemvW4FirstInstance &&
-           c.instance < kGemvW4FirstInstance + 6;
+           c.instance < kGemvW4FirstInstance + 2;
 }
 
 cudaError_t encode_gemv_w4_maps(const Problem& p, const nnjit_candidate& c, const void* A, const void* B,
@@ -341,7 +378,7 @@ cudaError_t encode_gemv_w4_maps(const Problem& p, const nnjit_candidate& c, cons
         return cudaErrorNotSupported;
     }
     const int i = c.instance - kGemvW4FirstInstance;
-    if (i < 0 || i >= 6 || p.M < 1 || p.M > 8) {
+    if (i < 0 || i >= 2 || p.M < 1 || p.M > 8) {
         *why = "not a 4-bit GEMV candidate";
         return cudaErrorInvalidValue;
     }
@@ -350,9 +387,9 @@ cudaError_t encode_gemv_w4_maps(const Problem& p, const nnjit_candidate& c, cons
     {
         const cuuint64_t dims[2] = {(cuuint64_t)((p.K + 7) / 8), (cuuint64_t)p.N};
         const cuuint64_t strides[1] = {(cuuint64_t)(p.ldb / 2)};
-        const cuuint32_t box[2] = {(cuuint32_t)(kKc / 8), (cuuint32_t)kRowsOf[i]};
+        const cuuint32_t box[2] = {(cuuint32_t)(kQuarter / 8), (cuuint32_t)kRowsOf[i]};
         if (enc(tw, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<char*>(blob), dims, strides, box, estr,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
             *why = "cuTensorMapEncodeTiled failed for the 4-bit codes";
             return cudaErrorInvalidValue;
@@ -372,7 +409,7 @@ cudaError_t encode_gemv_w4_maps(const Problem& p, const nnjit_candidate& c, cons
     {
         const cuuint64_t dims[2] = {(cuuint64_t)p.K, (cuuint64_t)p.M};
         const cuuint64_t strides[1] = {(cuuint64_t)(p.lda * 2)};
-        const cuuint32_t box[2] = {(cuuint32_t)kXBox, (cuuint32_t)p.M};
+        const cuuint32_t box[2] = {(cuuint32_t)kQuarter, (cuuint32_t)p.M};
         if (enc(tx, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(A), dims, strides, box, estr,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
@@ -387,11 +424,11 @@ cudaError_t launch_gemv_w4(const LaunchArgs& a) {
     const Problem& p = *a.p;
     const nnjit_candidate& c = *a.c;
     const int i = c.instance - kGemvW4FirstInstance;
-    if (i < 0 || i >= 6 || !a.tmap_a || !a.tmap_b || !a.tmap_c || p.dtype != NNJIT_W4_BF16 ||
+    if (i < 0 || i >= 2 || !a.tmap_a || !a.tmap_b || !a.tmap_c || p.dtype != NNJIT_W4_BF16 ||
         p.b_layout != NNJIT_B_NK)
         return cudaErrorInvalidValue;
-    if (p.M < 1 || p.M > kMaxMOf[i] || c.bn != kRowsOf[i] || c.stages < 2 || c.stages > kMaxStages ||
-        c.split_k < 1 || c.threads != kThreads || c.bk != kKc)
+    if (p.M < 1 || p.M > 8 || c.bn != kRowsOf[i] || c.stages < 2 || c.stages > kMaxStages || c.split_k < 1 ||
+        c.threads != kThreads || c.bk != kKc)
         return cudaErrorInvalidValue;
     GemvW4Params prm;
     prm.tmap_x = *a.tmap_a;
@@ -417,11 +454,11 @@ cudaError_t launch_gemv_w4(const LaunchArgs& a) {
     const int grid = (int)std::min<long long>(items, std::max(1, c.grid));
     prm.pf_chunks = 0;
     if (prm.b_const) {
-        const long long per_cta = kPrefetchBytes / grid / ((long long)kRowsOf[i] * kWRowBytes);
+        const long long per_cta = kPrefetchBytes / grid / ((long long)kRowsOf[i] * (kKc / 2));
         prm.pf_chunks = (int)std::min<long long>(per_cta, prm.cps);
     }
-    const int stage_bytes = kRowsOf[i] * (kWRowBytes + kGroupsPerStage * 2) + (int)p.M * kKc * 2;
-    const int smem = 128 + c.stages * stage_bytes;
+    const int stride = (kRowsOf[i] * (kKc / 2) + (int)p.M * kKc * 2 + kRowsOf[i] * kGroupsPerStage * 2 + 1023) / 1024 * 1024;
+    const int smem = 1024 + c.stages * stride;
     {
         std::lock_guard<std::mutex> lk(g_mu);
         if (g_smem[i] < smem) {

@@ -91,7 +91,7 @@ EncodeTiledFn get_encode_fn();
 // GEMV candidates whose weights are streamed by TMA (instances kGemvTmaFirstInstance..+5).
 bool gemv_uses_tma(const nnjit_candidate& c);
 cudaError_t launch_gemv_tma(const LaunchArgs& a);
-// GEMV candidates over 4-bit weights (instances kGemvW4FirstInstance..+5); LaunchArgs'
+// GEMV candidates over 4-bit weights (instances kGemvW4FirstInstance..+1); LaunchArgs'
 // tmap_a, tmap_b, tmap_c are the maps of x, the codes and the group scales.
 bool gemv_uses_w4(const nnjit_candidate& c);
 cudaError_t launch_gemv_w4(const LaunchArgs& a);

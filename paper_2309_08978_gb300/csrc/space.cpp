@@ -266,19 +266,19 @@ void ffma_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 // that set the bytes in flight per SM: threads per CTA, rows per warp, 16-byte loads in
 // flight per lane and row (unroll), and split-K.
 // ---------------------------------------------------------------------------------
-// 4-bit weights (NNJIT_W4_BF16): the TMA-fed kernel only.  A ring stage holds `rows`
-// weight rows x 1024 codes (512 bytes a row), their 8 group scales, and the matching
-// 1024-element slice of every row of x; axes rows per stage, ring stages, split-K.
+// 4-bit weights (NNJIT_W4_BF16): the TMA-fed tensor-core kernel only.  A ring stage
+// holds `rows` weight rows x 1024 codes (512 bytes a row, four 128-byte-swizzled boxes),
+// the 1024-element slice of every row of x and the rows' 8 group scales, padded to 1 KB;
+// axes rows per stage (16-row MMA tiles), ring stages, split-K.
 void gemv_w4_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_candidate>& v,
                    int64_t* naive) {
     using MC = ModelConstants;
     const int64_t M = std::max<int64_t>(p.M, 1), N = std::max<int64_t>(p.N, 1);
     const int64_t K = std::max<int64_t>(p.K, 1);
     const int64_t wbytes = N * K / 2 + ceil_div(K, 128) * N * 2;
-    const int maxm = M == 1 ? 1 : MC::kGemvMaxM;
     const int64_t chunks = ceil_div(K, MC::kGemvW4Kc);
-    *naive = 3 * 2 * 4;
-    for (int rows : {8, 16, 32}) {
+    *naive = 2 * 2 * 4;
+    for (int rows : {16, 32}) {
         const int64_t groups = ceil_div(N, rows);
         for (int stages : {4, 8}) {
             for (int split : {1, 2, 4, 8}) {
@@ -286,10 +286,12 @@ void gemv_w4_space(const Problem& p, const nnjit_device_limits& L, std::vector<n
                 if (split > 1 && (cps < 2 || (split - 1) * cps >= chunks ||
                                   groups * (split / 2) >= 2LL * L.sm_count))
                     continue;
-                const int64_t stage_bytes = rows * (MC::kGemvW4Kc / 2 + 16) + M * MC::kGemvW4Kc * 2;
-                const int64_t smem = 128 + stages * stage_bytes;
+                const int64_t stage_bytes =
+                    ceil_div(rows * (MC::kGemvW4Kc / 2 + 16) + M * MC::kGemvW4Kc * 2, 1024) * 1024;
+                // dynamic (1 KB alignment slack + ring) and static (barriers, partial sums)
+                const int64_t smem = 1024 + stages * stage_bytes + 256 + rows * 128;
                 if (smem > L.smem_per_block_optin) continue;
-                const int regs = maxm == 1 ? 72 : 104 + 5 * rows;  // ptxas: 58-68 / 144-252
+                const int regs = rows == 16 ? 88 : 112;  // ptxas: 84 / 110
                 const int blk = blocks_per_core(L, regs, MC::kGemvTmaThreads, (int)smem, 0);
                 if (blk < 1) continue;
                 const int64_t items = groups * split;
@@ -298,7 +300,7 @@ void gemv_w4_space(const Problem& p, const nnjit_device_limits& L, std::vector<n
                 nnjit_candidate c = blank();
                 c.family = NNJIT_FAMILY_GEMV;
                 c.bm = (int)M; c.bn = rows; c.bk = MC::kGemvW4Kc;
-                c.tm = rows / 4; c.tn = 1;
+                c.tm = rows / 16; c.tn = 1;
                 c.stages = stages;
                 c.split_k = split;
                 c.threads = MC::kGemvTmaThreads;
@@ -315,7 +317,7 @@ void gemv_w4_space(const Problem& p, const nnjit_device_limits& L, std::vector<n
                 if (split > 1)
                     cost += MC::kLaunchClk + ceil_div(2LL * split * M * N * 4, MC::kHbmBytesPerClk);
                 c.predicted_cost = cost;
-                c.instance = gemv_w4_instance(rows, maxm);
+                c.instance = gemv_w4_instance(rows);
                 v.push_back(c);
             }
         }
@@ -513,11 +515,9 @@ int gemv_instance(int b_layout, int rows, int unroll) {
     return ri * 2 + ui;
 }
 
-int gemv_w4_instance(int rows, int maxm) {
-    const int ri = rows == 8 ? 0 : rows == 16 ? 1 : rows == 32 ? 2 : -1;
-    const int mi = maxm == 1 ? 0 : maxm == ModelConstants::kGemvMaxM ? 1 : -1;
-    if (ri < 0 || mi < 0) return -1;
-    return kGemvW4FirstInstance + ri * 2 + mi;
+int gemv_w4_instance(int rows) {
+    const int ri = rows == 16 ? 0 : rows == 32 ? 1 : -1;
+    return ri < 0 ? -1 : kGemvW4FirstInstance + ri;
 }
 
 int gemv_tma_instance(int rows, int maxm) {

@@ -85,6 +85,6 @@ constexpr int kGemvTmaFirstInstance = 8;
 int gemv_tma_instance(int rows, int maxm);                     // 8..13, -1 if none
 // TMA-fed GEMV over 4-bit weights (NNJIT_W4_BF16): rows per stage 8/16/32, maxm 1 or 8.
 constexpr int kGemvW4FirstInstance = 14;
-int gemv_w4_instance(int rows, int maxm);                      // 14..19, -1 if none
+int gemv_w4_instance(int rows);                                // 14..15, -1 if none
 
 }  // namespace nnjit
