@@ -331,6 +331,29 @@ def run_ours(args, workload, rank, world, local_rank):
         nj.nnjit_cache_load(args.cache)
     items = []
     tune = {"budget_ms_per_shape": args.budget_ms, "shapes": []}
+    free_sizes = {}
+    if args.study:
+        # Sec. 5.1: fix the settings a one-variable-at-a-time microbenchmark finds
+        # consistently better (a 4096^3 product per tensor-core dtype plus the workload's
+        # own tensor-core products), then build every space with them
+        tc_shapes = [s for s in workload.shapes if dtype in ("bf16", "tf32") and s.M > 8]
+        descs = [nj.make_desc(4096, 4096, 4096, dt, "NK") for dt in ("bf16", "tf32")]
+        descs += [nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch, has_bias=s.has_bias)
+                  for s in tc_shapes]
+        for s in workload.shapes:
+            d = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch, has_bias=s.has_bias)
+            free_sizes[id(s)] = len(nj.nnjit_space_enumerate(d, lim)[0])
+        t0 = time.perf_counter()
+        fixed, report = nj.nnjit_settings_study(descs)
+        study_ms = 1000 * (time.perf_counter() - t0)
+        nj.nnjit_settings_set(fixed)
+        tune["settings"] = {
+            "fixed": fixed, "study_ms": round(study_ms, 1),
+            "products": [{"shape": [p["batch"], p["M"], p["N"], p["K"]], "dtype": p["dtype"],
+                          "space_size": p["space_size"], "best_us": round(p["best_us"], 3),
+                          "verdicts": {a: [e["value"], e["twin_value"], round(e["twin_us"], 3), e["verdict"]]
+                                       for a, e in p["settings"].items()}}
+                         for p in report["products"]]}
     for s in workload.shapes:
         A, B, bias = make_operands(s, workload.index, dtype)
         bflag = nj.NNJIT_PLAN_B_CONSTANT if s.b_is_weight else 0   # weights never change
@@ -342,6 +365,7 @@ def run_ours(args, workload, rank, world, local_rank):
         info = plan.describe()
         entry = {"shape": [s.batch, s.M, s.N, s.K], "plan_ms": round(plan_ms, 2),
                  "space_size": info["space_size"], "naive_space": info["naive_space"],
+                 **({"space_size_free": free_sizes[id(s)]} if id(s) in free_sizes else {}),
                  "chosen_index": info["chosen_index"], "family": info["family"],
                  "candidate": {k: info["candidate"][k] for k in ("bm", "bn", "bk", "stages", "split_k", "raster")}}
         if not args.no_sweep:
@@ -558,6 +582,8 @@ def main(argv=None):
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
     ap.add_argument("--budget-ms", type=float, default=2000.0, help="tuning budget per product")
     ap.add_argument("--no-sweep", action="store_true", help="skip the exhaustive sweep")
+    ap.add_argument("--study", action="store_true",
+                    help="run the fixed-settings microbenchmark first and plan with its settings")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--e2e-steps", type=int, default=200)

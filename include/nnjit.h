@@ -185,6 +185,29 @@ typedef struct {
 
 typedef struct nnjit_plan_s* nnjit_plan;
 
+/*
+ * Fixed settings (the primitive vector of Sec. 5.1): settings that offline
+ * microbenchmarks found consistently better are fixed before the lite space is built,
+ * which shrinks the space.  Each field is NNJIT_SETTING_FREE (searched; the default) or
+ * the one value kept.  They act on the tensor-core family only:
+ *   raster     tile order: 0 = M fastest, 1 = N fastest;
+ *   kgroup     k-blocks per ring slot (candidate bk / one 128-byte k-block): 1 or 2;
+ *   reduce     split-K reduction: 0 = second kernel, 1 = inside a cluster (DSMEM);
+ *   multicast  128 x 256 tiles as TMA-multicast pairs (cluster_m = 2, bm = 128): 0 or 1.
+ * A fixed value removes a candidate only where the same candidate with the fixed value
+ * (every other searched field equal: bm, bn, split_k and the other three settings) is
+ * in the space, so a setting never empties the space and never removes the only legal
+ * choice (for example kgroup = 2 keeps bn = 256 tiles, which exist only with 1).  The
+ * axes are applied in the order above.
+ */
+#define NNJIT_SETTING_FREE (-1)
+typedef struct {
+    int32_t raster;
+    int32_t kgroup;
+    int32_t reduce;
+    int32_t multicast;
+} nnjit_settings;
+
 /* ---------------------------------------------------------------------------------- */
 
 /* Static string for a status code.  Never NULL. */
@@ -205,7 +228,8 @@ nnjit_status nnjit_device_limits_query(int32_t device, nnjit_device_limits* out)
  * Table 1: enumerate power-of-two tiles (heuristic 2), keep those whose shared memory,
  * TMEM, register and thread usage fit the device, compute Block_core =
  * min(RegLimit, L1Limit, WarpLimit, ...), and order the survivors from most to fewest
- * blocks per core, then by the predicted cost.  Writes at most `capacity` candidates to
+ * blocks per core, then by the predicted cost; then drop what the process-wide fixed
+ * settings (nnjit_settings_set) exclude.  Writes at most `capacity` candidates to
  * `out` (may be NULL when capacity is 0), the full count to *count, and the size of the
  * unpruned space (every tile/stage/split combination of the family's axes before the
  * usage rules and heuristics) to *naive_count (may be NULL).
@@ -214,6 +238,34 @@ nnjit_status nnjit_device_limits_query(int32_t device, nnjit_device_limits* out)
 nnjit_status nnjit_space_enumerate(const nnjit_matmul_desc* d, const nnjit_device_limits* lim,
                                    nnjit_candidate* out, int32_t capacity, int32_t* count,
                                    int64_t* naive_count);
+
+/*
+ * Set (or, with s = NULL, clear) the process-wide fixed settings used by every later
+ * nnjit_space_enumerate and plan call; the plan cache keys include them.  INVALID_ARG for
+ * a value outside the field's range (FREE or the values listed above).  Thread-safe.
+ */
+nnjit_status nnjit_settings_set(const nnjit_settings* s);
+
+/* The current process-wide fixed settings. */
+nnjit_status nnjit_settings_get(nnjit_settings* out);
+
+/*
+ * One-variable-at-a-time microbenchmark (Sec. 5.1) over the products `descs[0..count)`
+ * on the current device: each product's full space (every setting searched, the current
+ * fixed settings ignored) is timed exhaustively as by NNJIT_PLAN_EXHAUSTIVE; then, from
+ * its fastest candidate, each setting is flipped alone and the two times compared.  A
+ * flip more than 2 % slower is a decisive vote for the fastest candidate's value; a
+ * smaller difference is a tie; a setting whose flipped twin is not in the space has no
+ * vote.  *out receives, per setting, the value every decisive vote agreed on, or FREE
+ * when there was no decisive vote or the votes disagreed.  Nothing is applied: pass *out
+ * to nnjit_settings_set.  `report` (may be NULL) receives a JSON object with each
+ * product's space size, fastest candidate and per-setting times and verdicts; the
+ * length it needs (with the NUL) is stored in *report_needed (may be NULL).  The plan
+ * cache is neither read nor written.  Synchronises the device.  INVALID_ARG for
+ * count < 1 or a bad descriptor; the first failing product's status otherwise.
+ */
+nnjit_status nnjit_settings_study(const nnjit_matmul_desc* descs, int32_t count, nnjit_settings* out,
+                                  char* report, size_t report_len, size_t* report_needed);
 
 /*
  * JIT-tune a plan for C[M,N] = A[M,K] . B[K,N] (B_KN, batch 1, packed, with a bias slot

@@ -518,8 +518,62 @@ def _gemv(p, lim):
     return out, 2 * 2 * 6
 
 
-def build_space(p: Problem, lim: dict):
-    """Ordered candidates (list of dicts with CANDIDATE_FIELDS) and the unpruned count."""
+SETTING_AXES = ("raster", "kgroup", "reduce", "multicast")
+SETTING_RANGE = {"raster": (0, 1), "kgroup": (1, 2), "reduce": (0, 1), "multicast": (0, 1)}
+
+
+def setting_value(p: Problem, c: dict, axis: str):
+    """The fixed-setting value of a tensor-core candidate (None for other families):
+    tile order, k-blocks per ring slot (bk over one 128-byte k-block), split-K reduction,
+    and whether it is a 128-row multicast pair."""
+    if c["family"] != FAMILY_TC:
+        return None
+    if axis == "raster":
+        return c["raster"]
+    if axis == "kgroup":
+        return c["bk"] // (128 // p.elem)
+    if axis == "reduce":
+        return c["reduce"]
+    return 1 if (c["bm"] == TC_BM and c["cluster_m"] == 2) else 0
+
+
+def _twins(p: Problem, a: dict, b: dict, axis: str) -> bool:
+    """a and b differ in `axis` and agree on every other searched field."""
+    if a["family"] != FAMILY_TC or b["family"] != FAMILY_TC:
+        return False
+    if (a["bm"], a["bn"], a["split_k"]) != (b["bm"], b["bn"], b["split_k"]):
+        return False
+    for o in SETTING_AXES:
+        if o != axis and setting_value(p, a, o) != setting_value(p, b, o):
+            return False
+    return setting_value(p, a, axis) != setting_value(p, b, axis)
+
+
+def apply_settings(p: Problem, cands: list, settings: dict | None) -> list:
+    """Sec. 5.1's fixed settings: for each fixed axis in SETTING_AXES order, drop a
+    candidate whose value differs when its twin with the fixed value is present."""
+    for axis in SETTING_AXES:
+        fixed = (settings or {}).get(axis, -1)
+        if fixed == -1:
+            continue
+        keep = []
+        for c in cands:
+            v = setting_value(p, c, axis)
+            drop = v is not None and v != fixed and any(
+                setting_value(p, t, axis) == fixed and _twins(p, c, t, axis) for t in cands)
+            if not drop:
+                keep.append(c)
+        cands = keep
+    return cands
+
+
+def build_space(p: Problem, lim: dict, settings: dict | None = None):
+    """Ordered candidates (list of dicts with CANDIDATE_FIELDS) and the unpruned count,
+    after the fixed settings (a dict axis -> value; -1 or absent: searched)."""
+    for axis, v in (settings or {}).items():
+        lo, hi = SETTING_RANGE[axis]
+        if v != -1 and not lo <= v <= hi:
+            raise SpaceError(INVALID_ARG)
     if (lim["sm_count"] <= 0 or lim["smem_per_sm"] <= 0 or lim["smem_per_block_optin"] <= 0 or
             lim["regs_per_sm"] <= 0 or lim["max_threads_per_sm"] <= 0 or
             lim["max_blocks_per_sm"] <= 0 or lim["tmem_cols_per_sm"] < 0):
@@ -538,4 +592,4 @@ def build_space(p: Problem, lim: dict):
     # Sec. 5.2: from the most blocks per core to the fewest; then predicted cost; then
     # enumeration order (a stable sort)
     cands.sort(key=lambda c: (-c["blocks_per_sm"], c["predicted_cost"]))
-    return cands, naive
+    return apply_settings(p, cands, settings), naive

@@ -86,6 +86,7 @@ struct nnjit_plan_s {
     double tune_ms = 0.0;
     bool from_cache = false;
     bool timed = false;
+    nnjit_settings settings = nnjit::free_settings();  // the fixed settings its space was built with
     float* ws = nullptr;
     size_t ws_bytes = 0;
     int* err = nullptr;
@@ -139,6 +140,21 @@ std::map<std::string, CacheEntry>& cache() {
     return m;
 }
 
+// Process-wide fixed settings (nnjit_settings_set).
+std::mutex g_set_mu;
+nnjit_settings g_settings = free_settings();
+
+nnjit_settings current_settings() {
+    std::lock_guard<std::mutex> lk(g_set_mu);
+    return g_settings;
+}
+
+bool any_fixed(const nnjit_settings& s) {
+    for (int a = 0; a < kSettingAxes; ++a)
+        if (setting_of(s, a) != NNJIT_SETTING_FREE) return true;
+    return false;
+}
+
 std::mutex g_lim_mu;
 std::map<int, nnjit_device_limits> g_limits;
 std::map<int, std::string> g_dev_name;
@@ -170,7 +186,7 @@ nnjit_status query_limits(int dev, nnjit_device_limits* out) {
     return NNJIT_OK;
 }
 
-std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L) {
+std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L, const nnjit_settings& set) {
     char buf[512];
     std::string name;
     {
@@ -186,6 +202,10 @@ std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L) {
                   name.c_str(), L.cc_major, L.cc_minor, L.sm_count);
     std::string key = buf;
     if (p.epilogue != NNJIT_EPI_NONE) key += "|ep=" + std::to_string(p.epilogue);
+    if (any_fixed(set)) {
+        std::snprintf(buf, sizeof buf, "|set=%d,%d,%d,%d", set.raster, set.kgroup, set.reduce, set.multicast);
+        key += buf;
+    }
     return key;
 }
 
@@ -460,7 +480,7 @@ void free_plan(nnjit_plan pl) {
 
 nnjit_status plan_common(const nnjit_matmul_desc* d, nnjit_plan* out, Problem* prob,
                          nnjit_device_limits* L, int* dev, std::vector<nnjit_candidate>* space,
-                         int64_t* naive) {
+                         int64_t* naive, const nnjit_settings& set) {
     if (!out) return fail(NNJIT_ERR_INVALID_ARG, "out is NULL");
     *out = nullptr;
     std::string err;
@@ -472,7 +492,7 @@ nnjit_status plan_common(const nnjit_matmul_desc* d, nnjit_plan* out, Problem* p
     if (e != cudaSuccess) return cuda_fail(e, "context");
     st = query_limits(*dev, L);
     if (st != NNJIT_OK) return st;
-    st = build_space(*prob, *L, space, naive, &err);
+    st = build_space(*prob, *L, set, space, naive, &err);
     if (st != NNJIT_OK) return fail(st, err);
     return NNJIT_OK;
 }
@@ -603,7 +623,7 @@ nnjit_status nnjit_space_enumerate(const nnjit_matmul_desc* d, const nnjit_devic
     if (st != NNJIT_OK) return fail(st, err);
     std::vector<nnjit_candidate> v;
     int64_t naive = 0;
-    st = build_space(p, *lim, &v, &naive, &err);
+    st = build_space(p, *lim, current_settings(), &v, &naive, &err);
     if (st != NNJIT_OK) return fail(st, err);
     *count = (int32_t)v.size();
     for (int32_t i = 0; i < capacity && i < (int32_t)v.size(); ++i) out[i] = v[i];
@@ -611,7 +631,14 @@ nnjit_status nnjit_space_enumerate(const nnjit_matmul_desc* d, const nnjit_devic
     return NNJIT_OK;
 }
 
-nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, nnjit_plan* out) {
+}  // extern "C"
+
+namespace {
+
+// The body of nnjit_matmul_plan_ex with explicit fixed settings (the settings study
+// builds its spaces with every setting searched).
+nnjit_status plan_ex_impl(const nnjit_matmul_desc* d, double budget_ms, const nnjit_settings& set,
+                          nnjit_plan* out) {
     const double t0 = now_ms();
     if (!(budget_ms >= 0.0)) return fail(NNJIT_ERR_INVALID_ARG, "tune_budget_ms must be >= 0");
     Problem p;
@@ -619,7 +646,7 @@ nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, 
     int dev = 0;
     std::vector<nnjit_candidate> space;
     int64_t naive = 0;
-    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive);
+    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive, set);
     if (st != NNJIT_OK) return st;
     std::unique_ptr<nnjit_plan_s> pl(new nnjit_plan_s);
     pl->p = p;
@@ -627,8 +654,9 @@ nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, 
     pl->family = space[0].family;
     pl->space_size = (int)space.size();
     pl->naive = naive;
+    pl->settings = set;
     const bool use_cache = !(p.flags & NNJIT_PLAN_NO_CACHE) && !(p.flags & NNJIT_PLAN_EXHAUSTIVE);
-    const std::string key = cache_key(p, dev, L);
+    const std::string key = cache_key(p, dev, L, set);
     if (use_cache) {
         std::lock_guard<std::mutex> lk(g_cache_mu);
         auto it = cache().find(key);
@@ -741,6 +769,104 @@ nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, 
     return NNJIT_OK;
 }
 
+}  // namespace
+
+extern "C" {
+
+nnjit_status nnjit_matmul_plan_ex(const nnjit_matmul_desc* d, double budget_ms, nnjit_plan* out) {
+    return plan_ex_impl(d, budget_ms, current_settings(), out);
+}
+
+nnjit_status nnjit_settings_set(const nnjit_settings* s) {
+    const nnjit_settings v = s ? *s : free_settings();
+    std::string err;
+    if (!settings_valid(v, &err)) return fail(NNJIT_ERR_INVALID_ARG, err);
+    std::lock_guard<std::mutex> lk(g_set_mu);
+    g_settings = v;
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_settings_get(nnjit_settings* out) {
+    if (!out) return fail(NNJIT_ERR_INVALID_ARG, "out is NULL");
+    *out = current_settings();
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_settings_study(const nnjit_matmul_desc* descs, int32_t count, nnjit_settings* out,
+                                  char* report, size_t report_len, size_t* report_needed) {
+    if (!descs || count < 1 || !out) return fail(NNJIT_ERR_INVALID_ARG, "need descs, count >= 1 and out");
+    static const char* names[kSettingAxes] = {"raster", "kgroup", "reduce", "multicast"};
+    const nnjit_settings free_set = free_settings();
+    int vote[kSettingAxes];      // value every decisive vote agreed on; -1 none yet; -2 conflict
+    for (int a = 0; a < kSettingAxes; ++a) vote[a] = -1;
+    std::string js = "{\"products\":[";
+    char tmp[512];
+    for (int32_t i = 0; i < count; ++i) {
+        nnjit_matmul_desc d = descs[i];
+        d.flags |= NNJIT_PLAN_EXHAUSTIVE | NNJIT_PLAN_NO_CACHE;
+        nnjit_plan raw = nullptr;
+        nnjit_status st = plan_ex_impl(&d, 0.0, free_set, &raw);
+        if (st != NNJIT_OK) return st;
+        std::unique_ptr<nnjit_plan_s, void (*)(nnjit_plan)> pl(raw, free_plan);
+        const Problem& p = pl->p;
+        nnjit_device_limits L;
+        st = query_limits(pl->device, &L);
+        if (st != NNJIT_OK) return st;
+        std::vector<nnjit_candidate> space;
+        int64_t naive = 0;
+        std::string err;
+        st = build_space(p, L, free_set, &space, &naive, &err);
+        if (st != NNJIT_OK) return fail(st, err);
+        std::vector<double> us(space.size(), -1.0);
+        for (const auto& t : pl->timings)
+            if (t.first >= 0 && t.first < (int)space.size()) us[t.first] = t.second;
+        const int best = pl->chosen_index;
+        std::snprintf(tmp, sizeof tmp,
+                      "%s{\"M\":%lld,\"N\":%lld,\"K\":%lld,\"batch\":%lld,\"dtype\":%d,\"b_layout\":%d,"
+                      "\"space_size\":%d,\"best_index\":%d,\"best_us\":%.4f,\"best\":{\"bm\":%d,\"bn\":%d,"
+                      "\"split_k\":%d,\"raster\":%d,\"kgroup\":%d,\"reduce\":%d,\"multicast\":%d},\"settings\":{",
+                      i ? "," : "", (long long)p.M, (long long)p.N, (long long)p.K, (long long)p.batch, p.dtype,
+                      p.b_layout, (int)space.size(), best, us[best], space[best].bm, space[best].bn,
+                      space[best].split_k, candidate_setting(p, space[best], 0), candidate_setting(p, space[best], 1),
+                      candidate_setting(p, space[best], 2), candidate_setting(p, space[best], 3));
+        js += tmp;
+        for (int a = 0; a < kSettingAxes; ++a) {
+            int twin = -1;
+            for (int j = 0; j < (int)space.size() && twin < 0; ++j)
+                if (setting_twins(p, space[best], space[j], a)) twin = j;
+            const int mine = candidate_setting(p, space[best], a);
+            const char* verdict = "no twin";
+            if (twin >= 0 && us[twin] > 0.0 && us[best] > 0.0) {
+                if (us[twin] > 1.02 * us[best]) {
+                    verdict = "decisive";
+                    vote[a] = (vote[a] == -1 || vote[a] == mine) ? mine : -2;
+                } else {
+                    verdict = "tie";
+                }
+            }
+            std::snprintf(tmp, sizeof tmp, "%s\"%s\":{\"value\":%d,\"twin_value\":%d,\"twin_us\":%.4f,\"verdict\":\"%s\"}",
+                          a ? "," : "", names[a], mine, twin >= 0 ? candidate_setting(p, space[twin], a) : -1,
+                          twin >= 0 ? us[twin] : -1.0, verdict);
+            js += tmp;
+        }
+        js += "}}";
+    }
+    nnjit_settings res = free_set;
+    int* fields[kSettingAxes] = {&res.raster, &res.kgroup, &res.reduce, &res.multicast};
+    for (int a = 0; a < kSettingAxes; ++a) *fields[a] = vote[a] >= 0 ? vote[a] : NNJIT_SETTING_FREE;
+    std::snprintf(tmp, sizeof tmp, "],\"fixed\":{\"raster\":%d,\"kgroup\":%d,\"reduce\":%d,\"multicast\":%d}}",
+                  res.raster, res.kgroup, res.reduce, res.multicast);
+    js += tmp;
+    *out = res;
+    if (report_needed) *report_needed = js.size() + 1;
+    if (report && report_len > 0) {
+        const size_t n = std::min(report_len - 1, js.size());
+        std::memcpy(report, js.data(), n);
+        report[n] = '\0';
+    }
+    return NNJIT_OK;
+}
+
 nnjit_status nnjit_matmul_plan(int64_t M, int64_t N, int64_t K, nnjit_dtype dt, double budget_ms,
                                nnjit_plan* out) {
     nnjit_matmul_desc d{};
@@ -757,7 +883,8 @@ nnjit_status nnjit_matmul_plan_candidate(const nnjit_matmul_desc* d, int32_t ind
     int dev = 0;
     std::vector<nnjit_candidate> space;
     int64_t naive = 0;
-    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive);
+    const nnjit_settings set = current_settings();
+    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive, set);
     if (st != NNJIT_OK) return st;
     if (index < 0 || index >= (int32_t)space.size())
         return fail(NNJIT_ERR_INVALID_ARG, "candidate index out of range");
@@ -769,6 +896,7 @@ nnjit_status nnjit_matmul_plan_candidate(const nnjit_matmul_desc* d, int32_t ind
     pl->chosen_index = index;
     pl->space_size = (int)space.size();
     pl->naive = naive;
+    pl->settings = set;
     st = alloc_plan_buffers(pl.get());
     if (st != NNJIT_OK) { free_plan(pl.release()); return st; }
     *out = pl.release();
@@ -789,11 +917,13 @@ nnjit_status nnjit_matmul_plan_online(const nnjit_matmul_desc* d, nnjit_plan* ou
     int dev = 0;
     std::vector<nnjit_candidate> space;
     int64_t naive = 0;
-    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive);
+    const nnjit_settings set = current_settings();
+    nnjit_status st = plan_common(d, out, &p, &L, &dev, &space, &naive, set);
     if (st != NNJIT_OK) return st;
     std::unique_ptr<nnjit_plan_s> pl(new nnjit_plan_s);
     pl->p = p;
     pl->device = dev;
+    pl->settings = set;
     pl->family = space[0].family;
     pl->cand = space[0];
     pl->chosen_index = 0;
@@ -804,7 +934,7 @@ nnjit_status nnjit_matmul_plan_online(const nnjit_matmul_desc* d, nnjit_plan* ou
     o.active = !p.degenerate();
     o.space = space;
     o.samples.assign(space.size(), {});
-    o.key = (p.flags & NNJIT_PLAN_NO_CACHE) ? std::string() : cache_key(p, dev, L);
+    o.key = (p.flags & NNJIT_PLAN_NO_CACHE) ? std::string() : cache_key(p, dev, L, set);
     // the workspace serves every candidate of the queue
     nnjit_candidate widest = space[0];
     for (const auto& c : space)
@@ -917,13 +1047,14 @@ nnjit_status nnjit_plan_describe(nnjit_plan pl, char* buf, size_t len, size_t* n
                   "\"candidate\":{\"bm\":%d,\"bn\":%d,\"bk\":%d,\"tm\":%d,\"tn\":%d,\"stages\":%d,"
                   "\"split_k\":%d,\"raster\":%d,\"threads\":%d,\"smem_bytes\":%d,\"tmem_cols\":%d,"
                   "\"regs_per_thread\":%d,\"blocks_per_sm\":%d,\"grid\":%d,\"wave_eff_ppm\":%d,"
-                  "\"instance\":%d,\"predicted_cost\":%lld},\"timings_us\":[",
+                  "\"instance\":%d,\"predicted_cost\":%lld},\"settings\":[%d,%d,%d,%d],\"timings_us\":[",
                   (long long)p.M, (long long)p.N, (long long)p.K, (long long)p.batch, p.dtype,
                   p.b_layout, pl->family, pl->chosen_index, pl->space_size, (long long)pl->naive,
                   pl->tune_ms, pl->from_cache ? "true" : "false", pl->timed ? "true" : "false",
                   c.bm, c.bn, c.bk, c.tm, c.tn, c.stages, c.split_k, c.raster, c.threads,
                   c.smem_bytes, c.tmem_cols, c.regs_per_thread, c.blocks_per_sm, c.grid,
-                  c.wave_eff_ppm, c.instance, (long long)c.predicted_cost);
+                  c.wave_eff_ppm, c.instance, (long long)c.predicted_cost, pl->settings.raster,
+                  pl->settings.kgroup, pl->settings.reduce, pl->settings.multicast);
     s += tmp;
     for (size_t i = 0; i < pl->timings.size(); ++i) {
         std::snprintf(tmp, sizeof tmp, "%s[%d,%.4f]", i ? "," : "", pl->timings[i].first,

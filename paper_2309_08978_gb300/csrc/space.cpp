@@ -614,8 +614,76 @@ nnjit_status choose_family(const Problem& p, int* family, std::string* err) {
     return NNJIT_OK;
 }
 
-nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
+nnjit_settings free_settings() {
+    nnjit_settings s;
+    s.raster = s.kgroup = s.reduce = s.multicast = NNJIT_SETTING_FREE;
+    return s;
+}
+
+int setting_of(const nnjit_settings& s, int axis) {
+    switch (axis) {
+        case 0: return s.raster;
+        case 1: return s.kgroup;
+        case 2: return s.reduce;
+        case 3: return s.multicast;
+        default: return NNJIT_SETTING_FREE;
+    }
+}
+
+bool settings_valid(const nnjit_settings& s, std::string* err) {
+    const int lo[kSettingAxes] = {0, 1, 0, 0}, hi[kSettingAxes] = {1, 2, 1, 1};
+    const char* names[kSettingAxes] = {"raster", "kgroup", "reduce", "multicast"};
+    for (int a = 0; a < kSettingAxes; ++a) {
+        const int v = setting_of(s, a);
+        if (v != NNJIT_SETTING_FREE && (v < lo[a] || v > hi[a])) {
+            *err = std::string("setting ") + names[a] + " out of range";
+            return false;
+        }
+    }
+    return true;
+}
+
+int candidate_setting(const Problem& p, const nnjit_candidate& c, int axis) {
+    if (c.family != NNJIT_FAMILY_TC) return -1;
+    switch (axis) {
+        case 0: return c.raster;
+        case 1: return c.bk / (128 / p.elem_bytes());
+        case 2: return c.reduce;
+        case 3: return (c.bm == ModelConstants::kTcBM && c.cluster_m == 2) ? 1 : 0;
+        default: return -1;
+    }
+}
+
+bool setting_twins(const Problem& p, const nnjit_candidate& a, const nnjit_candidate& b, int axis) {
+    if (a.family != NNJIT_FAMILY_TC || b.family != NNJIT_FAMILY_TC) return false;
+    if (a.bm != b.bm || a.bn != b.bn || a.split_k != b.split_k) return false;
+    for (int o = 0; o < kSettingAxes; ++o)
+        if (o != axis && candidate_setting(p, a, o) != candidate_setting(p, b, o)) return false;
+    return candidate_setting(p, a, axis) != candidate_setting(p, b, axis);
+}
+
+void apply_settings(const Problem& p, const nnjit_settings& s, std::vector<nnjit_candidate>* v) {
+    for (int axis = 0; axis < kSettingAxes; ++axis) {
+        const int fixed = setting_of(s, axis);
+        if (fixed == NNJIT_SETTING_FREE) continue;
+        std::vector<nnjit_candidate> kept;
+        for (const auto& c : *v) {
+            bool drop = false;
+            if (c.family == NNJIT_FAMILY_TC && candidate_setting(p, c, axis) != fixed)
+                for (const auto& t : *v)
+                    if (candidate_setting(p, t, axis) == fixed && setting_twins(p, c, t, axis)) {
+                        drop = true;
+                        break;
+                    }
+            if (!drop) kept.push_back(c);
+        }
+        *v = std::move(kept);
+    }
+}
+
+nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim, const nnjit_settings& set,
                          std::vector<nnjit_candidate>* out, int64_t* naive, std::string* err) {
+    if (!settings_valid(set, err)) return NNJIT_ERR_INVALID_ARG;
     if (lim.sm_count <= 0 || lim.smem_per_sm <= 0 || lim.smem_per_block_optin <= 0 ||
         lim.regs_per_sm <= 0 || lim.max_threads_per_sm <= 0 || lim.max_blocks_per_sm <= 0 ||
         lim.tmem_cols_per_sm < 0) {
@@ -648,6 +716,7 @@ nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
         if (a.blocks_per_sm != b.blocks_per_sm) return a.blocks_per_sm > b.blocks_per_sm;
         return a.predicted_cost < b.predicted_cost;
     });
+    apply_settings(p, set, &v);
     *out = std::move(v);
     if (naive) *naive = nv;
     return NNJIT_OK;

@@ -68,8 +68,24 @@ nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string
 // Which family serves the problem (a1 of the hot path), or UNSUPPORTED with `err`.
 nnjit_status choose_family(const Problem& p, int* family, std::string* err);
 
-// Build the ordered lite space.  naive = size before pruning.
-nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim,
+// Fixed settings (nnjit_settings, the primitive vector of Sec. 5.1).  Axis a of a
+// tensor-core candidate: 0 raster, 1 k-blocks per ring slot, 2 split-K reduction,
+// 3 multicast pair; -1 for candidates of other families.
+constexpr int kSettingAxes = 4;
+nnjit_settings free_settings();
+int setting_of(const nnjit_settings& s, int axis);
+bool settings_valid(const nnjit_settings& s, std::string* err);
+int candidate_setting(const Problem& p, const nnjit_candidate& c, int axis);
+// True if a and b are the same candidate but for axis `axis` (every other searched field
+// equal: bm, bn, split_k and the other settings).
+bool setting_twins(const Problem& p, const nnjit_candidate& a, const nnjit_candidate& b, int axis);
+// Drop, axis by axis in order, every candidate whose value differs from a fixed one while
+// its twin with the fixed value is in the space.  Order is preserved.
+void apply_settings(const Problem& p, const nnjit_settings& s, std::vector<nnjit_candidate>* v);
+
+// Build the ordered lite space, then apply the fixed settings.  naive = size before
+// pruning.
+nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim, const nnjit_settings& set,
                          std::vector<nnjit_candidate>* out, int64_t* naive, std::string* err);
 
 // Precompiled-instance index helpers (kept in one place so the registry and the space
@@ -83,7 +99,7 @@ int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if non
 // TMA-fed GEMV (B as [N][K]): rows per stage 8/16/32, M <= maxm (1 or 8).
 constexpr int kGemvTmaFirstInstance = 8;
 int gemv_tma_instance(int rows, int maxm);                     // 8..13, -1 if none
-// TMA-fed GEMV over 4-bit weights (NNJIT_W4_BF16): rows per stage 8/16/32, maxm 1 or 8.
+// TMA-fed GEMV over 4-bit weights (NNJIT_W4_BF16): rows per stage 16/32.
 constexpr int kGemvW4FirstInstance = 14;
 int gemv_w4_instance(int rows);                                // 14..15, -1 if none
 

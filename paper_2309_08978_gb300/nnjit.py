@@ -71,6 +71,14 @@ class nnjit_candidate(ctypes.Structure):
                         ("cluster_m", ctypes.c_int32)]
 
 
+NNJIT_SETTING_FREE = -1
+SETTING_AXES = ("raster", "kgroup", "reduce", "multicast")
+
+
+class nnjit_settings(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in SETTING_AXES]
+
+
 def struct_to_dict(s) -> dict:
     return {name: getattr(s, name) for name, _ in s._fields_}
 
@@ -123,6 +131,10 @@ def load_library(path: str = LIB_PATH):
             "nnjit_cache_save": [ctypes.c_char_p],
             "nnjit_cache_load": [ctypes.c_char_p, P(i32)],
             "nnjit_w4_layout": [i64, i64, i64, P(i64), P(i64)],
+            "nnjit_settings_set": [P(nnjit_settings)],
+            "nnjit_settings_get": [P(nnjit_settings)],
+            "nnjit_settings_study": [P(nnjit_matmul_desc), i32, P(nnjit_settings), ctypes.c_char_p,
+                                     ctypes.c_size_t, P(ctypes.c_size_t)],
         }
         for name, args in sigs.items():
             f = getattr(lib, name)
@@ -361,3 +373,38 @@ def nnjit_cache_load(path: str) -> int:
     n = ctypes.c_int32(0)
     _check(load_library().nnjit_cache_load(os.fsencode(path), ctypes.byref(n)), "nnjit_cache_load")
     return n.value
+
+
+def nnjit_settings_set(settings: dict | None):
+    """Fix settings process-wide ({axis: value}; missing axes stay searched); None clears."""
+    lib = load_library()
+    if settings is None:
+        _check(lib.nnjit_settings_set(None), "nnjit_settings_set")
+        return
+    unknown = set(settings) - set(SETTING_AXES)
+    if unknown:
+        raise ValueError(f"unknown settings {sorted(unknown)}")
+    s = nnjit_settings(*[int(settings.get(a, NNJIT_SETTING_FREE)) for a in SETTING_AXES])
+    _check(lib.nnjit_settings_set(ctypes.byref(s)), "nnjit_settings_set")
+
+
+def nnjit_settings_get() -> dict:
+    s = nnjit_settings()
+    _check(load_library().nnjit_settings_get(ctypes.byref(s)), "nnjit_settings_get")
+    return struct_to_dict(s)
+
+
+def nnjit_settings_study(descs) -> tuple[dict, dict]:
+    """Run the one-variable-at-a-time settings study over `descs`; returns (settings it
+    recommends, the JSON report as a dict).  Nothing is applied."""
+    lib = load_library()
+    arr = (nnjit_matmul_desc * len(descs))(*descs)
+    out = nnjit_settings()
+    need = ctypes.c_size_t(0)
+    size = 4096 + 4096 * len(descs)      # the report takes well under 1 KB per product
+    buf = ctypes.create_string_buffer(size)
+    _check(lib.nnjit_settings_study(arr, len(descs), ctypes.byref(out), buf, size, ctypes.byref(need)),
+           "nnjit_settings_study")
+    if need.value > size:
+        raise RuntimeError(f"settings report truncated ({need.value} > {size} bytes)")
+    return struct_to_dict(out), json.loads(buf.value.decode())

@@ -117,3 +117,21 @@ def test_w4_layout_matches_the_documented_blob(lib):
         with pytest.raises(nj.NnjitError) as ei:
             nj.nnjit_w4_layout(*bad)
         assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
+
+
+def test_settings_roundtrip_and_validation(lib):
+    """nnjit_settings_set/get: values round-trip, out-of-range values are refused without
+    changing the current settings, NULL clears (host only)."""
+    import paper_2309_08978_gb300 as nj
+    assert nj.nnjit_settings_get() == {"raster": -1, "kgroup": -1, "reduce": -1, "multicast": -1}
+    try:
+        nj.nnjit_settings_set({"raster": 1, "multicast": 0})
+        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": -1, "multicast": 0}
+        for bad in ({"kgroup": 0}, {"kgroup": 3}, {"raster": 2}, {"reduce": -2}, {"multicast": 5}):
+            with pytest.raises(nj.NnjitError) as ei:
+                nj.nnjit_settings_set(bad)
+            assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
+        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": -1, "multicast": 0}
+    finally:
+        nj.nnjit_settings_set(None)
+    assert nj.nnjit_settings_get()["raster"] == -1

@@ -165,3 +165,47 @@ def test_online_plan_serves_exact_results_while_it_tunes():
         i2 = p2.describe()
         assert i2["from_cache"] is True and i2["chosen_index"] == prog["current_index"]
     nj.nnjit_cache_clear()
+
+
+def test_settings_study_and_fixed_settings():
+    """The one-variable-at-a-time study (Sec. 5.1) times each product's full space, and
+    each setting's verdict is consistent with the times it reports; the settings it
+    recommends shrink the spaces (never to zero), are part of the plan-cache key and
+    the plan description, and a plan from the shrunk space stays exact."""
+    descs = [nj.make_desc(512, 2304, 768, "tf32", "NK", has_bias=True),
+             nj.make_desc(1024, 1024, 1024, "bf16", "NK")]
+    rec, report = nj.nnjit_settings_study(descs)
+    assert set(rec) == set(nj.SETTING_AXES)
+    assert len(report["products"]) == 2
+    lim = nj.nnjit_device_limits_query(0)
+    for prod, d in zip(report["products"], descs):
+        cands, _ = nj.nnjit_space_enumerate(d, lim)
+        assert prod["space_size"] == len(cands)
+        for axis, ev in prod["settings"].items():
+            assert ev["value"] == prod["best"][axis]
+            if ev["verdict"] == "decisive":
+                assert ev["twin_us"] > 1.02 * prod["best_us"]
+                assert rec[axis] in (-1, ev["value"])
+            elif ev["verdict"] == "tie":
+                assert ev["twin_us"] <= 1.02 * prod["best_us"]
+    for axis, v in rec.items():
+        votes = {p["settings"][axis]["value"] for p in report["products"]
+                 if p["settings"][axis]["verdict"] == "decisive"}
+        assert (v == -1) == (len(votes) != 1) and (v == -1 or votes == {v})
+    # apply a fixed setting set (the recommended one, or a hand-picked one when the study
+    # found nothing decisive) and check the shrunk space and a plan from it
+    fixed = {a: v for a, v in rec.items() if v != -1} or {"raster": 0, "kgroup": 2}
+    full = [len(nj.nnjit_space_enumerate(d, lim)[0]) for d in descs]
+    nj.nnjit_settings_set(fixed)
+    try:
+        shrunk = [len(nj.nnjit_space_enumerate(d, lim)[0]) for d in descs]
+        assert all(1 <= s <= f for s, f in zip(shrunk, full))
+        shape = Shape("t", 512, 2304, 768, 1, "NK", True)
+        A, B, bias = make_operands(shape, 31, "tf32", ints=True)
+        with nj.nnjit_matmul_plan_ex(descs[0], 200.0) as plan:
+            info = plan.describe()
+            assert info["settings"] == [fixed.get(a, -1) for a in nj.SETTING_AXES]
+            C = run_plan(plan, A, B, bias, 512, 2304)
+        compare(C, A, B, bias, "NK", "tf32", exact=True)
+    finally:
+        nj.nnjit_settings_set(None)

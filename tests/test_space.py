@@ -133,3 +133,80 @@ def test_space_invariants_on_gb300():
             assert c["instance"] >= 0
         keys = [tuple(c[k] for k in osp.CANDIDATE_FIELDS) for c in cands]
         assert len(set(keys)) == len(keys)
+
+
+SETTINGS_CASES = [
+    {"raster": 0}, {"raster": 1}, {"kgroup": 2}, {"kgroup": 1, "reduce": 1},
+    {"reduce": 0, "multicast": 1}, {"multicast": 0, "raster": 1},
+    {"raster": 0, "kgroup": 2, "reduce": 1, "multicast": 1},
+]
+
+
+@pytest.mark.parametrize("settings", SETTINGS_CASES, ids=lambda s: ",".join(f"{k}={v}" for k, v in s.items()))
+def test_library_space_with_fixed_settings_equals_oracle(settings):
+    """Sec. 5.1's fixed settings prune the same candidates in both implementations."""
+    import paper_2309_08978_gb300 as nj
+    from paper_2309_08978_gb300.build_lib import build
+    build()
+    L = _limits(GB300)
+    nj.nnjit_settings_set(settings)
+    try:
+        checked = 0
+        for prob in _problems():
+            desc = nj.make_desc(prob["M"], prob["N"], prob["K"], prob["dtype"], prob["b_layout"],
+                                batch=prob.get("batch", 1), has_bias=prob.get("has_bias", 0),
+                                lda=prob.get("lda", 0), ldb=prob.get("ldb", 0), ldc=prob.get("ldc", 0),
+                                stride_c=prob.get("stride_c", 0))
+            try:
+                want, _ = osp.build_space(osp.resolve(**prob), GB300, settings)
+            except osp.SpaceError:
+                continue
+            got, _ = nj.nnjit_space_enumerate(desc, L)
+            assert [{k: g[k] for k in osp.CANDIDATE_FIELDS} for g in got] == want, (prob, settings)
+            checked += 1
+        assert checked >= 30
+    finally:
+        nj.nnjit_settings_set(None)
+
+
+def test_fixed_settings_prune_only_where_a_twin_exists():
+    """A fixed setting keeps the space non-empty and ordered (a subsequence of the free
+    space), removes every candidate with the other value whose twin is present, and
+    keeps the only legal choice (kgroup = 2 keeps the 256-wide tiles, which exist only
+    with one k-block per slot)."""
+    seen_bn256 = False
+    for prob in _problems():
+        try:
+            p = osp.resolve(**prob)
+            free, _ = osp.build_space(p, GB300)
+        except osp.SpaceError:
+            continue
+        for settings in SETTINGS_CASES:
+            fixed, _ = osp.build_space(p, GB300, settings)
+            assert fixed, (prob, settings)
+            it = iter(free)
+            assert all(any(c == f for f in it) for c in fixed)          # ordered subsequence
+            for axis, v in settings.items():
+                for c in fixed:
+                    w = osp.setting_value(p, c, axis)
+                    if w is not None and w != v:
+                        assert not any(osp.setting_value(p, t, axis) == v and osp._twins(p, c, t, axis)
+                                       for t in fixed), (prob, settings, c)
+            if settings.get("kgroup") == 2:
+                wide = [c for c in free if c["family"] == osp.FAMILY_TC and c["bn"] == 256]
+                seen_bn256 |= bool(wide)
+                assert all(c in fixed for c in wide if settings.keys() == {"kgroup"})
+    assert seen_bn256
+
+
+def test_setting_values_of_candidates():
+    """The setting accessors read what the candidates encode: bk = 2 k-blocks of 128 bytes
+    for kgroup 2 (64 bf16 elements per k-block), multicast only for 128-row pairs."""
+    p = osp.resolve(M=4096, N=4096, K=4096, dtype=osp.BF16, b_layout=osp.B_NK)
+    cands, _ = osp.build_space(p, GB300)
+    kg = {osp.setting_value(p, c, "kgroup") for c in cands}
+    assert kg == {1, 2}
+    assert all(c["bk"] == 64 * osp.setting_value(p, c, "kgroup") for c in cands)
+    pairs = [c for c in cands if c["cluster_m"] == 2]
+    assert {osp.setting_value(p, c, "multicast") for c in pairs} == {0, 1}   # CTA pairs and multicast pairs
+    assert all(osp.setting_value(p, c, "multicast") == (c["bm"] == 128) for c in pairs)
