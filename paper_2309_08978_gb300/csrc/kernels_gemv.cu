@@ -260,21 +260,50 @@ const GemvKernel kGemvKernels[8] = {
 std::mutex g_gemv_mu;
 int g_gemv_smem[8] = {0};
 
+// Fixed-order sum of the split-K partials (s = 0, 1, ... per element; + bias, activation)
+// into C.  With vec4, four consecutive columns per thread in 16-byte accesses (N, ldc and
+// stride_c multiples of 4; C, bias and the workspace 16-byte aligned).
 __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, long long batch_mn,
                                      int M, int N, long long ldc, long long stride_c,
-                                     const float* __restrict__ bias, int act, float* __restrict__ C) {
+                                     const float* __restrict__ bias, int act, int vec4, float* __restrict__ C) {
     ptx::griddep_wait();
     if (threadIdx.x == 0) ptx::griddep_launch_dependents();
+    const long long step = (long long)gridDim.x * blockDim.x;
+    if (vec4) {
+        const int n4 = N >> 2;
+        const long long total = batch_mn >> 2;
+        for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < total; i += step) {
+            const long long row = i / n4;  // batch item * M + m
+            const int c = (int)(i - row * n4) << 2;
+            const long long e = row * N + c;
+            float4 v = *reinterpret_cast<const float4*>(ws + e);
+            for (int s = 1; s < split; ++s) {
+                const float4 w = *reinterpret_cast<const float4*>(ws + (long long)s * batch_mn + e);
+                v.x += w.x; v.y += w.y; v.z += w.z; v.w += w.w;
+            }
+            if (bias) {
+                const float4 b4 = *reinterpret_cast<const float4*>(bias + c);
+                v.x += b4.x; v.y += b4.y; v.z += b4.z; v.w += b4.w;
+            }
+            if (act != NNJIT_EPI_NONE) {
+                v.x = apply_act(v.x, act); v.y = apply_act(v.y, act);
+                v.z = apply_act(v.z, act); v.w = apply_act(v.w, act);
+            }
+            const long long b = row / M;
+            const int m = (int)(row - b * M);
+            *reinterpret_cast<float4*>(C + b * stride_c + (long long)m * ldc + c) = v;
+        }
+        return;
+    }
     const long long mn = (long long)M * N;
-    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < batch_mn;
-         i += (long long)gridDim.x * blockDim.x) {
+    for (long long i = blockIdx.x * (long long)blockDim.x + threadIdx.x; i < batch_mn; i += step) {
         float v = ws[i];
         for (int s = 1; s < split; ++s) v += ws[(long long)s * batch_mn + i];
         const long long b = i / mn;
         const long long r = i % mn;
         const int m = (int)(r / N), n = (int)(r % N);
         if (bias) v += bias[n];
-        C[b * stride_c + (long long)m * ldc + n] = apply_act(v, act);
+        C[b * stride_c + (long long)m * ldc + n] = act != NNJIT_EPI_NONE ? apply_act(v, act) : v;
     }
 }
 
@@ -376,8 +405,11 @@ cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, c
                                  float* C, cudaStream_t s) {
     const long long n = p.batch * p.M * p.N;
     if (n == 0) return cudaSuccess;
-    return launch_pdl(splitk_reduce_kernel, dim3(grid_for(n, 256)), dim3(256), 0, s, ws, split, n,
-                      (int)p.M, (int)p.N, p.ldc, p.stride_c, bias, p.epilogue, C);
+    auto a16 = [](const void* q) { return (reinterpret_cast<uintptr_t>(q) & 15) == 0; };
+    const int vec4 = (p.N % 4 == 0 && p.ldc % 4 == 0 && p.stride_c % 4 == 0 && a16(C) && a16(ws) &&
+                      (!bias || a16(bias))) ? 1 : 0;
+    return launch_pdl(splitk_reduce_kernel, dim3(grid_for(vec4 ? n / 4 : n, 256)), dim3(256), 0, s, ws, split,
+                      n, (int)p.M, (int)p.N, p.ldc, p.stride_c, bias, p.epilogue, vec4, C);
 }
 
 cudaError_t launch_fill_bias(const Problem& p, const float* bias, float* C, cudaStream_t s) {

@@ -295,7 +295,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
                 }
-                apply_act32(v, p.act);
                 if (p.tma_store) {
                     uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
                     if (lane == 0) ptx::bulk_wait_read<1>();
@@ -304,6 +303,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                     for (int j = 0; j < 8; ++j)
                         *reinterpret_cast<float4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
                             make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                    if (p.act != NNJIT_EPI_NONE) act_row128(buf + lane * 128, p.act);
                     ptx::fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
@@ -322,6 +322,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                         for (int j = 0; j < 32; ++j)
                             if (col0 + j < p.N) dst[j] = v[j];
                     }
+                    if (p.act != NNJIT_EPI_NONE) act_written(dst, min(32, p.N - col0), p.act);
                 }
             };
             auto bias_of = [&](int c) {
