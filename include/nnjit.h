@@ -89,12 +89,17 @@ typedef enum {
  * Elementwise activation applied to every output after the bias, inside the kernel that
  * writes C (the epilogue fusion of a Linear with its activation; in split-K plans the
  * reduction applies it once the slices are summed):  C = act(A * Bt + bias).
+ * Or-ed with NNJIT_EPI_RESIDUAL, the kernel that writes C also adds the value C held
+ * before the call (a residual connection; C must then be initialised by the caller):
+ *   C = act(A * Bt + bias) + C.
+ * Partial sums of split-K plans go to the plan's workspace; C is read and written once.
  */
 typedef enum {
     NNJIT_EPI_NONE = 0,
     NNJIT_EPI_RELU = 1,  /* max(x, 0) */
     NNJIT_EPI_GELU = 2,  /* x * Phi(x) = 0.5 x (1 + erf(x / sqrt(2)))  (exact, erf form) */
-    NNJIT_EPI_SILU = 3   /* x * sigmoid(x) = x / (1 + exp(-x)) */
+    NNJIT_EPI_SILU = 3,  /* x * sigmoid(x) = x / (1 + exp(-x)) */
+    NNJIT_EPI_RESIDUAL = 0x10
 } nnjit_epilogue;
 
 /* Kernel families of the lite space. */

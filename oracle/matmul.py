@@ -91,12 +91,14 @@ def to_f64(x: np.ndarray) -> np.ndarray:
 
 
 def matmul(A: np.ndarray, B: np.ndarray, bias: np.ndarray | None = None,
-           b_layout: int = B_KN, nthreads: int = 0, act: str = "none"):
+           b_layout: int = B_KN, nthreads: int = 0, act: str = "none", residual=None):
     """Reference product.
 
     A: [M,K] or [batch,M,K]; B: [K,N] / [N,K] (KN / NK), optionally with a leading batch
     dimension.  uint16 arrays are bf16 bit patterns.  bias: [N] or None.  act: an
     activation of oracle.epilogue applied in FP64 after the bias (the fused epilogue).
+    residual: None, or the prior content of C (shape of the result), added after the
+    activation (the residual epilogue: C = act(A.Bt + bias) + C).
     Returns (C64, C32): float64 and float32 arrays of shape [M,N] or [batch,M,N].
     """
     A64, B64 = to_f64(A), to_f64(B)
@@ -138,6 +140,11 @@ def matmul(A: np.ndarray, B: np.ndarray, bias: np.ndarray | None = None,
     if act != "none":
         from .epilogue import apply
         C = apply(C, act)
+    if residual is not None:
+        R = np.asarray(residual, dtype=np.float64)
+        if R.shape != C.shape:
+            raise ValueError(f"residual shape {R.shape} != result shape {C.shape}")
+        C = C + R
     return C, C.astype(np.float32)
 
 

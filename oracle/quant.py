@@ -35,6 +35,7 @@ def dequant(blob: np.ndarray, N: int, K: int, ldb: int = 0) -> np.ndarray:
 
 
 def matmul(x_bits: np.ndarray, blob: np.ndarray, N: int, K: int, ldb: int = 0, bias=None,
-           act: str = "none", nthreads: int = 0):
-    """(C64, C32) of x (bf16 bit patterns [M][K]) times the dequantised W^T (+ bias, act)."""
-    return _matmul(x_bits, dequant(blob, N, K, ldb), bias, B_NK, nthreads, act)
+           act: str = "none", nthreads: int = 0, residual=None):
+    """(C64, C32) of x (bf16 bit patterns [M][K]) times the dequantised W^T (+ bias, act,
+    + residual)."""
+    return _matmul(x_bits, dequant(blob, N, K, ldb), bias, B_NK, nthreads, act, residual)

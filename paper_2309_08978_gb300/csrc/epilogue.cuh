@@ -1,6 +1,7 @@
 // The elementwise activation a kernel applies to each output after the bias
-// (nnjit_epilogue).  `act` is uniform across a launch, so the switch costs one predictable
-// branch per element.
+// (nnjit_epilogue).  Kernels receive the epilogue code: the activation in bits 0-3 and
+// NNJIT_EPI_RESIDUAL (add the output's prior value after the activation).  The code is
+// uniform across a launch, so each switch costs one predictable branch.
 //
 // The epilogue runs on the 4 warps that drain TMEM, so a long per-element computation is
 // on the critical path of every tile; both transcendental activations therefore use a
@@ -38,7 +39,7 @@ __device__ __forceinline__ float silu_fast(float x) {
 // A chunk of 32 outputs of one thread: one switch per chunk, then 32 independent
 // evaluations the compiler can interleave (a switch per element serialises them).
 __device__ __forceinline__ void apply_act32(float (&v)[32], int act) {
-    switch (act) {
+    switch (act & 15) {
         case NNJIT_EPI_RELU:
 #pragma unroll
             for (int j = 0; j < 32; ++j) v[j] = fmaxf(v[j], 0.0f);
@@ -64,7 +65,7 @@ __device__ __forceinline__ void apply_act32(float (&v)[32], int act) {
 // that slowed plans without an activation by 0.2-0.7 us per product.
 __device__ __forceinline__ void act_row128(void* row128, int act) {
     float4* r = static_cast<float4*>(row128);
-    switch (act) {
+    switch (act & 15) {
         case NNJIT_EPI_RELU:
 #pragma unroll 1
             for (int u = 0; u < 8; ++u) {
@@ -91,21 +92,53 @@ __device__ __forceinline__ void act_row128(void* row128, int act) {
     }
 }
 
-__device__ __forceinline__ void act_written(float* dst, int n, int act) {
+// The epilogue of a staged row (plain order, n <= 32 values) written element by element to
+// dst: activation, then with NNJIT_EPI_RESIDUAL the value dst held before.
+__device__ __forceinline__ void epi_store_row(const float* row, int code, float* dst, int n) {
+    const int act = code & 15;
+    const bool res = (code & NNJIT_EPI_RESIDUAL) != 0;
 #pragma unroll 1
     for (int j = 0; j < n; ++j) {
-        const float x = dst[j];
-        dst[j] = act == NNJIT_EPI_RELU ? fmaxf(x, 0.0f) : act == NNJIT_EPI_GELU ? gelu_as7126(x) : silu_fast(x);
+        const float x = row[j];
+        float y = act == NNJIT_EPI_RELU ? fmaxf(x, 0.0f)
+                  : act == NNJIT_EPI_GELU ? gelu_as7126(x)
+                  : act == NNJIT_EPI_SILU ? silu_fast(x) : x;
+        if (res) y += dst[j];
+        dst[j] = y;
+    }
+}
+
+// With NNJIT_EPI_RESIDUAL: add the prior content of a thread's output segment (n <= 32
+// columns at dst, 16-byte aligned) to its staged 128-byte row, whose logical 16-byte unit j
+// sits at unit j ^ swz (the 128-byte swizzle of the TMA-store staging).
+__device__ __forceinline__ void residual_row128(void* row128, int swz, const float* dst, int n) {
+    float4* r = static_cast<float4*>(row128);
+    if (n >= 32) {
+#pragma unroll 1
+        for (int j = 0; j < 8; ++j) {
+            const float4 o = *reinterpret_cast<const float4*>(dst + 4 * j);
+            float4& s = r[j ^ swz];
+            s.x += o.x; s.y += o.y; s.z += o.z; s.w += o.w;
+        }
+    } else {
+#pragma unroll 1
+        for (int j = 0; j < n; ++j) reinterpret_cast<float*>(&r[(j >> 2) ^ swz])[j & 3] += dst[j];
     }
 }
 
 __device__ __forceinline__ float apply_act(float v, int act) {
-    switch (act) {
+    switch (act & 15) {
         case NNJIT_EPI_RELU: return fmaxf(v, 0.0f);
         case NNJIT_EPI_GELU: return gelu_as7126(v);
         case NNJIT_EPI_SILU: return silu_fast(v);
         default: return v;
     }
+}
+
+// One output element: act(v), plus the element's prior value *c with NNJIT_EPI_RESIDUAL.
+__device__ __forceinline__ float epi_out(float v, int code, const float* c) {
+    const float y = apply_act(v, code);
+    return (code & NNJIT_EPI_RESIDUAL) ? y + *c : y;
 }
 
 }  // namespace nnjit

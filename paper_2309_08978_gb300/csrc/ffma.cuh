@@ -140,7 +140,7 @@ __global__ void __launch_bounds__((BM / TM) * (BN / TN))
             const int gn = n0 + tx * TN + j;
             if (gn < p.N) {
                 const float v = bias ? acc[i][j] + __ldg(bias + gn) : acc[i][j];
-                dst[gn] = p.split == 1 ? apply_act(v, p.act) : v;
+                dst[gn] = p.split == 1 ? epi_out(v, p.act, dst + gn) : v;
             }
         }
     }

@@ -169,7 +169,8 @@ __global__ void __launch_bounds__(256) gemv_nk_kernel(const GemvParams p) {
                 for (int m = 0; m < kMaxM; ++m) {
                     if (m >= M) continue;
                     if (p.split == 1)
-                        p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act);
+                        p.C[(long long)m * p.ldc + n] = epi_out(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act,
+                                                                p.C + (long long)m * p.ldc + n);
                     else
                         p.ws[((long long)s * M + m) * p.N + n] = acc[r][m];
                 }
@@ -244,7 +245,7 @@ __global__ void __launch_bounds__(256) gemv_kn_kernel(const GemvParams p) {
         float v = 0.0f;
         for (int w = 0; w < warps; ++w) v += red[((long long)w * M + m) * 256 + col];
         if (p.split == 1)
-            p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? v + p.bias[n] : v, p.act);
+            p.C[(long long)m * p.ldc + n] = epi_out(p.bias ? v + p.bias[n] : v, p.act, p.C + (long long)m * p.ldc + n);
         else
             p.ws[((long long)s * M + m) * p.N + n] = v;
     }
@@ -285,13 +286,18 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, lo
                 const float4 b4 = *reinterpret_cast<const float4*>(bias + c);
                 v.x += b4.x; v.y += b4.y; v.z += b4.z; v.w += b4.w;
             }
-            if (act != NNJIT_EPI_NONE) {
+            if ((act & 15) != NNJIT_EPI_NONE) {
                 v.x = apply_act(v.x, act); v.y = apply_act(v.y, act);
                 v.z = apply_act(v.z, act); v.w = apply_act(v.w, act);
             }
             const long long b = row / M;
             const int m = (int)(row - b * M);
-            *reinterpret_cast<float4*>(C + b * stride_c + (long long)m * ldc + c) = v;
+            float4* out = reinterpret_cast<float4*>(C + b * stride_c + (long long)m * ldc + c);
+            if (act & NNJIT_EPI_RESIDUAL) {
+                const float4 o = *out;
+                v.x += o.x; v.y += o.y; v.z += o.z; v.w += o.w;
+            }
+            *out = v;
         }
         return;
     }
@@ -303,7 +309,8 @@ __global__ void splitk_reduce_kernel(const float* __restrict__ ws, int split, lo
         const long long r = i % mn;
         const int m = (int)(r / N), n = (int)(r % N);
         if (bias) v += bias[n];
-        C[b * stride_c + (long long)m * ldc + n] = act != NNJIT_EPI_NONE ? apply_act(v, act) : v;
+        float* out = C + b * stride_c + (long long)m * ldc + n;
+        *out = act != NNJIT_EPI_NONE ? epi_out(v, act, out) : v;
     }
 }
 
@@ -316,7 +323,8 @@ __global__ void fill_bias_kernel(long long total, int M, int N, long long ldc, l
          i += (long long)gridDim.x * blockDim.x) {
         const long long b = i / mn, r = i % mn;
         const int m = (int)(r / N), n = (int)(r % N);
-        C[b * stride_c + (long long)m * ldc + n] = apply_act(bias ? bias[n] : 0.0f, act);
+        float* out = C + b * stride_c + (long long)m * ldc + n;
+        *out = epi_out(bias ? bias[n] : 0.0f, act, out);
     }
 }
 

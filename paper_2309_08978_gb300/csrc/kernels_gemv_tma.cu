@@ -252,7 +252,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
                 for (int m = 0; m < MAXM; ++m) {
                     if (m >= M) continue;
                     if (p.split == 1)
-                        p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act);
+                        p.C[(long long)m * p.ldc + n] = epi_out(p.bias ? acc[r][m] + p.bias[n] : acc[r][m], p.act,
+                                                                p.C + (long long)m * p.ldc + n);
                     else
                         p.ws[((long long)w.s * M + m) * p.N + n] = acc[r][m];
                 }

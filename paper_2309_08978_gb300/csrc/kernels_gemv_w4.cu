@@ -345,7 +345,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
                 if (n >= p.N) continue;
                 const float v = ((red[0][row][m] + red[1][row][m]) + red[2][row][m]) + red[3][row][m];
                 if (p.split == 1)
-                    p.C[(long long)m * p.ldc + n] = apply_act(p.bias ? v + p.bias[n] : v, p.act);
+                    p.C[(long long)m * p.ldc + n] = epi_out(p.bias ? v + p.bias[n] : v, p.act, p.C + (long long)m * p.ldc + n);
                 else
                     p.ws[((long long)w.s * M + m) * p.N + n] = v;
             }

@@ -303,7 +303,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                     for (int j = 0; j < 8; ++j)
                         *reinterpret_cast<float4*>(buf + lane * 128 + ((j ^ (lane & 7)) << 4)) =
                             make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
-                    if (p.act != NNJIT_EPI_NONE) act_row128(buf + lane * 128, p.act);
+                    if ((p.act & 15) != NNJIT_EPI_NONE) act_row128(buf + lane * 128, p.act);
+                    if ((p.act & NNJIT_EPI_RESIDUAL) && row < p.M && col0 < p.N)
+                        residual_row128(buf + lane * 128, lane & 7, dst_row + col0, p.N - col0);
                     ptx::fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
@@ -313,7 +315,17 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                     ++chunk_ctr;
                 } else if (row < p.M) {
                     float* dst = dst_row + col0;
-                    if (col0 + 32 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
+                    if (p.act != NNJIT_EPI_NONE) {
+                        // stage the row (this thread's own 128 bytes of the idle staging
+                        // buffer), then activation and residual element by element
+                        if (col0 < p.N) {
+                            float* srow = reinterpret_cast<float*>(stage_buf + lane * 128);
+#pragma unroll
+                            for (int j = 0; j < 32; j += 4)
+                                *reinterpret_cast<float4*>(srow + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
+                            epi_store_row(srow, p.act, dst, min(32, p.N - col0));
+                        }
+                    } else if (col0 + 32 <= p.N && (reinterpret_cast<uintptr_t>(dst) & 15) == 0) {
 #pragma unroll
                         for (int j = 0; j < 32; j += 4)
                             *reinterpret_cast<float4*>(dst + j) = make_float4(v[j], v[j + 1], v[j + 2], v[j + 3]);
@@ -322,7 +334,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                         for (int j = 0; j < 32; ++j)
                             if (col0 + j < p.N) dst[j] = v[j];
                     }
-                    if (p.act != NNJIT_EPI_NONE) act_written(dst, min(32, p.N - col0), p.act);
                 }
             };
             auto bias_of = [&](int c) {

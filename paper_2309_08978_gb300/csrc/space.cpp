@@ -534,7 +534,9 @@ nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string
     if (d->dtype < NNJIT_F32_FFMA || d->dtype > NNJIT_W4_BF16) { *err = "unknown dtype"; return NNJIT_ERR_INVALID_ARG; }
     if (d->b_layout != NNJIT_B_KN && d->b_layout != NNJIT_B_NK) { *err = "unknown b_layout"; return NNJIT_ERR_INVALID_ARG; }
     if (d->has_bias != 0 && d->has_bias != 1) { *err = "has_bias must be 0 or 1"; return NNJIT_ERR_INVALID_ARG; }
-    if (d->epilogue < NNJIT_EPI_NONE || d->epilogue > NNJIT_EPI_SILU) { *err = "unknown epilogue"; return NNJIT_ERR_INVALID_ARG; }
+    if ((d->epilogue & ~(NNJIT_EPI_RESIDUAL | 15)) != 0 || (d->epilogue & 15) > NNJIT_EPI_SILU) {
+        *err = "unknown epilogue"; return NNJIT_ERR_INVALID_ARG;
+    }
     const int64_t lim = (int64_t)1 << 31;
     if (d->M >= lim || d->N >= lim || d->K >= lim || d->batch >= lim) {
         *err = "dimensions must be < 2^31"; return NNJIT_ERR_INVALID_ARG;

@@ -31,6 +31,7 @@ NNJIT_EPI_NONE = 0
 NNJIT_EPI_RELU = 1
 NNJIT_EPI_GELU = 2
 NNJIT_EPI_SILU = 3
+NNJIT_EPI_RESIDUAL = 0x10
 
 NNJIT_B_KN = 0
 NNJIT_B_NK = 1
@@ -202,7 +203,9 @@ EPILOGUES = {"none": 0, "relu": 1, "gelu": 2, "silu": 3}
 
 
 def make_desc(M, N, K, dtype, b_layout="KN", batch=1, has_bias=False, flags=0, lda=0, ldb=0,
-              ldc=0, stride_a=0, stride_b=0, stride_c=0, epilogue="none") -> nnjit_matmul_desc:
+              ldc=0, stride_a=0, stride_b=0, stride_c=0, epilogue="none",
+              residual=False) -> nnjit_matmul_desc:
+    """`epilogue`: an activation name or code; `residual`: C = act(A.Bt + bias) + C."""
     d = nnjit_matmul_desc()
     d.M, d.N, d.K, d.batch = M, N, K, batch
     d.dtype = DTYPES[dtype] if isinstance(dtype, str) else dtype
@@ -211,7 +214,8 @@ def make_desc(M, N, K, dtype, b_layout="KN", batch=1, has_bias=False, flags=0, l
     d.stride_a, d.stride_b, d.stride_c = stride_a, stride_b, stride_c
     d.has_bias = 1 if has_bias else 0
     d.flags = flags
-    d.epilogue = EPILOGUES[epilogue] if isinstance(epilogue, str) else epilogue
+    d.epilogue = (EPILOGUES[epilogue] if isinstance(epilogue, str) else epilogue) | \
+        (NNJIT_EPI_RESIDUAL if residual else 0)
     return d
 
 

@@ -49,8 +49,8 @@ def plan_run_batched(plan, dA, dB, C):
     nj.nnjit_matmul_run_batched(plan, dA, dB, C)
 
 
-def compare(C_gpu, A, B, bias, b_layout, dtype, exact=False, act="none"):
-    ref64, ref32 = oracle.matmul(A, B, bias, layout_code(b_layout), act=act)
+def compare(C_gpu, A, B, bias, b_layout, dtype, exact=False, act="none", residual=None):
+    ref64, ref32 = oracle.matmul(A, B, bias, layout_code(b_layout), act=act, residual=residual)
     assert C_gpu.shape == ref64.shape
     assert np.all(np.isfinite(C_gpu)), "non-finite output (unwritten element?)"
     if exact:

@@ -57,7 +57,8 @@ def test_invalid_descriptors(lib):
            nj.make_desc(4, 4, 4, 7), nj.make_desc(4, 4, 4, "bf16", b_layout=5),
            nj.make_desc(4, 4, 8, "bf16", lda=4), nj.make_desc(4, 8, 4, "bf16", "KN", ldb=4),
            nj.make_desc(4, 8, 4, "bf16", ldc=7), nj.make_desc(4, 4, 4, "bf16", epilogue=9),
-           nj.make_desc(4, 4, 4, "bf16", epilogue=-1)]
+           nj.make_desc(4, 4, 4, "bf16", epilogue=-1), nj.make_desc(4, 4, 4, "bf16", epilogue=0x14),
+           nj.make_desc(4, 4, 4, "bf16", epilogue=0x30)]
     for d in bad:
         with pytest.raises(nj.NnjitError) as ei:
             nj.nnjit_space_enumerate(d, L)

@@ -425,3 +425,95 @@ def test_w4_refusals():
         with pytest.raises(nj.NnjitError) as ei:
             nj.nnjit_space_enumerate(d, L)
         assert ei.value.status == nj.NNJIT_ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("case", EPI_CASES, ids=_ids)
+def test_residual_epilogue_every_candidate(case):
+    """C = act(A.B + bias) + C: the kernel that writes C adds the value C held before (split-K
+    plans: the reduction, once).  Every candidate, ReLU + an integer residual on integer
+    inputs (exact); the top-ranked plan with GELU + a random residual (tolerance)."""
+    torch = pytest.importorskip("torch")
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    Ai, Bi, biasi = make_operands(shape, 32, dtype, ints=True)
+    Ar, Br, biasr = make_operands(shape, 33, dtype)
+    Ri = np.random.default_rng(7).integers(-8, 9, (M, N)).astype(np.float32)
+    Rr = np.random.default_rng(8).normal(0.0, 1.0, (M, N)).astype(np.float32)
+    lim = nj.nnjit_device_limits_query(0)
+    desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, epilogue="relu", residual=True,
+                        flags=nj.NNJIT_PLAN_NO_CACHE)
+    cands, _ = nj.nnjit_space_enumerate(desc, lim)
+    for i, c in enumerate(cands):
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            C = run_plan(plan, Ai, Bi, biasi, M, N, C=torch.from_numpy(Ri.copy()).cuda())
+        try:
+            compare(C, Ai, Bi, biasi, layout, dtype, exact=True, act="relu", residual=Ri)
+        except AssertionError as e:
+            raise AssertionError(f"candidate {i} {c}: {e}") from None
+    desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, epilogue="gelu", residual=True,
+                        flags=nj.NNJIT_PLAN_NO_CACHE)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        C = run_plan(plan, Ar, Br, biasr, M, N, C=torch.from_numpy(Rr.copy()).cuda())
+    compare(C, Ar, Br, biasr, layout, dtype, act="gelu", residual=Rr)
+
+
+def test_residual_edge_cases():
+    """Residual with direct stores (ldc = N + 1 rules the TMA store out), batched outputs
+    (stride_c), K = 0 (C = bias + C), no activation, and a 4-bit weight GEMV."""
+    torch = pytest.importorskip("torch")
+    lim = nj.nnjit_device_limits_query(0)
+    rng = np.random.default_rng(9)
+    # direct stores, bf16 and tf32 tensor-core tiles
+    for dtype in ("bf16", "tf32"):
+        M, N, K = 130, 72, 64
+        shape = Shape("t", M, N, K, 1, "NK", True)
+        A, B, bias = make_operands(shape, 34, dtype, ints=True)
+        R = rng.integers(-8, 9, (M, N + 1)).astype(np.float32)
+        desc = nj.make_desc(M, N, K, dtype, "NK", has_bias=True, ldc=N + 1, residual=True,
+                            flags=nj.NNJIT_PLAN_NO_CACHE)
+        cands, _ = nj.nnjit_space_enumerate(desc, lim)
+        for i in range(len(cands)):
+            Cd = torch.from_numpy(R.copy()).cuda()
+            with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+                plan.run(dev(A), dev(B), dev(bias), Cd)
+                torch.cuda.synchronize()
+                plan.check()
+            Cn = Cd.cpu().numpy()
+            assert np.array_equal(Cn[:, N], R[:, N])                    # the gap is untouched
+            compare(np.ascontiguousarray(Cn[:, :N]), A, B, bias, "NK", dtype, exact=True,
+                    residual=R[:, :N])
+    # batched (no bias), every candidate
+    shape = Shape("t", 100, 96, 64, 3, "NK", False)
+    A, B, _ = make_operands(shape, 35, "bf16", ints=True)
+    R = rng.integers(-8, 9, (3, 100, 96)).astype(np.float32)
+    desc = nj.make_desc(100, 96, 64, "bf16", "NK", batch=3, residual=True, flags=nj.NNJIT_PLAN_NO_CACHE)
+    cands, _ = nj.nnjit_space_enumerate(desc, lim)
+    for i in range(len(cands)):
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            C = run_plan(plan, A, B, None, 100, 96, batch=3, C=torch.from_numpy(R.copy()).cuda())
+        compare(C, A, B, None, "NK", "bf16", exact=True, residual=R)
+    # K = 0: C = bias + C
+    bias = rng.integers(-8, 9, 40).astype(np.float32)
+    R = rng.integers(-8, 9, (5, 40)).astype(np.float32)
+    desc = nj.make_desc(5, 40, 0, "bf16", "NK", has_bias=True, residual=True, flags=nj.NNJIT_PLAN_NO_CACHE)
+    with nj.nnjit_matmul_plan_ex(desc, 0.0) as plan:
+        Cd = torch.from_numpy(R.copy()).cuda()
+        plan.run(dev(np.zeros((5, 1), np.uint16)), dev(np.zeros((40, 1), np.uint16)), dev(bias), Cd)
+        torch.cuda.synchronize()
+        plan.check()
+    assert np.array_equal(Cd.cpu().numpy(), R + bias)
+    # 4-bit weights, every candidate
+    from synthetic import make_w4_operands
+    from oracle.quant import matmul as w4_matmul
+    M, N, K = 2, 520, 4096
+    shape = Shape("t", M, N, K, 1, "NK", True)
+    x, blob, bias = make_w4_operands(shape, 36, ints=True)
+    R = rng.integers(-8, 9, (M, N)).astype(np.float32)
+    desc = nj.make_desc(M, N, K, "w4_bf16", "NK", has_bias=True, epilogue="relu", residual=True,
+                        flags=nj.NNJIT_PLAN_NO_CACHE)
+    cands, _ = nj.nnjit_space_enumerate(desc, lim)
+    _, want = w4_matmul(x, blob, N, K, 0, bias, "relu", residual=R)
+    for i in range(len(cands)):
+        with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+            C = run_plan(plan, x, blob, bias, M, N, C=torch.from_numpy(R.copy()).cuda())
+        assert np.array_equal(C, want), i

@@ -299,3 +299,21 @@ def test_w4_matmul_small_integers_bruteforce():
     C64, _ = w4_matmul(x_bits, blob, N, K)
     want = [[sum(int(xi[m, k]) * (int(codes[n, k]) - 8) for k in range(K)) for n in range(N)] for m in range(M)]
     assert np.array_equal(C64, np.array(want, dtype=np.float64))
+
+
+def test_residual_is_added_after_the_activation():
+    """C = act(A.Bt + bias) + R: with A = 0 the result is act(bias) + R; relu on integer
+    sums then an integer residual stays exact; a residual of the wrong shape is refused."""
+    from oracle.epilogue import apply
+    bias = np.array([-2.0, 0.5, 3.0], dtype=np.float32)
+    R = np.arange(6, dtype=np.float32).reshape(2, 3) - 2.5
+    C64, C32 = oracle.matmul(np.zeros((2, 4), np.float32), np.ones((4, 3), np.float32), bias,
+                             oracle.B_KN, act="gelu", residual=R)
+    assert np.array_equal(C64, apply(np.broadcast_to(bias.astype(np.float64), (2, 3)), "gelu") + R)
+    A = np.array([[1, -2], [3, 1]], np.float32)
+    B = np.array([[1, 1], [2, -1]], np.float32)
+    R = np.array([[10, -10], [0, 7]], np.float32)
+    C64, _ = oracle.matmul(A, B, None, oracle.B_KN, act="relu", residual=R)
+    assert np.array_equal(C64, np.array([[10.0, -7.0], [5.0, 9.0]]))
+    with pytest.raises(ValueError):
+        oracle.matmul(A, B, None, oracle.B_KN, residual=np.zeros((2, 3), np.float32))
