@@ -370,6 +370,30 @@ nnjit_status nnjit_plan_candidate(nnjit_plan p, nnjit_candidate* out);
 nnjit_status nnjit_plan_destroy(nnjit_plan p);
 
 /*
+ * Fused attention (the QK^T -> softmax -> PV neighbours of the attention BatchMatMuls of
+ * Table 3, K2 and K3): for each of `batch` independent problems (batch x heads),
+ *   S = scale * Q K^T,  P = softmax over each row of S (keys j masked off are left out),
+ *   O = P V,
+ * without writing S or P to memory.  Q [batch][Lq][d], K and V [batch][Lk][d] packed
+ * bfloat16, O [batch][Lq][d] packed float32, all device pointers the caller owns, 16-byte
+ * aligned.  d is 64 or 128.  With causal = 1 query i sees keys j <= i + (Lk - Lq) (the
+ * causal mask aligned to the last key, as in decoding with a cache); a query that sees no
+ * key gets O = 0.  The scores are accumulated in float32 from exact bfloat16 products;
+ * P is rounded to bfloat16 for the P V product, whose sums are float32.  Lq, Lk >= 0
+ * (0 is a no-op), batch >= 1, Lq, Lk, batch < 2^31.  INVALID_ARG for a bad descriptor or
+ * NULL pointer, UNSUPPORTED for another d or unaligned pointers.  Asynchronous on
+ * `stream`; allocates nothing.
+ */
+typedef struct {
+    int64_t batch, Lq, Lk, d;
+    int32_t causal;
+    float scale;
+} nnjit_attention_desc;
+
+nnjit_status nnjit_attention(const nnjit_attention_desc* desc, const void* Q, const void* K,
+                             const void* V, float* O, void* stream);
+
+/*
  * Decode GEMV that allocates nothing (the paper has no counterpart; this serves callers
  * that cannot allocate device memory when they run a product, e.g. a process whose
  * device memory a framework's caching allocator has already reserved, or a decode loop

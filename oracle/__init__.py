@@ -10,6 +10,9 @@ written from the paper:
     plain Python, plus the Blackwell readings of those rules used by the library.
   * ``epilogue`` -- the activations a kernel may apply after the bias (textbook
     definitions of ReLU, GELU and SiLU in FP64).
+  * ``quant``   -- 4-bit weights with bf16 group scales, dequantised in FP64.
+  * ``attention`` -- softmax attention between the two attention BatchMatMuls (Table 3,
+    K2 and K3), its definition in FP64.
 
 Only tests/, ``__graft_entry__.smoke()`` and bench.py's CPU-baseline / reference legs
 may import this package.  The GPU library shares no code with it.

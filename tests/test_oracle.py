@@ -317,3 +317,72 @@ def test_residual_is_added_after_the_activation():
     assert np.array_equal(C64, np.array([[10.0, -7.0], [5.0, 9.0]]))
     with pytest.raises(ValueError):
         oracle.matmul(A, B, None, oracle.B_KN, residual=np.zeros((2, 3), np.float32))
+
+
+# ---------------------------------------------------------------- attention
+
+def _bf(x):
+    return f32_to_bf16_bits(np.asarray(x, dtype=np.float32))
+
+
+def test_attention_bruteforce_tiny():
+    """Pure-Python loops with math.exp on a tiny causal and non-causal case."""
+    import math
+    from oracle.attention import attention
+    rng = np.random.default_rng(10)
+    Q = rng.integers(-3, 4, (1, 3, 4)).astype(np.float32)
+    K = rng.integers(-3, 4, (1, 5, 4)).astype(np.float32)
+    V = rng.integers(-3, 4, (1, 5, 4)).astype(np.float32)
+    for causal in (False, True):
+        O = attention(_bf(Q), _bf(K), _bf(V), 0.5, causal)
+        for i in range(3):
+            last = i + 2 if causal else 4
+            s = [0.5 * sum(float(Q[0, i, c]) * float(K[0, j, c]) for c in range(4)) for j in range(last + 1)]
+            mx = max(s)
+            w = [math.exp(x - mx) for x in s]
+            tot = sum(w)
+            for c in range(4):
+                want = sum(w[j] / tot * float(V[0, j, c]) for j in range(last + 1))
+                assert abs(O[0, i, c] - want) < 1e-12
+
+
+def test_attention_closed_forms():
+    """One key: O = that value row.  Q = 0: uniform weights, O = the mean of the visible
+    value rows (prefix means when causal).  A dominant key takes all the weight.  Causal
+    with Lq > Lk: queries that see no key get 0, and query Lq - Lk sees key 0 only."""
+    from oracle.attention import attention
+    rng = np.random.default_rng(11)
+    V = rng.integers(-4, 5, (2, 6, 8)).astype(np.float32)
+    K = rng.integers(-4, 5, (2, 6, 8)).astype(np.float32)
+    Q = rng.integers(-4, 5, (2, 3, 8)).astype(np.float32)
+    O = attention(_bf(Q), _bf(K[:, :1]), _bf(V[:, :1]), 0.125)
+    assert np.array_equal(O, np.broadcast_to(V[:, :1].astype(np.float64), O.shape))
+    O = attention(_bf(np.zeros((2, 6, 8))), _bf(K), _bf(V), 1.0, causal=True)
+    want = np.cumsum(V.astype(np.float64), axis=1) / np.arange(1, 7)[None, :, None]
+    assert np.max(np.abs(O - want)) < 1e-12
+    Kd = np.zeros((1, 4, 8), np.float32)
+    Kd[0, 2] = 64.0
+    Qd = np.full((1, 2, 8), 64.0, np.float32)
+    O = attention(_bf(Qd), _bf(Kd), _bf(V[:1, :4]), 1.0)
+    assert np.max(np.abs(O - V[0, 2].astype(np.float64))) < 1e-12
+    O = attention(_bf(Q[:1, :3]), _bf(K[:1, :2]), _bf(V[:1, :2]), 0.5, causal=True)
+    assert np.array_equal(O[0, 0], np.zeros(8))
+    assert np.array_equal(O[0, 1], V[0, 0].astype(np.float64))
+
+
+def test_attention_invariances():
+    """Permuting keys and values together leaves O unchanged; adding one vector u to every
+    key shifts each row's scores by a constant (softmax is shift-invariant); with every
+    value row equal to ones, O is one (the weights sum to one)."""
+    from oracle.attention import attention
+    rng = np.random.default_rng(12)
+    Q = rng.integers(-2, 3, (3, 5, 16)).astype(np.float32)
+    K = rng.integers(-2, 3, (3, 7, 16)).astype(np.float32)
+    V = rng.normal(0.0, 1.0, (3, 7, 16)).astype(np.float32)
+    O = attention(_bf(Q), _bf(K), _bf(V), 0.25)
+    perm = rng.permutation(7)
+    assert np.max(np.abs(attention(_bf(Q), _bf(K[:, perm]), _bf(V[:, perm]), 0.25) - O)) < 1e-12
+    u = rng.integers(-2, 3, 16).astype(np.float32)
+    assert np.max(np.abs(attention(_bf(Q), _bf(K + u), _bf(V), 0.25) - O)) < 1e-12
+    ones = attention(_bf(Q), _bf(K), _bf(np.ones_like(V)), 0.25, causal=True)
+    assert np.max(np.abs(ones - 1.0)) < 1e-12
