@@ -9,6 +9,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <cmath>
 #include <chrono>
 #include <cstdio>
 #include <cstdlib>
@@ -594,6 +595,24 @@ const char* nnjit_status_string(nnjit_status s) {
 const char* nnjit_last_error(void) { return t_last_error.c_str(); }
 
 int32_t nnjit_version(void) { return 100; }
+
+nnjit_status nnjit_attention(const nnjit_attention_desc* d, const void* Q, const void* K, const void* V,
+                             float* O, void* stream) {
+    if (!d) return fail(NNJIT_ERR_INVALID_ARG, "descriptor is NULL");
+    const int64_t lim = (int64_t)1 << 31;
+    if (d->batch < 1 || d->Lq < 0 || d->Lk < 0 || d->batch >= lim || d->Lq >= lim || d->Lk >= lim)
+        return fail(NNJIT_ERR_INVALID_ARG, "need batch >= 1 and 0 <= Lq, Lk < 2^31");
+    if (d->causal != 0 && d->causal != 1) return fail(NNJIT_ERR_INVALID_ARG, "causal must be 0 or 1");
+    if (!std::isfinite(d->scale)) return fail(NNJIT_ERR_INVALID_ARG, "scale must be finite");
+    if (d->d != 64 && d->d != 128) return fail(NNJIT_ERR_UNSUPPORTED, "head dimension must be 64 or 128");
+    if (d->Lq == 0) return NNJIT_OK;
+    if (!Q || !O || (d->Lk > 0 && (!K || !V))) return fail(NNJIT_ERR_INVALID_ARG, "NULL pointer");
+    auto a16 = [](const void* p) { return !p || (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
+    if (!a16(Q) || !a16(K) || !a16(V) || !a16(O)) return fail(NNJIT_ERR_UNSUPPORTED, "pointers must be 16-byte aligned");
+    cudaError_t e = launch_attention(*d, Q, K, V, O, static_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+    return NNJIT_OK;
+}
 
 nnjit_status nnjit_w4_layout(int64_t N, int64_t K, int64_t ldb, int64_t* scale_offset_bytes,
                              int64_t* total_bytes) {

@@ -107,4 +107,8 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
                                   const void* B, CUtensorMap* ta, CUtensorMap* tb,
                                   const char** why);
 
+// Fused attention (nnjit_attention); the descriptor is validated by the caller.
+cudaError_t launch_attention(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
+                             float* O, cudaStream_t stream);
+
 }  // namespace nnjit

@@ -72,6 +72,11 @@ class nnjit_candidate(ctypes.Structure):
                         ("cluster_m", ctypes.c_int32)]
 
 
+class nnjit_attention_desc(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int64), ("Lq", ctypes.c_int64), ("Lk", ctypes.c_int64),
+                ("d", ctypes.c_int64), ("causal", ctypes.c_int32), ("scale", ctypes.c_float)]
+
+
 NNJIT_SETTING_FREE = -1
 SETTING_AXES = ("raster", "kgroup", "reduce", "multicast")
 
@@ -133,6 +138,7 @@ def load_library(path: str = LIB_PATH):
             "nnjit_cache_load": [ctypes.c_char_p, P(i32)],
             "nnjit_w4_layout": [i64, i64, i64, P(i64), P(i64)],
             "nnjit_settings_set": [P(nnjit_settings)],
+            "nnjit_attention": [P(nnjit_attention_desc), vp, vp, vp, vp, vp],
             "nnjit_settings_get": [P(nnjit_settings)],
             "nnjit_settings_study": [P(nnjit_matmul_desc), i32, P(nnjit_settings), ctypes.c_char_p,
                                      ctypes.c_size_t, P(ctypes.c_size_t)],
@@ -412,3 +418,15 @@ def nnjit_settings_study(descs) -> tuple[dict, dict]:
     if need.value > size:
         raise RuntimeError(f"settings report truncated ({need.value} > {size} bytes)")
     return struct_to_dict(out), json.loads(buf.value.decode())
+
+
+def nnjit_attention(Q, K, V, O, causal=False, scale=None, stream=None):
+    """O = softmax(scale Q K^T) V per leading index (batch x heads).  Q [B][Lq][d], K and V
+    [B][Lk][d] bf16 tensors, O [B][Lq][d] float32 (device tensors); scale defaults to
+    1 / sqrt(d)."""
+    B, Lq, d = Q.shape
+    Lk = K.shape[1]
+    desc = nnjit_attention_desc(B, Lq, Lk, d, 1 if causal else 0,
+                                float(scale) if scale is not None else 1.0 / float(d) ** 0.5)
+    _check(load_library().nnjit_attention(ctypes.byref(desc), _ptr(Q), _ptr(K), _ptr(V), _ptr(O),
+                                          _stream(stream)), "nnjit_attention")
