@@ -380,18 +380,30 @@ nnjit_status nnjit_plan_destroy(nnjit_plan p);
  * causal mask aligned to the last key, as in decoding with a cache); a query that sees no
  * key gets O = 0.  The scores are accumulated in float32 from exact bfloat16 products;
  * P is rounded to bfloat16 for the P V product, whose sums are float32.  Lq, Lk >= 0
- * (0 is a no-op), batch >= 1, Lq, Lk, batch < 2^31.  INVALID_ARG for a bad descriptor or
- * NULL pointer, UNSUPPORTED for another d or unaligned pointers.  Asynchronous on
- * `stream`; allocates nothing.
+ * (Lq = 0 is a no-op), batch >= 1, Lq, Lk, batch < 2^31.  `kernel` selects the
+ * implementation: NNJIT_ATTN_AUTO (0) and NNJIT_ATTN_TCGEN05 (1) run the tensor-memory
+ * kernel (128 queries per CTA, scores and outputs in TMEM, bounded waits), NNJIT_ATTN_MMA
+ * (2) the warp-level MMA kernel (64 queries per CTA, no waits).  INVALID_ARG for a bad
+ * descriptor or NULL pointer, UNSUPPORTED for another d or unaligned pointers.
+ * Asynchronous on `stream`; allocates nothing.  An expired wait inside the tensor-memory
+ * kernel is reported by nnjit_attention_check.
  */
+typedef enum { NNJIT_ATTN_AUTO = 0, NNJIT_ATTN_TCGEN05 = 1, NNJIT_ATTN_MMA = 2 } nnjit_attention_kernel;
+
 typedef struct {
     int64_t batch, Lq, Lk, d;
     int32_t causal;
     float scale;
+    int32_t kernel;  /* nnjit_attention_kernel */
 } nnjit_attention_desc;
 
 nnjit_status nnjit_attention(const nnjit_attention_desc* desc, const void* Q, const void* K,
                              const void* V, float* O, void* stream);
+
+/* Synchronise the current device and report whether any tensor-memory attention kernel
+ * since the last check gave up on a wait (NNJIT_ERR_TIMEOUT, with the wait's code in
+ * nnjit_last_error); clears the record. */
+nnjit_status nnjit_attention_check(void);
 
 /*
  * Decode GEMV that allocates nothing (the paper has no counterpart; this serves callers

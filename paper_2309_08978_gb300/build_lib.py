@@ -18,7 +18,7 @@ LIB = os.path.join(BUILD, "libnnjit.so")
 INCLUDE = os.path.join(ROOT, "include")
 
 CUDA_SOURCES = ["capi.cu", "kernels_tc.cu", "kernels_tc2.cu", "kernels_gemv.cu", "kernels_gemv_tma.cu", "kernels_gemv_w4.cu", "kernels_ffma.cu",
-                "kernels_ffma_kn.cu", "kernels_ffma_nk.cu", "noalloc.cu", "attention.cu"]
+                "kernels_ffma_kn.cu", "kernels_ffma_nk.cu", "noalloc.cu", "attention.cu", "attention_tc.cu"]
 CXX_SOURCES = ["space.cpp"]
 HEADERS = ["space.h", "launch.h", "ptx.cuh", "ffma.cuh", "epilogue.cuh"]
 

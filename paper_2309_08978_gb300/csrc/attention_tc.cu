@@ -1,0 +1,422 @@
+// Fused attention on the 5th-generation tensor cores (nnjit_attention, kernel 1):
+// O = softmax(scale Q K^T) V per batch x head without writing the scores.
+//
+// One CTA takes 128 queries of one problem; 6 warps:
+//   warp 0     TMA producer: the Q tile once, then key and value blocks of 128 rows
+//              through an S-slot ring (128-byte swizzle; keys K-major, values MN-major);
+//   warp 1     allocates TMEM and issues, from one thread, S_j = Q K_j^T (M = 128,
+//              N = 128, K = d) into one of two TMEM score buffers, and O_j = P_j V_j
+//              (M = 128, N = d, K = 128) into one of two TMEM output buffers;
+//   warps 2-9  softmax: warps w and w + 4 share TMEM lane quarter w % 4 (32 query rows)
+//              and split each row in two halves of 64 keys and d / 2 output columns.
+//              Row maximum over S_j (first pass over TMEM; the halves' maxima meet through
+//              shared memory behind a barrier of the warp pair), then p = 2^(s - m)
+//              written as bf16 into a shared-memory P buffer in the MMA's K-major
+//              swizzled layout (second pass), and, one block behind, the running output
+//              O = O * 2^(m_old - m_new) + O_j accumulated in registers.
+// The score and output buffers, P and the ring are double-buffered so that the tensor
+// cores work on block j + 1 while the softmax warps work on block j.  Keys past Lk and,
+// with the causal mask, keys past i + (Lk - Lq) score -inf; blocks a CTA cannot see are
+// skipped.  Every wait is bounded: on expiry the watchdog word is set, the CTA's abort
+// flag raised, and every role leaves after draining what it issued.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstdint>
+
+#include "../../include/nnjit.h"
+#include "launch.h"
+#include "ptx.cuh"
+
+namespace nnjit {
+
+namespace {
+
+__device__ int g_attn_watchdog;  // first expired wait's code (0: none)
+
+constexpr int kQ = 128;   // queries per CTA
+constexpr int kKV = 128;  // keys per block
+constexpr int kThreads = 320;  // producer, MMA issuer, 8 softmax warps
+constexpr int kErrProd = 0x301, kErrMmaQ = 0x311, kErrMmaKv = 0x312, kErrMmaS = 0x313, kErrMmaP = 0x314;
+constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrDrain = 0x331;
+
+template <int D>
+struct Cfg {
+    static constexpr int kStages = D == 64 ? 3 : 2;
+    static constexpr uint32_t kQBytes = kQ * D * 2;
+    static constexpr uint32_t kKBytes = kKV * D * 2;
+    static constexpr uint32_t kVBytes = kKV * D * 2;
+    static constexpr uint32_t kStageBytes = kKBytes + kVBytes;
+    static constexpr uint32_t kPBytes = kQ * kKV * 2;
+    static constexpr uint32_t kSmem = 1024 + kQBytes + kStages * kStageBytes + 2 * kPBytes;
+};
+
+struct Params {
+    CUtensorMap tq, tk, tv;
+    float* O;
+    int Lq, Lk, causal, qblocks;
+    float scale_log2;
+};
+
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    uint32_t r;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+    return r;
+}
+
+// 32 lanes x 16 consecutive 32-bit TMEM columns (thread t: lane base + t), and the wait.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]),
+                   "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]),
+                   "+r"(r[14]), "+r"(r[15])
+                 :
+                 : "memory");
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
+                 : "memory");
+}
+
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_constant__ Params p) {
+    using C = Cfg<D>;
+    constexpr int S = C::kStages;
+    constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
+    extern __shared__ uint8_t raw[];
+    __shared__ __align__(8) uint64_t bars[16];
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_word;
+    // [half][row]: partial row maxima, then sums.  One buffer is enough: a pair barrier
+    // (the vote on the next wait) separates each read from the next write.
+    __shared__ float red[2][kQ];
+    volatile int* abort_flag = &abort_word;
+    int* err = &g_attn_watchdog;
+
+    const uint32_t base = (ptx::smem_u32(raw) + 1023u) & ~1023u;
+    const uint32_t sQ = base, sKV = base + C::kQBytes, sP = sKV + S * C::kStageBytes;
+    auto sK = [&](int s) { return sKV + (uint32_t)s * C::kStageBytes; };
+    auto sV = [&](int s) { return sKV + (uint32_t)s * C::kStageBytes + C::kKBytes; };
+    auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
+    const uint32_t q_full = bar(0), drain_bar = bar(15);
+    auto kv_full = [&](int s) { return bar(1 + s); };
+    auto kv_empty = [&](int s) { return bar(4 + s); };
+    auto s_full = [&](int i) { return bar(7 + i); };
+    auto s_empty = [&](int i) { return bar(9 + i); };
+    auto p_full = [&](int i) { return bar(11 + i); };
+    auto o_full = [&](int i) { return bar(13 + i); };
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int b = (int)(blockIdx.x / p.qblocks);
+    const int q0 = (int)(blockIdx.x % p.qblocks) * kQ;
+    const int shift = p.Lk - p.Lq;
+    int kv_end = p.Lk;
+    if (p.causal) kv_end = min(p.Lk, max(0, min(q0 + kQ, p.Lq) - 1 + shift + 1));
+    const int nblocks = (kv_end + kKV - 1) / kKV;
+
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(q_full, 1);
+        for (int s = 0; s < S; ++s) {
+            ptx::mbar_init(kv_full(s), 1);
+            ptx::mbar_init(kv_empty(s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            ptx::mbar_init(s_full(i), 1);
+            ptx::mbar_init(s_empty(i), 256);
+            ptx::mbar_init(p_full(i), 256);
+            ptx::mbar_init(o_full(i), 1);
+        }
+        ptx::mbar_init(drain_bar, 1);
+        abort_word = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(&tmem_slot), 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0 && nblocks > 0) {
+            ptx::prefetch_tmap(&p.tq);
+            ptx::prefetch_tmap(&p.tk);
+            ptx::prefetch_tmap(&p.tv);
+            ptx::mbar_arrive_expect_tx(q_full, C::kQBytes);
+            for (int kb = 0; kb < kDB; ++kb) ptx::tma_load_3d(sQ + kb * 16384u, &p.tq, kb * 64, q0, b, q_full);
+            uint32_t armed = 0, armed_parity = 0;
+            int stage = 0;
+            uint32_t phase = 0;
+            for (int j = 0; j < nblocks; ++j) {
+                if (!ptx::mbar_wait(kv_empty(stage), phase ^ 1u, abort_flag, err, kErrProd)) break;
+                ptx::mbar_arrive_expect_tx(kv_full(stage), C::kStageBytes);
+                for (int kb = 0; kb < kDB; ++kb)
+                    ptx::tma_load_3d(sK(stage) + kb * 16384u, &p.tk, kb * 64, j * kKV, b, kv_full(stage));
+                for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
+                    for (int a = 0; a < kDB; ++a)    // 64 columns of d per swizzle atom
+                        ptx::tma_load_3d(sV(stage) + kb * (D * 128u) + a * 8192u, &p.tv, a * 64, j * kKV + kb * 64,
+                                         b, kv_full(stage));
+                armed |= 1u << stage;
+                armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
+                if (++stage == S) {
+                    stage = 0;
+                    phase ^= 1u;
+                }
+            }
+            volatile int no_abort = 0;
+            ptx::mbar_wait(q_full, 0, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int s = 0; s < S; ++s)
+                if (armed & (1u << s))
+                    ptx::mbar_wait(kv_full(s), (armed_parity >> s) & 1u, &no_abort, err, kErrDrain,
+                                   ptx::kWaitLimitNs / 4);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        if (lane == 0 && nblocks > 0) {
+            constexpr uint32_t kIdescS = ptx::instr_desc(1u, false, kQ, kKV);
+            constexpr uint32_t kIdescO = ptx::instr_desc(1u, true, kQ, D);
+            bool ok = ptx::mbar_wait(q_full, 0, abort_flag, err, kErrMmaQ);
+            ptx::tc_fence_after();
+            auto issue_s = [&](int j) -> bool {
+                const int sb = j & 1, st = j % S;
+                if (j >= 2 && !ptx::mbar_wait(s_empty(sb), ((j - 2) >> 1) & 1, abort_flag, err, kErrMmaS))
+                    return false;
+                if (!ptx::mbar_wait(kv_full(st), (uint32_t)((j / S) & 1), abort_flag, err, kErrMmaKv)) return false;
+                ptx::tc_fence_after();
+                const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
+#pragma unroll
+                for (int kb = 0; kb < kDB; ++kb) {
+                    const uint64_t ad = ptx::smem_desc(sQ + kb * 16384u, 16, 1024);
+                    const uint64_t bd = ptx::smem_desc(sK(st) + kb * 16384u, 16, 1024);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        ptx::mma_ss<0>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdescS, (kb | kk) ? 1u : 0u);
+                }
+                ptx::tc_commit(s_full(sb));
+                return true;
+            };
+            if (ok) ok = issue_s(0);
+            for (int j = 0; ok && j < nblocks; ++j) {
+                if (j + 1 < nblocks && !issue_s(j + 1)) break;
+                if (!ptx::mbar_wait(p_full(j & 1), (j >> 1) & 1, abort_flag, err, kErrMmaP)) break;
+                ptx::tc_fence_after();
+                const int st = j % S;
+                const uint32_t o_tmem = tmem + 2u * kKV + (uint32_t)(j & 1) * D;
+#pragma unroll
+                for (int kb = 0; kb < 2; ++kb) {
+                    const uint64_t ad = ptx::smem_desc(sP + (uint32_t)(j & 1) * C::kPBytes + kb * 16384u, 16, 1024);
+                    const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)
+                        ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (kb | kk) ? 1u : 0u);
+                }
+                ptx::tc_commit(o_full(j & 1));
+                ptx::tc_commit(kv_empty(st));
+            }
+            // every MMA issued here has completed before TMEM is freed
+            ptx::tc_commit(drain_bar);
+            volatile int no_abort = 0;
+            ptx::mbar_wait(drain_bar, 0, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+        }
+    } else {
+        // ------------------------------------------------------------ softmax warps
+        const int q = warp & 3;
+        const int half = (warp - 2) >> 2;
+        const int row = q * 32 + lane;
+        const int qrow = q0 + row;
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
+        constexpr int kOH = D / 2;                             // output columns of this half
+        float o[kOH];
+#pragma unroll
+        for (int c = 0; c < kOH; ++c) o[c] = 0.0f;
+        float m = -INFINITY, l = 0.0f, alpha_prev = 0.0f;
+        bool ok = true;
+        // barrier of the two warps of lane quarter q; the vote keeps them leaving together
+        auto pair_any = [&](bool v) -> bool {
+            uint32_t r;
+            asm volatile(
+                "{\n\t.reg .pred a, b;\n\t"
+                "setp.ne.u32 a, %1, 0;\n\t"
+                "barrier.cta.red.or.pred b, %2, 64, a;\n\t"
+                "selp.u32 %0, 1, 0, b;\n\t}"
+                : "=r"(r)
+                : "r"((uint32_t)v), "r"(1 + q)
+                : "memory");
+            return r != 0;
+        };
+        // the output of block jb (one behind the softmax) into the running sum
+        auto accumulate = [&](int jb) -> bool {
+            const bool ready = ptx::mbar_wait(o_full(jb & 1), (jb >> 1) & 1, abort_flag, err, kErrSoftO);
+            if (pair_any(!ready)) return false;
+            ptx::tc_fence_after();
+            const uint32_t ob = tmem + lane_base + 2u * kKV + (uint32_t)(jb & 1) * D + (uint32_t)(half * kOH);
+#pragma unroll
+            for (int c = 0; c < kOH / 16; ++c) {
+                uint32_t r[16];
+                tmem_ld16(ob + c * 16, r);
+                tmem_wait16(r);
+#pragma unroll
+                for (int i = 0; i < 16; ++i) o[c * 16 + i] = fmaf(o[c * 16 + i], alpha_prev, __uint_as_float(r[i]));
+            }
+            ptx::tc_fence_before();
+            return true;
+        };
+        for (int j = 0; j < nblocks; ++j) {
+            const int sb = j & 1;
+            const bool ready = ptx::mbar_wait(s_full(sb), (j >> 1) & 1, abort_flag, err, kErrSoftS);
+            if (pair_any(!ready)) {
+                ok = false;
+                break;
+            }
+            ptx::tc_fence_after();
+            const uint32_t sa = tmem + lane_base + (uint32_t)sb * kKV + (uint32_t)(half * 64);
+            // columns 0..lim of this half are visible
+            const int lim = min(last, p.Lk - 1) - j * kKV - half * 64;
+            // pass 1: this half's maximum (scaled, base 2), then the row's
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t r[16];
+                tmem_ld16(sa + c * 16, r);
+                tmem_wait16(r);
+#pragma unroll
+                for (int i = 0; i < 16; ++i)
+                    if (c * 16 + i <= lim) mx = fmaxf(mx, __fmul_rn(__uint_as_float(r[i]), p.scale_log2));
+            }
+            red[half][row] = mx;
+            asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+            mx = fmaxf(mx, red[half ^ 1][row]);
+            const float mn = fmaxf(m, mx);
+            const float basev = mn == -INFINITY ? 0.0f : mn;  // no visible key yet: every p is 0
+            const float alpha = ex2(m - basev);
+            m = mn;
+            l *= alpha;
+            // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: this half is
+            // the row's 128-byte segment of K-block `half`; 16-byte chunk u at u ^ (row % 8))
+            const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)half * 16384u + (uint32_t)row * 128u;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {  // 16 keys per chunk: two 16-byte chunks of P
+                uint32_t r[16];
+                tmem_ld16(sa + c * 16, r);
+                tmem_wait16(r);
+                uint32_t pk[8];
+#pragma unroll
+                for (int i = 0; i < 16; i += 2) {
+                    const int col = c * 16 + i;
+                    // the product rounded as in the first pass (no contraction into an FMA), so
+                    // the row's maximum gives exactly 2^0 = 1
+                    const float p0 =
+                        col <= lim ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(r[i]), p.scale_log2), basev)) : 0.0f;
+                    const float p1 =
+                        col + 1 <= lim ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(r[i + 1]), p.scale_log2), basev)) : 0.0f;
+                    l += p0 + p1;
+                    pk[i >> 1] = pack_bf16(p0, p1);
+                }
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const uint32_t ch = (uint32_t)(c * 2 + u);
+                    st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
+                                 pk[4 * u + 3]);
+                }
+            }
+            ptx::tc_fence_before();
+            ptx::mbar_arrive(s_empty(sb));
+            ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
+            ptx::mbar_arrive(p_full(sb));
+            if (j >= 1 && !accumulate(j - 1)) {
+                ok = false;
+                break;
+            }
+            alpha_prev = alpha;
+        }
+        if (ok && nblocks > 0) ok = accumulate(nblocks - 1);
+        // the row sum is the two halves' sums (both relative to the same maximum)
+        red[half][row] = l;
+        asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+        l += red[half ^ 1][row];
+        if (qrow < p.Lq) {
+            const float inv = (ok && l > 0.0f) ? 1.0f / l : 0.0f;
+            float* dst = p.O + ((size_t)b * p.Lq + qrow) * D + half * kOH;
+#pragma unroll
+            for (int c = 0; c < kOH; c += 4)
+                *reinterpret_cast<float4*>(dst + c) = make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
+        }
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem, 512);
+}
+
+}  // namespace
+
+cudaError_t attention_watchdog_take(int* word) {
+    cudaError_t e = cudaMemcpyFromSymbol(word, g_attn_watchdog, sizeof(int));
+    if (e != cudaSuccess || *word == 0) return e;
+    const int zero = 0;
+    return cudaMemcpyToSymbol(g_attn_watchdog, &zero, sizeof(int));
+}
+
+cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
+                                float* O, cudaStream_t stream) {
+    const int qblocks = (int)((d.Lq + kQ - 1) / kQ);
+    const long long ctas = (long long)qblocks * d.batch;
+    if (ctas <= 0) return cudaSuccess;
+    if (ctas >= (1LL << 31)) return cudaErrorInvalidValue;
+    if (d.Lk == 0) return cudaMemsetAsync(O, 0, (size_t)d.batch * d.Lq * d.d * sizeof(float), stream);
+    EncodeTiledFn enc = get_encode_fn();
+    if (!enc) return cudaErrorNotSupported;
+    Params p;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    auto encode = [&](CUtensorMap* m, const void* ptr, long long rows, cuuint32_t box_rows) {
+        const cuuint64_t dims[3] = {(cuuint64_t)d.d, (cuuint64_t)rows, (cuuint64_t)d.batch};
+        const cuuint64_t strides[2] = {(cuuint64_t)(d.d * 2), (cuuint64_t)(rows * d.d * 2)};
+        const cuuint32_t box[3] = {64, box_rows, 1};
+        return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(ptr), dims, strides, box, estr,
+                   CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    };
+    if (!encode(&p.tq, Q, d.Lq, kQ) || !encode(&p.tk, K, d.Lk, kKV) || !encode(&p.tv, V, d.Lk, 64))
+        return cudaErrorInvalidValue;
+    p.O = O;
+    p.Lq = (int)d.Lq;
+    p.Lk = (int)d.Lk;
+    p.causal = d.causal;
+    p.qblocks = qblocks;
+    p.scale_log2 = d.scale * 1.4426950408889634f;
+    static bool attr_set[2] = {false, false};
+    const int i = d.d == 64 ? 0 : 1;
+    const int smem = i == 0 ? (int)Cfg<64>::kSmem : (int)Cfg<128>::kSmem;
+    if (!attr_set[i]) {
+        cudaError_t e = cudaFuncSetAttribute(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>,
+                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        attr_set[i] = true;
+    }
+    return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3((unsigned)ctas),
+                      dim3(kThreads), (size_t)smem, stream, p);
+}
+
+}  // namespace nnjit

@@ -605,12 +605,28 @@ nnjit_status nnjit_attention(const nnjit_attention_desc* d, const void* Q, const
     if (d->causal != 0 && d->causal != 1) return fail(NNJIT_ERR_INVALID_ARG, "causal must be 0 or 1");
     if (!std::isfinite(d->scale)) return fail(NNJIT_ERR_INVALID_ARG, "scale must be finite");
     if (d->d != 64 && d->d != 128) return fail(NNJIT_ERR_UNSUPPORTED, "head dimension must be 64 or 128");
+    if (d->kernel < NNJIT_ATTN_AUTO || d->kernel > NNJIT_ATTN_MMA) return fail(NNJIT_ERR_INVALID_ARG, "unknown kernel");
     if (d->Lq == 0) return NNJIT_OK;
     if (!Q || !O || (d->Lk > 0 && (!K || !V))) return fail(NNJIT_ERR_INVALID_ARG, "NULL pointer");
     auto a16 = [](const void* p) { return !p || (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
     if (!a16(Q) || !a16(K) || !a16(V) || !a16(O)) return fail(NNJIT_ERR_UNSUPPORTED, "pointers must be 16-byte aligned");
-    cudaError_t e = launch_attention(*d, Q, K, V, O, static_cast<cudaStream_t>(stream));
+    cudaError_t e = d->kernel == NNJIT_ATTN_MMA ? launch_attention(*d, Q, K, V, O, static_cast<cudaStream_t>(stream))
+                                                : launch_attention_tc(*d, Q, K, V, O, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_attention_check(void) {
+    cudaError_t e = cudaDeviceSynchronize();
+    if (e != cudaSuccess) return cuda_fail(e, "attention check");
+    int word = 0;
+    e = attention_watchdog_take(&word);
+    if (e != cudaSuccess) return cuda_fail(e, "attention watchdog read");
+    if (word != 0) {
+        char msg[64];
+        std::snprintf(msg, sizeof msg, "attention wait expired (code 0x%x)", word);
+        return fail(NNJIT_ERR_TIMEOUT, msg);
+    }
     return NNJIT_OK;
 }
 

@@ -107,8 +107,13 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
                                   const void* B, CUtensorMap* ta, CUtensorMap* tb,
                                   const char** why);
 
-// Fused attention (nnjit_attention); the descriptor is validated by the caller.
+// Fused attention (nnjit_attention); the descriptor is validated by the caller.  The
+// warp-level MMA kernel, and the tensor-memory kernel with its watchdog word.
 cudaError_t launch_attention(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
                              float* O, cudaStream_t stream);
+cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
+                                float* O, cudaStream_t stream);
+// Read and clear the tensor-memory kernel's watchdog word (synchronous).
+cudaError_t attention_watchdog_take(int* word);
 
 }  // namespace nnjit

@@ -74,7 +74,11 @@ class nnjit_candidate(ctypes.Structure):
 
 class nnjit_attention_desc(ctypes.Structure):
     _fields_ = [("batch", ctypes.c_int64), ("Lq", ctypes.c_int64), ("Lk", ctypes.c_int64),
-                ("d", ctypes.c_int64), ("causal", ctypes.c_int32), ("scale", ctypes.c_float)]
+                ("d", ctypes.c_int64), ("causal", ctypes.c_int32), ("scale", ctypes.c_float),
+                ("kernel", ctypes.c_int32)]
+
+
+NNJIT_ATTN_AUTO, NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA = 0, 1, 2
 
 
 NNJIT_SETTING_FREE = -1
@@ -139,6 +143,7 @@ def load_library(path: str = LIB_PATH):
             "nnjit_w4_layout": [i64, i64, i64, P(i64), P(i64)],
             "nnjit_settings_set": [P(nnjit_settings)],
             "nnjit_attention": [P(nnjit_attention_desc), vp, vp, vp, vp, vp],
+            "nnjit_attention_check": [],
             "nnjit_settings_get": [P(nnjit_settings)],
             "nnjit_settings_study": [P(nnjit_matmul_desc), i32, P(nnjit_settings), ctypes.c_char_p,
                                      ctypes.c_size_t, P(ctypes.c_size_t)],
@@ -420,13 +425,17 @@ def nnjit_settings_study(descs) -> tuple[dict, dict]:
     return struct_to_dict(out), json.loads(buf.value.decode())
 
 
-def nnjit_attention(Q, K, V, O, causal=False, scale=None, stream=None):
+def nnjit_attention(Q, K, V, O, causal=False, scale=None, stream=None, kernel=NNJIT_ATTN_AUTO):
     """O = softmax(scale Q K^T) V per leading index (batch x heads).  Q [B][Lq][d], K and V
     [B][Lk][d] bf16 tensors, O [B][Lq][d] float32 (device tensors); scale defaults to
-    1 / sqrt(d)."""
+    1 / sqrt(d); kernel: NNJIT_ATTN_AUTO / _TCGEN05 / _MMA."""
     B, Lq, d = Q.shape
     Lk = K.shape[1]
     desc = nnjit_attention_desc(B, Lq, Lk, d, 1 if causal else 0,
-                                float(scale) if scale is not None else 1.0 / float(d) ** 0.5)
+                                float(scale) if scale is not None else 1.0 / float(d) ** 0.5, kernel)
     _check(load_library().nnjit_attention(ctypes.byref(desc), _ptr(Q), _ptr(K), _ptr(V), _ptr(O),
                                           _stream(stream)), "nnjit_attention")
+
+
+def nnjit_attention_check():
+    _check(load_library().nnjit_attention_check(), "nnjit_attention_check")

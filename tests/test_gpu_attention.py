@@ -25,11 +25,14 @@ def _dev(bits):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
 
 
-def _run(Q, K, V, causal, scale):
+KERNELS = {"tcgen05": 1, "mma": 2}
+
+
+def _run(Q, K, V, causal, scale, kernel=1):
     B, Lq, d = Q.shape
     O = torch.full((B, Lq, d), float("nan"), dtype=torch.float32, device="cuda")
-    nj.nnjit_attention(_dev(Q), _dev(K), _dev(V), O, causal=causal, scale=scale)
-    torch.cuda.synchronize()
+    nj.nnjit_attention(_dev(Q), _dev(K), _dev(V), O, causal=causal, scale=scale, kernel=kernel)
+    nj.nnjit_attention_check()
     return O.cpu().numpy()
 
 
@@ -38,12 +41,13 @@ CASES = [(2, 64, 64, 64, False), (3, 100, 130, 64, False), (2, 128, 128, 128, Tr
          (2, 1, 300, 128, True), (2, 333, 333, 128, False), (1, 65, 1, 64, False)]
 
 
+@pytest.mark.parametrize("kernel", list(KERNELS))
 @pytest.mark.parametrize("case", CASES, ids=lambda c: "b{}-q{}-k{}-d{}{}".format(*c[:4], "-causal" if c[4] else ""))
-def test_attention_matches_oracle(case):
+def test_attention_matches_oracle(case, kernel):
     B, Lq, Lk, d, causal = case
     Q, K, V = _bf16((B, Lq, d), 1), _bf16((B, Lk, d), 2), _bf16((B, Lk, d), 3)
     scale = 1.0 / np.sqrt(d)
-    O = _run(Q, K, V, causal, scale)
+    O = _run(Q, K, V, causal, scale, KERNELS[kernel])
     ref = attention_ref(Q, K, V, scale, causal)
     assert np.all(np.isfinite(O))
     if causal and Lq > Lk:
@@ -51,20 +55,21 @@ def test_attention_matches_oracle(case):
     assert oracle.rel_fro(O, ref) <= TOL
 
 
-def test_attention_exact_special_cases():
+@pytest.mark.parametrize("kernel", list(KERNELS))
+def test_attention_exact_special_cases(kernel):
     """One key: every weight is exactly 1, so O is the value row bit for bit.  Lk = 0:
     O = 0.  Lq = 0: nothing is written."""
     V = _bf16((3, 1, 128), 4)
-    O = _run(_bf16((3, 77, 128), 5), _bf16((3, 1, 128), 6), V, False, 0.3)
+    O = _run(_bf16((3, 77, 128), 5), _bf16((3, 1, 128), 6), V, False, 0.3, KERNELS[kernel])
     want = oracle.bf16_bits_to_f64(V).astype(np.float32)
     assert np.array_equal(O, np.broadcast_to(want, O.shape))
     Q = _bf16((2, 10, 64), 7)
     O = torch.full((2, 10, 64), float("nan"), device="cuda")
     nj.nnjit_attention(_dev(Q), _dev(np.zeros((2, 1, 64), np.uint16)), _dev(np.zeros((2, 1, 64), np.uint16)),
-                       O, scale=1.0)   # Lk = 1 with zero values
+                       O, scale=1.0, kernel=KERNELS[kernel])   # Lk = 1 with zero values
     torch.cuda.synchronize()
     assert np.array_equal(O.cpu().numpy(), np.zeros((2, 10, 64), np.float32))
-    desc = nj.nnjit_attention_desc(2, 10, 0, 64, 0, 1.0)
+    desc = nj.nnjit_attention_desc(2, 10, 0, 64, 0, 1.0, KERNELS[kernel])
     O.fill_(float("nan"))
     lib = nj.load_library()
     assert lib.nnjit_attention(desc, _dev(Q).data_ptr(), None, None, O.data_ptr(), None) == 0
@@ -78,21 +83,23 @@ def test_attention_refusals():
     p = x.data_ptr()
     for d, st in (((1, 4, 4, 96, 0, 1.0), nj.NNJIT_ERR_UNSUPPORTED), ((0, 4, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
                   ((1, 4, 4, 64, 2, 1.0), nj.NNJIT_ERR_INVALID_ARG), ((1, -1, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
-                  ((1, 4, 4, 64, 0, float("inf")), nj.NNJIT_ERR_INVALID_ARG)):
+                  ((1, 4, 4, 64, 0, float("inf")), nj.NNJIT_ERR_INVALID_ARG),
+                  ((1, 4, 4, 64, 0, 1.0, 3), nj.NNJIT_ERR_INVALID_ARG)):
         assert lib.nnjit_attention(nj.nnjit_attention_desc(*d), p, p, p, p, None) == st
     assert lib.nnjit_attention(nj.nnjit_attention_desc(1, 4, 4, 64, 0, 1.0), p + 4, p, p, p, None) == \
         nj.NNJIT_ERR_UNSUPPORTED
 
 
+@pytest.mark.parametrize("kernel", list(KERNELS))
 @pytest.mark.parametrize("shape", [(128, 256, 256, 64, False), (128, 1024, 1024, 128, True)],
                          ids=["t5_large_heads", "llama2_prefill_heads"])
-def test_attention_full_size_sampled_heads(shape):
+def test_attention_full_size_sampled_heads(shape, kernel):
     """The attention of the T5-large layer (8 x 16 heads, 256 tokens, d = 64) and of the
     Llama-2 prefill (4 x 32 heads, 1024 tokens, d = 128, causal), run in full; five heads
     compared with the oracle."""
     B, Lq, Lk, d, causal = shape
     Q, K, V = _bf16((B, Lq, d), 8), _bf16((B, Lk, d), 9), _bf16((B, Lk, d), 10)
-    O = _run(Q, K, V, causal, 1.0 / np.sqrt(d))
+    O = _run(Q, K, V, causal, 1.0 / np.sqrt(d), KERNELS[kernel])
     heads = [0, 1, B // 2, B - 2, B - 1]
     ref = attention_ref(Q[heads], K[heads], V[heads], 1.0 / np.sqrt(d), causal)
     assert oracle.rel_fro(O[heads], ref) <= TOL
