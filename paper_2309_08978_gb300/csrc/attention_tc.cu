@@ -22,6 +22,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstdint>
 
@@ -55,7 +56,7 @@ struct Cfg {
 struct Params {
     CUtensorMap tq, tk, tv;
     float* O;
-    int Lq, Lk, causal, qblocks;
+    int Lq, Lk, causal, qblocks, batch;
     float scale_log2;
 };
 
@@ -89,6 +90,21 @@ __device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
                  : "memory");
 }
 
+// 32 lanes x 64 consecutive 32-bit TMEM columns in one load, and its wait.
+__device__ __forceinline__ void tmem_ld64(uint32_t taddr, uint32_t (&r)[64]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x64.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63}, [%64];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31]), "=r"(r[32]), "=r"(r[33]), "=r"(r[34]), "=r"(r[35]), "=r"(r[36]), "=r"(r[37]), "=r"(r[38]), "=r"(r[39]), "=r"(r[40]), "=r"(r[41]), "=r"(r[42]), "=r"(r[43]), "=r"(r[44]), "=r"(r[45]), "=r"(r[46]), "=r"(r[47]), "=r"(r[48]), "=r"(r[49]), "=r"(r[50]), "=r"(r[51]), "=r"(r[52]), "=r"(r[53]), "=r"(r[54]), "=r"(r[55]), "=r"(r[56]), "=r"(r[57]), "=r"(r[58]), "=r"(r[59]), "=r"(r[60]), "=r"(r[61]), "=r"(r[62]), "=r"(r[63])
+        : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait64(uint32_t (&r)[64]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]), "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15]), "+r"(r[16]), "+r"(r[17]), "+r"(r[18]), "+r"(r[19]), "+r"(r[20]), "+r"(r[21]), "+r"(r[22]), "+r"(r[23]), "+r"(r[24]), "+r"(r[25]), "+r"(r[26]), "+r"(r[27]), "+r"(r[28]), "+r"(r[29]), "+r"(r[30]), "+r"(r[31]), "+r"(r[32]), "+r"(r[33]), "+r"(r[34]), "+r"(r[35]), "+r"(r[36]), "+r"(r[37]), "+r"(r[38]), "+r"(r[39]), "+r"(r[40]), "+r"(r[41]), "+r"(r[42]), "+r"(r[43]), "+r"(r[44]), "+r"(r[45]), "+r"(r[46]), "+r"(r[47]), "+r"(r[48]), "+r"(r[49]), "+r"(r[50]), "+r"(r[51]), "+r"(r[52]), "+r"(r[53]), "+r"(r[54]), "+r"(r[55]), "+r"(r[56]), "+r"(r[57]), "+r"(r[58]), "+r"(r[59]), "+r"(r[60]), "+r"(r[61]), "+r"(r[62]), "+r"(r[63])
+                 :
+                 : "memory");
+}
+
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
                  : "memory");
@@ -100,7 +116,7 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
     constexpr int S = C::kStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
-    __shared__ __align__(8) uint64_t bars[16];
+    __shared__ __align__(8) uint64_t bars[17];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
     // [half][row]: partial row maxima, then sums.  One buffer is enough: a pair barrier
@@ -114,7 +130,7 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
     auto sK = [&](int s) { return sKV + (uint32_t)s * C::kStageBytes; };
     auto sV = [&](int s) { return sKV + (uint32_t)s * C::kStageBytes + C::kKBytes; };
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
-    const uint32_t q_full = bar(0), drain_bar = bar(15);
+    const uint32_t q_full = bar(0), q_empty = bar(16), drain_bar = bar(15);
     auto kv_full = [&](int s) { return bar(1 + s); };
     auto kv_empty = [&](int s) { return bar(4 + s); };
     auto s_full = [&](int i) { return bar(7 + i); };
@@ -123,15 +139,21 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
     auto o_full = [&](int i) { return bar(13 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int b = (int)(blockIdx.x / p.qblocks);
-    const int q0 = (int)(blockIdx.x % p.qblocks) * kQ;
     const int shift = p.Lk - p.Lq;
-    int kv_end = p.Lk;
-    if (p.causal) kv_end = min(p.Lk, max(0, min(q0 + kQ, p.Lq) - 1 + shift + 1));
-    const int nblocks = (kv_end + kKV - 1) / kKV;
+    const int items = p.qblocks * p.batch;
+    // Work item -> (problem, first query, key blocks).  Items run heaviest first: with the
+    // causal mask the last query blocks see the most keys.
+    auto decode = [&](int it, int& bb, int& qq0) {
+        bb = it % p.batch;
+        qq0 = (p.qblocks - 1 - it / p.batch) * kQ;
+        int kv_end = p.Lk;
+        if (p.causal) kv_end = min(p.Lk, max(0, min(qq0 + kQ, p.Lq) - 1 + shift + 1));
+        return (kv_end + kKV - 1) / kKV;
+    };
 
     if (threadIdx.x == 0) {
         ptx::mbar_init(q_full, 1);
+        ptx::mbar_init(q_empty, 1);
         for (int s = 0; s < S; ++s) {
             ptx::mbar_init(kv_full(s), 1);
             ptx::mbar_init(kv_empty(s), 1);
@@ -159,50 +181,60 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
 
     if (warp == 0) {
         // ------------------------------------------------------------ TMA producer
-        if (lane == 0 && nblocks > 0) {
+        if (lane == 0) {
             ptx::prefetch_tmap(&p.tq);
             ptx::prefetch_tmap(&p.tk);
             ptx::prefetch_tmap(&p.tv);
-            ptx::mbar_arrive_expect_tx(q_full, C::kQBytes);
-            for (int kb = 0; kb < kDB; ++kb) ptx::tma_load_3d(sQ + kb * 16384u, &p.tq, kb * 64, q0, b, q_full);
-            uint32_t armed = 0, armed_parity = 0;
-            int stage = 0;
-            uint32_t phase = 0;
-            for (int j = 0; j < nblocks; ++j) {
-                if (!ptx::mbar_wait(kv_empty(stage), phase ^ 1u, abort_flag, err, kErrProd)) break;
-                ptx::mbar_arrive_expect_tx(kv_full(stage), C::kStageBytes);
-                for (int kb = 0; kb < kDB; ++kb)
-                    ptx::tma_load_3d(sK(stage) + kb * 16384u, &p.tk, kb * 64, j * kKV, b, kv_full(stage));
-                for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
-                    for (int a = 0; a < kDB; ++a)    // 64 columns of d per swizzle atom
-                        ptx::tma_load_3d(sV(stage) + kb * (D * 128u) + a * 8192u, &p.tv, a * 64, j * kKV + kb * 64,
-                                         b, kv_full(stage));
-                armed |= 1u << stage;
-                armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
-                if (++stage == S) {
-                    stage = 0;
-                    phase ^= 1u;
+            uint32_t armed = 0, armed_parity = 0, q_armed = 0;
+            int g = 0, nq = 0;  // key blocks and Q tiles loaded so far
+            bool ok = true;
+            for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+                int bb, qq0;
+                const int nblocks = decode(it, bb, qq0);
+                if (nblocks == 0) continue;
+                // the Q buffer is free once the previous item's score MMAs have completed
+                if (nq > 0 && !ptx::mbar_wait(q_empty, (nq - 1) & 1, abort_flag, err, kErrProd)) break;
+                ptx::mbar_arrive_expect_tx(q_full, C::kQBytes);
+                for (int kb = 0; kb < kDB; ++kb) ptx::tma_load_3d(sQ + kb * 16384u, &p.tq, kb * 64, qq0, bb, q_full);
+                q_armed = 1;
+                ++nq;
+                for (int j = 0; j < nblocks; ++j, ++g) {
+                    const int stage = g % S;
+                    const uint32_t phase = (uint32_t)(g / S) & 1u;
+                    if (!ptx::mbar_wait(kv_empty(stage), phase ^ 1u, abort_flag, err, kErrProd)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::mbar_arrive_expect_tx(kv_full(stage), C::kStageBytes);
+                    for (int kb = 0; kb < kDB; ++kb)
+                        ptx::tma_load_3d(sK(stage) + kb * 16384u, &p.tk, kb * 64, j * kKV, bb, kv_full(stage));
+                    for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
+                        for (int a = 0; a < kDB; ++a)    // 64 columns of d per swizzle atom
+                            ptx::tma_load_3d(sV(stage) + kb * (D * 128u) + a * 8192u, &p.tv, a * 64,
+                                             j * kKV + kb * 64, bb, kv_full(stage));
+                    armed |= 1u << stage;
+                    armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
                 }
             }
+            // drain: every copy issued here has landed before the CTA may exit
             volatile int no_abort = 0;
-            ptx::mbar_wait(q_full, 0, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
-            for (int s = 0; s < S; ++s)
-                if (armed & (1u << s))
-                    ptx::mbar_wait(kv_full(s), (armed_parity >> s) & 1u, &no_abort, err, kErrDrain,
+            if (q_armed) ptx::mbar_wait(q_full, (uint32_t)(nq - 1) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int st = 0; st < S; ++st)
+                if (armed & (1u << st))
+                    ptx::mbar_wait(kv_full(st), (armed_parity >> st) & 1u, &no_abort, err, kErrDrain,
                                    ptx::kWaitLimitNs / 4);
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0 && nblocks > 0) {
+        if (lane == 0) {
             constexpr uint32_t kIdescS = ptx::instr_desc(1u, false, kQ, kKV);
             constexpr uint32_t kIdescO = ptx::instr_desc(1u, true, kQ, D);
-            bool ok = ptx::mbar_wait(q_full, 0, abort_flag, err, kErrMmaQ);
-            ptx::tc_fence_after();
-            auto issue_s = [&](int j) -> bool {
-                const int sb = j & 1, st = j % S;
-                if (j >= 2 && !ptx::mbar_wait(s_empty(sb), ((j - 2) >> 1) & 1, abort_flag, err, kErrMmaS))
+            // S_g = Q K_g^T into score buffer g % 2
+            auto issue_s = [&](int g) -> bool {
+                const int sb = g & 1, st = g % S;
+                if (g >= 2 && !ptx::mbar_wait(s_empty(sb), ((g - 2) >> 1) & 1, abort_flag, err, kErrMmaS))
                     return false;
-                if (!ptx::mbar_wait(kv_full(st), (uint32_t)((j / S) & 1), abort_flag, err, kErrMmaKv)) return false;
+                if (!ptx::mbar_wait(kv_full(st), (uint32_t)((g / S) & 1), abort_flag, err, kErrMmaKv)) return false;
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
 #pragma unroll
@@ -216,23 +248,44 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                 ptx::tc_commit(s_full(sb));
                 return true;
             };
-            if (ok) ok = issue_s(0);
-            for (int j = 0; ok && j < nblocks; ++j) {
-                if (j + 1 < nblocks && !issue_s(j + 1)) break;
-                if (!ptx::mbar_wait(p_full(j & 1), (j >> 1) & 1, abort_flag, err, kErrMmaP)) break;
+            int g = 0, nq = 0;
+            bool ok = true;
+            for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+                int bb, qq0;
+                const int nblocks = decode(it, bb, qq0);
+                if (nblocks == 0) continue;
+                if (!ptx::mbar_wait(q_full, nq & 1, abort_flag, err, kErrMmaQ)) break;
+                ++nq;
                 ptx::tc_fence_after();
-                const int st = j % S;
-                const uint32_t o_tmem = tmem + 2u * kKV + (uint32_t)(j & 1) * D;
+                if (!issue_s(g)) break;
+                for (int j = 0; j < nblocks; ++j, ++g) {
+                    if (j + 1 < nblocks) {
+                        if (!issue_s(g + 1)) {
+                            ok = false;
+                            break;
+                        }
+                    } else {
+                        ptx::tc_commit(q_empty);  // every score MMA of the item is issued
+                    }
+                    if (!ptx::mbar_wait(p_full(g & 1), (g >> 1) & 1, abort_flag, err, kErrMmaP)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    const int st = g % S;
+                    const uint32_t o_tmem = tmem + 2u * kKV + (uint32_t)(g & 1) * D;
 #pragma unroll
-                for (int kb = 0; kb < 2; ++kb) {
-                    const uint64_t ad = ptx::smem_desc(sP + (uint32_t)(j & 1) * C::kPBytes + kb * 16384u, 16, 1024);
-                    const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
+                    for (int kb = 0; kb < 2; ++kb) {
+                        const uint64_t ad =
+                            ptx::smem_desc(sP + (uint32_t)(g & 1) * C::kPBytes + kb * 16384u, 16, 1024);
+                        const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (kb | kk) ? 1u : 0u);
+                        for (int kk = 0; kk < 4; ++kk)
+                            ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (kb | kk) ? 1u : 0u);
+                    }
+                    ptx::tc_commit(o_full(g & 1));
+                    ptx::tc_commit(kv_empty(st));
                 }
-                ptx::tc_commit(o_full(j & 1));
-                ptx::tc_commit(kv_empty(st));
             }
             // every MMA issued here has completed before TMEM is freed
             ptx::tc_commit(drain_bar);
@@ -244,15 +297,8 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
         const int q = warp & 3;
         const int half = (warp - 2) >> 2;
         const int row = q * 32 + lane;
-        const int qrow = q0 + row;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
-        constexpr int kOH = D / 2;                             // output columns of this half
-        float o[kOH];
-#pragma unroll
-        for (int c = 0; c < kOH; ++c) o[c] = 0.0f;
-        float m = -INFINITY, l = 0.0f, alpha_prev = 0.0f;
-        bool ok = true;
+        constexpr int kOH = D / 2;  // output columns of this half
         // barrier of the two warps of lane quarter q; the vote keeps them leaving together
         auto pair_any = [&](bool v) -> bool {
             uint32_t r;
@@ -266,102 +312,122 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                 : "memory");
             return r != 0;
         };
-        // the output of block jb (one behind the softmax) into the running sum
-        auto accumulate = [&](int jb) -> bool {
-            const bool ready = ptx::mbar_wait(o_full(jb & 1), (jb >> 1) & 1, abort_flag, err, kErrSoftO);
-            if (pair_any(!ready)) return false;
-            ptx::tc_fence_after();
-            const uint32_t ob = tmem + lane_base + 2u * kKV + (uint32_t)(jb & 1) * D + (uint32_t)(half * kOH);
+        int g = 0;
+        bool ok = true;
+        for (int it = blockIdx.x; it < items; it += gridDim.x) {
+            int bb, qq0;
+            const int nblocks = decode(it, bb, qq0);
+            const int qrow = qq0 + row;
+            const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
+            float o[kOH];
 #pragma unroll
-            for (int c = 0; c < kOH / 16; ++c) {
-                uint32_t r[16];
-                tmem_ld16(ob + c * 16, r);
-                tmem_wait16(r);
+            for (int c = 0; c < kOH; ++c) o[c] = 0.0f;
+            float m = -INFINITY, l = 0.0f, alpha_prev = 0.0f;
+            // the output of global block gb (one behind the softmax) into the running sum
+            auto accumulate = [&](int gb) -> bool {
+                const bool ready = ptx::mbar_wait(o_full(gb & 1), (gb >> 1) & 1, abort_flag, err, kErrSoftO);
+                if (pair_any(!ready)) return false;
+                ptx::tc_fence_after();
+                const uint32_t ob = tmem + lane_base + 2u * kKV + (uint32_t)(gb & 1) * D + (uint32_t)(half * kOH);
+                if constexpr (kOH == 64) {
+                    uint32_t r[64];
+                    tmem_ld64(ob, r);
+                    tmem_wait64(r);
 #pragma unroll
-                for (int i = 0; i < 16; ++i) o[c * 16 + i] = fmaf(o[c * 16 + i], alpha_prev, __uint_as_float(r[i]));
+                    for (int i = 0; i < 64; ++i) o[i] = fmaf(o[i], alpha_prev, __uint_as_float(r[i]));
+                } else {
+#pragma unroll
+                    for (int c = 0; c < kOH / 16; ++c) {
+                        uint32_t r[16];
+                        tmem_ld16(ob + c * 16, r);
+                        tmem_wait16(r);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) o[c * 16 + i] = fmaf(o[c * 16 + i], alpha_prev, __uint_as_float(r[i]));
+                    }
+                }
+                ptx::tc_fence_before();
+                return true;
+            };
+            for (int j = 0; ok && j < nblocks; ++j, ++g) {
+                const int sb = g & 1;
+                const bool ready = ptx::mbar_wait(s_full(sb), (g >> 1) & 1, abort_flag, err, kErrSoftS);
+                if (pair_any(!ready)) {
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+                const uint32_t sa = tmem + lane_base + (uint32_t)sb * kKV + (uint32_t)(half * 64);
+                // this half of the row's scores, in one TMEM load kept for both passes
+                uint32_t sr[64];
+                tmem_ld64(sa, sr);
+                tmem_wait64(sr);
+                ptx::tc_fence_before();
+                ptx::mbar_arrive(s_empty(sb));  // the score buffer may take S_{g+2} now
+                // columns 0..lim of this half are visible
+                const int lim = min(last, p.Lk - 1) - j * kKV - half * 64;
+                // pass 1: this half's maximum (scaled, base 2), then the row's
+                float mx = -INFINITY;
+#pragma unroll
+                for (int i = 0; i < 64; ++i)
+                    if (i <= lim) mx = fmaxf(mx, __fmul_rn(__uint_as_float(sr[i]), p.scale_log2));
+                red[half][row] = mx;
+                asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+                mx = fmaxf(mx, red[half ^ 1][row]);
+                const float mn = fmaxf(m, mx);
+                const float basev = mn == -INFINITY ? 0.0f : mn;  // no visible key yet: every p is 0
+                const float alpha = ex2(m - basev);
+                m = mn;
+                l *= alpha;
+                // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: this half is
+                // the row's 128-byte segment of K-block `half`; 16-byte chunk u at u ^ (row % 8))
+                const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)half * 16384u + (uint32_t)row * 128u;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {  // 16 keys per chunk: two 16-byte chunks of P
+                    uint32_t pk[8];
+#pragma unroll
+                    for (int i = 0; i < 16; i += 2) {
+                        const int col = c * 16 + i;
+                        // the product rounded as in the first pass (no contraction into an FMA),
+                        // so the row's maximum gives exactly 2^0 = 1
+                        const float p0 =
+                            col <= lim ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(sr[col]), p.scale_log2), basev)) : 0.0f;
+                        const float p1 = col + 1 <= lim
+                                             ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(sr[col + 1]), p.scale_log2), basev))
+                                             : 0.0f;
+                        l += p0 + p1;
+                        pk[i >> 1] = pack_bf16(p0, p1);
+                    }
+#pragma unroll
+                    for (int u = 0; u < 2; ++u) {
+                        const uint32_t ch = (uint32_t)(c * 2 + u);
+                        st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
+                                     pk[4 * u + 3]);
+                    }
+                }
+                ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
+                ptx::mbar_arrive(p_full(sb));
+                if (j >= 1 && !accumulate(g - 1)) {
+                    ok = false;
+                    break;
+                }
+                alpha_prev = alpha;
             }
-            ptx::tc_fence_before();
-            return true;
-        };
-        for (int j = 0; j < nblocks; ++j) {
-            const int sb = j & 1;
-            const bool ready = ptx::mbar_wait(s_full(sb), (j >> 1) & 1, abort_flag, err, kErrSoftS);
-            if (pair_any(!ready)) {
-                ok = false;
-                break;
-            }
-            ptx::tc_fence_after();
-            const uint32_t sa = tmem + lane_base + (uint32_t)sb * kKV + (uint32_t)(half * 64);
-            // columns 0..lim of this half are visible
-            const int lim = min(last, p.Lk - 1) - j * kKV - half * 64;
-            // pass 1: this half's maximum (scaled, base 2), then the row's
-            float mx = -INFINITY;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t r[16];
-                tmem_ld16(sa + c * 16, r);
-                tmem_wait16(r);
-#pragma unroll
-                for (int i = 0; i < 16; ++i)
-                    if (c * 16 + i <= lim) mx = fmaxf(mx, __fmul_rn(__uint_as_float(r[i]), p.scale_log2));
-            }
-            red[half][row] = mx;
+            if (ok && nblocks > 0) ok = accumulate(g - 1);
+            // the row sum is the two halves' sums (both relative to the same maximum)
+            red[half][row] = l;
             asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
-            mx = fmaxf(mx, red[half ^ 1][row]);
-            const float mn = fmaxf(m, mx);
-            const float basev = mn == -INFINITY ? 0.0f : mn;  // no visible key yet: every p is 0
-            const float alpha = ex2(m - basev);
-            m = mn;
-            l *= alpha;
-            // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: this half is
-            // the row's 128-byte segment of K-block `half`; 16-byte chunk u at u ^ (row % 8))
-            const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)half * 16384u + (uint32_t)row * 128u;
+            l += red[half ^ 1][row];
+            if (qrow < p.Lq) {
+                const float inv = (ok && l > 0.0f) ? 1.0f / l : 0.0f;
+                float* dst = p.O + ((size_t)bb * p.Lq + qrow) * D + half * kOH;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {  // 16 keys per chunk: two 16-byte chunks of P
-                uint32_t r[16];
-                tmem_ld16(sa + c * 16, r);
-                tmem_wait16(r);
-                uint32_t pk[8];
-#pragma unroll
-                for (int i = 0; i < 16; i += 2) {
-                    const int col = c * 16 + i;
-                    // the product rounded as in the first pass (no contraction into an FMA), so
-                    // the row's maximum gives exactly 2^0 = 1
-                    const float p0 =
-                        col <= lim ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(r[i]), p.scale_log2), basev)) : 0.0f;
-                    const float p1 =
-                        col + 1 <= lim ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(r[i + 1]), p.scale_log2), basev)) : 0.0f;
-                    l += p0 + p1;
-                    pk[i >> 1] = pack_bf16(p0, p1);
-                }
-#pragma unroll
-                for (int u = 0; u < 2; ++u) {
-                    const uint32_t ch = (uint32_t)(c * 2 + u);
-                    st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
-                                 pk[4 * u + 3]);
-                }
+                for (int c = 0; c < kOH; c += 4)
+                    *reinterpret_cast<float4*>(dst + c) =
+                        make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
             }
-            ptx::tc_fence_before();
-            ptx::mbar_arrive(s_empty(sb));
-            ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
-            ptx::mbar_arrive(p_full(sb));
-            if (j >= 1 && !accumulate(j - 1)) {
-                ok = false;
-                break;
-            }
-            alpha_prev = alpha;
-        }
-        if (ok && nblocks > 0) ok = accumulate(nblocks - 1);
-        // the row sum is the two halves' sums (both relative to the same maximum)
-        red[half][row] = l;
-        asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
-        l += red[half ^ 1][row];
-        if (qrow < p.Lq) {
-            const float inv = (ok && l > 0.0f) ? 1.0f / l : 0.0f;
-            float* dst = p.O + ((size_t)b * p.Lq + qrow) * D + half * kOH;
-#pragma unroll
-            for (int c = 0; c < kOH; c += 4)
-                *reinterpret_cast<float4*>(dst + c) = make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
+            // the next item's first maximum is written only after both halves read this sum
+            asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+            if (!ok) break;
         }
     }
     ptx::tc_fence_before();
@@ -405,6 +471,7 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     p.Lk = (int)d.Lk;
     p.causal = d.causal;
     p.qblocks = qblocks;
+    p.batch = (int)d.batch;
     p.scale_log2 = d.scale * 1.4426950408889634f;
     static bool attr_set[2] = {false, false};
     const int i = d.d == 64 ? 0 : 1;
@@ -415,7 +482,16 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
         if (e != cudaSuccess) return e;
         attr_set[i] = true;
     }
-    return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3((unsigned)ctas),
+    // persistent: one CTA per SM (the CTA holds all of the SM's tensor memory)
+    static int sms = 0;
+    if (sms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (sms <= 0) sms = 1;
+    }
+    const unsigned grid = (unsigned)std::min<long long>(ctas, sms);
+    return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3(grid),
                       dim3(kThreads), (size_t)smem, stream, p);
 }
 
