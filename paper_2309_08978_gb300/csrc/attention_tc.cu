@@ -365,11 +365,25 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                 ptx::mbar_arrive(s_empty(sb));  // the score buffer may take S_{g+2} now
                 // columns 0..lim of this half are visible
                 const int lim = min(last, p.Lk - 1) - j * kKV - half * 64;
-                // pass 1: this half's maximum (scaled, base 2), then the row's
-                float mx = -INFINITY;
+                // pass 1: scale to base 2 in place (-inf where masked), this half's maximum
+                // (four independent partial maxima), then the row's
+                float mxv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                if (lim >= 63) {  // every column of this half is visible
 #pragma unroll
-                for (int i = 0; i < 64; ++i)
-                    if (i <= lim) mx = fmaxf(mx, __fmul_rn(__uint_as_float(sr[i]), p.scale_log2));
+                    for (int i = 0; i < 64; ++i) {
+                        const float x = __fmul_rn(__uint_as_float(sr[i]), p.scale_log2);
+                        sr[i] = __float_as_uint(x);
+                        mxv[i & 3] = fmaxf(mxv[i & 3], x);
+                    }
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 64; ++i) {
+                        const float x = i <= lim ? __fmul_rn(__uint_as_float(sr[i]), p.scale_log2) : -INFINITY;
+                        sr[i] = __float_as_uint(x);
+                        mxv[i & 3] = fmaxf(mxv[i & 3], x);
+                    }
+                }
+                float mx = fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3]));
                 red[half][row] = mx;
                 asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
                 mx = fmaxf(mx, red[half ^ 1][row]);
@@ -381,20 +395,17 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                 // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: this half is
                 // the row's 128-byte segment of K-block `half`; 16-byte chunk u at u ^ (row % 8))
                 const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)half * 16384u + (uint32_t)row * 128u;
+                float lv[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // partial sums (shorter dependency chains)
 #pragma unroll
                 for (int c = 0; c < 4; ++c) {  // 16 keys per chunk: two 16-byte chunks of P
                     uint32_t pk[8];
 #pragma unroll
                     for (int i = 0; i < 16; i += 2) {
                         const int col = c * 16 + i;
-                        // the product rounded as in the first pass (no contraction into an FMA),
-                        // so the row's maximum gives exactly 2^0 = 1
-                        const float p0 =
-                            col <= lim ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(sr[col]), p.scale_log2), basev)) : 0.0f;
-                        const float p1 = col + 1 <= lim
-                                             ? ex2(__fsub_rn(__fmul_rn(__uint_as_float(sr[col + 1]), p.scale_log2), basev))
-                                             : 0.0f;
-                        l += p0 + p1;
+                        // the maximum itself gives exactly 2^0 = 1; masked columns 2^-inf = 0
+                        const float p0 = ex2(__fsub_rn(__uint_as_float(sr[col]), basev));
+                        const float p1 = ex2(__fsub_rn(__uint_as_float(sr[col + 1]), basev));
+                        lv[(i >> 1) & 3] += p0 + p1;
                         pk[i >> 1] = pack_bf16(p0, p1);
                     }
 #pragma unroll
@@ -404,6 +415,7 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                                      pk[4 * u + 3]);
                     }
                 }
+                l += (lv[0] + lv[1]) + (lv[2] + lv[3]);
                 ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
                 ptx::mbar_arrive(p_full(sb));
                 if (j >= 1 && !accumulate(g - 1)) {
