@@ -7,10 +7,11 @@
 //   warp 1     allocates TMEM and issues, from one thread, S_j = Q K_j^T (M = 128,
 //              N = 128, K = d) into one of two TMEM score buffers, and O_j = P_j V_j
 //              (M = 128, N = d, K = 128) into one of two TMEM output buffers;
-//   warps 2-9  softmax: warps w and w + 4 share TMEM lane quarter w % 4 (32 query rows)
-//              and split each row in two halves of 64 keys and d / 2 output columns.
-//              Row maximum over S_j (first pass over TMEM; the halves' maxima meet through
-//              shared memory behind a barrier of the warp pair), then p = 2^(s - m)
+//   warps 2-   softmax: the kSplit warps w, w + 4, ... share TMEM lane quarter w % 4 (32
+//              query rows) and split each row in kSplit parts of 128 / kSplit keys and
+//              d / kSplit output columns (kSplit = 2).  Row
+//              maximum over S_j (first pass over TMEM; the parts' maxima meet through
+//              shared memory behind a barrier of those warps), then p = 2^(s - m)
 //              written as bf16 into a shared-memory P buffer in the MMA's K-major
 //              swizzled layout (second pass), and, one block behind, the running output
 //              O = O * 2^(m_old - m_new) + O_j accumulated in registers.
@@ -38,7 +39,13 @@ __device__ int g_attn_watchdog;  // first expired wait's code (0: none)
 
 constexpr int kQ = 128;   // queries per CTA
 constexpr int kKV = 128;  // keys per block
-constexpr int kThreads = 320;  // producer, MMA issuer, 8 softmax warps
+// Softmax warps per TMEM lane quarter.  Two: four (measured with d = 64) ran slower, the
+// extra barriers and per-part overhead outweighing the extra warps; with d = 128 the ring
+// and buffers leave no room for a four-part exchange buffer either.
+template <int D>
+__host__ __device__ constexpr int split_of() { return 2; }
+template <int D>
+__host__ __device__ constexpr int threads_of() { return 64 + 128 * split_of<D>(); }
 constexpr int kErrProd = 0x301, kErrMmaQ = 0x311, kErrMmaKv = 0x312, kErrMmaS = 0x313, kErrMmaP = 0x314;
 constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrDrain = 0x331;
 
@@ -111,17 +118,19 @@ __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t
 }
 
 template <int D>
-__global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_constant__ Params p) {
+__global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const __grid_constant__ Params p) {
     using C = Cfg<D>;
+    constexpr int kSplit = split_of<D>();
+    constexpr int kCols = kKV / kSplit;  // score columns of a row per softmax thread
     constexpr int S = C::kStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
     __shared__ __align__(8) uint64_t bars[17];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
-    // [half][row]: partial row maxima, then sums.  One buffer is enough: a pair barrier
+    // [part][row]: partial row maxima, then sums.  One buffer is enough: a group barrier
     // (the vote on the next wait) separates each read from the next write.
-    __shared__ float red[2][kQ];
+    __shared__ float red[kSplit][kQ];
     volatile int* abort_flag = &abort_word;
     int* err = &g_attn_watchdog;
 
@@ -160,8 +169,8 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(s_full(i), 1);
-            ptx::mbar_init(s_empty(i), 256);
-            ptx::mbar_init(p_full(i), 256);
+            ptx::mbar_init(s_empty(i), 128 * kSplit);
+            ptx::mbar_init(p_full(i), 128 * kSplit);
             ptx::mbar_init(o_full(i), 1);
         }
         ptx::mbar_init(drain_bar, 1);
@@ -294,23 +303,36 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
         }
     } else {
         // ------------------------------------------------------------ softmax warps
-        const int q = warp & 3;
-        const int half = (warp - 2) >> 2;
+        const int q = warp & 3;                 // TMEM lane quarter
+        const int part = (warp - 2) >> 2;       // which kCols columns of the row
         const int row = q * 32 + lane;
         const uint32_t lane_base = (uint32_t)(q * 32) << 16;
-        constexpr int kOH = D / 2;  // output columns of this half
-        // barrier of the two warps of lane quarter q; the vote keeps them leaving together
-        auto pair_any = [&](bool v) -> bool {
+        constexpr int kOP = D / kSplit;         // output columns of this part
+        // barrier of the kSplit warps of lane quarter q; the vote keeps them leaving together
+        auto group_any = [&](bool v) -> bool {
             uint32_t r;
             asm volatile(
                 "{\n\t.reg .pred a, b;\n\t"
                 "setp.ne.u32 a, %1, 0;\n\t"
-                "barrier.cta.red.or.pred b, %2, 64, a;\n\t"
+                "barrier.cta.red.or.pred b, %2, %3, a;\n\t"
                 "selp.u32 %0, 1, 0, b;\n\t}"
                 : "=r"(r)
-                : "r"((uint32_t)v), "r"(1 + q)
+                : "r"((uint32_t)v), "r"(1 + q), "n"(32 * kSplit)
                 : "memory");
             return r != 0;
+        };
+        auto group_sync = [&]() { asm volatile("bar.sync %0, %1;" ::"r"(1 + q), "n"(32 * kSplit) : "memory"); };
+        // the maximum (op 0) or sum (op 1) of the row's kSplit partial values
+        auto row_reduce = [&](float v, int op) -> float {
+            red[part][row] = v;
+            group_sync();
+            float r = v;
+#pragma unroll
+            for (int k = 1; k < kSplit; ++k) {
+                const float w = red[(part + k) % kSplit][row];
+                r = op == 0 ? fmaxf(r, w) : r + w;
+            }
+            return r;
         };
         int g = 0;
         bool ok = true;
@@ -319,17 +341,17 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
             const int nblocks = decode(it, bb, qq0);
             const int qrow = qq0 + row;
             const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
-            float o[kOH];
+            float o[kOP];
 #pragma unroll
-            for (int c = 0; c < kOH; ++c) o[c] = 0.0f;
+            for (int c = 0; c < kOP; ++c) o[c] = 0.0f;
             float m = -INFINITY, l = 0.0f, alpha_prev = 0.0f;
             // the output of global block gb (one behind the softmax) into the running sum
             auto accumulate = [&](int gb) -> bool {
                 const bool ready = ptx::mbar_wait(o_full(gb & 1), (gb >> 1) & 1, abort_flag, err, kErrSoftO);
-                if (pair_any(!ready)) return false;
+                if (group_any(!ready)) return false;
                 ptx::tc_fence_after();
-                const uint32_t ob = tmem + lane_base + 2u * kKV + (uint32_t)(gb & 1) * D + (uint32_t)(half * kOH);
-                if constexpr (kOH == 64) {
+                const uint32_t ob = tmem + lane_base + 2u * kKV + (uint32_t)(gb & 1) * D + (uint32_t)(part * kOP);
+                if constexpr (kOP == 64) {
                     uint32_t r[64];
                     tmem_ld64(ob, r);
                     tmem_wait64(r);
@@ -337,7 +359,7 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                     for (int i = 0; i < 64; ++i) o[i] = fmaf(o[i], alpha_prev, __uint_as_float(r[i]));
                 } else {
 #pragma unroll
-                    for (int c = 0; c < kOH / 16; ++c) {
+                    for (int c = 0; c < kOP / 16; ++c) {
                         uint32_t r[16];
                         tmem_ld16(ob + c * 16, r);
                         tmem_wait16(r);
@@ -351,69 +373,75 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
             for (int j = 0; ok && j < nblocks; ++j, ++g) {
                 const int sb = g & 1;
                 const bool ready = ptx::mbar_wait(s_full(sb), (g >> 1) & 1, abort_flag, err, kErrSoftS);
-                if (pair_any(!ready)) {
+                if (group_any(!ready)) {
                     ok = false;
                     break;
                 }
                 ptx::tc_fence_after();
-                const uint32_t sa = tmem + lane_base + (uint32_t)sb * kKV + (uint32_t)(half * 64);
-                // this half of the row's scores, in one TMEM load kept for both passes
-                uint32_t sr[64];
-                tmem_ld64(sa, sr);
-                tmem_wait64(sr);
+                const uint32_t sa = tmem + lane_base + (uint32_t)sb * kKV + (uint32_t)(part * kCols);
+                // this part of the row's scores, in one TMEM load kept for both passes
+                uint32_t sr[kCols];
+                if constexpr (kCols == 64) {
+                    tmem_ld64(sa, sr);
+                    tmem_wait64(sr);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < kCols / 16; ++c) {
+                        uint32_t r[16];
+                        tmem_ld16(sa + c * 16, r);
+                        tmem_wait16(r);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) sr[c * 16 + i] = r[i];
+                    }
+                }
                 ptx::tc_fence_before();
                 ptx::mbar_arrive(s_empty(sb));  // the score buffer may take S_{g+2} now
-                // columns 0..lim of this half are visible
-                const int lim = min(last, p.Lk - 1) - j * kKV - half * 64;
-                // pass 1: scale to base 2 in place (-inf where masked), this half's maximum
+                // columns 0..lim of this part are visible
+                const int lim = min(last, p.Lk - 1) - j * kKV - part * kCols;
+                // pass 1: scale to base 2 in place (-inf where masked), this part's maximum
                 // (four independent partial maxima), then the row's
                 float mxv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                if (lim >= 63) {  // every column of this half is visible
+                if (lim >= kCols - 1) {  // every column of this part is visible
 #pragma unroll
-                    for (int i = 0; i < 64; ++i) {
+                    for (int i = 0; i < kCols; ++i) {
                         const float x = __fmul_rn(__uint_as_float(sr[i]), p.scale_log2);
                         sr[i] = __float_as_uint(x);
                         mxv[i & 3] = fmaxf(mxv[i & 3], x);
                     }
                 } else {
 #pragma unroll
-                    for (int i = 0; i < 64; ++i) {
+                    for (int i = 0; i < kCols; ++i) {
                         const float x = i <= lim ? __fmul_rn(__uint_as_float(sr[i]), p.scale_log2) : -INFINITY;
                         sr[i] = __float_as_uint(x);
                         mxv[i & 3] = fmaxf(mxv[i & 3], x);
                     }
                 }
-                float mx = fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3]));
-                red[half][row] = mx;
-                asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
-                mx = fmaxf(mx, red[half ^ 1][row]);
+                const float mx = row_reduce(fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3])), 0);
                 const float mn = fmaxf(m, mx);
                 const float basev = mn == -INFINITY ? 0.0f : mn;  // no visible key yet: every p is 0
                 const float alpha = ex2(m - basev);
                 m = mn;
                 l *= alpha;
-                // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: this half is
-                // the row's 128-byte segment of K-block `half`; 16-byte chunk u at u ^ (row % 8))
-                const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)half * 16384u + (uint32_t)row * 128u;
+                // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: keys
+                // part * kCols .. of the row lie in K-block kb = part * kCols / 64; 16-byte
+                // chunk u of the row's 128 bytes of a K-block sits at u ^ (row % 8))
+                const int kb = (part * kCols) >> 6;
+                const int u0 = ((part * kCols) & 63) >> 3;
+                const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)kb * 16384u + (uint32_t)row * 128u;
                 float lv[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // partial sums (shorter dependency chains)
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {  // 16 keys per chunk: two 16-byte chunks of P
-                    uint32_t pk[8];
+                for (int c = 0; c < kCols / 8; ++c) {  // 8 keys = one 16-byte chunk of P
+                    uint32_t pk[4];
 #pragma unroll
-                    for (int i = 0; i < 16; i += 2) {
-                        const int col = c * 16 + i;
+                    for (int i = 0; i < 8; i += 2) {
                         // the maximum itself gives exactly 2^0 = 1; masked columns 2^-inf = 0
-                        const float p0 = ex2(__fsub_rn(__uint_as_float(sr[col]), basev));
-                        const float p1 = ex2(__fsub_rn(__uint_as_float(sr[col + 1]), basev));
+                        const float p0 = ex2(__fsub_rn(__uint_as_float(sr[c * 8 + i]), basev));
+                        const float p1 = ex2(__fsub_rn(__uint_as_float(sr[c * 8 + i + 1]), basev));
                         lv[(i >> 1) & 3] += p0 + p1;
                         pk[i >> 1] = pack_bf16(p0, p1);
                     }
-#pragma unroll
-                    for (int u = 0; u < 2; ++u) {
-                        const uint32_t ch = (uint32_t)(c * 2 + u);
-                        st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[4 * u], pk[4 * u + 1], pk[4 * u + 2],
-                                     pk[4 * u + 3]);
-                    }
+                    const uint32_t ch = (uint32_t)(u0 + c);
+                    st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[0], pk[1], pk[2], pk[3]);
                 }
                 l += (lv[0] + lv[1]) + (lv[2] + lv[3]);
                 ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
@@ -425,20 +453,18 @@ __global__ void __launch_bounds__(kThreads, 1) attention_tc_kernel(const __grid_
                 alpha_prev = alpha;
             }
             if (ok && nblocks > 0) ok = accumulate(g - 1);
-            // the row sum is the two halves' sums (both relative to the same maximum)
-            red[half][row] = l;
-            asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
-            l += red[half ^ 1][row];
+            // the row sum is the parts' sums (all relative to the same maximum)
+            l = row_reduce(l, 1);
             if (qrow < p.Lq) {
                 const float inv = (ok && l > 0.0f) ? 1.0f / l : 0.0f;
-                float* dst = p.O + ((size_t)bb * p.Lq + qrow) * D + half * kOH;
+                float* dst = p.O + ((size_t)bb * p.Lq + qrow) * D + part * kOP;
 #pragma unroll
-                for (int c = 0; c < kOH; c += 4)
+                for (int c = 0; c < kOP; c += 4)
                     *reinterpret_cast<float4*>(dst + c) =
                         make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
             }
-            // the next item's first maximum is written only after both halves read this sum
-            asm volatile("bar.sync %0, 64;" ::"r"(1 + q) : "memory");
+            // the next item's first maximum is written only after every part read this sum
+            group_sync();
             if (!ok) break;
         }
     }
@@ -504,7 +530,7 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     }
     const unsigned grid = (unsigned)std::min<long long>(ctas, sms);
     return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3(grid),
-                      dim3(kThreads), (size_t)smem, stream, p);
+                      dim3(i == 0 ? threads_of<64>() : threads_of<128>()), (size_t)smem, stream, p);
 }
 
 }  // namespace nnjit
