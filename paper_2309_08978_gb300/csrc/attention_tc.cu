@@ -125,7 +125,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     constexpr int S = C::kStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
-    __shared__ __align__(8) uint64_t bars[17];
+    __shared__ __align__(8) uint64_t bars[24];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
     // [part][row]: partial row maxima, then sums.  One buffer is enough: a group barrier
@@ -135,17 +135,22 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     int* err = &g_attn_watchdog;
 
     const uint32_t base = (ptx::smem_u32(raw) + 1023u) & ~1023u;
-    const uint32_t sQ = base, sKV = base + C::kQBytes, sP = sKV + S * C::kStageBytes;
-    auto sK = [&](int s) { return sKV + (uint32_t)s * C::kStageBytes; };
-    auto sV = [&](int s) { return sKV + (uint32_t)s * C::kStageBytes + C::kKBytes; };
+    // separate key and value rings of S slots each: a key slot is free once its score
+    // product has completed, well before the value slot of the same block
+    const uint32_t sQ = base, sKR = base + C::kQBytes, sVR = sKR + S * C::kKBytes;
+    const uint32_t sP = sVR + S * C::kVBytes;
+    auto sK = [&](int s) { return sKR + (uint32_t)s * C::kKBytes; };
+    auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
-    const uint32_t q_full = bar(0), q_empty = bar(16), drain_bar = bar(15);
-    auto kv_full = [&](int s) { return bar(1 + s); };
-    auto kv_empty = [&](int s) { return bar(4 + s); };
-    auto s_full = [&](int i) { return bar(7 + i); };
-    auto s_empty = [&](int i) { return bar(9 + i); };
-    auto p_full = [&](int i) { return bar(11 + i); };
-    auto o_full = [&](int i) { return bar(13 + i); };
+    const uint32_t q_full = bar(0), q_empty = bar(1), drain_bar = bar(2);
+    auto k_full = [&](int s) { return bar(3 + s); };
+    auto k_empty = [&](int s) { return bar(6 + s); };
+    auto v_full = [&](int s) { return bar(9 + s); };
+    auto v_empty = [&](int s) { return bar(12 + s); };
+    auto s_full = [&](int i) { return bar(15 + i); };
+    auto s_empty = [&](int i) { return bar(17 + i); };
+    auto p_full = [&](int i) { return bar(19 + i); };
+    auto o_full = [&](int i) { return bar(21 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int shift = p.Lk - p.Lq;
@@ -164,8 +169,10 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
         ptx::mbar_init(q_full, 1);
         ptx::mbar_init(q_empty, 1);
         for (int s = 0; s < S; ++s) {
-            ptx::mbar_init(kv_full(s), 1);
-            ptx::mbar_init(kv_empty(s), 1);
+            ptx::mbar_init(k_full(s), 1);
+            ptx::mbar_init(k_empty(s), 1);
+            ptx::mbar_init(v_full(s), 1);
+            ptx::mbar_init(v_empty(s), 1);
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(s_full(i), 1);
@@ -194,9 +201,26 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             ptx::prefetch_tmap(&p.tq);
             ptx::prefetch_tmap(&p.tk);
             ptx::prefetch_tmap(&p.tv);
-            uint32_t armed = 0, armed_parity = 0, q_armed = 0;
+            uint32_t k_armed = 0, k_par = 0, v_armed = 0, v_par = 0, q_armed = 0;
             int g = 0, nq = 0;  // key blocks and Q tiles loaded so far
             bool ok = true;
+            // the value block of global block gv (problem vb, first key vk0): issued one key
+            // block behind, so that a wait for a value slot never holds back the next keys
+            int gv = -1, vb = 0, vk0 = 0;
+            auto load_v = [&]() -> bool {
+                const int st = gv % S;
+                const uint32_t ph = (uint32_t)(gv / S) & 1u;
+                if (!ptx::mbar_wait(v_empty(st), ph ^ 1u, abort_flag, err, kErrProd)) return false;
+                ptx::mbar_arrive_expect_tx(v_full(st), C::kVBytes);
+                for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
+                    for (int a = 0; a < kDB; ++a)    // 64 columns of d per swizzle atom
+                        ptx::tma_load_3d(sV(st) + kb * (D * 128u) + a * 8192u, &p.tv, a * 64, vk0 + kb * 64, vb,
+                                         v_full(st));
+                v_armed |= 1u << st;
+                v_par = (v_par & ~(1u << st)) | (ph << st);
+                gv = -1;
+                return true;
+            };
             for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
                 int bb, qq0;
                 const int nblocks = decode(it, bb, qq0);
@@ -208,30 +232,37 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 q_armed = 1;
                 ++nq;
                 for (int j = 0; j < nblocks; ++j, ++g) {
-                    const int stage = g % S;
-                    const uint32_t phase = (uint32_t)(g / S) & 1u;
-                    if (!ptx::mbar_wait(kv_empty(stage), phase ^ 1u, abort_flag, err, kErrProd)) {
+                    const int st = g % S;
+                    const uint32_t ph = (uint32_t)(g / S) & 1u;
+                    if (!ptx::mbar_wait(k_empty(st), ph ^ 1u, abort_flag, err, kErrProd)) {
                         ok = false;
                         break;
                     }
-                    ptx::mbar_arrive_expect_tx(kv_full(stage), C::kStageBytes);
+                    ptx::mbar_arrive_expect_tx(k_full(st), C::kKBytes);
                     for (int kb = 0; kb < kDB; ++kb)
-                        ptx::tma_load_3d(sK(stage) + kb * 16384u, &p.tk, kb * 64, j * kKV, bb, kv_full(stage));
-                    for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
-                        for (int a = 0; a < kDB; ++a)    // 64 columns of d per swizzle atom
-                            ptx::tma_load_3d(sV(stage) + kb * (D * 128u) + a * 8192u, &p.tv, a * 64,
-                                             j * kKV + kb * 64, bb, kv_full(stage));
-                    armed |= 1u << stage;
-                    armed_parity = (armed_parity & ~(1u << stage)) | (phase << stage);
+                        ptx::tma_load_3d(sK(st) + kb * 16384u, &p.tk, kb * 64, j * kKV, bb, k_full(st));
+                    k_armed |= 1u << st;
+                    k_par = (k_par & ~(1u << st)) | (ph << st);
+                    if (gv >= 0 && !load_v()) {
+                        ok = false;
+                        break;
+                    }
+                    gv = g;
+                    vb = bb;
+                    vk0 = j * kKV;
                 }
+                // the item's last value block before the next item's Q tile and keys
+                if (ok && gv >= 0 && !load_v()) ok = false;
             }
             // drain: every copy issued here has landed before the CTA may exit
             volatile int no_abort = 0;
             if (q_armed) ptx::mbar_wait(q_full, (uint32_t)(nq - 1) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
-            for (int st = 0; st < S; ++st)
-                if (armed & (1u << st))
-                    ptx::mbar_wait(kv_full(st), (armed_parity >> st) & 1u, &no_abort, err, kErrDrain,
-                                   ptx::kWaitLimitNs / 4);
+            for (int st = 0; st < S; ++st) {
+                if (k_armed & (1u << st))
+                    ptx::mbar_wait(k_full(st), (k_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+                if (v_armed & (1u << st))
+                    ptx::mbar_wait(v_full(st), (v_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -243,7 +274,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 const int sb = g & 1, st = g % S;
                 if (g >= 2 && !ptx::mbar_wait(s_empty(sb), ((g - 2) >> 1) & 1, abort_flag, err, kErrMmaS))
                     return false;
-                if (!ptx::mbar_wait(kv_full(st), (uint32_t)((g / S) & 1), abort_flag, err, kErrMmaKv)) return false;
+                if (!ptx::mbar_wait(k_full(st), (uint32_t)((g / S) & 1), abort_flag, err, kErrMmaKv)) return false;
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
 #pragma unroll
@@ -255,6 +286,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                         ptx::mma_ss<0>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdescS, (kb | kk) ? 1u : 0u);
                 }
                 ptx::tc_commit(s_full(sb));
+                ptx::tc_commit(k_empty(st));  // the key slot is free once S_g has completed
                 return true;
             };
             int g = 0, nq = 0;
@@ -276,12 +308,13 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     } else {
                         ptx::tc_commit(q_empty);  // every score MMA of the item is issued
                     }
-                    if (!ptx::mbar_wait(p_full(g & 1), (g >> 1) & 1, abort_flag, err, kErrMmaP)) {
+                    const int st = g % S;
+                    if (!ptx::mbar_wait(p_full(g & 1), (g >> 1) & 1, abort_flag, err, kErrMmaP) ||
+                        !ptx::mbar_wait(v_full(st), (uint32_t)((g / S) & 1), abort_flag, err, kErrMmaKv)) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
-                    const int st = g % S;
                     const uint32_t o_tmem = tmem + 2u * kKV + (uint32_t)(g & 1) * D;
 #pragma unroll
                     for (int kb = 0; kb < 2; ++kb) {
@@ -293,7 +326,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                             ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (kb | kk) ? 1u : 0u);
                     }
                     ptx::tc_commit(o_full(g & 1));
-                    ptx::tc_commit(kv_empty(st));
+                    ptx::tc_commit(v_empty(st));
                 }
             }
             // every MMA issued here has completed before TMEM is freed
