@@ -53,11 +53,14 @@ template <int D>
 struct Cfg {
     static constexpr int kStages = D == 64 ? 3 : 2;
     static constexpr uint32_t kQBytes = kQ * D * 2;
+    // Q buffers: two with d = 64, so the next item's Q tile loads during this item; one
+    // with d = 128 (the key, value and P buffers take the rest of the shared memory)
+    static constexpr int kQBuf = D == 64 ? 2 : 1;
     static constexpr uint32_t kKBytes = kKV * D * 2;
     static constexpr uint32_t kVBytes = kKV * D * 2;
     static constexpr uint32_t kStageBytes = kKBytes + kVBytes;
     static constexpr uint32_t kPBytes = kQ * kKV * 2;
-    static constexpr uint32_t kSmem = 1024 + kQBytes + kStages * kStageBytes + 2 * kPBytes;
+    static constexpr uint32_t kSmem = 1024 + kQBuf * kQBytes + kStages * kStageBytes + 2 * kPBytes;
 };
 
 struct Params {
@@ -125,7 +128,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     constexpr int S = C::kStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
-    __shared__ __align__(8) uint64_t bars[24];
+    __shared__ __align__(8) uint64_t bars[25];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
     // [part][row]: partial row maxima, then sums.  One buffer is enough: a group barrier
@@ -137,12 +140,16 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     const uint32_t base = (ptx::smem_u32(raw) + 1023u) & ~1023u;
     // separate key and value rings of S slots each: a key slot is free once its score
     // product has completed, well before the value slot of the same block
-    const uint32_t sQ = base, sKR = base + C::kQBytes, sVR = sKR + S * C::kKBytes;
+    constexpr int QB = C::kQBuf;
+    auto sQ = [&](int i) { return base + (uint32_t)i * C::kQBytes; };
+    const uint32_t sKR = base + QB * C::kQBytes, sVR = sKR + S * C::kKBytes;
     const uint32_t sP = sVR + S * C::kVBytes;
     auto sK = [&](int s) { return sKR + (uint32_t)s * C::kKBytes; };
     auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
-    const uint32_t q_full = bar(0), q_empty = bar(1), drain_bar = bar(2);
+    const uint32_t drain_bar = bar(2);
+    auto q_full = [&](int i) { return i == 0 ? bar(0) : bar(23); };
+    auto q_empty = [&](int i) { return i == 0 ? bar(1) : bar(24); };
     auto k_full = [&](int s) { return bar(3 + s); };
     auto k_empty = [&](int s) { return bar(6 + s); };
     auto v_full = [&](int s) { return bar(9 + s); };
@@ -166,8 +173,10 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     };
 
     if (threadIdx.x == 0) {
-        ptx::mbar_init(q_full, 1);
-        ptx::mbar_init(q_empty, 1);
+        for (int i = 0; i < QB; ++i) {
+            ptx::mbar_init(q_full(i), 1);
+            ptx::mbar_init(q_empty(i), 1);
+        }
         for (int s = 0; s < S; ++s) {
             ptx::mbar_init(k_full(s), 1);
             ptx::mbar_init(k_empty(s), 1);
@@ -201,7 +210,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             ptx::prefetch_tmap(&p.tq);
             ptx::prefetch_tmap(&p.tk);
             ptx::prefetch_tmap(&p.tv);
-            uint32_t k_armed = 0, k_par = 0, v_armed = 0, v_par = 0, q_armed = 0;
+            uint32_t k_armed = 0, k_par = 0, v_armed = 0, v_par = 0, q_armed = 0, q_par = 0;
             int g = 0, nq = 0;  // key blocks and Q tiles loaded so far
             bool ok = true;
             // the value block of global block gv (problem vb, first key vk0): issued one key
@@ -225,11 +234,15 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 int bb, qq0;
                 const int nblocks = decode(it, bb, qq0);
                 if (nblocks == 0) continue;
-                // the Q buffer is free once the previous item's score MMAs have completed
-                if (nq > 0 && !ptx::mbar_wait(q_empty, (nq - 1) & 1, abort_flag, err, kErrProd)) break;
-                ptx::mbar_arrive_expect_tx(q_full, C::kQBytes);
-                for (int kb = 0; kb < kDB; ++kb) ptx::tma_load_3d(sQ + kb * 16384u, &p.tq, kb * 64, qq0, bb, q_full);
-                q_armed = 1;
+                // a Q buffer is free once the score MMAs of the item that used it have completed
+                const int qi = nq % QB;
+                const uint32_t qph = (uint32_t)(nq / QB) & 1u;
+                if (nq >= QB && !ptx::mbar_wait(q_empty(qi), qph ^ 1u, abort_flag, err, kErrProd)) break;
+                ptx::mbar_arrive_expect_tx(q_full(qi), C::kQBytes);
+                for (int kb = 0; kb < kDB; ++kb)
+                    ptx::tma_load_3d(sQ(qi) + kb * 16384u, &p.tq, kb * 64, qq0, bb, q_full(qi));
+                q_armed |= 1u << qi;
+                q_par = (q_par & ~(1u << qi)) | (qph << qi);
                 ++nq;
                 for (int j = 0; j < nblocks; ++j, ++g) {
                     const int st = g % S;
@@ -256,7 +269,9 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             }
             // drain: every copy issued here has landed before the CTA may exit
             volatile int no_abort = 0;
-            if (q_armed) ptx::mbar_wait(q_full, (uint32_t)(nq - 1) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int i = 0; i < QB; ++i)
+                if (q_armed & (1u << i))
+                    ptx::mbar_wait(q_full(i), (q_par >> i) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
             for (int st = 0; st < S; ++st) {
                 if (k_armed & (1u << st))
                     ptx::mbar_wait(k_full(st), (k_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
@@ -269,6 +284,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
         if (lane == 0) {
             constexpr uint32_t kIdescS = ptx::instr_desc(1u, false, kQ, kKV);
             constexpr uint32_t kIdescO = ptx::instr_desc(1u, true, kQ, D);
+            uint32_t q_addr = sQ(0);  // the current item's Q tile
             // S_g = Q K_g^T into score buffer g % 2
             auto issue_s = [&](int g) -> bool {
                 const int sb = g & 1, st = g % S;
@@ -279,7 +295,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
 #pragma unroll
                 for (int kb = 0; kb < kDB; ++kb) {
-                    const uint64_t ad = ptx::smem_desc(sQ + kb * 16384u, 16, 1024);
+                    const uint64_t ad = ptx::smem_desc(q_addr + kb * 16384u, 16, 1024);
                     const uint64_t bd = ptx::smem_desc(sK(st) + kb * 16384u, 16, 1024);
 #pragma unroll
                     for (int kk = 0; kk < 4; ++kk)
@@ -295,7 +311,9 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 int bb, qq0;
                 const int nblocks = decode(it, bb, qq0);
                 if (nblocks == 0) continue;
-                if (!ptx::mbar_wait(q_full, nq & 1, abort_flag, err, kErrMmaQ)) break;
+                const int qi = nq % QB;
+                if (!ptx::mbar_wait(q_full(qi), (uint32_t)(nq / QB) & 1u, abort_flag, err, kErrMmaQ)) break;
+                q_addr = sQ(qi);
                 ++nq;
                 ptx::tc_fence_after();
                 if (!issue_s(g)) break;
@@ -306,7 +324,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                             break;
                         }
                     } else {
-                        ptx::tc_commit(q_empty);  // every score MMA of the item is issued
+                        ptx::tc_commit(q_empty(qi));  // every score MMA of the item is issued
                     }
                     const int st = g % S;
                     if (!ptx::mbar_wait(p_full(g & 1), (g >> 1) & 1, abort_flag, err, kErrMmaP) ||
