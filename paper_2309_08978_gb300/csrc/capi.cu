@@ -596,8 +596,23 @@ const char* nnjit_last_error(void) { return t_last_error.c_str(); }
 
 int32_t nnjit_version(void) { return 100; }
 
-nnjit_status nnjit_attention(const nnjit_attention_desc* d, const void* Q, const void* K, const void* V,
-                             float* O, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Kernel choices recorded by nnjit_attention_tune, keyed by shape, mask and device.
+std::mutex g_attn_mu;
+std::map<std::string, int> g_attn_choice;
+
+std::string attention_key(const nnjit_attention_desc& d, int dev) {
+    char buf[160];
+    std::snprintf(buf, sizeof buf, "attn|%lld,%lld,%lld,%lld|c%d|dev%d", (long long)d.batch, (long long)d.Lq,
+                  (long long)d.Lk, (long long)d.d, d.causal, dev);
+    return buf;
+}
+
+nnjit_status attention_validate(const nnjit_attention_desc* d, const void* Q, const void* K, const void* V,
+                                const float* O) {
     if (!d) return fail(NNJIT_ERR_INVALID_ARG, "descriptor is NULL");
     const int64_t lim = (int64_t)1 << 31;
     if (d->batch < 1 || d->Lq < 0 || d->Lk < 0 || d->batch >= lim || d->Lq >= lim || d->Lk >= lim)
@@ -610,9 +625,87 @@ nnjit_status nnjit_attention(const nnjit_attention_desc* d, const void* Q, const
     if (!Q || !O || (d->Lk > 0 && (!K || !V))) return fail(NNJIT_ERR_INVALID_ARG, "NULL pointer");
     auto a16 = [](const void* p) { return !p || (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
     if (!a16(Q) || !a16(K) || !a16(V) || !a16(O)) return fail(NNJIT_ERR_UNSUPPORTED, "pointers must be 16-byte aligned");
-    cudaError_t e = d->kernel == NNJIT_ATTN_MMA ? launch_attention(*d, Q, K, V, O, static_cast<cudaStream_t>(stream))
-                                                : launch_attention_tc(*d, Q, K, V, O, static_cast<cudaStream_t>(stream));
+    return NNJIT_OK;
+}
+
+cudaError_t attention_launch(const nnjit_attention_desc& d, int kernel, const void* Q, const void* K,
+                             const void* V, float* O, cudaStream_t s) {
+    return kernel == NNJIT_ATTN_MMA ? launch_attention(d, Q, K, V, O, s) : launch_attention_tc(d, Q, K, V, O, s);
+}
+
+}  // namespace
+
+extern "C" {
+
+nnjit_status nnjit_attention(const nnjit_attention_desc* d, const void* Q, const void* K, const void* V,
+                             float* O, void* stream) {
+    nnjit_status st = attention_validate(d, Q, K, V, O);
+    if (st != NNJIT_OK || d->Lq == 0) return st;
+    int kernel = d->kernel;
+    if (kernel == NNJIT_ATTN_AUTO) {
+        kernel = NNJIT_ATTN_TCGEN05;
+        int dev = 0;
+        cudaGetDevice(&dev);
+        std::lock_guard<std::mutex> lk(g_attn_mu);
+        auto it = g_attn_choice.find(attention_key(*d, dev));
+        if (it != g_attn_choice.end()) kernel = it->second;
+    }
+    cudaError_t e = attention_launch(*d, kernel, Q, K, V, O, static_cast<cudaStream_t>(stream));
     if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_attention_tune(const nnjit_attention_desc* d, const void* Q, const void* K, const void* V,
+                                  float* O, int32_t reps, double* times_us, int32_t* chosen) {
+    nnjit_status st = attention_validate(d, Q, K, V, O);
+    if (st != NNJIT_OK) return st;
+    if (reps < 1 || reps > 100) return fail(NNJIT_ERR_INVALID_ARG, "reps must be 1..100");
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    const int kernels[2] = {NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA};
+    double med[2] = {0.0, 0.0};
+    if (d->Lq > 0) {
+        cudaStream_t s = nullptr;
+        if ((e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking)) != cudaSuccess) return cuda_fail(e, "stream");
+        cudaEvent_t e0 = nullptr, e1 = nullptr;
+        cudaEventCreate(&e0);
+        cudaEventCreate(&e1);
+        for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
+            e = attention_launch(*d, kernels[k], Q, K, V, O, s);  // warm-up
+            std::vector<double> trials;
+            for (int t = 0; t < 3 && e == cudaSuccess; ++t) {
+                cudaEventRecord(e0, s);
+                for (int r = 0; r < reps && e == cudaSuccess; ++r) e = attention_launch(*d, kernels[k], Q, K, V, O, s);
+                cudaEventRecord(e1, s);
+                if (e == cudaSuccess) e = cudaEventSynchronize(e1);
+                float ms = 0.f;
+                cudaEventElapsedTime(&ms, e0, e1);
+                trials.push_back(1000.0 * ms / reps);
+            }
+            if (e == cudaSuccess) {
+                std::sort(trials.begin(), trials.end());
+                med[k] = trials[1];
+            }
+        }
+        cudaEventDestroy(e0);
+        cudaEventDestroy(e1);
+        cudaStreamDestroy(s);
+        if (e != cudaSuccess) return cuda_fail(e, "attention tuning");
+        int word = 0;
+        if ((e = attention_watchdog_take(&word)) != cudaSuccess) return cuda_fail(e, "attention watchdog read");
+        if (word != 0) return fail(NNJIT_ERR_TIMEOUT, "attention wait expired while tuning");
+    }
+    const int best = med[1] < med[0] ? NNJIT_ATTN_MMA : NNJIT_ATTN_TCGEN05;
+    {
+        std::lock_guard<std::mutex> lk(g_attn_mu);
+        g_attn_choice[attention_key(*d, dev)] = best;
+    }
+    if (times_us) {
+        times_us[0] = med[0];
+        times_us[1] = med[1];
+    }
+    if (chosen) *chosen = best;
     return NNJIT_OK;
 }
 

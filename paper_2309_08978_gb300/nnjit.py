@@ -144,6 +144,7 @@ def load_library(path: str = LIB_PATH):
             "nnjit_settings_set": [P(nnjit_settings)],
             "nnjit_attention": [P(nnjit_attention_desc), vp, vp, vp, vp, vp],
             "nnjit_attention_check": [],
+            "nnjit_attention_tune": [P(nnjit_attention_desc), vp, vp, vp, vp, i32, P(ctypes.c_double), P(i32)],
             "nnjit_settings_get": [P(nnjit_settings)],
             "nnjit_settings_study": [P(nnjit_matmul_desc), i32, P(nnjit_settings), ctypes.c_char_p,
                                      ctypes.c_size_t, P(ctypes.c_size_t)],
@@ -439,3 +440,16 @@ def nnjit_attention(Q, K, V, O, causal=False, scale=None, stream=None, kernel=NN
 
 def nnjit_attention_check():
     _check(load_library().nnjit_attention_check(), "nnjit_attention_check")
+
+
+def nnjit_attention_tune(Q, K, V, O, causal=False, scale=None, reps=20):
+    """Time both attention kernels on these buffers (O is overwritten) and record the faster
+    for later kernel=AUTO calls; returns (times_us (tensor-memory, warp-MMA), chosen)."""
+    B, Lq, d = Q.shape
+    desc = nnjit_attention_desc(B, Lq, K.shape[1], d, 1 if causal else 0,
+                                float(scale) if scale is not None else 1.0 / float(d) ** 0.5, 0)
+    times = (ctypes.c_double * 2)()
+    chosen = ctypes.c_int32(0)
+    _check(load_library().nnjit_attention_tune(ctypes.byref(desc), _ptr(Q), _ptr(K), _ptr(V), _ptr(O), reps,
+                                               times, ctypes.byref(chosen)), "nnjit_attention_tune")
+    return (times[0], times[1]), chosen.value

@@ -103,3 +103,19 @@ def test_attention_full_size_sampled_heads(shape, kernel):
     heads = [0, 1, B // 2, B - 2, B - 1]
     ref = attention_ref(Q[heads], K[heads], V[heads], 1.0 / np.sqrt(d), causal)
     assert oracle.rel_fro(O[heads], ref) <= TOL
+
+
+def test_attention_tune_records_the_faster_kernel():
+    """nnjit_attention_tune times both kernels on the caller's buffers and records the faster
+    one for the shape; AUTO calls then use it and stay within the oracle's tolerance."""
+    B, Lq, Lk, d = 4, 200, 260, 64
+    Q, K, V = _bf16((B, Lq, d), 11), _bf16((B, Lk, d), 12), _bf16((B, Lk, d), 13)
+    dQ, dK, dV = _dev(Q), _dev(K), _dev(V)
+    O = torch.empty((B, Lq, d), dtype=torch.float32, device="cuda")
+    (t_tc, t_mma), chosen = nj.nnjit_attention_tune(dQ, dK, dV, O, causal=True, reps=5)
+    assert t_tc > 0 and t_mma > 0
+    assert chosen == (nj.NNJIT_ATTN_MMA if t_mma < t_tc else nj.NNJIT_ATTN_TCGEN05)
+    O.fill_(float("nan"))
+    nj.nnjit_attention(dQ, dK, dV, O, causal=True)          # AUTO: the recorded kernel
+    nj.nnjit_attention_check()
+    assert oracle.rel_fro(O.cpu().numpy(), attention_ref(Q, K, V, 1.0 / np.sqrt(d), True)) <= TOL
