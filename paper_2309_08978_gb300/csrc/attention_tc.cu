@@ -115,6 +115,18 @@ __device__ __forceinline__ void tmem_wait64(uint32_t (&r)[64]) {
                  : "memory");
 }
 
+// 32 lanes x 64 (or 32) consecutive 32-bit TMEM columns stored from registers, and the
+// wait for this thread's outstanding stores.
+__device__ __forceinline__ void tmem_st64(uint32_t taddr, const uint32_t (&r)[64]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32, %33, %34, %35, %36, %37, %38, %39, %40, %41, %42, %43, %44, %45, %46, %47, %48, %49, %50, %51, %52, %53, %54, %55, %56, %57, %58, %59, %60, %61, %62, %63, %64};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31]), "r"(r[32]), "r"(r[33]), "r"(r[34]), "r"(r[35]), "r"(r[36]), "r"(r[37]), "r"(r[38]), "r"(r[39]), "r"(r[40]), "r"(r[41]), "r"(r[42]), "r"(r[43]), "r"(r[44]), "r"(r[45]), "r"(r[46]), "r"(r[47]), "r"(r[48]), "r"(r[49]), "r"(r[50]), "r"(r[51]), "r"(r[52]), "r"(r[53]), "r"(r[54]), "r"(r[55]), "r"(r[56]), "r"(r[57]), "r"(r[58]), "r"(r[59]), "r"(r[60]), "r"(r[61]), "r"(r[62]), "r"(r[63])
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+                 : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
 __device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
     asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
                  : "memory");
@@ -333,7 +345,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                         break;
                     }
                     ptx::tc_fence_after();
-                    const uint32_t o_tmem = tmem + 2u * kKV + (uint32_t)(g & 1) * D;
+                    const uint32_t o_tmem = tmem + 2u * kKV;  // O accumulates over the item's blocks
 #pragma unroll
                     for (int kb = 0; kb < 2; ++kb) {
                         const uint64_t ad =
@@ -341,7 +353,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                         const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk)
-                            ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (kb | kk) ? 1u : 0u);
+                            ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (j | kb | kk) ? 1u : 0u);
                     }
                     ptx::tc_commit(o_full(g & 1));
                     ptx::tc_commit(v_empty(st));
@@ -392,35 +404,12 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             const int nblocks = decode(it, bb, qq0);
             const int qrow = qq0 + row;
             const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
-            float o[kOP];
-#pragma unroll
-            for (int c = 0; c < kOP; ++c) o[c] = 0.0f;
-            float m = -INFINITY, l = 0.0f, alpha_prev = 0.0f;
-            // the output of global block gb (one behind the softmax) into the running sum
-            auto accumulate = [&](int gb) -> bool {
-                const bool ready = ptx::mbar_wait(o_full(gb & 1), (gb >> 1) & 1, abort_flag, err, kErrSoftO);
-                if (group_any(!ready)) return false;
-                ptx::tc_fence_after();
-                const uint32_t ob = tmem + lane_base + 2u * kKV + (uint32_t)(gb & 1) * D + (uint32_t)(part * kOP);
-                if constexpr (kOP == 64) {
-                    uint32_t r[64];
-                    tmem_ld64(ob, r);
-                    tmem_wait64(r);
-#pragma unroll
-                    for (int i = 0; i < 64; ++i) o[i] = fmaf(o[i], alpha_prev, __uint_as_float(r[i]));
-                } else {
-#pragma unroll
-                    for (int c = 0; c < kOP / 16; ++c) {
-                        uint32_t r[16];
-                        tmem_ld16(ob + c * 16, r);
-                        tmem_wait16(r);
-#pragma unroll
-                        for (int i = 0; i < 16; ++i) o[c * 16 + i] = fmaf(o[c * 16 + i], alpha_prev, __uint_as_float(r[i]));
-                    }
-                }
-                ptx::tc_fence_before();
-                return true;
-            };
+            // The output accumulates in TMEM (the P V products add onto it); the row keeps
+            // its base m (p = 2^(x - m)) until a block's maximum exceeds it by more than
+            // 2^8, and only then is the TMEM row rescaled by 2^(m_old - m_new) (values up
+            // to 2^8 are harmless to bf16 P and float32 sums).
+            float m = -INFINITY, l = 0.0f;
+            const uint32_t orow = tmem + lane_base + 2u * kKV + (uint32_t)(part * kOP);
             for (int j = 0; ok && j < nblocks; ++j, ++g) {
                 const int sb = g & 1;
                 const bool ready = ptx::mbar_wait(s_full(sb), (g >> 1) & 1, abort_flag, err, kErrSoftS);
@@ -468,11 +457,15 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     }
                 }
                 const float mx = row_reduce(fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3])), 0);
-                const float mn = fmaxf(m, mx);
-                const float basev = mn == -INFINITY ? 0.0f : mn;  // no visible key yet: every p is 0
-                const float alpha = ex2(m - basev);
-                m = mn;
-                l *= alpha;
+                // a new base only when the maximum outgrows the current one by 2^8
+                const bool rebase = mx > m + 8.0f;  // (always for the first visible key: m = -inf)
+                float alpha = 1.0f;
+                if (rebase) {
+                    alpha = ex2(m - mx);  // 0 while m = -inf
+                    m = mx;
+                    l *= alpha;
+                }
+                const float basev = m == -INFINITY ? 0.0f : m;  // no visible key yet: every p is 0
                 // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: keys
                 // part * kCols .. of the row lie in K-block kb = part * kCols / 64; 16-byte
                 // chunk u of the row's 128 bytes of a K-block sits at u ^ (row % 8))
@@ -485,7 +478,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     uint32_t pk[4];
 #pragma unroll
                     for (int i = 0; i < 8; i += 2) {
-                        // the maximum itself gives exactly 2^0 = 1; masked columns 2^-inf = 0
+                        // the maximum gives exactly 2^0 = 1 when it is the base; masked 2^-inf = 0
                         const float p0 = ex2(__fsub_rn(__uint_as_float(sr[c * 8 + i]), basev));
                         const float p1 = ex2(__fsub_rn(__uint_as_float(sr[c * 8 + i + 1]), basev));
                         lv[(i >> 1) & 3] += p0 + p1;
@@ -495,25 +488,70 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[0], pk[1], pk[2], pk[3]);
                 }
                 l += (lv[0] + lv[1]) + (lv[2] + lv[3]);
+                // O (the P V products of this item's earlier blocks) is complete in TMEM; P_g went to
+                // the other P buffer meanwhile
+                if (j >= 1) {
+                    const bool done = ptx::mbar_wait(o_full((g - 1) & 1), ((g - 1) >> 1) & 1, abort_flag, err, kErrSoftO);
+                    if (group_any(!done)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    // rescale the warp's rows of O in TMEM when any of them took a new base
+                    if (__any_sync(0xffffffffu, rebase)) {
+                        if constexpr (kOP == 64) {
+                            uint32_t r[64];
+                            tmem_ld64(orow, r);
+                            tmem_wait64(r);
+#pragma unroll
+                            for (int i = 0; i < 64; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                            tmem_st64(orow, r);
+                        } else {
+                            uint32_t r[32];
+                            ptx::tmem_ld32(orow, r);
+                            ptx::tmem_wait_ld(r);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                            tmem_st32(orow, r);
+                        }
+                        tmem_wait_st();
+                    }
+                }
+                ptx::tc_fence_before();         // the rescaled O is stored before P V_g runs
                 ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
                 ptx::mbar_arrive(p_full(sb));
-                if (j >= 1 && !accumulate(g - 1)) {
-                    ok = false;
-                    break;
-                }
-                alpha_prev = alpha;
             }
-            if (ok && nblocks > 0) ok = accumulate(g - 1);
-            // the row sum is the parts' sums (all relative to the same maximum)
+            // the row sum is the parts' sums (all relative to the same base)
             l = row_reduce(l, 1);
-            if (qrow < p.Lq) {
-                const float inv = (ok && l > 0.0f) ? 1.0f / l : 0.0f;
-                float* dst = p.O + ((size_t)bb * p.Lq + qrow) * D + part * kOP;
-#pragma unroll
-                for (int c = 0; c < kOP; c += 4)
-                    *reinterpret_cast<float4*>(dst + c) =
-                        make_float4(o[c] * inv, o[c + 1] * inv, o[c + 2] * inv, o[c + 3] * inv);
+            // the item's output: O from TMEM once its last P V product has completed
+            bool have_o = false;
+            if (ok && nblocks > 0) {
+                const bool done = ptx::mbar_wait(o_full((g - 1) & 1), ((g - 1) >> 1) & 1, abort_flag, err, kErrSoftO);
+                ok = !group_any(!done);
+                have_o = ok;
+                if (ok) ptx::tc_fence_after();
             }
+            const float inv = (have_o && l > 0.0f) ? 1.0f / l : 0.0f;
+            float* dst = p.O + ((size_t)bb * p.Lq + qrow) * D + part * kOP;
+#pragma unroll
+            for (int c0 = 0; c0 < kOP; c0 += 32) {
+                uint32_t r[32];
+                if (have_o) {
+                    ptx::tmem_ld32(orow + c0, r);
+                    ptx::tmem_wait_ld(r);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) r[i] = 0u;
+                }
+                if (qrow < p.Lq) {
+#pragma unroll
+                    for (int c = 0; c < 32; c += 4)
+                        *reinterpret_cast<float4*>(dst + c0 + c) =
+                            make_float4(__uint_as_float(r[c]) * inv, __uint_as_float(r[c + 1]) * inv,
+                                        __uint_as_float(r[c + 2]) * inv, __uint_as_float(r[c + 3]) * inv);
+                }
+            }
+            ptx::tc_fence_before();  // the next item's first P V overwrites O
             // the next item's first maximum is written only after every part read this sum
             group_sync();
             if (!ok) break;
