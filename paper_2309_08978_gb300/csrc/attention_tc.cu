@@ -51,16 +51,14 @@ constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrDrain = 0x331;
 
 template <int D>
 struct Cfg {
-    static constexpr int kStages = D == 64 ? 3 : 2;
+    static constexpr int kStages = D == 64 ? 4 : 2;
     static constexpr uint32_t kQBytes = kQ * D * 2;
-    // Q buffers: two with d = 64, so the next item's Q tile loads during this item; one
-    // with d = 128 (the key, value and P buffers take the rest of the shared memory)
-    static constexpr int kQBuf = D == 64 ? 2 : 1;
+    // two Q buffers, so that the next item's Q tile loads during this item
+    static constexpr int kQBuf = 2;
     static constexpr uint32_t kKBytes = kKV * D * 2;
     static constexpr uint32_t kVBytes = kKV * D * 2;
     static constexpr uint32_t kStageBytes = kKBytes + kVBytes;
-    static constexpr uint32_t kPBytes = kQ * kKV * 2;
-    static constexpr uint32_t kSmem = 1024 + kQBuf * kQBytes + kStages * kStageBytes + 2 * kPBytes;
+    static constexpr uint32_t kSmem = 1024 + kQBuf * kQBytes + kStages * kStageBytes;
 };
 
 struct Params {
@@ -127,11 +125,6 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
 }
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c, uint32_t d) {
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c), "r"(d)
-                 : "memory");
-}
-
 template <int D>
 __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const __grid_constant__ Params p) {
     using C = Cfg<D>;
@@ -140,7 +133,10 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     constexpr int S = C::kStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
-    __shared__ __align__(8) uint64_t bars[25];
+    // q_full, q_empty (2 each), drain, k_full, k_empty, v_full, v_empty (S each), s_full,
+    // s_empty, p_full, o_full (2 each)
+    __shared__ __align__(8) uint64_t bars[5 + 4 * C::kStages + 8];
+    static_assert(C::kQBuf <= 2, "two Q barrier pairs");
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
     // [part][row]: partial row maxima, then sums.  One buffer is enough: a group barrier
@@ -155,21 +151,20 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     constexpr int QB = C::kQBuf;
     auto sQ = [&](int i) { return base + (uint32_t)i * C::kQBytes; };
     const uint32_t sKR = base + QB * C::kQBytes, sVR = sKR + S * C::kKBytes;
-    const uint32_t sP = sVR + S * C::kVBytes;
     auto sK = [&](int s) { return sKR + (uint32_t)s * C::kKBytes; };
     auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
-    const uint32_t drain_bar = bar(2);
-    auto q_full = [&](int i) { return i == 0 ? bar(0) : bar(23); };
-    auto q_empty = [&](int i) { return i == 0 ? bar(1) : bar(24); };
-    auto k_full = [&](int s) { return bar(3 + s); };
-    auto k_empty = [&](int s) { return bar(6 + s); };
-    auto v_full = [&](int s) { return bar(9 + s); };
-    auto v_empty = [&](int s) { return bar(12 + s); };
-    auto s_full = [&](int i) { return bar(15 + i); };
-    auto s_empty = [&](int i) { return bar(17 + i); };
-    auto p_full = [&](int i) { return bar(19 + i); };
-    auto o_full = [&](int i) { return bar(21 + i); };
+    const uint32_t drain_bar = bar(4);
+    auto q_full = [&](int i) { return bar(i); };
+    auto q_empty = [&](int i) { return bar(2 + i); };
+    auto k_full = [&](int s) { return bar(5 + s); };
+    auto k_empty = [&](int s) { return bar(5 + S + s); };
+    auto v_full = [&](int s) { return bar(5 + 2 * S + s); };
+    auto v_empty = [&](int s) { return bar(5 + 3 * S + s); };
+    auto s_full = [&](int i) { return bar(5 + 4 * S + i); };
+    auto s_empty = [&](int i) { return bar(7 + 4 * S + i); };
+    auto p_full = [&](int i) { return bar(9 + 4 * S + i); };
+    auto o_full = [&](int i) { return bar(11 + 4 * S + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int shift = p.Lk - p.Lq;
@@ -346,14 +341,14 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     }
                     ptx::tc_fence_after();
                     const uint32_t o_tmem = tmem + 2u * kKV;  // O accumulates over the item's blocks
+                    const uint32_t p_tmem = o_tmem + D + (uint32_t)(g & 1) * (kKV / 2);  // P_g, bf16 pairs
 #pragma unroll
                     for (int kb = 0; kb < 2; ++kb) {
-                        const uint64_t ad =
-                            ptx::smem_desc(sP + (uint32_t)(g & 1) * C::kPBytes + kb * 16384u, 16, 1024);
                         const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
 #pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)
-                            ptx::mma_ss<0>(o_tmem, ad + 2 * kk, bd + 128 * kk, kIdescO, (j | kb | kk) ? 1u : 0u);
+                        for (int kk = 0; kk < 4; ++kk)  // keys kb * 64 + kk * 16 .. + 15: 8 columns of P
+                            ptx::mma_ts_f16(o_tmem, p_tmem + kb * 32 + kk * 8, bd + 128 * kk, kIdescO,
+                                            (j | kb | kk) ? 1u : 0u);
                     }
                     ptx::tc_commit(o_full(g & 1));
                     ptx::tc_commit(v_empty(st));
@@ -466,26 +461,23 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     l *= alpha;
                 }
                 const float basev = m == -INFINITY ? 0.0f : m;  // no visible key yet: every p is 0
-                // pass 2: p = 2^(s - m) as bf16 into P (K-major, 128-byte swizzle: keys
-                // part * kCols .. of the row lie in K-block kb = part * kCols / 64; 16-byte
-                // chunk u of the row's 128 bytes of a K-block sits at u ^ (row % 8))
-                const int kb = (part * kCols) >> 6;
-                const int u0 = ((part * kCols) & 63) >> 3;
-                const uint32_t seg = sP + (uint32_t)sb * C::kPBytes + (uint32_t)kb * 16384u + (uint32_t)row * 128u;
+                // pass 2: p = 2^(s - m) as bf16 into P in TMEM (the row's lane; keys 2c, 2c + 1
+                // of the block in column c of P buffer g % 2), the A operand of P V
+                const uint32_t pcol = tmem + lane_base + 2u * kKV + D + (uint32_t)sb * (kKV / 2) +
+                                      (uint32_t)(part * kCols / 2);
                 float lv[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // partial sums (shorter dependency chains)
 #pragma unroll
-                for (int c = 0; c < kCols / 8; ++c) {  // 8 keys = one 16-byte chunk of P
-                    uint32_t pk[4];
+                for (int c0 = 0; c0 < kCols; c0 += 64) {  // 64 keys = 32 columns of P per store
+                    uint32_t pk[32];
 #pragma unroll
-                    for (int i = 0; i < 8; i += 2) {
+                    for (int i = 0; i < 64; i += 2) {
                         // the maximum gives exactly 2^0 = 1 when it is the base; masked 2^-inf = 0
-                        const float p0 = ex2(__fsub_rn(__uint_as_float(sr[c * 8 + i]), basev));
-                        const float p1 = ex2(__fsub_rn(__uint_as_float(sr[c * 8 + i + 1]), basev));
+                        const float p0 = ex2(__fsub_rn(__uint_as_float(sr[c0 + i]), basev));
+                        const float p1 = ex2(__fsub_rn(__uint_as_float(sr[c0 + i + 1]), basev));
                         lv[(i >> 1) & 3] += p0 + p1;
                         pk[i >> 1] = pack_bf16(p0, p1);
                     }
-                    const uint32_t ch = (uint32_t)(u0 + c);
-                    st_shared_v4(seg + ((ch ^ (uint32_t)(row & 7)) << 4), pk[0], pk[1], pk[2], pk[3]);
+                    tmem_st32(pcol + (uint32_t)(c0 / 2), pk);
                 }
                 l += (lv[0] + lv[1]) + (lv[2] + lv[3]);
                 // O (the P V products of this item's earlier blocks) is complete in TMEM; P_g went to
@@ -514,11 +506,10 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                             for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
                             tmem_st32(orow, r);
                         }
-                        tmem_wait_st();
                     }
                 }
-                ptx::tc_fence_before();         // the rescaled O is stored before P V_g runs
-                ptx::fence_proxy_async_smem();  // P is read by the tensor cores (async proxy)
+                tmem_wait_st();
+                ptx::tc_fence_before();  // P_g and the rescaled O are stored before P V_g runs
                 ptx::mbar_arrive(p_full(sb));
             }
             // the row sum is the parts' sums (all relative to the same base)

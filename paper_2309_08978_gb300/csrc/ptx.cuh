@@ -232,6 +232,18 @@ __host__ __device__ constexpr uint32_t instr_desc(uint32_t fmt, bool b_mn_major,
            ((n >> 3) << 17) | ((m >> 4) << 24);
 }
 
+// kind::f16 with the A operand (M rows = TMEM lanes, K bf16 values packed two per 32-bit
+// column, the lower k in the low half) read from tensor memory and B from shared memory.
+__device__ __forceinline__ void mma_ts_f16(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                           uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 template <int kKind>  // 0: kind::f16 (bf16 operands), 1: kind::tf32
 __device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                        uint32_t accumulate) {

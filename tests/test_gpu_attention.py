@@ -38,7 +38,9 @@ def _run(Q, K, V, causal, scale, kernel=1):
 
 CASES = [(2, 64, 64, 64, False), (3, 100, 130, 64, False), (2, 128, 128, 128, True),
          (1, 70, 200, 64, True), (1, 200, 70, 128, True), (4, 256, 256, 64, False),
-         (2, 1, 300, 128, True), (2, 333, 333, 128, False), (1, 65, 1, 64, False)]
+         (2, 1, 300, 128, True), (2, 333, 333, 128, False), (1, 65, 1, 64, False),
+         # more query blocks than SMs: persistent CTAs take several items each
+         (160, 130, 200, 64, True), (90, 256, 130, 128, False)]
 
 
 @pytest.mark.parametrize("kernel", list(KERNELS))
