@@ -51,14 +51,15 @@ constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrDrain = 0x331;
 
 template <int D>
 struct Cfg {
-    static constexpr int kStages = D == 64 ? 4 : 2;
+    // key and value ring slots (a third key slot with d = 128 measured no faster)
+    static constexpr int kKStages = D == 64 ? 4 : 2;
+    static constexpr int kVStages = D == 64 ? 4 : 2;
     static constexpr uint32_t kQBytes = kQ * D * 2;
     // two Q buffers, so that the next item's Q tile loads during this item
     static constexpr int kQBuf = 2;
     static constexpr uint32_t kKBytes = kKV * D * 2;
     static constexpr uint32_t kVBytes = kKV * D * 2;
-    static constexpr uint32_t kStageBytes = kKBytes + kVBytes;
-    static constexpr uint32_t kSmem = 1024 + kQBuf * kQBytes + kStages * kStageBytes;
+    static constexpr uint32_t kSmem = 1024 + kQBuf * kQBytes + kKStages * kKBytes + kVStages * kVBytes;
 };
 
 struct Params {
@@ -72,6 +73,33 @@ __device__ __forceinline__ float ex2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
     return y;
+}
+
+// Packed pairs of f32 (the Blackwell f32x2 add and multiply: one instruction for two lanes
+// worth of work, each half rounded as the scalar operation would be), and the three-input
+// maximum.
+__device__ __forceinline__ uint64_t f2(uint32_t lo, uint32_t hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+    return r;
+}
+__device__ __forceinline__ void f2_split(uint64_t v, uint32_t& lo, uint32_t& hi) {
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t f2_mul(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ uint64_t f2_add(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+__device__ __forceinline__ float max3(float a, float b, float c) {
+    float r;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(r) : "f"(a), "f"(b), "f"(c));
+    return r;
 }
 
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
@@ -130,12 +158,12 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     using C = Cfg<D>;
     constexpr int kSplit = split_of<D>();
     constexpr int kCols = kKV / kSplit;  // score columns of a row per softmax thread
-    constexpr int S = C::kStages;
+    constexpr int SK = C::kKStages, SV = C::kVStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
-    // q_full, q_empty (2 each), drain, k_full, k_empty, v_full, v_empty (S each), s_full,
-    // s_empty, p_full, o_full (2 each)
-    __shared__ __align__(8) uint64_t bars[5 + 4 * C::kStages + 8];
+    // q_full, q_empty (2 each), drain, k_full, k_empty (SK each), v_full, v_empty (SV
+    // each), s_full, s_empty, p_full, o_full (2 each)
+    __shared__ __align__(8) uint64_t bars[5 + 2 * C::kKStages + 2 * C::kVStages + 8];
     static_assert(C::kQBuf <= 2, "two Q barrier pairs");
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
@@ -150,7 +178,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     // product has completed, well before the value slot of the same block
     constexpr int QB = C::kQBuf;
     auto sQ = [&](int i) { return base + (uint32_t)i * C::kQBytes; };
-    const uint32_t sKR = base + QB * C::kQBytes, sVR = sKR + S * C::kKBytes;
+    const uint32_t sKR = base + QB * C::kQBytes, sVR = sKR + SK * C::kKBytes;
     auto sK = [&](int s) { return sKR + (uint32_t)s * C::kKBytes; };
     auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
@@ -158,13 +186,14 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     auto q_full = [&](int i) { return bar(i); };
     auto q_empty = [&](int i) { return bar(2 + i); };
     auto k_full = [&](int s) { return bar(5 + s); };
-    auto k_empty = [&](int s) { return bar(5 + S + s); };
-    auto v_full = [&](int s) { return bar(5 + 2 * S + s); };
-    auto v_empty = [&](int s) { return bar(5 + 3 * S + s); };
-    auto s_full = [&](int i) { return bar(5 + 4 * S + i); };
-    auto s_empty = [&](int i) { return bar(7 + 4 * S + i); };
-    auto p_full = [&](int i) { return bar(9 + 4 * S + i); };
-    auto o_full = [&](int i) { return bar(11 + 4 * S + i); };
+    auto k_empty = [&](int s) { return bar(5 + SK + s); };
+    constexpr int kVB = 5 + 2 * SK, kSB = kVB + 2 * SV;
+    auto v_full = [&](int s) { return bar(kVB + s); };
+    auto v_empty = [&](int s) { return bar(kVB + SV + s); };
+    auto s_full = [&](int i) { return bar(kSB + i); };
+    auto s_empty = [&](int i) { return bar(kSB + 2 + i); };
+    auto p_full = [&](int i) { return bar(kSB + 4 + i); };
+    auto o_full = [&](int i) { return bar(kSB + 6 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int shift = p.Lk - p.Lq;
@@ -184,9 +213,11 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             ptx::mbar_init(q_full(i), 1);
             ptx::mbar_init(q_empty(i), 1);
         }
-        for (int s = 0; s < S; ++s) {
+        for (int s = 0; s < SK; ++s) {
             ptx::mbar_init(k_full(s), 1);
             ptx::mbar_init(k_empty(s), 1);
+        }
+        for (int s = 0; s < SV; ++s) {
             ptx::mbar_init(v_full(s), 1);
             ptx::mbar_init(v_empty(s), 1);
         }
@@ -224,8 +255,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             // block behind, so that a wait for a value slot never holds back the next keys
             int gv = -1, vb = 0, vk0 = 0;
             auto load_v = [&]() -> bool {
-                const int st = gv % S;
-                const uint32_t ph = (uint32_t)(gv / S) & 1u;
+                const int st = gv % SV;
+                const uint32_t ph = (uint32_t)(gv / SV) & 1u;
                 if (!ptx::mbar_wait(v_empty(st), ph ^ 1u, abort_flag, err, kErrProd)) return false;
                 ptx::mbar_arrive_expect_tx(v_full(st), C::kVBytes);
                 for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
@@ -252,8 +283,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 q_par = (q_par & ~(1u << qi)) | (qph << qi);
                 ++nq;
                 for (int j = 0; j < nblocks; ++j, ++g) {
-                    const int st = g % S;
-                    const uint32_t ph = (uint32_t)(g / S) & 1u;
+                    const int st = g % SK;
+                    const uint32_t ph = (uint32_t)(g / SK) & 1u;
                     if (!ptx::mbar_wait(k_empty(st), ph ^ 1u, abort_flag, err, kErrProd)) {
                         ok = false;
                         break;
@@ -279,12 +310,12 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             for (int i = 0; i < QB; ++i)
                 if (q_armed & (1u << i))
                     ptx::mbar_wait(q_full(i), (q_par >> i) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
-            for (int st = 0; st < S; ++st) {
+            for (int st = 0; st < SK; ++st)
                 if (k_armed & (1u << st))
                     ptx::mbar_wait(k_full(st), (k_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int st = 0; st < SV; ++st)
                 if (v_armed & (1u << st))
                     ptx::mbar_wait(v_full(st), (v_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
-            }
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
@@ -294,10 +325,10 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             uint32_t q_addr = sQ(0);  // the current item's Q tile
             // S_g = Q K_g^T into score buffer g % 2
             auto issue_s = [&](int g) -> bool {
-                const int sb = g & 1, st = g % S;
+                const int sb = g & 1, st = g % SK;
                 if (g >= 2 && !ptx::mbar_wait(s_empty(sb), ((g - 2) >> 1) & 1, abort_flag, err, kErrMmaS))
                     return false;
-                if (!ptx::mbar_wait(k_full(st), (uint32_t)((g / S) & 1), abort_flag, err, kErrMmaKv)) return false;
+                if (!ptx::mbar_wait(k_full(st), (uint32_t)((g / SK) & 1), abort_flag, err, kErrMmaKv)) return false;
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
 #pragma unroll
@@ -333,9 +364,9 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     } else {
                         ptx::tc_commit(q_empty(qi));  // every score MMA of the item is issued
                     }
-                    const int st = g % S;
+                    const int st = g % SV;
                     if (!ptx::mbar_wait(p_full(g & 1), (g >> 1) & 1, abort_flag, err, kErrMmaP) ||
-                        !ptx::mbar_wait(v_full(st), (uint32_t)((g / S) & 1), abort_flag, err, kErrMmaKv)) {
+                        !ptx::mbar_wait(v_full(st), (uint32_t)((g / SV) & 1), abort_flag, err, kErrMmaKv)) {
                         ok = false;
                         break;
                     }
@@ -436,19 +467,24 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 // pass 1: scale to base 2 in place (-inf where masked), this part's maximum
                 // (four independent partial maxima), then the row's
                 float mxv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                const uint32_t cb = __float_as_uint(p.scale_log2);
+                const uint64_t c2 = f2(cb, cb);
                 if (lim >= kCols - 1) {  // every column of this part is visible
 #pragma unroll
-                    for (int i = 0; i < kCols; ++i) {
-                        const float x = __fmul_rn(__uint_as_float(sr[i]), p.scale_log2);
-                        sr[i] = __float_as_uint(x);
-                        mxv[i & 3] = fmaxf(mxv[i & 3], x);
+                    for (int i = 0; i < kCols; i += 2) {  // two columns per packed multiply
+                        f2_split(f2_mul(f2(sr[i], sr[i + 1]), c2), sr[i], sr[i + 1]);
+                        mxv[(i >> 1) & 3] =
+                            max3(mxv[(i >> 1) & 3], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
                     }
                 } else {
+                    const uint32_t ninf = __float_as_uint(-INFINITY);
 #pragma unroll
-                    for (int i = 0; i < kCols; ++i) {
-                        const float x = i <= lim ? __fmul_rn(__uint_as_float(sr[i]), p.scale_log2) : -INFINITY;
-                        sr[i] = __float_as_uint(x);
-                        mxv[i & 3] = fmaxf(mxv[i & 3], x);
+                    for (int i = 0; i < kCols; i += 2) {
+                        f2_split(f2_mul(f2(sr[i], sr[i + 1]), c2), sr[i], sr[i + 1]);
+                        if (i > lim) sr[i] = ninf;
+                        if (i + 1 > lim) sr[i + 1] = ninf;
+                        mxv[(i >> 1) & 3] =
+                            max3(mxv[(i >> 1) & 3], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
                     }
                 }
                 const float mx = row_reduce(fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3])), 0);
@@ -465,21 +501,30 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 // of the block in column c of P buffer g % 2), the A operand of P V
                 const uint32_t pcol = tmem + lane_base + 2u * kKV + D + (uint32_t)sb * (kKV / 2) +
                                       (uint32_t)(part * kCols / 2);
-                float lv[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // partial sums (shorter dependency chains)
+                // packed partial sums: two pairs of lanes (shorter dependency chains)
+                uint64_t lv2[2] = {0ull, 0ull};
+                const uint32_t nb = __float_as_uint(-basev);  // x + (-m) rounds as x - m
+                const uint64_t nb2 = f2(nb, nb);
 #pragma unroll
                 for (int c0 = 0; c0 < kCols; c0 += 64) {  // 64 keys = 32 columns of P per store
                     uint32_t pk[32];
 #pragma unroll
                     for (int i = 0; i < 64; i += 2) {
                         // the maximum gives exactly 2^0 = 1 when it is the base; masked 2^-inf = 0
-                        const float p0 = ex2(__fsub_rn(__uint_as_float(sr[c0 + i]), basev));
-                        const float p1 = ex2(__fsub_rn(__uint_as_float(sr[c0 + i + 1]), basev));
-                        lv[(i >> 1) & 3] += p0 + p1;
+                        uint32_t d0, d1;
+                        f2_split(f2_add(f2(sr[c0 + i], sr[c0 + i + 1]), nb2), d0, d1);
+                        const float p0 = ex2(__uint_as_float(d0)), p1 = ex2(__uint_as_float(d1));
+                        lv2[(i >> 1) & 1] = f2_add(lv2[(i >> 1) & 1], f2(__float_as_uint(p0), __float_as_uint(p1)));
                         pk[i >> 1] = pack_bf16(p0, p1);
                     }
                     tmem_st32(pcol + (uint32_t)(c0 / 2), pk);
                 }
-                l += (lv[0] + lv[1]) + (lv[2] + lv[3]);
+                {
+                    uint32_t a0, a1, b0, b1;
+                    f2_split(lv2[0], a0, a1);
+                    f2_split(lv2[1], b0, b1);
+                    l += (__uint_as_float(a0) + __uint_as_float(a1)) + (__uint_as_float(b0) + __uint_as_float(b1));
+                }
                 // O (the P V products of this item's earlier blocks) is complete in TMEM; P_g went to
                 // the other P buffer meanwhile
                 if (j >= 1) {
