@@ -46,7 +46,7 @@ template <int D>
 __host__ __device__ constexpr int split_of() { return 2; }
 template <int D>
 __host__ __device__ constexpr int threads_of() { return 64 + 128 * split_of<D>(); }
-constexpr int kErrProd = 0x301, kErrMmaQ = 0x311, kErrMmaKv = 0x312, kErrMmaS = 0x313, kErrMmaP = 0x314;
+constexpr int kErrProd = 0x301, kErrMmaQ = 0x311, kErrMmaKv = 0x312, kErrMmaP = 0x314;
 constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrDrain = 0x331;
 
 template <int D>
@@ -162,8 +162,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
     // q_full, q_empty (2 each), drain, k_full, k_empty (SK each), v_full, v_empty (SV
-    // each), s_full, s_empty, p_full, o_full (2 each)
-    __shared__ __align__(8) uint64_t bars[5 + 2 * C::kKStages + 2 * C::kVStages + 8];
+    // each), s_full, p_full, o_full (2 each)
+    __shared__ __align__(8) uint64_t bars[5 + 2 * C::kKStages + 2 * C::kVStages + 6];
     static_assert(C::kQBuf <= 2, "two Q barrier pairs");
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
@@ -191,9 +191,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     auto v_full = [&](int s) { return bar(kVB + s); };
     auto v_empty = [&](int s) { return bar(kVB + SV + s); };
     auto s_full = [&](int i) { return bar(kSB + i); };
-    auto s_empty = [&](int i) { return bar(kSB + 2 + i); };
-    auto p_full = [&](int i) { return bar(kSB + 4 + i); };
-    auto o_full = [&](int i) { return bar(kSB + 6 + i); };
+    auto p_full = [&](int i) { return bar(kSB + 2 + i); };
+    auto o_full = [&](int i) { return bar(kSB + 4 + i); };
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int shift = p.Lk - p.Lq;
@@ -223,8 +222,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
         }
         for (int i = 0; i < 2; ++i) {
             ptx::mbar_init(s_full(i), 1);
-            ptx::mbar_init(s_empty(i), 128 * kSplit);
-            ptx::mbar_init(p_full(i), 128 * kSplit);
+            ptx::mbar_init(p_full(i), 4 * kSplit);  // one arrival per softmax warp
             ptx::mbar_init(o_full(i), 1);
         }
         ptx::mbar_init(drain_bar, 1);
@@ -326,8 +324,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             // S_g = Q K_g^T into score buffer g % 2
             auto issue_s = [&](int g) -> bool {
                 const int sb = g & 1, st = g % SK;
-                if (g >= 2 && !ptx::mbar_wait(s_empty(sb), ((g - 2) >> 1) & 1, abort_flag, err, kErrMmaS))
-                    return false;
+                // Score buffer g % 2 is free: the softmax read S_{g-2} before releasing P_{g-2},
+                // and P_{g-2} V_{g-2} was issued (after that release) before this product.
                 if (!ptx::mbar_wait(k_full(st), (uint32_t)((g / SK) & 1), abort_flag, err, kErrMmaKv)) return false;
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
@@ -461,7 +459,6 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                     }
                 }
                 ptx::tc_fence_before();
-                ptx::mbar_arrive(s_empty(sb));  // the score buffer may take S_{g+2} now
                 // columns 0..lim of this part are visible
                 const int lim = min(last, p.Lk - 1) - j * kKV - part * kCols;
                 // pass 1: scale to base 2 in place (-inf where masked), this part's maximum
@@ -555,7 +552,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 }
                 tmem_wait_st();
                 ptx::tc_fence_before();  // P_g and the rescaled O are stored before P V_g runs
-                ptx::mbar_arrive(p_full(sb));
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(p_full(sb));  // one arrival per warp
             }
             // the row sum is the parts' sums (all relative to the same base)
             l = row_reduce(l, 1);
