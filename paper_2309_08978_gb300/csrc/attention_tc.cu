@@ -1,25 +1,26 @@
 // Fused attention on the 5th-generation tensor cores (nnjit_attention, kernel 1):
 // O = softmax(scale Q K^T) V per batch x head without writing the scores.
 //
-// One CTA takes 128 queries of one problem; 6 warps:
-//   warp 0     TMA producer: the Q tile once, then key and value blocks of 128 rows
-//              through an S-slot ring (128-byte swizzle; keys K-major, values MN-major);
-//   warp 1     allocates TMEM and issues, from one thread, S_j = Q K_j^T (M = 128,
-//              N = 128, K = d) into one of two TMEM score buffers, and O_j = P_j V_j
-//              (M = 128, N = d, K = 128) into one of two TMEM output buffers;
-//   warps 2-   softmax: the kSplit warps w, w + 4, ... share TMEM lane quarter w % 4 (32
-//              query rows) and split each row in kSplit parts of 128 / kSplit keys and
-//              d / kSplit output columns (kSplit = 2).  Row
-//              maximum over S_j (first pass over TMEM; the parts' maxima meet through
-//              shared memory behind a barrier of those warps), then p = 2^(s - m)
-//              written as bf16 into a shared-memory P buffer in the MMA's K-major
-//              swizzled layout (second pass), and, one block behind, the running output
-//              O = O * 2^(m_old - m_new) + O_j accumulated in registers.
-// The score and output buffers, P and the ring are double-buffered so that the tensor
-// cores work on block j + 1 while the softmax warps work on block j.  Keys past Lk and,
-// with the causal mask, keys past i + (Lk - Lq) score -inf; blocks a CTA cannot see are
-// skipped.  Every wait is bounded: on expiry the watchdog word is set, the CTA's abort
-// flag raised, and every role leaves after draining what it issued.
+// A persistent CTA per SM loops over (problem, 128-query block) items; 10 warps:
+//   warp 0     TMA producer: an item's Q tile (two Q buffers), then its key and value
+//              blocks of 128 rows through separate key and value rings (128-byte
+//              swizzle; keys K-major, values MN-major), values one key block behind;
+//   warp 1     allocates TMEM and issues, from one thread, S_g = Q K_g^T (M = 128,
+//              N = 128, K = d) into TMEM score buffer g % 2, a block ahead, and
+//              O += P_g V_g (M = 128, N = d, K = 128) with P_g read from TMEM as the A
+//              operand, into the item's TMEM output;
+//   warps 2-9  softmax: the two warps w, w + 4 share TMEM lane quarter w % 4 (32 query
+//              rows) and split each row in two parts of 64 keys and d / 2 output
+//              columns.  Row maximum over S_g (first pass; the parts' maxima meet
+//              through shared memory behind a barrier of the two warps), then
+//              p = 2^(s - m) stored as bf16 pairs into TMEM P buffer g % 2 (second
+//              pass).  A row keeps its base m until a block's maximum exceeds it by
+//              more than 2^8; only then is its TMEM output rescaled in place.
+// The score and P buffers are double-buffered so that the tensor cores work on block
+// g + 1 while the softmax warps work on block g.  Keys past Lk and, with the causal mask,
+// keys past i + (Lk - Lq) score -inf; blocks a query block cannot see are skipped.  Every
+// wait is bounded: on expiry the watchdog word is set, the CTA's abort flag raised, and
+// every role leaves after draining what it issued.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -59,11 +60,15 @@ struct Cfg {
     static constexpr int kQBuf = 2;
     static constexpr uint32_t kKBytes = kKV * D * 2;
     static constexpr uint32_t kVBytes = kKV * D * 2;
-    static constexpr uint32_t kSmem = 1024 + kQBuf * kQBytes + kKStages * kKBytes + kVStages * kVBytes;
+    // output staging: one 32 x 32 f32 tile (4 KB, 128-byte swizzle) per softmax warp, stored
+    // to global memory by TMA (whole 128-byte row segments instead of one row per lane)
+    static constexpr uint32_t kOStage = 4096;
+    static constexpr uint32_t kSmem =
+        1024 + kQBuf * kQBytes + kKStages * kKBytes + kVStages * kVBytes + 8 * kOStage;
 };
 
 struct Params {
-    CUtensorMap tq, tk, tv;
+    CUtensorMap tq, tk, tv, to;
     float* O;
     int Lq, Lk, causal, qblocks, batch;
     float scale_log2;
@@ -141,6 +146,11 @@ __device__ __forceinline__ void tmem_wait64(uint32_t (&r)[64]) {
                  : "memory");
 }
 
+__device__ __forceinline__ void st_shared_f4(uint32_t addr, float a, float b, float c, float d) {
+    asm volatile("st.shared.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "f"(a), "f"(b), "f"(c), "f"(d)
+                 : "memory");
+}
+
 // 32 lanes x 64 (or 32) consecutive 32-bit TMEM columns stored from registers, and the
 // wait for this thread's outstanding stores.
 __device__ __forceinline__ void tmem_st64(uint32_t taddr, const uint32_t (&r)[64]) {
@@ -181,6 +191,7 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     const uint32_t sKR = base + QB * C::kQBytes, sVR = sKR + SK * C::kKBytes;
     auto sK = [&](int s) { return sKR + (uint32_t)s * C::kKBytes; };
     auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
+    const uint32_t sO = sVR + SV * C::kVBytes;  // 8 output staging tiles
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
     const uint32_t drain_bar = bar(4);
     auto q_full = [&](int i) { return bar(i); };
@@ -566,7 +577,10 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
                 if (ok) ptx::tc_fence_after();
             }
             const float inv = (have_o && l > 0.0f) ? 1.0f / l : 0.0f;
-            float* dst = p.O + ((size_t)bb * p.Lq + qrow) * D + part * kOP;
+            // 32 x 32 tiles of the warp's rows and this part's columns: staged with the
+            // 128-byte swizzle (16-byte chunk c of row r at c ^ (r % 8)) and stored by TMA,
+            // which leaves rows past Lq unwritten
+            const uint32_t stage = sO + (uint32_t)(warp - 2) * C::kOStage;
 #pragma unroll
             for (int c0 = 0; c0 < kOP; c0 += 32) {
                 uint32_t r[32];
@@ -577,12 +591,18 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
 #pragma unroll
                     for (int i = 0; i < 32; ++i) r[i] = 0u;
                 }
-                if (qrow < p.Lq) {
+                if (lane == 0) ptx::bulk_wait_all_read();  // the tile's previous store has read it
+                __syncwarp();
 #pragma unroll
-                    for (int c = 0; c < 32; c += 4)
-                        *reinterpret_cast<float4*>(dst + c0 + c) =
-                            make_float4(__uint_as_float(r[c]) * inv, __uint_as_float(r[c + 1]) * inv,
-                                        __uint_as_float(r[c + 2]) * inv, __uint_as_float(r[c + 3]) * inv);
+                for (int c = 0; c < 8; ++c)
+                    st_shared_f4(stage + (uint32_t)lane * 128u + ((uint32_t)(c ^ (lane & 7)) << 4),
+                                 __uint_as_float(r[4 * c]) * inv, __uint_as_float(r[4 * c + 1]) * inv,
+                                 __uint_as_float(r[4 * c + 2]) * inv, __uint_as_float(r[4 * c + 3]) * inv);
+                ptx::fence_proxy_async_smem();  // the tile is read by the TMA (async proxy)
+                __syncwarp();
+                if (lane == 0) {
+                    ptx::tma_store_3d(&p.to, stage, part * kOP + c0, qq0 + q * 32, bb);
+                    ptx::bulk_commit();
                 }
             }
             ptx::tc_fence_before();  // the next item's first P V overwrites O
@@ -590,6 +610,8 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
             group_sync();
             if (!ok) break;
         }
+        if (lane == 0) ptx::bulk_wait_all();  // every output store has completed
+        __syncwarp();
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -627,6 +649,15 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     };
     if (!encode(&p.tq, Q, d.Lq, kQ) || !encode(&p.tk, K, d.Lk, kKV) || !encode(&p.tv, V, d.Lk, 64))
         return cudaErrorInvalidValue;
+    {  // O: f32 [batch, Lq, d], stored in 32 x 32 tiles (128-byte rows, 128-byte swizzle)
+        const cuuint64_t dims[3] = {(cuuint64_t)d.d, (cuuint64_t)d.Lq, (cuuint64_t)d.batch};
+        const cuuint64_t strides[2] = {(cuuint64_t)(d.d * 4), (cuuint64_t)(d.Lq * d.d * 4)};
+        const cuuint32_t box[3] = {32, 32, 1};
+        if (enc(&p.to, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, O, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
     p.O = O;
     p.Lq = (int)d.Lq;
     p.Lk = (int)d.Lk;
