@@ -386,9 +386,10 @@ def run_attention(args, name, rank, world, local_rank):
     peak_t = peaks["bf16_tflops_sustained"] if sustained and peaks.get("bf16_tflops_sustained") else peaks["bf16_tflops"]
     ach = flops / dur_s / 1e12
     alg_bytes = set_bytes
+    kernel_key = f"attention {tune['chosen']} d{d} B{B} Lq{Lq} Lk{Lk}" + (" causal" if causal else "")
     roof = {"bound": "tensor", "achieved": round(ach, 2), "peak": round(peak_t, 1), "unit": "TFLOP/s",
-            "frac": round(ach / peak_t, 4), "traffic": None,
-            "kernel": f"attention {tune['chosen']} d{d} B{B} Lq{Lq} Lk{Lk}" + (" causal" if causal else ""),
+            "frac": round(ach / peak_t, 4), "traffic": lookup_traffic(kernel_key),
+            "kernel": kernel_key,
             "peak_source": ("sustained" if sustained else "burst") + f" bf16 ({peaks['source']})",
             "units_per_launch": f"{flops} flop, {alg_bytes} algorithmic bytes"}
 
