@@ -38,7 +38,7 @@ namespace {
 
 __device__ int g_attn_watchdog;  // first expired wait's code (0: none)
 
-constexpr int kQ = 128;   // queries per CTA
+constexpr int kQ = 128;   // queries per work item (a CTA loops over items)
 constexpr int kKV = 128;  // keys per block
 // Softmax warps per TMEM lane quarter.  Two: one (whole rows per thread, no exchange of
 // maxima) measured 60.7 against 55.4 us on the Llama prefill heads, four (d = 64) slower
