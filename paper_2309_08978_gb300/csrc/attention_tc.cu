@@ -25,6 +25,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 
@@ -629,7 +630,8 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     p.qblocks = qblocks;
     p.batch = (int)d.batch;
     p.scale_log2 = d.scale * 1.4426950408889634f;
-    static bool attr_set[2] = {false, false};
+    // set once per head dimension (concurrent first calls both set it, which is harmless)
+    static std::atomic<bool> attr_set[2] = {{false}, {false}};
     const int i = d.d == 64 ? 0 : 1;
     const int smem = i == 0 ? (int)Cfg<64>::kSmem : (int)Cfg<128>::kSmem;
     if (!attr_set[i]) {
@@ -639,12 +641,14 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
         attr_set[i] = true;
     }
     // persistent: one CTA per SM (the CTA holds all of the SM's tensor memory)
-    static int sms = 0;
+    static std::atomic<int> sms_cached{0};
+    int sms = sms_cached.load();
     if (sms == 0) {
         int dev = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
         if (sms <= 0) sms = 1;
+        sms_cached.store(sms);
     }
     const unsigned grid = (unsigned)std::min<long long>(ctas, sms);
     return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3(grid),
