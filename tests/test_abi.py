@@ -136,3 +136,27 @@ def test_settings_roundtrip_and_validation(lib):
     finally:
         nj.nnjit_settings_set(None)
     assert nj.nnjit_settings_get()["raster"] == -1
+
+
+def test_attention_refusals_without_a_gpu(lib):
+    """nnjit_attention checks its descriptor and pointers before any CUDA call: invalid
+    sizes, flags, kernels and NULL pointers give INVALID_ARG, an unsupported head dimension
+    or a pointer off a 16-byte boundary UNSUPPORTED, and Lq = 0 returns OK with nothing to
+    do.  The pointers are never dereferenced on these paths."""
+    import paper_2309_08978_gb300 as nj
+    f = nj.load_library().nnjit_attention
+    p = 1 << 20  # a 16-byte-aligned address, never touched
+    cases = (((1, 4, 4, 96, 0, 1.0), nj.NNJIT_ERR_UNSUPPORTED), ((0, 4, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
+             ((1, 4, 4, 64, 2, 1.0), nj.NNJIT_ERR_INVALID_ARG), ((1, -1, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
+             ((1, 4, -2, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
+             ((1, 4, 4, 64, 0, float("nan")), nj.NNJIT_ERR_INVALID_ARG),
+             ((1, 4, 4, 64, 0, 1.0, 3), nj.NNJIT_ERR_INVALID_ARG), ((1, 4, 4, 64, 0, 1.0, -1), nj.NNJIT_ERR_INVALID_ARG))
+    for d, st in cases:
+        assert f(nj.nnjit_attention_desc(*d), p, p, p, p, None) == st, d
+    desc = nj.nnjit_attention_desc(1, 4, 4, 64, 0, 1.0)
+    assert f(desc, p + 4, p, p, p, None) == nj.NNJIT_ERR_UNSUPPORTED
+    assert f(desc, p, p, p, p + 8, None) == nj.NNJIT_ERR_UNSUPPORTED
+    assert f(desc, None, p, p, p, None) == nj.NNJIT_ERR_INVALID_ARG
+    assert f(desc, p, None, p, p, None) == nj.NNJIT_ERR_INVALID_ARG
+    assert f(None, p, p, p, p, None) == nj.NNJIT_ERR_INVALID_ARG
+    assert f(nj.nnjit_attention_desc(2, 0, 5, 128, 1, 1.0), None, None, None, None, None) == nj.NNJIT_OK
