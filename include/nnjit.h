@@ -182,10 +182,9 @@ typedef struct {
     int32_t reduce;          /* split-K reduction: 0 = partials in the plan's workspace, summed
                                 by a second kernel; 1 = TC only, inside a thread-block cluster
                                 of split_k CTAs through distributed shared memory */
-    int32_t cluster_m;       /* TC only: 2 = a cluster of two CTAs; with bm = 128 they take
-                                vertically adjacent tiles and share each B tile by TMA
-                                multicast, with bm = 256 they compute one 256-row tile with
-                                tcgen05 cta_group::2 MMAs; else 1 */
+    int32_t cluster_m;       /* TC only: 2 = a cluster of two CTAs on two SMs computing one
+                                256-row tile (bm = 256) with tcgen05 cta_group::2 MMAs;
+                                else 1 */
 } nnjit_candidate;
 
 typedef struct nnjit_plan_s* nnjit_plan;
@@ -197,10 +196,9 @@ typedef struct nnjit_plan_s* nnjit_plan;
  * the one value kept.  They act on the tensor-core family only:
  *   raster     tile order: 0 = M fastest, 1 = N fastest;
  *   kgroup     k-blocks per ring slot (candidate bk / one 128-byte k-block): 1 or 2;
- *   reduce     split-K reduction: 0 = second kernel, 1 = inside a cluster (DSMEM);
- *   multicast  128 x 256 tiles as TMA-multicast pairs (cluster_m = 2, bm = 128): 0 or 1.
+ *   reduce     split-K reduction: 0 = second kernel, 1 = inside a cluster (DSMEM).
  * A fixed value removes a candidate only where the same candidate with the fixed value
- * (every other searched field equal: bm, bn, split_k and the other three settings) is
+ * (every other searched field equal: bm, bn, split_k and the other two settings) is
  * in the space, so a setting never empties the space and never removes the only legal
  * choice (for example kgroup = 2 keeps bn = 256 tiles, which exist only with 1).  The
  * axes are applied in the order above.
@@ -210,7 +208,6 @@ typedef struct {
     int32_t raster;
     int32_t kgroup;
     int32_t reduce;
-    int32_t multicast;
 } nnjit_settings;
 
 /* ---------------------------------------------------------------------------------- */
@@ -429,7 +426,8 @@ nnjit_status nnjit_attention_tune(const nnjit_attention_desc* desc, const void* 
  *
  * C[m,n] = sum_k x[m,k] * W[n,k] (+ bias[n]) for 1 <= M <= 8, with x [M][K] and W [N][K]
  * packed bf16, C [M][N] packed float32, bias float32[N] or NULL, all device pointers the
- * caller owns; K % 8 == 0 and x, W 16-byte aligned.  K is split into split_k slices
+ * caller owns; K % 8 == 0, x and W 16-byte aligned, C and bias 4-byte aligned (else
+ * UNSUPPORTED).  K is split into split_k slices
  * (1..64) whose float32 partial sums are kept in one fixed device array inside the
  * library of NNJIT_NOALLOC_SCRATCH_FLOATS floats (4 MiB, held by every GPU that loads
  * the library until the process exits) and then added in slice order.  Requests with

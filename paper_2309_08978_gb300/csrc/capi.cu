@@ -204,7 +204,7 @@ std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L, c
     std::string key = buf;
     if (p.epilogue != NNJIT_EPI_NONE) key += "|ep=" + std::to_string(p.epilogue);
     if (any_fixed(set)) {
-        std::snprintf(buf, sizeof buf, "|set=%d,%d,%d,%d", set.raster, set.kgroup, set.reduce, set.multicast);
+        std::snprintf(buf, sizeof buf, "|set=%d,%d,%d", set.raster, set.kgroup, set.reduce);
         key += buf;
     }
     return key;
@@ -923,7 +923,7 @@ nnjit_status nnjit_settings_get(nnjit_settings* out) {
 nnjit_status nnjit_settings_study(const nnjit_matmul_desc* descs, int32_t count, nnjit_settings* out,
                                   char* report, size_t report_len, size_t* report_needed) {
     if (!descs || count < 1 || !out) return fail(NNJIT_ERR_INVALID_ARG, "need descs, count >= 1 and out");
-    static const char* names[kSettingAxes] = {"raster", "kgroup", "reduce", "multicast"};
+    static const char* names[kSettingAxes] = {"raster", "kgroup", "reduce"};
     const nnjit_settings free_set = free_settings();
     int vote[kSettingAxes];      // value every decisive vote agreed on; -1 none yet; -2 conflict
     for (int a = 0; a < kSettingAxes; ++a) vote[a] = -1;
@@ -952,11 +952,11 @@ nnjit_status nnjit_settings_study(const nnjit_matmul_desc* descs, int32_t count,
         std::snprintf(tmp, sizeof tmp,
                       "%s{\"M\":%lld,\"N\":%lld,\"K\":%lld,\"batch\":%lld,\"dtype\":%d,\"b_layout\":%d,"
                       "\"space_size\":%d,\"best_index\":%d,\"best_us\":%.4f,\"best\":{\"bm\":%d,\"bn\":%d,"
-                      "\"split_k\":%d,\"raster\":%d,\"kgroup\":%d,\"reduce\":%d,\"multicast\":%d},\"settings\":{",
+                      "\"split_k\":%d,\"raster\":%d,\"kgroup\":%d,\"reduce\":%d},\"settings\":{",
                       i ? "," : "", (long long)p.M, (long long)p.N, (long long)p.K, (long long)p.batch, p.dtype,
                       p.b_layout, (int)space.size(), best, us[best], space[best].bm, space[best].bn,
                       space[best].split_k, candidate_setting(p, space[best], 0), candidate_setting(p, space[best], 1),
-                      candidate_setting(p, space[best], 2), candidate_setting(p, space[best], 3));
+                      candidate_setting(p, space[best], 2));
         js += tmp;
         for (int a = 0; a < kSettingAxes; ++a) {
             int twin = -1;
@@ -980,10 +980,10 @@ nnjit_status nnjit_settings_study(const nnjit_matmul_desc* descs, int32_t count,
         js += "}}";
     }
     nnjit_settings res = free_set;
-    int* fields[kSettingAxes] = {&res.raster, &res.kgroup, &res.reduce, &res.multicast};
+    int* fields[kSettingAxes] = {&res.raster, &res.kgroup, &res.reduce};
     for (int a = 0; a < kSettingAxes; ++a) *fields[a] = vote[a] >= 0 ? vote[a] : NNJIT_SETTING_FREE;
-    std::snprintf(tmp, sizeof tmp, "],\"fixed\":{\"raster\":%d,\"kgroup\":%d,\"reduce\":%d,\"multicast\":%d}}",
-                  res.raster, res.kgroup, res.reduce, res.multicast);
+    std::snprintf(tmp, sizeof tmp, "],\"fixed\":{\"raster\":%d,\"kgroup\":%d,\"reduce\":%d}}",
+                  res.raster, res.kgroup, res.reduce);
     js += tmp;
     *out = res;
     if (report_needed) *report_needed = js.size() + 1;
@@ -1175,14 +1175,14 @@ nnjit_status nnjit_plan_describe(nnjit_plan pl, char* buf, size_t len, size_t* n
                   "\"candidate\":{\"bm\":%d,\"bn\":%d,\"bk\":%d,\"tm\":%d,\"tn\":%d,\"stages\":%d,"
                   "\"split_k\":%d,\"raster\":%d,\"threads\":%d,\"smem_bytes\":%d,\"tmem_cols\":%d,"
                   "\"regs_per_thread\":%d,\"blocks_per_sm\":%d,\"grid\":%d,\"wave_eff_ppm\":%d,"
-                  "\"instance\":%d,\"predicted_cost\":%lld},\"settings\":[%d,%d,%d,%d],\"timings_us\":[",
+                  "\"instance\":%d,\"predicted_cost\":%lld},\"settings\":[%d,%d,%d],\"timings_us\":[",
                   (long long)p.M, (long long)p.N, (long long)p.K, (long long)p.batch, p.dtype,
                   p.b_layout, pl->family, pl->chosen_index, pl->space_size, (long long)pl->naive,
                   pl->tune_ms, pl->from_cache ? "true" : "false", pl->timed ? "true" : "false",
                   c.bm, c.bn, c.bk, c.tm, c.tn, c.stages, c.split_k, c.raster, c.threads,
                   c.smem_bytes, c.tmem_cols, c.regs_per_thread, c.blocks_per_sm, c.grid,
                   c.wave_eff_ppm, c.instance, (long long)c.predicted_cost, pl->settings.raster,
-                  pl->settings.kgroup, pl->settings.reduce, pl->settings.multicast);
+                  pl->settings.kgroup, pl->settings.reduce);
     s += tmp;
     for (size_t i = 0; i < pl->timings.size(); ++i) {
         std::snprintf(tmp, sizeof tmp, "%s[%d,%.4f]", i ? "," : "", pl->timings[i].first,
@@ -1223,7 +1223,7 @@ int32_t nnjit_cache_size(void) {
 // File format: a header line, then one line per entry:
 //   key \t 20 candidate integers \t chosen_index space_size naive tune_ms timed \t
 //   n (index us)*n
-static const char* kCacheHeader = "nnjit-plan-cache v2";
+static const char* kCacheHeader = "nnjit-plan-cache v3";
 
 nnjit_status nnjit_cache_save(const char* path) {
     if (!path) return fail(NNJIT_ERR_INVALID_ARG, "path is NULL");

@@ -57,19 +57,17 @@ struct TileCoord {
     int b, s, tm, tn;
 };
 
-// Kernel modes: persistent CTAs (slices of a tile are separate work items), cluster
+// Kernel modes: persistent CTAs (slices of a tile are separate work items) and cluster
 // split-K (the split_k consecutive CTAs of a cluster share one output tile, CTA rank =
-// K slice), and multicast pairs (a cluster of 2 CTAs takes the two vertically adjacent
-// tiles 2*mp and 2*mp + 1 of one tile column; work item = pair).
+// K slice).
 constexpr int kModePersistent = 0;
 constexpr int kModeClusterSplitK = 1;
-constexpr int kModeMcastPair = 2;
 
 // Work item t -> (batch, K slice, tile row, tile column).
 template <int kMode>
-__device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p, int rank) {
+__device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p) {
     TileCoord c;
-    const int rows = kMode == kModeMcastPair ? (p.tiles_m + 1) / 2 : p.tiles_m;
+    const int rows = p.tiles_m;
     const int per = rows * p.tiles_n;
     int r, q;
     if constexpr (kMode == kModeClusterSplitK) {
@@ -90,7 +88,6 @@ __device__ __forceinline__ TileCoord decode_tile(int t, const TcParams& p, int r
         c.tn = r % p.tiles_n;
         c.tm = r / p.tiles_n;
     }
-    if constexpr (kMode == kModeMcastPair) c.tm = 2 * c.tm + rank;
     return c;
 }
 
@@ -107,7 +104,6 @@ constexpr int kErrDrain = 0x131;
 template <int kKind, bool kBMn, int BN, int kMode, int BM, int KG>
 __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_constant__ TcParams p) {
     constexpr bool kCluster = kMode == kModeClusterSplitK;
-    constexpr bool kMcast = kMode == kModeMcastPair;
     static_assert(BM == 128 || (BM == 64 && kMode == kModePersistent), "BM 64 tiles run persistent only");
     static_assert(KG == 1 || (KG == 2 && kMode == kModePersistent && BN <= 128),
                   "k-block groups: persistent tiles with BN <= 128");
@@ -156,41 +152,24 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         kb0 = (int)((long long)tc.s * p.num_kb / p.split);
         kb1 = (int)((long long)(tc.s + 1) * p.num_kb / p.split);
     };
-    // Multicast pairs: this CTA's rank in its cluster; work items are pairs.
-    const int rank = kMcast ? (int)ptx::cluster_ctarank() : 0;
-    const int t_begin = kMcast ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
-    const int t_step = kMcast ? (int)(gridDim.x >> 1) : (int)gridDim.x;
-    // B tile of k-block kb into the ring slot at `sb`.  In a multicast pair each CTA
-    // fetches one half of the tile and the copy lands in both CTAs' slots.
+    const int t_begin = (int)blockIdx.x;
+    const int t_step = (int)gridDim.x;
+    // B tile of k-block kb into the ring slot at `sb`.
     auto load_b = [&](uint32_t sb, const TileCoord& tc, int kb, uint32_t bar) {
         if constexpr (!kBMn) {
-            if constexpr (kMcast) {
-                constexpr int kHalf = BN / 2;
-                ptx::tma_load_3d_mc(sb + rank * kHalf * 128, &p.tmap_b, kb * BK, tc.tn * BN + rank * kHalf,
-                                    tc.b, bar, 0x3);
-            } else {
-                ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, bar);
-            }
+            ptx::tma_load_3d(sb, &p.tmap_b, kb * BK, tc.tn * BN, tc.b, bar);
         } else {
             constexpr int kBoxes = BN / kAtom;
-            constexpr int kPer = kMcast ? kBoxes / 2 : kBoxes;
 #pragma unroll
-            for (int i = 0; i < kPer; ++i) {
-                const int j = (kMcast ? rank * kPer : 0) + i;
-                if constexpr (kMcast)
-                    ptx::tma_load_3d_mc(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b,
-                                        bar, 0x3);
-                else
-                    ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b, bar);
-            }
+            for (int j = 0; j < kBoxes; ++j)
+                ptx::tma_load_3d(sb + j * (BK * 128), &p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b, bar);
         }
     };
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
             ptx::mbar_init(full_bar(s), 1);
-            // multicast pairs: a slot is free once both CTAs' MMAs have read it
-            ptx::mbar_init(empty_bar(s), kMcast ? 2 : 1);
+            ptx::mbar_init(empty_bar(s), 1);
         }
         for (int a = 0; a < 2; ++a) {
             ptx::mbar_init(tfull_bar(a), 1);
@@ -208,13 +187,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         // previous kernel may still be running: an L2 prefetch writes nothing, and L2 is
         // where the previous kernel's stores land, so no stale copy can result.
         if (t_begin < p.total_tiles) {
-            const TileCoord tc = decode_tile<kMode>(t_begin, p, rank);
+            const TileCoord tc = decode_tile<kMode>(t_begin, p);
             int kb0, kb1;
             kb_range(tc, kb0, kb1);
             for (int kb = kb0; kb < kb1 && kb < kb0 + S * KG; ++kb) {
                 ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm * BM, tc.b);
                 if constexpr (!kBMn) {
-                    ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN + (kMcast ? rank * (BN / 2) : 0), tc.b);
+                    ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN, tc.b);
                 } else {
                     for (int j = 0; j < BN / kAtom; ++j)
                         ptx::tma_prefetch_l2_3d(&p.tmap_b, tc.tn * BN + j * kAtom, kb * BK, tc.b);
@@ -230,15 +209,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     __syncthreads();
     ptx::tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
-    // multicast pairs: the partner's barriers must be initialised before any copy or
-    // commit of this CTA can reach them
-    if constexpr (kMcast) ptx::cluster_sync();
     // With a constant B the producer arms the first ring and starts its B tiles before
     // the dependency wait (the ring is empty, so no "empty" wait is needed); the loop
     // below then only adds the A tiles of those stages.
     int b_preloaded = 0;  // ring slots whose B tiles are already requested
     if (p.b_const && warp == 0 && t_begin < p.total_tiles) {
-        const TileCoord tc = decode_tile<kMode>(t_begin, p, rank);
+        const TileCoord tc = decode_tile<kMode>(t_begin, p);
         int kb0, kb1;
         kb_range(tc, kb0, kb1);
         b_preloaded = min(S, (kb1 - kb0 + KG - 1) / KG);
@@ -265,7 +241,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         bool ok = true;
         int issued = 0;  // ring slots filled so far by this CTA
         for (int t = t_begin; ok && t < p.total_tiles; t += t_step) {
-            const TileCoord tc = decode_tile<kMode>(t, p, rank);
+            const TileCoord tc = decode_tile<kMode>(t, p);
             int kb0, kb1;
             kb_range(tc, kb0, kb1);
             for (int g0 = kb0; g0 < kb1; g0 += KG) {
@@ -315,7 +291,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                                       : ptx::smem_desc(smem_base + kABytes, 16, 1024);
         constexpr uint32_t kBStep = kBMn ? (kUmmaK * 128) >> 4 : 32 >> 4;  // per MMA along K
         for (int t = t_begin; ok && t < p.total_tiles; t += t_step, ++iter) {
-            const TileCoord tc = decode_tile<kMode>(t, p, rank);
+            const TileCoord tc = decode_tile<kMode>(t, p);
             int kb0, kb1;
             kb_range(tc, kb0, kb1);
             const uint32_t acc = iter & 1u;
@@ -345,10 +321,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                                                    (g0 > kb0 || j > 0 || kk > 0) ? 1u : 0u);
                         }
                     }
-                    if constexpr (kMcast)
-                        ptx::tc_commit_mc(empty_bar(stage), 0x3);  // frees the slot in both CTAs
-                    else
-                        ptx::tc_commit(empty_bar(stage));
+                    ptx::tc_commit(empty_bar(stage));
                 }
                 __syncwarp();
                 if (++stage == S) {
@@ -379,7 +352,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
         uint32_t iter = 0;
         const long long MN = (long long)p.M * p.N;
         for (int t = t_begin; t < p.total_tiles; t += t_step, ++iter) {
-            const TileCoord tc = decode_tile<kMode>(t, p, rank);
+            const TileCoord tc = decode_tile<kMode>(t, p);
             const uint32_t acc = iter & 1u;
             const uint32_t acc_phase = (iter >> 1) & 1u;
             if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
@@ -520,7 +493,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             }
         }
         ptx::cluster_sync();
-        const TileCoord tc = decode_tile<kModeClusterSplitK>(blockIdx.x, p, 0);
+        const TileCoord tc = decode_tile<kModeClusterSplitK>(blockIdx.x, p);
         constexpr int kVec = BN / 4;
         const float* recv = reinterpret_cast<const float*>(smem);
         float* Cb = p.C + (long long)tc.b * p.stride_c;
@@ -551,9 +524,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
-    // multicast pairs: neither CTA leaves while the other may still copy into it or
-    // signal its barriers
-    if constexpr (kMcast) ptx::cluster_sync();
     if (warp == 1) ptx::tmem_dealloc(tmem_base, kTmemCols);
 }
 
@@ -561,11 +531,10 @@ using TcKernel = void (*)(TcParams);
 
 // Instance table, indexed as tc_instance(): variant * 12 + (dtype_i * 2 + kn) * 3 + bn_i
 // for variant 0 = 128-row persistent, 1 = 128-row cluster split-K, 2 = 64-row persistent;
-// then 36 + dtype_i * 2 + kn for the 128 x 256 multicast pairs; then
-// 40 + (dtype_i * 2 + kn) * 2 + bn_i for 128-row persistent tiles with BN = 64, 128 and
-// two k-blocks per ring slot.  (With BN = 256 the tensor pipe, not the issue path, sets
-// the pace, and halving the number of slots only shortens the lookahead.)
-constexpr int kNumTcInstances = 48;
+// then 36 + (dtype_i * 2 + kn) * 2 + bn_i for 128-row persistent tiles with BN = 64, 128
+// and two k-blocks per ring slot.  (With BN = 256 the tensor pipe, not the issue path,
+// sets the pace, and halving the number of slots only shortens the lookahead.)
+constexpr int kNumTcInstances = 44;
 #define NNJIT_TC_ROW(K, MN, MODE, BM)                                                  \
     tc_gemm_kernel<K, MN, 64, MODE, BM, 1>, tc_gemm_kernel<K, MN, 128, MODE, BM, 1>, \
         tc_gemm_kernel<K, MN, 256, MODE, BM, 1>
@@ -577,8 +546,6 @@ const TcKernel kTcKernels[kNumTcInstances] = {
     NNJIT_TC_ROW(1, false, 1, 128), NNJIT_TC_ROW(1, true, 1, 128),
     NNJIT_TC_ROW(0, false, 0, 64),  NNJIT_TC_ROW(0, true, 0, 64),
     NNJIT_TC_ROW(1, false, 0, 64),  NNJIT_TC_ROW(1, true, 0, 64),
-    tc_gemm_kernel<0, false, 256, 2, 128, 1>, tc_gemm_kernel<0, true, 256, 2, 128, 1>,
-    tc_gemm_kernel<1, false, 256, 2, 128, 1>, tc_gemm_kernel<1, true, 256, 2, 128, 1>,
     NNJIT_TC_KG2(0, false), NNJIT_TC_KG2(0, true), NNJIT_TC_KG2(1, false), NNJIT_TC_KG2(1, true),
 };
 #undef NNJIT_TC_ROW
@@ -644,8 +611,8 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
         cuuint32_t box[3];
         if (p.b_layout == NNJIT_B_NK) {
             dims[0] = (cuuint64_t)p.K; dims[1] = (cuuint64_t)p.N;
-            // a multicast pair fetches each B tile in two halves
-            box[0] = bk; box[1] = (cuuint32_t)(c.bn / (c.cluster_m == 2 ? 2 : 1));
+            // each CTA of a pair tile (bm = 256) loads its own half of the B tile
+            box[0] = bk; box[1] = (cuuint32_t)(c.bm == 256 ? c.bn / 2 : c.bn);
         } else {
             dims[0] = (cuuint64_t)p.N; dims[1] = (cuuint64_t)p.K;
             box[0] = 128 / e; box[1] = bk;
@@ -694,15 +661,13 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     if (c.instance < 0 || c.instance >= kNumTcInstances || !a.tmap_a || !a.tmap_b)
         return cudaErrorInvalidValue;
     const bool cluster = c.instance >= 12 && c.instance < 24;
-    const bool mcast = c.instance >= 36 && c.instance < 40;
-    const int kg = c.instance >= 40 ? 2 : 1;  // k-blocks per ring slot
+    const int kg = c.instance >= 36 ? 2 : 1;  // k-blocks per ring slot
     const int bk = 128 / p.elem_bytes();      // K elements per k-block
     if ((c.instance >= 24 && c.instance < 36) != (c.bm == 64) || (c.bm != 64 && c.bm != 128))
         return cudaErrorInvalidValue;
     if (c.bk != bk * kg || (kg == 2 && (c.bm != 128 || c.bn > 128 || c.reduce != 0)))
         return cudaErrorInvalidValue;
-    if (mcast != (c.cluster_m == 2) || (mcast && (c.bn != 256 || c.split_k != 1 || c.grid < 2 || (c.grid & 1))))
-        return cudaErrorInvalidValue;
+    if (c.cluster_m != 1) return cudaErrorInvalidValue;
     if (cluster != (c.reduce == 1)) return cudaErrorInvalidValue;
     if (cluster && (c.split_k < 2 || c.split_k > 8 || (c.split_k & (c.split_k - 1)) != 0))
         return cudaErrorInvalidValue;
@@ -728,24 +693,21 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     prm.split = c.split_k;
     prm.tiles_m = (int)((p.M + c.bm - 1) / c.bm);
     prm.tiles_n = (int)((p.N + c.bn - 1) / c.bn);
-    // work items: tiles (x K slices), or pairs of vertically adjacent tiles
-    const long long total = mcast ? (long long)p.batch * ((prm.tiles_m + 1) / 2) * prm.tiles_n
-                                  : (long long)p.batch * c.split_k * prm.tiles_m * prm.tiles_n;
+    // work items: tiles x K slices
+    const long long total = (long long)p.batch * c.split_k * prm.tiles_m * prm.tiles_n;
     if (total >= (1LL << 31)) return cudaErrorInvalidValue;
     if (c.split_k > prm.num_kb) return cudaErrorInvalidValue;  // every split owns >= 1 k-block
     prm.total_tiles = (int)total;
     prm.stages = c.stages;
     prm.raster = c.raster;
     // persistent: at most the candidate's grid; cluster mode: one CTA per (tile, slice)
-    const int grid = cluster ? (int)total
-                     : mcast ? (int)std::min<long long>(2 * total, c.grid)
-                             : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
+    const int grid = cluster ? (int)total : (int)std::min<long long>(total, c.grid > 0 ? c.grid : total);
     // ring + alignment slack + barriers/TMEM slot/abort flag
     const int stage_bytes = kg * (c.bm + c.bn) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     cudaError_t e = prepare_tc_instance(c.instance, smem);
     if (e != cudaSuccess) return e;
-    if (!cluster && !mcast)
+    if (!cluster)
         return launch_pdl(kTcKernels[c.instance], dim3(grid), dim3(kThreads), smem, a.stream, prm);
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);
@@ -756,7 +718,7 @@ cudaError_t launch_tc(const LaunchArgs& a) {
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     attr[1].id = cudaLaunchAttributeClusterDimension;
-    attr[1].val.clusterDim.x = mcast ? 2u : (unsigned)c.split_k;
+    attr[1].val.clusterDim.x = (unsigned)c.split_k;
     attr[1].val.clusterDim.y = 1;
     attr[1].val.clusterDim.z = 1;
     cfg.attrs = attr;

@@ -66,7 +66,8 @@ extern "C" nnjit_status nnjit_gemv_bf16_noalloc(int64_t M, int64_t N, int64_t K,
     }
     if (K % 8 != 0 || (reinterpret_cast<uintptr_t>(x) & 15) || (reinterpret_cast<uintptr_t>(W) & 15) ||
         (reinterpret_cast<uintptr_t>(C) & 3) || (bias && (reinterpret_cast<uintptr_t>(bias) & 3))) {
-        set_last_error("nnjit_gemv_bf16_noalloc: needs K % 8 == 0 and 16-byte aligned x and W");
+        set_last_error("nnjit_gemv_bf16_noalloc: needs K % 8 == 0, x and W 16-byte aligned, "
+                       "C and bias 4-byte aligned");
         return NNJIT_ERR_UNSUPPORTED;
     }
     // The partials of all K slices must fit the library's scratch array.

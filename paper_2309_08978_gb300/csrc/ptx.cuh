@@ -139,17 +139,6 @@ __device__ __forceinline__ void tma_prefetch_l2_2d(const void* tmap, int c0, int
                  : "memory");
 }
 
-// As tma_load_3d, but the tile lands at the same shared-memory offset in every CTA of
-// the cluster named in `mask`, and completes bytes on each one's barrier at `bar`.
-__device__ __forceinline__ void tma_load_3d_mc(uint32_t dst, const void* tmap, int c0, int c1, int c2,
-                                               uint32_t bar, uint16_t mask) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster"
-        " [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(bar), "h"(mask)
-        : "memory");
-}
-
 // Bring a 3-D tile into L2 (no shared-memory write, no completion to wait for).
 __device__ __forceinline__ void tma_prefetch_l2_3d(const void* tmap, int c0, int c1, int c2) {
     asm volatile("cp.async.bulk.prefetch.tensor.3d.L2.global.tile [%0, {%1, %2, %3}];" ::"l"(
@@ -268,15 +257,6 @@ __device__ __forceinline__ void mma_ss(uint32_t d_tmem, uint64_t adesc, uint64_t
 __device__ __forceinline__ void tc_commit(uint32_t bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
-        : "memory");
-}
-
-// As tc_commit, arriving on the barrier at the same offset in every CTA named in `mask`.
-__device__ __forceinline__ void tc_commit_mc(uint32_t bar, uint16_t mask) {
-    asm volatile(
-        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64"
-        " [%0], %1;" ::"r"(bar),
-        "h"(mask)
         : "memory");
 }
 

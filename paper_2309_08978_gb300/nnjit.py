@@ -82,7 +82,7 @@ NNJIT_ATTN_AUTO, NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA = 0, 1, 2
 
 
 NNJIT_SETTING_FREE = -1
-SETTING_AXES = ("raster", "kgroup", "reduce", "multicast")
+SETTING_AXES = ("raster", "kgroup", "reduce")
 
 
 class nnjit_settings(ctypes.Structure):

@@ -85,7 +85,7 @@ def test_cache_file_format(lib, tmp_path):
     nj.nnjit_cache_clear()
     empty = tmp_path / "empty.cache"
     nj.nnjit_cache_save(str(empty))
-    assert empty.read_text().splitlines() == ["nnjit-plan-cache v2"]
+    assert empty.read_text().splitlines() == ["nnjit-plan-cache v3"]
     assert nj.nnjit_cache_load(str(empty)) == 0
     bad = tmp_path / "bad.cache"
     bad.write_text("something else\n")
@@ -96,13 +96,13 @@ def test_cache_file_format(lib, tmp_path):
     entry = ("t=matmul|s=1,2,3,1|dt=2|bl=1|ld=3,3,2|st=3,6,2|bias=0|dev=X,cc103,sm152\t"
              "1 128 256 64 0 0 4 1 0 192 230656 512 72 1 1 1000000 2 9 0 1\t0 6 336 12.5 1\t2 0 3.5 1 4.25\n")
     good = tmp_path / "good.cache"
-    good.write_text("nnjit-plan-cache v2\n" + entry)
+    good.write_text("nnjit-plan-cache v3\n" + entry)
     assert nj.nnjit_cache_load(str(good)) == 1
     assert nj.nnjit_cache_size() == 1
     out = tmp_path / "out.cache"
     nj.nnjit_cache_save(str(out))
     lines = out.read_text().splitlines()
-    assert lines[0] == "nnjit-plan-cache v2" and lines[1].split("\t")[0] == entry.split("\t")[0]
+    assert lines[0] == "nnjit-plan-cache v3" and lines[1].split("\t")[0] == entry.split("\t")[0]
     assert lines[1].split("\t")[1] == entry.split("\t")[1]
     nj.nnjit_cache_clear()
     assert nj.nnjit_cache_size() == 0
@@ -124,15 +124,15 @@ def test_settings_roundtrip_and_validation(lib):
     """nnjit_settings_set/get: values round-trip, out-of-range values are refused without
     changing the current settings, NULL clears (host only)."""
     import paper_2309_08978_gb300 as nj
-    assert nj.nnjit_settings_get() == {"raster": -1, "kgroup": -1, "reduce": -1, "multicast": -1}
+    assert nj.nnjit_settings_get() == {"raster": -1, "kgroup": -1, "reduce": -1}
     try:
-        nj.nnjit_settings_set({"raster": 1, "multicast": 0})
-        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": -1, "multicast": 0}
-        for bad in ({"kgroup": 0}, {"kgroup": 3}, {"raster": 2}, {"reduce": -2}, {"multicast": 5}):
+        nj.nnjit_settings_set({"raster": 1, "reduce": 0})
+        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": 0}
+        for bad in ({"kgroup": 0}, {"kgroup": 3}, {"raster": 2}, {"reduce": -2}, {"reduce": 5}):
             with pytest.raises(nj.NnjitError) as ei:
                 nj.nnjit_settings_set(bad)
             assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
-        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": -1, "multicast": 0}
+        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": 0}
     finally:
         nj.nnjit_settings_set(None)
     assert nj.nnjit_settings_get()["raster"] == -1

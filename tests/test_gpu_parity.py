@@ -185,7 +185,8 @@ def test_constant_b_flag_is_exact(case):
     # the first few candidates, plus every tensor-core one with two k-blocks per ring slot
     # (whose preloaded B tiles are grouped two to a barrier)
     picks = sorted(set(range(min(len(cands), 6))) |
-                   {i for i, c in enumerate(cands) if c["family"] == nj.NNJIT_FAMILY_TC and c["instance"] >= 40})
+                   {i for i, c in enumerate(cands) if c["family"] == nj.NNJIT_FAMILY_TC and
+                    (c["bk"] * (2 if dtype == "bf16" else 4) == 256 or c["cluster_m"] == 2)})
     for i in picks:
         with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
             C = run_plan(plan, A, B, bias, M, N)
@@ -275,24 +276,26 @@ def test_gemv_tma_writes_after_the_previous_kernel():
         p1.destroy()
 
 
-PAIR_CASES = [("bf16", 2048, 2560, 192, "NK"), ("bf16", 2176, 2560, 136, "KN"),
-              ("tf32", 2048, 2560, 64, "NK"), ("tf32", 2200, 2560, 40, "KN")]
+FULL_WAVE_CASES = [("bf16", 2048, 2560, 192, "NK"), ("bf16", 2176, 2560, 136, "KN"),
+                   ("tf32", 2048, 2560, 64, "NK"), ("tf32", 2200, 2560, 40, "KN")]
 
 
-@pytest.mark.parametrize("case", PAIR_CASES, ids=_ids)
-def test_multicast_pairs_exact(case):
-    """Two CTAs of a cluster take vertically adjacent 128 x 256 tiles and share each B tile
-    through TMA multicast (each fetches one half).  Includes an odd number of tile rows,
-    where the second tile of the last pair lies entirely past M."""
+@pytest.mark.parametrize("case", FULL_WAVE_CASES, ids=_ids)
+def test_full_wave_shapes_every_candidate_exact(case):
+    """Shapes with more tiles than SMs, so persistent CTAs take several tiles and the
+    accumulator barriers cycle: every candidate (CTA-pair tiles included where B is
+    [N][K]), with and without a constant B.  Includes an odd number of 256-row tile
+    rows, where the last pair tile lies partly past M."""
     dtype, M, N, K, layout = case
     shape = Shape("t", M, N, K, 1, layout, True)
     A, B, bias = make_operands(shape, 14, dtype, ints=True)
     for flags in (0, nj.NNJIT_PLAN_B_CONSTANT):
         desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, flags=flags)
         cands, _ = nj.nnjit_space_enumerate(desc, nj.nnjit_device_limits_query(0))
-        pairs = [i for i, c in enumerate(cands) if c["cluster_m"] == 2]
-        assert pairs, "expected multicast-pair candidates for a full-wave shape"
-        for i in pairs:
+        assert all(c["cluster_m"] == 1 or c["bm"] == 256 for c in cands)
+        if layout == "NK":
+            assert any(c["cluster_m"] == 2 for c in cands), "expected CTA-pair candidates"
+        for i in range(len(cands)):
             with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
                 C = run_plan(plan, A, B, bias, M, N)
             compare(C, A, B, bias, layout, dtype, exact=True)
