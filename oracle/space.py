@@ -37,10 +37,12 @@ TC_BM = 128
 TC_FIXED_SMEM = 1024 + 256 + 32768   # alignment slack, barriers, epilogue staging
 TC_MAX_STAGES = 8
 TC_PAIR_ACC_COLS = 512        # TMEM columns of the CTA-pair tile kernel (2 x 256)
-TC_PAIR_FIRST = 48            # instance ids of the CTA-pair tile kernel (bf16, tf32)
+TC_PAIR_FIRST = 44            # instance ids of the CTA-pair tile kernel (bf16, tf32)
 MMA_N256_CLK = 128            # tensor pipe: one M = 128, N = 256 MMA instruction
 MMA_ISSUE_CLK = 57            # issuing thread: one tcgen05.mma
 SLOT_SYNC_CLK = 226           # issuing thread: one ring-slot barrier wait + commit
+ISSUE_SHOW = 8                # 1/8 of the issue path is not hidden behind the feed
+DSMEM_REDUCE_BYTES_PER_CLK = 5   # cluster split-K partial exchange and sum, per SM
 GEMV_MAX_M = 8
 GEMV_MAX_SMEM = 64 * 1024
 GEMV_TMA_KC = 256             # K elements per ring stage of the TMA-fed GEMV
@@ -191,11 +193,9 @@ def _blank():
     return c
 
 
-def tc_instance(dtype, b_layout, bn, cluster, bm, mcast=False, kg=1):
+def tc_instance(dtype, b_layout, bn, cluster, bm, kg=1):
     if kg == 2:
-        return 40 + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 2 + {64: 0, 128: 1}[bn]
-    if mcast:
-        return 36 + (0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)
+        return 36 + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 2 + {64: 0, 128: 1}[bn]
     variant = 2 if bm == 64 else (1 if cluster else 0)
     return variant * 12 + ((0 if dtype == BF16 else 1) * 2 + (1 if b_layout == B_KN else 0)) * 3 + \
         {64: 0, 128: 1, 256: 2}[bn]
@@ -269,12 +269,12 @@ def _tc(p, lim):
                     # per k-block: tensor pipe, issuing thread, operand feed
                     t_tensor = 4 * max(MMA_N256_CLK // 4, MMA_N256_CLK * bn // 256)
                     t_issue = 4 * MMA_ISSUE_CLK + SLOT_SYNC_CLK // kg
-                    t_kb = max(t_tensor, t_issue, cdiv(kb_bytes, FEED_BYTES_PER_CLK))
+                    t_kb = max(t_tensor, t_issue, cdiv(kb_bytes, FEED_BYTES_PER_CLK)) + t_issue // ISSUE_SHOW
                     cost = waves * t_kb * cdiv(num_kb, split)
                     if split > 1 and reduce == 0:
                         cost += LAUNCH_CLK + cdiv(2 * split * p.batch * M * N * 4, HBM_BYTES_PER_CLK)
                     if split > 1 and reduce == 1:
-                        cost += waves * (TC_BM * bn * 4 // FEED_BYTES_PER_CLK)
+                        cost += waves * (TC_BM * bn * 4 // DSMEM_REDUCE_BYTES_PER_CLK)
                     c.update(family=FAMILY_TC, bm=bm, bn=bn, bk=bk * kg, stages=stages, split_k=split,
                              raster=raster, threads=TC_THREADS, smem_bytes=smem, tmem_cols=tmem,
                              regs_per_thread=TC_REGS, blocks_per_sm=blk,
@@ -282,17 +282,6 @@ def _tc(p, lim):
                              instance=tc_instance(p.dtype, p.b_layout, bn, reduce, bm, kg=kg),
                              predicted_cost=cost, reduce=reduce)
                     out.append(c)
-                    # multicast pair: two CTAs of a cluster share each B tile
-                    if bm == TC_BM and bn == 256 and split == 1 and tiles >= lim["sm_count"]:
-                        m = dict(c)
-                        pairs = p.batch * cdiv(tiles_m, 2) * tiles_n
-                        live = min(pairs, max(1, slots // 2))
-                        pw = cdiv(pairs, live)
-                        feed = cdiv(kb_bytes - bn * 128 // 2, FEED_BYTES_PER_CLK)
-                        m.update(cluster_m=2, grid=2 * live, wave_eff_ppm=pairs * 1000000 // (pw * live),
-                                 predicted_cost=pw * max(t_tensor, t_issue, feed) * num_kb,
-                                 instance=tc_instance(p.dtype, p.b_layout, bn, 0, bm, True, kg))
-                        out.append(m)
     # 256 x 256 tiles on CTA pairs (tcgen05 cta_group::2), B as [N][K]: an SM receives its
     # 128 rows of A and half of the B tile per k-block; one thread issues for both SMs
     if p.b_layout == B_NK and M > TC_BM and lim["sm_count"] >= 2:
@@ -309,7 +298,8 @@ def _tc(p, lim):
                     continue
                 live = min(pairs, max(1, lim["sm_count"] * blk // 2))
                 waves = cdiv(pairs, live)
-                t_kb = max(4 * MMA_N256_CLK, 4 * MMA_ISSUE_CLK + SLOT_SYNC_CLK, cdiv(kb_bytes, FEED_BYTES_PER_CLK))
+                t_issue = 4 * MMA_ISSUE_CLK + SLOT_SYNC_CLK
+                t_kb = max(4 * MMA_N256_CLK, t_issue, cdiv(kb_bytes, FEED_BYTES_PER_CLK)) + t_issue // ISSUE_SHOW
                 c = _blank()
                 c.update(family=FAMILY_TC, bm=256, bn=256, bk=bk, stages=stages, raster=raster,
                          threads=TC_THREADS, smem_bytes=smem, tmem_cols=tmem, regs_per_thread=TC_REGS,
@@ -518,23 +508,21 @@ def _gemv(p, lim):
     return out, 2 * 2 * 6
 
 
-SETTING_AXES = ("raster", "kgroup", "reduce", "multicast")
-SETTING_RANGE = {"raster": (0, 1), "kgroup": (1, 2), "reduce": (0, 1), "multicast": (0, 1)}
+SETTING_AXES = ("raster", "kgroup", "reduce")
+SETTING_RANGE = {"raster": (0, 1), "kgroup": (1, 2), "reduce": (0, 1)}
 
 
 def setting_value(p: Problem, c: dict, axis: str):
     """The fixed-setting value of a tensor-core candidate (None for other families):
-    tile order, k-blocks per ring slot (bk over one 128-byte k-block), split-K reduction,
-    and whether it is a 128-row multicast pair."""
+    tile order, k-blocks per ring slot (bk over one 128-byte k-block) and split-K
+    reduction."""
     if c["family"] != FAMILY_TC:
         return None
     if axis == "raster":
         return c["raster"]
     if axis == "kgroup":
         return c["bk"] // (128 // p.elem)
-    if axis == "reduce":
-        return c["reduce"]
-    return 1 if (c["bm"] == TC_BM and c["cluster_m"] == 2) else 0
+    return c["reduce"]
 
 
 def _twins(p: Problem, a: dict, b: dict, axis: str) -> bool:

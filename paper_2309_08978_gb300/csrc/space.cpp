@@ -58,7 +58,7 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
     const int64_t num_kb = ceil_div(K, BK);
     const int bns[3] = {64, 128, 256};
     const int splits[4] = {1, 2, 4, 8};
-    // BM x BN x stages x split x raster x reduce x pair x k-blocks per ring slot
+    // BM x BN x stages x split x raster x reduce x CTA pair x k-blocks per ring slot
     *naive = 2 * 3 * (MC::kTcMaxStages - 1) * 4 * 2 * 2 * 2 * 2;
     for (int BM : {MC::kTcBM, 64})
     for (int bn : bns)
@@ -116,37 +116,21 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 // instruction takes kMmaN256Clk * N / 256, at least a quarter of that),
                 // the issuing thread (kMmaIssueClk per instruction plus one barrier wait
                 // and commit per ring slot) and the operand feed (bytes over the per-SM
-                // L2 feed)
+                // L2 feed), plus the share of the issue path that the feed does not hide
                 const int64_t t_tensor = 4LL * std::max(MC::kMmaN256Clk / 4, MC::kMmaN256Clk * bn / 256);
                 const int64_t t_issue = 4LL * MC::kMmaIssueClk + MC::kSlotSyncClk / kg;
                 const int64_t t_kb = std::max(std::max(t_tensor, t_issue),
-                                              ceil_div(kb_bytes, MC::kFeedBytesPerClk));
+                                              ceil_div(kb_bytes, MC::kFeedBytesPerClk)) +
+                                     t_issue / MC::kIssueShowDiv;
                 int64_t cost = waves * t_kb * ceil_div(num_kb, split);
                 if (split > 1 && reduce == 0)
                     cost += MC::kLaunchClk +
                             ceil_div(2LL * split * p.batch * M * N * 4, MC::kHbmBytesPerClk);
-                if (split > 1 && reduce == 1)
-                    cost += waves * (128LL * bn * 4 / MC::kFeedBytesPerClk);  // DSMEM reduction
+                if (split > 1 && reduce == 1)  // DSMEM reduction of the partial tiles
+                    cost += waves * (128LL * bn * 4 / MC::kDsmemReduceBytesPerClk);
                 c.predicted_cost = cost;
-                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM, 0, kg);
+                c.instance = tc_instance(p.dtype, p.b_layout, bn, reduce, BM, kg);
                 v.push_back(c);
-                // Multicast pair of the same tile: for full waves of 128 x 256 tiles, two
-                // CTAs of a cluster take vertically adjacent tiles and share each B tile,
-                // halving the B bytes each SM pulls from L2 (32 instead of 48 KB per k-block).
-                if (BM == MC::kTcBM && bn == 256 && split == 1 && tiles >= L.sm_count) {
-                    nnjit_candidate m = c;
-                    m.cluster_m = 2;
-                    const int64_t pairs = p.batch * ceil_div(tiles_m, 2) * tiles_n;
-                    const int64_t pair_slots = std::max<int64_t>(1, slots / 2);
-                    const int64_t live_pairs = std::min(pairs, pair_slots);
-                    const int64_t pwaves = ceil_div(pairs, live_pairs);
-                    m.grid = (int32_t)(2 * live_pairs);
-                    m.wave_eff_ppm = (int32_t)(pairs * 1000000 / (pwaves * live_pairs));
-                    const int64_t feed = ceil_div(kb_bytes - bn * 128 / 2, MC::kFeedBytesPerClk);
-                    m.predicted_cost = pwaves * std::max(std::max(t_tensor, t_issue), feed) * num_kb;
-                    m.instance = tc_instance(p.dtype, p.b_layout, bn, 0, BM, 1, kg);
-                    v.push_back(m);
-                }
             }
         }
     }
@@ -182,7 +166,8 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 c.wave_eff_ppm = (int32_t)(pairs * 1000000 / (waves * live));
                 const int64_t t_tensor = 4LL * MC::kMmaN256Clk;
                 const int64_t t_issue = 4LL * MC::kMmaIssueClk + MC::kSlotSyncClk;
-                const int64_t t_kb = std::max(std::max(t_tensor, t_issue), ceil_div(kb_bytes, MC::kFeedBytesPerClk));
+                const int64_t t_kb = std::max(std::max(t_tensor, t_issue), ceil_div(kb_bytes, MC::kFeedBytesPerClk)) +
+                                     t_issue / MC::kIssueShowDiv;
                 c.predicted_cost = waves * t_kb * num_kb;
                 c.instance = kTcPairFirstInstance + (p.dtype == NNJIT_BF16 ? 0 : 1);
                 v.push_back(c);
@@ -479,16 +464,15 @@ void gemv_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnji
 
 }  // namespace
 
-int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast, int kg) {
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int kg) {
     const int bi = bn == 64 ? 0 : bn == 128 ? 1 : bn == 256 ? 2 : -1;
     if (bi < 0 || (bm != 64 && bm != 128) || (bm == 64 && cluster)) return -1;
     const int di = dtype == NNJIT_BF16 ? 0 : 1;
     if (kg == 2) {
-        if (bm != 128 || cluster || mcast || bn > 128) return -1;
-        return 40 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 2 + bi;
+        if (bm != 128 || cluster || bn > 128) return -1;
+        return 36 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 2 + bi;
     }
     if (kg != 1) return -1;
-    if (mcast) return (bn == 256 && bm == 128 && !cluster) ? 36 + di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0) : -1;
     const int variant = bm == 64 ? 2 : cluster ? 1 : 0;
     return variant * 12 + (di * 2 + (b_layout == NNJIT_B_KN ? 1 : 0)) * 3 + bi;
 }
@@ -618,7 +602,7 @@ nnjit_status choose_family(const Problem& p, int* family, std::string* err) {
 
 nnjit_settings free_settings() {
     nnjit_settings s;
-    s.raster = s.kgroup = s.reduce = s.multicast = NNJIT_SETTING_FREE;
+    s.raster = s.kgroup = s.reduce = NNJIT_SETTING_FREE;
     return s;
 }
 
@@ -627,14 +611,13 @@ int setting_of(const nnjit_settings& s, int axis) {
         case 0: return s.raster;
         case 1: return s.kgroup;
         case 2: return s.reduce;
-        case 3: return s.multicast;
         default: return NNJIT_SETTING_FREE;
     }
 }
 
 bool settings_valid(const nnjit_settings& s, std::string* err) {
-    const int lo[kSettingAxes] = {0, 1, 0, 0}, hi[kSettingAxes] = {1, 2, 1, 1};
-    const char* names[kSettingAxes] = {"raster", "kgroup", "reduce", "multicast"};
+    const int lo[kSettingAxes] = {0, 1, 0}, hi[kSettingAxes] = {1, 2, 1};
+    const char* names[kSettingAxes] = {"raster", "kgroup", "reduce"};
     for (int a = 0; a < kSettingAxes; ++a) {
         const int v = setting_of(s, a);
         if (v != NNJIT_SETTING_FREE && (v < lo[a] || v > hi[a])) {
@@ -651,7 +634,6 @@ int candidate_setting(const Problem& p, const nnjit_candidate& c, int axis) {
         case 0: return c.raster;
         case 1: return c.bk / (128 / p.elem_bytes());
         case 2: return c.reduce;
-        case 3: return (c.bm == ModelConstants::kTcBM && c.cluster_m == 2) ? 1 : 0;
         default: return -1;
     }
 }

@@ -55,6 +55,10 @@ struct ModelConstants {
     static constexpr int kMmaN256Clk = 128;           // tensor pipe: one M = 128, N = 256 MMA
     static constexpr int kMmaIssueClk = 57;           // issuing thread: one tcgen05.mma
     static constexpr int kSlotSyncClk = 226;          // issuing thread: ring-slot wait + commit
+    static constexpr int kIssueShowDiv = 8;           // 1/8 of the issue path is not hidden
+                                                      // behind the operand feed
+    static constexpr int kDsmemReduceBytesPerClk = 5; // cluster split-K: partial-tile exchange
+                                                      // and sum through DSMEM, per SM
     static constexpr int kGemvMaxM = 8;
     static constexpr int kGemvMaxSmem = 64 * 1024;
     static constexpr int kGemvTmaKc = 256;           // K elements per TMA GEMV ring stage
@@ -69,9 +73,9 @@ nnjit_status resolve_problem(const nnjit_matmul_desc* d, Problem* p, std::string
 nnjit_status choose_family(const Problem& p, int* family, std::string* err);
 
 // Fixed settings (nnjit_settings, the primitive vector of Sec. 5.1).  Axis a of a
-// tensor-core candidate: 0 raster, 1 k-blocks per ring slot, 2 split-K reduction,
-// 3 multicast pair; -1 for candidates of other families.
-constexpr int kSettingAxes = 4;
+// tensor-core candidate: 0 raster, 1 k-blocks per ring slot, 2 split-K reduction; -1 for
+// candidates of other families.
+constexpr int kSettingAxes = 3;
 nnjit_settings free_settings();
 int setting_of(const nnjit_settings& s, int axis);
 bool settings_valid(const nnjit_settings& s, std::string* err);
@@ -91,9 +95,9 @@ nnjit_status build_space(const Problem& p, const nnjit_device_limits& lim, const
 // Precompiled-instance index helpers (kept in one place so the registry and the space
 // agree).
 // kg: k-blocks per ring slot (2 only for 128-row persistent tiles with BN <= 128)
-int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int mcast, int kg = 1);  // 0..47
-// 256 x 256 tiles on CTA pairs (tcgen05 cta_group::2), B as [N][K]: 48 (bf16), 49 (tf32).
-constexpr int kTcPairFirstInstance = 48;
+int tc_instance(int dtype, int b_layout, int bn, int cluster, int bm, int kg = 1);  // 0..43
+// 256 x 256 tiles on CTA pairs (tcgen05 cta_group::2), B as [N][K]: 44 (bf16), 45 (tf32).
+constexpr int kTcPairFirstInstance = 44;
 int ffma_instance(int tm, int bm, int bn, int bk, int b_layout);  // 0..23, -1 if none
 int gemv_instance(int b_layout, int rows, int unroll);        // 0..7, -1 if none
 // TMA-fed GEMV (B as [N][K]): rows per stage 8/16/32, M <= maxm (1 or 8).

@@ -137,8 +137,8 @@ def test_space_invariants_on_gb300():
 
 SETTINGS_CASES = [
     {"raster": 0}, {"raster": 1}, {"kgroup": 2}, {"kgroup": 1, "reduce": 1},
-    {"reduce": 0, "multicast": 1}, {"multicast": 0, "raster": 1},
-    {"raster": 0, "kgroup": 2, "reduce": 1, "multicast": 1},
+    {"reduce": 0}, {"reduce": 1, "raster": 1},
+    {"raster": 0, "kgroup": 2, "reduce": 1},
 ]
 
 
@@ -201,12 +201,75 @@ def test_fixed_settings_prune_only_where_a_twin_exists():
 
 def test_setting_values_of_candidates():
     """The setting accessors read what the candidates encode: bk = 2 k-blocks of 128 bytes
-    for kgroup 2 (64 bf16 elements per k-block), multicast only for 128-row pairs."""
+    for kgroup 2 (64 bf16 elements per k-block); the only two-CTA clusters are the
+    256-row CTA-pair tiles."""
     p = osp.resolve(M=4096, N=4096, K=4096, dtype=osp.BF16, b_layout=osp.B_NK)
     cands, _ = osp.build_space(p, GB300)
     kg = {osp.setting_value(p, c, "kgroup") for c in cands}
     assert kg == {1, 2}
     assert all(c["bk"] == 64 * osp.setting_value(p, c, "kgroup") for c in cands)
     pairs = [c for c in cands if c["cluster_m"] == 2]
-    assert {osp.setting_value(p, c, "multicast") for c in pairs} == {0, 1}   # CTA pairs and multicast pairs
-    assert all(osp.setting_value(p, c, "multicast") == (c["bm"] == 128) for c in pairs)
+    assert pairs and all(c["bm"] == 256 and c["bn"] == 256 for c in pairs)
+
+
+BLACKWELL = os.path.join(os.path.dirname(__file__), "golden", "blackwell_usage.txt")
+_DT = {"bf16": osp.BF16, "tf32": osp.TF32, "f32_ffma": osp.F32_FFMA, "w4_bf16": osp.W4_BF16}
+_FAM = {"tc": osp.FAMILY_TC, "ffma": osp.FAMILY_FFMA, "gemv": osp.FAMILY_GEMV}
+
+
+def _blackwell_rows(kind):
+    for line in open(BLACKWELL):
+        if line.startswith("#") or not line.strip():
+            continue
+        head, *rest = [part.strip() for part in line.split("|")]
+        fam, dt, lay, M, N, K = head.split()
+        if (fam == "order") != (kind == "order"):
+            continue
+        prob = dict(M=int(M), N=int(N), K=int(K), dtype=_DT[dt],
+                    b_layout=osp.B_NK if lay == "NK" else osp.B_KN)
+        if kind == "order":
+            yield prob, [[int(v) for v in r.split()] for r in rest]
+        else:
+            pick = {k: int(v) for k, v in (t.split("=") for t in rest[0].split())}
+            want = {k: int(v) for k, v in (t.split("=") for t in rest[1].split())}
+            yield fam, prob, pick, want
+
+
+def _both_spaces(prob):
+    """The library's space (host only, GB300 limits) and the oracle restatement's."""
+    import paper_2309_08978_gb300 as nj
+    p = osp.resolve(**prob)
+    ours, _ = osp.build_space(p, GB300)
+    lay = "NK" if prob["b_layout"] == osp.B_NK else "KN"
+    dt = {v: k for k, v in _DT.items()}[prob["dtype"]]
+    lib, _ = nj.nnjit_space_enumerate(nj.make_desc(prob["M"], prob["N"], prob["K"], dt, lay),
+                                      _limits(GB300))
+    return {"oracle": ours, "library": lib}
+
+
+@pytest.mark.parametrize("fam,prob,pick,want", list(_blackwell_rows("usage")),
+                         ids=lambda v: str(v) if not isinstance(v, dict) else
+                         ",".join(f"{k}={x}" for k, x in v.items() if k in ("M", "N", "K", "bm", "bn",
+                                                                          "bk", "split_k", "reduce",
+                                                                          "stages", "tm")))
+def test_blackwell_usage_matches_hand_worked_values(fam, prob, pick, want):
+    """Stages, shared memory, TMEM columns, registers, blocks per SM, grid, wave efficiency
+    and the ordering cost of chosen candidates, worked by hand from the usage formulas
+    (tests/golden/blackwell_usage.txt), for the library and the oracle restatement alike."""
+    for who, space in _both_spaces(prob).items():
+        hits = [c for c in space if c["family"] == _FAM[fam] and all(c[k] == v for k, v in pick.items())]
+        assert len(hits) == 1, f"{who}: {len(hits)} candidates match {pick}"
+        got = {k: hits[0][k] for k in want}
+        assert got == want, f"{who}: {got} != {want}"
+
+
+@pytest.mark.parametrize("prob,order", list(_blackwell_rows("order")))
+def test_evaluation_order_matches_hand_ordering(prob, order):
+    """The 4096^3 BF16 space, index by index, in the order worked out by hand (blocks per
+    SM, then the cost, then enumeration order)."""
+    for who, space in _both_spaces(prob).items():
+        assert len(space) == len(order), f"{who}: {len(space)} candidates"
+        for idx, bm, bn, bk, raster, cluster in order:
+            c = space[idx]
+            assert (c["bm"], c["bn"], c["bk"], c["raster"], c["cluster_m"]) == (bm, bn, bk, raster, cluster), \
+                f"{who}: index {idx} is {c}"
