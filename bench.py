@@ -1,15 +1,20 @@
 """Benchmark of the JIT-tuned MatMul hot path on one workload (one JSON line on stdout).
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload NAME] [--budget-ms B] [--no-sweep]
+    python bench.py [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME] [--tune-budget-ms B] [--no-sweep]
 
-A step is one pass of the workload's products (for the default workload, the four
-Linears of a BART-base encoder layer at batch 4 x seq 128, TF32) over one batch of
-synthetic input.  Plans are tuned first (the JIT phase, timed separately and reported
-under "tune"); the timed region then runs K steps.  Each product's K launches run as a
-block of CUDA-graph replays that rotate over enough operand copies to exceed the L2, so
-operands come from HBM; CUDA events at the block boundaries give every kernel's average
-launch duration.  Under torchrun each rank runs its own replica (weak scaling).
+A step is one pass of the workload's products over one batch of synthetic input.  The
+default workload is the Llama-2-7B decoder block prefill at batch 4 x seq 1024 (M = 4096,
+BF16): the four Linears (qkv, o-proj, gate/up, down) and the two attention BatchMatMuls
+(QK^T and PV over 128 batch x heads).  Plans are tuned first under one total budget (the
+JIT phase, timed separately and reported under "tune", with the exhaustive sweep of the
+same spaces beside it); the timed region then runs K steps.  Each product's K launches
+run as a block of CUDA-graph replays that rotate over enough operand copies to exceed the
+L2, so operands come from HBM; CUDA events at the block boundaries give every kernel's
+average launch duration.
+
+The operator runs on one GPU: --gpus above 1 (or a torchrun world above 1) prints an
+"unavailable" line and exits 0 without touching a GPU.
 
 --impl reference times the oracle (the plain CPU definition) on the host cores on the
 same workload and metric.
@@ -29,10 +34,9 @@ ROOT = os.path.dirname(os.path.abspath(__file__))
 if ROOT not in sys.path:
     sys.path.insert(0, ROOT)
 
-DEFAULT_WORKLOAD = "bart_base_encoder_m512"
+DEFAULT_WORKLOAD = "llama2_7b_prefill_m4096"
 METRIC = "GEMM TFLOP/s (GEMV GB/s) vs GB300 roofline per shape; JIT tune time to plan"
-TF32_OVER_BF16 = 1.1 / 2.25     # nominal dense TF32 / BF16 tensor rates
-FFMA_PEAK_NOTE = "FP32 FFMA: 152 SMs x 128 FMA/clk x 2 x SM clock"
+TF32_OVER_BF16 = 1.1 / 2.25     # nominal dense TF32 / BF16 tensor rates (fallback only)
 
 
 def log(*a):
@@ -58,20 +62,73 @@ def shape_bytes(s, dtype):
     return b + (4 * s.N if s.has_bias else 0)
 
 
-def max_over_ranks(x: float, world: int, device=None) -> float:
-    """The largest of every rank's value (the slowest rank's time); identity at world 1."""
-    if world <= 1:
-        return float(x)
+def job_throughput(flops_per_step: int, steps: int, ms: float) -> float:
+    """TFLOP/s of `steps` steps of `flops_per_step` in `ms` milliseconds."""
+    return flops_per_step * steps / (ms / 1e3) / 1e12
+
+
+def prefix_curve(times_us: dict, n: int) -> dict:
+    """pick/best had the tuner timed only a prefix of the ordered space: for the first k
+    candidates (k = 1, 2, 3, 5, 10) and the first 10 / 25 / 50 % of the space, the best
+    time among them over the best time of the whole space."""
+    best = min(times_us.values())
+    out = {}
+
+    def ratio(k):
+        seen = [t for i, t in times_us.items() if i < k]
+        return round(min(seen) / best, 4) if seen else None
+
+    for k in (1, 2, 3, 5, 10):
+        out[f"first_{k}"] = ratio(min(k, n))
+    for pct in (10, 25, 50):
+        out[f"first_{pct}pct"] = ratio(max(1, math.ceil(pct * n / 100)))
+    return out
+
+
+def workload_config(workload, args) -> dict:
+    """The "config" object of the JSON line: the same for both arms."""
+    return {"workload": workload.key, "title": workload.title, "epilogue": args.epilogue,
+            "shapes": [[s.batch, s.M, s.N, s.K, s.b_layout] for s in workload.shapes],
+            "parallelism": "single GPU",
+            "l2": "each product rotates over operand copies totalling >= 3 x L2 (inputs larger "
+                  "than L2), so every timed launch reads its operands from HBM",
+            "schedule": "per product: K launches as CUDA-graph replays, products in sequence"}
+
+
+def probe_peaks(dtype, dev):
+    """Measured dense peaks for the non-BF16 paths, taken on this GPU at bench start:
+    TF32 = torch.matmul on float32 8192^3 with TF32 allowed, FP32 FFMA = the same with
+    TF32 off (cuBLAS SGEMM), each the best of several CUDA-event-timed launches."""
     import torch
-    import torch.distributed as dist
-    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
-    dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    return float(t.item())
-
-
-def job_throughput(world: int, flops_per_step: int, steps: int, ms: float) -> float:
-    """Whole-job TFLOP/s: every replica ran `steps` steps; `ms` is the slowest rank's time."""
-    return world * flops_per_step * steps / (ms / 1e3) / 1e12
+    if dtype not in ("tf32", "f32_ffma"):
+        return {}
+    n = 8192
+    a = torch.randn(n, n, device=dev)
+    b = torch.randn(n, n, device=dev)
+    out = {}
+    old = torch.backends.cuda.matmul.allow_tf32
+    try:
+        for name, tf32, reps in (("tf32_tflops", True, 10), ("ffma_tflops", False, 4)):
+            torch.backends.cuda.matmul.allow_tf32 = tf32
+            for _ in range(2):
+                torch.matmul(a, b)
+            torch.cuda.synchronize()
+            best = float("inf")
+            for _ in range(reps):
+                e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                e0.record()
+                torch.matmul(a, b)
+                e1.record()
+                torch.cuda.synchronize()
+                best = min(best, e0.elapsed_time(e1))
+            out[name] = round(2 * n ** 3 / (best / 1e3) / 1e12, 2)
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = old
+    del a, b
+    torch.cuda.empty_cache()
+    out["how"] = ("torch.matmul float32 8192^3 (cuBLAS), TF32 allowed / not allowed, best of "
+                  "10 / 4 launches, CUDA events, on this GPU at bench start")
+    return out
 
 
 def kernel_key(s, dtype, cand):
@@ -118,17 +175,31 @@ def sustained_run(clocks) -> bool:
             clocks["sm_mhz"] < 0.95 * clocks["sm_max_mhz"])
 
 
-def dtype_peak_tflops(dtype, peaks, sm_mhz, sustained=False):
-    """Tensor peak for the dtype: the measured BF16 figure (burst for a kernel timed in a
-    short region, sustained under the power cap), scaled by the nominal TF32/BF16 ratio for
-    TF32; FP32 FFMA from the unit count and the SM clock."""
+def peak_source(dtype, peaks, sustained, probes):
+    """Where the tensor peak of the roofline comes from, in words."""
+    if dtype == "tf32" and probes.get("tf32_tflops"):
+        return "TF32 probe (cuBLAS float32 8192^3 with TF32, measured at bench start)"
+    if dtype == "f32_ffma" and probes.get("ffma_tflops"):
+        return "FP32 FFMA probe (cuBLAS SGEMM 8192^3, measured at bench start)"
+    kind = ("sustained" if sustained else "burst") + " bf16"
+    if dtype == "tf32":
+        kind += " x nominal tf32/bf16 ratio"
+    return f"{kind} ({peaks['source']})"
+
+
+def dtype_peak_tflops(dtype, peaks, sm_mhz, sustained=False, probes=None, sm_count=152):
+    """Dense peak for the dtype.  BF16: the measured figure (burst for a kernel timed in a
+    short region, sustained under the power cap).  TF32 and FP32 FFMA: the probes taken at
+    bench start (probe_peaks); without them, TF32 = BF16 x the nominal TF32/BF16 ratio and
+    FFMA = SMs x 128 FMA/clk x 2 x the SM clock."""
+    probes = probes or {}
     bf16 = peaks["bf16_tflops_sustained"] if sustained and peaks.get("bf16_tflops_sustained") \
         else peaks["bf16_tflops"]
     if dtype == "bf16":
         return bf16
     if dtype == "tf32":
-        return bf16 * TF32_OVER_BF16
-    return 152 * 128 * 2 * sm_mhz * 1e6 / 1e12
+        return probes.get("tf32_tflops") or bf16 * TF32_OVER_BF16
+    return probes.get("ffma_tflops") or sm_count * 128 * 2 * sm_mhz * 1e6 / 1e12
 
 
 class ClockSampler:
@@ -243,7 +314,7 @@ def run_reference(args, workload, rank):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": 1000 * total / len(timings), "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": workload.key, "shapes": [[s.batch, s.M, s.N, s.K] for s in workload.shapes]},
+        "config": workload_config(workload, args),
         "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": cores, "kind": "oracle",
                          "sample": sample},
         "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
@@ -304,17 +375,17 @@ def attention_flops(B, Lq, Lk, d, causal):
     return 4 * d * B * pairs
 
 
-def run_attention(args, name, rank, world, local_rank):
+def run_attention(args, name):
     import numpy as np
     import torch
     import paper_2309_08978_gb300 as nj
     from synthetic import f32_to_bf16_bits, normal
 
     B, Lq, Lk, d, causal = ATTENTION_WORKLOADS[name]
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
     peaks = load_peaks()
-    lim = nj.nnjit_device_limits_query(local_rank)
+    lim = nj.nnjit_device_limits_query(0)
     scale = 1.0 / math.sqrt(d)
 
     def bf16(shape, seed):
@@ -359,12 +430,9 @@ def run_attention(args, name, rank, world, local_rank):
     with torch.cuda.stream(stream):
         block(args.warmup)
     torch.cuda.synchronize()
-    sampler = ClockSampler(local_rank)
+    sampler = ClockSampler(0)
     sampler.start()
     time.sleep(0.3)
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     t_wall = time.perf_counter()
@@ -375,15 +443,12 @@ def run_attention(args, name, rank, world, local_rank):
         e1.record(stream)
     stream.synchronize()
     torch.cuda.nvtx.range_pop()
-    if world > 1:
-        import torch.distributed as dist
-        dist.barrier()
     torch.cuda.synchronize()
     wall = time.perf_counter() - t_wall
     clocks = sampler.stop()
-    ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
+    ms = e0.elapsed_time(e1)
     flops = attention_flops(B, Lq, Lk, d, causal)
-    value = job_throughput(world, flops, args.steps, ms)
+    value = job_throughput(flops, args.steps, ms)
     dur_s = ms / 1e3 / args.steps
     sustained = sustained_run(clocks)
     peak_t = peaks["bf16_tflops_sustained"] if sustained and peaks.get("bf16_tflops_sustained") else peaks["bf16_tflops"]
@@ -458,11 +523,11 @@ def run_attention(args, name, rank, world, local_rank):
             e2e_step()
         f1.record(stream)
     stream.synchronize()
-    e2e_ms = max_over_ranks(f0.elapsed_time(f1), world, dev)
-    e2e_value = job_throughput(world, flops, e2e_steps, e2e_ms)
+    e2e_ms = f0.elapsed_time(f1)
+    e2e_value = job_throughput(flops, e2e_steps, e2e_ms)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if not args.no_cpu_baseline:
         from oracle.attention import attention as attention_ref
         t_used, heads = 0.0, 0
         while t_used < args.cpu_seconds and heads < B:
@@ -476,12 +541,12 @@ def run_attention(args, name, rank, world, local_rank):
                          "per-row softmax loop)"}
 
     line = {
-        "metric": ATTN_METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
+        "metric": ATTN_METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 6),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded SplitMix64 N(0,1) Q, K, V; no trained weights)",
         "config": {"workload": name, "batch_heads": B, "Lq": Lq, "Lk": Lk, "d": d, "causal": causal,
-                   "scale": scale, "parallelism": f"replicas{world}",
+                   "scale": scale, "parallelism": "single GPU",
                    "l2": f"rotates over {nsets} input/output copies (>= 3 x L2), so operands stream from HBM"},
         "roofline": roof,
         "tune": tune,
@@ -496,8 +561,7 @@ def run_attention(args, name, rank, world, local_rank):
     }
     if cpu is not None:
         line["cpu_baseline"] = cpu
-    if rank == 0:
-        print(json.dumps(line), flush=True)
+    print(json.dumps(line), flush=True)
     return 0
 
 
@@ -518,18 +582,19 @@ def custom_workload(ap, spec):
     return Workload(f"custom_{M}x{N}x{K}_{dtype}_{layout}", 5, f"custom product {spec}", (dtype,), (shape,))
 
 
-def run_ours(args, workload, rank, world, local_rank):
+def run_ours(args, workload):
     import numpy as np
     import torch
     import paper_2309_08978_gb300 as nj
     from synthetic import make_operands
 
-    torch.cuda.set_device(local_rank)
-    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(0)
+    dev = torch.device("cuda", 0)
     dtype = workload.dtypes[-1]
     peaks = load_peaks()
-    lim = nj.nnjit_device_limits_query(local_rank)
+    lim = nj.nnjit_device_limits_query(0)
     l2 = lim.l2_bytes
+    probes = probe_peaks(dtype, dev)
 
     def to_dev(x):
         if x is None:
@@ -551,7 +616,8 @@ def run_ours(args, workload, rank, world, local_rank):
     if args.cache and os.path.exists(args.cache):
         nj.nnjit_cache_load(args.cache)
     items = []
-    tune = {"budget_ms_per_shape": args.budget_ms, "shapes": []}
+    tune = {"budget_ms_total": args.tune_budget_ms, "shapes": []}
+    budget_left = args.tune_budget_ms
     free_sizes = {}
     if args.study:
         # Sec. 5.1: fix the settings a one-variable-at-a-time microbenchmark finds
@@ -575,16 +641,20 @@ def run_ours(args, workload, rank, world, local_rank):
                           "verdicts": {a: [e["value"], e["twin_value"], round(e["twin_us"], 3), e["verdict"]]
                                        for a, e in p["settings"].items()}}
                          for p in report["products"]]}
-    for s in workload.shapes:
+    for si, s in enumerate(workload.shapes):
         A, B, bias = make_operands(s, workload.index, dtype)
         bflag = nj.NNJIT_PLAN_B_CONSTANT if s.b_is_weight else 0   # weights never change
         desc = nj.make_desc(s.M, s.N, s.K, dtype, s.b_layout, batch=s.batch,
                             has_bias=s.has_bias, flags=bflag, epilogue=args.epilogue)
+        # the total budget is shared out evenly over the products still to plan
+        budget = max(0.0, budget_left / (len(workload.shapes) - si))
         t0 = time.perf_counter()
-        plan = nj.nnjit_matmul_plan_ex(desc, args.budget_ms)
+        plan = nj.nnjit_matmul_plan_ex(desc, budget)
         plan_ms = 1000 * (time.perf_counter() - t0)
+        budget_left -= plan_ms
         info = plan.describe()
-        entry = {"shape": [s.batch, s.M, s.N, s.K], "plan_ms": round(plan_ms, 2),
+        entry = {"shape": [s.batch, s.M, s.N, s.K], "budget_ms": round(budget, 1), "plan_ms": round(plan_ms, 2),
+                 "timed": len(info["timings_us"]),
                  "space_size": info["space_size"], "naive_space": info["naive_space"],
                  **({"space_size_free": free_sizes[id(s)]} if id(s) in free_sizes else {}),
                  "chosen_index": info["chosen_index"], "family": info["family"],
@@ -604,7 +674,8 @@ def run_ours(args, workload, rank, world, local_rank):
             entry.update({"sweep_ms": round(sweep_ms, 2), "best_index": best_i,
                           "best_us": round(times[best_i], 3),
                           "pick_us": round(pick, 3) if pick is not None else None,
-                          "pick_over_best": round(pick / times[best_i], 4) if pick else None})
+                          "pick_over_best": round(pick / times[best_i], 4) if pick else None,
+                          "prefix_curve": prefix_curve(times, info["space_size"])})
         tune["shapes"].append(entry)
         nsets = int(min(64, max(1, math.ceil(3 * l2 / shape_bytes(s, dtype)))))
         if s.batch > 1:
@@ -621,11 +692,16 @@ def run_ours(args, workload, rank, world, local_rank):
         items.append({"shape": s, "plan": plan, "sets": sets, "host": (A, B, bias),
                       "launches": launches, "family": info["family"]})
     tune["total_plan_ms"] = round(sum(e["plan_ms"] for e in tune["shapes"]), 2)
+    tune["within_budget"] = tune["total_plan_ms"] <= args.tune_budget_ms
     if args.cache:
         nj.nnjit_cache_save(args.cache)
     ratios = [e["pick_over_best"] for e in tune["shapes"] if e.get("pick_over_best")]
     if ratios:
         tune["max_pick_over_best"] = max(ratios)
+    curves = [e["prefix_curve"] for e in tune["shapes"] if e.get("prefix_curve")]
+    if curves:
+        # the worst product at each prefix length
+        tune["prefix_curve_max"] = {k: max(c[k] for c in curves) for k in curves[0]}
     torch.cuda.synchronize()
 
     stream = torch.cuda.Stream(device=dev)
@@ -664,12 +740,9 @@ def run_ours(args, workload, rank, world, local_rank):
     torch.cuda.synchronize()
 
     def barrier():
-        if world > 1:
-            import torch.distributed as dist
-            dist.barrier()
         torch.cuda.synchronize()
 
-    sampler = ClockSampler(local_rank)
+    sampler = ClockSampler(0)
     sampler.start()
     time.sleep(0.3)
     barrier()
@@ -687,13 +760,13 @@ def run_ours(args, workload, rank, world, local_rank):
     wall = time.perf_counter() - t_wall
     clocks = sampler.stop()
     per_item_ms = [evs[i].elapsed_time(evs[i + 1]) for i in range(len(items))]
-    total_ms = max_over_ranks(sum(per_item_ms), world, dev)
+    total_ms = sum(per_item_ms)
     for it in items:
         it["plan"].check()
 
     flops_step = sum(it["shape"].flops for it in items)
     ms_per_step = total_ms / args.steps
-    value = job_throughput(world, flops_step, args.steps, total_ms)
+    value = job_throughput(flops_step, args.steps, total_ms)
 
     # ---- roofline of the dominant kernel (largest share of the timed region)
     dom = max(range(len(items)), key=lambda i: per_item_ms[i])
@@ -702,7 +775,7 @@ def run_ours(args, workload, rank, world, local_rank):
     alg_bytes = shape_bytes(ds, dtype)
     sm_mhz = clocks["sm_mhz"] if clocks else 1900.0
     sustained = sustained_run(clocks)
-    peak_t = dtype_peak_tflops(dtype, peaks, sm_mhz, sustained)
+    peak_t = dtype_peak_tflops(dtype, peaks, sm_mhz, sustained, probes, lim.sm_count)
     ai = ds.flops / alg_bytes
     ridge = peak_t * 1e12 / (peaks["hbm_gbs"] * 1e9)
     if items[dom]["family"] == nj.NNJIT_FAMILY_GEMV or ai < ridge:
@@ -715,18 +788,19 @@ def run_ours(args, workload, rank, world, local_rank):
                 "unit": "TFLOP/s", "frac": round(ach / peak_t, 4)}
     dom_key = kernel_key(ds, dtype, items[dom]["plan"].candidate())
     roof.update({"traffic": lookup_traffic(dom_key), "kernel": dom_key,
-                 "peak_source": (("sustained" if sustained else "burst") + " bf16 " +
-                                 ("x nominal tf32/bf16 ratio " if dtype == "tf32" else "") +
-                                 f"({peaks['source']})") if roof["unit"] == "TFLOP/s"
+                 "peak_source": peak_source(dtype, peaks, sustained, probes) if roof["unit"] == "TFLOP/s"
                                 else f"copy bandwidth ({peaks['source']})",
                  "units_per_launch": f"{ds.flops} flop, {alg_bytes} algorithmic bytes"})
     per_shape = []
     for i, it in enumerate(items):
         s = it["shape"]
         d = per_item_ms[i] / 1e3 / args.steps
+        tf, gb = s.flops / d / 1e12, shape_bytes(s, dtype) / d / 1e9
+        hbm_bound = it["family"] == nj.NNJIT_FAMILY_GEMV or s.flops / shape_bytes(s, dtype) < ridge
         per_shape.append({"shape": [s.batch, s.M, s.N, s.K], "us": round(d * 1e6, 3),
-                          "tflops": round(s.flops / d / 1e12, 2),
-                          "gbs": round(shape_bytes(s, dtype) / d / 1e9, 1),
+                          "tflops": round(tf, 2), "gbs": round(gb, 1),
+                          "bound": "hbm" if hbm_bound else "tensor",
+                          "frac": round(gb / peaks["hbm_gbs"] if hbm_bound else tf / peak_t, 4),
                           "share": round(per_item_ms[i] / sum(per_item_ms), 4)})
 
     # ---- end to end through the C ABI with host buffers (copies inside the region)
@@ -755,25 +829,21 @@ def run_ours(args, workload, rank, world, local_rank):
         e1.record(stream)
     stream.synchronize()
     barrier()
-    e2e_ms = max_over_ranks(e0.elapsed_time(e1), world, dev)
-    e2e_value = job_throughput(world, flops_step, e2e_steps, e2e_ms)
+    e2e_ms = e0.elapsed_time(e1)
+    e2e_value = job_throughput(flops_step, e2e_steps, e2e_ms)
 
     cpu = None
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+    if not args.no_cpu_baseline:
         cpu = cpu_baseline(workload, dtype, seconds=args.cpu_seconds, act=args.epilogue)
 
-    l2_note = ("each product rotates over " + ", ".join(str(len(it["sets"])) for it in items) +
-               f" operand copies (>= 3 x L2 = {3 * l2 / 2**20:.0f} MiB per product), so "
-               "operands stream from HBM")
     line = {
-        "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": world,
+        "metric": METRIC, "value": round(value, 3), "unit": "TFLOP/s", "n_gpus": 1,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": dtype,
         "data": "synthetic (seeded SplitMix64, the workload's distributions; no trained weights)",
-        "config": {"workload": workload.key, "title": workload.title, "epilogue": args.epilogue,
-                   "shapes": [[s.batch, s.M, s.N, s.K, s.b_layout] for s in workload.shapes],
-                   "parallelism": f"replicas{world}", "l2": l2_note,
-                   "schedule": "per product: K launches as CUDA-graph replays, products in sequence"},
+        "config": workload_config(workload, args),
+        "operand_copies": {"per_product": [len(it["sets"]) for it in items],
+                           "l2_bytes": l2, "rule": "copies x operand bytes >= 3 x L2 per product"},
         "roofline": roof,
         "per_shape": per_shape,
         "tune": tune,
@@ -787,21 +857,23 @@ def run_ours(args, workload, rank, world, local_rank):
     }
     if cpu is not None:
         line["cpu_baseline"] = cpu
+    if probes:
+        line["peak_probes"] = probes
     for it in items:
         it["plan"].destroy()
-    if rank == 0:
-        print(json.dumps(line), flush=True)
+    print(json.dumps(line), flush=True)
     return 0
 
 
 def main(argv=None):
     ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=50000)
-    ap.add_argument("--warmup", type=int, default=500)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD)
-    ap.add_argument("--budget-ms", type=float, default=2000.0, help="tuning budget per product")
+    ap.add_argument("--tune-budget-ms", type=float, default=30000.0,
+                    help="total tuning budget of the workload, shared out over its products")
     ap.add_argument("--no-sweep", action="store_true", help="skip the exhaustive sweep")
     ap.add_argument("--study", action="store_true",
                     help="run the fixed-settings microbenchmark first and plan with its settings")
@@ -821,6 +893,15 @@ def main(argv=None):
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
     from synthetic import WORKLOADS
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    if args.impl == "ours" and (world > 1 or args.gpus > 1):
+        # the operator runs on one GPU; several GPUs would only run independent replicas
+        if rank == 0:
+            print(json.dumps({"metric": METRIC, "n_gpus": max(world, args.gpus), "unavailable":
+                              "single-GPU library: every product runs on one GPU, no multi-GPU "
+                              "path is built"}), flush=True)
+        return 0
     if args.workload in ATTENTION_WORKLOADS:
         if args.impl == "reference":
             print(json.dumps({"impl": "reference", "unavailable": "the reference arm covers the MatMul "
@@ -828,8 +909,7 @@ def main(argv=None):
             return 0
         import __graft_entry__
         __graft_entry__.build()
-        return run_attention(args, args.workload, int(os.environ.get("RANK", "0")),
-                             int(os.environ.get("WORLD_SIZE", "1")), int(os.environ.get("LOCAL_RANK", "0")))
+        return run_attention(args, args.workload)
     workload = WORKLOADS[args.workload]
     if args.shape:
         workload = custom_workload(ap, args.shape)
@@ -839,24 +919,11 @@ def main(argv=None):
         if not shapes:
             ap.error(f"--only: no product named {args.only} in {args.workload}")
         workload = dataclasses.replace(workload, shapes=shapes)
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         return run_reference(args, workload, rank)
-    if world > 1:
-        import torch
-        import torch.distributed as dist
-        torch.cuda.set_device(local_rank)
-        dist.init_process_group("nccl")
     import __graft_entry__
     __graft_entry__.build()
-    try:
-        return run_ours(args, workload, rank, world, local_rank)
-    finally:
-        if world > 1:
-            import torch.distributed as dist
-            dist.destroy_process_group()
+    return run_ours(args, workload)
 
 
 if __name__ == "__main__":

@@ -36,9 +36,43 @@ def test_attention_flops_closed_forms():
 
 
 def test_job_throughput():
-    # 2 replicas x 1e12 flop x 10 steps in 5 ms = 4000 TFLOP/s
-    assert bench.job_throughput(2, 10**12, 10, 5.0) == pytest.approx(4000.0)
-    assert bench.max_over_ranks(3.5, 1) == 3.5
+    # 1e12 flop x 10 steps in 5 ms = 2000 TFLOP/s
+    assert bench.job_throughput(10**12, 10, 5.0) == pytest.approx(2000.0)
+
+
+def test_prefix_curve():
+    # candidate 3 of 8 is the fastest: prefixes shorter than 4 see 12 us at best
+    times = {0: 20.0, 1: 12.0, 2: 15.0, 3: 10.0, 4: 11.0, 5: 30.0, 6: 10.5, 7: 40.0}
+    c = bench.prefix_curve(times, 8)
+    assert c["first_1"] == 2.0 and c["first_2"] == 1.2 and c["first_3"] == 1.2
+    assert c["first_5"] == 1.0 and c["first_10"] == 1.0
+    assert c["first_10pct"] == 2.0       # ceil(0.8) = 1 candidate
+    assert c["first_25pct"] == 1.2       # 2 candidates
+    assert c["first_50pct"] == 1.0       # 4 candidates
+    # untimed (failed) candidates are skipped
+    assert bench.prefix_curve({1: 5.0, 2: 4.0}, 3)["first_1"] is None
+
+
+def test_more_than_one_gpu_is_refused_without_touching_a_gpu(capsys, monkeypatch):
+    import json
+    monkeypatch.delenv("WORLD_SIZE", raising=False)
+    assert bench.main(["--gpus", "2"]) == 0
+    line = json.loads(capsys.readouterr().out.strip())
+    assert line["n_gpus"] == 2 and "unavailable" in line
+    monkeypatch.setenv("WORLD_SIZE", "4")
+    monkeypatch.setenv("RANK", "1")
+    assert bench.main([]) == 0
+    assert capsys.readouterr().out == ""         # only rank 0 prints
+
+
+def test_both_arms_share_the_config():
+    import argparse
+    w = WORKLOADS[bench.DEFAULT_WORKLOAD]
+    args = argparse.Namespace(epilogue="none")
+    cfg = bench.workload_config(w, args)
+    assert cfg["workload"] == "llama2_7b_prefill_m4096"
+    assert cfg["shapes"][2] == [1, 4096, 22016, 4096, "NK"]
+    assert cfg == bench.workload_config(w, args)
 
 
 def test_shape_bytes_bart_qkv():
