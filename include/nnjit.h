@@ -401,7 +401,11 @@ nnjit_status nnjit_attention(const nnjit_attention_desc* desc, const void* Q, co
 
 /* Synchronise the current device and report whether any tensor-memory attention kernel
  * since the last check gave up on a wait (NNJIT_ERR_TIMEOUT, with the wait's code in
- * nnjit_last_error); clears the record. */
+ * nnjit_last_error); clears the record.  The record is one word per device, shared by
+ * every attention call on that device (unlike a matmul plan's own watchdog word): with
+ * calls from several streams or threads, one caller's check can report, and clears,
+ * another caller's expired wait, so callers that need to tell their calls apart must
+ * serialise them with their checks (nnjit_attention_tune checks, and clears, it too). */
 nnjit_status nnjit_attention_check(void);
 
 /*

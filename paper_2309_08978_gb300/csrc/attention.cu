@@ -18,12 +18,12 @@
 // O / (row sum), 0 for a query that sees no key.
 #include <cuda_runtime.h>
 
-#include <atomic>
 
 #include <cmath>
 #include <cstdint>
 
 #include "../../include/nnjit.h"
+#include "launch.h"
 
 namespace nnjit {
 
@@ -281,15 +281,11 @@ cudaError_t launch_attention(const nnjit_attention_desc& d, const void* Q, const
     if (ctas <= 0) return cudaSuccess;
     if (ctas >= (1LL << 31)) return cudaErrorInvalidValue;
     const int smem = 5 * 64 * (int)d.d * 2;  // Q tile + two K and two V slots
-    // set once per head dimension (concurrent first calls both set it, which is harmless)
-    static std::atomic<bool> attr_set[2] = {{false}, {false}};
     const int i = d.d == 64 ? 0 : 1;
-    if (!attr_set[i]) {
-        cudaError_t e = cudaFuncSetAttribute(i == 0 ? attention_kernel<64> : attention_kernel<128>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
-        attr_set[i] = true;
-    }
+    cudaError_t e = ensure_dynamic_smem(
+        i == 0 ? reinterpret_cast<const void*>(attention_kernel<64>) : reinterpret_cast<const void*>(attention_kernel<128>),
+        smem);
+    if (e != cudaSuccess) return e;
     if (i == 0)
         attention_kernel<64><<<(unsigned)ctas, kWarps * 32, smem, stream>>>(p);
     else

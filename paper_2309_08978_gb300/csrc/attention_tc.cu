@@ -25,7 +25,6 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
-#include <atomic>
 #include <cmath>
 #include <cstdint>
 
@@ -630,26 +629,14 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     p.qblocks = qblocks;
     p.batch = (int)d.batch;
     p.scale_log2 = d.scale * 1.4426950408889634f;
-    // set once per head dimension (concurrent first calls both set it, which is harmless)
-    static std::atomic<bool> attr_set[2] = {{false}, {false}};
     const int i = d.d == 64 ? 0 : 1;
     const int smem = i == 0 ? (int)Cfg<64>::kSmem : (int)Cfg<128>::kSmem;
-    if (!attr_set[i]) {
-        cudaError_t e = cudaFuncSetAttribute(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
-        attr_set[i] = true;
-    }
+    cudaError_t e = ensure_dynamic_smem(
+        i == 0 ? reinterpret_cast<const void*>(attention_tc_kernel<64>) : reinterpret_cast<const void*>(attention_tc_kernel<128>),
+        smem);
+    if (e != cudaSuccess) return e;
     // persistent: one CTA per SM (the CTA holds all of the SM's tensor memory)
-    static std::atomic<int> sms_cached{0};
-    int sms = sms_cached.load();
-    if (sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-        if (sms <= 0) sms = 1;
-        sms_cached.store(sms);
-    }
+    const int sms = current_sm_count();
     const unsigned grid = (unsigned)std::min<long long>(ctas, sms);
     return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3(grid),
                       dim3(i == 0 ? threads_of<64>() : threads_of<128>()), (size_t)smem, stream, p);

@@ -71,6 +71,37 @@ FaultSpec read_fault() {
 namespace nnjit {
 // Record a failure detail for nnjit_last_error() from other translation units.
 void set_last_error(const char* msg) { t_last_error = msg; }
+
+namespace {
+std::mutex g_attr_mu;
+std::map<std::pair<int, const void*>, int> g_dyn_smem;  // (device, function) -> bytes set
+std::map<int, int> g_sm_count;                          // device -> SMs
+}  // namespace
+
+cudaError_t ensure_dynamic_smem(const void* func, int smem_bytes) {
+    if (smem_bytes <= 48 * 1024) return cudaSuccess;  // within the default limit
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    std::lock_guard<std::mutex> lk(g_attr_mu);
+    int& have = g_dyn_smem[{dev, func}];
+    if (have >= smem_bytes) return cudaSuccess;
+    e = cudaFuncSetAttribute(func, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
+    if (e == cudaSuccess) have = smem_bytes;
+    return e;
+}
+
+int current_sm_count() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return 1;
+    std::lock_guard<std::mutex> lk(g_attr_mu);
+    auto it = g_sm_count.find(dev);
+    if (it != g_sm_count.end()) return it->second;
+    int sms = 0;
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms <= 0) sms = 1;
+    g_sm_count[dev] = sms;
+    return sms;
+}
 }  // namespace nnjit
 
 // ------------------------------------------------------------------------ plan

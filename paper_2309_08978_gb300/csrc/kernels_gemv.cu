@@ -11,7 +11,6 @@
 
 #include <cstdint>
 #include <algorithm>
-#include <mutex>
 
 #include "epilogue.cuh"
 #include "launch.h"
@@ -258,8 +257,6 @@ const GemvKernel kGemvKernels[8] = {
     gemv_nk_kernel<4, 2>, gemv_nk_kernel<4, 4>, gemv_kn_kernel<2>,    gemv_kn_kernel<4>,
 };
 
-std::mutex g_gemv_mu;
-int g_gemv_smem[8] = {0};
 
 // Fixed-order sum of the split-K partials (s = 0, 1, ... per element; + bias, activation)
 // into C.  With vec4, four consecutive columns per thread in 16-byte accesses (N, ldc and
@@ -363,12 +360,7 @@ int grid_for(long long n, int threads) {
 cudaError_t prepare_gemv_instance(int instance, int smem_bytes) {
     if (instance < 0 || instance >= 8) return cudaErrorInvalidValue;
     if (smem_bytes <= 48 * 1024) return cudaSuccess;
-    std::lock_guard<std::mutex> lk(g_gemv_mu);
-    if (g_gemv_smem[instance] >= smem_bytes) return cudaSuccess;
-    cudaError_t e = cudaFuncSetAttribute(kGemvKernels[instance],
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
-    if (e == cudaSuccess) g_gemv_smem[instance] = smem_bytes;
-    return e;
+    return ensure_dynamic_smem(reinterpret_cast<const void*>(kGemvKernels[instance]), smem_bytes);
 }
 
 cudaError_t launch_gemv(const LaunchArgs& a) {

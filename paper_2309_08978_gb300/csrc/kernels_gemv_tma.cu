@@ -20,7 +20,6 @@
 
 #include <algorithm>
 #include <cstdint>
-#include <mutex>
 
 #include "epilogue.cuh"
 #include "launch.h"
@@ -272,8 +271,6 @@ const GemvTmaKernel kKernels[6] = {
 const int kRowsOf[6] = {8, 8, 16, 16, 32, 32};
 const int kMaxMOf[6] = {1, 8, 1, 8, 1, 8};
 
-std::mutex g_mu;
-int g_smem[6] = {0};
 
 }  // namespace
 
@@ -360,14 +357,8 @@ cudaError_t launch_gemv_tma(const LaunchArgs& a) {
         prm.pf_chunks = (int)std::min<long long>(per_cta, prm.cps);
     }
     const int smem = 128 + c.stages * (kRowsOf[i] + (int)p.M) * kRowBytes;
-    {
-        std::lock_guard<std::mutex> lk(g_mu);
-        if (g_smem[i] < smem) {
-            cudaError_t e = cudaFuncSetAttribute(kKernels[i], cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-            if (e != cudaSuccess) return e;
-            g_smem[i] = smem;
-        }
-    }
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kKernels[i]), smem);
+    if (e != cudaSuccess) return e;
     return launch_pdl(kKernels[i], dim3(grid), dim3(kThreads), smem, a.stream, prm);
 }
 

@@ -35,7 +35,6 @@
 
 #include <algorithm>
 #include <cstdint>
-#include <mutex>
 
 #include "epilogue.cuh"
 #include "launch.h"
@@ -360,8 +359,6 @@ using GemvW4Kernel = void (*)(GemvW4Params);
 const GemvW4Kernel kKernels[2] = {gemv_w4_kernel<16>, gemv_w4_kernel<32>};
 const int kRowsOf[2] = {16, 32};
 
-std::mutex g_mu;
-int g_smem[2] = {0, 0};
 
 }  // namespace
 
@@ -459,14 +456,8 @@ cudaError_t launch_gemv_w4(const LaunchArgs& a) {
     }
     const int stride = (kRowsOf[i] * (kKc / 2) + (int)p.M * kKc * 2 + kRowsOf[i] * kGroupsPerStage * 2 + 1023) / 1024 * 1024;
     const int smem = 1024 + c.stages * stride;
-    {
-        std::lock_guard<std::mutex> lk(g_mu);
-        if (g_smem[i] < smem) {
-            cudaError_t e = cudaFuncSetAttribute(kKernels[i], cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-            if (e != cudaSuccess) return e;
-            g_smem[i] = smem;
-        }
-    }
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kKernels[i]), smem);
+    if (e != cudaSuccess) return e;
     return launch_pdl(kKernels[i], dim3(grid), dim3(kThreads), smem, a.stream, prm);
 }
 

@@ -551,9 +551,6 @@ const TcKernel kTcKernels[kNumTcInstances] = {
 #undef NNJIT_TC_ROW
 #undef NNJIT_TC_KG2
 
-std::mutex g_prep_mu;
-int g_prepared_smem[kNumTcInstances] = {0};
-
 }  // namespace
 
 EncodeTiledFn get_encode_fn() {
@@ -572,12 +569,7 @@ EncodeTiledFn get_encode_fn() {
 
 cudaError_t prepare_tc_instance(int instance, int smem_bytes) {
     if (instance < 0 || instance >= kNumTcInstances) return cudaErrorInvalidValue;
-    std::lock_guard<std::mutex> lk(g_prep_mu);
-    if (g_prepared_smem[instance] >= smem_bytes) return cudaSuccess;
-    cudaError_t e = cudaFuncSetAttribute(kTcKernels[instance],
-                                         cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes);
-    if (e == cudaSuccess) g_prepared_smem[instance] = smem_bytes;
-    return e;
+    return ensure_dynamic_smem(reinterpret_cast<const void*>(kTcKernels[instance]), smem_bytes);
 }
 
 cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, const void* A,

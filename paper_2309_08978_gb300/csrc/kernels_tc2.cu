@@ -25,7 +25,6 @@
 
 #include <algorithm>
 #include <cstdint>
-#include <mutex>
 
 #include "epilogue.cuh"
 #include "launch.h"
@@ -382,8 +381,6 @@ using Tc2Kernel = void (*)(Tc2Params);
 // Instance table, indexed as instance - kTcPairFirstInstance: dtype_i (bf16, tf32).
 const Tc2Kernel kKernels[2] = {tc2_gemm_kernel<0, 256, kPairAccBuffers>, tc2_gemm_kernel<1, 256, kPairAccBuffers>};
 
-std::mutex g_mu;
-int g_smem[2] = {0, 0};
 
 }  // namespace
 
@@ -424,12 +421,8 @@ cudaError_t launch_tc_pair(const LaunchArgs& a) {
     const int stage_bytes = (128 + 128) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     {
-        std::lock_guard<std::mutex> lk(g_mu);
-        if (g_smem[i] < smem) {
-            cudaError_t e = cudaFuncSetAttribute(kKernels[i], cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-            if (e != cudaSuccess) return e;
-            g_smem[i] = smem;
-        }
+        cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kKernels[i]), smem);
+        if (e != cudaSuccess) return e;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(grid);

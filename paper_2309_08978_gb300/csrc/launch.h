@@ -68,7 +68,15 @@ cudaError_t launch_fill_scratch(void* dst, int64_t n_elems, int elem_bytes, uint
 // Write `bytes` of `buf` (evicts the L2 between timed repetitions).
 cudaError_t launch_l2_flush(void* buf, int64_t bytes, cudaStream_t s);
 
-// One-time per-process kernel attribute setup (opt-in shared memory).  Idempotent.
+// Opt-in dynamic shared memory of `func` on the current device.  The attribute belongs to
+// a device's context, so the sizes already set are recorded per (device, function):
+// cudaFuncSetAttribute runs the first time a device needs a size beyond the default or
+// beyond what was set there before.  Thread-safe; idempotent.
+cudaError_t ensure_dynamic_smem(const void* func, int smem_bytes);
+// Number of SMs of the current device (looked up once per device).
+int current_sm_count();
+
+// Kernel attribute setup of one instance on the current device (ensure_dynamic_smem).
 cudaError_t prepare_tc_instance(int instance, int smem_bytes);
 cudaError_t prepare_gemv_instance(int instance, int smem_bytes);
 
