@@ -815,22 +815,44 @@ def run_ours(args, workload):
     h2d = sum(h[0].numel() * h[0].element_size() + h[1].numel() * h[1].element_size() +
               (h[2].numel() * 4 if h[2] is not None else 0) for h in hosts)
     d2h = sum(h[3].numel() * 4 for h in hosts)
-    with torch.cuda.stream(stream):
+    plans = [it["plan"] for it in items]
+    cols = list(zip(*hosts))          # hA, hB, hbias, hC lists
+    has_bias = any(x is not None for x in cols[2])
+
+    def e2e_step():
+        nj.nnjit_matmul_run_host_seq(plans, cols[0], cols[1], cols[2] if has_bias else None, cols[3], stream)
+
+    def e2e_serial_step():
         for it, h in zip(items, hosts):
             nj.nnjit_matmul_run_host(it["plan"], *h, stream)
-    stream.synchronize()
-    barrier()
-    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        e0.record(stream)
-        for _ in range(e2e_steps):
-            for it, h in zip(items, hosts):
-                nj.nnjit_matmul_run_host(it["plan"], *h, stream)
-        e1.record(stream)
-    stream.synchronize()
-    barrier()
-    e2e_ms = e0.elapsed_time(e1)
+
+    def time_e2e(step_fn):
+        with torch.cuda.stream(stream):
+            step_fn()
+        stream.synchronize()
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(e2e_steps):
+                step_fn()
+            e1.record(stream)
+        stream.synchronize()
+        barrier()
+        return e0.elapsed_time(e1)
+
+    e2e_ms = time_e2e(e2e_step)
     e2e_value = job_throughput(flops_step, e2e_steps, e2e_ms)
+    serial_ms = time_e2e(e2e_serial_step)
+    # every product's result must have come back intact: compare the host copy with the
+    # device-side result of the same plan on the same operands
+    for it, h in zip(items, hosts):
+        A, B, bias, C = it["sets"][0]
+        it["plan"].run(A, B, bias, C, stream)
+    stream.synchronize()
+    for it, h in zip(items, hosts):
+        if not torch.equal(it["sets"][0][3].cpu(), h[3]):
+            raise RuntimeError("end-to-end result differs from the device-side result")
 
     cpu = None
     if not args.no_cpu_baseline:
@@ -849,8 +871,12 @@ def run_ours(args, workload):
         "tune": tune,
         "e2e": {"value": round(e2e_value, 3), "unit": "TFLOP/s", "h2d_bytes_per_step": h2d,
                 "d2h_bytes_per_step": d2h, "steps": e2e_steps,
-                "how": "nnjit_matmul_run_host per product: pinned host -> device copies, kernel, "
-                       "device -> host copy of C, all inside the timed region"},
+                "how": "nnjit_matmul_run_host_seq over the step's products: pinned host -> device "
+                       "copies of every A, B (and bias) on a copy-in stream, the kernels, and every "
+                       "C copied back on a copy-out stream, overlapped, all inside the timed region",
+                "serial_value": round(job_throughput(flops_step, e2e_steps, serial_ms), 3),
+                "serial_how": "nnjit_matmul_run_host per product (copies, kernel, copy back on one "
+                              "stream, one product after another); context"},
         "gpu_launches": int(args.steps * sum(it["launches"] for it in items)),
         "clocks": clocks,
         "wall_s": round(wall, 3),

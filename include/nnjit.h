@@ -347,6 +347,32 @@ nnjit_status nnjit_matmul_run_batched(nnjit_plan p, const void* A, const void* B
 nnjit_status nnjit_matmul_run_host(nnjit_plan p, const void* hA, const void* hB,
                                    const float* hbias, float* hC, void* stream);
 
+/*
+ * End-to-end form over a sequence of `count` products with HOST buffers (for instance the
+ * Linears of a layer whose weights and activations come from host memory): product i is
+ * nnjit_matmul_run_host(plans[i], hA[i], hB[i], hbias ? hbias[i] : NULL, hC[i]), but the
+ * transfers of different products overlap each other and the kernels: the inputs of the
+ * products are copied in, in order, on a host-to-device stream of the library, and each
+ * result is copied out, in order, on a device-to-host stream of the library as soon as
+ * its kernels finish, while the kernels run on `stream`.  The sequence's whole cost is
+ * about the longer of the two copy directions plus one product's exposed head and tail,
+ * instead of the sum of every copy and kernel.
+ * Ordering: nothing of the call starts before the work already queued on `stream`, and
+ * work queued on `stream` after the call starts after the last result has reached the
+ * host, so the caller synchronises `stream` before reading any hC[i].  Within the call
+ * the inputs of later products may be read before earlier results are written: no hC[i]
+ * may overlap any hA[j], hB[j] or hbias[j].  A plan may appear more than once (its
+ * staging buffers are then reused in order).  Every plan must belong to the current
+ * device and be packed (else INVALID_ARG / UNSUPPORTED, checked before anything is
+ * queued); hbias may be NULL (no bias anywhere) and hbias[i] may be NULL.  Host buffers
+ * should be page-locked.  The copy streams and events are created on the first call on a
+ * device and kept until exit; calls from several threads on one device are serialised
+ * while they queue their work.  Never synchronises.
+ */
+nnjit_status nnjit_matmul_run_host_seq(int32_t count, const nnjit_plan* plans, const void* const* hA,
+                                       const void* const* hB, const float* const* hbias,
+                                       float* const* hC, void* stream);
+
 /* Synchronise the plan's device and read its watchdog word: TIMEOUT if any kernel of
  * this plan stopped on an expired wait since the last check (the word is then reset). */
 nnjit_status nnjit_plan_check(nnjit_plan p);

@@ -244,7 +244,15 @@ std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L, c
 // Split-K partials go to a workspace unless they are reduced inside a cluster.
 bool uses_workspace(const nnjit_candidate& c) { return c.split_k > 1 && c.reduce == 0; }
 
+// A CTA-pair candidate whose tail tiles are split into K-slices (reduce 2).
+bool pair_tail_split(const nnjit_candidate& c) { return c.cluster_m == 2 && c.reduce == 2; }
+
 size_t ws_bytes_for(const Problem& p, const nnjit_candidate& c) {
+    if (pair_tail_split(c)) {
+        const int64_t pairs = std::max(1, c.grid / 2);
+        const int64_t total = p.batch * ((p.M + 255) / 256) * ((p.N + 255) / 256);
+        return (size_t)tc2_tail_ws_bytes(total % pairs, c.split_k);
+    }
     if (!uses_workspace(c)) return 0;
     return (size_t)c.split_k * (size_t)p.batch * (size_t)p.M * (size_t)p.N * sizeof(float);
 }
@@ -370,6 +378,8 @@ nnjit_status make_scratch(const Problem& p, const std::vector<nnjit_candidate>& 
     if ((err = cudaMalloc(&s->C.p, sets * r256(s->c_elems * 4))) != cudaSuccess) return cuda_fail(err, "scratch C");
     if ((err = cudaMalloc(&s->bias.p, r256((size_t)p.N * 4))) != cudaSuccess) return cuda_fail(err, "scratch bias");
     if (ws_max && (err = cudaMalloc(&s->ws.p, ws_max)) != cudaSuccess) return cuda_fail(err, "scratch workspace");
+    // tail-split candidates keep hand-off counters in the workspace: zero before first use
+    if (ws_max && (err = cudaMemset(s->ws.p, 0, ws_max)) != cudaSuccess) return cuda_fail(err, "scratch workspace");
     if ((err = launch_fill_scratch(s->A.p, (int64_t)(sets * r256(s->a_elems * e) / e), e, 1u, 0)) != cudaSuccess ||
         (err = launch_fill_scratch(s->B.p, (int64_t)(sets * r256(s->b_elems * e) / e), e, 2u, 0)) != cudaSuccess ||
         (err = launch_fill_scratch(s->bias.p, p.N, 4, 3u, 0)) != cudaSuccess)
@@ -417,7 +427,11 @@ bool time_candidate(nnjit_plan pl, const nnjit_candidate& c, const Scratch& sc, 
         int word = 0;
         cudaMemcpy(&word, pl->err, sizeof(int), cudaMemcpyDeviceToHost);
         if (fault.kind == 2 && fault.index == idx) word = 0x1FF;
-        if (word != 0) cudaMemset(pl->err, 0, sizeof(int));
+        if (word != 0) {
+            cudaMemset(pl->err, 0, sizeof(int));
+            // a stopped tail-split launch may have left hand-off counters raised
+            if (ws && pair_tail_split(c)) cudaMemset(ws, 0, ws_bytes_for(p, c));
+        }
         return word != 0;
     };
     nnjit_status st = launch(0);
@@ -489,6 +503,8 @@ nnjit_status alloc_plan_buffers(nnjit_plan pl) {
     pl->ws_bytes = ws_bytes_for(pl->p, pl->cand);
     if (pl->ws_bytes) {
         e = cudaMalloc(&pl->ws, pl->ws_bytes);
+        if (e != cudaSuccess) return cuda_fail(e, "split-K workspace");
+        e = cudaMemset(pl->ws, 0, pl->ws_bytes);  // tail-split hand-off counters start at zero
         if (e != cudaSuccess) return cuda_fail(e, "split-K workspace");
     }
     return NNJIT_OK;
@@ -1129,9 +1145,11 @@ nnjit_status nnjit_matmul_run_batched(nnjit_plan p, const void* A, const void* B
     return nnjit_matmul_run(p, A, B, nullptr, C, stream);
 }
 
-nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB,
-                                   const float* hbias, float* hC, void* stream) {
-    if (!pl) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+namespace {
+
+// Byte sizes of a packed plan's host operands and its device staging buffers (allocated on
+// first use and kept by the plan).  UNSUPPORTED for plans with padded strides.
+nnjit_status host_staging(nnjit_plan pl, size_t* a_bytes, size_t* b_bytes, size_t* c_bytes) {
     const Problem& p = pl->p;
     const int64_t b_rows = p.b_layout == NNJIT_B_KN ? p.K : p.N;
     const int64_t b_cols = p.b_layout == NNJIT_B_KN ? p.N : p.K;
@@ -1139,21 +1157,49 @@ nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB
                         p.ldc == std::max<int64_t>(p.N, 1) && p.stride_a == p.M * p.lda &&
                         p.stride_b == b_rows * p.ldb && p.stride_c == p.M * p.ldc;
     if (!packed) return fail(NNJIT_ERR_UNSUPPORTED, "run_host needs a packed plan");
-    if (p.M == 0 || p.N == 0) return NNJIT_OK;
-    if (!hC || (p.K > 0 && (!hA || !hB))) return fail(NNJIT_ERR_INVALID_ARG, "NULL host buffer");
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
     const size_t e = (size_t)p.elem_bytes();
-    const size_t a_bytes = (size_t)(p.batch * p.M * p.K) * e;
-    const size_t b_bytes = (size_t)p.b_bytes();
-    const size_t c_bytes = (size_t)(p.batch * p.M * p.N) * 4;
-    {
-        std::lock_guard<std::mutex> lk(pl->mu);
-        cudaError_t err = cudaSuccess;
-        if (!pl->hA && a_bytes && (err = cudaMalloc(&pl->hA, a_bytes)) != cudaSuccess) return cuda_fail(err, "staging A");
-        if (!pl->hB && b_bytes && (err = cudaMalloc(&pl->hB, b_bytes)) != cudaSuccess) return cuda_fail(err, "staging B");
-        if (!pl->hbias && (err = cudaMalloc(&pl->hbias, (size_t)p.N * 4)) != cudaSuccess) return cuda_fail(err, "staging bias");
-        if (!pl->hC && (err = cudaMalloc(&pl->hC, c_bytes)) != cudaSuccess) return cuda_fail(err, "staging C");
-    }
+    *a_bytes = (size_t)(p.batch * p.M * p.K) * e;
+    *b_bytes = (size_t)p.b_bytes();
+    *c_bytes = (size_t)(p.batch * p.M * p.N) * 4;
+    if (p.M == 0 || p.N == 0) return NNJIT_OK;
+    std::lock_guard<std::mutex> lk(pl->mu);
+    cudaError_t err = cudaSuccess;
+    if (!pl->hA && *a_bytes && (err = cudaMalloc(&pl->hA, *a_bytes)) != cudaSuccess) return cuda_fail(err, "staging A");
+    if (!pl->hB && *b_bytes && (err = cudaMalloc(&pl->hB, *b_bytes)) != cudaSuccess) return cuda_fail(err, "staging B");
+    if (!pl->hbias && (err = cudaMalloc(&pl->hbias, (size_t)p.N * 4)) != cudaSuccess) return cuda_fail(err, "staging bias");
+    if (!pl->hC && (err = cudaMalloc(&pl->hC, *c_bytes)) != cudaSuccess) return cuda_fail(err, "staging C");
+    return NNJIT_OK;
+}
+
+// Copy streams (host to device, device to host) and a pool of events of one device, used
+// by nnjit_matmul_run_host_seq; `mu` serialises the calls that enqueue on them.
+struct CopyLanes {
+    std::mutex mu;
+    cudaStream_t in = nullptr, out = nullptr;
+    std::vector<cudaEvent_t> events;
+};
+std::mutex g_lanes_mu;
+std::map<int, std::unique_ptr<CopyLanes>> g_lanes;
+
+CopyLanes* copy_lanes(int dev) {
+    std::lock_guard<std::mutex> lk(g_lanes_mu);
+    auto& l = g_lanes[dev];
+    if (!l) l.reset(new CopyLanes);
+    return l.get();
+}
+
+}  // namespace
+
+nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB,
+                                   const float* hbias, float* hC, void* stream) {
+    if (!pl) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+    const Problem& p = pl->p;
+    size_t a_bytes = 0, b_bytes = 0, c_bytes = 0;
+    if (!hC && p.M > 0 && p.N > 0) return fail(NNJIT_ERR_INVALID_ARG, "NULL host buffer");
+    if (p.M > 0 && p.N > 0 && p.K > 0 && (!hA || !hB)) return fail(NNJIT_ERR_INVALID_ARG, "NULL host buffer");
+    nnjit_status st = host_staging(pl, &a_bytes, &b_bytes, &c_bytes);
+    if (st != NNJIT_OK || p.M == 0 || p.N == 0) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
     cudaError_t err;
     if (a_bytes && (err = cudaMemcpyAsync(pl->hA, hA, a_bytes, cudaMemcpyHostToDevice, s)) != cudaSuccess)
         return cuda_fail(err, "copy A");
@@ -1161,10 +1207,95 @@ nnjit_status nnjit_matmul_run_host(nnjit_plan pl, const void* hA, const void* hB
         return cuda_fail(err, "copy B");
     if (hbias && (err = cudaMemcpyAsync(pl->hbias, hbias, (size_t)p.N * 4, cudaMemcpyHostToDevice, s)) != cudaSuccess)
         return cuda_fail(err, "copy bias");
-    nnjit_status st = run_impl(pl, pl->hA, pl->hB, hbias ? pl->hbias : nullptr, pl->hC, s);
+    st = run_impl(pl, pl->hA, pl->hB, hbias ? pl->hbias : nullptr, pl->hC, s);
     if (st != NNJIT_OK) return st;
     if ((err = cudaMemcpyAsync(hC, pl->hC, c_bytes, cudaMemcpyDeviceToHost, s)) != cudaSuccess)
         return cuda_fail(err, "copy C");
+    return NNJIT_OK;
+}
+
+nnjit_status nnjit_matmul_run_host_seq(int32_t count, const nnjit_plan* plans, const void* const* hA,
+                                       const void* const* hB, const float* const* hbias,
+                                       float* const* hC, void* stream) {
+    if (count < 0 || (count > 0 && (!plans || !hA || !hB || !hC)))
+        return fail(NNJIT_ERR_INVALID_ARG, "count < 0 or NULL array");
+    if (count == 0) return NNJIT_OK;
+    int dev = 0;
+    cudaError_t err = cudaGetDevice(&dev);
+    if (err != cudaSuccess) return cuda_fail(err, "current device");
+    std::vector<size_t> ab(count), bb(count), cb(count);
+    for (int32_t i = 0; i < count; ++i) {
+        nnjit_plan pl = plans[i];
+        if (!pl) return fail(NNJIT_ERR_INVALID_ARG, "plan is NULL");
+        if (pl->device != dev) return fail(NNJIT_ERR_INVALID_ARG, "every plan must belong to the current device");
+        const Problem& p = pl->p;
+        if (p.M > 0 && p.N > 0 && (!hC[i] || (p.K > 0 && (!hA[i] || !hB[i]))))
+            return fail(NNJIT_ERR_INVALID_ARG, "NULL host buffer");
+        nnjit_status st = host_staging(pl, &ab[i], &bb[i], &cb[i]);
+        if (st != NNJIT_OK) return st;
+    }
+    CopyLanes* L = copy_lanes(dev);
+    std::lock_guard<std::mutex> lk(L->mu);
+    if (!L->in && (err = cudaStreamCreateWithFlags(&L->in, cudaStreamNonBlocking)) != cudaSuccess)
+        return cuda_fail(err, "copy stream");
+    if (!L->out && (err = cudaStreamCreateWithFlags(&L->out, cudaStreamNonBlocking)) != cudaSuccess)
+        return cuda_fail(err, "copy stream");
+    // events: [0] the start, then per product: inputs landed, kernels done, result copied
+    const size_t need = 1 + 3 * (size_t)count;
+    while (L->events.size() < need) {
+        cudaEvent_t e;
+        if ((err = cudaEventCreateWithFlags(&e, cudaEventDisableTiming)) != cudaSuccess)
+            return cuda_fail(err, "event");
+        L->events.push_back(e);
+    }
+    cudaEvent_t* ev = L->events.data();
+    auto ev_in = [&](int i) { return ev[1 + 3 * i]; };
+    auto ev_k = [&](int i) { return ev[2 + 3 * i]; };
+    auto ev_out = [&](int i) { return ev[3 + 3 * i]; };
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    // both copy streams start after the work already queued on `stream`
+    if ((err = cudaEventRecord(ev[0], s)) != cudaSuccess ||
+        (err = cudaStreamWaitEvent(L->in, ev[0], 0)) != cudaSuccess ||
+        (err = cudaStreamWaitEvent(L->out, ev[0], 0)) != cudaSuccess)
+        return cuda_fail(err, "stream join");
+    for (int32_t i = 0; i < count; ++i) {
+        nnjit_plan pl = plans[i];
+        const Problem& p = pl->p;
+        // an earlier product of the same plan: its staging buffers are reused, so this
+        // product's inputs wait for its kernels and this product's kernels for its result
+        int prev = -1;
+        for (int32_t j = i - 1; j >= 0 && prev < 0; --j)
+            if (plans[j] == pl) prev = j;
+        if (prev >= 0 && (err = cudaStreamWaitEvent(L->in, ev_k(prev), 0)) != cudaSuccess)
+            return cuda_fail(err, "stream join");
+        const bool work = p.M > 0 && p.N > 0;
+        if (work && ab[i] && (err = cudaMemcpyAsync(pl->hA, hA[i], ab[i], cudaMemcpyHostToDevice, L->in)) != cudaSuccess)
+            return cuda_fail(err, "copy A");
+        if (work && bb[i] && (err = cudaMemcpyAsync(pl->hB, hB[i], bb[i], cudaMemcpyHostToDevice, L->in)) != cudaSuccess)
+            return cuda_fail(err, "copy B");
+        const float* bias_i = hbias ? hbias[i] : nullptr;
+        if (work && bias_i &&
+            (err = cudaMemcpyAsync(pl->hbias, bias_i, (size_t)p.N * 4, cudaMemcpyHostToDevice, L->in)) != cudaSuccess)
+            return cuda_fail(err, "copy bias");
+        if ((err = cudaEventRecord(ev_in(i), L->in)) != cudaSuccess ||
+            (err = cudaStreamWaitEvent(s, ev_in(i), 0)) != cudaSuccess)
+            return cuda_fail(err, "stream join");
+        if (prev >= 0 && (err = cudaStreamWaitEvent(s, ev_out(prev), 0)) != cudaSuccess)
+            return cuda_fail(err, "stream join");
+        if (work) {
+            nnjit_status st = run_impl(pl, pl->hA, pl->hB, bias_i ? pl->hbias : nullptr, pl->hC, s);
+            if (st != NNJIT_OK) return st;
+        }
+        if ((err = cudaEventRecord(ev_k(i), s)) != cudaSuccess ||
+            (err = cudaStreamWaitEvent(L->out, ev_k(i), 0)) != cudaSuccess)
+            return cuda_fail(err, "stream join");
+        if (work && (err = cudaMemcpyAsync(hC[i], pl->hC, cb[i], cudaMemcpyDeviceToHost, L->out)) != cudaSuccess)
+            return cuda_fail(err, "copy C");
+        if ((err = cudaEventRecord(ev_out(i), L->out)) != cudaSuccess) return cuda_fail(err, "event");
+    }
+    // later work on `stream` starts after the last result has reached the host (the copy-out
+    // stream runs in order, so its last event covers every earlier copy)
+    if ((err = cudaStreamWaitEvent(s, ev_out(count - 1), 0)) != cudaSuccess) return cuda_fail(err, "stream join");
     return NNJIT_OK;
 }
 
@@ -1176,7 +1307,11 @@ nnjit_status nnjit_plan_check(nnjit_plan p) {
     cudaError_t e = cudaDeviceSynchronize();
     int word = 0;
     if (e == cudaSuccess) e = cudaMemcpy(&word, p->err, sizeof(int), cudaMemcpyDeviceToHost);
-    if (e == cudaSuccess && word != 0) cudaMemset(p->err, 0, sizeof(int));
+    if (e == cudaSuccess && word != 0) {
+        cudaMemset(p->err, 0, sizeof(int));
+        // a stopped tail-split launch may have left hand-off counters raised
+        if (p->ws && p->ws_bytes) cudaMemset(p->ws, 0, p->ws_bytes);
+    }
     if (cur != p->device) cudaSetDevice(cur);
     if (e != cudaSuccess) return cuda_fail(e, "plan check");
     if (word != 0) {

@@ -130,6 +130,7 @@ def load_library(path: str = LIB_PATH):
             "nnjit_matmul_run": [vp, vp, vp, vp, vp, vp],
             "nnjit_matmul_run_batched": [vp, vp, vp, vp, vp],
             "nnjit_matmul_run_host": [vp, vp, vp, vp, vp, vp],
+            "nnjit_matmul_run_host_seq": [i32, P(vp), P(vp), P(vp), P(vp), P(vp), vp],
             "nnjit_plan_check": [vp],
             "nnjit_plan_describe": [vp, ctypes.c_char_p, ctypes.c_size_t, P(ctypes.c_size_t)],
             "nnjit_plan_candidate": [vp, P(nnjit_candidate)],
@@ -327,6 +328,21 @@ def nnjit_matmul_run_host(plan: Plan, hA, hB, hbias, hC, stream=None):
     _check(load_library().nnjit_matmul_run_host(plan.handle, _ptr(hA), _ptr(hB), _ptr(hbias),
                                                 _ptr(hC), _stream(stream)),
            "nnjit_matmul_run_host")
+
+
+def nnjit_matmul_run_host_seq(plans, hAs, hBs, hbiases, hCs, stream=None):
+    """Sequence of products from host buffers with overlapped transfers (include/nnjit.h)."""
+    n = len(plans)
+    if not (len(hAs) == len(hBs) == len(hCs) == n) or (hbiases is not None and len(hbiases) != n):
+        raise ValueError("plans and buffer lists must have the same length")
+    vp = ctypes.c_void_p
+    arr_p = (vp * max(1, n))(*[p.handle for p in plans])
+    arr_a = (vp * max(1, n))(*[_ptr(x) for x in hAs])
+    arr_b = (vp * max(1, n))(*[_ptr(x) for x in hBs])
+    arr_c = (vp * max(1, n))(*[_ptr(x) for x in hCs])
+    arr_bias = None if hbiases is None else (vp * max(1, n))(*[_ptr(x) for x in hbiases])
+    _check(load_library().nnjit_matmul_run_host_seq(n, arr_p, arr_a, arr_b, arr_bias, arr_c, _stream(stream)),
+           "nnjit_matmul_run_host_seq")
 
 
 def nnjit_plan_check(plan: Plan):

@@ -160,3 +160,15 @@ def test_attention_refusals_without_a_gpu(lib):
     assert f(desc, p, None, p, p, None) == nj.NNJIT_ERR_INVALID_ARG
     assert f(None, p, p, p, p, None) == nj.NNJIT_ERR_INVALID_ARG
     assert f(nj.nnjit_attention_desc(2, 0, 5, 128, 1, 1.0), None, None, None, None, None) == nj.NNJIT_OK
+
+
+def test_run_host_seq_refusals_without_a_gpu(lib):
+    """nnjit_matmul_run_host_seq checks its arrays before any CUDA call: a negative count or
+    NULL arrays are INVALID_ARG, and count 0 is a no-op."""
+    import ctypes
+    import paper_2309_08978_gb300 as nj
+    f = nj.load_library().nnjit_matmul_run_host_seq
+    assert f(0, None, None, None, None, None, None) == nj.NNJIT_OK
+    assert f(-1, None, None, None, None, None, None) == nj.NNJIT_ERR_INVALID_ARG
+    assert f(2, None, None, None, None, None, None) == nj.NNJIT_ERR_INVALID_ARG
+    assert "NULL" in nj.nnjit_last_error()

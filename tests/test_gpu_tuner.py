@@ -114,6 +114,52 @@ def test_run_host_end_to_end():
         compare(hC.numpy(), A, B, bias, "KN", "tf32")
 
 
+def test_run_host_seq_overlapped_sequence():
+    """A sequence of products from host buffers with overlapped transfers: a tensor-core
+    product with bias, a GEMV, a batched product and the first plan again with new
+    inputs (its staging buffers are reused in order), all bit exact against the oracle on
+    integer inputs; then twice in a row to check that a second call waits for the first."""
+    import torch
+
+    def pinned(x):
+        if x is None:
+            return None
+        if x.dtype == np.uint16:
+            return torch.from_numpy(x.view(np.int16)).view(torch.bfloat16).pin_memory()
+        return torch.from_numpy(x).pin_memory()
+
+    specs = [(Shape("a", 300, 520, 264, 1, "NK", True), 41),
+             (Shape("b", 1, 1000, 512, 1, "NK", False), 42),
+             (Shape("c", 130, 72, 64, 3, "KN", False), 43),
+             (Shape("a", 300, 520, 264, 1, "NK", True), 44)]
+    plans = {}
+    items = []
+    for shape, seed in specs:
+        key = (shape.M, shape.N, shape.K, shape.batch, shape.b_layout)
+        if key not in plans:
+            desc = nj.make_desc(shape.M, shape.N, shape.K, "bf16", shape.b_layout, batch=shape.batch,
+                                has_bias=shape.has_bias, flags=nj.NNJIT_PLAN_NO_CACHE)
+            plans[key] = nj.nnjit_matmul_plan_ex(desc, 20.0)
+        A, B, bias = make_operands(shape, seed, "bf16", ints=True)
+        out = (shape.batch, shape.M, shape.N) if shape.batch > 1 else (shape.M, shape.N)
+        hC = torch.full(out, float("nan"), dtype=torch.float32).pin_memory()
+        items.append((plans[key], shape, A, B, bias, pinned(A), pinned(B), pinned(bias), hC))
+    try:
+        for _ in range(2):
+            for it in items:
+                it[8].fill_(float("nan"))
+            nj.nnjit_matmul_run_host_seq([it[0] for it in items], [it[5] for it in items],
+                                         [it[6] for it in items], [it[7] for it in items],
+                                         [it[8] for it in items])
+            torch.cuda.synchronize()
+            for plan, shape, A, B, bias, *_, hC in items:
+                plan.check()
+                compare(hC.numpy(), A, B, bias, shape.b_layout, "bf16", exact=True)
+    finally:
+        for p in plans.values():
+            p.destroy()
+
+
 def test_invalid_run_arguments():
     import torch
     with nj.nnjit_matmul_plan_ex(nj.make_desc(256, 256, 256, "bf16", "NK"), 0.0) as plan:
