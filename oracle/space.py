@@ -308,6 +308,17 @@ def _tc(p, lim):
                          predicted_cost=waves * t_kb * num_kb,
                          instance=TC_PAIR_FIRST + (0 if p.dtype == BF16 else 1))
                 out.append(c)
+                # tail split: the tiles past the last whole wave in `sl` K-slices each
+                full_waves, tail = pairs // live, pairs % live
+                for sl in (2, 4):
+                    if full_waves < 1 or tail == 0 or tail * sl > live or num_kb < 4 * sl:
+                        continue
+                    t = dict(c)
+                    t.update(split_k=sl, reduce=2,
+                             wave_eff_ppm=pairs * 1000000 * sl // (live * (full_waves * sl + 1)),
+                             predicted_cost=full_waves * t_kb * num_kb + t_kb * cdiv(num_kb, sl) +
+                             sl * (128 * 256 * 4 // FEED_BYTES_PER_CLK))
+                    out.append(t)
     return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2 * 2
 
 

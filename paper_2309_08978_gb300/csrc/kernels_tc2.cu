@@ -20,6 +20,19 @@
 //               the accumulator on the even CTA's "tmem_empty[acc]" (8 arrivals).
 // Every wait is bounded; on expiry the error word is set and the roles fall through to
 // the teardown (the producers wait, bounded, for their ring slots to drain first).
+//
+// Tail split (candidate reduce = 2, split_k = s): when the pair tiles do not fill a whole
+// number of waves of the resident pairs, the `tail` tiles of the last partial wave are
+// cut into s slices of their k-blocks, so that the last wave runs tail * s shorter work
+// items on up to all pairs instead of `tail` whole tiles on a few.  Work items are the
+// whole tiles first, then every tail tile's slices 0 .. s-2, then their last slices.  A
+// slice other than the last writes its raw accumulator to the plan's workspace and adds
+// one to a counter per (tail tile, CTA, epilogue warp) with release semantics; the last
+// slice of the tile waits (bounded) for s - 1 counts, adds the partials to its own
+// accumulator in slice order (so repeated runs give identical bits), applies bias,
+// activation and residual, stores C and resets its counter for the next launch.  Each
+// persistent pair takes items in increasing order and a last slice waits only for items
+// of lower index, which run on other pairs in the same final round, so every wait ends.
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -44,6 +57,7 @@ constexpr int kErrMmaTmemEmpty = 0x142;
 constexpr int kErrMmaFull = 0x143;
 constexpr int kErrEpiTmemFull = 0x144;
 constexpr int kErrDrain = 0x145;
+constexpr int kErrTailWait = 0x146;
 
 struct Tc2Params {
     CUtensorMap tmap_a;  // A: dims {K, M, batch}, box {BK, 128, 1}
@@ -58,10 +72,20 @@ struct Tc2Params {
     long long ldc, stride_c;
     int num_kb, tiles2_m, tiles_n, total, stages, raster;
     int act;  // nnjit_epilogue
+    // tail split: items = full + tail * slices (slices = 1: every item a whole tile)
+    int full, tail, slices, items;
+    float* part;    // [tail][slices - 1][2 CTAs][BN / 32 chunks][128 rows][32] partial sums
+    unsigned* cnt;  // [tail][2 CTAs][4 epilogue warps] hand-off counters, zero between launches
 };
 
 struct PairTile {
     int b, tm2, tn;
+};
+
+// One work item: a whole pair tile (slice = -1) or slice `slice` of tail tile `j`,
+// covering k-blocks [kb0, kb1).
+struct PairItem {
+    int tile, slice, j, kb0, kb1;
 };
 
 __device__ __forceinline__ PairTile decode(int t, const Tc2Params& p) {
@@ -77,6 +101,21 @@ __device__ __forceinline__ PairTile decode(int t, const Tc2Params& p) {
         c.tm2 = r / p.tiles_n;
     }
     return c;
+}
+
+__device__ __forceinline__ PairItem decode_item(int t, const Tc2Params& p) {
+    PairItem it;
+    if (t < p.full) {
+        it.tile = t; it.slice = -1; it.j = 0; it.kb0 = 0; it.kb1 = p.num_kb;
+        return it;
+    }
+    const int r = t - p.full;
+    it.slice = r / p.tail;
+    it.j = r % p.tail;
+    it.tile = p.full + it.j;
+    it.kb0 = (int)((long long)it.slice * p.num_kb / p.slices);
+    it.kb1 = (int)((long long)(it.slice + 1) * p.num_kb / p.slices);
+    return it;
 }
 
 // NB: accumulator buffers in TMEM (2: the epilogue of one tile overlaps the mainloop of
@@ -137,9 +176,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         ptx::prefetch_tmap(&p.tmap_a);
         ptx::prefetch_tmap(&p.tmap_b);
         if (p.tma_store) ptx::prefetch_tmap(&p.tmap_c);
-        if (t_begin < p.total) {
-            const PairTile tc = decode(t_begin, p);
-            for (int kb = 0; kb < p.num_kb && kb < S; ++kb) {
+        if (t_begin < p.items) {
+            const PairItem it = decode_item(t_begin, p);
+            const PairTile tc = decode(it.tile, p);
+            for (int kb = it.kb0; kb < it.kb1 && kb < it.kb0 + S; ++kb) {
                 ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm2 * 256 + row_off, tc.b);
                 ptx::tma_prefetch_l2_3d(&p.tmap_b, kb * BK, tc.tn * BN + bcol_off, tc.b);
             }
@@ -160,13 +200,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
     // With a constant B the first ring's B halves are requested before the dependency
     // wait; the even CTA arms those slots with the bytes of both CTAs' A and B.
     int b_preloaded = 0;
-    if (p.b_const && warp == 0 && t_begin < p.total) {
-        const PairTile tc = decode(t_begin, p);
-        b_preloaded = min(S, p.num_kb);
+    if (p.b_const && warp == 0 && t_begin < p.items) {
+        const PairItem it = decode_item(t_begin, p);
+        const PairTile tc = decode(it.tile, p);
+        b_preloaded = min(S, it.kb1 - it.kb0);
         if (lane == 0) {
             for (int i = 0; i < b_preloaded; ++i) {
                 if (leader) ptx::mbar_arrive_expect_tx(full_bar(i), 2 * kStageBytes);
-                ptx::tma_load_3d_pair(smem_base + i * kStageBytes + kABytes, &p.tmap_b, i * BK,
+                ptx::tma_load_3d_pair(smem_base + i * kStageBytes + kABytes, &p.tmap_b, (it.kb0 + i) * BK,
                                       tc.tn * BN + bcol_off, tc.b, leader_full(i));
             }
         }
@@ -181,9 +222,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         uint32_t phase = 0;
         bool ok = true;
         int issued = 0;
-        for (int t = t_begin; ok && t < p.total; t += t_step) {
-            const PairTile tc = decode(t, p);
-            for (int kb = 0; kb < p.num_kb; ++kb) {
+        for (int t = t_begin; ok && t < p.items; t += t_step) {
+            const PairItem it = decode_item(t, p);
+            const PairTile tc = decode(it.tile, p);
+            for (int kb = it.kb0; kb < it.kb1; ++kb) {
                 if (!ptx::mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, p.err, kErrProducerEmpty)) {
                     ok = false;
                     break;
@@ -223,7 +265,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
             bool ok = true;
             const uint64_t a_desc0 = ptx::smem_desc(smem_base, 16, 1024);
             const uint64_t b_desc0 = ptx::smem_desc(smem_base + kABytes, 16, 1024);
-            for (int t = t_begin; ok && t < p.total; t += t_step, ++iter) {
+            for (int t = t_begin; ok && t < p.items; t += t_step, ++iter) {
+                const PairItem it = decode_item(t, p);
                 const uint32_t acc = NB == 2 ? (iter & 1u) : 0u;
                 const uint32_t acc_phase = NB == 2 ? ((iter >> 1) & 1u) : (iter & 1u);
                 if (!ptx::mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty)) {
@@ -232,7 +275,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 }
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem_base + acc * BN;
-                for (int kb = 0; kb < p.num_kb; ++kb) {
+                for (int kb = it.kb0; kb < it.kb1; ++kb) {
                     if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull)) {
                         ok = false;
                         break;
@@ -243,7 +286,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                         const uint64_t ad = a_desc0 + off, bd = b_desc0 + off;
 #pragma unroll
                         for (int kk = 0; kk < kKSteps; ++kk)
-                            ptx::mma_pair<kKind>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                            ptx::mma_pair<kKind>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdesc, (kb > it.kb0 || kk > 0) ? 1u : 0u);
                         ptx::tc_commit_pair(empty_bar(stage), 0x3);  // frees the slot in both CTAs
                     }
                     __syncwarp();
@@ -272,24 +315,65 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         uint32_t iter = 0;
         const uint32_t leader_tempty0 = ptx::map_shared_rank(tempty_bar(0), 0);
         const uint32_t leader_tempty1 = ptx::map_shared_rank(tempty_bar(1), 0);
-        for (int t = t_begin; t < p.total; t += t_step, ++iter) {
-            const PairTile tc = decode(t, p);
+        constexpr int kChunks = BN / 32;
+        static_assert(kChunks % 2 == 0, "chunks are processed in pairs");
+        // this thread's 32 floats of chunk c of slice k of tail tile j in the workspace
+        auto part_chunk = [&](int j, int k, int c) {
+            const long long idx = ((((long long)j * (p.slices - 1) + k) * 2 + rank) * kChunks + c) * 128 + q * 32 + lane;
+            return reinterpret_cast<float4*>(p.part + idx * 32);
+        };
+        for (int t = t_begin; t < p.items; t += t_step, ++iter) {
+            const PairItem it = decode_item(t, p);
+            const PairTile tc = decode(it.tile, p);
+            // a slice other than the last hands its sum over; the last slice collects them
+            const bool partial = it.slice >= 0 && it.slice < p.slices - 1;
+            const bool last = it.slice >= 0 && it.slice == p.slices - 1;
+            unsigned* cnt = p.cnt + ((it.j * 2 + (int)rank) * 4 + q);
             const uint32_t acc = NB == 2 ? (iter & 1u) : 0u;
             const uint32_t acc_phase = NB == 2 ? ((iter >> 1) & 1u) : (iter & 1u);
             if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
             ptx::tc_fence_after();
+            if (last) {
+                bool ok = true;
+                if (lane == 0) ok = ptx::wait_counter(cnt, (uint32_t)(p.slices - 1), abort_flag, p.err, kErrTailWait);
+                if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
+                (void)ptx::ld_acquire_gpu(cnt);  // every lane orders its partial reads after the count
+            }
             const int row_base = tc.tm2 * 256 + row_off + q * 32;
             const int row = row_base + lane;
             const float* bias = p.bias;
             float* dst_row = p.C + (long long)tc.b * p.stride_c + (long long)row * p.ldc;
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN;
-            constexpr int kChunks = BN / 32;
-            static_assert(kChunks % 2 == 0, "chunks are processed in pairs");
             auto emit = [&](const uint32_t (&r)[32], float bl, int c) {
                 const int col0 = tc.tn * BN + c * 32;
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
+                if (partial) {  // raw sum of this slice's k-blocks to the workspace
+                    float4* dst = part_chunk(it.j, it.slice, c);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                    return;
+                }
+                if (last) {  // (partial 0 + partial 1 + ... + partial s-2) + own sum
+                    float w[32];
+                    const float4* src = part_chunk(it.j, 0, c);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        const float4 x = __ldcg(src + j);
+                        w[4 * j] = x.x; w[4 * j + 1] = x.y; w[4 * j + 2] = x.z; w[4 * j + 3] = x.w;
+                    }
+                    for (int k = 1; k < p.slices - 1; ++k) {
+                        src = part_chunk(it.j, k, c);
+#pragma unroll
+                        for (int j = 0; j < 8; ++j) {
+                            const float4 x = __ldcg(src + j);
+                            w[4 * j] += x.x; w[4 * j + 1] += x.y; w[4 * j + 2] += x.z; w[4 * j + 3] += x.w;
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = w[j] + v[j];
+                }
                 if (bias) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
@@ -364,6 +448,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 emit(rb, bb, c + 1);
                 if (c + 2 < kChunks) ptx::tmem_wait_ld(ra);
             }
+            if (partial) {  // publish this warp's rows of the slice
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) ptx::red_release_add_gpu(cnt, 1u);
+            }
+            if (last) {  // every partial has been read: ready for the next launch
+                __syncwarp();
+                if (lane == 0) *cnt = 0u;
+            }
         }
         if (p.tma_store && lane == 0) ptx::bulk_wait_all_read();
         __syncwarp();
@@ -390,8 +483,12 @@ cudaError_t launch_tc_pair(const LaunchArgs& a) {
     const int i = c.instance - kTcPairFirstInstance;
     const int di = p.dtype == NNJIT_BF16 ? 0 : 1;
     if (i != di || !a.tmap_a || !a.tmap_b || p.b_layout != NNJIT_B_NK) return cudaErrorInvalidValue;
-    if (c.bm != 256 || c.bn != 256 || c.cluster_m != 2 || c.split_k != 1 || c.reduce != 0 ||
-        c.stages < 2 || c.stages > kMaxStages || c.bk != 128 / p.elem_bytes())
+    if (c.bm != 256 || c.bn != 256 || c.cluster_m != 2 || c.stages < 2 || c.stages > kMaxStages ||
+        c.bk != 128 / p.elem_bytes())
+        return cudaErrorInvalidValue;
+    // unsplit (split_k 1, reduce 0) or tail split (reduce 2, split_k = slices of a tail tile)
+    const bool tail_split = c.reduce == 2;
+    if (tail_split ? (c.split_k < 2 || c.split_k > 8 || !a.ws) : (c.split_k != 1 || c.reduce != 0))
         return cudaErrorInvalidValue;
     Tc2Params prm;
     prm.tmap_a = *a.tmap_a;
@@ -418,6 +515,26 @@ cudaError_t launch_tc_pair(const LaunchArgs& a) {
     prm.stages = c.stages;
     prm.raster = c.raster;
     const int grid = (int)std::min<long long>(2 * total, c.grid);
+    prm.full = prm.total;
+    prm.tail = 0;
+    prm.slices = 1;
+    prm.part = nullptr;
+    prm.cnt = nullptr;
+    if (tail_split) {
+        // the tiles past the last whole wave of `pairs` resident pairs, each in split_k slices
+        const int pairs = grid / 2;
+        const int tail = prm.total % pairs;
+        if (prm.total <= pairs || tail == 0 || (long long)tail * c.split_k > pairs ||
+            prm.num_kb < 4 * c.split_k)
+            return cudaErrorInvalidValue;
+        prm.tail = tail;
+        prm.full = prm.total - tail;
+        prm.slices = c.split_k;
+        // workspace: the counters, then the partial sums (tc2_tail_ws_bytes)
+        prm.cnt = reinterpret_cast<unsigned*>(a.ws);
+        prm.part = a.ws + tc2_tail_cnt_floats(tail);
+    }
+    prm.items = prm.full + prm.tail * prm.slices;
     const int stage_bytes = (128 + 128) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     {

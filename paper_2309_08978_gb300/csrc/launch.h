@@ -51,8 +51,17 @@ struct LaunchArgs {
 cudaError_t launch_ffma(const LaunchArgs& a);
 cudaError_t launch_gemv(const LaunchArgs& a);
 cudaError_t launch_tc(const LaunchArgs& a);
-// CTA-pair (cta_group::2) tensor-core instances kTcPairFirstInstance.. (bf16, tf32).
+// CTA-pair (cta_group::2) tensor-core instances kTcPairFirstInstance.. (bf16, tf32).  A
+// tail-split candidate (reduce 2) takes its counters and partial sums from LaunchArgs::ws.
 cudaError_t launch_tc_pair(const LaunchArgs& a);
+// Workspace of a tail-split pair candidate with `tail` tiles of `slices` slices: per tail
+// tile 2 CTAs x 4 warps of counters (padded to 256 bytes in all), then (slices - 1) partial
+// 256 x 256 f32 tiles.  The counters must be zero before the first launch; every launch
+// that completes leaves them zero.
+inline int64_t tc2_tail_cnt_floats(int64_t tail) { return (tail * 8 + 63) / 64 * 64; }
+inline int64_t tc2_tail_ws_bytes(int64_t tail, int64_t slices) {
+    return (tc2_tail_cnt_floats(tail) + tail * (slices - 1) * 256 * 256) * 4;
+}
 
 // C[b,m,n] = sum_{s < split} ws[s][b][m][n] (+ bias[n]), s ascending.
 cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, const float* bias,

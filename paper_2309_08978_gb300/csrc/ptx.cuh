@@ -89,6 +89,43 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatil
     }
 }
 
+// ------------------------------------------------------------ global-memory hand-off
+// A 32-bit counter in global memory that CTAs of one grid use to hand data to each other:
+// producers add with release semantics after writing their data, the consumer waits with
+// acquire loads until the count it needs is reached (both at GPU scope).
+__device__ __forceinline__ void red_release_add_gpu(unsigned* p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const unsigned* p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Wait until *p >= target.  Bounded like mbar_wait: gives up if *abort_flag becomes
+// non-zero or after limit_ns, raising the abort flag and recording `code`.  Only the
+// waiting thread gets acquire ordering; other threads that read the handed-over data
+// must follow with their own ld_acquire_gpu of the counter.
+__device__ __forceinline__ bool wait_counter(const unsigned* p, uint32_t target, volatile int* abort_flag,
+                                             int* err_word, int code, uint64_t limit_ns = kWaitLimitNs) {
+    uint64_t t0 = 0;
+    for (uint32_t i = 1;; ++i) {
+        if (ld_acquire_gpu(p) >= target) return true;
+        if ((i & 255u) == 0) {
+            if (*abort_flag) return false;
+            const uint64_t now = globaltimer();
+            if (t0 == 0) {
+                t0 = now;
+            } else if (now - t0 > limit_ns) {
+                *abort_flag = 1;
+                if (err_word) atomicCAS(err_word, 0, code);
+                return false;
+            }
+        }
+    }
+}
+
 // ----------------------------------------------------------------------------- TMA
 __device__ __forceinline__ void prefetch_tmap(const void* tmap) {
     asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");

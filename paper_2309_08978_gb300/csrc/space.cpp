@@ -171,6 +171,21 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 c.predicted_cost = waves * t_kb * num_kb;
                 c.instance = kTcPairFirstInstance + (p.dtype == NNJIT_BF16 ? 0 : 1);
                 v.push_back(c);
+                // Tail split: the tiles past the last whole wave are cut into `sl` slices of
+                // their k-blocks, so the last wave takes 1/sl of a tile plus the hand-off of
+                // the partial sums (one 128-row x 256-column f32 partial per CTA written or
+                // read per slice, at the per-SM feed rate).
+                const int64_t full_waves = pairs / live, tail = pairs % live;
+                for (int sl : {2, 4}) {
+                    if (full_waves < 1 || tail == 0 || tail * sl > live || num_kb < 4LL * sl) continue;
+                    nnjit_candidate t = c;
+                    t.split_k = sl;
+                    t.reduce = 2;
+                    t.wave_eff_ppm = (int32_t)(pairs * 1000000 * sl / (live * (full_waves * sl + 1)));
+                    t.predicted_cost = full_waves * t_kb * num_kb + t_kb * ceil_div(num_kb, sl) +
+                                       sl * (128LL * 256 * 4 / MC::kFeedBytesPerClk);
+                    v.push_back(t);
+                }
             }
         }
     }

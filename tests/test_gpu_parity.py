@@ -520,3 +520,58 @@ def test_residual_edge_cases():
         with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
             C = run_plan(plan, x, blob, bias, M, N, C=torch.from_numpy(R.copy()).cuda())
         assert np.array_equal(C, want), i
+
+
+TAIL_CASES = [("bf16", 4096, 2560, 1024, "NK"), ("tf32", 4096, 2560, 512, "NK"),
+              ("bf16", 4200, 2300, 1040, "NK")]
+
+
+@pytest.mark.parametrize("case", TAIL_CASES, ids=_ids)
+def test_pair_tail_split_exact_repeated_and_in_graphs(case):
+    """CTA-pair tiles whose last partial wave is split into K-slices (reduce 2): the last
+    slice of each tail tile adds the other slices' partial sums from the workspace after
+    a counter hand-off, and resets the counters for the next launch.  Every tail-split
+    candidate must be bit exact on integer inputs (with bias, and with ReLU), on three
+    launches in a row and on two replays of a CUDA graph of two launches, ragged M and N
+    included (4200 x 2300: the last pair tile is partly past both edges)."""
+    import torch
+    dtype, M, N, K, layout = case
+    shape = Shape("t", M, N, K, 1, layout, True)
+    A, B, bias = make_operands(shape, 51, dtype, ints=True)
+    dA, dB, dbias = (torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).view(torch.bfloat16).cuda()
+                     if x.dtype == np.uint16 else torch.from_numpy(x).cuda() for x in (A, B, bias))
+    lim = nj.nnjit_device_limits_query(0)
+    for act in ("none", "relu"):
+        desc = nj.make_desc(M, N, K, dtype, layout, has_bias=True, epilogue=act, flags=nj.NNJIT_PLAN_NO_CACHE)
+        cands, _ = nj.nnjit_space_enumerate(desc, lim)
+        tails = [i for i, c in enumerate(cands) if c["reduce"] == 2]
+        assert tails, "expected tail-split candidates"
+        _, ref32 = oracle.matmul(A, B, bias, layout_code(layout), act=act)
+        for i in tails:
+            with nj.nnjit_matmul_plan_candidate(desc, i) as plan:
+                for rep in range(3):
+                    C = torch.full((M, N), float("nan"), dtype=torch.float32, device="cuda")
+                    plan.run(dA, dB, dbias, C)
+                    torch.cuda.synchronize()
+                    plan.check()
+                    got = C.cpu().numpy()
+                    bad = np.argwhere(got != ref32)
+                    assert bad.size == 0, f"candidate {i} {cands[i]} launch {rep}: {len(bad)} mismatches"
+                st = torch.cuda.Stream()
+                C1 = torch.empty((M, N), dtype=torch.float32, device="cuda")
+                C2 = torch.empty((M, N), dtype=torch.float32, device="cuda")
+                plan.run(dA, dB, dbias, C1, st)   # tensor maps cached outside the capture
+                plan.run(dA, dB, dbias, C2, st)
+                st.synchronize()
+                g = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(g, stream=st):
+                    plan.run(dA, dB, dbias, C1, st)
+                    plan.run(dA, dB, dbias, C2, st)
+                for rep in range(2):
+                    C1.fill_(float("nan"))
+                    C2.fill_(float("nan"))
+                    g.replay()
+                    torch.cuda.synchronize()
+                    plan.check()
+                    for Cx in (C1, C2):
+                        assert np.array_equal(Cx.cpu().numpy(), ref32), f"candidate {i} graph replay {rep}"
