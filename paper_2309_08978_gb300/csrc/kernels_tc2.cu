@@ -74,7 +74,7 @@ struct Tc2Params {
     int act;  // nnjit_epilogue
     // tail split: items = full + tail * slices (slices = 1: every item a whole tile)
     int full, tail, slices, items;
-    float* part;    // [tail][slices - 1][2 CTAs][BN / 32 chunks][128 rows][32] partial sums
+    float* part;    // [tail][slices - 1][2 CTAs][BN / 32 chunks][4 warps][8][32 lanes] float4 partials
     unsigned* cnt;  // [tail][2 CTAs][4 epilogue warps] hand-off counters, zero between launches
 };
 
@@ -317,10 +317,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         const uint32_t leader_tempty1 = ptx::map_shared_rank(tempty_bar(1), 0);
         constexpr int kChunks = BN / 32;
         static_assert(kChunks % 2 == 0, "chunks are processed in pairs");
-        // this thread's 32 floats of chunk c of slice k of tail tile j in the workspace
+        // This warp's block of chunk c of slice k of tail tile j in the workspace: 8 x 32
+        // float4, element [i][lane] = columns 4i .. 4i + 3 of the lane's row, so that each
+        // warp-wide access covers 512 contiguous bytes.
         auto part_chunk = [&](int j, int k, int c) {
-            const long long idx = ((((long long)j * (p.slices - 1) + k) * 2 + rank) * kChunks + c) * 128 + q * 32 + lane;
-            return reinterpret_cast<float4*>(p.part + idx * 32);
+            const long long blk = (((((long long)j * (p.slices - 1) + k) * 2 + rank) * kChunks + c) * 4) + q;
+            return reinterpret_cast<float4*>(p.part) + blk * 256 + lane;
         };
         for (int t = t_begin; t < p.items; t += t_step, ++iter) {
             const PairItem it = decode_item(t, p);
@@ -352,7 +354,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 if (partial) {  // raw sum of this slice's k-blocks to the workspace
                     float4* dst = part_chunk(it.j, it.slice, c);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) dst[j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                    for (int j = 0; j < 8; ++j) dst[32 * j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                     return;
                 }
                 if (last) {  // (partial 0 + partial 1 + ... + partial s-2) + own sum
@@ -360,14 +362,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                     const float4* src = part_chunk(it.j, 0, c);
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
-                        const float4 x = __ldcg(src + j);
+                        const float4 x = __ldcg(src + 32 * j);
                         w[4 * j] = x.x; w[4 * j + 1] = x.y; w[4 * j + 2] = x.z; w[4 * j + 3] = x.w;
                     }
                     for (int k = 1; k < p.slices - 1; ++k) {
                         src = part_chunk(it.j, k, c);
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
-                            const float4 x = __ldcg(src + j);
+                            const float4 x = __ldcg(src + 32 * j);
                             w[4 * j] += x.x; w[4 * j + 1] += x.y; w[4 * j + 2] += x.z; w[4 * j + 3] += x.w;
                         }
                     }
