@@ -308,17 +308,23 @@ def _tc(p, lim):
                          predicted_cost=waves * t_kb * num_kb,
                          instance=TC_PAIR_FIRST + (0 if p.dtype == BF16 else 1))
                 out.append(c)
-                # tail split: the tiles past the last whole wave in `sl` K-slices each
-                full_waves, tail = pairs // live, pairs % live
-                for sl in (2, 4):
-                    if full_waves < 1 or tail == 0 or tail * sl > live or num_kb < 4 * sl:
-                        continue
-                    t = dict(c)
-                    t.update(split_k=sl, reduce=2,
-                             wave_eff_ppm=pairs * 1000000 * sl // (live * (full_waves * sl + 1)),
-                             predicted_cost=full_waves * t_kb * num_kb + t_kb * cdiv(num_kb, sl) +
-                             sl * (128 * 256 * 4 // FEED_BYTES_PER_CLK))
-                    out.append(t)
+                # stream-K over the last waves: whole waves but the last as whole tiles, the
+                # k-blocks of the rest shared evenly by all pairs
+                pair_slots = max(1, lim["sm_count"] * blk // 2)
+                # only from two whole waves on (all-stream-K measured slower)
+                if pairs % pair_slots and pairs // pair_slots >= 2:
+                    waves_sk = pairs // pair_slots
+                    dp = (waves_sk - 1) * pair_slots
+                    iters = (pairs - dp) * num_kb
+                    share = iters // pair_slots
+                    if share >= 4:
+                        per_pair = cdiv(iters, pair_slots)
+                        t = dict(c)
+                        t.update(reduce=2, grid=2 * pair_slots,
+                                 wave_eff_ppm=pairs * num_kb * 1000000 // (dp * num_kb + pair_slots * per_pair),
+                                 predicted_cost=(dp // pair_slots) * t_kb * num_kb + t_kb * per_pair +
+                                 (1 + cdiv(num_kb, share)) * (128 * 256 * 4 // FEED_BYTES_PER_CLK))
+                        out.append(t)
     return out, 2 * 3 * (TC_MAX_STAGES - 1) * 4 * 2 * 2 * 2 * 2
 
 

@@ -244,15 +244,12 @@ std::string cache_key(const Problem& p, int dev, const nnjit_device_limits& L, c
 // Split-K partials go to a workspace unless they are reduced inside a cluster.
 bool uses_workspace(const nnjit_candidate& c) { return c.split_k > 1 && c.reduce == 0; }
 
-// A CTA-pair candidate whose tail tiles are split into K-slices (reduce 2).
-bool pair_tail_split(const nnjit_candidate& c) { return c.cluster_m == 2 && c.reduce == 2; }
+// A CTA-pair candidate with stream-K over its last waves (reduce 2).
+bool pair_stream_k(const nnjit_candidate& c) { return c.cluster_m == 2 && c.reduce == 2; }
 
 size_t ws_bytes_for(const Problem& p, const nnjit_candidate& c) {
-    if (pair_tail_split(c)) {
-        const int64_t pairs = std::max(1, c.grid / 2);
-        const int64_t total = p.batch * ((p.M + 255) / 256) * ((p.N + 255) / 256);
-        return (size_t)tc2_tail_ws_bytes(total % pairs, c.split_k);
-    }
+    (void)p;
+    if (pair_stream_k(c)) return (size_t)tc2_sk_ws_bytes(std::max(1, c.grid / 2));
     if (!uses_workspace(c)) return 0;
     return (size_t)c.split_k * (size_t)p.batch * (size_t)p.M * (size_t)p.N * sizeof(float);
 }
@@ -378,7 +375,7 @@ nnjit_status make_scratch(const Problem& p, const std::vector<nnjit_candidate>& 
     if ((err = cudaMalloc(&s->C.p, sets * r256(s->c_elems * 4))) != cudaSuccess) return cuda_fail(err, "scratch C");
     if ((err = cudaMalloc(&s->bias.p, r256((size_t)p.N * 4))) != cudaSuccess) return cuda_fail(err, "scratch bias");
     if (ws_max && (err = cudaMalloc(&s->ws.p, ws_max)) != cudaSuccess) return cuda_fail(err, "scratch workspace");
-    // tail-split candidates keep hand-off counters in the workspace: zero before first use
+    // stream-K candidates keep hand-off flags in the workspace: zero before first use
     if (ws_max && (err = cudaMemset(s->ws.p, 0, ws_max)) != cudaSuccess) return cuda_fail(err, "scratch workspace");
     if ((err = launch_fill_scratch(s->A.p, (int64_t)(sets * r256(s->a_elems * e) / e), e, 1u, 0)) != cudaSuccess ||
         (err = launch_fill_scratch(s->B.p, (int64_t)(sets * r256(s->b_elems * e) / e), e, 2u, 0)) != cudaSuccess ||
@@ -429,8 +426,8 @@ bool time_candidate(nnjit_plan pl, const nnjit_candidate& c, const Scratch& sc, 
         if (fault.kind == 2 && fault.index == idx) word = 0x1FF;
         if (word != 0) {
             cudaMemset(pl->err, 0, sizeof(int));
-            // a stopped tail-split launch may have left hand-off counters raised
-            if (ws && pair_tail_split(c)) cudaMemset(ws, 0, ws_bytes_for(p, c));
+            // a stopped stream-K launch may have left hand-off flags raised
+            if (ws && pair_stream_k(c)) cudaMemset(ws, 0, ws_bytes_for(p, c));
         }
         return word != 0;
     };
@@ -504,7 +501,7 @@ nnjit_status alloc_plan_buffers(nnjit_plan pl) {
     if (pl->ws_bytes) {
         e = cudaMalloc(&pl->ws, pl->ws_bytes);
         if (e != cudaSuccess) return cuda_fail(e, "split-K workspace");
-        e = cudaMemset(pl->ws, 0, pl->ws_bytes);  // tail-split hand-off counters start at zero
+        e = cudaMemset(pl->ws, 0, pl->ws_bytes);  // stream-K hand-off flags start at zero
         if (e != cudaSuccess) return cuda_fail(e, "split-K workspace");
     }
     return NNJIT_OK;
@@ -1309,7 +1306,7 @@ nnjit_status nnjit_plan_check(nnjit_plan p) {
     if (e == cudaSuccess) e = cudaMemcpy(&word, p->err, sizeof(int), cudaMemcpyDeviceToHost);
     if (e == cudaSuccess && word != 0) {
         cudaMemset(p->err, 0, sizeof(int));
-        // a stopped tail-split launch may have left hand-off counters raised
+        // a stopped stream-K launch may have left hand-off flags raised
         if (p->ws && p->ws_bytes) cudaMemset(p->ws, 0, p->ws_bytes);
     }
     if (cur != p->device) cudaSetDevice(cur);

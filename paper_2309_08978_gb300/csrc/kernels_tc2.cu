@@ -21,18 +21,22 @@
 // Every wait is bounded; on expiry the error word is set and the roles fall through to
 // the teardown (the producers wait, bounded, for their ring slots to drain first).
 //
-// Tail split (candidate reduce = 2, split_k = s): when the pair tiles do not fill a whole
-// number of waves of the resident pairs, the `tail` tiles of the last partial wave are
-// cut into s slices of their k-blocks, so that the last wave runs tail * s shorter work
-// items on up to all pairs instead of `tail` whole tiles on a few.  Work items are the
-// whole tiles first, then every tail tile's slices 0 .. s-2, then their last slices.  A
-// slice other than the last writes its raw accumulator to the plan's workspace and adds
-// one to a counter per (tail tile, CTA, epilogue warp) with release semantics; the last
-// slice of the tile waits (bounded) for s - 1 counts, adds the partials to its own
-// accumulator in slice order (so repeated runs give identical bits), applies bias,
-// activation and residual, stores C and resets its counter for the next launch.  Each
-// persistent pair takes items in increasing order and a last slice waits only for items
-// of lower index, which run on other pairs in the same final round, so every wait ends.
+// Stream-K over the last waves (candidate reduce = 2).  The pairs are persistent and
+// take tiles round-robin, so when the pair tiles are not a whole number of waves of the
+// P resident pairs the last wave runs a few tiles while the other pairs idle.  Then only
+// the first (waves - 1) * P tiles run whole ("dp" tiles, round-robin); the k-blocks of
+// the remaining tiles ("sk" tiles, between 1 and 2 waves' worth) are laid end to end and
+// cut into P equal ranges, pair p taking range p after its dp tiles.  A range may start
+// inside a tile (its first segment), hold whole tiles, and end inside a tile (its last
+// segment).  A segment that starts inside a tile writes its raw sum to the pair's slot
+// of the workspace and raises a flag per (CTA, epilogue warp) with release semantics: so
+// a pair writes at most one partial.  The segment that starts a tile's k-blocks but does
+// not reach their end finishes the tile: it waits (bounded) for the flags of the pairs
+// that cover the rest, adds their partials to its own sum in pair order (identical bits
+// on every run), applies bias, activation and residual, stores C and lowers the flags
+// for the next launch.  A finishing segment is the last of its pair and waits only for
+// first segments of later pairs, which never wait, so every wait ends.
+
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -57,7 +61,7 @@ constexpr int kErrMmaTmemEmpty = 0x142;
 constexpr int kErrMmaFull = 0x143;
 constexpr int kErrEpiTmemFull = 0x144;
 constexpr int kErrDrain = 0x145;
-constexpr int kErrTailWait = 0x146;
+constexpr int kErrSkWait = 0x146;
 
 struct Tc2Params {
     CUtensorMap tmap_a;  // A: dims {K, M, batch}, box {BK, 128, 1}
@@ -72,20 +76,16 @@ struct Tc2Params {
     long long ldc, stride_c;
     int num_kb, tiles2_m, tiles_n, total, stages, raster;
     int act;  // nnjit_epilogue
-    // tail split: items = full + tail * slices (slices = 1: every item a whole tile)
-    int full, tail, slices, items;
-    float* part;    // [tail][slices - 1][2 CTAs][BN / 32 chunks][4 warps][8][32 lanes] float4 partials
-    unsigned* cnt;  // [tail][2 CTAs][4 epilogue warps] hand-off counters, zero between launches
+    // stream-K: tiles [0, dp) whole and round-robin; the k-blocks of tiles [dp, total)
+    // split evenly over the pairs (dp = total: no stream-K)
+    int dp, pairs;
+    long long sk_iters;  // (total - dp) * num_kb
+    float* part;         // [pairs][2 CTAs][BN / 32 chunks][4 warps][8][32 lanes] float4 partials
+    unsigned* flag;      // [pairs][2 CTAs][4 epilogue warps], zero between launches
 };
 
 struct PairTile {
     int b, tm2, tn;
-};
-
-// One work item: a whole pair tile (slice = -1) or slice `slice` of tail tile `j`,
-// covering k-blocks [kb0, kb1).
-struct PairItem {
-    int tile, slice, j, kb0, kb1;
 };
 
 __device__ __forceinline__ PairTile decode(int t, const Tc2Params& p) {
@@ -103,19 +103,55 @@ __device__ __forceinline__ PairTile decode(int t, const Tc2Params& p) {
     return c;
 }
 
-__device__ __forceinline__ PairItem decode_item(int t, const Tc2Params& p) {
-    PairItem it;
-    if (t < p.full) {
-        it.tile = t; it.slice = -1; it.j = 0; it.kb0 = 0; it.kb1 = p.num_kb;
-        return it;
+// One segment of a pair's work: k-blocks [kb0, kb1) of tile `tile`.  role 0: the whole
+// tile; 1: a partial sum for another pair to finish (the pair's first stream-K segment,
+// starting inside the tile); 2: finish the tile, adding the partials of pairs
+// [p_lo, p_hi].
+struct Seg {
+    int tile, kb0, kb1, role, p_lo, p_hi;
+};
+struct SegIter {
+    int dp_next;
+    long long i, end;
+};
+
+__device__ __forceinline__ SegIter seg_begin(int pc, const Tc2Params& p) {
+    SegIter st;
+    st.dp_next = pc;
+    st.i = (long long)pc * p.sk_iters / p.pairs;
+    st.end = (long long)(pc + 1) * p.sk_iters / p.pairs;
+    return st;
+}
+
+// The pair whose stream-K range holds k-block iteration i: the largest q with
+// floor(q * T / P) <= i (only called with T = sk_iters > 0).
+__device__ __forceinline__ int sk_pair_of(long long i, const Tc2Params& p) {
+    return (int)(((i + 1) * p.pairs - 1) / p.sk_iters);
+}
+
+__device__ __forceinline__ bool seg_next(SegIter& st, Seg& sg, const Tc2Params& p) {
+    if (st.dp_next < p.dp) {
+        sg.tile = st.dp_next; sg.kb0 = 0; sg.kb1 = p.num_kb; sg.role = 0; sg.p_lo = sg.p_hi = 0;
+        st.dp_next += p.pairs;
+        return true;
     }
-    const int r = t - p.full;
-    it.slice = r / p.tail;
-    it.j = r % p.tail;
-    it.tile = p.full + it.j;
-    it.kb0 = (int)((long long)it.slice * p.num_kb / p.slices);
-    it.kb1 = (int)((long long)(it.slice + 1) * p.num_kb / p.slices);
-    return it;
+    if (st.i >= st.end) return false;
+    const long long t = st.i / p.num_kb;
+    sg.tile = p.dp + (int)t;
+    sg.kb0 = (int)(st.i - t * p.num_kb);
+    sg.kb1 = (int)min((long long)p.num_kb, sg.kb0 + (st.end - st.i));
+    sg.p_lo = sg.p_hi = 0;
+    if (sg.kb0 > 0) {
+        sg.role = 1;
+    } else if (sg.kb1 == p.num_kb) {
+        sg.role = 0;
+    } else {
+        sg.role = 2;
+        sg.p_lo = sk_pair_of(t * p.num_kb + sg.kb1, p);
+        sg.p_hi = sk_pair_of(t * p.num_kb + p.num_kb - 1, p);
+    }
+    st.i = t * p.num_kb + sg.kb1;
+    return true;
 }
 
 // NB: accumulator buffers in TMEM (2: the epilogue of one tile overlaps the mainloop of
@@ -141,7 +177,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
     uint64_t* bars = reinterpret_cast<uint64_t*>(epi_smem + kEpiStageBytes);
     // bars[0..S): full (used in the even CTA), [S..2S): empty, 2S..2S+1: tmem_full,
     // 2S+2..2S+3: tmem_empty (even CTA), 2S+4: drain (even CTA)
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kMaxStages + 5);
+    // bars[2 kMaxStages + 5 + q]: partial-tile copy of epilogue warp q (stream-K finisher)
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bars + 2 * kMaxStages + 9);
     volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -154,6 +191,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
     auto tfull_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + a); };
     auto tempty_bar = [&](int a) { return ptx::smem_u32(bars + 2 * S + 2 + a); };
     const uint32_t drain_bar = ptx::smem_u32(bars + 2 * S + 4);
+    auto pcopy_bar = [&](int q) { return ptx::smem_u32(bars + 2 * kMaxStages + 5 + q); };
     const int t_begin = (int)(blockIdx.x >> 1);
     const int t_step = (int)(gridDim.x >> 1);
 
@@ -167,6 +205,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
             ptx::mbar_init(tempty_bar(a), 8);  // 4 epilogue warps of each CTA
         }
         ptx::mbar_init(drain_bar, 1);
+        for (int q = 0; q < 4; ++q) ptx::mbar_init(pcopy_bar(q), 1);
         *abort_flag = 0;
         ptx::fence_barrier_init();
     }
@@ -176,8 +215,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         ptx::prefetch_tmap(&p.tmap_a);
         ptx::prefetch_tmap(&p.tmap_b);
         if (p.tma_store) ptx::prefetch_tmap(&p.tmap_c);
-        if (t_begin < p.items) {
-            const PairItem it = decode_item(t_begin, p);
+        SegIter st0 = seg_begin(t_begin, p);
+        Seg it;
+        if (seg_next(st0, it, p)) {
             const PairTile tc = decode(it.tile, p);
             for (int kb = it.kb0; kb < it.kb1 && kb < it.kb0 + S; ++kb) {
                 ptx::tma_prefetch_l2_3d(&p.tmap_a, kb * BK, tc.tm2 * 256 + row_off, tc.b);
@@ -200,8 +240,10 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
     // With a constant B the first ring's B halves are requested before the dependency
     // wait; the even CTA arms those slots with the bytes of both CTAs' A and B.
     int b_preloaded = 0;
-    if (p.b_const && warp == 0 && t_begin < p.items) {
-        const PairItem it = decode_item(t_begin, p);
+    SegIter st_first = seg_begin(t_begin, p);
+    Seg first;
+    if (p.b_const && warp == 0 && seg_next(st_first, first, p)) {
+        const Seg& it = first;
         const PairTile tc = decode(it.tile, p);
         b_preloaded = min(S, it.kb1 - it.kb0);
         if (lane == 0) {
@@ -222,8 +264,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         uint32_t phase = 0;
         bool ok = true;
         int issued = 0;
-        for (int t = t_begin; ok && t < p.items; t += t_step) {
-            const PairItem it = decode_item(t, p);
+        SegIter st = seg_begin(t_begin, p);
+        Seg it;
+        while (ok && seg_next(st, it, p)) {
             const PairTile tc = decode(it.tile, p);
             for (int kb = it.kb0; kb < it.kb1; ++kb) {
                 if (!ptx::mbar_wait(empty_bar(stage), phase ^ 1u, abort_flag, p.err, kErrProducerEmpty)) {
@@ -265,8 +308,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
             bool ok = true;
             const uint64_t a_desc0 = ptx::smem_desc(smem_base, 16, 1024);
             const uint64_t b_desc0 = ptx::smem_desc(smem_base + kABytes, 16, 1024);
-            for (int t = t_begin; ok && t < p.items; t += t_step, ++iter) {
-                const PairItem it = decode_item(t, p);
+            SegIter st = seg_begin(t_begin, p);
+            Seg it;
+            for (; ok && seg_next(st, it, p); ++iter) {
                 const uint32_t acc = NB == 2 ? (iter & 1u) : 0u;
                 const uint32_t acc_phase = NB == 2 ? ((iter >> 1) & 1u) : (iter & 1u);
                 if (!ptx::mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty)) {
@@ -317,29 +361,47 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
         const uint32_t leader_tempty1 = ptx::map_shared_rank(tempty_bar(1), 0);
         constexpr int kChunks = BN / 32;
         static_assert(kChunks % 2 == 0, "chunks are processed in pairs");
-        // This warp's block of chunk c of slice k of tail tile j in the workspace: 8 x 32
-        // float4, element [i][lane] = columns 4i .. 4i + 3 of the lane's row, so that each
-        // warp-wide access covers 512 contiguous bytes.
-        auto part_chunk = [&](int j, int k, int c) {
-            const long long blk = (((((long long)j * (p.slices - 1) + k) * 2 + rank) * kChunks + c) * 4) + q;
-            return reinterpret_cast<float4*>(p.part) + blk * 256 + lane;
+        // Pair pr's partial in the workspace, for this CTA and warp: kChunks blocks of 8 x 32
+        // float4 (32 KB, contiguous), element [c][i][lane] = columns 32c + 4i .. 32c + 4i + 3
+        // of the lane's row, so that each warp-wide access covers 512 contiguous bytes.
+        auto part_block = [&](int pr) {
+            return reinterpret_cast<float4*>(p.part) + (((long long)pr * 2 + rank) * 4 + q) * (kChunks * 256);
         };
-        for (int t = t_begin; t < p.items; t += t_step, ++iter) {
-            const PairItem it = decode_item(t, p);
+        auto part_chunk = [&](int pr, int c) { return part_block(pr) + c * 256 + lane; };
+        // A finisher reads its (single) partial from shared memory: the ring is idle once its
+        // last segment's MMAs have completed, and warp q's 32 KB go to ring offset 32 KB * q.
+        const float4* staged = reinterpret_cast<const float4*>(smem + q * (kChunks * 4096)) + lane;
+        auto flag_of = [&](int pr) { return p.flag + ((pr * 2 + (int)rank) * 4 + q); };
+        const int pc = t_begin;  // this pair
+        SegIter st = seg_begin(pc, p);
+        Seg it;
+        for (; seg_next(st, it, p); ++iter) {
             const PairTile tc = decode(it.tile, p);
-            // a slice other than the last hands its sum over; the last slice collects them
-            const bool partial = it.slice >= 0 && it.slice < p.slices - 1;
-            const bool last = it.slice >= 0 && it.slice == p.slices - 1;
-            unsigned* cnt = p.cnt + ((it.j * 2 + (int)rank) * 4 + q);
+            const bool partial = it.role == 1;  // hand the sum over to the tile's finisher
+            const bool last = it.role == 2;     // finish the tile with the other pairs' sums
             const uint32_t acc = NB == 2 ? (iter & 1u) : 0u;
             const uint32_t acc_phase = NB == 2 ? ((iter >> 1) & 1u) : (iter & 1u);
             if (!ptx::mbar_wait(tfull_bar(acc), acc_phase, abort_flag, p.err, kErrEpiTmemFull)) break;
             ptx::tc_fence_after();
             if (last) {
                 bool ok = true;
-                if (lane == 0) ok = ptx::wait_counter(cnt, (uint32_t)(p.slices - 1), abort_flag, p.err, kErrTailWait);
+                if (lane == 0)
+                    for (int pr = it.p_lo; ok && pr <= it.p_hi; ++pr)
+                        ok = ptx::wait_counter(flag_of(pr), 1u, abort_flag, p.err, kErrSkWait);
                 if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
-                (void)ptx::ld_acquire_gpu(cnt);  // every lane orders its partial reads after the count
+                for (int pr = it.p_lo; pr <= it.p_hi; ++pr)
+                    (void)ptx::ld_acquire_gpu(flag_of(pr));  // every lane orders its partial reads
+                if (it.p_lo == it.p_hi) {  // one partial: one bulk copy into the idle ring
+                    if (lane == 0) {
+                        ptx::fence_proxy_async_global();
+                        ptx::mbar_arrive_expect_tx(pcopy_bar(q), kChunks * 4096);
+                        ptx::bulk_copy_g2s(ptx::smem_u32(smem) + q * (kChunks * 4096), part_block(it.p_lo),
+                                           kChunks * 4096, pcopy_bar(q));
+                    }
+                    __syncwarp();
+                    const bool landed = ptx::mbar_wait(pcopy_bar(q), 0, abort_flag, p.err, kErrSkWait);
+                    if (!__all_sync(0xffffffffu, landed)) break;
+                }
             }
             const int row_base = tc.tm2 * 256 + row_off + q * 32;
             const int row = row_base + lane;
@@ -351,30 +413,27 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 float v[32];
 #pragma unroll
                 for (int j = 0; j < 32; ++j) v[j] = __uint_as_float(r[j]);
-                if (partial) {  // raw sum of this slice's k-blocks to the workspace
-                    float4* dst = part_chunk(it.j, it.slice, c);
+                if (partial) {  // raw sum of this segment's k-blocks to the pair's slot
+                    float4* dst = part_chunk(pc, c);
 #pragma unroll
                     for (int j = 0; j < 8; ++j) dst[32 * j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                     return;
                 }
-                if (last) {  // (partial 0 + partial 1 + ... + partial s-2) + own sum
-                    float w[32];
-                    const float4* src = part_chunk(it.j, 0, c);
+                if (last && it.p_lo == it.p_hi) {  // own sum + the staged partial
 #pragma unroll
                     for (int j = 0; j < 8; ++j) {
-                        const float4 x = __ldcg(src + 32 * j);
-                        w[4 * j] = x.x; w[4 * j + 1] = x.y; w[4 * j + 2] = x.z; w[4 * j + 3] = x.w;
+                        const float4 x = staged[c * 256 + 32 * j];
+                        v[4 * j] += x.x; v[4 * j + 1] += x.y; v[4 * j + 2] += x.z; v[4 * j + 3] += x.w;
                     }
-                    for (int k = 1; k < p.slices - 1; ++k) {
-                        src = part_chunk(it.j, k, c);
+                } else if (last) {  // ((own sum + partial of pair p_lo) + ...) + partial of pair p_hi
+                    for (int pr = it.p_lo; pr <= it.p_hi; ++pr) {
+                        const float4* src = part_chunk(pr, c);
 #pragma unroll
                         for (int j = 0; j < 8; ++j) {
                             const float4 x = __ldcg(src + 32 * j);
-                            w[4 * j] += x.x; w[4 * j + 1] += x.y; w[4 * j + 2] += x.z; w[4 * j + 3] += x.w;
+                            v[4 * j] += x.x; v[4 * j + 1] += x.y; v[4 * j + 2] += x.z; v[4 * j + 3] += x.w;
                         }
                     }
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) v[j] = w[j] + v[j];
                 }
                 if (bias) {
 #pragma unroll
@@ -450,14 +509,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 emit(rb, bb, c + 1);
                 if (c + 2 < kChunks) ptx::tmem_wait_ld(ra);
             }
-            if (partial) {  // publish this warp's rows of the slice
+            if (partial) {  // publish this warp's rows of the partial
                 __threadfence();
                 __syncwarp();
-                if (lane == 0) ptx::red_release_add_gpu(cnt, 1u);
+                if (lane == 0) ptx::red_release_add_gpu(flag_of(pc), 1u);
             }
             if (last) {  // every partial has been read: ready for the next launch
                 __syncwarp();
-                if (lane == 0) *cnt = 0u;
+                if (lane == 0)
+                    for (int pr = it.p_lo; pr <= it.p_hi; ++pr) *flag_of(pr) = 0u;
             }
         }
         if (p.tma_store && lane == 0) ptx::bulk_wait_all_read();
@@ -488,10 +548,11 @@ cudaError_t launch_tc_pair(const LaunchArgs& a) {
     if (c.bm != 256 || c.bn != 256 || c.cluster_m != 2 || c.stages < 2 || c.stages > kMaxStages ||
         c.bk != 128 / p.elem_bytes())
         return cudaErrorInvalidValue;
-    // unsplit (split_k 1, reduce 0) or tail split (reduce 2, split_k = slices of a tail tile)
-    const bool tail_split = c.reduce == 2;
-    if (tail_split ? (c.split_k < 2 || c.split_k > 8 || !a.ws) : (c.split_k != 1 || c.reduce != 0))
-        return cudaErrorInvalidValue;
+    // unsplit (reduce 0) or stream-K over the last waves (reduce 2); split_k is 1
+    const bool stream_k = c.reduce == 2;
+    if (c.split_k != 1 || (c.reduce != 0 && !stream_k) || (stream_k && !a.ws)) return cudaErrorInvalidValue;
+    // a stream-K finisher stages a partial (4 warps x 32 KB) in the idle ring
+    if (stream_k && c.stages * (128 + 128) * 128 < 4 * 32768) return cudaErrorInvalidValue;
     Tc2Params prm;
     prm.tmap_a = *a.tmap_a;
     prm.tmap_b = *a.tmap_b;
@@ -516,27 +577,25 @@ cudaError_t launch_tc_pair(const LaunchArgs& a) {
     prm.total = (int)total;
     prm.stages = c.stages;
     prm.raster = c.raster;
-    const int grid = (int)std::min<long long>(2 * total, c.grid);
-    prm.full = prm.total;
-    prm.tail = 0;
-    prm.slices = 1;
+    // unsplit: at most one pair per tile; stream-K: every pair of the candidate's grid
+    const int grid = stream_k ? c.grid : (int)std::min<long long>(2 * total, c.grid);
+    prm.pairs = grid / 2;
+    prm.dp = prm.total;
+    prm.sk_iters = 0;  // no stream-K region: every pair's range is empty
     prm.part = nullptr;
-    prm.cnt = nullptr;
-    if (tail_split) {
-        // the tiles past the last whole wave of `pairs` resident pairs, each in split_k slices
-        const int pairs = grid / 2;
-        const int tail = prm.total % pairs;
-        if (prm.total <= pairs || tail == 0 || (long long)tail * c.split_k > pairs ||
-            prm.num_kb < 4 * c.split_k)
-            return cudaErrorInvalidValue;
-        prm.tail = tail;
-        prm.full = prm.total - tail;
-        prm.slices = c.split_k;
-        // workspace: the counters, then the partial sums (tc2_tail_ws_bytes)
-        prm.cnt = reinterpret_cast<unsigned*>(a.ws);
-        prm.part = a.ws + tc2_tail_cnt_floats(tail);
+    prm.flag = nullptr;
+    if (stream_k) {
+        // whole waves but the last run as whole tiles; the rest (1 to 2 waves) stream-K
+        const int P = prm.pairs;
+        const int waves = prm.total / P;
+        if (prm.total % P == 0) return cudaErrorInvalidValue;
+        prm.dp = waves >= 1 ? (waves - 1) * P : 0;
+        prm.sk_iters = (long long)(prm.total - prm.dp) * prm.num_kb;
+        if (prm.sk_iters < (long long)P) return cudaErrorInvalidValue;
+        // workspace: the flags, then one partial tile per pair (tc2_sk_ws_bytes)
+        prm.flag = reinterpret_cast<unsigned*>(a.ws);
+        prm.part = a.ws + tc2_sk_flag_floats(P);
     }
-    prm.items = prm.full + prm.tail * prm.slices;
     const int stage_bytes = (128 + 128) * 128;
     const int smem = c.stages * stage_bytes + kEpiStageBytes + 1024 + 256;
     {

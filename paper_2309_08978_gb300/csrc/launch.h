@@ -52,16 +52,14 @@ cudaError_t launch_ffma(const LaunchArgs& a);
 cudaError_t launch_gemv(const LaunchArgs& a);
 cudaError_t launch_tc(const LaunchArgs& a);
 // CTA-pair (cta_group::2) tensor-core instances kTcPairFirstInstance.. (bf16, tf32).  A
-// tail-split candidate (reduce 2) takes its counters and partial sums from LaunchArgs::ws.
+// stream-K candidate (reduce 2) takes its flags and partial sums from LaunchArgs::ws.
 cudaError_t launch_tc_pair(const LaunchArgs& a);
-// Workspace of a tail-split pair candidate with `tail` tiles of `slices` slices: per tail
-// tile 2 CTAs x 4 warps of counters (padded to 256 bytes in all), then (slices - 1) partial
-// 256 x 256 f32 tiles.  The counters must be zero before the first launch; every launch
-// that completes leaves them zero.
-inline int64_t tc2_tail_cnt_floats(int64_t tail) { return (tail * 8 + 63) / 64 * 64; }
-inline int64_t tc2_tail_ws_bytes(int64_t tail, int64_t slices) {
-    return (tc2_tail_cnt_floats(tail) + tail * (slices - 1) * 256 * 256) * 4;
-}
+// Workspace of a stream-K pair candidate over `pairs` pairs: 2 CTAs x 4 warps of flags
+// per pair (padded to 256 bytes in all), then one 256 x 256 f32 partial tile per pair.
+// The flags must be zero before the first launch; every launch that completes leaves
+// them zero.
+inline int64_t tc2_sk_flag_floats(int64_t pairs) { return (pairs * 8 + 63) / 64 * 64; }
+inline int64_t tc2_sk_ws_bytes(int64_t pairs) { return (tc2_sk_flag_floats(pairs) + pairs * 256 * 256) * 4; }
 
 // C[b,m,n] = sum_{s < split} ws[s][b][m][n] (+ bias[n]), s ascending.
 cudaError_t launch_splitk_reduce(const float* ws, int split, const Problem& p, const float* bias,

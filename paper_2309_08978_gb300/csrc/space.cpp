@@ -171,20 +171,28 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 c.predicted_cost = waves * t_kb * num_kb;
                 c.instance = kTcPairFirstInstance + (p.dtype == NNJIT_BF16 ? 0 : 1);
                 v.push_back(c);
-                // Tail split: the tiles past the last whole wave are cut into `sl` slices of
-                // their k-blocks, so the last wave takes 1/sl of a tile plus the hand-off of
-                // the partial sums (one 128-row x 256-column f32 partial per CTA written or
-                // read per slice, at the per-SM feed rate).
-                const int64_t full_waves = pairs / live, tail = pairs % live;
-                for (int sl : {2, 4}) {
-                    if (full_waves < 1 || tail == 0 || tail * sl > live || num_kb < 4LL * sl) continue;
-                    nnjit_candidate t = c;
-                    t.split_k = sl;
-                    t.reduce = 2;
-                    t.wave_eff_ppm = (int32_t)(pairs * 1000000 * sl / (live * (full_waves * sl + 1)));
-                    t.predicted_cost = full_waves * t_kb * num_kb + t_kb * ceil_div(num_kb, sl) +
-                                       sl * (128LL * 256 * 4 / MC::kFeedBytesPerClk);
-                    v.push_back(t);
+                // Stream-K over the last waves: the whole waves but the last run as whole
+                // tiles, the k-blocks of the remaining tiles are shared evenly by all pairs;
+                // each pair hands at most one partial tile over, and a tile's finisher reads
+                // the partials of the pairs covering the rest of it (one 128-row x 256-column
+                // f32 partial per CTA each, at the per-SM feed rate).
+                // Only from two whole waves on: with fewer tiles (all of them stream-K) it
+                // measured slower than whole tiles on every T5-large product.
+                if (pairs % pair_slots != 0 && pairs / pair_slots >= 2) {
+                    const int64_t waves_sk = pairs / pair_slots;
+                    const int64_t dp = (waves_sk - 1) * pair_slots;
+                    const int64_t iters = (pairs - dp) * num_kb;
+                    const int64_t share = iters / pair_slots;
+                    if (share >= 4) {
+                        nnjit_candidate t = c;
+                        t.reduce = 2;
+                        t.grid = (int32_t)(2 * pair_slots);
+                        const int64_t per_pair = ceil_div(iters, pair_slots);
+                        t.wave_eff_ppm = (int32_t)(pairs * num_kb * 1000000 / (dp * num_kb + pair_slots * per_pair));
+                        t.predicted_cost = (dp / pair_slots) * t_kb * num_kb + t_kb * per_pair +
+                                           (1 + ceil_div(num_kb, share)) * (128LL * 256 * 4 / MC::kFeedBytesPerClk);
+                        v.push_back(t);
+                    }
                 }
             }
         }

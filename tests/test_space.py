@@ -266,10 +266,10 @@ def test_blackwell_usage_matches_hand_worked_values(fam, prob, pick, want):
 @pytest.mark.parametrize("prob,order", list(_blackwell_rows("order")))
 def test_evaluation_order_matches_hand_ordering(prob, order):
     """The 4096^3 BF16 space, index by index, in the order worked out by hand (blocks per
-    SM, then the cost, then enumeration order), tail-split CTA pairs included."""
+    SM, then the cost, then enumeration order), stream-K CTA pairs included."""
     for who, space in _both_spaces(prob).items():
         assert len(space) == len(order), f"{who}: {len(space)} candidates"
-        for idx, bm, bn, bk, split, raster, cluster in order:
+        for idx, bm, bn, bk, split, reduce, raster, cluster in order:
             c = space[idx]
-            assert (c["bm"], c["bn"], c["bk"], c["split_k"], c["raster"], c["cluster_m"]) == \
-                (bm, bn, bk, split, raster, cluster), f"{who}: index {idx} is {c}"
+            assert (c["bm"], c["bn"], c["bk"], c["split_k"], c["reduce"], c["raster"], c["cluster_m"]) == \
+                (bm, bn, bk, split, reduce, raster, cluster), f"{who}: index {idx} is {c}"
