@@ -311,7 +311,8 @@ def _tc(p, lim):
                 # stream-K over the last waves: whole waves but the last as whole tiles, the
                 # k-blocks of the rest shared evenly by all pairs
                 pair_slots = max(1, lim["sm_count"] * blk // 2)
-                # only from two whole waves on (all-stream-K measured slower)
+                # only from two whole waves on (with all tiles in stream-K the hand-offs sit
+                # on the critical path and the launch measured slower than whole tiles)
                 if pairs % pair_slots and pairs // pair_slots >= 2:
                     waves_sk = pairs // pair_slots
                     dp = (waves_sk - 1) * pair_slots

@@ -193,7 +193,6 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
     const uint32_t drain_bar = ptx::smem_u32(bars + 2 * S + 4);
     auto pcopy_bar = [&](int q) { return ptx::smem_u32(bars + 2 * kMaxStages + 5 + q); };
     const int t_begin = (int)(blockIdx.x >> 1);
-    const int t_step = (int)(gridDim.x >> 1);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < S; ++s) {
@@ -368,9 +367,12 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
             return reinterpret_cast<float4*>(p.part) + (((long long)pr * 2 + rank) * 4 + q) * (kChunks * 256);
         };
         auto part_chunk = [&](int pr, int c) { return part_block(pr) + c * 256 + lane; };
-        // A finisher reads its (single) partial from shared memory: the ring is idle once its
-        // last segment's MMAs have completed, and warp q's 32 KB go to ring offset 32 KB * q.
-        const float4* staged = reinterpret_cast<const float4*>(smem + q * (kChunks * 4096)) + lane;
+        // A finisher reads the partials from shared memory: the ring is idle once its last
+        // segment's MMAs have completed, and warp q stages them in its quarter of the ring,
+        // `cpr` chunks (4 KB each) of every partial per round.
+        const int stage_slots = S * (int)kStageBytes / 4 / 4096;
+        const uint32_t stage_u32 = ptx::smem_u32(smem) + (uint32_t)(q * stage_slots * 4096);
+        const float4* stage_f4 = reinterpret_cast<const float4*>(smem + q * stage_slots * 4096) + lane;
         auto flag_of = [&](int pr) { return p.flag + ((pr * 2 + (int)rank) * 4 + q); };
         const int pc = t_begin;  // this pair
         SegIter st = seg_begin(pc, p);
@@ -391,18 +393,15 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 if (!__shfl_sync(0xffffffffu, ok ? 1 : 0, 0)) break;
                 for (int pr = it.p_lo; pr <= it.p_hi; ++pr)
                     (void)ptx::ld_acquire_gpu(flag_of(pr));  // every lane orders its partial reads
-                if (it.p_lo == it.p_hi) {  // one partial: one bulk copy into the idle ring
-                    if (lane == 0) {
-                        ptx::fence_proxy_async_global();
-                        ptx::mbar_arrive_expect_tx(pcopy_bar(q), kChunks * 4096);
-                        ptx::bulk_copy_g2s(ptx::smem_u32(smem) + q * (kChunks * 4096), part_block(it.p_lo),
-                                           kChunks * 4096, pcopy_bar(q));
-                    }
-                    __syncwarp();
-                    const bool landed = ptx::mbar_wait(pcopy_bar(q), 0, abort_flag, p.err, kErrSkWait);
-                    if (!__all_sync(0xffffffffu, landed)) break;
-                }
+                if (lane == 0) ptx::fence_proxy_async_global();  // the copies read what the flags released
             }
+            // partials to stage per round: all chunks, half, or a quarter, as the ring allows
+            const int n_part = last ? it.p_hi - it.p_lo + 1 : 0;
+            const int cpr = !last ? 0 : n_part * kChunks <= stage_slots ? kChunks
+                                  : n_part * (kChunks / 2) <= stage_slots ? kChunks / 2
+                                  : n_part * 2 <= stage_slots ? 2 : 0;
+            uint32_t stage_phase = 0;
+            bool stage_ok = true;
             const int row_base = tc.tm2 * 256 + row_off + q * 32;
             const int row = row_base + lane;
             const float* bias = p.bias;
@@ -419,11 +418,14 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                     for (int j = 0; j < 8; ++j) dst[32 * j] = make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
                     return;
                 }
-                if (last && it.p_lo == it.p_hi) {  // own sum + the staged partial
+                if (last && cpr > 0) {  // ((own sum + staged partial of p_lo) + ...) + p_hi
+                    for (int k = 0; k < n_part; ++k) {
+                        const float4* src = stage_f4 + (k * cpr + c % cpr) * 256;
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const float4 x = staged[c * 256 + 32 * j];
-                        v[4 * j] += x.x; v[4 * j + 1] += x.y; v[4 * j + 2] += x.z; v[4 * j + 3] += x.w;
+                        for (int j = 0; j < 8; ++j) {
+                            const float4 x = src[32 * j];
+                            v[4 * j] += x.x; v[4 * j + 1] += x.y; v[4 * j + 2] += x.z; v[4 * j + 3] += x.w;
+                        }
                     }
                 } else if (last) {  // ((own sum + partial of pair p_lo) + ...) + partial of pair p_hi
                     for (int pr = it.p_lo; pr <= it.p_hi; ++pr) {
@@ -497,6 +499,24 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
             ptx::tmem_wait_ld(ra);
 #pragma unroll 1
             for (int c = 0; c < kChunks; c += 2) {
+                if (cpr > 0 && c % cpr == 0) {
+                    // stage chunks [c, c + cpr) of every partial: one bulk copy per partial
+                    __syncwarp();  // this warp's reads of the previous round are done
+                    if (lane == 0) {
+                        ptx::fence_proxy_async_smem();
+                        ptx::mbar_arrive_expect_tx(pcopy_bar(q), (uint32_t)(n_part * cpr * 4096));
+                        for (int k = 0; k < n_part; ++k)
+                            ptx::bulk_copy_g2s(stage_u32 + (uint32_t)(k * cpr * 4096), part_block(it.p_lo + k) + c * 256,
+                                               (uint32_t)(cpr * 4096), pcopy_bar(q));
+                    }
+                    __syncwarp();
+                    const bool landed = ptx::mbar_wait(pcopy_bar(q), stage_phase, abort_flag, p.err, kErrSkWait);
+                    stage_phase ^= 1u;
+                    if (!__all_sync(0xffffffffu, landed)) {
+                        stage_ok = false;
+                        break;
+                    }
+                }
                 ptx::tmem_ld32(tbase + (c + 1) * 32, rb);
                 bb = bias_of(c + 1);
                 emit(ra, ba, c);
@@ -509,6 +529,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                 emit(rb, bb, c + 1);
                 if (c + 2 < kChunks) ptx::tmem_wait_ld(ra);
             }
+            if (!stage_ok) break;
             if (partial) {  // publish this warp's rows of the partial
                 __threadfence();
                 __syncwarp();

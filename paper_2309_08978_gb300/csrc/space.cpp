@@ -176,8 +176,11 @@ void tc_space(const Problem& p, const nnjit_device_limits& L, std::vector<nnjit_
                 // each pair hands at most one partial tile over, and a tile's finisher reads
                 // the partials of the pairs covering the rest of it (one 128-row x 256-column
                 // f32 partial per CTA each, at the per-SM feed rate).
-                // Only from two whole waves on: with fewer tiles (all of them stream-K) it
-                // measured slower than whole tiles on every T5-large product.
+                // Only from two whole waves on.  With fewer tiles every tile is stream-K and
+                // the hand-offs sit on the critical path: a per-CTA timeline of T5-large wo
+                // (32 tiles) showed the MMAs done at 15 us against 22.5 us for whole tiles,
+                // but 2.5 us to publish a partial, 1.8 us to see its flag and 8 us to add two
+                // partials and store, so the launch ended later than with whole tiles.
                 if (pairs % pair_slots != 0 && pairs / pair_slots >= 2) {
                     const int64_t waves_sk = pairs / pair_slots;
                     const int64_t dp = (waves_sk - 1) * pair_slots;
