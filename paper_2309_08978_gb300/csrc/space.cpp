@@ -302,7 +302,7 @@ void gemv_w4_space(const Problem& p, const nnjit_device_limits& L, std::vector<n
                 // dynamic (1 KB alignment slack + ring) and static (barriers, partial sums)
                 const int64_t smem = 1024 + stages * stage_bytes + 256 + rows * 128;
                 if (smem > L.smem_per_block_optin) continue;
-                const int regs = rows == 16 ? 88 : 112;  // ptxas: 84 / 110
+                const int regs = rows == 16 ? 88 : 112;  // ptxas: 82 / 108
                 const int blk = blocks_per_core(L, regs, MC::kGemvTmaThreads, (int)smem, 0);
                 if (blk < 1) continue;
                 const int64_t items = groups * split;

@@ -363,7 +363,7 @@ def test_fused_activation_k0_applies_to_bias(act):
 
 
 W4_CASES = [(1, 4096, 4096, 0), (1, 4096, 11008, 0), (3, 1000, 2056, 2080), (8, 520, 4096, 0),
-            (2, 264, 640, 0)]
+            (2, 264, 640, 0), (5, 4008, 4096, 0)]
 
 
 def _w4_ids(c):
