@@ -372,6 +372,11 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             const uint32_t tbase = tmem_base + ((uint32_t)(q * 32) << 16) + acc * BN;
             constexpr int kChunks = BN / 32;
             static_assert(kChunks % 2 == 0, "chunks are processed in pairs");
+            // The CTA's last tile: its MMAs have completed and no load follows, so the ring
+            // is idle and each warp stages every chunk in its own part of it, with no wait
+            // for earlier stores (the tail of the launch is bound by stores in flight).
+            const bool ring_out = p.tma_store && t + t_step >= p.total_tiles &&
+                                  S * (int)kGroupBytes >= 4 * kChunks * 4096;
             // One 32-column chunk: bias (lane j fetched column j; broadcast by shuffles),
             // then the staged TMA store or the direct stores.
             auto emit = [&](const uint32_t (&r)[32], float bl, int c) {
@@ -384,8 +389,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                     for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
                 }
                 if (p.tma_store) {
-                    uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
-                    if (lane == 0) ptx::bulk_wait_read<1>();  // the store that used buf is done
+                    uint8_t* buf = ring_out ? smem + ((warp - 2) * kChunks + c) * 4096
+                                            : stage_buf + (chunk_ctr & 1u) * 4096;
+                    if (!ring_out && lane == 0) ptx::bulk_wait_read<1>();  // the store that used buf is done
                     __syncwarp();
                     if (row_lane) {
 #pragma unroll
@@ -402,7 +408,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
                         ptx::tma_store_3d(&p.tmap_c, ptx::smem_u32(buf), col0, tc.tm * BM + q * kRowsPerWarp, zc);
                         ptx::bulk_commit();
                     }
-                    ++chunk_ctr;
+                    if (!ring_out) ++chunk_ctr;
                 } else if (row_lane && row < p.M) {
                     float* dst = dst_row + col0;
                     if (act != NNJIT_EPI_NONE) {

@@ -402,6 +402,13 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                                   : n_part * 2 <= stage_slots ? 2 : 0;
             uint32_t stage_phase = 0;
             bool stage_ok = true;
+            // The pair's last segment (not a stream-K one): its MMAs have completed and no
+            // load follows, so the ring is idle and each warp stages every chunk in its own
+            // part of it, with no wait for earlier stores.
+            SegIter peek = st;
+            Seg after;
+            const bool ring_out = p.tma_store && !partial && !last && !seg_next(peek, after, p) &&
+                                  S * (int)kStageBytes >= 4 * kChunks * 4096;
             const int row_base = tc.tm2 * 256 + row_off + q * 32;
             const int row = row_base + lane;
             const float* bias = p.bias;
@@ -442,8 +449,8 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                     for (int j = 0; j < 32; ++j) v[j] += __shfl_sync(0xffffffffu, bl, j);
                 }
                 if (p.tma_store) {
-                    uint8_t* buf = stage_buf + (chunk_ctr & 1u) * 4096;
-                    if (lane == 0) ptx::bulk_wait_read<1>();
+                    uint8_t* buf = ring_out ? smem + (q * kChunks + c) * 4096 : stage_buf + (chunk_ctr & 1u) * 4096;
+                    if (!ring_out && lane == 0) ptx::bulk_wait_read<1>();
                     __syncwarp();
 #pragma unroll
                     for (int j = 0; j < 8; ++j)
@@ -458,7 +465,7 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
                         ptx::tma_store_3d(&p.tmap_c, ptx::smem_u32(buf), col0, row_base, tc.b);
                         ptx::bulk_commit();
                     }
-                    ++chunk_ctr;
+                    if (!ring_out) ++chunk_ctr;
                 } else if (row < p.M) {
                     float* dst = dst_row + col0;
                     if (p.act != NNJIT_EPI_NONE) {
