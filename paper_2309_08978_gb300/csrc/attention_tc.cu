@@ -39,6 +39,8 @@ namespace {
 __device__ int g_attn_watchdog;  // first expired wait's code (0: none)
 
 constexpr int kQ = 128;   // queries per work item (a CTA loops over items)
+// Bytes of Q, K, V and O that one group of problems may touch (about 3/4 of the 129 MB L2).
+constexpr long long kGroupL2Bytes = 96ll << 20;
 constexpr int kKV = 128;  // keys per block
 // Softmax warps per TMEM lane quarter.  Two: one (whole rows per thread, no exchange of
 // maxima) measured 60.7 against 55.4 us on the Llama prefill heads, four (d = 64) slower
@@ -71,6 +73,7 @@ struct Params {
     CUtensorMap tq, tk, tv, to;
     float* O;
     int Lq, Lk, causal, qblocks, batch;
+    int group;  // problems per item group (divides batch)
     float scale_log2;
 };
 
@@ -186,11 +189,16 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int shift = p.Lk - p.Lq;
     const int items = p.qblocks * p.batch;
-    // Work item -> (problem, first query, key blocks).  Items run heaviest first: with the
-    // causal mask the last query blocks see the most keys.
+    // Work item -> (problem, first query, key blocks).  The problems run in groups of
+    // p.group, sized on the host so that a group's Q, K, V and O fit in L2 together: the
+    // key and value blocks a problem's query blocks share are then read from DRAM once.
+    // Within a group the items run heaviest first: with the causal mask the last query
+    // blocks see the most keys.
     auto decode = [&](int it, int& bb, int& qq0) {
-        bb = it % p.batch;
-        qq0 = (p.qblocks - 1 - it / p.batch) * kQ;
+        const int per = p.group * p.qblocks;
+        const int g = it / per, r = it - g * per;
+        bb = g * p.group + r % p.group;
+        qq0 = (p.qblocks - 1 - r / p.group) * kQ;
         int kv_end = p.Lk;
         if (p.causal) kv_end = min(p.Lk, max(0, min(qq0 + kQ, p.Lq) - 1 + shift + 1));
         return (kv_end + kKV - 1) / kKV;
@@ -628,6 +636,12 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     p.causal = d.causal;
     p.qblocks = qblocks;
     p.batch = (int)d.batch;
+    // item groups: halve the group (while it divides the batch) until one group's Q, K, V
+    // (bf16) and O (f32) take at most kGroupL2Bytes
+    const long long per_problem = (long long)d.Lq * d.d * (2 + 4) + 2LL * d.Lk * d.d * 2;
+    long long group = d.batch;
+    while (group % 2 == 0 && group * per_problem > kGroupL2Bytes) group /= 2;
+    p.group = (int)group;
     p.scale_log2 = d.scale * 1.4426950408889634f;
     const int i = d.d == 64 ? 0 : 1;
     const int smem = i == 0 ? (int)Cfg<64>::kSmem : (int)Cfg<128>::kSmem;
