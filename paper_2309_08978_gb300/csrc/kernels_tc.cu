@@ -9,7 +9,8 @@
 // Warp roles (192 threads):
 //   warp 0      TMA producer: waits "empty[s]", arms "full[s]" with the stage bytes and
 //               issues the A and B tile loads.
-//   warp 1      TMEM owner and MMA issuer: waits "full[s]", issues BK/UMMA_K MMAs into
+//   warp 1      TMEM owner and MMA issuer (the whole warp waits and stays converged;
+//               one lane elected by elect.sync issues): waits "full[s]", issues BK/UMMA_K MMAs into
 //               accumulator buffer (tile & 1), commits to "empty[s]"; after the last
 //               k-block commits to "tmem_full[acc]".
 //   warps 2..5  epilogue: wait "tmem_full[acc]", tcgen05.ld 32 columns at a time, add
@@ -296,7 +297,9 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             kb_range(tc, kb0, kb1);
             const uint32_t acc = iter & 1u;
             const uint32_t acc_phase = (iter >> 1) & 1u;
-            if (!ptx::mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty)) {
+            // every lane waits; the warp leaves together if any lane's wait expired
+            if (!__all_sync(0xffffffffu,
+                            ptx::mbar_wait(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty))) {
                 ok = false;
                 break;
             }
@@ -304,38 +307,35 @@ __global__ void __launch_bounds__(kThreads, 1) tc_gemm_kernel(const __grid_const
             const uint32_t d_tmem = tmem_base + acc * BN;
             for (int g0 = kb0; g0 < kb1; g0 += KG) {
                 const int nk = min(KG, kb1 - g0);
-                if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull)) {
+                if (!__all_sync(0xffffffffu, ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull))) {
                     ok = false;
                     break;
                 }
                 ptx::tc_fence_after();
-                if (lane == 0) {
+                // the whole warp issues (one elected lane), so it stays converged
 #pragma unroll
-                    for (int j = 0; j < KG; ++j) {
-                        if (j < nk) {
-                            const uint64_t off = (uint64_t)((stage * kGroupBytes + j * kStageBytes) >> 4);
-                            const uint64_t ad = a_desc0 + off, bd = b_desc0 + off;
+                for (int j = 0; j < KG; ++j) {
+                    if (j < nk) {
+                        const uint64_t off = (uint64_t)((stage * kGroupBytes + j * kStageBytes) >> 4);
+                        const uint64_t ad = a_desc0 + off, bd = b_desc0 + off;
 #pragma unroll
-                            for (int kk = 0; kk < kKSteps; ++kk)
-                                ptx::mma_ss<kKind>(d_tmem, ad + 2 * kk, bd + kBStep * kk, kIdesc,
-                                                   (g0 > kb0 || j > 0 || kk > 0) ? 1u : 0u);
-                        }
+                        for (int kk = 0; kk < kKSteps; ++kk)
+                            ptx::mma_ss_elect<kKind>(d_tmem, ad + 2 * kk, bd + kBStep * kk, kIdesc,
+                                                     (g0 > kb0 || j > 0 || kk > 0) ? 1u : 0u);
                     }
-                    ptx::tc_commit(empty_bar(stage));
                 }
-                __syncwarp();
+                ptx::tc_commit_elect(empty_bar(stage));
                 if (++stage == S) {
                     stage = 0;
                     phase ^= 1u;
                 }
             }
             if (!ok) break;
-            if (lane == 0) ptx::tc_commit(tfull_bar(acc));
-            __syncwarp();
+            ptx::tc_commit_elect(tfull_bar(acc));
         }
-        // Drain: all MMAs this thread issued have completed before TMEM is released.
-        if (lane == 0) ptx::tc_commit(drain_bar);
+        // Drain: all MMAs the warp issued have completed before TMEM is released.
         __syncwarp();
+        ptx::tc_commit_elect(drain_bar);
         volatile int no_abort = 0;
         ptx::mbar_wait(drain_bar, 0, &no_abort, p.err, kErrDrain, ptx::kWaitLimitNs / 4);
     } else {

@@ -13,7 +13,8 @@
 //               barrier (whose producer arms it with both CTAs' bytes); a slot is
 //               refilled once the MMA has released it in this CTA ("empty[s]").
 //   warp 1      TMEM owner in each CTA (the pair allocation is done by one warp of each
-//               CTA); in the even CTA also the MMA issuer: waits "full[s]", issues 4 MMAs
+//               CTA); in the even CTA also the MMA issuer (the whole warp, converged; one
+//               lane elected by elect.sync issues): waits "full[s]", issues 4 MMAs
 //               per k-block, commits to "empty[s]" of both CTAs, and per tile to
 //               "tmem_full[acc]" of both CTAs.
 //   warps 2..5  epilogue of each CTA on its own 128 accumulator rows; each warp releases
@@ -312,39 +313,39 @@ __global__ void __launch_bounds__(kThreads, 1) tc2_gemm_kernel(const __grid_cons
             for (; ok && seg_next(st, it, p); ++iter) {
                 const uint32_t acc = NB == 2 ? (iter & 1u) : 0u;
                 const uint32_t acc_phase = NB == 2 ? ((iter >> 1) & 1u) : (iter & 1u);
-                if (!ptx::mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, abort_flag, p.err, kErrMmaTmemEmpty)) {
+                // every lane waits; the warp leaves together if any lane's wait expired
+                if (!__all_sync(0xffffffffu, ptx::mbar_wait_cluster(tempty_bar(acc), acc_phase ^ 1u, abort_flag,
+                                                                    p.err, kErrMmaTmemEmpty))) {
                     ok = false;
                     break;
                 }
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem_base + acc * BN;
                 for (int kb = it.kb0; kb < it.kb1; ++kb) {
-                    if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull)) {
+                    if (!__all_sync(0xffffffffu, ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrMmaFull))) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
-                    if (lane == 0) {
-                        const uint64_t off = (uint64_t)((stage * kStageBytes) >> 4);
-                        const uint64_t ad = a_desc0 + off, bd = b_desc0 + off;
+                    // the whole warp issues (one elected lane), so it stays converged
+                    const uint64_t off = (uint64_t)((stage * kStageBytes) >> 4);
+                    const uint64_t ad = a_desc0 + off, bd = b_desc0 + off;
 #pragma unroll
-                        for (int kk = 0; kk < kKSteps; ++kk)
-                            ptx::mma_pair<kKind>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdesc, (kb > it.kb0 || kk > 0) ? 1u : 0u);
-                        ptx::tc_commit_pair(empty_bar(stage), 0x3);  // frees the slot in both CTAs
-                    }
-                    __syncwarp();
+                    for (int kk = 0; kk < kKSteps; ++kk)
+                        ptx::mma_pair_elect<kKind>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdesc,
+                                                   (kb > it.kb0 || kk > 0) ? 1u : 0u);
+                    ptx::tc_commit_pair_elect(empty_bar(stage), 0x3);  // frees the slot in both CTAs
                     if (++stage == S) {
                         stage = 0;
                         phase ^= 1u;
                     }
                 }
                 if (!ok) break;
-                if (lane == 0) ptx::tc_commit_pair(tfull_bar(acc), 0x3);
-                __syncwarp();
+                ptx::tc_commit_pair_elect(tfull_bar(acc), 0x3);
             }
-            // Drain: all pair MMAs this thread issued have completed before TMEM is freed.
-            if (lane == 0) ptx::tc_commit_pair(drain_bar, 0x1);
+            // Drain: all pair MMAs the warp issued have completed before TMEM is freed.
             __syncwarp();
+            ptx::tc_commit_pair_elect(drain_bar, 0x1);
             volatile int no_abort = 0;
             ptx::mbar_wait(drain_bar, 0, &no_abort, p.err, kErrDrain, ptx::kWaitLimitNs / 4);
         }
