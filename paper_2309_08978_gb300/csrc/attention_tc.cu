@@ -5,7 +5,8 @@
 //   warp 0     TMA producer: an item's Q tile (two Q buffers), then its key and value
 //              blocks of 128 rows through separate key and value rings (128-byte
 //              swizzle; keys K-major, values MN-major), values one key block behind;
-//   warp 1     allocates TMEM and issues, from one thread, S_g = Q K_g^T (M = 128,
+//   warp 1     allocates TMEM and issues (the warp converged, one lane elected by
+//              elect.sync) S_g = Q K_g^T (M = 128,
 //              N = 128, K = d) into TMEM score buffer g % 2, a block ahead, and
 //              O += P_g V_g (M = 128, N = d, K = 128) with P_g read from TMEM as the A
 //              operand, into the item's TMEM output;
@@ -314,77 +315,81 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
         }
     } else if (warp == 1) {
         // ------------------------------------------------------------ MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t kIdescS = ptx::instr_desc(1u, false, kQ, kKV);
-            constexpr uint32_t kIdescO = ptx::instr_desc(1u, true, kQ, D);
-            uint32_t q_addr = sQ(0);  // the current item's Q tile
-            // S_g = Q K_g^T into score buffer g % 2
-            auto issue_s = [&](int g) -> bool {
-                const int sb = g & 1, st = g % SK;
-                // Score buffer g % 2 is free: the softmax read S_{g-2} before releasing P_{g-2},
-                // and P_{g-2} V_{g-2} was issued (after that release) before this product.
-                if (!ptx::mbar_wait(k_full(st), (uint32_t)((g / SK) & 1), abort_flag, err, kErrMmaKv)) return false;
-                ptx::tc_fence_after();
-                const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
+        // The whole warp runs the loop converged: every lane waits (the results are voted,
+        // so the warp leaves as one) and elect.sync picks the lane that issues.
+        auto wait_all = [&](uint32_t bar, uint32_t parity, int code) {
+            return __all_sync(0xffffffffu, ptx::mbar_wait(bar, parity, abort_flag, err, code));
+        };
+        constexpr uint32_t kIdescS = ptx::instr_desc(1u, false, kQ, kKV);
+        constexpr uint32_t kIdescO = ptx::instr_desc(1u, true, kQ, D);
+        uint32_t q_addr = sQ(0);  // the current item's Q tile
+        // S_g = Q K_g^T into score buffer g % 2
+        auto issue_s = [&](int g) -> bool {
+            const int sb = g & 1, st = g % SK;
+            // Score buffer g % 2 is free: the softmax read S_{g-2} before releasing P_{g-2},
+            // and P_{g-2} V_{g-2} was issued (after that release) before this product.
+            if (!wait_all(k_full(st), (uint32_t)((g / SK) & 1), kErrMmaKv)) return false;
+            ptx::tc_fence_after();
+            const uint32_t d_tmem = tmem + (uint32_t)sb * kKV;
 #pragma unroll
-                for (int kb = 0; kb < kDB; ++kb) {
-                    const uint64_t ad = ptx::smem_desc(q_addr + kb * 16384u, 16, 1024);
-                    const uint64_t bd = ptx::smem_desc(sK(st) + kb * 16384u, 16, 1024);
+            for (int kb = 0; kb < kDB; ++kb) {
+                const uint64_t ad = ptx::smem_desc(q_addr + kb * 16384u, 16, 1024);
+                const uint64_t bd = ptx::smem_desc(sK(st) + kb * 16384u, 16, 1024);
 #pragma unroll
-                    for (int kk = 0; kk < 4; ++kk)
-                        ptx::mma_ss<0>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdescS, (kb | kk) ? 1u : 0u);
-                }
-                ptx::tc_commit(s_full(sb));
-                ptx::tc_commit(k_empty(st));  // the key slot is free once S_g has completed
-                return true;
-            };
-            int g = 0, nq = 0;
-            bool ok = true;
-            for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
-                int bb, qq0;
-                const int nblocks = decode(it, bb, qq0);
-                if (nblocks == 0) continue;
-                const int qi = nq % QB;
-                if (!ptx::mbar_wait(q_full(qi), (uint32_t)(nq / QB) & 1u, abort_flag, err, kErrMmaQ)) break;
-                q_addr = sQ(qi);
-                ++nq;
-                ptx::tc_fence_after();
-                if (!issue_s(g)) break;
-                for (int j = 0; j < nblocks; ++j, ++g) {
-                    if (j + 1 < nblocks) {
-                        if (!issue_s(g + 1)) {
-                            ok = false;
-                            break;
-                        }
-                    } else {
-                        ptx::tc_commit(q_empty(qi));  // every score MMA of the item is issued
-                    }
-                    const int st = g % SV;
-                    if (!ptx::mbar_wait(p_full(g & 1), (g >> 1) & 1, abort_flag, err, kErrMmaP) ||
-                        !ptx::mbar_wait(v_full(st), (uint32_t)((g / SV) & 1), abort_flag, err, kErrMmaKv)) {
+                for (int kk = 0; kk < 4; ++kk)
+                    ptx::mma_ss_elect<0>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdescS, (kb | kk) ? 1u : 0u);
+            }
+            ptx::tc_commit_elect(s_full(sb));
+            ptx::tc_commit_elect(k_empty(st));  // the key slot is free once S_g has completed
+            return true;
+        };
+        int g = 0, nq = 0;
+        bool ok = true;
+        for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+            int bb, qq0;
+            const int nblocks = decode(it, bb, qq0);
+            if (nblocks == 0) continue;
+            const int qi = nq % QB;
+            if (!wait_all(q_full(qi), (uint32_t)(nq / QB) & 1u, kErrMmaQ)) break;
+            q_addr = sQ(qi);
+            ++nq;
+            ptx::tc_fence_after();
+            if (!issue_s(g)) break;
+            for (int j = 0; j < nblocks; ++j, ++g) {
+                if (j + 1 < nblocks) {
+                    if (!issue_s(g + 1)) {
                         ok = false;
                         break;
                     }
-                    ptx::tc_fence_after();
-                    const uint32_t o_tmem = tmem + 2u * kKV;  // O accumulates over the item's blocks
-                    const uint32_t p_tmem = o_tmem + D + (uint32_t)(g & 1) * (kKV / 2);  // P_g, bf16 pairs
-#pragma unroll
-                    for (int kb = 0; kb < 2; ++kb) {
-                        const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
-#pragma unroll
-                        for (int kk = 0; kk < 4; ++kk)  // keys kb * 64 + kk * 16 .. + 15: 8 columns of P
-                            ptx::mma_ts_f16(o_tmem, p_tmem + kb * 32 + kk * 8, bd + 128 * kk, kIdescO,
-                                            (j | kb | kk) ? 1u : 0u);
-                    }
-                    ptx::tc_commit(o_full(g & 1));
-                    ptx::tc_commit(v_empty(st));
+                } else {
+                    ptx::tc_commit_elect(q_empty(qi));  // every score MMA of the item is issued
                 }
+                const int st = g % SV;
+                if (!wait_all(p_full(g & 1), (g >> 1) & 1, kErrMmaP) ||
+                    !wait_all(v_full(st), (uint32_t)((g / SV) & 1), kErrMmaKv)) {
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+                const uint32_t o_tmem = tmem + 2u * kKV;  // O accumulates over the item's blocks
+                const uint32_t p_tmem = o_tmem + D + (uint32_t)(g & 1) * (kKV / 2);  // P_g, bf16 pairs
+#pragma unroll
+                for (int kb = 0; kb < 2; ++kb) {
+                    const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
+#pragma unroll
+                    for (int kk = 0; kk < 4; ++kk)  // keys kb * 64 + kk * 16 .. + 15: 8 columns of P
+                        ptx::mma_ts_f16_elect(o_tmem, p_tmem + kb * 32 + kk * 8, bd + 128 * kk, kIdescO,
+                                              (j | kb | kk) ? 1u : 0u);
+                }
+                ptx::tc_commit_elect(o_full(g & 1));
+                ptx::tc_commit_elect(v_empty(st));
             }
-            // every MMA issued here has completed before TMEM is freed
-            ptx::tc_commit(drain_bar);
-            volatile int no_abort = 0;
-            ptx::mbar_wait(drain_bar, 0, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
         }
+        // every MMA issued here has completed before TMEM is freed
+        __syncwarp();
+        ptx::tc_commit_elect(drain_bar);
+        volatile int no_abort = 0;
+        ptx::mbar_wait(drain_bar, 0, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
     } else {
         // ------------------------------------------------------------ softmax warps
         const int q = warp & 3;                 // TMEM lane quarter

@@ -195,7 +195,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
             for (int m = 0; m < MAXM; ++m) acc[r][m] = 0.0f;
         bool ok = true;
         for (int c = w.c0; c < w.c1; ++c) {
-            if (!ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrGemvFull)) {
+            // the warp's lanes agree on the outcome, so the warp stays converged
+            if (!__all_sync(0xffffffffu, ptx::mbar_wait(full_bar(stage), phase, abort_flag, p.err, kErrGemvFull))) {
                 ok = false;
                 break;
             }
@@ -222,8 +223,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_tma_kernel(const __grid_cons
                     }
                 }
             }
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(empty_bar(stage));
+            ptx::mbar_arrive_elect(empty_bar(stage));  // after every lane's reads of the stage
             if (++stage == S) {
                 stage = 0;
                 phase ^= 1u;

@@ -320,8 +320,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_w4_kernel(const __grid_const
                     acc[r][3] = fmaf(s1, d[3] + e[3], acc[r][3]);
                 }
             }
-            __syncwarp();
-            if (lane == 0) ptx::mbar_arrive(empty_bar(stage));
+            ptx::mbar_arrive_elect(empty_bar(stage));  // after every lane's reads of the stage
             if (++stage == S) {
                 stage = 0;
                 phase ^= 1u;
