@@ -91,8 +91,7 @@ def test_kernel_key_format():
 
 
 def test_traffic_table_lookup():
-    assert bench.lookup_traffic("tc tf32 1x512x768x3072 NK bm128 bn256 bk32 st4 split8 red0 rast1") > 0
-    assert bench.lookup_traffic("attention tcgen05 d128 B128 Lq1024 Lk1024 causal") > 0
+    assert bench.lookup_traffic("tc bf16 1x4096x22016x4096 NK bm256 bn256 bk64 st6 split1 red2 rast0") > 0
     assert bench.lookup_traffic("no such kernel") is None
     # every entry is "key | integer bytes"
     path = os.path.join(bench.ROOT, "profiles", "dram_traffic.txt")
