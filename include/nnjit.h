@@ -181,7 +181,8 @@ typedef struct {
     int64_t predicted_cost;  /* model cost used for ordering (arbitrary units, lower first) */
     int32_t reduce;          /* split-K reduction: 0 = partials in the plan's workspace, summed
                                 by a second kernel; 1 = TC only, inside a thread-block cluster
-                                of split_k CTAs through distributed shared memory */
+                                of split_k CTAs through distributed shared memory; 2 = CTA
+                                pairs only, stream-K over the last waves (split_k 1) */
     int32_t cluster_m;       /* TC only: 2 = a cluster of two CTAs on two SMs computing one
                                 256-row tile (bm = 256) with tcgen05 cta_group::2 MMAs;
                                 else 1 */
@@ -196,7 +197,8 @@ typedef struct nnjit_plan_s* nnjit_plan;
  * the one value kept.  They act on the tensor-core family only:
  *   raster     tile order: 0 = M fastest, 1 = N fastest;
  *   kgroup     k-blocks per ring slot (candidate bk / one 128-byte k-block): 1 or 2;
- *   reduce     split-K reduction: 0 = second kernel, 1 = inside a cluster (DSMEM).
+ *   reduce     split-K reduction: 0 = second kernel, 1 = inside a cluster (DSMEM),
+ *              2 = CTA-pair stream-K over the last waves.
  * A fixed value removes a candidate only where the same candidate with the fixed value
  * (every other searched field equal: bm, bn, split_k and the other two settings) is
  * in the space, so a setting never empties the space and never removes the only legal

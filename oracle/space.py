@@ -527,7 +527,7 @@ def _gemv(p, lim):
 
 
 SETTING_AXES = ("raster", "kgroup", "reduce")
-SETTING_RANGE = {"raster": (0, 1), "kgroup": (1, 2), "reduce": (0, 1)}
+SETTING_RANGE = {"raster": (0, 1), "kgroup": (1, 2), "reduce": (0, 2)}
 
 
 def setting_value(p: Problem, c: dict, axis: str):

@@ -642,7 +642,8 @@ int setting_of(const nnjit_settings& s, int axis) {
 }
 
 bool settings_valid(const nnjit_settings& s, std::string* err) {
-    const int lo[kSettingAxes] = {0, 1, 0}, hi[kSettingAxes] = {1, 2, 1};
+    // reduce: 0 second kernel, 1 cluster (DSMEM), 2 CTA-pair stream-K
+    const int lo[kSettingAxes] = {0, 1, 0}, hi[kSettingAxes] = {1, 2, 2};
     const char* names[kSettingAxes] = {"raster", "kgroup", "reduce"};
     for (int a = 0; a < kSettingAxes; ++a) {
         const int v = setting_of(s, a);

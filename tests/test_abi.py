@@ -128,7 +128,12 @@ def test_settings_roundtrip_and_validation(lib):
     try:
         nj.nnjit_settings_set({"raster": 1, "reduce": 0})
         assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": 0}
-        for bad in ({"kgroup": 0}, {"kgroup": 3}, {"raster": 2}, {"reduce": -2}, {"reduce": 5}):
+        # every reduction a candidate can carry is a legal fixed value (a settings study may
+        # vote for the CTA-pair stream-K one, 2)
+        nj.nnjit_settings_set({"raster": 1, "reduce": 2})
+        assert nj.nnjit_settings_get() == {"raster": 1, "kgroup": -1, "reduce": 2}
+        nj.nnjit_settings_set({"raster": 1, "reduce": 0})
+        for bad in ({"kgroup": 0}, {"kgroup": 3}, {"raster": 2}, {"reduce": -2}, {"reduce": 3}, {"reduce": 5}):
             with pytest.raises(nj.NnjitError) as ei:
                 nj.nnjit_settings_set(bad)
             assert ei.value.status == nj.NNJIT_ERR_INVALID_ARG
