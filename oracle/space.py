@@ -29,7 +29,7 @@ INVALID_ARG, UNSUPPORTED = 1, 2
 # model constants (readings of the paper's unstated relaxation ratio and cost model)
 FEED_BYTES_PER_CLK = 64       # per-SM L2 -> SM operand feed
 HBM_BYTES_PER_CLK = 3500      # chip-wide HBM bytes per SM clock
-LAUNCH_CLK = 2000             # one extra kernel launch
+LAUNCH_CLK = 4000             # one extra kernel launch (the split-K sum after the GEMM)
 REG_SHARE_PCT = 50            # Table 1's Reg_thread is this share of a thread's registers
 TC_REGS = 176                 # registers per thread of the tensor-core kernel (ptxas: 72-173)
 TC_THREADS = 192
