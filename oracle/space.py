@@ -179,7 +179,9 @@ def block_core(lim, regs, threads, smem, tmem):
     """Table 1's Block_core with the Blackwell resources: the fewest CTAs allowed by the
     register file, shared memory (the L1Limit), warps, tensor-memory columns, blocks."""
     reg_limit = lim["regs_per_sm"] // max(1, regs * threads)
-    l1_limit = lim["smem_per_sm"] // smem if smem > 0 else lim["max_blocks_per_sm"]
+    # each resident CTA also holds the SM's per-block shared-memory reservation
+    reserved = max(0, lim["smem_per_sm"] - lim["smem_per_block_optin"])
+    l1_limit = lim["smem_per_sm"] // (smem + reserved) if smem > 0 else lim["max_blocks_per_sm"]
     warp_limit = (lim["max_threads_per_sm"] // 32) // max(1, threads // 32)
     tmem_limit = lim["tmem_cols_per_sm"] // tmem if tmem > 0 else lim["max_blocks_per_sm"]
     return min(reg_limit, l1_limit, warp_limit, tmem_limit, lim["max_blocks_per_sm"])

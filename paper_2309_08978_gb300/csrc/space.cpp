@@ -23,7 +23,10 @@ int min4(int a, int b, int c, int d) { return std::min(std::min(a, b), std::min(
 // of the per-resource limits (registers, shared memory = L1Limit, warps, TMEM, blocks).
 int blocks_per_core(const nnjit_device_limits& L, int regs, int threads, int smem, int tmem) {
     const int reg_lim = L.regs_per_sm / std::max(1, regs * threads);
-    const int smem_lim = smem > 0 ? L.smem_per_sm / smem : L.max_blocks_per_sm;
+    // every resident CTA also holds the per-block reservation of the SM's shared memory
+    // (the difference between the SM's shared memory and the largest opt-in per block)
+    const int reserved = std::max(0, L.smem_per_sm - L.smem_per_block_optin);
+    const int smem_lim = smem > 0 ? L.smem_per_sm / (smem + reserved) : L.max_blocks_per_sm;
     const int warp_lim = (L.max_threads_per_sm / 32) / std::max(1, threads / 32);
     const int tmem_lim = tmem > 0 ? L.tmem_cols_per_sm / tmem : L.max_blocks_per_sm;
     return std::min(min4(reg_lim, smem_lim, warp_lim, tmem_lim), L.max_blocks_per_sm);
