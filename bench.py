@@ -407,11 +407,13 @@ def run_attention(args, name):
         Q, K, V, O = sets[k % nsets]
         nj.nnjit_attention(Q, K, V, O, causal=causal, scale=scale, stream=stream)
 
-    # the JIT phase: time both kernels on these buffers, keep the faster (kernel AUTO)
+    # the JIT phase: time the three kernels on these buffers, keep the fastest (kernel AUTO)
     t0 = time.perf_counter()
-    (t_tc, t_mma), chosen = nj.nnjit_attention_tune(Q0, K0, V0, sets[0][3], causal=causal, scale=scale, reps=10)
+    (t_tc, t_mma, t_tc2), chosen = nj.nnjit_attention_tune(Q0, K0, V0, sets[0][3], causal=causal, scale=scale,
+                                                           reps=10)
     tune = {"plan_ms": round(1000 * (time.perf_counter() - t0), 2), "tcgen05_us": round(t_tc, 3),
-            "mma_us": round(t_mma, 3), "chosen": {1: "tcgen05", 2: "mma"}[chosen]}
+            "mma_us": round(t_mma, 3), "tcgen05_2t_us": round(t_tc2, 3),
+            "chosen": {1: "tcgen05", 2: "mma", 3: "tcgen05_2t"}[chosen]}
     with torch.cuda.stream(stream):
         launch(0)
     torch.cuda.synchronize()

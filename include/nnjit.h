@@ -408,14 +408,21 @@ nnjit_status nnjit_plan_destroy(nnjit_plan p);
  * (Lq = 0 is a no-op), batch >= 1, Lq, Lk, batch < 2^31.  `kernel` selects the
  * implementation: NNJIT_ATTN_AUTO (0) and NNJIT_ATTN_TCGEN05 (1) run the tensor-memory
  * kernel (128 queries per CTA, scores and outputs in TMEM, bounded waits), NNJIT_ATTN_MMA
- * (2) the warp-level MMA kernel (64 queries per CTA, no waits); AUTO takes the kernel that
- * nnjit_attention_tune recorded as faster for the same (batch, Lq, Lk, d, causal) on the
- * current device, else the tensor-memory kernel.  INVALID_ARG for a bad
+ * (2) the warp-level MMA kernel (64 queries per CTA, no waits), NNJIT_ATTN_TCGEN05_2T (3)
+ * the tensor-memory kernel with two 128-query tiles per CTA sharing each key and value
+ * block (the tensor cores alternate between the tiles; bounded waits); AUTO takes the
+ * kernel that nnjit_attention_tune recorded as fastest for the same (batch, Lq, Lk, d,
+ * causal) on the current device, else the tensor-memory kernel (1).  INVALID_ARG for a bad
  * descriptor or NULL pointer, UNSUPPORTED for another d or unaligned pointers.
  * Asynchronous on `stream`; allocates nothing.  An expired wait inside the tensor-memory
  * kernel is reported by nnjit_attention_check.
  */
-typedef enum { NNJIT_ATTN_AUTO = 0, NNJIT_ATTN_TCGEN05 = 1, NNJIT_ATTN_MMA = 2 } nnjit_attention_kernel;
+typedef enum {
+    NNJIT_ATTN_AUTO = 0,
+    NNJIT_ATTN_TCGEN05 = 1,
+    NNJIT_ATTN_MMA = 2,
+    NNJIT_ATTN_TCGEN05_2T = 3
+} nnjit_attention_kernel;
 
 typedef struct {
     int64_t batch, Lq, Lk, d;
@@ -440,10 +447,11 @@ nnjit_status nnjit_attention_check(void);
  * JIT selection for fused attention (Sec. 3: evaluate the candidates on the device, keep
  * the fastest): runs each kernel on the caller's buffers (O is overwritten; the inputs
  * are only read), once to warm up and then `reps` (1..100) times per trial for three
- * trials, on a stream of its own, and records the one with the lower median time for
+ * trials, on a stream of its own, and records the one with the lowest median time for
  * (batch, Lq, Lk, d, causal) on the current device, where later calls with kernel = AUTO
- * find it.  *times_us (may be NULL) receives the two medians (tensor-memory, warp-MMA),
- * *chosen (may be NULL) the recorded kernel.  Synchronous.  Errors as nnjit_attention;
+ * find it.  *times_us (may be NULL; three doubles) receives the medians of kernels 1, 2
+ * and 3 (tensor-memory, warp-MMA, tensor-memory with two tiles), *chosen (may be NULL) the
+ * recorded kernel.  Synchronous.  Errors as nnjit_attention;
  * NNJIT_ERR_TIMEOUT if a tensor-memory wait expired while timing.
  */
 nnjit_status nnjit_attention_tune(const nnjit_attention_desc* desc, const void* Q, const void* K,

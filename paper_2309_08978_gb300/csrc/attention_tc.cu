@@ -596,6 +596,441 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
     if (warp == 1) ptx::tmem_dealloc(tmem, 512);
 }
 
+// ---------------------------------------------------------------------------------
+// Kernel 3: two query tiles per work item.  An item is 256 queries of one problem, tiles
+// A (rows 0..127) and B (rows 128..255), sharing every key and value block.  The tensor
+// cores alternate between the tiles: while the softmax warps of tile A turn S_A(j) into
+// P_A(j), the MMAs compute S_B(j) or P_B V, and the other way round.  TMEM holds S_A, S_B,
+// O_A and O_B (512 columns with d = 128); P_X(j) is written over the columns of S_X(j)
+// it was computed from (the softmax has read them), and S_X(j + 1) is issued only after
+// P_X(j) V(j), so the in-order tensor pipe reads P_X(j) before overwriting it.  Each
+// softmax thread holds a whole row (128 scores): no exchange of row maxima.
+//   warp 0     TMA producer: both Q tiles of an item (one barrier), then its key and
+//              value blocks through the key and value rings;
+//   warp 1     TMEM owner and MMA issuer (converged warp, elected lane);
+//   warps 2-5  softmax of tile A (TMEM lane quarter = warp % 4), warps 6-9 of tile B.
+// Every wait is bounded, as in kernel 1.
+template <int D>
+struct Cfg2 {
+    static constexpr int kKStages = 2;
+    static constexpr int kVStages = 2;
+    static constexpr uint32_t kQBytes = kQ * D * 2;  // one tile
+    static constexpr uint32_t kKBytes = kKV * D * 2;
+    static constexpr uint32_t kVBytes = kKV * D * 2;
+    static constexpr uint32_t kOStage = 4096;
+    static constexpr uint32_t kSmem = 1024 + 2 * kQBytes + kKStages * kKBytes + kVStages * kVBytes + 8 * kOStage;
+};
+
+template <int D>
+__global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_constant__ Params p) {
+    using C = Cfg2<D>;
+    constexpr int SK = C::kKStages, SV = C::kVStages;
+    constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
+    extern __shared__ uint8_t raw[];
+    // q_full, q_empty, drain, k_full/k_empty (SK each), v_full/v_empty (SV each), then per
+    // tile X: s_full[X], p_full[X], o_full[X]
+    __shared__ __align__(8) uint64_t bars[3 + 2 * SK + 2 * SV + 6];
+    __shared__ uint32_t tmem_slot;
+    __shared__ int abort_word;
+    volatile int* abort_flag = &abort_word;
+    int* err = &g_attn_watchdog;
+
+    const uint32_t base = (ptx::smem_u32(raw) + 1023u) & ~1023u;
+    auto sQ = [&](int x) { return base + (uint32_t)x * C::kQBytes; };
+    const uint32_t sKR = base + 2 * C::kQBytes, sVR = sKR + SK * C::kKBytes;
+    auto sK = [&](int s) { return sKR + (uint32_t)s * C::kKBytes; };
+    auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
+    const uint32_t sO = sVR + SV * C::kVBytes;  // 8 output staging tiles
+    auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
+    const uint32_t q_full = bar(0), q_empty = bar(1), drain_bar = bar(2);
+    auto k_full = [&](int s) { return bar(3 + s); };
+    auto k_empty = [&](int s) { return bar(3 + SK + s); };
+    constexpr int kVB = 3 + 2 * SK, kXB = kVB + 2 * SV;
+    auto v_full = [&](int s) { return bar(kVB + s); };
+    auto v_empty = [&](int s) { return bar(kVB + SV + s); };
+    auto s_full = [&](int x) { return bar(kXB + x); };
+    auto p_full = [&](int x) { return bar(kXB + 2 + x); };
+    auto o_full = [&](int x) { return bar(kXB + 4 + x); };
+    // TMEM: S_A at column 0, S_B at 128, O_A at 256, O_B at 256 + D
+    auto s_col = [&](int x) { return (uint32_t)x * kKV; };
+    auto o_col = [&](int x) { return 2u * kKV + (uint32_t)x * D; };
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int shift = p.Lk - p.Lq;
+    const int items = p.qblocks * p.batch;  // qblocks: 256-query blocks here
+    // Work item -> (problem, first query) and the key blocks tiles A and B see: as kernel
+    // 1's order (problem groups that fit in L2, heaviest first within a group).
+    auto decode = [&](int it, int& bb, int& qq0, int& na, int& nb) {
+        const int per = p.group * p.qblocks;
+        const int g = it / per, r = it - g * per;
+        bb = g * p.group + r % p.group;
+        qq0 = (p.qblocks - 1 - r / p.group) * (2 * kQ);
+        auto blocks = [&](int q0) {  // key blocks the rows q0 .. q0 + 127 (below Lq) see
+            if (q0 >= p.Lq) return 0;
+            int kv_end = p.Lk;
+            if (p.causal) kv_end = min(p.Lk, max(0, min(q0 + kQ, p.Lq) - 1 + shift + 1));
+            return (kv_end + kKV - 1) / kKV;
+        };
+        na = blocks(qq0);
+        nb = blocks(qq0 + kQ);
+    };
+
+    if (threadIdx.x == 0) {
+        ptx::mbar_init(q_full, 1);
+        ptx::mbar_init(q_empty, 1);
+        ptx::mbar_init(drain_bar, 1);
+        for (int s = 0; s < SK; ++s) {
+            ptx::mbar_init(k_full(s), 1);
+            ptx::mbar_init(k_empty(s), 1);
+        }
+        for (int s = 0; s < SV; ++s) {
+            ptx::mbar_init(v_full(s), 1);
+            ptx::mbar_init(v_empty(s), 1);
+        }
+        for (int x = 0; x < 2; ++x) {
+            ptx::mbar_init(s_full(x), 1);
+            ptx::mbar_init(p_full(x), 4);  // one arrival per softmax warp of the tile
+            ptx::mbar_init(o_full(x), 1);
+        }
+        abort_word = 0;
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(&tmem_slot), 512);
+        ptx::tmem_relinquish();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = tmem_slot;
+    ptx::griddep_wait();
+    if (threadIdx.x == 0) ptx::griddep_launch_dependents();
+
+    if (warp == 0) {
+        // ------------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            ptx::prefetch_tmap(&p.tq);
+            ptx::prefetch_tmap(&p.tk);
+            ptx::prefetch_tmap(&p.tv);
+            uint32_t k_armed = 0, k_par = 0, v_armed = 0, v_par = 0, q_armed = 0, q_par = 0;
+            int g = 0, nq = 0;  // key blocks and items loaded so far
+            bool ok = true;
+            int gv = -1, vb = 0, vk0 = 0;  // the value block issued one key block behind
+            auto load_v = [&]() -> bool {
+                const int st = gv % SV;
+                const uint32_t ph = (uint32_t)(gv / SV) & 1u;
+                if (!ptx::mbar_wait(v_empty(st), ph ^ 1u, abort_flag, err, kErrProd)) return false;
+                ptx::mbar_arrive_expect_tx(v_full(st), C::kVBytes);
+                for (int kb = 0; kb < 2; ++kb)       // 64 keys per K-block of P V
+                    for (int a = 0; a < kDB; ++a)    // 64 columns of d per swizzle atom
+                        ptx::tma_load_3d(sV(st) + kb * (D * 128u) + a * 8192u, &p.tv, a * 64, vk0 + kb * 64, vb,
+                                         v_full(st));
+                v_armed |= 1u << st;
+                v_par = (v_par & ~(1u << st)) | (ph << st);
+                gv = -1;
+                return true;
+            };
+            for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+                int bb, qq0, na, nb;
+                decode(it, bb, qq0, na, nb);
+                const int nmax = max(na, nb);
+                if (nmax == 0) continue;
+                // both Q tiles are free once every score MMA of the previous item has completed
+                const uint32_t qph = (uint32_t)nq & 1u;
+                if (nq >= 1 && !ptx::mbar_wait(q_empty, qph ^ 1u, abort_flag, err, kErrProd)) break;
+                ptx::mbar_arrive_expect_tx(q_full, 2 * C::kQBytes);
+                for (int x = 0; x < 2; ++x)
+                    for (int kb = 0; kb < kDB; ++kb)
+                        ptx::tma_load_3d(sQ(x) + kb * 16384u, &p.tq, kb * 64, qq0 + x * kQ, bb, q_full);
+                q_armed = 1;
+                q_par = qph;
+                ++nq;
+                for (int j = 0; j < nmax; ++j, ++g) {
+                    const int st = g % SK;
+                    const uint32_t ph = (uint32_t)(g / SK) & 1u;
+                    if (!ptx::mbar_wait(k_empty(st), ph ^ 1u, abort_flag, err, kErrProd)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::mbar_arrive_expect_tx(k_full(st), C::kKBytes);
+                    for (int kb = 0; kb < kDB; ++kb)
+                        ptx::tma_load_3d(sK(st) + kb * 16384u, &p.tk, kb * 64, j * kKV, bb, k_full(st));
+                    k_armed |= 1u << st;
+                    k_par = (k_par & ~(1u << st)) | (ph << st);
+                    if (gv >= 0 && !load_v()) {
+                        ok = false;
+                        break;
+                    }
+                    gv = g;
+                    vb = bb;
+                    vk0 = j * kKV;
+                }
+                if (ok && gv >= 0 && !load_v()) ok = false;  // the item's last value block
+            }
+            // drain: every copy issued here has landed before the CTA may exit
+            volatile int no_abort = 0;
+            if (q_armed) ptx::mbar_wait(q_full, q_par, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int st = 0; st < SK; ++st)
+                if (k_armed & (1u << st))
+                    ptx::mbar_wait(k_full(st), (k_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int st = 0; st < SV; ++st)
+                if (v_armed & (1u << st))
+                    ptx::mbar_wait(v_full(st), (v_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------------------ MMA issuer
+        auto wait_all = [&](uint32_t b, uint32_t parity, int code) {
+            return __all_sync(0xffffffffu, ptx::mbar_wait(b, parity, abort_flag, err, code));
+        };
+        constexpr uint32_t kIdescS = ptx::instr_desc(1u, false, kQ, kKV);
+        constexpr uint32_t kIdescO = ptx::instr_desc(1u, true, kQ, D);
+        // S_X = Q_X K^T of the key block in slot st into tile X's score columns
+        auto issue_s = [&](int x, int st) {
+            const uint32_t d_tmem = tmem + s_col(x);
+#pragma unroll
+            for (int kb = 0; kb < kDB; ++kb) {
+                const uint64_t ad = ptx::smem_desc(sQ(x) + kb * 16384u, 16, 1024);
+                const uint64_t bd = ptx::smem_desc(sK(st) + kb * 16384u, 16, 1024);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)
+                    ptx::mma_ss_elect<0>(d_tmem, ad + 2 * kk, bd + 2 * kk, kIdescS, (kb | kk) ? 1u : 0u);
+            }
+            ptx::tc_commit_elect(s_full(x));
+        };
+        // O_X += P_X V of the value block in slot st (P_X: bf16 pairs over S_X's columns)
+        auto issue_pv = [&](int x, int st, bool acc) {
+            const uint32_t o_tmem = tmem + o_col(x), p_tmem = tmem + s_col(x);
+#pragma unroll
+            for (int kb = 0; kb < 2; ++kb) {
+                const uint64_t bd = ptx::smem_desc(sV(st) + kb * (D * 128u), 8192, 1024, ptx::kLayoutSw128);
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk)  // keys kb * 64 + kk * 16 .. + 15: 8 columns of P
+                    ptx::mma_ts_f16_elect(o_tmem, p_tmem + kb * 32 + kk * 8, bd + 128 * kk, kIdescO,
+                                          (acc || kb || kk) ? 1u : 0u);
+            }
+            ptx::tc_commit_elect(o_full(x));
+        };
+        int g = 0, nq = 0;
+        int gx[2] = {0, 0};  // blocks of tile A / B so far (the parity of its barriers)
+        bool ok = true;
+        for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+            int bb, qq0, na, nb;
+            decode(it, bb, qq0, na, nb);
+            const int n[2] = {na, nb};
+            const int nmax = max(na, nb);
+            if (nmax == 0) continue;
+            if (!wait_all(q_full, (uint32_t)nq & 1u, kErrMmaQ)) break;
+            ++nq;
+            ptx::tc_fence_after();
+            // block 0's score products
+            if (!wait_all(k_full(g % SK), (uint32_t)((g / SK) & 1), kErrMmaKv)) break;
+            ptx::tc_fence_after();
+            for (int x = 0; x < 2; ++x)
+                if (n[x] > 0) issue_s(x, g % SK);
+            ptx::tc_commit_elect(k_empty(g % SK));
+            if (nmax == 1) ptx::tc_commit_elect(q_empty);
+            for (int j = 0; j < nmax; ++j, ++g) {
+                const int sv = g % SV, sk1 = (g + 1) % SK;
+                if (!wait_all(v_full(sv), (uint32_t)((g / SV) & 1), kErrMmaKv)) {
+                    ok = false;
+                    break;
+                }
+                const bool next = j + 1 < nmax;
+                bool k_ready = false;  // key block j + 1 landed (waited for before its first use)
+                for (int x = 0; x < 2 && ok; ++x) {
+                    if (j >= n[x]) continue;
+                    if (!wait_all(p_full(x), (uint32_t)gx[x] & 1u, kErrMmaP)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    issue_pv(x, sv, j > 0);
+                    ++gx[x];
+                    if (j + 1 < n[x]) {  // after P_X(j) V: the in-order pipe reads P_X(j) first
+                        if (!k_ready && !wait_all(k_full(sk1), (uint32_t)(((g + 1) / SK) & 1), kErrMmaKv)) {
+                            ok = false;
+                            break;
+                        }
+                        k_ready = true;
+                        ptx::tc_fence_after();
+                        issue_s(x, sk1);
+                    }
+                }
+                if (!ok) break;
+                ptx::tc_commit_elect(v_empty(sv));
+                if (next) ptx::tc_commit_elect(k_empty(sk1));
+                if (j + 2 == nmax) ptx::tc_commit_elect(q_empty);  // every score MMA of the item is issued
+            }
+        }
+        // every MMA issued here has completed before TMEM is freed
+        __syncwarp();
+        ptx::tc_commit_elect(drain_bar);
+        volatile int no_abort = 0;
+        ptx::mbar_wait(drain_bar, 0, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+    } else {
+        // ------------------------------------------------------------ softmax warps
+        const int x = (warp - 2) >> 2;  // tile A (0) or B (1)
+        const int q = warp & 3;         // TMEM lane quarter
+        const int row = q * 32 + lane;  // row of the tile
+        const uint32_t lane_base = (uint32_t)(q * 32) << 16;
+        const uint32_t srow = tmem + lane_base + s_col(x), orow = tmem + lane_base + o_col(x);
+        auto wait_warp = [&](uint32_t b, uint32_t parity, int code) {
+            return __all_sync(0xffffffffu, ptx::mbar_wait(b, parity, abort_flag, err, code));
+        };
+        int gx = 0;  // this tile's blocks so far (the parity of its barriers)
+        bool ok = true;
+        for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+            int bb, qq0, na, nb;
+            decode(it, bb, qq0, na, nb);
+            if (max(na, nb) == 0) continue;
+            const int nx = x ? nb : na;
+            const int qrow = qq0 + x * kQ + row;
+            const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
+            // The output accumulates in TMEM; the row keeps its base m (p = 2^(x - m)) until
+            // a block's maximum exceeds it by more than 2^8, and only then is its TMEM row
+            // of O rescaled by 2^(m_old - m_new).
+            float m = -INFINITY, l = 0.0f;
+            for (int j = 0; j < nx; ++j, ++gx) {
+                if (!wait_warp(s_full(x), (uint32_t)gx & 1u, kErrSoftS)) {
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+                uint32_t sr[kKV];  // the row's scores of this block
+                tmem_ld64(srow, *reinterpret_cast<uint32_t(*)[64]>(sr));
+                tmem_ld64(srow + 64, *reinterpret_cast<uint32_t(*)[64]>(sr + 64));
+                tmem_wait64(*reinterpret_cast<uint32_t(*)[64]>(sr));
+                tmem_wait64(*reinterpret_cast<uint32_t(*)[64]>(sr + 64));
+                ptx::tc_fence_before();
+                const int lim = min(last, p.Lk - 1) - j * kKV;  // columns 0..lim are visible
+                // pass 1: scale to base 2 in place (-inf where masked), the row's maximum
+                float mxv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
+                const uint32_t cb = __float_as_uint(p.scale_log2);
+                const uint64_t c2 = f2(cb, cb);
+                if (lim >= kKV - 1) {
+#pragma unroll
+                    for (int i = 0; i < kKV; i += 2) {
+                        f2_split(f2_mul(f2(sr[i], sr[i + 1]), c2), sr[i], sr[i + 1]);
+                        mxv[(i >> 1) & 3] =
+                            max3(mxv[(i >> 1) & 3], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
+                    }
+                } else {
+                    const uint32_t ninf = __float_as_uint(-INFINITY);
+#pragma unroll
+                    for (int i = 0; i < kKV; i += 2) {
+                        f2_split(f2_mul(f2(sr[i], sr[i + 1]), c2), sr[i], sr[i + 1]);
+                        if (i > lim) sr[i] = ninf;
+                        if (i + 1 > lim) sr[i + 1] = ninf;
+                        mxv[(i >> 1) & 3] =
+                            max3(mxv[(i >> 1) & 3], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
+                    }
+                }
+                const float mx = fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3]));
+                const bool rebase = mx > m + 8.0f;  // (always for the first visible key: m = -inf)
+                float alpha = 1.0f;
+                if (rebase) {
+                    alpha = ex2(m - mx);  // 0 while m = -inf
+                    m = mx;
+                    l *= alpha;
+                }
+                const float basev = m == -INFINITY ? 0.0f : m;  // no visible key yet: every p is 0
+                // pass 2: p = 2^(s - m) as bf16 pairs over the first 64 score columns (keys 2c,
+                // 2c + 1 in column c), the A operand of P V
+                uint64_t lv2[2] = {0ull, 0ull};
+                const uint32_t nb2u = __float_as_uint(-basev);  // x + (-m) rounds as x - m
+                const uint64_t nb2 = f2(nb2u, nb2u);
+#pragma unroll
+                for (int c0 = 0; c0 < kKV; c0 += 64) {
+                    uint32_t pk[32];
+#pragma unroll
+                    for (int i = 0; i < 64; i += 2) {
+                        uint32_t d0, d1;
+                        f2_split(f2_add(f2(sr[c0 + i], sr[c0 + i + 1]), nb2), d0, d1);
+                        const float p0 = ex2(__uint_as_float(d0)), p1 = ex2(__uint_as_float(d1));
+                        lv2[(i >> 1) & 1] = f2_add(lv2[(i >> 1) & 1], f2(__float_as_uint(p0), __float_as_uint(p1)));
+                        pk[i >> 1] = pack_bf16(p0, p1);
+                    }
+                    tmem_st32(srow + (uint32_t)(c0 / 2), pk);
+                }
+                {
+                    uint32_t a0, a1, b0, b1;
+                    f2_split(lv2[0], a0, a1);
+                    f2_split(lv2[1], b0, b1);
+                    l += (__uint_as_float(a0) + __uint_as_float(a1)) + (__uint_as_float(b0) + __uint_as_float(b1));
+                }
+                // O (the P V products of this item's earlier blocks) is complete in TMEM
+                if (j >= 1) {
+                    if (!wait_warp(o_full(x), (uint32_t)(gx - 1) & 1u, kErrSoftO)) {
+                        ok = false;
+                        break;
+                    }
+                    ptx::tc_fence_after();
+                    if (__any_sync(0xffffffffu, rebase)) {  // rescale the warp's rows of O
+#pragma unroll
+                        for (int c0 = 0; c0 < D; c0 += 32) {
+                            uint32_t r[32];
+                            ptx::tmem_ld32(orow + c0, r);
+                            ptx::tmem_wait_ld(r);
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * alpha);
+                            tmem_st32(orow + c0, r);
+                        }
+                    }
+                }
+                tmem_wait_st();
+                ptx::tc_fence_before();  // P_X(j) and the rescaled O are stored before P V runs
+                __syncwarp();
+                if (lane == 0) ptx::mbar_arrive(p_full(x));
+            }
+            if (!ok) break;
+            // the item's output: O from TMEM once its last P V product has completed
+            const bool have_o = nx > 0;
+            if (have_o) {
+                if (!wait_warp(o_full(x), (uint32_t)(gx - 1) & 1u, kErrSoftO)) {
+                    ok = false;
+                    break;
+                }
+                ptx::tc_fence_after();
+            }
+            const float inv = (have_o && l > 0.0f) ? 1.0f / l : 0.0f;
+            // 32 x 32 tiles of the warp's rows: staged with the 128-byte swizzle and stored by
+            // TMA, which leaves rows past Lq unwritten
+            const uint32_t stage = sO + (uint32_t)(warp - 2) * C::kOStage;
+#pragma unroll
+            for (int c0 = 0; c0 < D; c0 += 32) {
+                uint32_t r[32];
+                if (have_o) {
+                    ptx::tmem_ld32(orow + c0, r);
+                    ptx::tmem_wait_ld(r);
+                } else {
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) r[i] = 0u;
+                }
+                if (lane == 0) ptx::bulk_wait_all_read();  // the tile's previous store has read it
+                __syncwarp();
+#pragma unroll
+                for (int c = 0; c < 8; ++c)
+                    st_shared_f4(stage + (uint32_t)lane * 128u + ((uint32_t)(c ^ (lane & 7)) << 4),
+                                 __uint_as_float(r[4 * c]) * inv, __uint_as_float(r[4 * c + 1]) * inv,
+                                 __uint_as_float(r[4 * c + 2]) * inv, __uint_as_float(r[4 * c + 3]) * inv);
+                ptx::fence_proxy_async_smem();  // the tile is read by the TMA (async proxy)
+                __syncwarp();
+                if (lane == 0) {
+                    ptx::tma_store_3d(&p.to, stage, c0, qq0 + x * kQ + q * 32, bb);
+                    ptx::bulk_commit();
+                }
+            }
+            ptx::tc_fence_before();  // the next item's first P V overwrites O
+        }
+        if (lane == 0) ptx::bulk_wait_all();  // every output store has completed
+        __syncwarp();
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    if (warp == 1) ptx::tmem_dealloc(tmem, 512);
+}
+
 }  // namespace
 
 cudaError_t attention_watchdog_take(int* word) {
@@ -606,8 +1041,9 @@ cudaError_t attention_watchdog_take(int* word) {
 }
 
 cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
-                                float* O, cudaStream_t stream) {
-    const int qblocks = (int)((d.Lq + kQ - 1) / kQ);
+                                float* O, cudaStream_t stream, bool two_tiles) {
+    const int item_q = two_tiles ? 2 * kQ : kQ;  // queries per work item
+    const int qblocks = (int)((d.Lq + item_q - 1) / item_q);
     const long long ctas = (long long)qblocks * d.batch;
     if (ctas <= 0) return cudaSuccess;
     if (ctas >= (1LL << 31)) return cudaErrorInvalidValue;
@@ -648,17 +1084,23 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     while (group % 2 == 0 && group * per_problem > kGroupL2Bytes) group /= 2;
     p.group = (int)group;
     p.scale_log2 = d.scale * 1.4426950408889634f;
-    const int i = d.d == 64 ? 0 : 1;
-    const int smem = i == 0 ? (int)Cfg<64>::kSmem : (int)Cfg<128>::kSmem;
-    cudaError_t e = ensure_dynamic_smem(
-        i == 0 ? reinterpret_cast<const void*>(attention_tc_kernel<64>) : reinterpret_cast<const void*>(attention_tc_kernel<128>),
-        smem);
-    if (e != cudaSuccess) return e;
     // persistent: one CTA per SM (the CTA holds all of the SM's tensor memory)
     const int sms = current_sm_count();
     const unsigned grid = (unsigned)std::min<long long>(ctas, sms);
-    return launch_pdl(i == 0 ? attention_tc_kernel<64> : attention_tc_kernel<128>, dim3(grid),
-                      dim3(i == 0 ? threads_of<64>() : threads_of<128>()), (size_t)smem, stream, p);
+    void (*kern)(Params);
+    int smem, threads;
+    if (two_tiles) {
+        kern = d.d == 64 ? attention_tc2_kernel<64> : attention_tc2_kernel<128>;
+        smem = d.d == 64 ? (int)Cfg2<64>::kSmem : (int)Cfg2<128>::kSmem;
+        threads = 320;
+    } else {
+        kern = d.d == 64 ? attention_tc_kernel<64> : attention_tc_kernel<128>;
+        smem = d.d == 64 ? (int)Cfg<64>::kSmem : (int)Cfg<128>::kSmem;
+        threads = d.d == 64 ? threads_of<64>() : threads_of<128>();
+    }
+    cudaError_t e = ensure_dynamic_smem(reinterpret_cast<const void*>(kern), smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(kern, dim3(grid), dim3(threads), (size_t)smem, stream, p);
 }
 
 }  // namespace nnjit

@@ -664,7 +664,8 @@ nnjit_status attention_validate(const nnjit_attention_desc* d, const void* Q, co
     if (d->causal != 0 && d->causal != 1) return fail(NNJIT_ERR_INVALID_ARG, "causal must be 0 or 1");
     if (!std::isfinite(d->scale)) return fail(NNJIT_ERR_INVALID_ARG, "scale must be finite");
     if (d->d != 64 && d->d != 128) return fail(NNJIT_ERR_UNSUPPORTED, "head dimension must be 64 or 128");
-    if (d->kernel < NNJIT_ATTN_AUTO || d->kernel > NNJIT_ATTN_MMA) return fail(NNJIT_ERR_INVALID_ARG, "unknown kernel");
+    if (d->kernel < NNJIT_ATTN_AUTO || d->kernel > NNJIT_ATTN_TCGEN05_2T)
+        return fail(NNJIT_ERR_INVALID_ARG, "unknown kernel");
     if (d->Lq == 0) return NNJIT_OK;
     if (!Q || !O || (d->Lk > 0 && (!K || !V))) return fail(NNJIT_ERR_INVALID_ARG, "NULL pointer");
     auto a16 = [](const void* p) { return !p || (reinterpret_cast<uintptr_t>(p) & 15) == 0; };
@@ -674,7 +675,8 @@ nnjit_status attention_validate(const nnjit_attention_desc* d, const void* Q, co
 
 cudaError_t attention_launch(const nnjit_attention_desc& d, int kernel, const void* Q, const void* K,
                              const void* V, float* O, cudaStream_t s) {
-    return kernel == NNJIT_ATTN_MMA ? launch_attention(d, Q, K, V, O, s) : launch_attention_tc(d, Q, K, V, O, s);
+    if (kernel == NNJIT_ATTN_MMA) return launch_attention(d, Q, K, V, O, s);
+    return launch_attention_tc(d, Q, K, V, O, s, kernel == NNJIT_ATTN_TCGEN05_2T);
 }
 
 }  // namespace
@@ -707,15 +709,15 @@ nnjit_status nnjit_attention_tune(const nnjit_attention_desc* d, const void* Q, 
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
-    const int kernels[2] = {NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA};
-    double med[2] = {0.0, 0.0};
+    const int kernels[3] = {NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA, NNJIT_ATTN_TCGEN05_2T};
+    double med[3] = {0.0, 0.0, 0.0};
     if (d->Lq > 0) {
         cudaStream_t s = nullptr;
         if ((e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking)) != cudaSuccess) return cuda_fail(e, "stream");
         cudaEvent_t e0 = nullptr, e1 = nullptr;
         cudaEventCreate(&e0);
         cudaEventCreate(&e1);
-        for (int k = 0; k < 2 && e == cudaSuccess; ++k) {
+        for (int k = 0; k < 3 && e == cudaSuccess; ++k) {
             e = attention_launch(*d, kernels[k], Q, K, V, O, s);  // warm-up
             std::vector<double> trials;
             for (int t = 0; t < 3 && e == cudaSuccess; ++t) {
@@ -740,15 +742,16 @@ nnjit_status nnjit_attention_tune(const nnjit_attention_desc* d, const void* Q, 
         if ((e = attention_watchdog_take(&word)) != cudaSuccess) return cuda_fail(e, "attention watchdog read");
         if (word != 0) return fail(NNJIT_ERR_TIMEOUT, "attention wait expired while tuning");
     }
-    const int best = med[1] < med[0] ? NNJIT_ATTN_MMA : NNJIT_ATTN_TCGEN05;
+    int bk = 0;  // the lowest median (the first on a tie)
+    for (int k = 1; k < 3; ++k)
+        if (med[k] < med[bk]) bk = k;
+    const int best = kernels[bk];
     {
         std::lock_guard<std::mutex> lk(g_attn_mu);
         g_attn_choice[attention_key(*d, dev)] = best;
     }
-    if (times_us) {
-        times_us[0] = med[0];
-        times_us[1] = med[1];
-    }
+    if (times_us)
+        for (int k = 0; k < 3; ++k) times_us[k] = med[k];
     if (chosen) *chosen = best;
     return NNJIT_OK;
 }

@@ -126,8 +126,10 @@ cudaError_t encode_tc_tensor_maps(const Problem& p, const nnjit_candidate& c, co
 // warp-level MMA kernel, and the tensor-memory kernel with its watchdog word.
 cudaError_t launch_attention(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
                              float* O, cudaStream_t stream);
+// two_tiles: 256-query items of two 128-row tiles sharing the key and value blocks (kernel
+// NNJIT_ATTN_TCGEN05_2T); else 128-query items (NNJIT_ATTN_TCGEN05).
 cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, const void* K, const void* V,
-                                float* O, cudaStream_t stream);
+                                float* O, cudaStream_t stream, bool two_tiles = false);
 // Read and clear the tensor-memory kernel's watchdog word (synchronous).
 cudaError_t attention_watchdog_take(int* word);
 

@@ -78,7 +78,7 @@ class nnjit_attention_desc(ctypes.Structure):
                 ("kernel", ctypes.c_int32)]
 
 
-NNJIT_ATTN_AUTO, NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA = 0, 1, 2
+NNJIT_ATTN_AUTO, NNJIT_ATTN_TCGEN05, NNJIT_ATTN_MMA, NNJIT_ATTN_TCGEN05_2T = 0, 1, 2, 3
 
 
 NNJIT_SETTING_FREE = -1
@@ -445,7 +445,7 @@ def nnjit_settings_study(descs) -> tuple[dict, dict]:
 def nnjit_attention(Q, K, V, O, causal=False, scale=None, stream=None, kernel=NNJIT_ATTN_AUTO):
     """O = softmax(scale Q K^T) V per leading index (batch x heads).  Q [B][Lq][d], K and V
     [B][Lk][d] bf16 tensors, O [B][Lq][d] float32 (device tensors); scale defaults to
-    1 / sqrt(d); kernel: NNJIT_ATTN_AUTO / _TCGEN05 / _MMA."""
+    1 / sqrt(d); kernel: NNJIT_ATTN_AUTO / _TCGEN05 / _MMA / _TCGEN05_2T."""
     B, Lq, d = Q.shape
     Lk = K.shape[1]
     desc = nnjit_attention_desc(B, Lq, Lk, d, 1 if causal else 0,
@@ -459,13 +459,14 @@ def nnjit_attention_check():
 
 
 def nnjit_attention_tune(Q, K, V, O, causal=False, scale=None, reps=20):
-    """Time both attention kernels on these buffers (O is overwritten) and record the faster
-    for later kernel=AUTO calls; returns (times_us (tensor-memory, warp-MMA), chosen)."""
+    """Time the three attention kernels on these buffers (O is overwritten) and record the
+    fastest for later kernel=AUTO calls; returns (times_us (tensor-memory, warp-MMA,
+    two-tile tensor-memory), chosen)."""
     B, Lq, d = Q.shape
     desc = nnjit_attention_desc(B, Lq, K.shape[1], d, 1 if causal else 0,
                                 float(scale) if scale is not None else 1.0 / float(d) ** 0.5, 0)
-    times = (ctypes.c_double * 2)()
+    times = (ctypes.c_double * 3)()
     chosen = ctypes.c_int32(0)
     _check(load_library().nnjit_attention_tune(ctypes.byref(desc), _ptr(Q), _ptr(K), _ptr(V), _ptr(O), reps,
                                                times, ctypes.byref(chosen)), "nnjit_attention_tune")
-    return (times[0], times[1]), chosen.value
+    return (times[0], times[1], times[2]), chosen.value

@@ -155,7 +155,7 @@ def test_attention_refusals_without_a_gpu(lib):
              ((1, 4, 4, 64, 2, 1.0), nj.NNJIT_ERR_INVALID_ARG), ((1, -1, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
              ((1, 4, -2, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
              ((1, 4, 4, 64, 0, float("nan")), nj.NNJIT_ERR_INVALID_ARG),
-             ((1, 4, 4, 64, 0, 1.0, 3), nj.NNJIT_ERR_INVALID_ARG), ((1, 4, 4, 64, 0, 1.0, -1), nj.NNJIT_ERR_INVALID_ARG))
+             ((1, 4, 4, 64, 0, 1.0, 4), nj.NNJIT_ERR_INVALID_ARG), ((1, 4, 4, 64, 0, 1.0, -1), nj.NNJIT_ERR_INVALID_ARG))
     for d, st in cases:
         assert f(nj.nnjit_attention_desc(*d), p, p, p, p, None) == st, d
     desc = nj.nnjit_attention_desc(1, 4, 4, 64, 0, 1.0)

@@ -25,7 +25,7 @@ def _dev(bits):
     return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
 
 
-KERNELS = {"tcgen05": 1, "mma": 2}
+KERNELS = {"tcgen05": 1, "mma": 2, "tcgen05_2t": 3}
 
 
 def _run(Q, K, V, causal, scale, kernel=1):
@@ -86,7 +86,7 @@ def test_attention_refusals():
     for d, st in (((1, 4, 4, 96, 0, 1.0), nj.NNJIT_ERR_UNSUPPORTED), ((0, 4, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
                   ((1, 4, 4, 64, 2, 1.0), nj.NNJIT_ERR_INVALID_ARG), ((1, -1, 4, 64, 0, 1.0), nj.NNJIT_ERR_INVALID_ARG),
                   ((1, 4, 4, 64, 0, float("inf")), nj.NNJIT_ERR_INVALID_ARG),
-                  ((1, 4, 4, 64, 0, 1.0, 3), nj.NNJIT_ERR_INVALID_ARG)):
+                  ((1, 4, 4, 64, 0, 1.0, 4), nj.NNJIT_ERR_INVALID_ARG)):
         assert lib.nnjit_attention(nj.nnjit_attention_desc(*d), p, p, p, p, None) == st
     assert lib.nnjit_attention(nj.nnjit_attention_desc(1, 4, 4, 64, 0, 1.0), p + 4, p, p, p, None) == \
         nj.NNJIT_ERR_UNSUPPORTED
@@ -108,15 +108,16 @@ def test_attention_full_size_sampled_heads(shape, kernel):
 
 
 def test_attention_tune_records_the_faster_kernel():
-    """nnjit_attention_tune times both kernels on the caller's buffers and records the faster
-    one for the shape; AUTO calls then use it and stay within the oracle's tolerance."""
+    """nnjit_attention_tune times the three kernels on the caller's buffers and records the
+    fastest for the shape; AUTO calls then use it and stay within the oracle's tolerance."""
     B, Lq, Lk, d = 4, 200, 260, 64
     Q, K, V = _bf16((B, Lq, d), 11), _bf16((B, Lk, d), 12), _bf16((B, Lk, d), 13)
     dQ, dK, dV = _dev(Q), _dev(K), _dev(V)
     O = torch.empty((B, Lq, d), dtype=torch.float32, device="cuda")
-    (t_tc, t_mma), chosen = nj.nnjit_attention_tune(dQ, dK, dV, O, causal=True, reps=5)
-    assert t_tc > 0 and t_mma > 0
-    assert chosen == (nj.NNJIT_ATTN_MMA if t_mma < t_tc else nj.NNJIT_ATTN_TCGEN05)
+    times, chosen = nj.nnjit_attention_tune(dQ, dK, dV, O, causal=True, reps=5)
+    assert len(times) == 3 and all(t > 0 for t in times)
+    kernels = (nj.NNJIT_ATTN_TCGEN05, nj.NNJIT_ATTN_MMA, nj.NNJIT_ATTN_TCGEN05_2T)
+    assert chosen == kernels[min(range(3), key=lambda k: (times[k], k))]
     O.fill_(float("nan"))
     nj.nnjit_attention(dQ, dK, dV, O, causal=True)          # AUTO: the recorded kernel
     nj.nnjit_attention_check()
