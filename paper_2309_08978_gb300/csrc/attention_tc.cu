@@ -143,6 +143,10 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
     asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
                  : "memory");
 }
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
+    asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+                 : "memory");
+}
 __device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
 
 template <int D>
@@ -627,9 +631,9 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
     constexpr int SK = C::kKStages, SV = C::kVStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
-    // q_full, q_empty, drain, k_full/k_empty (SK each), v_full/v_empty (SV each), then per
-    // tile X: s_full[X], p_full[X], o_full[X]
-    __shared__ __align__(8) uint64_t bars[3 + 2 * SK + 2 * SV + 6];
+    // q_full[X], q_empty[X], drain, k_full/k_empty (SK each), v_full/v_empty (SV each),
+    // then per tile X: s_full[X], p_full[X], o_full[X]
+    __shared__ __align__(8) uint64_t bars[5 + 2 * SK + 2 * SV + 6];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
     volatile int* abort_flag = &abort_word;
@@ -642,10 +646,14 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
     auto sV = [&](int s) { return sVR + (uint32_t)s * C::kVBytes; };
     const uint32_t sO = sVR + SV * C::kVBytes;  // 8 output staging tiles
     auto bar = [&](int i) { return ptx::smem_u32(&bars[i]); };
-    const uint32_t q_full = bar(0), q_empty = bar(1), drain_bar = bar(2);
-    auto k_full = [&](int s) { return bar(3 + s); };
-    auto k_empty = [&](int s) { return bar(3 + SK + s); };
-    constexpr int kVB = 3 + 2 * SK, kXB = kVB + 2 * SV;
+    // each tile's Q buffer has its own pair of barriers, so that tile A's next Q tile
+    // loads as soon as A's last score product of the current item has completed
+    auto q_full = [&](int x) { return bar(x); };
+    auto q_empty = [&](int x) { return bar(2 + x); };
+    const uint32_t drain_bar = bar(4);
+    auto k_full = [&](int s) { return bar(5 + s); };
+    auto k_empty = [&](int s) { return bar(5 + SK + s); };
+    constexpr int kVB = 5 + 2 * SK, kXB = kVB + 2 * SV;
     auto v_full = [&](int s) { return bar(kVB + s); };
     auto v_empty = [&](int s) { return bar(kVB + SV + s); };
     auto s_full = [&](int x) { return bar(kXB + x); };
@@ -676,8 +684,10 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
     };
 
     if (threadIdx.x == 0) {
-        ptx::mbar_init(q_full, 1);
-        ptx::mbar_init(q_empty, 1);
+        for (int x = 0; x < 2; ++x) {
+            ptx::mbar_init(q_full(x), 1);
+            ptx::mbar_init(q_empty(x), 1);
+        }
         ptx::mbar_init(drain_bar, 1);
         for (int s = 0; s < SK; ++s) {
             ptx::mbar_init(k_full(s), 1);
@@ -713,8 +723,22 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             ptx::prefetch_tmap(&p.tk);
             ptx::prefetch_tmap(&p.tv);
             uint32_t k_armed = 0, k_par = 0, v_armed = 0, v_par = 0, q_armed = 0, q_par = 0;
-            int g = 0, nq = 0;  // key blocks and items loaded so far
+            int g = 0;                 // key blocks loaded so far
+            int nqt[2] = {0, 0};       // Q tiles loaded so far, per tile
             bool ok = true;
+            // tile x's Q buffer is free once the last score product of its previous item
+            // has completed
+            auto load_q = [&](int x, int bb, int row0) -> bool {
+                const uint32_t ph = (uint32_t)nqt[x] & 1u;
+                if (nqt[x] >= 1 && !ptx::mbar_wait(q_empty(x), ph ^ 1u, abort_flag, err, kErrProd)) return false;
+                ptx::mbar_arrive_expect_tx(q_full(x), C::kQBytes);
+                for (int kb = 0; kb < kDB; ++kb)
+                    ptx::tma_load_3d(sQ(x) + kb * 16384u, &p.tq, kb * 64, row0, bb, q_full(x));
+                q_armed |= 1u << x;
+                q_par = (q_par & ~(1u << x)) | (ph << x);
+                ++nqt[x];
+                return true;
+            };
             int gv = -1, vb = 0, vk0 = 0;  // the value block issued one key block behind
             auto load_v = [&]() -> bool {
                 const int st = gv % SV;
@@ -735,16 +759,9 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
                 decode(it, bb, qq0, na, nb);
                 const int nmax = max(na, nb);
                 if (nmax == 0) continue;
-                // both Q tiles are free once every score MMA of the previous item has completed
-                const uint32_t qph = (uint32_t)nq & 1u;
-                if (nq >= 1 && !ptx::mbar_wait(q_empty, qph ^ 1u, abort_flag, err, kErrProd)) break;
-                ptx::mbar_arrive_expect_tx(q_full, 2 * C::kQBytes);
-                for (int x = 0; x < 2; ++x)
-                    for (int kb = 0; kb < kDB; ++kb)
-                        ptx::tma_load_3d(sQ(x) + kb * 16384u, &p.tq, kb * 64, qq0 + x * kQ, bb, q_full);
-                q_armed = 1;
-                q_par = qph;
-                ++nq;
+                // order: Q_A, the first key block, Q_B (tile B's previous item ends a block
+                // later than tile A's), then the item's key and value blocks
+                if (na > 0 && !load_q(0, bb, qq0)) break;
                 for (int j = 0; j < nmax; ++j, ++g) {
                     const int st = g % SK;
                     const uint32_t ph = (uint32_t)(g / SK) & 1u;
@@ -757,6 +774,10 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
                         ptx::tma_load_3d(sK(st) + kb * 16384u, &p.tk, kb * 64, j * kKV, bb, k_full(st));
                     k_armed |= 1u << st;
                     k_par = (k_par & ~(1u << st)) | (ph << st);
+                    if (j == 0 && nb > 0 && !load_q(1, bb, qq0 + kQ)) {
+                        ok = false;
+                        break;
+                    }
                     if (gv >= 0 && !load_v()) {
                         ok = false;
                         break;
@@ -769,7 +790,9 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             }
             // drain: every copy issued here has landed before the CTA may exit
             volatile int no_abort = 0;
-            if (q_armed) ptx::mbar_wait(q_full, q_par, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
+            for (int x = 0; x < 2; ++x)
+                if (q_armed & (1u << x))
+                    ptx::mbar_wait(q_full(x), (q_par >> x) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
             for (int st = 0; st < SK; ++st)
                 if (k_armed & (1u << st))
                     ptx::mbar_wait(k_full(st), (k_par >> st) & 1u, &no_abort, err, kErrDrain, ptx::kWaitLimitNs / 4);
@@ -810,8 +833,9 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             }
             ptx::tc_commit_elect(o_full(x));
         };
-        int g = 0, nq = 0;
-        int gx[2] = {0, 0};  // blocks of tile A / B so far (the parity of its barriers)
+        int g = 0;
+        int nqt[2] = {0, 0};  // Q tiles used so far, per tile
+        int gx[2] = {0, 0};   // blocks of tile A / B so far (the parity of its barriers)
         bool ok = true;
         for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
             int bb, qq0, na, nb;
@@ -819,16 +843,21 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             const int n[2] = {na, nb};
             const int nmax = max(na, nb);
             if (nmax == 0) continue;
-            if (!wait_all(q_full, (uint32_t)nq & 1u, kErrMmaQ)) break;
-            ++nq;
-            ptx::tc_fence_after();
-            // block 0's score products
+            // block 0's score products, tile by tile as its Q tile lands
             if (!wait_all(k_full(g % SK), (uint32_t)((g / SK) & 1), kErrMmaKv)) break;
-            ptx::tc_fence_after();
-            for (int x = 0; x < 2; ++x)
-                if (n[x] > 0) issue_s(x, g % SK);
+            for (int x = 0; x < 2 && ok; ++x) {
+                if (n[x] == 0) continue;
+                if (!wait_all(q_full(x), (uint32_t)nqt[x] & 1u, kErrMmaQ)) {
+                    ok = false;
+                    break;
+                }
+                ++nqt[x];
+                ptx::tc_fence_after();
+                issue_s(x, g % SK);
+                if (n[x] == 1) ptx::tc_commit_elect(q_empty(x));  // the tile's only score product
+            }
+            if (!ok) break;
             ptx::tc_commit_elect(k_empty(g % SK));
-            if (nmax == 1) ptx::tc_commit_elect(q_empty);
             for (int j = 0; j < nmax; ++j, ++g) {
                 const int sv = g % SV, sk1 = (g + 1) % SK;
                 if (!wait_all(v_full(sv), (uint32_t)((g / SV) & 1), kErrMmaKv)) {
@@ -854,12 +883,12 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
                         k_ready = true;
                         ptx::tc_fence_after();
                         issue_s(x, sk1);
+                        if (j + 2 == n[x]) ptx::tc_commit_elect(q_empty(x));  // the tile's last score product
                     }
                 }
                 if (!ok) break;
                 ptx::tc_commit_elect(v_empty(sv));
                 if (next) ptx::tc_commit_elect(k_empty(sk1));
-                if (j + 2 == nmax) ptx::tc_commit_elect(q_empty);  // every score MMA of the item is issued
             }
         }
         // every MMA issued here has completed before TMEM is freed
@@ -886,71 +915,92 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             const int nx = x ? nb : na;
             const int qrow = qq0 + x * kQ + row;
             const int last = p.causal ? qrow + shift : p.Lk - 1;  // last key this row sees
-            // The output accumulates in TMEM; the row keeps its base m (p = 2^(x - m)) until
-            // a block's maximum exceeds it by more than 2^8, and only then is its TMEM row
-            // of O rescaled by 2^(m_old - m_new).
+            // The output accumulates in TMEM; the row keeps its base m, a raw score
+            // (p = 2^((s - m) c), c = scale log2(e)), until a block's maximum exceeds it by
+            // more than 8 / c (p > 2^8), and only then is its TMEM row of O rescaled by
+            // 2^((m_old - m_new) c).  s - m is formed first: the maximum gives exactly 1.
             float m = -INFINITY, l = 0.0f;
+            const float c = p.scale_log2, rebase_gap = 8.0f / c;
             for (int j = 0; j < nx; ++j, ++gx) {
                 if (!wait_warp(s_full(x), (uint32_t)gx & 1u, kErrSoftS)) {
                     ok = false;
                     break;
                 }
                 ptx::tc_fence_after();
-                uint32_t sr[kKV];  // the row's scores of this block
-                tmem_ld64(srow, *reinterpret_cast<uint32_t(*)[64]>(sr));
-                tmem_ld64(srow + 64, *reinterpret_cast<uint32_t(*)[64]>(sr + 64));
-                tmem_wait64(*reinterpret_cast<uint32_t(*)[64]>(sr));
-                tmem_wait64(*reinterpret_cast<uint32_t(*)[64]>(sr + 64));
-                ptx::tc_fence_before();
+                // The row's 128 scores are read from TMEM twice, in 32-column pieces with the
+                // next piece's load in flight while one is worked on (a few registers, no
+                // spills): pass 1 takes the maximum of the raw scores, pass 2 computes p.
+                uint32_t ra[32], rb[32];
                 const int lim = min(last, p.Lk - 1) - j * kKV;  // columns 0..lim are visible
-                // pass 1: scale to base 2 in place (-inf where masked), the row's maximum
                 float mxv[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
-                const uint32_t cb = __float_as_uint(p.scale_log2);
-                const uint64_t c2 = f2(cb, cb);
-                if (lim >= kKV - 1) {
+                ptx::tmem_ld32(srow, ra);
+                ptx::tmem_wait_ld(ra);
+                // the branch is taken by the whole warp: the TMEM loads and stores in it are
+                // warp-collective (.sync.aligned), and lim differs between rows
+                if (__all_sync(0xffffffffu, lim >= kKV - 1)) {
 #pragma unroll
-                    for (int i = 0; i < kKV; i += 2) {
-                        f2_split(f2_mul(f2(sr[i], sr[i + 1]), c2), sr[i], sr[i + 1]);
-                        mxv[(i >> 1) & 3] =
-                            max3(mxv[(i >> 1) & 3], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
+                    for (int k = 0; k < kKV / 32; ++k) {
+                        uint32_t(&cur)[32] = (k & 1) ? rb : ra;
+                        uint32_t(&nxt)[32] = (k & 1) ? ra : rb;
+                        if (k + 1 < kKV / 32) ptx::tmem_ld32(srow + 32u * (k + 1), nxt);
+#pragma unroll
+                        for (int i = 0; i < 32; i += 2)
+                            mxv[(i >> 1) & 3] = max3(mxv[(i >> 1) & 3], __uint_as_float(cur[i]), __uint_as_float(cur[i + 1]));
+                        if (k + 1 < kKV / 32) ptx::tmem_wait_ld(nxt);
                     }
                 } else {
+                    // a block on the mask's edge: masked scores become -inf, written back to
+                    // TMEM (so that pass 2 reads p = 0 there) before the second read
                     const uint32_t ninf = __float_as_uint(-INFINITY);
 #pragma unroll
-                    for (int i = 0; i < kKV; i += 2) {
-                        f2_split(f2_mul(f2(sr[i], sr[i + 1]), c2), sr[i], sr[i + 1]);
-                        if (i > lim) sr[i] = ninf;
-                        if (i + 1 > lim) sr[i + 1] = ninf;
-                        mxv[(i >> 1) & 3] =
-                            max3(mxv[(i >> 1) & 3], __uint_as_float(sr[i]), __uint_as_float(sr[i + 1]));
+                    for (int k = 0; k < kKV / 32; ++k) {
+                        uint32_t(&cur)[32] = (k & 1) ? rb : ra;
+                        uint32_t(&nxt)[32] = (k & 1) ? ra : rb;
+                        if (k + 1 < kKV / 32) ptx::tmem_ld32(srow + 32u * (k + 1), nxt);
+#pragma unroll
+                        for (int i = 0; i < 32; ++i)
+                            if (32 * k + i > lim) cur[i] = ninf;
+#pragma unroll
+                        for (int i = 0; i < 32; i += 2)
+                            mxv[(i >> 1) & 3] = max3(mxv[(i >> 1) & 3], __uint_as_float(cur[i]), __uint_as_float(cur[i + 1]));
+                        tmem_st32(srow + 32u * k, cur);
+                        if (k + 1 < kKV / 32) ptx::tmem_wait_ld(nxt);
                     }
+                    tmem_wait_st();
                 }
                 const float mx = fmaxf(fmaxf(mxv[0], mxv[1]), fmaxf(mxv[2], mxv[3]));
-                const bool rebase = mx > m + 8.0f;  // (always for the first visible key: m = -inf)
+                const bool rebase = mx > m + rebase_gap;  // (always for the first visible key: m = -inf)
                 float alpha = 1.0f;
                 if (rebase) {
-                    alpha = ex2(m - mx);  // 0 while m = -inf
+                    alpha = ex2((m - mx) * c);  // 0 while m = -inf
                     m = mx;
                     l *= alpha;
                 }
                 const float basev = m == -INFINITY ? 0.0f : m;  // no visible key yet: every p is 0
-                // pass 2: p = 2^(s - m) as bf16 pairs over the first 64 score columns (keys 2c,
-                // 2c + 1 in column c), the A operand of P V
+                // pass 2: p as bf16 pairs over the first 64 score columns (keys 2c, 2c + 1 in
+                // column c), the A operand of P V.  Piece k's p go to columns 16k..16k+15, whose
+                // scores were read before.
                 uint64_t lv2[2] = {0ull, 0ull};
-                const uint32_t nb2u = __float_as_uint(-basev);  // x + (-m) rounds as x - m
-                const uint64_t nb2 = f2(nb2u, nb2u);
+                const uint32_t cb = __float_as_uint(c), nb2u = __float_as_uint(-basev);
+                const uint64_t c2 = f2(cb, cb), nb2 = f2(nb2u, nb2u);
+                ptx::tmem_ld32(srow, ra);
+                ptx::tmem_wait_ld(ra);
 #pragma unroll
-                for (int c0 = 0; c0 < kKV; c0 += 64) {
-                    uint32_t pk[32];
+                for (int k = 0; k < kKV / 32; ++k) {
+                    uint32_t(&cur)[32] = (k & 1) ? rb : ra;
+                    uint32_t(&nxt)[32] = (k & 1) ? ra : rb;
+                    if (k + 1 < kKV / 32) ptx::tmem_ld32(srow + 32u * (k + 1), nxt);
+                    uint32_t pk[16];
 #pragma unroll
-                    for (int i = 0; i < 64; i += 2) {
+                    for (int i = 0; i < 32; i += 2) {
                         uint32_t d0, d1;
-                        f2_split(f2_add(f2(sr[c0 + i], sr[c0 + i + 1]), nb2), d0, d1);
+                        f2_split(f2_mul(f2_add(f2(cur[i], cur[i + 1]), nb2), c2), d0, d1);
                         const float p0 = ex2(__uint_as_float(d0)), p1 = ex2(__uint_as_float(d1));
                         lv2[(i >> 1) & 1] = f2_add(lv2[(i >> 1) & 1], f2(__float_as_uint(p0), __float_as_uint(p1)));
                         pk[i >> 1] = pack_bf16(p0, p1);
                     }
-                    tmem_st32(srow + (uint32_t)(c0 / 2), pk);
+                    tmem_st16(srow + 16u * k, pk);
+                    if (k + 1 < kKV / 32) ptx::tmem_wait_ld(nxt);
                 }
                 {
                     uint32_t a0, a1, b0, b1;
