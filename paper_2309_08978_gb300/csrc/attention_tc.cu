@@ -26,6 +26,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <cmath>
 #include <cstdint>
 
@@ -39,6 +40,14 @@ namespace {
 
 __device__ int g_attn_watchdog;  // first expired wait's code (0: none)
 
+// Work counters of the two-tile kernel: a launch uses slot Params::sched (the launcher
+// cycles through the slots).  CTA b takes item b first, then (when there are more items
+// than CTAs) items G + [0]++ in turn, so a CTA whose items run long takes fewer; a CTA
+// that has taken its last item counts itself in [1], and the last one zeroes both for the
+// slot's next launch.  Launches that run at the same time need different slots.
+constexpr int kSchedSlots = 64;
+__device__ unsigned g_attn_sched[kSchedSlots][2];
+
 constexpr int kQ = 128;   // queries per work item (a CTA loops over items)
 // Bytes of Q, K, V and O that one group of problems may touch (about 3/4 of the 129 MB L2).
 constexpr long long kGroupL2Bytes = 96ll << 20;
@@ -51,7 +60,7 @@ __host__ __device__ constexpr int split_of() { return 2; }
 template <int D>
 __host__ __device__ constexpr int threads_of() { return 64 + 128 * split_of<D>(); }
 constexpr int kErrProd = 0x301, kErrMmaQ = 0x311, kErrMmaKv = 0x312, kErrMmaP = 0x314;
-constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrDrain = 0x331;
+constexpr int kErrSoftS = 0x321, kErrSoftO = 0x322, kErrItem = 0x323, kErrDrain = 0x331;
 
 template <int D>
 struct Cfg {
@@ -76,6 +85,7 @@ struct Params {
     int Lq, Lk, causal, qblocks, batch;
     int group;  // problems per item group (divides batch)
     float scale_log2;
+    int sched;  // two-tile kernel: its work-counter slot
 };
 
 __device__ __forceinline__ float ex2(float x) {
@@ -631,9 +641,11 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
     constexpr int SK = C::kKStages, SV = C::kVStages;
     constexpr int kDB = D / 64;  // 64-element (128-byte) column blocks of d
     extern __shared__ uint8_t raw[];
+    constexpr int kIR = 4;  // item ring: the items the producer has taken ahead
     // q_full[X], q_empty[X], drain, k_full/k_empty (SK each), v_full/v_empty (SV each),
-    // then per tile X: s_full[X], p_full[X], o_full[X]
-    __shared__ __align__(8) uint64_t bars[5 + 2 * SK + 2 * SV + 6];
+    // per tile X: s_full[X], p_full[X], o_full[X]; then i_full/i_empty (kIR each)
+    __shared__ __align__(8) uint64_t bars[5 + 2 * SK + 2 * SV + 6 + 2 * kIR];
+    __shared__ int item_ring[kIR];
     __shared__ uint32_t tmem_slot;
     __shared__ int abort_word;
     volatile int* abort_flag = &abort_word;
@@ -659,6 +671,8 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
     auto s_full = [&](int x) { return bar(kXB + x); };
     auto p_full = [&](int x) { return bar(kXB + 2 + x); };
     auto o_full = [&](int x) { return bar(kXB + 4 + x); };
+    auto i_full = [&](int s) { return bar(kXB + 6 + s); };
+    auto i_empty = [&](int s) { return bar(kXB + 6 + kIR + s); };
     // TMEM: S_A at column 0, S_B at 128, O_A at 256, O_B at 256 + D
     auto s_col = [&](int x) { return (uint32_t)x * kKV; };
     auto o_col = [&](int x) { return 2u * kKV + (uint32_t)x * D; };
@@ -683,6 +697,19 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
         nb = blocks(qq0 + kQ);
     };
 
+    // Items are handed out dynamically: the producer takes the next item index from the
+    // launch's work counter and publishes it in the item ring; the other roles read the
+    // same sequence from the ring (an index past the last item ends every role's loop).
+    auto next_item = [&](int n) -> int {  // the n-th item of this CTA (MMA and softmax warps)
+        const int s = n % kIR;
+        if (!__all_sync(0xffffffffu, ptx::mbar_wait(i_full(s), (uint32_t)(n / kIR) & 1u, abort_flag, err, kErrItem)))
+            return -1;
+        const int it = *reinterpret_cast<volatile int*>(&item_ring[s]);
+        __syncwarp();
+        if ((threadIdx.x & 31) == 0) ptx::mbar_arrive(i_empty(s));
+        return it;
+    };
+
     if (threadIdx.x == 0) {
         for (int x = 0; x < 2; ++x) {
             ptx::mbar_init(q_full(x), 1);
@@ -701,6 +728,10 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             ptx::mbar_init(s_full(x), 1);
             ptx::mbar_init(p_full(x), 4);  // one arrival per softmax warp of the tile
             ptx::mbar_init(o_full(x), 1);
+        }
+        for (int s = 0; s < kIR; ++s) {
+            ptx::mbar_init(i_full(s), 1);
+            ptx::mbar_init(i_empty(s), 9);  // the MMA warp and the eight softmax warps
         }
         abort_word = 0;
         ptx::fence_barrier_init();
@@ -754,7 +785,22 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
                 gv = -1;
                 return true;
             };
-            for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+            for (int n = 0; ok; ++n) {
+                // take the next item: its ring slot is free once every role has read item n - kIR
+                const int s = n % kIR;
+                if (n >= kIR && !ptx::mbar_wait(i_empty(s), ((uint32_t)(n / kIR) & 1u) ^ 1u, abort_flag, err, kErrProd))
+                    break;
+                // the first item is the CTA's own index (no wait on the counter before the
+                // first loads); the later ones come from the counter, which counts past the grid
+                int it = -1;
+                if (n == 0)
+                    it = (int)blockIdx.x;
+                else if (items > (int)gridDim.x)
+                    it = (int)gridDim.x + (int)atomicAdd(&g_attn_sched[p.sched][0], 1u);
+                if (it >= items) it = -1;
+                item_ring[s] = it;
+                ptx::mbar_arrive(i_full(s));  // (release: the index is visible to the waiters)
+                if (it < 0) break;
                 int bb, qq0, na, nb;
                 decode(it, bb, qq0, na, nb);
                 const int nmax = max(na, nb);
@@ -787,6 +833,17 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
                     vk0 = j * kKV;
                 }
                 if (ok && gv >= 0 && !load_v()) ok = false;  // the item's last value block
+            }
+            if (items > (int)gridDim.x) {
+                // this CTA takes no more items; the last CTA to get here zeroes the counter
+                // for the slot's next launch (every other CTA has taken its last item)
+                unsigned* c = g_attn_sched[p.sched];
+                __threadfence();
+                if (atomicAdd(&c[1], 1u) == gridDim.x - 1) {
+                    __threadfence();
+                    atomicExch(&c[0], 0u);
+                    atomicExch(&c[1], 0u);
+                }
             }
             // drain: every copy issued here has landed before the CTA may exit
             volatile int no_abort = 0;
@@ -837,7 +894,9 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
         int nqt[2] = {0, 0};  // Q tiles used so far, per tile
         int gx[2] = {0, 0};   // blocks of tile A / B so far (the parity of its barriers)
         bool ok = true;
-        for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+        for (int ni = 0; ok; ++ni) {
+            const int it = next_item(ni);
+            if (it < 0) break;
             int bb, qq0, na, nb;
             decode(it, bb, qq0, na, nb);
             const int n[2] = {na, nb};
@@ -908,7 +967,9 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
         };
         int gx = 0;  // this tile's blocks so far (the parity of its barriers)
         bool ok = true;
-        for (int it = blockIdx.x; ok && it < items; it += gridDim.x) {
+        for (int ni = 0; ok; ++ni) {
+            const int it = next_item(ni);
+            if (it < 0) break;
             int bb, qq0, na, nb;
             decode(it, bb, qq0, na, nb);
             if (max(na, nb) == 0) continue;
@@ -1134,6 +1195,8 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
     while (group % 2 == 0 && group * per_problem > kGroupL2Bytes) group /= 2;
     p.group = (int)group;
     p.scale_log2 = d.scale * 1.4426950408889634f;
+    static std::atomic<unsigned> next_sched{0};
+    p.sched = two_tiles ? (int)(next_sched.fetch_add(1u) % kSchedSlots) : 0;
     // persistent: one CTA per SM (the CTA holds all of the SM's tensor memory)
     const int sms = current_sm_count();
     const unsigned grid = (unsigned)std::min<long long>(ctas, sms);

@@ -122,3 +122,40 @@ def test_attention_tune_records_the_faster_kernel():
     nj.nnjit_attention(dQ, dK, dV, O, causal=True)          # AUTO: the recorded kernel
     nj.nnjit_attention_check()
     assert oracle.rel_fro(O.cpu().numpy(), attention_ref(Q, K, V, 1.0 / np.sqrt(d), True)) <= TOL
+
+
+def test_two_tile_work_counter_resets():
+    """The two-tile kernel hands its items out from a per-launch work counter that the last
+    CTA to finish taking items zeroes.  More launches than counter slots, and replays of one
+    captured launch (the same slot every time), all give the first launch's output bit for
+    bit; the first output matches the oracle on sampled heads."""
+    B, Lq, Lk, d = 160, 600, 650, 64           # 160 x 3 items of 256 queries > the SM count
+    Q, K, V = _bf16((B, Lq, d), 14), _bf16((B, Lk, d), 15), _bf16((B, Lk, d), 16)
+    dQ, dK, dV = _dev(Q), _dev(K), _dev(V)
+    kern = KERNELS["tcgen05_2t"]
+    O0 = torch.full((B, Lq, d), float("nan"), dtype=torch.float32, device="cuda")
+    nj.nnjit_attention(dQ, dK, dV, O0, causal=True, kernel=kern)
+    nj.nnjit_attention_check()
+    first = O0.cpu().numpy()
+    heads = [0, 77, B - 1]
+    assert oracle.rel_fro(first[heads], attention_ref(Q[heads], K[heads], V[heads], 1.0 / np.sqrt(d), True)) <= TOL
+    O = torch.empty_like(O0)
+    for _ in range(70):                        # the launcher cycles through 64 slots
+        O.fill_(float("nan"))
+        nj.nnjit_attention(dQ, dK, dV, O, causal=True, kernel=kern)
+    nj.nnjit_attention_check()
+    assert np.array_equal(O.cpu().numpy(), first)
+    st = torch.cuda.Stream()
+    st.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(st):
+        Og = torch.full_like(O0, float("nan"))
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=st):
+            nj.nnjit_attention(dQ, dK, dV, Og, causal=True, kernel=kern)
+        for _ in range(3):
+            Og.fill_(float("nan"))
+            g.replay()
+    torch.cuda.current_stream().wait_stream(st)
+    torch.cuda.synchronize()
+    nj.nnjit_attention_check()
+    assert np.array_equal(Og.cpu().numpy(), first)
