@@ -81,6 +81,7 @@ struct Cfg {
 
 struct Params {
     CUtensorMap tq, tk, tv, to;
+    CUtensorMap to16;  // O in 32 x 16 pieces (64-byte rows, 64-byte swizzle): the two-tile kernel
     float* O;
     int Lq, Lk, causal, qblocks, batch;
     int group;  // problems per item group (divides batch)
@@ -151,6 +152,20 @@ __device__ __forceinline__ void st_shared_f4(uint32_t addr, float a, float b, fl
 // this thread's outstanding stores.
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32]) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+                 : "memory");
+}
+// 32 lanes x 16 consecutive 32-bit TMEM columns, and the wait for them.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+                   "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+                 : "r"(taddr));
+}
+__device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
+    asm volatile("tcgen05.wait::ld.sync.aligned;"
+                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
+                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
+                 :
                  : "memory");
 }
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
@@ -1104,30 +1119,33 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
                 ptx::tc_fence_after();
             }
             const float inv = (have_o && l > 0.0f) ? 1.0f / l : 0.0f;
-            // 32 x 32 tiles of the warp's rows: staged with the 128-byte swizzle and stored by
-            // TMA, which leaves rows past Lq unwritten
+            // 32 x 16 pieces of the warp's rows, staged alternately in the two 2 KB halves of
+            // the warp's buffer with the 64-byte swizzle (16-byte chunk c of row r at
+            // c ^ (r / 2 % 4)) and stored by TMA, which leaves rows past Lq unwritten: a store
+            // may still be reading one half while the warp fills the other
             const uint32_t stage = sO + (uint32_t)(warp - 2) * C::kOStage;
 #pragma unroll
-            for (int c0 = 0; c0 < D; c0 += 32) {
-                uint32_t r[32];
+            for (int c0 = 0; c0 < D; c0 += 16) {
+                uint32_t r[16];
                 if (have_o) {
-                    ptx::tmem_ld32(orow + c0, r);
-                    ptx::tmem_wait_ld(r);
+                    tmem_ld16(orow + c0, r);
+                    tmem_wait16(r);
                 } else {
 #pragma unroll
-                    for (int i = 0; i < 32; ++i) r[i] = 0u;
+                    for (int i = 0; i < 16; ++i) r[i] = 0u;
                 }
-                if (lane == 0) ptx::bulk_wait_all_read();  // the tile's previous store has read it
+                const uint32_t buf = stage + (uint32_t)((c0 / 16) & 1) * 2048u;
+                if (lane == 0) ptx::bulk_wait_read<1>();  // the store before last (this half) has read it
                 __syncwarp();
 #pragma unroll
-                for (int c = 0; c < 8; ++c)
-                    st_shared_f4(stage + (uint32_t)lane * 128u + ((uint32_t)(c ^ (lane & 7)) << 4),
+                for (int c = 0; c < 4; ++c)
+                    st_shared_f4(buf + (uint32_t)lane * 64u + ((uint32_t)(c ^ ((lane >> 1) & 3)) << 4),
                                  __uint_as_float(r[4 * c]) * inv, __uint_as_float(r[4 * c + 1]) * inv,
                                  __uint_as_float(r[4 * c + 2]) * inv, __uint_as_float(r[4 * c + 3]) * inv);
-                ptx::fence_proxy_async_smem();  // the tile is read by the TMA (async proxy)
+                ptx::fence_proxy_async_smem();  // the piece is read by the TMA (async proxy)
                 __syncwarp();
                 if (lane == 0) {
-                    ptx::tma_store_3d(&p.to, stage, c0, qq0 + x * kQ + q * 32, bb);
+                    ptx::tma_store_3d(&p.to16, buf, c0, qq0 + x * kQ + q * 32, bb);
                     ptx::bulk_commit();
                 }
             }
@@ -1179,6 +1197,11 @@ cudaError_t launch_attention_tc(const nnjit_attention_desc& d, const void* Q, co
         const cuuint32_t box[3] = {32, 32, 1};
         if (enc(&p.to, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, O, dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+        const cuuint32_t box16[3] = {16, 32, 1};
+        if (enc(&p.to16, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, O, dims, strides, box16, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
             return cudaErrorInvalidValue;
     }
