@@ -154,20 +154,6 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&r)[32
     asm volatile("tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]), "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]), "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
                  : "memory");
 }
-// 32 lanes x 16 consecutive 32-bit TMEM columns, and the wait for them.
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
-    asm volatile("tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
-                 : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
-                   "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-                 : "r"(taddr));
-}
-__device__ __forceinline__ void tmem_wait16(uint32_t (&r)[16]) {
-    asm volatile("tcgen05.wait::ld.sync.aligned;"
-                 : "+r"(r[0]), "+r"(r[1]), "+r"(r[2]), "+r"(r[3]), "+r"(r[4]), "+r"(r[5]), "+r"(r[6]), "+r"(r[7]),
-                   "+r"(r[8]), "+r"(r[9]), "+r"(r[10]), "+r"(r[11]), "+r"(r[12]), "+r"(r[13]), "+r"(r[14]), "+r"(r[15])
-                 :
-                 : "memory");
-}
 __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&r)[16]) {
     asm volatile("tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr), "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]), "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
                  : "memory");
@@ -1123,17 +1109,22 @@ __global__ void __launch_bounds__(320, 1) attention_tc2_kernel(const __grid_cons
             // the warp's buffer with the 64-byte swizzle (16-byte chunk c of row r at
             // c ^ (r / 2 % 4)) and stored by TMA, which leaves rows past Lq unwritten: a store
             // may still be reading one half while the warp fills the other
+            // (the row's D output columns come from TMEM in one round trip first)
             const uint32_t stage = sO + (uint32_t)(warp - 2) * C::kOStage;
+            uint32_t ro[D];
+            if (have_o) {
+#pragma unroll
+                for (int c0 = 0; c0 < D; c0 += 32)
+                    ptx::tmem_ld32(orow + c0, *reinterpret_cast<uint32_t(*)[32]>(ro + c0));
+#pragma unroll
+                for (int c0 = 0; c0 < D; c0 += 32) ptx::tmem_wait_ld(*reinterpret_cast<uint32_t(*)[32]>(ro + c0));
+            } else {
+#pragma unroll
+                for (int i = 0; i < D; ++i) ro[i] = 0u;
+            }
 #pragma unroll
             for (int c0 = 0; c0 < D; c0 += 16) {
-                uint32_t r[16];
-                if (have_o) {
-                    tmem_ld16(orow + c0, r);
-                    tmem_wait16(r);
-                } else {
-#pragma unroll
-                    for (int i = 0; i < 16; ++i) r[i] = 0u;
-                }
+                const uint32_t* r = ro + c0;
                 const uint32_t buf = stage + (uint32_t)((c0 / 16) & 1) * 2048u;
                 if (lane == 0) ptx::bulk_wait_read<1>();  // the store before last (this half) has read it
                 __syncwarp();
