@@ -410,7 +410,11 @@ nnjit_status nnjit_plan_destroy(nnjit_plan p);
  * kernel (128 queries per CTA, scores and outputs in TMEM, bounded waits), NNJIT_ATTN_MMA
  * (2) the warp-level MMA kernel (64 queries per CTA, no waits), NNJIT_ATTN_TCGEN05_2T (3)
  * the tensor-memory kernel with two 128-query tiles per CTA sharing each key and value
- * block (the tensor cores alternate between the tiles; bounded waits); AUTO takes the
+ * block (the tensor cores alternate between the tiles; bounded waits; when there are more
+ * work items than CTAs, the CTAs take them from a work counter in device memory: each
+ * call uses the next of 64 counter slots, which the call leaves at zero, so calls that
+ * run at the same time on different streams use different slots, while one captured
+ * graph replayed on two streams at once would share its slot and is not supported); AUTO takes the
  * kernel that nnjit_attention_tune recorded as fastest for the same (batch, Lq, Lk, d,
  * causal) on the current device, else the tensor-memory kernel (1).  INVALID_ARG for a bad
  * descriptor or NULL pointer, UNSUPPORTED for another d or unaligned pointers.
