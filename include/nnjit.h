@@ -416,7 +416,8 @@ nnjit_status nnjit_plan_destroy(nnjit_plan p);
  * run at the same time on different streams use different slots, while one captured
  * graph replayed on two streams at once would share its slot and is not supported); AUTO takes the
  * kernel that nnjit_attention_tune recorded as fastest for the same (batch, Lq, Lk, d,
- * causal) on the current device, else the tensor-memory kernel (1).  INVALID_ARG for a bad
+ * causal) on the current device, else the two-tile kernel (3) when batch * ceil(Lq / 256)
+ * is at least half the device's SM count and the tensor-memory kernel (1) otherwise.  INVALID_ARG for a bad
  * descriptor or NULL pointer, UNSUPPORTED for another d or unaligned pointers.
  * Asynchronous on `stream`; allocates nothing.  An expired wait inside the tensor-memory
  * kernel is reported by nnjit_attention_check.

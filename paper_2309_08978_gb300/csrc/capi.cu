@@ -689,7 +689,11 @@ nnjit_status nnjit_attention(const nnjit_attention_desc* d, const void* Q, const
     if (st != NNJIT_OK || d->Lq == 0) return st;
     int kernel = d->kernel;
     if (kernel == NNJIT_ATTN_AUTO) {
-        kernel = NNJIT_ATTN_TCGEN05;
+        // without a record: the two-tile kernel once its 256-query items fill at least half
+        // of the SMs (it was the faster on both benchmark shapes), else the one-tile kernel,
+        // whose 128-query items give small problems twice the CTAs
+        const long long items2 = d->batch * ((d->Lq + 255) / 256);
+        kernel = 2 * items2 >= current_sm_count() ? NNJIT_ATTN_TCGEN05_2T : NNJIT_ATTN_TCGEN05;
         int dev = 0;
         cudaGetDevice(&dev);
         std::lock_guard<std::mutex> lk(g_attn_mu);

@@ -159,3 +159,20 @@ def test_two_tile_work_counter_resets():
     torch.cuda.synchronize()
     nj.nnjit_attention_check()
     assert np.array_equal(Og.cpu().numpy(), first)
+
+
+def test_attention_auto_without_a_record():
+    """Without a tuning record, AUTO runs the two-tile kernel when its 256-query items fill
+    at least half of the SMs and the one-tile tensor-memory kernel otherwise: bit for bit
+    the chosen kernel's output."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    for B, kern in ((sms, KERNELS["tcgen05_2t"]), (2, KERNELS["tcgen05"])):
+        Lq, Lk, d = 200, 300, 64
+        Q, K, V = _bf16((B, Lq, d), 17), _bf16((B, Lk, d), 18), _bf16((B, Lk, d), 19)
+        dQ, dK, dV = _dev(Q), _dev(K), _dev(V)
+        want = torch.full((B, Lq, d), float("nan"), dtype=torch.float32, device="cuda")
+        got = torch.full_like(want, float("nan"))
+        nj.nnjit_attention(dQ, dK, dV, want, kernel=kern)
+        nj.nnjit_attention(dQ, dK, dV, got)                  # AUTO, no record for this shape
+        nj.nnjit_attention_check()
+        assert torch.equal(got, want)
