@@ -619,12 +619,16 @@ __global__ void __launch_bounds__(threads_of<D>(), 1) attention_tc_kernel(const 
 // O_A and O_B (512 columns with d = 128); P_X(j) is written over the columns of S_X(j)
 // it was computed from (the softmax has read them), and S_X(j + 1) is issued only after
 // P_X(j) V(j), so the in-order tensor pipe reads P_X(j) before overwriting it.  Each
-// softmax thread holds a whole row (128 scores): no exchange of row maxima.
-//   warp 0     TMA producer: both Q tiles of an item (one barrier), then its key and
-//              value blocks through the key and value rings;
+// softmax thread owns a whole row (no exchange of row maxima), read from TMEM in 32-column
+// pieces.
+//   warp 0     TMA producer: takes the items (its own index first, then from the launch's
+//              work counter) and publishes them in the item ring; per item Q_A, the first
+//              key block, Q_B (each tile's Q buffer with its own barriers), then the key
+//              and value blocks through the key and value rings;
 //   warp 1     TMEM owner and MMA issuer (converged warp, elected lane);
 //   warps 2-5  softmax of tile A (TMEM lane quarter = warp % 4), warps 6-9 of tile B.
-// Every wait is bounded, as in kernel 1.
+// The MMA and softmax warps read the items from the ring in the producer's order.  Every
+// wait is bounded, as in kernel 1.
 template <int D>
 struct Cfg2 {
     static constexpr int kKStages = 2;
